@@ -1,0 +1,246 @@
+/*
+ * sn.h -- C ABI of the GB300 routine-selecting CNN inference library
+ * (SoftNeuro, arXiv 2110.06037, reimplemented for sm_103a).
+ *
+ * The calls follow the paper's statement of the tuning problem (Alg. 1,
+ * "Input: a 1-in-1-out net {L_i}, layer-wise optimal routines {F_i},
+ * {F^a_ij}, a routine schema set Lambda; Output: the optimal routine path
+ * S*"):
+ *   sn_graph_create / sn_add_layer  build the net            (section III-B)
+ *   sn_profile                      measures T(r)            (section III-C)
+ *   sn_get/set_cost_table           the profiling data T(r), T(r^a)
+ *   sn_select_path                  DPRS (Alg. 1) or brute force (Def. 2)
+ *   sn_run                          inference with the tuned path
+ *
+ * Conventions for every call:
+ *   - Every function returns sn_status; no C++ exception, abort or CUDA error
+ *     crosses this boundary.  On a status other than SN_OK the graph is left
+ *     as it was and sn_last_error() gives a message (thread-local, valid until
+ *     the next call on the same thread).
+ *   - Pointers named *_dev are device pointers on the current CUDA device;
+ *     all other pointers are host pointers.  `stream` is a cudaStream_t
+ *     (NULL = the legacy default stream).  The library launches only on that
+ *     stream and never synchronises the device; calls that must read results
+ *     back (profiling, SN_OPT_CHECK) synchronise that stream only.
+ *   - Host arrays passed in are copied; the caller keeps ownership.  Device
+ *     memory the library needs (weights in each schema, activations,
+ *     workspace) comes from the allocator given to sn_graph_create (or
+ *     cudaMalloc when none is given) and is released by sn_graph_destroy.
+ *   - Tensor extents are always given as logical (N, C, H, W); the schema's
+ *     layout says how they are stored (NCHW or NHWC, dense, row-major).
+ *   - Costs are int64 nanoseconds; SN_COST_INF (INT64_MAX) = infeasible.
+ */
+#ifndef SN_H
+#define SN_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define SN_API __attribute__((visibility("default")))
+#else
+#define SN_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct sn_graph sn_graph; /* opaque, owned by the library */
+
+typedef enum {
+    SN_OK = 0,
+    SN_EINVAL = 1,        /* bad argument, size or layer parameter            */
+    SN_ENOMEM = 2,        /* the allocator returned NULL                      */
+    SN_ECUDA = 3,         /* a CUDA runtime/driver call failed                */
+    SN_EUNSUPPORTED = 4,  /* valid request this build cannot serve            */
+    SN_ESTATE = 5,        /* call out of order (e.g. sn_run before a path)    */
+    SN_ETIMEOUT = 6,      /* a device-side bounded wait gave up               */
+    SN_EINFEASIBLE = 7    /* no routine path with finite cost exists          */
+} sn_status;
+
+#define SN_COST_INF INT64_MAX
+
+/* Routine schema (section III-C): the platform is always this GPU, so a
+ * schema is the pair (data type, layout).  Two adjacent layers whose routines
+ * have different schemas are joined by an adapt routine that casts and/or
+ * permutes the blob. */
+typedef enum { SN_F32 = 0, SN_F16 = 1, SN_BF16 = 2 } sn_dtype;
+typedef enum { SN_NCHW = 0, SN_NHWC = 1 } sn_layout;
+typedef struct { int32_t dtype; int32_t layout; } sn_schema;
+
+/* Layer types (section III-B); activations are fused layer attributes (the
+ * importer's ReLU fusion, section III-A). */
+typedef enum {
+    SN_L_CONV2 = 0,   /* 2-D convolution (cross-correlation) + bias + act      */
+    SN_L_DWCONV2 = 1, /* depthwise conv2: groups = c_in = c_out                */
+    SN_L_MAXPOOL = 2, /* max pooling, -inf padding                             */
+    SN_L_GAP = 3,     /* global average pooling -> N x C x 1 x 1               */
+    SN_L_ADD = 4,     /* elementwise sum of two blobs + act                    */
+    SN_L_DENSE = 5    /* y = W x + b on an N x C x 1 x 1 blob                  */
+} sn_layer_type;
+
+typedef enum { SN_ACT_NONE = 0, SN_ACT_RELU = 1, SN_ACT_RELU6 = 2 } sn_act;
+
+/* conv2 / dwconv2 parameters: output extent P = floor((H + 2ph - dh(kh-1) - 1)/sh) + 1. */
+typedef struct {
+    int32_t c_in, c_out, kh, kw, sh, sw, ph, pw, dh, dw, groups, act;
+} sn_conv_params;
+typedef struct { int32_t kh, kw, sh, sw, ph, pw; } sn_pool_params;
+typedef struct { int32_t act; } sn_add_params;
+typedef struct { int32_t in_features, out_features, act; } sn_dense_params;
+
+/* Device allocator hooks (e.g. the PyTorch caching allocator).  alloc returns
+ * a device pointer aligned to >= 256 bytes or NULL; free releases it. */
+typedef void *(*sn_alloc_fn)(size_t bytes, void *ctx);
+typedef void (*sn_free_fn)(void *ptr, void *ctx);
+
+/*
+ * Create an empty net with one input blob of logical shape in_nchw, stored in
+ * in_schema, whose output will be produced in out_schema.  schemas[0..n) is
+ * the schema set Lambda the routines may use (section IV-A).  The input and
+ * output are the net's auxiliary layers L_1 and L_n (section IV-E): one
+ * zero-cost routine each, in in_schema / out_schema.
+ * alloc/free may both be NULL (cudaMalloc/cudaFree are used).
+ * Errors: SN_EINVAL (bad shape or schema, n_schemas < 1, only one of alloc/free).
+ */
+SN_API sn_status sn_graph_create(const int64_t in_nchw[4], sn_schema in_schema, sn_schema out_schema,
+                          const sn_schema *schemas, int32_t n_schemas, sn_alloc_fn alloc,
+                          sn_free_fn free_fn, void *alloc_ctx, sn_graph **out);
+
+/*
+ * Append a layer (section III-B).  params points to the struct for the type
+ * (sn_conv_params for CONV2/DWCONV2, sn_pool_params, sn_add_params,
+ * sn_dense_params; NULL for GAP).  inputs[0..n_inputs) are ids returned by
+ * earlier calls, -1 = the net input (ADD takes two, the others one).
+ * weights: host fp32, conv [c_out][c_in/groups][kh][kw], dense [out][in];
+ * bias: host fp32 [c_out] or NULL (zeros).  Both are copied.  The last layer
+ * added is the net output.  *out_layer_id receives the new layer's id.
+ * Errors: SN_EINVAL (shape mismatch, bad parameter), SN_ESTATE (after the
+ * net was finalised by sn_profile/sn_get_cost_table/sn_select_path/...).
+ */
+SN_API sn_status sn_add_layer(sn_graph *g, int32_t type, const void *params, const int32_t *inputs,
+                       int32_t n_inputs, const float *weights, const float *bias,
+                       int32_t *out_layer_id);
+
+/* ---------------- the cost table (profiling data, section III-C) ----------
+ * After finalisation the net has n_layers = (layers added) + 2 internal
+ * layers in topological order: 0 is the input layer, n_layers-1 the output
+ * layer and layer id u returned by sn_add_layer is internal layer u+1.
+ * Each layer has candidate routines (routine id, routine-parameter
+ * combination "variant", schema index); each edge (src, dst) has an adapt
+ * cost for every ordered schema pair (void adapt = 0 on the diagonal).
+ * Schema indices run over the graph's schema universe: Lambda in the order
+ * given, then in_schema and out_schema if they are not in Lambda. */
+typedef struct {
+    int32_t routine;  /* routine id, see sn_routine_name()                */
+    int32_t variant;  /* routine-parameter combination index              */
+    int32_t schema;   /* schema index                                      */
+    int32_t layer;    /* internal layer index                              */
+    int64_t cost_ns;  /* T(r); SN_COST_INF until profiled or set           */
+} sn_candidate;
+
+typedef struct {
+    int32_t n_layers, n_schemas, n_edges, n_candidates;
+    sn_candidate *candidates; /* [n_candidates], grouped by layer, ascending  */
+    int32_t *edges;           /* [n_edges][2] = (src, dst) internal layers    */
+    int64_t *adapt_cost;      /* [n_edges][n_schemas (from)][n_schemas (to)]  */
+} sn_cost_table;
+
+/* Finalise the net if needed and report the table.  With t->candidates,
+ * t->edges and t->adapt_cost all NULL only the four sizes are written;
+ * otherwise the caller provides arrays of those sizes and they are filled. */
+SN_API sn_status sn_get_cost_table(sn_graph *g, sn_cost_table *t);
+/* Overwrite every candidate cost and adapt cost from t (sizes must match the
+ * graph's; the routine/variant/schema/layer fields are checked, not copied).
+ * Lets a caller inject or reuse profiling data.  Errors: SN_EINVAL. */
+SN_API sn_status sn_set_cost_table(sn_graph *g, const sn_cost_table *t);
+/* Schema universe queries. */
+SN_API sn_status sn_get_schema(sn_graph *g, int32_t index, sn_schema *out, int32_t *n_schemas);
+
+/* ---------------- profiling (section III-C) --------------------------------
+ * Unit profiling times every candidate of every layer, deduplicated by layer
+ * signature, on scratch buffers: `warmup` untimed launches, then the median
+ * of `iters` launches timed with CUDA events on `stream`, rounded to ns.
+ * Every adapt (blob shape, from, to) is timed the same way.  With topk > 0,
+ * integrated profiling then re-times the topk best candidates per (layer,
+ * schema) inside whole-net passes (one pass per schema and rank, `passes`
+ * repetitions, median) and replaces their unit times.  Synchronises stream. */
+typedef struct {
+    int32_t warmup;   /* default 3  */
+    int32_t iters;    /* default 20 */
+    int32_t topk;     /* default 2; 0 = unit profiling only */
+    int32_t passes;   /* default 5  */
+} sn_profile_opts;
+SN_API sn_status sn_profile(sn_graph *g, const sn_profile_opts *opts, void *stream);
+
+/* ---------------- path selection (section IV) ------------------------------ */
+#define SN_SELECT_DPRS 0  /* Alg. 1                                            */
+#define SN_SELECT_BRUTE 1 /* exhaustive argmin of Def. 2 (small nets only)     */
+
+typedef struct {
+    int64_t total_ns;   /* T(S*)                                          */
+    int32_t n_layers;   /* in: capacity of the arrays; out: n_layers       */
+    int32_t *schema;    /* [n_layers] chosen schema index per layer, or NULL */
+    int32_t *candidate; /* [n_layers] chosen candidate index (global index
+                           into the cost table's candidates), or NULL       */
+} sn_path;
+
+/* Select S* from the current cost table and make it the path sn_run uses.
+ * Errors: SN_EINFEASIBLE (every path has infinite cost), SN_EUNSUPPORTED
+ * (brute force on a net with too many assignments), SN_EINVAL. */
+SN_API sn_status sn_select_path(sn_graph *g, int32_t method, sn_path *out);
+/* Force a path: candidate[i] is a global candidate index of layer i for
+ * every internal layer (tests use this to run one routine in isolation). */
+SN_API sn_status sn_set_path(sn_graph *g, const int32_t *candidate, int32_t n_layers);
+
+/* ---------------- inference --------------------------------------------- */
+#define SN_OPT_CUDA_GRAPH 0 /* 1 = replay the launch sequence as a CUDA graph    */
+#define SN_OPT_CHECK 1      /* 1 = sync stream after sn_run and read the device
+                               error word (SN_ETIMEOUT / SN_ECUDA on failure)    */
+SN_API sn_status sn_set_option(sn_graph *g, int32_t option, int64_t value);
+
+/* Run the net with the selected path: in_dev holds the input in in_schema,
+ * out_dev receives the output in out_schema (both caller-owned device
+ * buffers of the full tensor size).  The first call after a path change
+ * builds the plan (adapt insertion, buffers, weight copies per schema).
+ * Errors: SN_ESTATE (no path), SN_ENOMEM, SN_ECUDA, SN_ETIMEOUT. */
+SN_API sn_status sn_run(sn_graph *g, const void *in_dev, void *out_dev, void *stream);
+
+/* sn_run with a CUDA event pair around every launch of the plan; after the
+ * stream has finished (this call synchronises it) layer_ms[i] holds the time
+ * of layer i's routine and edge_ms[e] that of edge e's adapt (0 if void).
+ * Either array may be NULL.  Sizes: n_layers and n_edges. */
+SN_API sn_status sn_run_timed(sn_graph *g, const void *in_dev, void *out_dev, void *stream,
+                       float *layer_ms, float *edge_ms);
+
+/* Logical output shape of internal layer `layer` (N, C, H, W). */
+SN_API sn_status sn_layer_shape(sn_graph *g, int32_t layer, int64_t out_nchw[4]);
+
+/* Save / restore the tuned state (cost table + selected path) as JSON.  A
+ * loaded file must describe the same net (same layers and candidates). */
+SN_API sn_status sn_save_plan(sn_graph *g, const char *path);
+SN_API sn_status sn_load_plan(sn_graph *g, const char *path);
+
+SN_API void sn_graph_destroy(sn_graph *g);
+
+/* ---------------- routines and adapts used directly ------------------------ */
+/* Routine descriptor "cuda:<dtype>.<layout>/<algorithm>" style name of a
+ * routine id (section III-C), or NULL for an unknown id. */
+SN_API const char *sn_routine_name(int32_t routine);
+/* Human-readable routine parameters of (routine, variant), e.g. "bn=128". */
+SN_API const char *sn_variant_name(int32_t routine, int32_t variant);
+
+/* Adapt routine on its own (section III-C, jobs (2) and (3)): convert the
+ * N x C x H x W blob x_dev stored in `from` into y_dev stored in `to`
+ * (layout permutation and/or round-to-nearest-even cast; bit-exact).
+ * Errors: SN_EINVAL, SN_ECUDA. */
+SN_API sn_status sn_convert(const void *x_dev, sn_schema from, void *y_dev, sn_schema to,
+                     const int64_t nchw[4], void *stream);
+
+SN_API const char *sn_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* SN_H */

@@ -1,0 +1,523 @@
+// extern "C" boundary of the library (declared in include/sn.h).  Every entry
+// point catches C++ exceptions and turns them into a status, so nothing but
+// an sn_status crosses the ABI.
+#include <cstdio>
+#include <cstring>
+#include <fstream>
+#include <sstream>
+#include <string>
+
+#include "sn_internal.h"
+
+namespace sn {
+const char *last_error();
+sn_status add_layer(Graph *g, int32_t type, const void *params, const int32_t *inputs,
+                    int32_t n_inputs, const float *weights, const float *bias, int32_t *out_id);
+}  // namespace sn
+
+using namespace sn;
+
+#define SN_GUARD(...)                                                    \
+    try {                                                                \
+        __VA_ARGS__                                                      \
+    } catch (const std::bad_alloc &) {                                   \
+        return fail(SN_ENOMEM, "host allocation failed");                \
+    } catch (const std::exception &ex) {                                 \
+        return fail(SN_EINVAL, std::string("internal error: ") + ex.what()); \
+    } catch (...) {                                                      \
+        return fail(SN_EINVAL, "internal error");                        \
+    }
+
+extern "C" {
+
+const char *sn_last_error(void) { return last_error(); }
+
+const char *sn_routine_name(int32_t routine) { return routine_name(routine); }
+
+const char *sn_variant_name(int32_t routine, int32_t variant) {
+    if (!routine_name(routine)) return nullptr;
+    return variant_name(routine, variant);
+}
+
+sn_status sn_graph_create(const int64_t in_nchw[4], sn_schema in_schema, sn_schema out_schema,
+                          const sn_schema *schemas, int32_t n_schemas, sn_alloc_fn alloc,
+                          sn_free_fn free_fn, void *alloc_ctx, sn_graph **out) {
+    SN_GUARD({
+        if (!out || !in_nchw || !schemas || n_schemas < 1 || n_schemas > 16)
+            return fail(SN_EINVAL, "sn_graph_create: bad arguments");
+        *out = nullptr;
+        if ((alloc == nullptr) != (free_fn == nullptr))
+            return fail(SN_EINVAL, "sn_graph_create: give both alloc and free, or neither");
+        for (int k = 0; k < 4; ++k)
+            if (in_nchw[k] < 1) return fail(SN_EINVAL, "sn_graph_create: input extents must be >= 1");
+        if (!schema_valid(in_schema) || !schema_valid(out_schema))
+            return fail(SN_EINVAL, "sn_graph_create: invalid in/out schema");
+        auto *g = new Graph();
+        g->in_shape = {in_nchw[0], in_nchw[1], in_nchw[2], in_nchw[3]};
+        g->in_schema = in_schema;
+        g->out_schema = out_schema;
+        for (int32_t i = 0; i < n_schemas; ++i) {
+            if (!schema_valid(schemas[i])) {
+                delete g;
+                return fail(SN_EINVAL, "sn_graph_create: invalid schema in Lambda");
+            }
+            for (auto &s : g->schemas)
+                if (schema_eq(s, schemas[i])) {
+                    delete g;
+                    return fail(SN_EINVAL, "sn_graph_create: duplicate schema in Lambda");
+                }
+            g->schemas.push_back(schemas[i]);
+        }
+        g->n_lambda = n_schemas;
+        auto find_or_add = [&](sn_schema s) {
+            for (size_t i = 0; i < g->schemas.size(); ++i)
+                if (schema_eq(g->schemas[i], s)) return (int32_t)i;
+            g->schemas.push_back(s);
+            return (int32_t)g->schemas.size() - 1;
+        };
+        g->in_schema_idx = find_or_add(in_schema);
+        g->out_schema_idx = find_or_add(out_schema);
+        g->alloc = alloc;
+        g->free_fn = free_fn;
+        g->alloc_ctx = alloc_ctx;
+        *out = reinterpret_cast<sn_graph *>(g);
+        return SN_OK;
+    })
+}
+
+static Graph *G(sn_graph *g) { return reinterpret_cast<Graph *>(g); }
+
+sn_status sn_add_layer(sn_graph *g, int32_t type, const void *params, const int32_t *inputs,
+                       int32_t n_inputs, const float *weights, const float *bias,
+                       int32_t *out_layer_id) {
+    SN_GUARD({
+        if (!g || !out_layer_id) return fail(SN_EINVAL, "sn_add_layer: NULL argument");
+        return add_layer(G(g), type, params, inputs, n_inputs, weights, bias, out_layer_id);
+    })
+}
+
+sn_status sn_get_cost_table(sn_graph *gg, sn_cost_table *t) {
+    SN_GUARD({
+        if (!gg || !t) return fail(SN_EINVAL, "sn_get_cost_table: NULL argument");
+        Graph *g = G(gg);
+        sn_status rc = graph_finalize(g);
+        if (rc != SN_OK) return rc;
+        const bool sizes_only = !t->candidates && !t->edges && !t->adapt_cost;
+        if (!sizes_only) {
+            if (t->n_layers != g->n_layers() || t->n_schemas != g->n_schemas() ||
+                t->n_edges != (int32_t)g->edges.size() || t->n_candidates != (int32_t)g->cands.size())
+                return fail(SN_EINVAL, "sn_get_cost_table: array sizes do not match the graph");
+            if (t->candidates)
+                for (size_t c = 0; c < g->cands.size(); ++c) {
+                    const Candidate &k = g->cands[c];
+                    t->candidates[c] = {k.routine, k.variant, k.schema, k.layer, k.cost};
+                }
+            if (t->edges)
+                for (size_t e = 0; e < g->edges.size(); ++e) {
+                    t->edges[2 * e] = g->edges[e].first;
+                    t->edges[2 * e + 1] = g->edges[e].second;
+                }
+            if (t->adapt_cost)
+                std::memcpy(t->adapt_cost, g->adapt_cost.data(), g->adapt_cost.size() * sizeof(int64_t));
+        }
+        t->n_layers = g->n_layers();
+        t->n_schemas = g->n_schemas();
+        t->n_edges = (int32_t)g->edges.size();
+        t->n_candidates = (int32_t)g->cands.size();
+        return SN_OK;
+    })
+}
+
+sn_status sn_set_cost_table(sn_graph *gg, const sn_cost_table *t) {
+    SN_GUARD({
+        if (!gg || !t || !t->candidates || !t->adapt_cost)
+            return fail(SN_EINVAL, "sn_set_cost_table: NULL argument");
+        Graph *g = G(gg);
+        sn_status rc = graph_finalize(g);
+        if (rc != SN_OK) return rc;
+        if (t->n_layers != g->n_layers() || t->n_schemas != g->n_schemas() ||
+            t->n_edges != (int32_t)g->edges.size() || t->n_candidates != (int32_t)g->cands.size())
+            return fail(SN_EINVAL, "sn_set_cost_table: sizes do not match the graph");
+        for (size_t c = 0; c < g->cands.size(); ++c) {
+            const Candidate &k = g->cands[c];
+            const sn_candidate &x = t->candidates[c];
+            if (x.routine != k.routine || x.variant != k.variant || x.schema != k.schema || x.layer != k.layer)
+                return fail(SN_EINVAL, "sn_set_cost_table: candidate " + std::to_string(c) + " differs");
+            if (x.cost_ns < 0) return fail(SN_EINVAL, "sn_set_cost_table: negative cost");
+        }
+        const int32_t ns = g->n_schemas();
+        for (size_t e = 0; e < g->edges.size(); ++e)
+            for (int32_t a = 0; a < ns; ++a) {
+                if (t->adapt_cost[(e * ns + a) * ns + a] != 0)
+                    return fail(SN_EINVAL, "sn_set_cost_table: void adapt must cost 0");
+                for (int32_t b = 0; b < ns; ++b)
+                    if (t->adapt_cost[(e * ns + a) * ns + b] < 0)
+                        return fail(SN_EINVAL, "sn_set_cost_table: negative adapt cost");
+            }
+        for (size_t c = 0; c < g->cands.size(); ++c) g->cands[c].cost = t->candidates[c].cost_ns;
+        std::memcpy(g->adapt_cost.data(), t->adapt_cost, g->adapt_cost.size() * sizeof(int64_t));
+        return SN_OK;
+    })
+}
+
+sn_status sn_get_schema(sn_graph *gg, int32_t index, sn_schema *out, int32_t *n_schemas) {
+    SN_GUARD({
+        if (!gg) return fail(SN_EINVAL, "sn_get_schema: NULL graph");
+        Graph *g = G(gg);
+        if (n_schemas) *n_schemas = g->n_schemas();
+        if (out) {
+            if (index < 0 || index >= g->n_schemas()) return fail(SN_EINVAL, "schema index out of range");
+            *out = g->schemas[index];
+        }
+        return SN_OK;
+    })
+}
+
+sn_status sn_profile(sn_graph *gg, const sn_profile_opts *opts, void *stream) {
+    SN_GUARD({
+        if (!gg) return fail(SN_EINVAL, "sn_profile: NULL graph");
+        Graph *g = G(gg);
+        sn_status rc = graph_finalize(g);
+        if (rc != SN_OK) return rc;
+        sn_profile_opts o{3, 20, 2, 5};
+        if (opts) o = *opts;
+        if (o.warmup < 0 || o.iters < 1 || o.topk < 0 || o.passes < 1 || o.iters > 10000)
+            return fail(SN_EINVAL, "sn_profile: bad options");
+        return profile_graph(g, o, static_cast<cudaStream_t>(stream));
+    })
+}
+
+static sn_status fill_path(Graph *g, const std::vector<int32_t> &schema_of, int64_t total, sn_path *out) {
+    std::vector<int64_t> F;
+    std::vector<int32_t> argF;
+    fastest_per_schema(*g, F, argF);
+    const int32_t n = g->n_layers(), ns = g->n_schemas();
+    std::vector<int32_t> pc(n);
+    for (int32_t i = 0; i < n; ++i) {
+        pc[i] = argF[(size_t)i * ns + schema_of[i]];
+        if (pc[i] < 0) return fail(SN_EINFEASIBLE, "selected schema has no routine");
+    }
+    g->path_cand = pc;
+    g->path_total = total;
+    g->has_path = true;
+    invalidate_plan(g);
+    if (out) {
+        if ((out->schema || out->candidate) && out->n_layers < n)
+            return fail(SN_EINVAL, "sn_path arrays too small");
+        out->total_ns = total;
+        out->n_layers = n;
+        for (int32_t i = 0; i < n; ++i) {
+            if (out->schema) out->schema[i] = schema_of[i];
+            if (out->candidate) out->candidate[i] = pc[i];
+        }
+    }
+    return SN_OK;
+}
+
+sn_status sn_select_path(sn_graph *gg, int32_t method, sn_path *out) {
+    SN_GUARD({
+        if (!gg) return fail(SN_EINVAL, "sn_select_path: NULL graph");
+        Graph *g = G(gg);
+        sn_status rc = graph_finalize(g);
+        if (rc != SN_OK) return rc;
+        std::vector<int32_t> schema_of;
+        int64_t total = kInf;
+        if (method == SN_SELECT_DPRS) rc = select_dprs(*g, schema_of, total);
+        else if (method == SN_SELECT_BRUTE) rc = select_brute(*g, schema_of, total);
+        else return fail(SN_EINVAL, "sn_select_path: unknown method");
+        if (rc != SN_OK) return rc;
+        return fill_path(g, schema_of, total, out);
+    })
+}
+
+sn_status sn_set_path(sn_graph *gg, const int32_t *candidate, int32_t n_layers) {
+    SN_GUARD({
+        if (!gg || !candidate) return fail(SN_EINVAL, "sn_set_path: NULL argument");
+        Graph *g = G(gg);
+        sn_status rc = graph_finalize(g);
+        if (rc != SN_OK) return rc;
+        const int32_t n = g->n_layers();
+        if (n_layers != n) return fail(SN_EINVAL, "sn_set_path: wrong number of layers");
+        int64_t total = 0;
+        std::vector<int32_t> sch(n);
+        for (int32_t i = 0; i < n; ++i) {
+            const int32_t c = candidate[i];
+            if (c < g->cand_begin[i] || c >= g->cand_begin[i + 1])
+                return fail(SN_EINVAL, "sn_set_path: candidate " + std::to_string(c) +
+                                           " does not belong to layer " + std::to_string(i));
+            sch[i] = g->cands[c].schema;
+            total = sat_add(total, g->cands[c].cost);
+        }
+        for (size_t e = 0; e < g->edges.size(); ++e) {
+            auto [u, v] = g->edges[e];
+            if (sch[u] != sch[v]) total = sat_add(total, g->adapt((int32_t)e, sch[u], sch[v]));
+        }
+        g->path_cand.assign(candidate, candidate + n);
+        g->path_total = total;
+        g->has_path = true;
+        invalidate_plan(g);
+        return SN_OK;
+    })
+}
+
+sn_status sn_set_option(sn_graph *gg, int32_t option, int64_t value) {
+    SN_GUARD({
+        if (!gg) return fail(SN_EINVAL, "sn_set_option: NULL graph");
+        Graph *g = G(gg);
+        if (option == SN_OPT_CUDA_GRAPH) {
+            g->opt_graph = value ? 1 : 0;
+            if (g->gexec) {
+                cudaGraphExecDestroy(g->gexec);
+                g->gexec = nullptr;
+            }
+        } else if (option == SN_OPT_CHECK) {
+            g->opt_check = value ? 1 : 0;
+        } else {
+            return fail(SN_EINVAL, "sn_set_option: unknown option");
+        }
+        return SN_OK;
+    })
+}
+
+static sn_status check_device(Graph *g, cudaStream_t st) {
+    (void)g;
+    SN_CUDA_TRY(cudaStreamSynchronize(st));
+    int word = 0;
+    SN_CUDA_TRY(cudaMemcpy(&word, k::device_error_word(), sizeof(int), cudaMemcpyDeviceToHost));
+    if (word) {
+        const int zero = 0;
+        cudaMemcpy(k::device_error_word(), &zero, sizeof(int), cudaMemcpyHostToDevice);
+        return fail(SN_ETIMEOUT, "device error word set: " + std::to_string(word) +
+                                     " (a bounded wait in a kernel gave up)");
+    }
+    return SN_OK;
+}
+
+sn_status sn_run(sn_graph *gg, const void *in_dev, void *out_dev, void *stream) {
+    SN_GUARD({
+        if (!gg || !in_dev || !out_dev) return fail(SN_EINVAL, "sn_run: NULL argument");
+        Graph *g = G(gg);
+        if (!g->has_path) return fail(SN_ESTATE, "sn_run: select or set a routine path first");
+        cudaStream_t st = static_cast<cudaStream_t>(stream);
+        if (!g->plan_valid) {
+            sn_status rc = build_plan(g, st);
+            if (rc != SN_OK) return rc;
+        }
+        sn_status rc = SN_OK;
+        if (g->opt_graph && st != nullptr) {
+            if (!g->gexec || g->gexec_in != in_dev || g->gexec_out != out_dev || g->gexec_stream != st) {
+                if (g->gexec) {
+                    cudaGraphExecDestroy(g->gexec);
+                    g->gexec = nullptr;
+                }
+                cudaGraph_t graph = nullptr;
+                SN_CUDA_TRY(cudaStreamBeginCapture(st, cudaStreamCaptureModeThreadLocal));
+                rc = run_plan(g, in_dev, out_dev, st, nullptr);
+                cudaError_t ce = cudaStreamEndCapture(st, &graph);
+                if (rc != SN_OK) {
+                    if (graph) cudaGraphDestroy(graph);
+                    return rc;
+                }
+                if (ce != cudaSuccess) return fail(SN_ECUDA, std::string("graph capture: ") + cudaGetErrorString(ce));
+                ce = cudaGraphInstantiate(&g->gexec, graph, 0);
+                cudaGraphDestroy(graph);
+                if (ce != cudaSuccess) {
+                    g->gexec = nullptr;
+                    return fail(SN_ECUDA, std::string("graph instantiate: ") + cudaGetErrorString(ce));
+                }
+                g->gexec_in = in_dev;
+                g->gexec_out = out_dev;
+                g->gexec_stream = st;
+            }
+            SN_CUDA_TRY(cudaGraphLaunch(g->gexec, st));
+        } else {
+            rc = run_plan(g, in_dev, out_dev, st, nullptr);
+            if (rc != SN_OK) return rc;
+        }
+        if (g->opt_check) return check_device(g, st);
+        return SN_OK;
+    })
+}
+
+sn_status sn_run_timed(sn_graph *gg, const void *in_dev, void *out_dev, void *stream,
+                       float *layer_ms, float *edge_ms) {
+    SN_GUARD({
+        if (!gg || !in_dev || !out_dev) return fail(SN_EINVAL, "sn_run_timed: NULL argument");
+        Graph *g = G(gg);
+        if (!g->has_path) return fail(SN_ESTATE, "sn_run_timed: select or set a routine path first");
+        cudaStream_t st = static_cast<cudaStream_t>(stream);
+        if (!g->plan_valid) {
+            sn_status rc = build_plan(g, st);
+            if (rc != SN_OK) return rc;
+        }
+        std::vector<cudaEvent_t> evs(2 * g->plan.size());
+        for (auto &e : evs) SN_CUDA_TRY(cudaEventCreate(&e));
+        sn_status rc = run_plan(g, in_dev, out_dev, st, &evs);
+        cudaError_t ce = cudaStreamSynchronize(st);
+        if (rc == SN_OK && ce == cudaSuccess) {
+            if (layer_ms)
+                for (int32_t i = 0; i < g->n_layers(); ++i) layer_ms[i] = 0.f;
+            if (edge_ms)
+                for (size_t e = 0; e < g->edges.size(); ++e) edge_ms[e] = 0.f;
+            for (size_t q = 0; q < g->plan.size(); ++q) {
+                float t = 0;
+                cudaEventElapsedTime(&t, evs[2 * q], evs[2 * q + 1]);
+                const PlanOp &op = g->plan[q];
+                if (op.kind == PlanOp::LAYER && layer_ms) layer_ms[op.layer] += t;
+                if (op.kind == PlanOp::ADAPT && edge_ms && op.edge >= 0) edge_ms[op.edge] += t;
+            }
+        }
+        for (auto &e : evs) cudaEventDestroy(e);
+        if (rc != SN_OK) return rc;
+        if (ce != cudaSuccess) return fail(SN_ECUDA, std::string("sn_run_timed: ") + cudaGetErrorString(ce));
+        if (g->opt_check) return check_device(g, st);
+        return SN_OK;
+    })
+}
+
+sn_status sn_layer_shape(sn_graph *gg, int32_t layer, int64_t out_nchw[4]) {
+    SN_GUARD({
+        if (!gg || !out_nchw) return fail(SN_EINVAL, "sn_layer_shape: NULL argument");
+        Graph *g = G(gg);
+        sn_status rc = graph_finalize(g);
+        if (rc != SN_OK) return rc;
+        if (layer < 0 || layer >= g->n_layers()) return fail(SN_EINVAL, "layer out of range");
+        const Shape &s = g->layers[layer].out;
+        out_nchw[0] = s.n, out_nchw[1] = s.c, out_nchw[2] = s.h, out_nchw[3] = s.w;
+        return SN_OK;
+    })
+}
+
+// ---- plan files: a small JSON document with integer arrays ----
+sn_status sn_save_plan(sn_graph *gg, const char *path) {
+    SN_GUARD({
+        if (!gg || !path) return fail(SN_EINVAL, "sn_save_plan: NULL argument");
+        Graph *g = G(gg);
+        sn_status rc = graph_finalize(g);
+        if (rc != SN_OK) return rc;
+        std::ofstream f(path);
+        if (!f) return fail(SN_EINVAL, std::string("cannot open ") + path);
+        f << "{\n \"format\": \"softneuro-gb300-plan-1\",\n";
+        f << " \"n_layers\": " << g->n_layers() << ",\n \"n_schemas\": " << g->n_schemas()
+          << ",\n \"n_edges\": " << g->edges.size() << ",\n \"n_candidates\": " << g->cands.size() << ",\n";
+        f << " \"candidates\": [";
+        for (size_t c = 0; c < g->cands.size(); ++c) {
+            const Candidate &k = g->cands[c];
+            f << (c ? ", " : "") << "[" << k.routine << ", " << k.variant << ", " << k.schema << ", "
+              << k.layer << ", " << k.cost << "]";
+        }
+        f << "],\n \"adapt_cost\": [";
+        for (size_t i = 0; i < g->adapt_cost.size(); ++i) f << (i ? ", " : "") << g->adapt_cost[i];
+        f << "],\n \"path\": [";
+        if (g->has_path)
+            for (size_t i = 0; i < g->path_cand.size(); ++i) f << (i ? ", " : "") << g->path_cand[i];
+        f << "],\n \"total_ns\": " << (g->has_path ? g->path_total : -1) << "\n}\n";
+        if (!f) return fail(SN_EINVAL, "write failed");
+        return SN_OK;
+    })
+}
+
+static bool read_int_array(const std::string &doc, const std::string &key, std::vector<int64_t> &out) {
+    const size_t k = doc.find("\"" + key + "\"");
+    if (k == std::string::npos) return false;
+    size_t p = doc.find('[', k);
+    if (p == std::string::npos) return false;
+    int depth = 0;
+    std::string num;
+    out.clear();
+    for (; p < doc.size(); ++p) {
+        const char ch = doc[p];
+        if (ch == '[') {
+            ++depth;
+        } else if (ch == ']' || ch == ',') {
+            if (!num.empty()) {
+                out.push_back(std::stoll(num));
+                num.clear();
+            }
+            if (ch == ']' && --depth == 0) return true;
+        } else if ((ch >= '0' && ch <= '9') || ch == '-') {
+            num += ch;
+        }
+    }
+    return false;
+}
+
+static bool read_int(const std::string &doc, const std::string &key, int64_t &v) {
+    const size_t k = doc.find("\"" + key + "\"");
+    if (k == std::string::npos) return false;
+    size_t p = doc.find(':', k);
+    if (p == std::string::npos) return false;
+    v = std::stoll(doc.substr(p + 1));
+    return true;
+}
+
+sn_status sn_load_plan(sn_graph *gg, const char *path) {
+    SN_GUARD({
+        if (!gg || !path) return fail(SN_EINVAL, "sn_load_plan: NULL argument");
+        Graph *g = G(gg);
+        sn_status rc = graph_finalize(g);
+        if (rc != SN_OK) return rc;
+        std::ifstream f(path);
+        if (!f) return fail(SN_EINVAL, std::string("cannot open ") + path);
+        std::stringstream ss;
+        ss << f.rdbuf();
+        const std::string doc = ss.str();
+        int64_t nl, ns, ne, nc, total;
+        std::vector<int64_t> cands, ac, pth;
+        if (!read_int(doc, "n_layers", nl) || !read_int(doc, "n_schemas", ns) || !read_int(doc, "n_edges", ne) ||
+            !read_int(doc, "n_candidates", nc) || !read_int(doc, "total_ns", total) ||
+            !read_int_array(doc, "candidates", cands) || !read_int_array(doc, "adapt_cost", ac) ||
+            !read_int_array(doc, "path", pth))
+            return fail(SN_EINVAL, "sn_load_plan: malformed plan file");
+        if (nl != g->n_layers() || ns != g->n_schemas() || ne != (int64_t)g->edges.size() ||
+            nc != (int64_t)g->cands.size() || cands.size() != (size_t)nc * 5 || ac.size() != g->adapt_cost.size())
+            return fail(SN_EINVAL, "sn_load_plan: plan describes a different net");
+        for (size_t c = 0; c < g->cands.size(); ++c) {
+            const Candidate &k = g->cands[c];
+            if (cands[5 * c] != k.routine || cands[5 * c + 1] != k.variant || cands[5 * c + 2] != k.schema ||
+                cands[5 * c + 3] != k.layer)
+                return fail(SN_EINVAL, "sn_load_plan: candidate list differs");
+        }
+        if (!pth.empty()) {
+            if ((int64_t)pth.size() != nl) return fail(SN_EINVAL, "sn_load_plan: bad path length");
+            for (int32_t i = 0; i < g->n_layers(); ++i)
+                if (pth[i] < g->cand_begin[i] || pth[i] >= g->cand_begin[i + 1])
+                    return fail(SN_EINVAL, "sn_load_plan: path candidate out of range");
+        }
+        for (size_t c = 0; c < g->cands.size(); ++c) g->cands[c].cost = cands[5 * c + 4];
+        for (size_t i = 0; i < ac.size(); ++i) g->adapt_cost[i] = ac[i];
+        if (!pth.empty()) {
+            g->path_cand.assign(pth.begin(), pth.end());
+            g->path_total = total;
+            g->has_path = true;
+        } else {
+            g->has_path = false;
+        }
+        invalidate_plan(g);
+        return SN_OK;
+    })
+}
+
+void sn_graph_destroy(sn_graph *g) {
+    try {
+        delete G(g);
+    } catch (...) {
+    }
+}
+
+sn_status sn_convert(const void *x_dev, sn_schema from, void *y_dev, sn_schema to,
+                     const int64_t nchw[4], void *stream) {
+    SN_GUARD({
+        if (!x_dev || !y_dev || !nchw) return fail(SN_EINVAL, "sn_convert: NULL argument");
+        if (!schema_valid(from) || !schema_valid(to)) return fail(SN_EINVAL, "sn_convert: invalid schema");
+        for (int k = 0; k < 4; ++k)
+            if (nchw[k] < 0) return fail(SN_EINVAL, "sn_convert: negative extent");
+        const Shape s{nchw[0], nchw[1], nchw[2], nchw[3]};
+        if (s.numel() == 0) return SN_OK;
+        SN_CUDA_TRY(k::convert(x_dev, from.dtype, from.layout, y_dev, to.dtype, to.layout, s,
+                               static_cast<cudaStream_t>(stream)));
+        return SN_OK;
+    })
+}
+
+}  // extern "C"

@@ -1,0 +1,274 @@
+// Net construction and finalisation (section III-B: net = DAG of layers with
+// one input and one output; section IV-A: layers L_1..L_n in topological
+// order; section IV-E: auxiliary zero-cost input/output layers).
+#include <algorithm>
+#include <cstring>
+
+#include "sn_internal.h"
+
+namespace sn {
+
+static thread_local std::string g_last_error;
+
+void set_error(const std::string &msg) { g_last_error = msg; }
+sn_status fail(sn_status s, const std::string &msg) {
+    g_last_error = msg;
+    return s;
+}
+const char *last_error() { return g_last_error.c_str(); }
+
+std::string schema_str(sn_schema s) {
+    static const char *dt[] = {"f32", "f16", "bf16"};
+    static const char *ly[] = {"nchw", "nhwc"};
+    if (!schema_valid(s)) return "invalid";
+    return std::string(dt[s.dtype]) + "." + ly[s.layout];
+}
+
+static int64_t out_dim(int64_t in, int64_t k, int64_t s, int64_t p, int64_t d) {
+    const int64_t span = d * (k - 1) + 1;
+    if (in + 2 * p < span) return 0;
+    return (in + 2 * p - span) / s + 1;
+}
+
+Graph::~Graph() {
+    if (gexec) cudaGraphExecDestroy(gexec);
+    for (auto &b : slots) dev_free(this, &b);
+    for (auto &kv : weight_cache) dev_free(this, &kv.second);
+    for (auto &kv : bias_cache) dev_free(this, &kv.second);
+    dev_free(this, &workspace);
+}
+
+sn_status dev_alloc(Graph *g, size_t bytes, Buffer *b) {
+    b->bytes = bytes;
+    b->ptr = nullptr;
+    if (bytes == 0) return SN_OK;
+    const size_t rounded = (bytes + 255) & ~size_t(255);
+    if (g->alloc) {
+        b->ptr = g->alloc(rounded, g->alloc_ctx);
+        if (!b->ptr) return fail(SN_ENOMEM, "allocator returned NULL for " + std::to_string(rounded) + " bytes");
+        if (reinterpret_cast<uintptr_t>(b->ptr) & 255u) {
+            g->free_fn(b->ptr, g->alloc_ctx);
+            b->ptr = nullptr;
+            return fail(SN_EINVAL, "allocator returned a pointer not aligned to 256 bytes");
+        }
+        return SN_OK;
+    }
+    cudaError_t e = cudaMalloc(&b->ptr, rounded);
+    if (e != cudaSuccess) {
+        b->ptr = nullptr;
+        return fail(e == cudaErrorMemoryAllocation ? SN_ENOMEM : SN_ECUDA,
+                    std::string("cudaMalloc: ") + cudaGetErrorString(e));
+    }
+    return SN_OK;
+}
+
+void dev_free(Graph *g, Buffer *b) {
+    if (!b->ptr) return;
+    if (g->free_fn) g->free_fn(b->ptr, g->alloc_ctx);
+    else cudaFree(b->ptr);
+    b->ptr = nullptr;
+    b->bytes = 0;
+}
+
+void invalidate_plan(Graph *g) {
+    g->plan_valid = false;
+    g->plan.clear();
+    if (g->gexec) {
+        cudaGraphExecDestroy(g->gexec);
+        g->gexec = nullptr;
+    }
+}
+
+// ---------------------------------------------------------------------------
+// layer validation + shape inference
+// ---------------------------------------------------------------------------
+static sn_status infer_shape(Layer &L, const std::vector<Shape> &in) {
+    switch (L.type) {
+    case SN_L_CONV2:
+    case SN_L_DWCONV2: {
+        const sn_conv_params &p = L.conv;
+        if (in.size() != 1) return fail(SN_EINVAL, "conv2 takes one input");
+        if (p.kh < 1 || p.kw < 1 || p.sh < 1 || p.sw < 1 || p.ph < 0 || p.pw < 0 || p.dh < 1 ||
+            p.dw < 1 || p.groups < 1 || p.c_in < 1 || p.c_out < 1)
+            return fail(SN_EINVAL, "conv2: invalid parameter");
+        if (p.act < SN_ACT_NONE || p.act > SN_ACT_RELU6) return fail(SN_EINVAL, "conv2: bad act");
+        if (in[0].c != p.c_in) return fail(SN_EINVAL, "conv2: input channels != c_in");
+        if (p.c_in % p.groups || p.c_out % p.groups)
+            return fail(SN_EINVAL, "conv2: groups must divide c_in and c_out");
+        if (L.type == SN_L_DWCONV2 && !(p.groups == p.c_in && p.c_in == p.c_out))
+            return fail(SN_EINVAL, "dwconv2: requires groups == c_in == c_out");
+        const int64_t P = out_dim(in[0].h, p.kh, p.sh, p.ph, p.dh);
+        const int64_t Q = out_dim(in[0].w, p.kw, p.sw, p.pw, p.dw);
+        if (P < 1 || Q < 1) return fail(SN_EINVAL, "conv2: empty output");
+        L.out = {in[0].n, p.c_out, P, Q};
+        L.act = p.act;
+        return SN_OK;
+    }
+    case SN_L_MAXPOOL: {
+        const sn_pool_params &p = L.pool;
+        if (in.size() != 1) return fail(SN_EINVAL, "maxpool takes one input");
+        if (p.kh < 1 || p.kw < 1 || p.sh < 1 || p.sw < 1 || p.ph < 0 || p.pw < 0 ||
+            p.ph >= p.kh || p.pw >= p.kw)
+            return fail(SN_EINVAL, "maxpool: invalid parameter (padding must be < kernel)");
+        const int64_t P = out_dim(in[0].h, p.kh, p.sh, p.ph, 1);
+        const int64_t Q = out_dim(in[0].w, p.kw, p.sw, p.pw, 1);
+        if (P < 1 || Q < 1) return fail(SN_EINVAL, "maxpool: empty output");
+        L.out = {in[0].n, in[0].c, P, Q};
+        return SN_OK;
+    }
+    case SN_L_GAP:
+        if (in.size() != 1) return fail(SN_EINVAL, "gap takes one input");
+        L.out = {in[0].n, in[0].c, 1, 1};
+        return SN_OK;
+    case SN_L_ADD:
+        if (in.size() != 2) return fail(SN_EINVAL, "add takes two inputs");
+        if (!(in[0] == in[1])) return fail(SN_EINVAL, "add: input shapes differ");
+        if (L.act < SN_ACT_NONE || L.act > SN_ACT_RELU6) return fail(SN_EINVAL, "add: bad act");
+        L.out = in[0];
+        return SN_OK;
+    case SN_L_DENSE:
+        if (in.size() != 1) return fail(SN_EINVAL, "dense takes one input");
+        if (in[0].h != 1 || in[0].w != 1 || in[0].c != L.dense_in || L.dense_out < 1)
+            return fail(SN_EINVAL, "dense: input must be N x in_features x 1 x 1");
+        if (L.act < SN_ACT_NONE || L.act > SN_ACT_RELU6) return fail(SN_EINVAL, "dense: bad act");
+        L.out = {in[0].n, L.dense_out, 1, 1};
+        return SN_OK;
+    default:
+        return fail(SN_EINVAL, "unknown layer type");
+    }
+}
+
+sn_status add_layer(Graph *g, int32_t type, const void *params, const int32_t *inputs,
+                    int32_t n_inputs, const float *weights, const float *bias, int32_t *out_id) {
+    if (g->finalized) return fail(SN_ESTATE, "net already finalised; no more layers");
+    if (n_inputs < 1 || n_inputs > 2 || !inputs) return fail(SN_EINVAL, "bad inputs");
+    Layer L;
+    L.type = type;
+    std::vector<Shape> in;
+    for (int32_t i = 0; i < n_inputs; ++i) {
+        const int32_t id = inputs[i];
+        if (id < -1 || id >= (int32_t)g->user.size()) return fail(SN_EINVAL, "input id out of range");
+        L.inputs.push_back(id + 1);  // internal index
+        in.push_back(id < 0 ? g->in_shape : g->user[id].out);
+    }
+    int64_t wn = 0, bn = 0;
+    switch (type) {
+    case SN_L_CONV2:
+    case SN_L_DWCONV2:
+        if (!params) return fail(SN_EINVAL, "conv2 needs params");
+        std::memcpy(&L.conv, params, sizeof(sn_conv_params));
+        wn = (int64_t)L.conv.c_out * (L.conv.groups > 0 ? L.conv.c_in / L.conv.groups : 0) *
+             L.conv.kh * L.conv.kw;
+        bn = L.conv.c_out;
+        break;
+    case SN_L_MAXPOOL:
+        if (!params) return fail(SN_EINVAL, "maxpool needs params");
+        std::memcpy(&L.pool, params, sizeof(sn_pool_params));
+        break;
+    case SN_L_GAP:
+        break;
+    case SN_L_ADD:
+        L.act = params ? static_cast<const sn_add_params *>(params)->act : SN_ACT_NONE;
+        break;
+    case SN_L_DENSE: {
+        if (!params) return fail(SN_EINVAL, "dense needs params");
+        auto *p = static_cast<const sn_dense_params *>(params);
+        L.dense_in = p->in_features;
+        L.dense_out = p->out_features;
+        L.act = p->act;
+        wn = (int64_t)L.dense_in * L.dense_out;
+        bn = L.dense_out;
+        break;
+    }
+    default:
+        return fail(SN_EINVAL, "unknown layer type");
+    }
+    sn_status s = infer_shape(L, in);
+    if (s != SN_OK) return s;
+    if (wn > 0) {
+        if (!weights) return fail(SN_EINVAL, "layer needs weights");
+        L.weight.assign(weights, weights + wn);
+        L.bias.assign(bn, 0.0f);
+        if (bias) L.bias.assign(bias, bias + bn);
+    }
+    g->user.push_back(std::move(L));
+    *out_id = (int32_t)g->user.size() - 1;
+    return SN_OK;
+}
+
+// ---------------------------------------------------------------------------
+// finalisation: internal layers, edges, candidates
+// ---------------------------------------------------------------------------
+sn_status graph_finalize(Graph *g) {
+    if (g->finalized) return SN_OK;
+    const int32_t m = (int32_t)g->user.size();
+    std::vector<Layer> L;
+    Layer in_l;
+    in_l.type = -1;
+    in_l.out = g->in_shape;
+    L.push_back(in_l);
+    for (auto &u : g->user) L.push_back(u);
+    Layer out_l;
+    out_l.type = -2;
+    out_l.inputs = {m};  // last user layer (internal index m), or the input when m == 0
+    out_l.out = m ? g->user[m - 1].out : g->in_shape;
+    L.push_back(out_l);
+    const int32_t n = (int32_t)L.size();
+
+    // 1-in-1-out: every layer must reach the output (section IV-A)
+    std::vector<char> reach(n, 0);
+    reach[n - 1] = 1;
+    for (int32_t i = n - 1; i >= 0; --i)
+        if (reach[i])
+            for (int32_t j : L[i].inputs) reach[j] = 1;
+    for (int32_t i = 0; i < n; ++i)
+        if (!reach[i])
+            return fail(SN_EINVAL, "layer " + std::to_string(i - 1) +
+                                       " does not reach the net output (net must be 1-in-1-out)");
+
+    std::vector<std::pair<int32_t, int32_t>> edges;
+    for (int32_t i = 0; i < n; ++i)
+        for (int32_t j : L[i].inputs) edges.push_back({j, i});
+
+    std::vector<Candidate> cands;
+    std::vector<int32_t> begin(n + 1, 0);
+    for (int32_t i = 0; i < n; ++i) {
+        begin[i] = (int32_t)cands.size();
+        if (i == 0) {
+            cands.push_back({R_IO, 0, g->in_schema_idx, 0, 0});
+            continue;
+        }
+        if (i == n - 1) {
+            cands.push_back({R_IO, 0, g->out_schema_idx, n - 1, 0});
+            continue;
+        }
+        std::vector<Shape> in;
+        for (int32_t j : L[i].inputs) in.push_back(L[j].out);
+        for (int32_t r = 1; r < R_COUNT; ++r) {
+            if (r == R_ADAPT) continue;
+            for (int32_t s = 0; s < g->n_lambda; ++s) {
+                const int32_t nv = routine_variants(r, L[i], in, g->schemas[s]);
+                for (int32_t v = 0; v < nv; ++v) cands.push_back({r, v, s, i, kInf});
+            }
+        }
+        if ((int32_t)cands.size() == begin[i])
+            return fail(SN_EINFEASIBLE, "layer " + std::to_string(i - 1) +
+                                            " has no routine in any schema of Lambda");
+    }
+    begin[n] = (int32_t)cands.size();
+
+    const int32_t ns = g->n_schemas();
+    std::vector<int64_t> ac((size_t)edges.size() * ns * ns, kInf);
+    for (size_t e = 0; e < edges.size(); ++e)
+        for (int32_t a = 0; a < ns; ++a) ac[(e * ns + a) * ns + a] = 0;  // void adapt
+
+    g->layers = std::move(L);
+    g->edges = std::move(edges);
+    g->cands = std::move(cands);
+    g->cand_begin = std::move(begin);
+    g->adapt_cost = std::move(ac);
+    g->finalized = true;
+    return SN_OK;
+}
+
+}  // namespace sn

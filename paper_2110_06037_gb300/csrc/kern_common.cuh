@@ -1,0 +1,71 @@
+// Device helpers shared by the kernel translation units.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+
+#include <cstdint>
+
+#include "sn_internal.h"
+
+namespace sn {
+namespace k {
+
+template <typename T> __device__ __forceinline__ float ldf(const T *p);
+template <> __device__ __forceinline__ float ldf<float>(const float *p) { return *p; }
+template <> __device__ __forceinline__ float ldf<__half>(const __half *p) { return __half2float(*p); }
+template <> __device__ __forceinline__ float ldf<__nv_bfloat16>(const __nv_bfloat16 *p) {
+    return __bfloat162float(*p);
+}
+
+// round-to-nearest-even stores
+template <typename T> __device__ __forceinline__ void stf(T *p, float v);
+template <> __device__ __forceinline__ void stf<float>(float *p, float v) { *p = v; }
+template <> __device__ __forceinline__ void stf<__half>(__half *p, float v) { *p = __float2half_rn(v); }
+template <> __device__ __forceinline__ void stf<__nv_bfloat16>(__nv_bfloat16 *p, float v) {
+    *p = __float2bfloat16_rn(v);
+}
+
+template <typename T> __device__ __forceinline__ T cvt(float v);
+template <> __device__ __forceinline__ float cvt<float>(float v) { return v; }
+template <> __device__ __forceinline__ __half cvt<__half>(float v) { return __float2half_rn(v); }
+template <> __device__ __forceinline__ __nv_bfloat16 cvt<__nv_bfloat16>(float v) {
+    return __float2bfloat16_rn(v);
+}
+
+__device__ __forceinline__ float act_apply(float v, int act) {
+    if (act == SN_ACT_RELU) return fmaxf(v, 0.0f);
+    if (act == SN_ACT_RELU6) return fminf(fmaxf(v, 0.0f), 6.0f);
+    return v;
+}
+
+inline unsigned grid_for(int64_t n, int block, int64_t cap = 152LL * 64) {
+    int64_t g = (n + block - 1) / block;
+    if (g > cap) g = cap;
+    if (g < 1) g = 1;
+    return (unsigned)g;
+}
+
+// dispatch a runtime dtype to a C++ type
+#define SN_DT_SWITCH(dt, T, ...)                          \
+    switch (dt) {                                         \
+    case SN_F32: { using T = float; __VA_ARGS__; break; } \
+    case SN_F16: { using T = __half; __VA_ARGS__; break; } \
+    default: { using T = __nv_bfloat16; __VA_ARGS__; break; } \
+    }
+
+struct ConvDims {
+    int32_t N, C, H, W, K, P, Q, R, S, sh, sw, ph, pw, dh, dw, groups, act;
+};
+
+inline ConvDims conv_dims(const LaunchArgs &a) {
+    const sn_conv_params &p = a.layer->conv;
+    const Shape &i = a.in_shapes[0];
+    const Shape &o = a.layer->out;
+    return ConvDims{(int32_t)i.n, (int32_t)i.c, (int32_t)i.h, (int32_t)i.w, (int32_t)o.c, (int32_t)o.h,
+                    (int32_t)o.w, p.kh, p.kw, p.sh, p.sw, p.ph, p.pw, p.dh, p.dw, p.groups, p.act};
+}
+
+}  // namespace k
+}  // namespace sn

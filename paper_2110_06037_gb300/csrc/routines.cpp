@@ -1,0 +1,166 @@
+// Routine registry (section III-C): which routines can serve a layer in a
+// schema, their routine-parameter combinations ("variants"), the weight
+// format each expects, and dispatch to the kernels.
+//
+// Every routine reads its inputs and writes its output in its own schema;
+// conversions between schemas are separate adapt routines on the edges.
+#include <string>
+
+#include "sn_internal.h"
+
+namespace sn {
+
+const char *routine_name(int32_t r) {
+    switch (r) {
+    case R_IO: return "io";
+    case R_CONV_DIRECT: return "conv2/direct";
+    case R_CONV_IGEMM: return "conv2/igemm_simt";
+    case R_CONV_WINO: return "conv2/wino_f2x2_3x3";
+    case R_CONV_TC: return "conv2/igemm_tc";
+    case R_DW_DIRECT: return "dwconv2/direct";
+    case R_MAXPOOL: return "maxpool/direct";
+    case R_GAP: return "gap/reduce";
+    case R_ADD: return "add/eltwise";
+    case R_DENSE: return "dense/simt";
+    case R_ADAPT: return "adapt/convert";
+    default: return nullptr;
+    }
+}
+
+const char *variant_name(int32_t r, int32_t v) {
+    switch (r) {
+    case R_CONV_IGEMM: return v == 0 ? "tile=64x64" : "tile=128x64";
+    case R_CONV_WINO: return v == 0 ? "gemm=simt" : "gemm=tc";
+    case R_CONV_TC: return k::conv_tc_variant_name(v);
+    default: return v == 0 ? "" : "?";
+    }
+}
+
+static bool is_conv(const Layer &l) { return l.type == SN_L_CONV2; }
+
+int32_t routine_variants(int32_t r, const Layer &l, const std::vector<Shape> &in, sn_schema s) {
+    const sn_conv_params &p = l.conv;
+    switch (r) {
+    case R_CONV_DIRECT:
+        return is_conv(l) ? 1 : 0;
+    case R_CONV_IGEMM:
+        return (is_conv(l) && p.groups == 1) ? 2 : 0;
+    case R_CONV_WINO:
+        return (is_conv(l) && p.groups == 1 && p.kh == 3 && p.kw == 3 && p.sh == 1 && p.sw == 1 &&
+                p.dh == 1 && p.dw == 1 && p.ph <= 2 && p.pw <= 2)
+                   ? 1
+                   : 0;
+    case R_CONV_TC:
+        return is_conv(l) ? k::conv_tc_variants(l, in[0], s) : 0;
+    case R_DW_DIRECT:
+        return l.type == SN_L_DWCONV2 ? 1 : 0;
+    case R_MAXPOOL:
+        return l.type == SN_L_MAXPOOL ? 1 : 0;
+    case R_GAP:
+        return l.type == SN_L_GAP ? 1 : 0;
+    case R_ADD:
+        return l.type == SN_L_ADD ? 1 : 0;
+    case R_DENSE:
+        return l.type == SN_L_DENSE ? 1 : 0;
+    default:
+        return 0;
+    }
+}
+
+size_t routine_workspace(int32_t r, int32_t v, const Layer &l, const std::vector<Shape> &in,
+                         sn_schema s) {
+    (void)v;
+    if (r == R_CONV_WINO) return k::conv_wino_ws(l, in[0], s);
+    return 0;
+}
+
+// weight format of (routine, layout)
+static int weight_format_of(int32_t r, sn_schema s) {
+    switch (r) {
+    case R_CONV_DIRECT: return s.layout == SN_NCHW ? k::W_KCRS : k::W_RSCK;
+    case R_CONV_IGEMM: return s.layout == SN_NCHW ? k::W_KCRS : k::W_KRSC;
+    case R_CONV_WINO: return k::W_WINO;
+    case R_CONV_TC: return k::W_KRSC;
+    case R_DW_DIRECT: return s.layout == SN_NCHW ? k::W_KCRS : k::W_RSCK;
+    case R_DENSE: return k::W_KCRS;
+    default: return -1;
+    }
+}
+
+sn_status prepare_weights(Graph *g, int32_t li, int32_t r, int32_t v, sn_schema s,
+                          const void **wt, const float **bias, cudaStream_t st) {
+    (void)v;
+    *wt = nullptr;
+    *bias = nullptr;
+    const Layer &L = g->layers[li];
+    if (L.weight.empty()) return SN_OK;
+    const int fmt = weight_format_of(r, s);
+    if (fmt < 0) return SN_OK;
+    int64_t K, Cg, R, S;
+    if (L.type == SN_L_DENSE) {
+        K = L.dense_out, Cg = L.dense_in, R = S = 1;
+    } else {
+        K = L.conv.c_out, Cg = L.conv.c_in / L.conv.groups, R = L.conv.kh, S = L.conv.kw;
+    }
+    // bias: fp32 on the device, shared by every routine of the layer
+    auto bit = g->bias_cache.find(li);
+    if (bit == g->bias_cache.end()) {
+        Buffer b;
+        sn_status rc = dev_alloc(g, L.bias.size() * sizeof(float), &b);
+        if (rc != SN_OK) return rc;
+        SN_CUDA_TRY(cudaMemcpyAsync(b.ptr, L.bias.data(), L.bias.size() * sizeof(float),
+                                    cudaMemcpyHostToDevice, st));
+        bit = g->bias_cache.emplace(li, b).first;
+    }
+    *bias = static_cast<const float *>(bit->second.ptr);
+
+    const std::string key = std::to_string(li) + "/" + std::to_string(fmt) + "/" + std::to_string(s.dtype);
+    auto it = g->weight_cache.find(key);
+    if (it != g->weight_cache.end()) {
+        *wt = it->second.ptr;
+        return SN_OK;
+    }
+    const int64_t elems = (fmt == k::W_WINO) ? 16 * K * Cg : K * Cg * R * S;
+    Buffer src, dst;
+    sn_status rc = dev_alloc(g, (size_t)K * Cg * R * S * sizeof(float), &src);
+    if (rc != SN_OK) return rc;
+    rc = dev_alloc(g, (size_t)elems * dtype_size(s.dtype), &dst);
+    if (rc != SN_OK) {
+        dev_free(g, &src);
+        return rc;
+    }
+    cudaError_t e = cudaMemcpyAsync(src.ptr, L.weight.data(), L.weight.size() * sizeof(float),
+                                    cudaMemcpyHostToDevice, st);
+    if (e == cudaSuccess)
+        e = k::weight_format(static_cast<const float *>(src.ptr), dst.ptr, fmt, s.dtype, K, Cg, R, S, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);  // src is freed next
+    dev_free(g, &src);
+    if (e != cudaSuccess) {
+        dev_free(g, &dst);
+        return fail(SN_ECUDA, std::string("weight preparation: ") + cudaGetErrorString(e));
+    }
+    g->weight_cache.emplace(key, dst);
+    *wt = dst.ptr;
+    return SN_OK;
+}
+
+sn_status launch_routine(const LaunchArgs &a) {
+    cudaError_t e = cudaSuccess;
+    switch (a.routine) {
+    case R_CONV_DIRECT: e = k::conv_direct(a); break;
+    case R_CONV_IGEMM: e = k::conv_igemm(a); break;
+    case R_CONV_WINO: e = k::conv_wino(a); break;
+    case R_CONV_TC: e = k::conv_tc(a); break;
+    case R_DW_DIRECT: e = k::dwconv(a); break;
+    case R_MAXPOOL: e = k::maxpool(a); break;
+    case R_GAP: e = k::gap(a); break;
+    case R_ADD: e = k::add(a); break;
+    case R_DENSE: e = k::dense(a); break;
+    default: return fail(SN_EINVAL, "launch of a non-launchable routine");
+    }
+    if (e != cudaSuccess)
+        return fail(SN_ECUDA, std::string(routine_name(a.routine)) + ": " + cudaGetErrorString(e));
+    return SN_OK;
+}
+
+}  // namespace sn

@@ -1,0 +1,438 @@
+// Plan construction, execution and profiling.
+//
+// Plan (inference with the tuned path, section III-A step 3): every layer
+// runs its selected routine; an adapt routine is inserted on every edge whose
+// endpoint schemas differ (section III-C; one conversion per edge, as Def. 1
+// charges one adapt per edge).  Activations live in graph-owned buffers; the
+// net input and output are the caller's buffers.
+//
+// Profiling (section III-C): unit profiling of every candidate, deduplicated
+// by layer signature, then integrated profiling of the best candidates per
+// (layer, schema) inside whole-net passes.
+#include <algorithm>
+#include <cstdio>
+#include <cstring>
+#include <sstream>
+#include <string>
+
+#include "sn_internal.h"
+
+namespace sn {
+
+static sn_status schema_slot(Graph *g, Shape s, sn_schema sc) {
+    g->slots.push_back({});
+    g->slot_shape.push_back(s);
+    g->slot_schema.push_back(sc);
+    return SN_OK;
+}
+
+sn_status build_plan(Graph *g, cudaStream_t st) {
+    if (!g->has_path) return fail(SN_ESTATE, "no routine path selected");
+    invalidate_plan(g);
+    for (auto &b : g->slots) dev_free(g, &b);
+    g->slots.clear();
+    g->slot_shape.clear();
+    g->slot_schema.clear();
+    const int32_t n = g->n_layers();
+    std::vector<sn_schema> sch(n);
+    for (int32_t i = 0; i < n; ++i) sch[i] = g->schemas[g->cands[g->path_cand[i]].schema];
+    schema_slot(g, g->in_shape, g->in_schema);              // slot 0: caller's input
+    schema_slot(g, g->layers[n - 1].out, g->out_schema);    // slot 1: caller's output
+    std::vector<int32_t> out_slot(n, -1);
+    out_slot[0] = 0;
+    const int32_t last = n - 2;  // last user layer (0 if none)
+    size_t ws = 0;
+    for (int32_t i = 1; i < n; ++i) {
+        const Layer &L = g->layers[i];
+        PlanOp op;
+        op.kind = PlanOp::LAYER;
+        op.layer = i;
+        op.cand = g->path_cand[i];
+        for (size_t k = 0; k < L.inputs.size(); ++k) {
+            const int32_t j = L.inputs[k];
+            int32_t e = -1;
+            for (size_t q = 0; q < g->edges.size(); ++q)
+                if (g->edges[q].first == j && g->edges[q].second == i) {
+                    e = (int32_t)q;
+                    if (k == 1 && L.inputs[0] == j) {  // second edge of add(x, x)
+                        for (size_t q2 = q + 1; q2 < g->edges.size(); ++q2)
+                            if (g->edges[q2].first == j && g->edges[q2].second == i) {
+                                e = (int32_t)q2;
+                                break;
+                            }
+                    }
+                    break;
+                }
+            int32_t src = out_slot[j];
+            const bool same = schema_eq(sch[j], sch[i]);
+            if (i == n - 1) {
+                // output layer: adapt into the caller's buffer unless the last
+                // layer already wrote there
+                if (!same || j == 0) {
+                    PlanOp a;
+                    a.kind = PlanOp::ADAPT;
+                    a.layer = i;
+                    a.edge = e;
+                    a.in_slots = {src};
+                    a.out_slot = 1;
+                    g->plan.push_back(a);
+                }
+                continue;
+            }
+            if (!same) {
+                schema_slot(g, g->layers[j].out, sch[i]);
+                PlanOp a;
+                a.kind = PlanOp::ADAPT;
+                a.layer = i;
+                a.edge = e;
+                a.in_slots = {src};
+                a.out_slot = (int32_t)g->slots.size() - 1;
+                g->plan.push_back(a);
+                src = a.out_slot;
+            }
+            op.in_slots.push_back(src);
+        }
+        if (i == n - 1) break;
+        if (i == last && schema_eq(sch[i], g->out_schema)) {
+            op.out_slot = 1;
+        } else {
+            schema_slot(g, L.out, sch[i]);
+            op.out_slot = (int32_t)g->slots.size() - 1;
+        }
+        out_slot[i] = op.out_slot;
+        const Candidate &c = g->cands[op.cand];
+        std::vector<Shape> in;
+        for (int32_t j : L.inputs) in.push_back(g->layers[j].out);
+        ws = std::max(ws, routine_workspace(c.routine, c.variant, L, in, sch[i]));
+        sn_status rc = prepare_weights(g, i, c.routine, c.variant, sch[i], &op.wt, &op.bias, st);
+        if (rc != SN_OK) return rc;
+        g->plan.push_back(op);
+    }
+    for (size_t s = 2; s < g->slots.size(); ++s) {
+        const size_t bytes = (size_t)g->slot_shape[s].numel() * dtype_size(g->slot_schema[s].dtype);
+        sn_status rc = dev_alloc(g, bytes, &g->slots[s]);
+        if (rc != SN_OK) return rc;
+    }
+    if (ws > g->workspace.bytes) {
+        dev_free(g, &g->workspace);
+        sn_status rc = dev_alloc(g, ws, &g->workspace);
+        if (rc != SN_OK) return rc;
+    }
+    g->plan_valid = true;
+    return SN_OK;
+}
+
+static sn_status launch_op(Graph *g, const PlanOp &op, const void *in, void *out,
+                           cudaStream_t st) {
+    auto ptr = [&](int32_t s) -> void * {
+        if (s == 0) return const_cast<void *>(in);
+        if (s == 1) return out;
+        return g->slots[s].ptr;
+    };
+    if (op.kind == PlanOp::ADAPT) {
+        const int32_t si = op.in_slots[0], so = op.out_slot;
+        const sn_schema a = g->slot_schema[si], b = g->slot_schema[so];
+        cudaError_t e = k::convert(ptr(si), a.dtype, a.layout, ptr(so), b.dtype, b.layout,
+                                   g->slot_shape[si], st);
+        if (e != cudaSuccess) return fail(SN_ECUDA, std::string("adapt: ") + cudaGetErrorString(e));
+        return SN_OK;
+    }
+    const Layer &L = g->layers[op.layer];
+    const Candidate &c = g->cands[op.cand];
+    LaunchArgs a;
+    a.g = g;
+    a.layer = &L;
+    a.routine = c.routine;
+    a.variant = c.variant;
+    a.schema = g->schemas[c.schema];
+    for (size_t k = 0; k < op.in_slots.size(); ++k) {
+        a.in[k] = ptr(op.in_slots[k]);
+        a.in_shapes.push_back(g->layers[L.inputs[k]].out);
+    }
+    a.out = ptr(op.out_slot);
+    a.wt = op.wt;
+    a.bias = op.bias;
+    a.ws = g->workspace.ptr;
+    a.ws_bytes = g->workspace.bytes;
+    a.stream = st;
+    return launch_routine(a);
+}
+
+sn_status run_plan(Graph *g, const void *in, void *out, cudaStream_t st,
+                   std::vector<cudaEvent_t> *evs) {
+    if (!g->plan_valid) {
+        sn_status rc = build_plan(g, st);
+        if (rc != SN_OK) return rc;
+    }
+    for (size_t i = 0; i < g->plan.size(); ++i) {
+        if (evs) SN_CUDA_TRY(cudaEventRecord((*evs)[2 * i], st));
+        sn_status rc = launch_op(g, g->plan[i], in, out, st);
+        if (rc != SN_OK) return rc;
+        if (evs) SN_CUDA_TRY(cudaEventRecord((*evs)[2 * i + 1], st));
+    }
+    return SN_OK;
+}
+
+// ---------------------------------------------------------------------------
+// profiling
+// ---------------------------------------------------------------------------
+namespace {
+
+struct Scratch {
+    Buffer in0, in1, out;
+};
+
+sn_status ensure(Graph *g, Buffer &b, size_t bytes) {
+    if (b.bytes >= bytes && b.ptr) return SN_OK;
+    dev_free(g, &b);
+    return dev_alloc(g, bytes, &b);
+}
+
+template <class F>
+sn_status time_median(int warm, int iters, cudaStream_t st, F launch, int64_t *ns_out) {
+    for (int i = 0; i < warm; ++i) {
+        sn_status rc = launch();
+        if (rc != SN_OK) return rc;
+    }
+    std::vector<cudaEvent_t> ev(2 * iters);
+    for (auto &e : ev) SN_CUDA_TRY(cudaEventCreate(&e));
+    sn_status rc = SN_OK;
+    for (int i = 0; i < iters && rc == SN_OK; ++i) {
+        cudaEventRecord(ev[2 * i], st);
+        rc = launch();
+        cudaEventRecord(ev[2 * i + 1], st);
+    }
+    cudaError_t e = cudaStreamSynchronize(st);
+    std::vector<float> ms;
+    if (rc == SN_OK && e == cudaSuccess)
+        for (int i = 0; i < iters; ++i) {
+            float t = 0;
+            cudaEventElapsedTime(&t, ev[2 * i], ev[2 * i + 1]);
+            ms.push_back(t);
+        }
+    for (auto &x : ev) cudaEventDestroy(x);
+    if (rc != SN_OK) return rc;
+    if (e != cudaSuccess) return fail(SN_ECUDA, std::string("profiling: ") + cudaGetErrorString(e));
+    std::sort(ms.begin(), ms.end());
+    const double med = iters % 2 ? ms[iters / 2] : 0.5 * (ms[iters / 2 - 1] + ms[iters / 2]);
+    *ns_out = std::max<int64_t>(1, (int64_t)(med * 1e6 + 0.5));
+    return SN_OK;
+}
+
+std::string signature(const Graph *g, int32_t i, const Candidate &c) {
+    const Layer &L = g->layers[i];
+    std::ostringstream o;
+    o << L.type << ':';
+    for (int32_t j : L.inputs) {
+        const Shape &s = g->layers[j].out;
+        o << s.n << 'x' << s.c << 'x' << s.h << 'x' << s.w << ';';
+    }
+    const sn_conv_params &p = L.conv;
+    o << p.c_in << ',' << p.c_out << ',' << p.kh << ',' << p.kw << ',' << p.sh << ',' << p.sw << ','
+      << p.ph << ',' << p.pw << ',' << p.dh << ',' << p.dw << ',' << p.groups << ',' << L.act << ','
+      << L.pool.kh << ',' << L.pool.sh << ',' << L.pool.ph << ',' << L.dense_in << ',' << L.dense_out
+      << '|' << c.routine << '/' << c.variant << '/' << c.schema;
+    return o.str();
+}
+
+}  // namespace
+
+sn_status profile_graph(Graph *g, const sn_profile_opts &o, cudaStream_t st) {
+    const int32_t n = g->n_layers(), ns = g->n_schemas();
+    size_t max_bytes = 0;
+    for (int32_t i = 0; i < n; ++i)
+        max_bytes = std::max(max_bytes, (size_t)g->layers[i].out.numel() * 4);
+    Scratch sc;
+    sn_status rc = SN_OK;
+    auto cleanup = [&]() {
+        dev_free(g, &sc.in0);
+        dev_free(g, &sc.in1);
+        dev_free(g, &sc.out);
+    };
+    if ((rc = ensure(g, sc.in0, max_bytes)) != SN_OK || (rc = ensure(g, sc.in1, max_bytes)) != SN_OK ||
+        (rc = ensure(g, sc.out, max_bytes)) != SN_OK) {
+        cleanup();
+        return rc;
+    }
+    // scratch inputs: small deterministic values (fp32 patterns reinterpreted
+    // per dtype are not needed: fill each dtype's worth of elements)
+    std::map<std::string, int64_t> seen;
+    // --- unit profiling of layer routines ---
+    for (int32_t i = 1; i < n - 1 && rc == SN_OK; ++i) {
+        const Layer &L = g->layers[i];
+        std::vector<Shape> in;
+        for (int32_t j : L.inputs) in.push_back(g->layers[j].out);
+        for (int32_t c = g->cand_begin[i]; c < g->cand_begin[i + 1] && rc == SN_OK; ++c) {
+            Candidate &cd = g->cands[c];
+            const std::string sig = signature(g, i, cd);
+            auto it = seen.find(sig);
+            if (it != seen.end()) {
+                cd.cost = it->second;
+                continue;
+            }
+            const sn_schema s = g->schemas[cd.schema];
+            LaunchArgs a;
+            a.g = g;
+            a.layer = &L;
+            a.routine = cd.routine;
+            a.variant = cd.variant;
+            a.schema = s;
+            a.in_shapes = in;
+            a.in[0] = sc.in0.ptr;
+            a.in[1] = sc.in1.ptr;
+            a.out = sc.out.ptr;
+            a.stream = st;
+            if (k::fill_pattern(sc.in0.ptr, s.dtype, in[0].numel(), 1234u + i, 1.0f, st) != cudaSuccess ||
+                (in.size() > 1 &&
+                 k::fill_pattern(sc.in1.ptr, s.dtype, in[1].numel(), 99u + i, 1.0f, st) != cudaSuccess)) {
+                rc = fail(SN_ECUDA, "profiling: fill failed");
+                break;
+            }
+            rc = prepare_weights(g, i, cd.routine, cd.variant, s, &a.wt, &a.bias, st);
+            if (rc != SN_OK) break;
+            const size_t ws = routine_workspace(cd.routine, cd.variant, L, in, s);
+            if (ws > g->workspace.bytes) {
+                invalidate_plan(g);
+                dev_free(g, &g->workspace);
+                if ((rc = dev_alloc(g, ws, &g->workspace)) != SN_OK) break;
+            }
+            a.ws = g->workspace.ptr;
+            a.ws_bytes = g->workspace.bytes;
+            int64_t t = kInf;
+            rc = time_median(o.warmup, o.iters, st, [&]() { return launch_routine(a); }, &t);
+            if (rc != SN_OK) break;
+            cd.cost = t;
+            seen.emplace(sig, t);
+        }
+    }
+    // --- unit profiling of adapt routines: every edge, every ordered pair ---
+    std::vector<int64_t> F;
+    std::vector<int32_t> argF;
+    fastest_per_schema(*g, F, argF);
+    std::map<std::string, int64_t> seen_a;
+    for (size_t e = 0; e < g->edges.size() && rc == SN_OK; ++e) {
+        auto [j, i] = g->edges[e];
+        const Shape s = g->layers[j].out;
+        for (int32_t a = 0; a < ns && rc == SN_OK; ++a) {
+            if (F[(size_t)j * ns + a] == kInf) continue;
+            for (int32_t b = 0; b < ns && rc == SN_OK; ++b) {
+                if (a == b || F[(size_t)i * ns + b] == kInf) continue;
+                std::ostringstream key;
+                key << s.n << 'x' << s.c << 'x' << s.h << 'x' << s.w << ':' << a << '>' << b;
+                auto it = seen_a.find(key.str());
+                if (it != seen_a.end()) {
+                    g->adapt((int32_t)e, a, b) = it->second;
+                    continue;
+                }
+                const sn_schema A = g->schemas[a], B = g->schemas[b];
+                if (k::fill_pattern(sc.in0.ptr, A.dtype, s.numel(), 7u, 1.0f, st) != cudaSuccess) {
+                    rc = fail(SN_ECUDA, "profiling: fill failed");
+                    break;
+                }
+                int64_t t = kInf;
+                rc = time_median(o.warmup, o.iters, st, [&]() -> sn_status {
+                    cudaError_t ce = k::convert(sc.in0.ptr, A.dtype, A.layout, sc.out.ptr, B.dtype,
+                                                B.layout, s, st);
+                    return ce == cudaSuccess ? SN_OK : fail(SN_ECUDA, cudaGetErrorString(ce));
+                }, &t);
+                if (rc != SN_OK) break;
+                g->adapt((int32_t)e, a, b) = t;
+                seen_a.emplace(key.str(), t);
+            }
+        }
+    }
+    cleanup();
+    if (rc != SN_OK) return rc;
+
+    // --- integrated profiling: top-k per (layer, schema) in whole-net passes ---
+    if (o.topk <= 0) return SN_OK;
+    const bool had_path = g->has_path;
+    const std::vector<int32_t> saved_path = g->path_cand;
+    const int64_t saved_total = g->path_total;
+    // ranked candidates per (layer, schema) by unit time
+    std::vector<std::vector<std::vector<int32_t>>> ranked(n, std::vector<std::vector<int32_t>>(ns));
+    for (int32_t i = 0; i < n; ++i) {
+        for (int32_t c = g->cand_begin[i]; c < g->cand_begin[i + 1]; ++c)
+            if (g->cands[c].cost != kInf) ranked[i][g->cands[c].schema].push_back(c);
+        for (auto &v : ranked[i])
+            std::stable_sort(v.begin(), v.end(), [&](int32_t x, int32_t y) {
+                return g->cands[x].cost < g->cands[y].cost;
+            });
+    }
+    Buffer xin, xout;
+    if ((rc = dev_alloc(g, (size_t)g->in_shape.numel() * dtype_size(g->in_schema.dtype), &xin)) != SN_OK)
+        return rc;
+    if ((rc = dev_alloc(g, (size_t)g->layers[n - 1].out.numel() * dtype_size(g->out_schema.dtype), &xout)) !=
+        SN_OK) {
+        dev_free(g, &xin);
+        return rc;
+    }
+    k::fill_pattern(xin.ptr, g->in_schema.dtype, g->in_shape.numel(), 5u, 1.0f, st);
+    std::vector<std::vector<float>> insitu(g->cands.size());
+    for (int32_t lam = 0; lam < g->n_lambda && rc == SN_OK; ++lam) {
+        for (int32_t r = 0; r < o.topk && rc == SN_OK; ++r) {
+            std::vector<int32_t> pc(n);
+            bool any = false;
+            for (int32_t i = 0; i < n; ++i) {
+                const auto &v = ranked[i][lam];
+                if (i == 0 || i == n - 1) {
+                    pc[i] = g->cand_begin[i];
+                } else if (!v.empty()) {
+                    pc[i] = v[std::min<size_t>(r, v.size() - 1)];
+                    any = any || (size_t)r < v.size();
+                } else {  // no routine in this schema: best overall
+                    int32_t best = g->cand_begin[i];
+                    for (int32_t c = g->cand_begin[i]; c < g->cand_begin[i + 1]; ++c)
+                        if (g->cands[c].cost < g->cands[best].cost) best = c;
+                    pc[i] = best;
+                }
+            }
+            if (!any) continue;
+            g->path_cand = pc;
+            g->has_path = true;
+            if ((rc = build_plan(g, st)) != SN_OK) break;
+            std::vector<cudaEvent_t> evs(2 * g->plan.size());
+            for (auto &e : evs) cudaEventCreate(&e);
+            std::vector<std::vector<float>> per_op(g->plan.size());
+            for (int32_t w = 0; w < o.warmup && rc == SN_OK; ++w)
+                rc = run_plan(g, xin.ptr, xout.ptr, st, nullptr);
+            for (int32_t p = 0; p < o.passes && rc == SN_OK; ++p) {
+                rc = run_plan(g, xin.ptr, xout.ptr, st, &evs);
+                if (rc != SN_OK) break;
+                if (cudaStreamSynchronize(st) != cudaSuccess) {
+                    rc = fail(SN_ECUDA, "integrated profiling: stream failed");
+                    break;
+                }
+                for (size_t q = 0; q < g->plan.size(); ++q) {
+                    float t = 0;
+                    cudaEventElapsedTime(&t, evs[2 * q], evs[2 * q + 1]);
+                    per_op[q].push_back(t);
+                }
+            }
+            for (auto &e : evs) cudaEventDestroy(e);
+            if (rc != SN_OK) break;
+            for (size_t q = 0; q < g->plan.size(); ++q) {
+                const PlanOp &op = g->plan[q];
+                if (op.kind != PlanOp::LAYER) continue;
+                auto v = per_op[q];
+                std::sort(v.begin(), v.end());
+                insitu[op.cand].push_back(v[v.size() / 2]);
+            }
+        }
+    }
+    dev_free(g, &xin);
+    dev_free(g, &xout);
+    for (size_t c = 0; c < insitu.size(); ++c) {
+        if (insitu[c].empty()) continue;
+        auto v = insitu[c];
+        std::sort(v.begin(), v.end());
+        g->cands[c].cost = std::max<int64_t>(1, (int64_t)(v[v.size() / 2] * 1e6 + 0.5));
+    }
+    g->has_path = had_path;
+    g->path_cand = saved_path;
+    g->path_total = saved_total;
+    invalidate_plan(g);
+    return rc;
+}
+
+}  // namespace sn

@@ -1,0 +1,227 @@
+// Internal declarations of the routine-selecting inference core.
+#pragma once
+
+#include <cuda_runtime.h>
+
+#include <cstdint>
+#include <map>
+#include <memory>
+#include <string>
+#include <vector>
+
+#include "../../include/sn.h"
+
+namespace sn {
+
+constexpr int64_t kInf = INT64_MAX;
+
+inline int64_t sat_add(int64_t a, int64_t b) { return (a == kInf || b == kInf) ? kInf : a + b; }
+
+// -------------------------------------------------------------------------
+// error reporting
+// -------------------------------------------------------------------------
+struct Error {
+    sn_status status;
+    std::string msg;
+};
+void set_error(const std::string &msg);
+sn_status fail(sn_status s, const std::string &msg);
+#define SN_CUDA_TRY(expr)                                                              \
+    do {                                                                               \
+        cudaError_t _e = (expr);                                                       \
+        if (_e != cudaSuccess)                                                         \
+            return ::sn::fail(SN_ECUDA, std::string(#expr) + ": " + cudaGetErrorString(_e)); \
+    } while (0)
+
+// -------------------------------------------------------------------------
+// tensors
+// -------------------------------------------------------------------------
+struct Shape {
+    int64_t n = 0, c = 0, h = 0, w = 0;
+    int64_t numel() const { return n * c * h * w; }
+    bool operator==(const Shape &o) const { return n == o.n && c == o.c && h == o.h && w == o.w; }
+};
+
+inline int dtype_size(int dt) { return dt == SN_F32 ? 4 : 2; }
+inline bool schema_eq(sn_schema a, sn_schema b) { return a.dtype == b.dtype && a.layout == b.layout; }
+inline bool schema_valid(sn_schema s) {
+    return s.dtype >= SN_F32 && s.dtype <= SN_BF16 && s.layout >= SN_NCHW && s.layout <= SN_NHWC;
+}
+std::string schema_str(sn_schema s);
+
+// -------------------------------------------------------------------------
+// routine registry (section III-C: routines, descriptors, routine parameters)
+// -------------------------------------------------------------------------
+enum RoutineId : int32_t {
+    R_IO = 0,            // auxiliary input/output layer, zero cost (section IV-E)
+    R_CONV_DIRECT = 1,   // direct convolution, one output per thread
+    R_CONV_IGEMM = 2,    // implicit GEMM on CUDA cores (FFMA), register-tiled
+    R_CONV_WINO = 3,     // Winograd F(2x2,3x3) childnet: wgenc -> wgconv -> wgdec
+    R_CONV_TC = 4,       // implicit GEMM on tcgen05 tensor cores, TMA-fed (NHWC)
+    R_DW_DIRECT = 5,     // depthwise conv
+    R_MAXPOOL = 6,
+    R_GAP = 7,
+    R_ADD = 8,
+    R_DENSE = 9,         // dense on CUDA cores
+    R_ADAPT = 10,        // adapt layer (cast / layout change)
+    R_COUNT = 11
+};
+
+// -------------------------------------------------------------------------
+// graph (section III-B)
+// -------------------------------------------------------------------------
+struct Layer {
+    int32_t type = -1;         // sn_layer_type, or -1 = input aux, -2 = output aux
+    sn_conv_params conv{};     // CONV2 / DWCONV2
+    sn_pool_params pool{};     // MAXPOOL
+    int32_t act = SN_ACT_NONE; // ADD / DENSE / CONV
+    int32_t dense_in = 0, dense_out = 0;
+    std::vector<int32_t> inputs;  // internal layer indices
+    Shape out;
+    std::vector<float> weight, bias;  // host fp32 copies
+};
+
+struct Candidate {
+    int32_t routine, variant, schema, layer;
+    int64_t cost;
+};
+
+struct Buffer {  // device allocation owned by the graph
+    void *ptr = nullptr;
+    size_t bytes = 0;
+};
+
+struct PlanOp {
+    enum Kind { LAYER, ADAPT } kind;
+    int32_t layer = -1;    // LAYER: internal layer; ADAPT: consumer layer
+    int32_t edge = -1;     // ADAPT: edge index
+    int32_t cand = -1;     // LAYER: candidate index
+    std::vector<int32_t> in_slots;
+    int32_t out_slot = -1;
+    const void *wt = nullptr;      // LAYER: prepared weights
+    const float *bias = nullptr;   // LAYER: fp32 bias
+};
+
+struct Graph;
+
+// A launchable routine instance: everything a kernel needs, resolved.
+struct LaunchArgs {
+    const Graph *g;
+    const Layer *layer;
+    int32_t routine, variant;
+    sn_schema schema;
+    std::vector<Shape> in_shapes;
+    const void *in[2] = {nullptr, nullptr};
+    void *out = nullptr;
+    const void *wt = nullptr;   // prepared weights in the routine's format
+    const float *bias = nullptr;
+    void *ws = nullptr;         // workspace
+    size_t ws_bytes = 0;
+    cudaStream_t stream = nullptr;
+};
+
+struct Graph {
+    Shape in_shape;
+    sn_schema in_schema{}, out_schema{};
+    std::vector<sn_schema> schemas;   // universe: Lambda, then in/out if absent
+    int32_t n_lambda = 0;             // |Lambda| (first entries of `schemas`)
+    int32_t in_schema_idx = 0, out_schema_idx = 0;
+    sn_alloc_fn alloc = nullptr;
+    sn_free_fn free_fn = nullptr;
+    void *alloc_ctx = nullptr;
+
+    std::vector<Layer> user;          // as added
+    bool finalized = false;
+    std::vector<Layer> layers;        // internal: [input, user..., output]
+    std::vector<std::pair<int32_t, int32_t>> edges;
+    std::vector<Candidate> cands;     // grouped by layer
+    std::vector<int32_t> cand_begin;  // [n_layers + 1]
+    std::vector<int64_t> adapt_cost;  // [n_edges][ns][ns]
+
+    bool has_path = false;
+    std::vector<int32_t> path_cand;   // per layer
+    int64_t path_total = kInf;
+
+    // plan (built lazily by sn_run)
+    bool plan_valid = false;
+    std::vector<PlanOp> plan;
+    std::vector<Buffer> slots;        // activation buffers; slot 0 = in, 1 = out (external)
+    std::vector<Shape> slot_shape;
+    std::vector<sn_schema> slot_schema;
+    std::map<std::string, Buffer> weight_cache;  // key: layer/format/dtype
+    std::map<int32_t, Buffer> bias_cache;        // per layer fp32 bias
+    Buffer workspace;
+    int opt_graph = 0, opt_check = 0;
+    cudaGraphExec_t gexec = nullptr;
+    const void *gexec_in = nullptr;
+    void *gexec_out = nullptr;
+    cudaStream_t gexec_stream = nullptr;
+
+    ~Graph();
+    int32_t n_layers() const { return (int32_t)layers.size(); }
+    int32_t n_schemas() const { return (int32_t)schemas.size(); }
+    int64_t &adapt(int32_t e, int32_t a, int32_t b) {
+        return adapt_cost[((size_t)e * schemas.size() + a) * schemas.size() + b];
+    }
+    int64_t adapt(int32_t e, int32_t a, int32_t b) const {
+        return adapt_cost[((size_t)e * schemas.size() + a) * schemas.size() + b];
+    }
+};
+
+sn_status graph_finalize(Graph *g);
+sn_status dev_alloc(Graph *g, size_t bytes, Buffer *b);
+void dev_free(Graph *g, Buffer *b);
+void invalidate_plan(Graph *g);
+
+// routine applicability: variants of `routine` that can serve `layer` in `s`
+int32_t routine_variants(int32_t routine, const Layer &layer, const std::vector<Shape> &in,
+                         sn_schema s);
+const char *routine_name(int32_t routine);
+const char *variant_name(int32_t routine, int32_t variant);
+size_t routine_workspace(int32_t routine, int32_t variant, const Layer &layer,
+                         const std::vector<Shape> &in, sn_schema s);
+// prepare weights for (layer, routine, variant, schema); returns device pointer
+sn_status prepare_weights(Graph *g, int32_t li, int32_t routine, int32_t variant, sn_schema s,
+                          const void **wt, const float **bias, cudaStream_t st);
+sn_status launch_routine(const LaunchArgs &a);
+
+// selection (section IV)
+sn_status select_dprs(const Graph &g, std::vector<int32_t> &schema_of, int64_t &total);
+sn_status select_brute(const Graph &g, std::vector<int32_t> &schema_of, int64_t &total);
+void fastest_per_schema(const Graph &g, std::vector<int64_t> &F, std::vector<int32_t> &argF);
+
+// plan + run
+sn_status build_plan(Graph *g, cudaStream_t st);
+sn_status run_plan(Graph *g, const void *in, void *out, cudaStream_t st,
+                   std::vector<cudaEvent_t> *evs);
+sn_status profile_graph(Graph *g, const sn_profile_opts &o, cudaStream_t st);
+
+// -------------------------------------------------------------------------
+// kernels (launchers; all asynchronous on `st`)
+// -------------------------------------------------------------------------
+namespace k {
+cudaError_t convert(const void *x, int dt_in, int lay_in, void *y, int dt_out, int lay_out,
+                    Shape s, cudaStream_t st);
+cudaError_t fill_pattern(void *y, int dt, int64_t n, uint32_t seed, float scale,
+                         cudaStream_t st);
+// weight re-layout / cast from fp32 KCRS (device) into a routine format
+enum WFormat { W_KCRS = 0, W_RSCK = 1, W_KRSC = 2, W_WINO = 3 };
+cudaError_t weight_format(const float *w_kcrs, void *out, int fmt, int dt, int64_t K,
+                          int64_t Cg, int64_t R, int64_t S, cudaStream_t st);
+
+cudaError_t conv_direct(const LaunchArgs &a);
+cudaError_t conv_igemm(const LaunchArgs &a);
+cudaError_t conv_wino(const LaunchArgs &a);
+size_t conv_wino_ws(const Layer &l, const Shape &in, sn_schema s);
+cudaError_t conv_tc(const LaunchArgs &a);
+int32_t conv_tc_variants(const Layer &l, const Shape &in, sn_schema s);
+const char *conv_tc_variant_name(int32_t v);
+cudaError_t dwconv(const LaunchArgs &a);
+cudaError_t maxpool(const LaunchArgs &a);
+cudaError_t gap(const LaunchArgs &a);
+cudaError_t add(const LaunchArgs &a);
+cudaError_t dense(const LaunchArgs &a);
+int *device_error_word();  // device address of the library's error word
+}  // namespace k
+
+}  // namespace sn

@@ -1,0 +1,135 @@
+"""End-to-end on the GPU: profile -> DPRS -> run, against the oracle.
+
+  * tiny CNN, fp32 (routine paths small enough to enumerate): the DPRS path on
+    the profiled cost table equals the oracle's exhaustive search, and the
+    output matches the oracle within 1e-4; random forced paths (mixed
+    schemas, adapts on edges) match as well.
+  * MobileNetV2 b1 fp16, ResNet-50 b1 fp16: DPRS equals the oracle's exact
+    block-wise search on the profiled table; output within 2e-2.
+  * ResNet-50 b32 bf16: sampled images of the batch against the oracle.
+"""
+import numpy as np
+import pytest
+
+import oracle
+import synth
+from oracle.net import run_net
+from oracle.paths import blockwise_search
+from paper_2110_06037_gb300 import SN_OPT_CUDA_GRAPH, SN_SELECT_BRUTE, SN_SELECT_DPRS, build_graph
+
+from gpu_helpers import TOL, from_device, maxrel, to_device
+from test_dprs import oracle_layer_cost
+
+pytestmark = pytest.mark.gpu
+
+F32 = [("f32", "nchw"), ("f32", "nhwc")]
+F16 = [("f16", "nchw"), ("f16", "nhwc")]
+BF16 = [("bf16", "nchw"), ("bf16", "nhwc")]
+
+
+def _profile_select_run(layers, x, in_schema, out_schema, schemas, exhaustive, warmup=1, iters=5):
+    import torch
+    g = build_graph(layers, x.shape, in_schema, out_schema, schemas)
+    g.profile(warmup=warmup, iters=iters, topk=2, passes=3)
+    t = g.cost_table()
+    lc = oracle_layer_cost(t)
+    if exhaustive:
+        ref_total, ref_asg, nmin = oracle.brute_force(lc, t["edges"], t["adapt"])
+    else:
+        ref_total, ref_asg = blockwise_search(lc, t["edges"], t["adapt"])
+        nmin = None
+    total, sch, cand = g.select_path(SN_SELECT_DPRS)
+    assert total == ref_total
+    assert oracle.path_cost(lc, t["edges"], t["adapt"], sch) == ref_total
+    if nmin == 1:
+        assert list(sch) == list(ref_asg)
+    y = g.run(to_device(x, in_schema))
+    torch.cuda.synchronize()
+    return g, from_device(y, out_schema)
+
+
+def test_tiny_cnn_fp32_profile_dprs_run():
+    x, layers = synth.tiny_cnn()
+    g, got = _profile_select_run(layers, x, ("f32", "nchw"), ("f32", "nchw"), F32, exhaustive=True)
+    total_b, _, _ = g.select_path(SN_SELECT_BRUTE)
+    total_d, _, _ = g.select_path(SN_SELECT_DPRS)
+    assert total_b == total_d
+    ref = run_net(layers, x, "f32")
+    assert maxrel(got, ref) <= TOL["f32"]
+
+
+def test_tiny_cnn_random_forced_paths():
+    import torch
+    x, layers = synth.tiny_cnn()
+    ref = run_net(layers, x, "f32")
+    g = build_graph(layers, x.shape, ("f32", "nchw"), ("f32", "nhwc"), F32)
+    t = g.cost_table()
+    rng = np.random.default_rng(0)
+    xd = to_device(x, ("f32", "nchw"))
+    for _ in range(12):
+        pc = [int(rng.choice(np.flatnonzero(t["layer"] == i))) for i in range(t["n_layers"])]
+        g.set_path(pc)
+        y = g.run(xd)
+        torch.cuda.synchronize()
+        assert maxrel(from_device(y, ("f32", "nhwc")), ref) <= TOL["f32"]
+
+
+def test_mixed_precision_schemas_tiny():
+    """fp16 and fp32 schemas in one net: adapts cast between them."""
+    import torch
+    x, layers = synth.tiny_cnn()
+    sch = [("f32", "nchw"), ("f16", "nhwc")]
+    g = build_graph(layers, x.shape, ("f32", "nchw"), ("f32", "nchw"), sch)
+    t = g.cost_table()
+    rng = np.random.default_rng(1)
+    xd = to_device(x, ("f32", "nchw"))
+    ref = run_net(layers, x, "f32")
+    for _ in range(6):
+        pc = [int(rng.choice(np.flatnonzero(t["layer"] == i))) for i in range(t["n_layers"])]
+        g.set_path(pc)
+        y = g.run(xd)
+        torch.cuda.synchronize()
+        assert maxrel(from_device(y, ("f32", "nchw")), ref) <= TOL["f16"]
+
+
+def test_mobilenet_v2_b1_fp16():
+    x, layers = synth.mobilenet_v2(1)
+    g, got = _profile_select_run(layers, x, ("f16", "nchw"), ("f16", "nchw"), F16, exhaustive=False)
+    ref = run_net(layers, x, "f16")
+    assert maxrel(got, ref) <= TOL["f16"]
+
+
+def test_resnet50_b1_fp16_and_graph_replay():
+    import torch
+    x, layers = synth.resnet50(1)
+    g, got = _profile_select_run(layers, x, ("f16", "nchw"), ("f16", "nchw"), F16, exhaustive=False)
+    ref = run_net(layers, x, "f16")
+    assert maxrel(got, ref) <= TOL["f16"]
+    # CUDA-graph replay gives the same bits as eager launches
+    xd = to_device(x, ("f16", "nchw"))
+    s = torch.cuda.Stream()
+    with torch.cuda.stream(s):
+        y1 = g.run(xd)
+        g.set_option(SN_OPT_CUDA_GRAPH, 1)
+        y2 = g.run(xd)
+        y3 = g.run(xd)
+    s.synchronize()
+    assert torch.equal(y1, y2) and torch.equal(y2, y3)
+
+
+def test_resnet50_b32_bf16_sampled():
+    import torch
+    x, layers = synth.resnet50(32)
+    g = build_graph(layers, x.shape, ("bf16", "nchw"), ("bf16", "nchw"), BF16)
+    g.profile(warmup=1, iters=3, topk=1, passes=2)
+    t = g.cost_table()
+    lc = oracle_layer_cost(t)
+    ref_total, _ = blockwise_search(lc, t["edges"], t["adapt"])
+    total, sch, _ = g.select_path(SN_SELECT_DPRS)
+    assert total == ref_total
+    y = g.run(to_device(x, ("bf16", "nchw")))
+    torch.cuda.synchronize()
+    got = from_device(y, ("bf16", "nchw"))
+    for n in (0, 31):
+        ref = run_net(layers, x[n:n + 1], "bf16")
+        assert maxrel(got[n:n + 1], ref) <= TOL["bf16"]

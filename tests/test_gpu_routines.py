@@ -1,0 +1,145 @@
+"""Per-routine parity on the GPU through the C ABI: every routine of every
+layer type, in every schema it serves, against the oracle on the same stored
+inputs.  Adapt conversions are checked bit for bit."""
+import numpy as np
+import pytest
+
+import oracle
+import synth
+from oracle.net import run_layer
+from paper_2110_06037_gb300 import build_graph, convert
+
+from gpu_helpers import TOL, find_candidate, from_device, maxrel, raw_bits, stored_values, to_device
+
+pytestmark = pytest.mark.gpu
+
+DTS = ("f32", "f16", "bf16")
+LAYS = ("nchw", "nhwc")
+SCHEMAS = [(d, l) for d in DTS for l in LAYS]
+
+
+def run_one(layer, x, schema, routine, variant):
+    """Build a one-layer net in `schema`, force (routine, variant), run, return fp64 NCHW."""
+    import torch
+    spec = dict(layer)
+    spec["inputs"] = [-1] * (2 if layer["type"] == "add" else 1)
+    g = build_graph([spec], x.shape, schema, schema, [schema])
+    t = g.cost_table()
+    c = find_candidate(t, 1, routine, variant, 0)
+    if c is None:
+        return None
+    cands = [int(np.flatnonzero(t["layer"] == 0)[0]), c, int(np.flatnonzero(t["layer"] == 2)[0])]
+    g.set_path(cands)
+    xd = to_device(x, schema)
+    y = g.run(xd)
+    torch.cuda.synchronize()
+    return from_device(y, schema)
+
+
+def ref_one(layer, x, dt):
+    xs = stored_values(x, dt)
+    ins = [xs, xs] if layer["type"] == "add" else [xs]
+    return run_layer(layer, ins, dt)
+
+
+CONV_CASES = [
+    # N, C, H, W, K, k, s, p, d, groups
+    (1, 3, 32, 32, 16, 3, 1, 1, 1, 1),
+    (1, 16, 32, 32, 32, 3, 2, 1, 1, 1),
+    (2, 24, 9, 11, 40, 3, 1, 1, 1, 1),     # ragged tiles
+    (1, 64, 14, 14, 64, 1, 1, 0, 1, 1),
+    (2, 32, 7, 7, 48, 1, 2, 0, 1, 1),
+    (1, 8, 10, 10, 8, 3, 1, 1, 1, 2),      # groups
+    (1, 3, 23, 23, 16, 7, 2, 3, 1, 1),     # stem-like 7x7 s2
+    (1, 8, 12, 12, 8, 3, 1, 2, 2, 1),      # dilation
+    (1, 130, 5, 5, 66, 3, 1, 1, 1, 1),     # channels past a tile edge
+    (1, 16, 1, 1, 8, 3, 1, 1, 1, 1),       # 1x1 image, 3x3 kernel (padding only)
+]
+ROUTINES = [("conv2/direct", 0), ("conv2/igemm_simt", 0), ("conv2/igemm_simt", 1), ("conv2/wino_f2x2_3x3", 0)]
+
+
+@pytest.mark.parametrize("case", CONV_CASES)
+@pytest.mark.parametrize("schema", SCHEMAS)
+def test_conv_routines(case, schema):
+    N, C, H, W, K, k, s, p, d, g = case
+    rng = np.random.default_rng(abs(hash((case, schema))) % 2**32)
+    x = rng.standard_normal((N, C, H, W)).astype(np.float32)
+    layer = synth.conv(C, K, k, s, p, act="relu", groups=g, d=d)
+    layer["weight"] = (rng.standard_normal((K, C // g, k, k)) * np.sqrt(2.0 / (C // g * k * k))).astype(np.float32)
+    layer["bias"] = (rng.standard_normal(K) * 0.1).astype(np.float32)
+    ref = ref_one(layer, x, schema[0])
+    ran = 0
+    for rname, v in ROUTINES:
+        got = run_one(layer, x, schema, rname, v)
+        if got is None:
+            continue
+        ran += 1
+        err = maxrel(got, ref)
+        assert err <= TOL[schema[0]], (rname, v, err)
+    assert ran >= 1
+
+
+DW_CASES = [(1, 32, 16, 16, 1), (2, 24, 9, 9, 2), (1, 144, 28, 28, 1), (1, 40, 7, 7, 2), (1, 8, 1, 1, 1)]
+
+
+@pytest.mark.parametrize("case", DW_CASES)
+@pytest.mark.parametrize("schema", SCHEMAS)
+def test_depthwise(case, schema):
+    N, C, H, W, s = case
+    rng = np.random.default_rng(abs(hash((case, schema))) % 2**32)
+    x = rng.standard_normal((N, C, H, W)).astype(np.float32)
+    layer = synth.dwconv(C, 3, s, act="relu6")
+    layer["weight"] = (rng.standard_normal((C, 1, 3, 3)) * np.sqrt(2 / 9)).astype(np.float32)
+    layer["bias"] = (rng.standard_normal(C) * 0.1).astype(np.float32)
+    got = run_one(layer, x, schema, "dwconv2/direct", 0)
+    assert maxrel(got, ref_one(layer, x, schema[0])) <= TOL[schema[0]]
+
+
+@pytest.mark.parametrize("schema", SCHEMAS)
+def test_pool_gap_add_dense(schema):
+    rng = np.random.default_rng(3)
+    x = rng.standard_normal((2, 16, 13, 11)).astype(np.float32)
+    mp = synth.maxpool(3, 2, 1)
+    got = run_one(mp, x, schema, "maxpool/direct", 0)
+    # max pooling selects a stored value: exact
+    assert np.array_equal(got, ref_one(mp, x, schema[0]))
+    gp = synth.gap()
+    assert maxrel(run_one(gp, x, schema, "gap/reduce", 0), ref_one(gp, x, schema[0])) <= TOL[schema[0]]
+    ad = synth.add(act="relu")
+    assert maxrel(run_one(ad, x, schema, "add/eltwise", 0), ref_one(ad, x, schema[0])) <= TOL[schema[0]]
+    xd = rng.standard_normal((3, 70, 1, 1)).astype(np.float32)
+    de = synth.dense(70, 33)
+    de["weight"] = (rng.standard_normal((33, 70)) * 0.2).astype(np.float32)
+    de["bias"] = (rng.standard_normal(33) * 0.1).astype(np.float32)
+    assert maxrel(run_one(de, xd, schema, "dense/simt", 0), ref_one(de, xd, schema[0])) <= TOL[schema[0]]
+
+
+CONVERT_SHAPES = [(2, 5, 7, 9), (1, 64, 56, 56), (3, 130, 1, 1), (1, 3, 65, 67)]
+
+
+@pytest.mark.parametrize("shape", CONVERT_SHAPES)
+def test_convert_bit_exact(shape):
+    import torch
+    rng = np.random.default_rng(11)
+    x = (rng.standard_normal(shape) * 3).astype(np.float32)
+    flat = x.reshape(-1)
+    flat[: min(6, flat.size)] = np.array([7e4, -1e5, 3e-8, -6e-6, 65520.0, 0.0], np.float32)[: min(6, flat.size)]
+    for d_in in DTS:
+        for l_in in LAYS:
+            xd = to_device(x, (d_in, l_in))
+            vin = stored_values(x, d_in).astype(np.float32)
+            for d_out in DTS:
+                for l_out in LAYS:
+                    y = convert(xd, (d_in, l_in), (d_out, l_out), shape)
+                    torch.cuda.synchronize()
+                    ref = oracle.to_bits(vin, d_out)
+                    if l_out == "nhwc":
+                        ref = oracle.nchw_to_nhwc(ref)
+                    got = raw_bits(y).reshape(ref.shape)
+                    assert np.array_equal(got, ref.view(got.dtype)), (d_in, l_in, d_out, l_out)
+
+
+def test_convert_empty_is_noop():
+    import torch
+    x = torch.zeros(4, device="cuda")
+    convert(x, ("f32", "nchw"), ("f16", "nhwc"), (0, 3, 4, 4), out=torch.zeros(1, device="cuda", dtype=torch.float16))

@@ -1,0 +1,113 @@
+"""Host-side behaviour of the C ABI: validation, call order, cost-table and
+plan-file round trips.  CPU only (no kernel is launched)."""
+import numpy as np
+import pytest
+
+import synth
+from paper_2110_06037_gb300 import SN_SELECT_DPRS, SnError, build_graph, _sn
+from paper_2110_06037_gb300.api import Graph
+
+S2 = [("f32", "nchw"), ("f32", "nhwc")]
+
+
+def tiny():
+    x, layers = synth.tiny_cnn()
+    return x, build_graph(layers, x.shape, ("f32", "nchw"), ("f32", "nchw"), S2, torch_alloc=False)
+
+
+def test_shapes_and_candidates():
+    x, g = tiny()
+    t = g.cost_table()
+    assert t["n_layers"] == 8 and t["n_schemas"] == 2
+    assert g.layer_shape(1) == (1, 16, 32, 32)
+    assert g.layer_shape(2) == (1, 32, 16, 16)
+    assert g.layer_shape(6) == (1, 10, 1, 1)
+    assert g.layer_shape(7) == (1, 10, 1, 1)
+    # Winograd only on the 3x3 stride-1 conv, tensor cores never in fp32
+    names = {(int(t["layer"][c]), _sn.routine_name(int(t["routine"][c]))) for c in range(len(t["cost"]))}
+    assert (1, "conv2/wino_f2x2_3x3") in names and (2, "conv2/wino_f2x2_3x3") not in names
+    assert not any(n == "conv2/igemm_tc" for _, n in names)
+    assert np.all(t["cost"][t["routine"] != 0] == _sn.COST_INF)
+
+
+def test_invalid_layers_rejected():
+    g = Graph((1, 3, 8, 8), ("f32", "nchw"), ("f32", "nchw"), S2, torch_alloc=False)
+    bad = dict(c_in=4, c_out=8, kh=3, kw=3, sh=1, sw=1, ph=1, pw=1)
+    with pytest.raises(SnError) as e:
+        g.add_layer(_sn.SN_L_CONV2, bad, (-1,), np.zeros((8, 4, 3, 3)), None)
+    assert e.value.status == _sn.SN_EINVAL
+    with pytest.raises(SnError):
+        g.add_layer(_sn.SN_L_CONV2, dict(bad, c_in=3), (5,), np.zeros((8, 3, 3, 3)), None)
+    with pytest.raises(SnError):
+        g.add_layer(_sn.SN_L_CONV2, dict(bad, c_in=3, kh=11, ph=0), (-1,), np.zeros((8, 3, 11, 3)), None)
+    with pytest.raises(SnError):
+        g.add_layer(_sn.SN_L_DENSE, dict(in_features=3, out_features=2), (-1,), np.zeros((2, 3)), None)
+    l0 = g.add_layer(_sn.SN_L_CONV2, dict(bad, c_in=3), (-1,), np.zeros((8, 3, 3, 3)), None)
+    with pytest.raises(SnError):  # shapes differ
+        g.add_layer(_sn.SN_L_ADD, {"act": "none"}, (-1, l0))
+
+
+def test_dead_end_layer_is_rejected():
+    g = Graph((1, 4, 4, 4), ("f32", "nchw"), ("f32", "nchw"), S2, torch_alloc=False)
+    p = dict(c_in=4, c_out=4, kh=1, kw=1, sh=1, sw=1, ph=0, pw=0)
+    g.add_layer(_sn.SN_L_CONV2, p, (-1,), np.zeros((4, 4, 1, 1)), None)
+    g.add_layer(_sn.SN_L_CONV2, p, (-1,), np.zeros((4, 4, 1, 1)), None)  # layer 0 is now a dead end
+    with pytest.raises(SnError) as e:
+        g.cost_table()
+    assert e.value.status == _sn.SN_EINVAL
+
+
+def test_call_order():
+    x, g = tiny()
+    with pytest.raises(SnError) as e:
+        _sn.check(_sn.lib().sn_run(g.h, 1, 1, None))
+    assert e.value.status == _sn.SN_ESTATE
+    with pytest.raises(SnError) as e:  # all costs unknown -> infeasible
+        g.select_path(SN_SELECT_DPRS)
+    assert e.value.status == _sn.SN_EINFEASIBLE
+    with pytest.raises(SnError) as e:  # finalised: no more layers
+        g.add_layer(_sn.SN_L_GAP, None, (0,))
+    assert e.value.status == _sn.SN_ESTATE
+
+
+def test_cost_table_validation_and_roundtrip(tmp_path):
+    x, g = tiny()
+    t = g.cost_table()
+    rng = np.random.default_rng(0)
+    t["cost"] = np.where(t["routine"] == 0, 0, rng.integers(1, 100, len(t["cost"]))).astype(np.int64)
+    a = rng.integers(1, 50, t["adapt"].shape).astype(np.int64)
+    for e in range(a.shape[0]):
+        np.fill_diagonal(a[e], 0)
+    t["adapt"] = a
+    g.set_cost_table(t)
+    t2 = g.cost_table()
+    assert np.array_equal(t2["cost"], t["cost"]) and np.array_equal(t2["adapt"], a)
+    bad = dict(t)
+    bad["adapt"] = a.copy()
+    bad["adapt"][0, 0, 0] = 5  # void adapt must be 0
+    with pytest.raises(SnError):
+        g.set_cost_table(bad)
+    bad = dict(t)
+    bad["schema"] = t["schema"].copy()
+    bad["schema"][3] ^= 1
+    with pytest.raises(SnError):
+        g.set_cost_table(bad)
+    assert np.array_equal(g.cost_table()["cost"], t["cost"])  # unchanged after errors
+    tot, sch, cand = g.select_path(SN_SELECT_DPRS)
+    p = tmp_path / "plan.json"
+    g.save_plan(p)
+    x2, g2 = tiny()
+    g2.load_plan(p)
+    t3 = g2.cost_table()
+    assert np.array_equal(t3["cost"], t["cost"]) and np.array_equal(t3["adapt"], a)
+    g2.save_plan(tmp_path / "plan2.json")
+    assert open(p).read() == open(tmp_path / "plan2.json").read()
+
+
+def test_set_path_validation():
+    x, g = tiny()
+    t = g.cost_table()
+    with pytest.raises(SnError):
+        g.set_path(np.zeros(t["n_layers"], np.int32))  # candidate 0 belongs to layer 0 only
+    first = [int(np.flatnonzero(t["layer"] == i)[0]) for i in range(t["n_layers"])]
+    g.set_path(first)
