@@ -1,0 +1,376 @@
+"""Benchmark: ResNet-50 inference with the DPRS-selected routine path on GB300.
+
+One step = one inference of a 32 x 3 x 224 x 224 bf16 batch through the whole
+routine path (every layer routine and adapt), replayed as a CUDA graph.
+Tuning (profiling + DPRS) runs once before the timed region and is reported
+separately.  Inputs are seeded synthetic tensors shaped like the paper's
+workloads (no trained weights or datasets are available).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+--impl reference times the CPU oracle (plain fp64) on the same workload and
+metric, one image per step as a bounded sample.  Multi-GPU: independent
+replicas (one batch per rank, no collective on the data path).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+METRIC = "ResNet-50 b1 latency (ms), b32 images/s; conv TFLOP/s & GB/s vs peak"
+WORKLOAD = "ResNet-50 v1.5 inference, batch 32, 3x224x224 bf16, DPRS path over {bf16 NCHW, bf16 NHWC}"
+FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0, "sm_max_mhz": 2070.0}
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return d, "measured"
+    return FALLBACK, "fallback"
+
+
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled during the timed region."""
+    Q = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+         "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+         "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.Q}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if not self.proc:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for l in self.lines:
+            f = [x.strip() for x in l.split(",")]
+            if len(f) < 7:
+                continue
+            try:
+                sm.append(float(f[0]))
+                mx.append(float(f[1]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[3:7]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def conv_work(layers, in_shape, elem=2):
+    """Algorithmic FLOPs and bytes of every layer (inputs, weights, output once)."""
+    shapes = []
+    work = []
+    for l in layers:
+        ins = [in_shape if j < 0 else shapes[j] for j in l["inputs"]]
+        n, c, h, w = ins[0]
+        p = l["params"]
+        if l["type"] in ("conv2", "dwconv2"):
+            g = p["groups"]
+            P = (h + 2 * p["ph"] - p.get("dh", 1) * (p["kh"] - 1) - 1) // p["sh"] + 1
+            Q = (w + 2 * p["pw"] - p.get("dw", 1) * (p["kw"] - 1) - 1) // p["sw"] + 1
+            K = p["c_out"]
+            out = (n, K, P, Q)
+            fl = 2 * n * K * P * Q * (c // g) * p["kh"] * p["kw"]
+            by = elem * (n * c * h * w + n * K * P * Q + K * (c // g) * p["kh"] * p["kw"]) + 4 * K
+        elif l["type"] == "maxpool":
+            P = (h + 2 * p["ph"] - p["kh"]) // p["sh"] + 1
+            Q = (w + 2 * p["pw"] - p["kw"]) // p["sw"] + 1
+            out = (n, c, P, Q)
+            fl, by = 0, elem * (n * c * h * w + n * c * P * Q)
+        elif l["type"] == "gap":
+            out = (n, c, 1, 1)
+            fl, by = n * c * h * w, elem * (n * c * h * w + n * c)
+        elif l["type"] == "add":
+            out = ins[0]
+            fl, by = n * c * h * w, 3 * elem * n * c * h * w
+        else:  # dense
+            out = (n, p["out_features"], 1, 1)
+            fl = 2 * n * p["in_features"] * p["out_features"]
+            by = elem * (n * p["in_features"] + n * p["out_features"] + p["in_features"] * p["out_features"])
+        shapes.append(out)
+        work.append((fl, by))
+    return work, shapes
+
+
+def run_reference(args, ws, rank):
+    """The CPU oracle on the same workload: one image per step (bounded sample)."""
+    if rank != 0:
+        return
+    import synth
+    from oracle.net import run_net
+    x, layers = synth.resnet50(32)
+    xs = x[:1]
+    for _ in range(max(0, args.warmup and 1)):
+        run_net(layers, xs, "bf16")
+    times = []
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        run_net(layers, xs, "bf16")
+        times.append(time.perf_counter() - t0)
+    sec = sum(times) / len(times)
+    v = 1.0 / sec
+    cores = os.cpu_count()
+    line = {"impl": "reference", "metric": METRIC, "value": v, "unit": "images/s", "n_gpus": ws,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": sec * 1e3, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": WORKLOAD + " (oracle: 1 image per step)", "batch": 32},
+            "cpu_baseline": {"value": v, "unit": "images/s", "cores": cores, "kind": "oracle",
+                             "sample": "1 of the 32 images per step, fp64 oracle, OpenMP over all host cores"},
+            "e2e": {"value": v, "unit": "images/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+
+
+def cpu_baseline_sample():
+    import synth
+    from oracle.net import run_net
+    x, layers = synth.resnet50(32)
+    xs = x[:1]
+    t0 = time.perf_counter()
+    n = 0
+    while True:
+        run_net(layers, xs, "bf16")
+        n += 1
+        if time.perf_counter() - t0 > 10.0 or n >= 3:
+            break
+    sec = (time.perf_counter() - t0) / n
+    return {"value": 1.0 / sec, "unit": "images/s", "cores": os.cpu_count(), "kind": "oracle",
+            "sample": f"{n} single-image passes of the 32-image batch, fp64 oracle, OpenMP over all host cores"}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--batch", type=int, default=32)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-b1", action="store_true")
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3)
+    ws, rank, local = dist_env()
+    if args.impl == "reference":
+        return run_reference(args, ws, rank)
+
+    import torch
+    import synth
+    import paper_2110_06037_gb300 as sn
+    from paper_2110_06037_gb300 import routine_name
+
+    torch.cuda.set_device(local)
+    dist = None
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    pk, pk_kind = peaks()
+
+    # ---------------- tune: profile + DPRS ----------------
+    x, layers = synth.resnet50(args.batch)
+    sch = [("bf16", "nchw"), ("bf16", "nhwc")]
+    stream = torch.cuda.Stream()
+    t_tune0 = time.perf_counter()
+    with torch.cuda.stream(stream):
+        g = sn.build_graph(layers, x.shape, ("bf16", "nchw"), ("bf16", "nchw"), sch)
+        g.profile(warmup=3, iters=10, topk=2, passes=3)
+        total, schemas, cands = g.select_path(sn.SN_SELECT_DPRS)
+    stream.synchronize()
+    tune_s = time.perf_counter() - t_tune0
+
+    xd = torch.from_numpy(x).to(torch.bfloat16).cuda()
+    out = g.new_output()
+    flush = torch.empty(256 * 1024 * 1024, dtype=torch.uint8, device="cuda")  # > L2 (129 MB)
+    g.set_option(sn.SN_OPT_CUDA_GRAPH, 1)
+    with torch.cuda.stream(stream):
+        for _ in range(args.warmup):
+            g.run(xd, out)
+    stream.synchronize()
+    n_ops, n_kern = g.plan_stats(stream)
+
+    # ---------------- timed region (device, per-step events, L2 flushed between steps) -------
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    clocks = ClockSampler(local)
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    torch.cuda.nvtx.range_push("sn_timed")
+    with torch.cuda.stream(stream):
+        for i in range(args.steps):
+            flush.zero_()
+            ev[i][0].record(stream)
+            g.run(xd, out)
+            ev[i][1].record(stream)
+    torch.cuda.synchronize()
+    torch.cuda.nvtx.range_pop()
+    if dist:
+        dist.barrier()
+    clk = clocks.stop()
+    step_ms = [a.elapsed_time(b) for a, b in ev]
+    ms = sum(step_ms) / len(step_ms)
+    if dist:
+        t = torch.tensor([ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    value = ws * args.batch / (ms / 1e3)
+
+    # ---------------- e2e through the public API with host buffers ----------------
+    xh = torch.from_numpy(x).to(torch.bfloat16).pin_memory()
+    oh = torch.empty(out.shape, dtype=out.dtype).pin_memory()
+    xin = torch.empty_like(xd)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        for _ in range(2):
+            xin.copy_(xh, non_blocking=True)
+            g.run(xin, out)
+            oh.copy_(out, non_blocking=True)
+        stream.synchronize()
+        e0.record(stream)
+        for _ in range(args.steps):
+            xin.copy_(xh, non_blocking=True)
+            g.run(xin, out)
+            oh.copy_(out, non_blocking=True)
+        e1.record(stream)
+    stream.synchronize()
+    e2e_ms = e0.elapsed_time(e1) / args.steps
+    e2e = {"value": args.batch / (e2e_ms / 1e3), "unit": "images/s",
+           "h2d_bytes_per_step": xh.numel() * xh.element_size(),
+           "d2h_bytes_per_step": oh.numel() * oh.element_size()}
+
+    # ---------------- per-routine device time (events around every launch) ----------------
+    g.set_option(sn.SN_OPT_CUDA_GRAPH, 0)
+    t = g.cost_table()
+    layer_ms = np.zeros(t["n_layers"])
+    edge_ms = np.zeros(len(t["edges"]))
+    reps = max(3, min(args.steps, 10))
+    with torch.cuda.stream(stream):
+        for _ in range(reps):
+            flush.zero_()
+            _, lm, em = g.run_timed(xd, out)
+            layer_ms += lm
+            edge_ms += em[: len(edge_ms)]
+    layer_ms /= reps
+    edge_ms /= reps
+    work, _ = conv_work(layers, x.shape)
+    per_routine = {}
+    for i in range(1, t["n_layers"] - 1):
+        c = int(cands[i])
+        r = routine_name(int(t["routine"][c]))
+        d = per_routine.setdefault(r, {"ms": 0.0, "flop": 0, "bytes": 0, "launches": 0})
+        d["ms"] += float(layer_ms[i])
+        d["flop"] += work[i - 1][0]
+        d["bytes"] += work[i - 1][1]
+        d["launches"] += 1
+    if edge_ms.sum() > 0:
+        per_routine["adapt/convert"] = {"ms": float(edge_ms.sum()), "flop": 0, "bytes": 0,
+                                        "launches": int((edge_ms > 0).sum())}
+    dom = max(per_routine, key=lambda r: per_routine[r]["ms"])
+    d = per_routine[dom]
+    sustained = pk.get("bf16_tflops_sustained", pk["bf16_tflops"])
+    if dom == "conv2/igemm_tc":
+        achieved = d["flop"] / (d["ms"] / 1e3) / 1e12
+        roof = {"bound": "tensor", "achieved": achieved, "peak": sustained, "unit": "TFLOP/s",
+                "frac": achieved / sustained, "traffic": None}
+    elif dom in ("conv2/igemm_simt", "conv2/direct", "conv2/wino_f2x2_3x3"):
+        ffma_peak = 2 * 128 * 152 * pk.get("sm_max_mhz", 2070.0) / 1e6  # TFLOP/s fp32 FFMA
+        achieved = d["flop"] / (d["ms"] / 1e3) / 1e12
+        roof = {"bound": "alu", "achieved": achieved, "peak": ffma_peak, "unit": "TFLOP/s",
+                "frac": achieved / ffma_peak, "traffic": None}
+    else:
+        achieved = d["bytes"] / (d["ms"] / 1e3) / 1e9
+        roof = {"bound": "hbm", "achieved": achieved, "peak": pk["hbm_gbs"], "unit": "GB/s",
+                "frac": achieved / pk["hbm_gbs"], "traffic": None}
+    roof["kernel"] = dom
+    roof["peak_source"] = f"{pk_kind} (MEASURED_PEAKS.json)" if pk_kind == "measured" else "fallback"
+
+    # ---------------- ResNet-50 b1 latency (fp16, CUDA graph) ----------------
+    b1 = None
+    if not args.no_b1:
+        x1, layers1 = synth.resnet50(1)
+        s16 = [("f16", "nchw"), ("f16", "nhwc")]
+        with torch.cuda.stream(stream):
+            g1 = sn.build_graph(layers1, x1.shape, ("f16", "nchw"), ("f16", "nchw"), s16)
+            g1.profile(warmup=3, iters=10, topk=2, passes=3)
+            g1.select_path(sn.SN_SELECT_DPRS)
+            g1.set_option(sn.SN_OPT_CUDA_GRAPH, 1)
+            x1d = torch.from_numpy(x1).to(torch.float16).cuda()
+            o1 = g1.new_output()
+            for _ in range(5):
+                g1.run(x1d, o1)
+        stream.synchronize()
+        lat = []
+        for _ in range(20):
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            with torch.cuda.stream(stream):
+                flush.zero_()
+                a.record(stream)
+                g1.run(x1d, o1)
+                b.record(stream)
+            stream.synchronize()
+            lat.append(a.elapsed_time(b))
+        b1 = {"mean_ms": statistics.mean(lat), "std_ms": statistics.pstdev(lat), "median_ms": statistics.median(lat)}
+
+    cpu = None
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline_sample()
+
+    if rank == 0:
+        line = {"metric": METRIC, "value": value, "unit": "images/s", "n_gpus": ws, "steps": args.steps,
+                "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+                "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+                "config": {"workload": WORKLOAD, "batch": args.batch, "parallelism": f"replicas x{ws}",
+                           "l2": "flushed between steps (256 MB write outside the step events)",
+                           "timing": "CUDA events around each step on the launching stream, CUDA-graph replay"},
+                "e2e": e2e, "gpu_launches": n_kern * args.steps, "roofline": roof, "cpu_baseline": cpu,
+                "clocks": clk, "tuning_s": tune_s, "path_cost_ns": total,
+                "r50_b1_fp16_latency": b1,
+                "per_routine_ms": {k: round(v["ms"], 4) for k, v in per_routine.items()}}
+        print(json.dumps(line))
+    if dist:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

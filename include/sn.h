@@ -214,6 +214,12 @@ SN_API sn_status sn_run(sn_graph *g, const void *in_dev, void *out_dev, void *st
 SN_API sn_status sn_run_timed(sn_graph *g, const void *in_dev, void *out_dev, void *stream,
                        float *layer_ms, float *edge_ms);
 
+/* Launch statistics of the current plan (built on `stream` if needed): the
+ * number of plan operations (layer routines + adapts) and of CUDA kernels
+ * that one sn_run launches.  Either output may be NULL.
+ * Errors: SN_ESTATE (no path), plus those of plan building. */
+SN_API sn_status sn_plan_stats(sn_graph *g, int32_t *n_ops, int32_t *n_kernels, void *stream);
+
 /* Logical output shape of internal layer `layer` (N, C, H, W). */
 SN_API sn_status sn_layer_shape(sn_graph *g, int32_t layer, int64_t out_nchw[4]);
 

@@ -90,6 +90,7 @@ SIGNATURES = {
     "sn_run_timed": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.POINTER(C.c_float),
                                C.POINTER(C.c_float)]),
     "sn_layer_shape": (C.c_int, [C.c_void_p, C.c_int32, C.POINTER(C.c_int64)]),
+    "sn_plan_stats": (C.c_int, [C.c_void_p, C.POINTER(C.c_int32), C.POINTER(C.c_int32), C.c_void_p]),
     "sn_save_plan": (C.c_int, [C.c_void_p, C.c_char_p]),
     "sn_load_plan": (C.c_int, [C.c_void_p, C.c_char_p]),
     "sn_graph_destroy": (None, [C.c_void_p]),

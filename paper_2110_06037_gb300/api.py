@@ -175,6 +175,12 @@ class Graph:
         check(lib().sn_layer_shape(self.h, i, s))
         return tuple(s)
 
+    def plan_stats(self, stream=None):
+        """(plan operations, CUDA kernels) that one run launches."""
+        ops, kern = C.c_int32(), C.c_int32()
+        check(lib().sn_plan_stats(self.h, C.byref(ops), C.byref(kern), _stream_ptr(stream)))
+        return ops.value, kern.value
+
     def save_plan(self, path):
         check(lib().sn_save_plan(self.h, str(path).encode()))
 

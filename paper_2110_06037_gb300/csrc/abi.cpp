@@ -375,6 +375,30 @@ sn_status sn_run_timed(sn_graph *gg, const void *in_dev, void *out_dev, void *st
     })
 }
 
+sn_status sn_plan_stats(sn_graph *gg, int32_t *n_ops, int32_t *n_kernels, void *stream) {
+    SN_GUARD({
+        if (!gg) return fail(SN_EINVAL, "sn_plan_stats: NULL graph");
+        Graph *g = G(gg);
+        if (!g->has_path) return fail(SN_ESTATE, "sn_plan_stats: select or set a routine path first");
+        if (!g->plan_valid) {
+            sn_status rc = build_plan(g, static_cast<cudaStream_t>(stream));
+            if (rc != SN_OK) return rc;
+        }
+        int32_t kern = 0;
+        for (const PlanOp &op : g->plan) {
+            if (op.kind == PlanOp::ADAPT) {
+                kern += 1;
+            } else {
+                const Candidate &c = g->cands[op.cand];
+                kern += kernels_per_launch(c.routine, c.variant);
+            }
+        }
+        if (n_ops) *n_ops = (int32_t)g->plan.size();
+        if (n_kernels) *n_kernels = kern;
+        return SN_OK;
+    })
+}
+
 sn_status sn_layer_shape(sn_graph *gg, int32_t layer, int64_t out_nchw[4]) {
     SN_GUARD({
         if (!gg || !out_nchw) return fail(SN_EINVAL, "sn_layer_shape: NULL argument");

@@ -144,6 +144,12 @@ sn_status prepare_weights(Graph *g, int32_t li, int32_t r, int32_t v, sn_schema 
     return SN_OK;
 }
 
+int32_t kernels_per_launch(int32_t r, int32_t v) {
+    (void)v;
+    if (r == R_CONV_WINO) return 3;  // wgenc, wgconv, wgdec
+    return 1;
+}
+
 sn_status launch_routine(const LaunchArgs &a) {
     cudaError_t e = cudaSuccess;
     switch (a.routine) {

@@ -184,6 +184,7 @@ size_t routine_workspace(int32_t routine, int32_t variant, const Layer &layer,
 sn_status prepare_weights(Graph *g, int32_t li, int32_t routine, int32_t variant, sn_schema s,
                           const void **wt, const float **bias, cudaStream_t st);
 sn_status launch_routine(const LaunchArgs &a);
+int32_t kernels_per_launch(int32_t routine, int32_t variant);
 
 // selection (section IV)
 sn_status select_dprs(const Graph &g, std::vector<int32_t> &schema_of, int64_t &total);
