@@ -111,3 +111,15 @@ def test_set_path_validation():
         g.set_path(np.zeros(t["n_layers"], np.int32))  # candidate 0 belongs to layer 0 only
     first = [int(np.flatnonzero(t["layer"] == i)[0]) for i in range(t["n_layers"])]
     g.set_path(first)
+
+
+def test_tc_not_offered_where_it_cannot_run():
+    for C, dt, lay, s, H in [(3, "f16", "nhwc", 1, 8), (64, "f32", "nhwc", 1, 8), (64, "f16", "nchw", 1, 8),
+                             (64, "bf16", "nhwc", 2, 7)]:
+        layer = synth.conv(C, 64, 3, s, 1)
+        layer["weight"] = np.zeros((64, C, 3, 3), np.float32)
+        layer["bias"] = np.zeros(64, np.float32)
+        g = build_graph([dict(layer, inputs=[-1])], (1, C, H, H), (dt, lay), (dt, lay), [(dt, lay)],
+                        torch_alloc=False)
+        t = g.cost_table()
+        assert not any(_sn.routine_name(int(r)) == "conv2/igemm_tc" for r in t["routine"])
