@@ -244,6 +244,43 @@ SN_API const char *sn_variant_name(int32_t routine, int32_t variant);
 SN_API sn_status sn_convert(const void *x_dev, sn_schema from, void *y_dev, sn_schema to,
                      const int64_t nchw[4], void *stream);
 
+/* ---------------- allocation-free Winograd convolution --------------------
+ * The paper has no counterpart to this call; it exists for callers that
+ * cannot allocate device memory at the point where they run a layer: plug-ins
+ * inside a host application that owns every device allocation, services
+ * whose memory budget is fixed at start-up, or latency-critical loops where a
+ * cudaMalloc (and its implicit synchronisation) is not acceptable.
+ *
+ * It computes the same conv2 as the graph's "conv2/wino_f2x2_3x3" routine
+ * (3x3 kernel, stride 1, dilation 1, groups 1, zero padding `pad` on both
+ * axes, bias + act), using the same kernels, but its scratch (the transformed
+ * filter U and the Winograd buffers V and M) lives in one fixed device array
+ * of SN_NOALLOC_SCRATCH_BYTES that is part of the library image: every GPU
+ * that loads the library holds that memory until the process exits.  The
+ * call itself never allocates: no cudaMalloc, no cudaFree, no allocator hook.
+ *
+ *   x_dev    input, logical N x C x H x W stored in `schema` (caller-owned)
+ *   w_dev    device fp32 weights [c_out][C][3][3] (caller-owned)
+ *   bias_dev device fp32 [c_out] (required)
+ *   y_dev    output, N x c_out x P x Q in `schema`, P = H + 2 pad - 2
+ *   act      sn_act
+ *   stream   cudaStream_t the kernels are launched on (asynchronous)
+ *
+ * The first call on a device resolves the array's device address (one
+ * cudaGetSymbolAddress with that device current); make that first call
+ * before any stream capture.  All calls share the one array and it keeps the
+ * previous call's contents; every element a call reads is first written by
+ * the same call, so nothing needs clearing.  Calls that can overlap on the
+ * GPU (different streams, or host threads without ordering) race on the
+ * array: serialise them.
+ * Errors: SN_EINVAL (NULL pointer, bad extent, schema, pad or act),
+ * SN_EUNSUPPORTED (the scratch need exceeds SN_NOALLOC_SCRATCH_BYTES; nothing
+ * is launched), SN_ECUDA. */
+#define SN_NOALLOC_SCRATCH_BYTES (32u * 1024u * 1024u)
+SN_API sn_status sn_conv2d_wino_noalloc(const void *x_dev, sn_schema schema, const int64_t in_nchw[4],
+                                        int32_t c_out, int32_t pad, int32_t act, const float *w_dev,
+                                        const float *bias_dev, void *y_dev, void *stream);
+
 SN_API const char *sn_last_error(void);
 
 #ifdef __cplusplus

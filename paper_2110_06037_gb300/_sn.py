@@ -97,8 +97,11 @@ SIGNATURES = {
     "sn_routine_name": (C.c_char_p, [C.c_int32]),
     "sn_variant_name": (C.c_char_p, [C.c_int32, C.c_int32]),
     "sn_convert": (C.c_int, [C.c_void_p, sn_schema, C.c_void_p, sn_schema, C.POINTER(C.c_int64), C.c_void_p]),
+    "sn_conv2d_wino_noalloc": (C.c_int, [C.c_void_p, sn_schema, C.POINTER(C.c_int64), C.c_int32, C.c_int32,
+                                         C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p]),
     "sn_last_error": (C.c_char_p, []),
 }
+NOALLOC_SCRATCH_BYTES = 32 * 1024 * 1024
 
 _lib = None
 

@@ -59,6 +59,9 @@ struct ConvDims {
     int32_t N, C, H, W, K, P, Q, R, S, sh, sw, ph, pw, dh, dw, groups, act;
 };
 
+cudaError_t conv_wino_buffers(const ConvDims &d, sn_schema s, const void *x, const void *u, const float *bias,
+                              void *y, float *V, float *Mx, cudaStream_t st);
+
 inline ConvDims conv_dims(const LaunchArgs &a) {
     const sn_conv_params &p = a.layer->conv;
     const Shape &i = a.in_shapes[0];

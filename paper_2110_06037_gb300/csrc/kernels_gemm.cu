@@ -357,5 +357,26 @@ cudaError_t conv_wino(const LaunchArgs &a) {
     return cudaGetLastError();
 }
 
+// The three Winograd stages on caller-provided buffers (used by the
+// allocation-free entry point): U [16][K][C] in the schema dtype, V and Mx fp32.
+cudaError_t conv_wino_buffers(const ConvDims &d, sn_schema s, const void *x, const void *u, const float *bias,
+                              void *y, float *V, float *Mx, cudaStream_t st) {
+    const WinoDims wd = wino_dims(d);
+    dim3 ggrid((unsigned)((wd.T + 63) / 64), (unsigned)((d.K + 63) / 64), 16);
+    if (ggrid.y > 65535) return cudaErrorInvalidValue;
+    SN_DT_SWITCH(s.dtype, T, {
+        if (s.layout == SN_NHWC)
+            wino_input_kernel<T, true><<<grid_for(wd.T * d.C, 256), 256, 0, st>>>((const T *)x, V, wd);
+        else
+            wino_input_kernel<T, false><<<grid_for(wd.T * d.C, 256), 256, 0, st>>>((const T *)x, V, wd);
+        gemm_nt_simt<T><<<ggrid, 256, 0, st>>>(V, (const T *)u, Mx, wd.T, d.K, d.C);
+        if (s.layout == SN_NHWC)
+            wino_output_kernel<T, true><<<grid_for(wd.T * d.K, 256), 256, 0, st>>>(Mx, bias, (T *)y, wd);
+        else
+            wino_output_kernel<T, false><<<grid_for(wd.T * d.K, 256), 256, 0, st>>>(Mx, bias, (T *)y, wd);
+    });
+    return cudaGetLastError();
+}
+
 }  // namespace k
 }  // namespace sn
