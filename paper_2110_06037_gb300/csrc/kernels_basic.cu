@@ -60,6 +60,22 @@ __global__ void __launch_bounds__(256) transpose_kernel(const Ti *__restrict__ x
     }
 }
 
+// few channels (C <= 16): one thread per pixel moves all of its channels;
+// the planar side is read/written coalesced across threads, the interleaved
+// side as C consecutive elements per thread (C * 32 contiguous per warp)
+template <typename Ti, typename To, bool TO_NHWC>
+__global__ void permute_small_c_kernel(const Ti *__restrict__ x, To *__restrict__ y, int64_t N, int C, int64_t HW) {
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < N * HW;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t n = i / HW, hw = i % HW;
+        for (int c = 0; c < C; ++c) {
+            const int64_t planar = (n * C + c) * HW + hw, inter = i * C + c;
+            if (TO_NHWC) stf<To>(y + inter, ldf<Ti>(x + planar));
+            else stf<To>(y + planar, ldf<Ti>(x + inter));
+        }
+    }
+}
+
 template <typename Ti, typename To>
 static cudaError_t convert_t(const void *x, int lay_in, void *y, int lay_out, Shape s,
                              cudaStream_t st) {
@@ -76,6 +92,16 @@ static cudaError_t convert_t(const void *x, int lay_in, void *y, int lay_out, Sh
             return cudaMemcpyAsync(y, x, bytes, cudaMemcpyDeviceToDevice, st);
         }
         cast_kernel<Ti, To><<<grid_for(n, 256), 256, 0, st>>>((const Ti *)x, (To *)y, n);
+        return cudaGetLastError();
+    }
+    if (s.c <= 16) {
+        const int64_t px = s.n * s.h * s.w;
+        if (lay_in == SN_NCHW)
+            permute_small_c_kernel<Ti, To, true><<<grid_for(px, 256), 256, 0, st>>>((const Ti *)x, (To *)y, s.n,
+                                                                                     (int)s.c, s.h * s.w);
+        else
+            permute_small_c_kernel<Ti, To, false><<<grid_for(px, 256), 256, 0, st>>>((const Ti *)x, (To *)y, s.n,
+                                                                                      (int)s.c, s.h * s.w);
         return cudaGetLastError();
     }
     // NCHW -> NHWC: per image [C][HW] -> [HW][C]; NHWC -> NCHW: [HW][C] -> [C][HW]
@@ -130,6 +156,7 @@ __global__ void weight_perm_kernel(const float *__restrict__ w, T *__restrict__ 
         int64_t o;
         if (fmt == W_KCRS) o = i;
         else if (fmt == W_RSCK) o = ((r * S + s) * Cg + c) * K + kk;
+        else if (fmt == W_KRSC_PAD64) o = kk * ((Cg * R * S + 63) / 64 * 64) + (r * S + s) * Cg + c;
         else o = ((kk * R + r) * S + s) * Cg + c;  // W_KRSC
         stf<T>(out + o, w[i]);
     }
@@ -165,6 +192,11 @@ cudaError_t weight_format(const float *w, void *out, int fmt, int dt, int64_t K,
         if (R != 3 || S != 3) return cudaErrorInvalidValue;
         SN_DT_SWITCH(dt, T, weight_wino_kernel<T><<<grid_for(K * Cg, 256), 256, 0, st>>>(w, (T *)out, K, Cg));
         return cudaGetLastError();
+    }
+    if (fmt == W_KRSC_PAD64) {  // rows padded with zeros to a multiple of 64 taps
+        const int64_t kpad = (Cg * R * S + 63) / 64 * 64;
+        cudaError_t e = cudaMemsetAsync(out, 0, (size_t)K * kpad * dtype_size(dt), st);
+        if (e != cudaSuccess) return e;
     }
     SN_DT_SWITCH(dt, T,
                  weight_perm_kernel<T><<<grid_for(K * Cg * R * S, 256), 256, 0, st>>>(w, (T *)out, fmt, K, Cg, R, S));
@@ -350,12 +382,54 @@ __global__ void maxpool_kernel(const T *__restrict__ x, T *__restrict__ y, int N
     }
 }
 
+// NHWC, 16 bytes of channels per thread (8 x 16-bit or 4 x fp32 lanes)
+template <typename T>
+__global__ void maxpool_nhwc_vec(const uint4 *__restrict__ x, uint4 *__restrict__ y, int N, int C16, int H, int W,
+                                 int P, int Q, int kh, int kw, int sh, int sw, int ph, int pw) {
+    constexpr int E = 16 / sizeof(T);
+    const int64_t total = (int64_t)N * P * Q * C16;
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const int cv = (int)(i % C16);
+        const int64_t pix = i / C16;
+        const int q = (int)(pix % Q), p = (int)((pix / Q) % P);
+        const int64_t n = pix / ((int64_t)Q * P);
+        float m[E];
+#pragma unroll
+        for (int e = 0; e < E; ++e) m[e] = -INFINITY;
+        for (int r = 0; r < kh; ++r) {
+            const int h = p * sh - ph + r;
+            if (h < 0 || h >= H) continue;
+            for (int s = 0; s < kw; ++s) {
+                const int ww = q * sw - pw + s;
+                if (ww < 0 || ww >= W) continue;
+                const uint4 v = x[((n * H + h) * W + ww) * C16 + cv];
+                const T *pv = reinterpret_cast<const T *>(&v);
+#pragma unroll
+                for (int e = 0; e < E; ++e) m[e] = fmaxf(m[e], ldf<T>(pv + e));
+            }
+        }
+        uint4 o;
+        T *po = reinterpret_cast<T *>(&o);
+#pragma unroll
+        for (int e = 0; e < E; ++e) po[e] = cvt<T>(m[e]);  // exact: m is one of the stored values
+        y[i] = o;
+    }
+}
+
 cudaError_t maxpool(const LaunchArgs &a) {
     const Shape &i = a.in_shapes[0], &o = a.layer->out;
     const sn_pool_params &p = a.layer->pool;
     const int64_t total = o.numel();
     SN_DT_SWITCH(a.schema.dtype, T, {
-        if (a.schema.layout == SN_NHWC)
+        const int64_t cb = i.c * (int64_t)sizeof(T);
+        if (a.schema.layout == SN_NHWC && cb % 16 == 0 && (uintptr_t)a.in[0] % 16 == 0 &&
+            (uintptr_t)a.out % 16 == 0) {
+            const int c16 = (int)(cb / 16);
+            maxpool_nhwc_vec<T><<<grid_for(o.n * o.h * o.w * c16, 256), 256, 0, a.stream>>>(
+                (const uint4 *)a.in[0], (uint4 *)a.out, (int)i.n, c16, (int)i.h, (int)i.w, (int)o.h, (int)o.w,
+                p.kh, p.kw, p.sh, p.sw, p.ph, p.pw);
+        } else if (a.schema.layout == SN_NHWC)
             maxpool_kernel<T, true><<<grid_for(total, 256), 256, 0, a.stream>>>(
                 (const T *)a.in[0], (T *)a.out, (int)i.n, (int)i.c, (int)i.h, (int)i.w, (int)o.h, (int)o.w,
                 p.kh, p.kw, p.sh, p.sw, p.ph, p.pw);

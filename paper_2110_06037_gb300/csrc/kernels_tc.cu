@@ -4,7 +4,7 @@
 // GEMM view (NHWC activations, KRSC weights, fp16/bf16 in, fp32 accumulate):
 //   D[m, k] = sum_{r, s, c} A[m, (r, s, c)] * B[k, (r, s, c)]
 //   m = output pixel (n, p, q), k = output channel.
-// One CTA computes a 128 x BN tile of D.  The K loop runs over filter taps
+// A tile of D is 128 pixels x BN channels.  The K loop runs over filter taps
 // (r, s) and 64-channel blocks; every step stages
 //   A: the 128 output pixels' input pixels for that tap, 64 channels
 //      (one TMA box of a 4-D [N, H, W, C] tensor map: the tile is a
@@ -16,11 +16,15 @@
 // Both land in shared memory in the 128-byte-swizzled K-major layout that
 // tcgen05.mma reads directly.
 //
-// Warp roles (192 threads): warp 0 = TMA producer (+ TMEM allocation),
-// warp 1 = MMA issuer (one thread), warps 2-5 = epilogue (TMEM -> registers
-// -> bias + activation -> fp16/bf16 -> global).  Every mbarrier wait is
-// bounded; on expiry the kernel records an error code in the library's error
-// word, waits (bounded) for its own copies and MMAs, frees TMEM and exits.
+// The kernel is persistent: one CTA per SM walks the tiles (A-sharing tiles
+// adjacent), with two TMEM accumulators so that the epilogue of one tile
+// overlaps the main loop of the next.  Warp roles (192 threads): warp 0 =
+// TMA producer (+ TMEM allocation), warp 1 = MMA issuer (one thread), warps
+// 2-5 = epilogue: TMEM -> registers -> bias + activation -> fp16/bf16 ->
+// 64-byte-swizzled staging in shared memory -> TMA tensor store (clipped at
+// the tensor edges).  Every mbarrier wait is bounded; on expiry the kernel
+// records an error code in the library's error word, waits (bounded) for its
+// own copies and MMAs, frees TMEM and exits.
 #include <cuda.h>
 
 #include <algorithm>
@@ -40,17 +44,19 @@ constexpr int BM = 128;
 constexpr int BK = 64;
 constexpr int THREADS = 192;
 constexpr long long WAIT_LIMIT = 4000000000LL;  // SM cycles (~2 s)
-enum : int { ERR_TMA_WAIT = 0x10, ERR_MMA_WAIT = 0x20, ERR_ACC_WAIT = 0x40 };
+constexpr uint32_t STG_BYTES = 32 * 32 * 2;    // one epilogue staging buffer: 32 rows x 32 channels
+enum : int { ERR_TMA_WAIT = 0x10, ERR_MMA_WAIT = 0x20, ERR_ACC_WAIT = 0x40, ERR_EPI_WAIT = 0x80 };
 
 struct Params {
     int32_t N, H, W, C, K, P, Q, R, S;
     int32_t stride, ph, pw, dh, dw;
     int32_t cblocks, kiters;
-    int32_t BW, BH, BNI, tq, tp;
+    int32_t BW, BH, BNI, tq, tp;   // pixel-tile geometry (implicit mode)
+    int32_t sbw, sbh, sbn;         // 32-row sub-box of a tile written by one epilogue warp
+    int32_t mtiles, ntiles;
     int64_t M;
     int32_t act;
     const float *bias;
-    void *y;
     int *err;  // the library's device error word
 };
 
@@ -181,56 +187,95 @@ __device__ __forceinline__ uint32_t pack2<__nv_bfloat16>(float a, float b) {
     return *reinterpret_cast<uint32_t *>(&h);
 }
 
+
+__device__ __forceinline__ void mbar_arrive(uint64_t *b) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(su32(b)) : "memory");
+}
+__device__ __forceinline__ void fence_proxy_async_smem() {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap *m, const void *src, int c0, int c1) {
+    asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.tile.bulk_group [%0, {%2, %3}], [%1];"
+                 ::"l"(reinterpret_cast<uint64_t>(m)), "r"(su32(src)), "r"(c0), "r"(c1)
+                 : "memory");
+}
+__device__ __forceinline__ void tma_store_4d(const CUtensorMap *m, const void *src, int c0, int c1, int c2, int c3) {
+    asm volatile("cp.async.bulk.tensor.4d.global.shared::cta.tile.bulk_group [%0, {%2, %3, %4, %5}], [%1];"
+                 ::"l"(reinterpret_cast<uint64_t>(m)), "r"(su32(src)), "r"(c0), "r"(c1), "r"(c2), "r"(c3)
+                 : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+// at most one store group may still be reading shared memory
+__device__ __forceinline__ void bulk_wait_read_1() { asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+
+struct TileCoord {
+    int n0;          // first output channel
+    int64_t m0;      // plain mode: first pixel row
+    int q0, p0, i0;  // implicit mode: box origin (q, p, image)
+};
+
+__device__ __forceinline__ TileCoord tile_coord(const Params &p, int t, int bn, bool implicit) {
+    TileCoord c;
+    const int mt = t / p.ntiles, nt = t - mt * p.ntiles;  // A-sharing tiles are adjacent
+    c.n0 = nt * bn;
+    c.m0 = 0;
+    c.q0 = c.p0 = c.i0 = 0;
+    if (implicit) {
+        int bx = mt;
+        const int bq = bx % p.tq;
+        bx /= p.tq;
+        const int bp = bx % p.tp;
+        bx /= p.tp;
+        c.q0 = bq * p.BW;
+        c.p0 = bp * p.BH;
+        c.i0 = bx * p.BNI;
+    } else {
+        c.m0 = (int64_t)mt * BM;
+    }
+    return c;
+}
+
 // --------------------------------------------------------------------- kernel
 template <typename T, int BN, int STAGES, bool IMPLICIT>
 __global__ void __launch_bounds__(THREADS, 1)
     conv_tc_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ CUtensorMap mA1,
                    const __grid_constant__ CUtensorMap mA2, const __grid_constant__ CUtensorMap mA3,
-                   const __grid_constant__ CUtensorMap mB, const Params p) {
+                   const __grid_constant__ CUtensorMap mB, const __grid_constant__ CUtensorMap mY,
+                   const Params p) {
     constexpr uint32_t A_BYTES = BM * BK * 2;
     constexpr uint32_t B_BYTES = BN * BK * 2;
     constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
-    constexpr uint32_t TMEM_COLS = BN;
+    constexpr uint32_t TMEM_COLS = 2 * BN;  // two accumulators
     extern __shared__ uint8_t smem_raw[];
     __shared__ __align__(8) uint64_t full_bar[STAGES];
     __shared__ __align__(8) uint64_t empty_bar[STAGES];
-    __shared__ __align__(8) uint64_t acc_bar;
+    __shared__ __align__(8) uint64_t accf_bar[2];  // MMA -> epilogue: accumulator ready
+    __shared__ __align__(8) uint64_t acce_bar[2];  // epilogue -> MMA: accumulator drained
     __shared__ uint32_t tmem_sh;
     __shared__ volatile int abort_sh;
     __shared__ int issued_sh, consumed_sh;
-    __shared__ float bias_sh[BN];
 
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint8_t *stg = smem + STAGES * STAGE_BYTES;  // 4 warps x 2 staging buffers, 1024-B aligned
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-    const int n0 = blockIdx.y * BN;
-    int64_t m0 = 0;
-    int q0 = 0, p0 = 0, i0 = 0;
-    if (IMPLICIT) {
-        int bx = blockIdx.x;
-        const int bq = bx % p.tq;
-        bx /= p.tq;
-        const int bp = bx % p.tp;
-        bx /= p.tp;
-        q0 = bq * p.BW;
-        p0 = bp * p.BH;
-        i0 = bx * p.BNI;
-    } else {
-        m0 = (int64_t)blockIdx.x * BM;
-    }
+    const int total = p.mtiles * p.ntiles;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
             mbar_init(&full_bar[s], 1);
             mbar_init(&empty_bar[s], 1);
         }
-        mbar_init(&acc_bar, 1);
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&accf_bar[b], 1);
+            mbar_init(&acce_bar[b], 4);  // one arrival per epilogue warp
+        }
         abort_sh = 0;
         issued_sh = 0;
         consumed_sh = 0;
         fence_mbar_init();
     }
     if (warp == 0) tmem_alloc(&tmem_sh, TMEM_COLS);
-    for (int j = threadIdx.x; j < BN; j += THREADS) bias_sh[j] = (n0 + j < p.K) ? p.bias[n0 + j] : 0.f;
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -238,109 +283,139 @@ __global__ void __launch_bounds__(THREADS, 1)
 
     if (warp == 0) {
         if (lane == 0) {  // ---------------- TMA producer
-            int it = 0;
-            for (; it < p.kiters; ++it) {
-                const int s = it % STAGES;
-                const uint32_t ph = (uint32_t)(it / STAGES) & 1u;
-                if (!mbar_wait(&empty_bar[s], ph ^ 1u)) {
-                    atomicOr(p.err, ERR_TMA_WAIT);
-                    abort_sh = 1;
-                    break;
-                }
-                if (abort_sh) break;
-                uint8_t *sa = smem + s * STAGE_BYTES;
-                uint8_t *sb = sa + A_BYTES;
-                const int tap = it / p.cblocks, cb = it - tap * p.cblocks;
-                const int r = tap / p.S, ss = tap - r * p.S;
-                const int c0 = cb * BK;
-                mbar_expect_tx(&full_bar[s], STAGE_BYTES);
-                if (IMPLICIT) {
-                    const int oh = r * p.dh - p.ph, ow = ss * p.dw - p.pw;
-                    if (p.stride == 1) {
-                        tma_4d(sa, &mA0, &full_bar[s], c0, q0 + ow, p0 + oh, i0);
-                    } else {  // stride 2: even/odd sub-lattice maps
-                        const int bh = oh & 1, bw = ow & 1;
-                        const int ah = (oh - bh) / 2, aw = (ow - bw) / 2;
-                        const CUtensorMap *m = bh ? (bw ? &mA3 : &mA2) : (bw ? &mA1 : &mA0);
-                        tma_4d(sa, m, &full_bar[s], c0, q0 + aw, p0 + ah, i0);
+            int g = 0;
+            bool stop = false;
+            for (int t = blockIdx.x; t < total && !stop; t += gridDim.x) {
+                const TileCoord tc = tile_coord(p, t, BN, IMPLICIT);
+                for (int it = 0; it < p.kiters; ++it, ++g) {
+                    const int s = g % STAGES;
+                    const uint32_t ph = (uint32_t)(g / STAGES) & 1u;
+                    if (!mbar_wait(&empty_bar[s], ph ^ 1u)) {
+                        atomicOr(p.err, ERR_TMA_WAIT);
+                        abort_sh = 1;
                     }
-                } else {
-                    tma_2d(sa, &mA0, &full_bar[s], c0, (int)m0);
+                    if (abort_sh) {
+                        stop = true;
+                        break;
+                    }
+                    uint8_t *sa = smem + s * STAGE_BYTES;
+                    uint8_t *sb = sa + A_BYTES;
+                    const int tap = it / p.cblocks, cb = it - tap * p.cblocks;
+                    const int r = tap / p.S, ss = tap - r * p.S;
+                    const int c0 = cb * BK;
+                    mbar_expect_tx(&full_bar[s], STAGE_BYTES);
+                    if (IMPLICIT) {
+                        const int oh = r * p.dh - p.ph, ow = ss * p.dw - p.pw;
+                        if (p.stride == 1) {
+                            tma_4d(sa, &mA0, &full_bar[s], c0, tc.q0 + ow, tc.p0 + oh, tc.i0);
+                        } else {  // stride 2: even/odd sub-lattice maps
+                            const int bh = oh & 1, bw = ow & 1;
+                            const int ah = (oh - bh) / 2, aw = (ow - bw) / 2;
+                            const CUtensorMap *m = bh ? (bw ? &mA3 : &mA2) : (bw ? &mA1 : &mA0);
+                            tma_4d(sa, m, &full_bar[s], c0, tc.q0 + aw, tc.p0 + ah, tc.i0);
+                        }
+                    } else {
+                        tma_2d(sa, &mA0, &full_bar[s], c0, (int)tc.m0);
+                    }
+                    tma_3d(sb, &mB, &full_bar[s], c0, tap, tc.n0);
                 }
-                tma_3d(sb, &mB, &full_bar[s], c0, tap, n0);
             }
-            issued_sh = it;
+            issued_sh = g;
         }
     } else if (warp == 1) {
         if (lane == 0) {  // ---------------- MMA issuer
             const uint32_t idesc = idesc_f16<T>(BM, BN);
-            int it = 0;
-            for (; it < p.kiters; ++it) {
-                const int s = it % STAGES;
-                const uint32_t ph = (uint32_t)(it / STAGES) & 1u;
-                if (!mbar_wait(&full_bar[s], ph)) {
-                    atomicOr(p.err, ERR_MMA_WAIT);
+            int g = 0, lt = 0;
+            bool stop = false;
+            for (int t = blockIdx.x; t < total && !stop; t += gridDim.x, ++lt) {
+                const int b = lt & 1;
+                const uint32_t aph = (uint32_t)(lt >> 1) & 1u;
+                if (!mbar_wait(&acce_bar[b], aph ^ 1u)) {
+                    atomicOr(p.err, ERR_EPI_WAIT);
                     abort_sh = 1;
                     break;
                 }
                 tc_fence_after();
-                const uint32_t sa = su32(smem + s * STAGE_BYTES), sb = sa + A_BYTES;
+                const uint32_t d = tmem + (uint32_t)(b * BN);
+                for (int it = 0; it < p.kiters; ++it, ++g) {
+                    const int s = g % STAGES;
+                    const uint32_t ph = (uint32_t)(g / STAGES) & 1u;
+                    if (!mbar_wait(&full_bar[s], ph)) {
+                        atomicOr(p.err, ERR_MMA_WAIT);
+                        abort_sh = 1;
+                        stop = true;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t sa = su32(smem + s * STAGE_BYTES), sb = sa + A_BYTES;
 #pragma unroll
-                for (int k = 0; k < BK / 16; ++k)
-                    umma(tmem, sdesc_sw128(sa + k * 32), sdesc_sw128(sb + k * 32), idesc, (it | k) ? 1u : 0u);
-                umma_commit(&empty_bar[s]);  // frees the stage once these MMAs have read it
+                    for (int k = 0; k < BK / 16; ++k)
+                        umma(d, sdesc_sw128(sa + k * 32), sdesc_sw128(sb + k * 32), idesc, (it | k) ? 1u : 0u);
+                    umma_commit(&empty_bar[s]);  // frees the stage once these MMAs have read it
+                }
+                if (!stop) umma_commit(&accf_bar[b]);
             }
-            consumed_sh = it;
-            if (it == p.kiters) umma_commit(&acc_bar);
+            consumed_sh = g;
         }
     } else {  // ---------------- epilogue: warps 2..5
-        const int g = warp & 3;  // TMEM lanes 32g..32g+31 belong to this warp
-        const int row = g * 32 + lane;
-        const bool ok = mbar_wait(&acc_bar, 0);
-        if (!ok) {
-            if (lane == 0) atomicOr(p.err, ERR_ACC_WAIT);
-            abort_sh = 1;
-        } else {
-            tc_fence_after();
-            bool valid;
-            int64_t off;
-            if (IMPLICIT) {
-                const int wq = row % p.BW, hp = (row / p.BW) % p.BH, ni = row / (p.BW * p.BH);
-                const int q = q0 + wq, pp = p0 + hp, n = i0 + ni;
-                valid = q < p.Q && pp < p.P && n < p.N;
-                off = (((int64_t)n * p.P + pp) * p.Q + q) * p.K;
-            } else {
-                const int64_t m = m0 + row;
-                valid = m < p.M;
-                off = m * p.K;
+        const int g4 = warp & 3;  // TMEM lanes 32*g4 .. +31 belong to this warp
+        uint8_t *my_stg = stg + (warp - 2) * 2 * STG_BYTES;
+        const int r0 = g4 * 32;  // first tile row of this warp
+        // origin of this warp's 32-row sub-box inside the tile (implicit mode)
+        const int wq0 = IMPLICIT ? r0 % p.BW : 0;
+        const int hp0 = IMPLICIT ? (r0 / p.BW) % p.BH : 0;
+        const int ni0 = IMPLICIT ? r0 / (p.BW * p.BH) : 0;
+        int lt = 0, chunk = 0;
+        for (int t = blockIdx.x; t < total; t += gridDim.x, ++lt) {
+            const int b = lt & 1;
+            const uint32_t aph = (uint32_t)(lt >> 1) & 1u;
+            if (!mbar_wait(&accf_bar[b], aph)) {
+                if (lane == 0) atomicOr(p.err, ERR_ACC_WAIT);
+                abort_sh = 1;
+                break;
             }
-            T *yrow = static_cast<T *>(p.y) + off + n0;
+            tc_fence_after();
+            const TileCoord tc = tile_coord(p, t, BN, IMPLICIT);
 #pragma unroll 1
-            for (int c = 0; c < BN; c += 32) {
+            for (int c = 0; c < BN && tc.n0 + c < p.K; c += 32, ++chunk) {
                 uint32_t v[32];
                 __syncwarp();
-                tmem_ld32(tmem + ((uint32_t)(g * 32) << 16) + (uint32_t)c, v);
-                if (valid && n0 + c < p.K) {
-                float f[32];
+                tmem_ld32(tmem + ((uint32_t)r0 << 16) + (uint32_t)(b * BN + c), v);
+                const float bl = (tc.n0 + c + lane < p.K) ? p.bias[tc.n0 + c + lane] : 0.f;
+                uint32_t w[16];
 #pragma unroll
-                for (int j = 0; j < 32; ++j) f[j] = act_apply(__uint_as_float(v[j]) + bias_sh[c + j], p.act);
-                if (n0 + c + 32 <= p.K) {
-                    uint4 *dst = reinterpret_cast<uint4 *>(yrow + c);
-#pragma unroll
-                    for (int q4 = 0; q4 < 4; ++q4) {
-                        uint4 w;
-                        w.x = pack2<T>(f[8 * q4 + 0], f[8 * q4 + 1]);
-                        w.y = pack2<T>(f[8 * q4 + 2], f[8 * q4 + 3]);
-                        w.z = pack2<T>(f[8 * q4 + 4], f[8 * q4 + 5]);
-                        w.w = pack2<T>(f[8 * q4 + 6], f[8 * q4 + 7]);
-                        dst[q4] = w;
-                    }
-                } else {
-                    for (int j = 0; j < 32 && n0 + c + j < p.K; ++j) stf<T>(yrow + c + j, f[j]);
+                for (int j = 0; j < 16; ++j) {
+                    const float f0 = act_apply(__uint_as_float(v[2 * j]) + __shfl_sync(0xffffffffu, bl, 2 * j), p.act);
+                    const float f1 =
+                        act_apply(__uint_as_float(v[2 * j + 1]) + __shfl_sync(0xffffffffu, bl, 2 * j + 1), p.act);
+                    w[j] = pack2<T>(f0, f1);
                 }
+                uint8_t *buf = my_stg + (chunk & 1) * STG_BYTES;
+                if (lane == 0) bulk_wait_read_1();  // the store that used this buffer has read it
+                __syncwarp();
+                // row `lane` (64 B = four 16-B chunks), 64-byte swizzle: chunk j -> j ^ ((row >> 1) & 3)
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    uint4 q4 = make_uint4(w[4 * j], w[4 * j + 1], w[4 * j + 2], w[4 * j + 3]);
+                    *reinterpret_cast<uint4 *>(buf + lane * 64 + ((j ^ ((lane >> 1) & 3)) << 4)) = q4;
+                }
+                fence_proxy_async_smem();
+                __syncwarp();
+                if (lane == 0) {
+                    if (IMPLICIT)
+                        tma_store_4d(&mY, buf, tc.n0 + c, tc.q0 + wq0, tc.p0 + hp0, tc.i0 + ni0);
+                    else
+                        tma_store_2d(&mY, buf, tc.n0 + c, (int)(tc.m0 + r0));
+                    bulk_commit();
                 }
             }
+            // every TMEM read of accumulator b is done: hand it back to the MMA warp
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&acce_bar[b]);
         }
+        if (lane == 0) bulk_wait_all();
+        __syncwarp();
     }
 
     tc_fence_before();
@@ -348,11 +423,11 @@ __global__ void __launch_bounds__(THREADS, 1)
     if (warp == 0) {
         if (abort_sh && lane == 0) {
             // let this CTA's own copies and MMAs land before its memory goes away
-            for (int it = consumed_sh; it < issued_sh; ++it)
-                mbar_wait(&full_bar[it % STAGES], (uint32_t)(it / STAGES) & 1u);
+            for (int g = consumed_sh; g < issued_sh; ++g)
+                mbar_wait(&full_bar[g % STAGES], (uint32_t)(g / STAGES) & 1u);
             if (consumed_sh > 0) {
-                const int it = consumed_sh - 1;
-                mbar_wait(&empty_bar[it % STAGES], (uint32_t)(it / STAGES) & 1u);
+                const int g = consumed_sh - 1;
+                mbar_wait(&empty_bar[g % STAGES], (uint32_t)(g / STAGES) & 1u);
             }
         }
         __syncwarp();
@@ -381,7 +456,8 @@ static EncodeTiled encoder() {
 }
 
 static bool encode(CUtensorMap *m, int dt, int rank, const void *base, const uint64_t *dims,
-                   const uint64_t *strides_bytes, const uint32_t *box) {
+                   const uint64_t *strides_bytes, const uint32_t *box,
+                   CUtensorMapSwizzle sw = CU_TENSOR_MAP_SWIZZLE_128B) {
     EncodeTiled fn = encoder();
     if (!fn) return false;
     cuuint64_t gd[5], gs[4];
@@ -393,9 +469,8 @@ static bool encode(CUtensorMap *m, int dt, int rank, const void *base, const uin
         if (i < rank - 1) gs[i] = strides_bytes[i];
     }
     const CUtensorMapDataType t = dt == SN_F16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
-    return fn(m, t, (cuuint32_t)rank, const_cast<void *>(base), gd, gs, bx, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
-              CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+    return fn(m, t, (cuuint32_t)rank, const_cast<void *>(base), gd, gs, bx, es, CU_TENSOR_MAP_INTERLEAVE_NONE, sw,
+              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 struct Config {
@@ -417,7 +492,7 @@ static std::vector<Config> configs(const Layer &l, const Shape &in, sn_schema s)
     std::vector<int> bns;
     if (K <= 64) bns = {64};
     else if (K <= 128) bns = {64, 128};
-    else bns = {128, 256};
+    else bns = {64, 128, 256};
     const bool plain = c.kh == 1 && c.kw == 1 && c.sh == 1 && c.ph == 0 && c.pw == 0;
     if (plain) {
         for (int bn : bns) out.push_back({false, bn, 0, 0, 0});
@@ -446,11 +521,21 @@ static std::vector<Config> configs(const Layer &l, const Shape &in, sn_schema s)
     return out;
 }
 
+static int num_sms() {
+    static int n = 0;
+    if (!n) {
+        int dev = 0;
+        cudaGetDevice(&dev);
+        if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 1;
+    }
+    return n;
+}
+
 template <typename T, int BN, bool IMPLICIT>
-static cudaError_t launch(const CUtensorMap *mA, const CUtensorMap &mB, const Params &p, dim3 grid,
+static cudaError_t launch(const CUtensorMap *mA, const CUtensorMap &mB, const CUtensorMap &mY, const Params &p,
                           cudaStream_t st) {
     constexpr int STAGES = BN == 256 ? 4 : (BN == 128 ? 6 : 8);
-    constexpr size_t smem = (size_t)STAGES * (BM * BK * 2 + BN * BK * 2) + 1024;
+    constexpr size_t smem = (size_t)STAGES * (BM * BK * 2 + BN * BK * 2) + 8 * STG_BYTES + 1024;
     auto kern = conv_tc_kernel<T, BN, STAGES, IMPLICIT>;
     static bool attr = false;
     if (!attr) {
@@ -458,7 +543,9 @@ static cudaError_t launch(const CUtensorMap *mA, const CUtensorMap &mB, const Pa
         if (e != cudaSuccess) return e;
         attr = true;
     }
-    kern<<<grid, THREADS, smem, st>>>(mA[0], mA[1], mA[2], mA[3], mB, p);
+    const int total = p.mtiles * p.ntiles;
+    const unsigned grid = (unsigned)std::min(total, num_sms());
+    kern<<<grid, THREADS, smem, st>>>(mA[0], mA[1], mA[2], mA[3], mB, mY, p);
     return cudaGetLastError();
 }
 
@@ -490,28 +577,30 @@ cudaError_t conv_tc(const LaunchArgs &a) {
     p.kiters = p.R * p.S * p.cblocks;
     p.act = c.act;
     p.bias = a.bias;
-    p.y = a.out;
     p.err = device_error_word();
     p.M = in.n * (int64_t)in.h * in.w;
+    p.ntiles = (p.K + cf.BN - 1) / cf.BN;
     const int dt = a.schema.dtype;
     const uint64_t es = 2;
-    CUtensorMap mA[4], mB;
-    // B: weights [K][R*S][C]
-    {
+    CUtensorMap mA[4], mB, mY;
+    {  // B: weights [K][R*S][C]
         const uint64_t dims[3] = {(uint64_t)p.C, (uint64_t)(p.R * p.S), (uint64_t)p.K};
         const uint64_t str[2] = {p.C * es, (uint64_t)p.R * p.S * p.C * es};
         const uint32_t box[3] = {BK, 1, (uint32_t)cf.BN};
         if (!encode(&mB, dt, 3, a.wt, dims, str, box)) return cudaErrorInvalidValue;
     }
-    dim3 grid;
-    grid.y = (unsigned)((p.K + cf.BN - 1) / cf.BN);
+    const int64_t Mout = (int64_t)p.N * p.P * p.Q;
     if (!cf.implicit) {
         const uint64_t dims[2] = {(uint64_t)p.C, (uint64_t)p.M};
         const uint64_t str[1] = {p.C * es};
         const uint32_t box[2] = {BK, BM};
         if (!encode(&mA[0], dt, 2, a.in[0], dims, str, box)) return cudaErrorInvalidValue;
         mA[1] = mA[2] = mA[3] = mA[0];
-        grid.x = (unsigned)((p.M + BM - 1) / BM);
+        const uint64_t ydims[2] = {(uint64_t)p.K, (uint64_t)Mout};
+        const uint64_t ystr[1] = {p.K * es};
+        const uint32_t ybox[2] = {32, 32};
+        if (!encode(&mY, dt, 2, a.out, ydims, ystr, ybox, CU_TENSOR_MAP_SWIZZLE_64B)) return cudaErrorInvalidValue;
+        p.mtiles = (int)((p.M + BM - 1) / BM);
     } else {
         p.BW = cf.BW, p.BH = cf.BH, p.BNI = cf.BNI;
         p.tq = (p.Q + cf.BW - 1) / cf.BW;
@@ -533,13 +622,21 @@ cudaError_t conv_tc(const LaunchArgs &a) {
                     if (!encode(&mA[bh * 2 + bw], dt, 4, base, dims, str, box)) return cudaErrorInvalidValue;
                 }
         }
-        grid.x = (unsigned)((int64_t)p.tq * p.tp * tn);
+        // the 32-row sub-box each epilogue warp stores
+        p.sbw = std::min(cf.BW, 32);
+        p.sbh = std::min(cf.BH, 32 / p.sbw);
+        p.sbn = 32 / (p.sbw * p.sbh);
+        const uint64_t ydims[4] = {(uint64_t)p.K, (uint64_t)p.Q, (uint64_t)p.P, (uint64_t)p.N};
+        const uint64_t ystr[3] = {p.K * es, (uint64_t)p.Q * p.K * es, (uint64_t)p.P * p.Q * p.K * es};
+        const uint32_t ybox[4] = {32, (uint32_t)p.sbw, (uint32_t)p.sbh, (uint32_t)p.sbn};
+        if (!encode(&mY, dt, 4, a.out, ydims, ystr, ybox, CU_TENSOR_MAP_SWIZZLE_64B)) return cudaErrorInvalidValue;
+        p.mtiles = p.tq * p.tp * tn;
     }
-    if (grid.y > 65535 || grid.x == 0) return cudaErrorInvalidValue;
+    if (p.mtiles <= 0 || (int64_t)p.mtiles * p.ntiles > INT32_MAX) return cudaErrorInvalidValue;
     const bool bf = dt == SN_BF16;
 #define SN_TC_LAUNCH(TT, BNV)                                                                     \
-    return cf.implicit ? launch<TT, BNV, true>(mA, mB, p, grid, a.stream)                          \
-                       : launch<TT, BNV, false>(mA, mB, p, grid, a.stream)
+    return cf.implicit ? launch<TT, BNV, true>(mA, mB, mY, p, a.stream)                            \
+                       : launch<TT, BNV, false>(mA, mB, mY, p, a.stream)
     if (bf) {
         if (cf.BN == 64) SN_TC_LAUNCH(__nv_bfloat16, 64);
         if (cf.BN == 128) SN_TC_LAUNCH(__nv_bfloat16, 128);
@@ -550,6 +647,112 @@ cudaError_t conv_tc(const LaunchArgs &a) {
         SN_TC_LAUNCH(__half, 256);
     }
 #undef SN_TC_LAUNCH
+}
+
+// ---------------------------------------------------------------------------
+// childnet routines built on the tensor-core GEMM (section III-D)
+// ---------------------------------------------------------------------------
+
+// 1x1 stride-1 conv2 of c_in -> c_out channels: the plain GEMM path of conv_tc
+static Layer gemm_layer(int c_in, int c_out, int act, Shape out) {
+    Layer g;
+    g.type = SN_L_CONV2;
+    g.conv = sn_conv_params{c_in, c_out, 1, 1, 1, 1, 0, 0, 1, 1, 1, act};
+    g.act = act;
+    g.out = out;
+    return g;
+}
+
+static int64_t im2col_kpad(const Layer &l) {
+    return ((int64_t)l.conv.c_in / l.conv.groups * l.conv.kh * l.conv.kw + 63) / 64 * 64;
+}
+
+// im2col -> GEMM: for layers the implicit routine cannot take (few input
+// channels such as an RGB stem, odd sizes with stride 2)
+int32_t conv_im2col_tc_variants(const Layer &l, const Shape &in, sn_schema s) {
+    const sn_conv_params &c = l.conv;
+    if (l.type != SN_L_CONV2 || c.groups != 1 || s.dtype == SN_F32 || s.layout != SN_NHWC) return 0;
+    if (c.c_out % 8) return 0;
+    if (!tc::configs(l, in, s).empty()) return 0;  // the implicit routine serves this layer
+    const Layer gl = gemm_layer((int)im2col_kpad(l), c.c_out, c.act, l.out);
+    const Shape gin{l.out.n, im2col_kpad(l), l.out.h, l.out.w};
+    return (int32_t)tc::configs(gl, gin, s).size();
+}
+
+size_t conv_im2col_tc_ws(const Layer &l, const Shape &in, sn_schema s) {
+    (void)in;
+    return (size_t)l.out.n * l.out.h * l.out.w * im2col_kpad(l) * dtype_size(s.dtype);
+}
+
+// A[m][kk] = x[n, p*sh - ph + r*dh, q*sw - pw + s*dw, c], kk = (r*S + s)*C + c,
+// zero outside the image and for kk >= C*R*S; 8 taps (16 bytes) per thread
+template <typename T>
+__global__ void im2col_nhwc_kernel(const T *__restrict__ x, T *__restrict__ A, ConvDims d, int kpad, int64_t M) {
+    const int g8 = kpad / 8;
+    const int crs = d.C * d.R * d.S;
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < M * g8;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t m = i / g8;
+        const int k0 = (int)(i % g8) * 8;
+        const int q = (int)(m % d.Q), p = (int)((m / d.Q) % d.P);
+        const int64_t n = m / ((int64_t)d.Q * d.P);
+        uint4 o;
+        T *po = reinterpret_cast<T *>(&o);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            const int kk = k0 + e;
+            float v = 0.f;
+            if (kk < crs) {
+                const int c = kk % d.C, rs = kk / d.C, r = rs / d.S, s = rs % d.S;
+                const int h = p * d.sh - d.ph + r * d.dh, w = q * d.sw - d.pw + s * d.dw;
+                if (h >= 0 && h < d.H && w >= 0 && w < d.W) v = ldf<T>(x + ((n * d.H + h) * d.W + w) * d.C + c);
+            }
+            po[e] = cvt<T>(v);  // exact: v is a stored value or zero
+        }
+        reinterpret_cast<uint4 *>(A)[i] = o;
+    }
+}
+
+cudaError_t conv_im2col_tc(const LaunchArgs &a) {
+    const Layer &l = *a.layer;
+    const ConvDims d = conv_dims(a);
+    const int64_t kpad = im2col_kpad(l);
+    const int64_t M = (int64_t)d.N * d.P * d.Q;
+    const size_t need = (size_t)M * kpad * dtype_size(a.schema.dtype);
+    if (!a.ws || a.ws_bytes < need || (uintptr_t)a.ws % 16) return cudaErrorInvalidValue;
+    SN_DT_SWITCH(a.schema.dtype, T,
+                 im2col_nhwc_kernel<T><<<grid_for(M * (kpad / 8), 256), 256, 0, a.stream>>>(
+                     (const T *)a.in[0], (T *)a.ws, d, (int)kpad, M));
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    const Layer gl = gemm_layer((int)kpad, d.K, d.act, l.out);
+    LaunchArgs g = a;
+    g.layer = &gl;
+    g.routine = R_CONV_TC;
+    g.in_shapes = {Shape{l.out.n, kpad, l.out.h, l.out.w}};
+    g.in[0] = a.ws;
+    g.ws = nullptr;
+    g.ws_bytes = 0;
+    return conv_tc(g);
+}
+
+// dense = reshape -> 1x1 conv2 -> reshape on an N x C x 1 x 1 blob (identical
+// bytes in NCHW and NHWC), run as the tensor-core GEMM
+int32_t dense_tc_variants(const Layer &l, const Shape &in, sn_schema s) {
+    if (l.type != SN_L_DENSE || s.dtype == SN_F32) return 0;
+    const sn_schema nhwc{s.dtype, SN_NHWC};
+    const Layer gl = gemm_layer(l.dense_in, l.dense_out, l.act, l.out);
+    return (int32_t)tc::configs(gl, in, nhwc).size();
+}
+
+cudaError_t dense_tc(const LaunchArgs &a) {
+    const Layer &l = *a.layer;
+    const Layer gl = gemm_layer(l.dense_in, l.dense_out, l.act, l.out);
+    LaunchArgs g = a;
+    g.layer = &gl;
+    g.routine = R_CONV_TC;
+    g.schema = sn_schema{a.schema.dtype, SN_NHWC};
+    return conv_tc(g);
 }
 
 }  // namespace k

@@ -23,6 +23,8 @@ const char *routine_name(int32_t r) {
     case R_ADD: return "add/eltwise";
     case R_DENSE: return "dense/simt";
     case R_ADAPT: return "adapt/convert";
+    case R_CONV_IM2COL_TC: return "conv2/im2col_tc";
+    case R_DENSE_TC: return "dense/gemm_tc";
     default: return nullptr;
     }
 }
@@ -31,7 +33,9 @@ const char *variant_name(int32_t r, int32_t v) {
     switch (r) {
     case R_CONV_IGEMM: return v == 0 ? "tile=64x64" : "tile=128x64";
     case R_CONV_WINO: return v == 0 ? "gemm=simt" : "gemm=tc";
-    case R_CONV_TC: return k::conv_tc_variant_name(v);
+    case R_CONV_TC:
+    case R_CONV_IM2COL_TC:
+    case R_DENSE_TC: return k::conv_tc_variant_name(v);
     default: return v == 0 ? "" : "?";
     }
 }
@@ -62,6 +66,10 @@ int32_t routine_variants(int32_t r, const Layer &l, const std::vector<Shape> &in
         return l.type == SN_L_ADD ? 1 : 0;
     case R_DENSE:
         return l.type == SN_L_DENSE ? 1 : 0;
+    case R_CONV_IM2COL_TC:
+        return is_conv(l) ? k::conv_im2col_tc_variants(l, in[0], s) : 0;
+    case R_DENSE_TC:
+        return l.type == SN_L_DENSE ? k::dense_tc_variants(l, in[0], s) : 0;
     default:
         return 0;
     }
@@ -71,6 +79,7 @@ size_t routine_workspace(int32_t r, int32_t v, const Layer &l, const std::vector
                          sn_schema s) {
     (void)v;
     if (r == R_CONV_WINO) return k::conv_wino_ws(l, in[0], s);
+    if (r == R_CONV_IM2COL_TC) return k::conv_im2col_tc_ws(l, in[0], s);
     return 0;
 }
 
@@ -83,6 +92,8 @@ static int weight_format_of(int32_t r, sn_schema s) {
     case R_CONV_TC: return k::W_KRSC;
     case R_DW_DIRECT: return s.layout == SN_NCHW ? k::W_KCRS : k::W_RSCK;
     case R_DENSE: return k::W_KCRS;
+    case R_CONV_IM2COL_TC: return k::W_KRSC_PAD64;
+    case R_DENSE_TC: return k::W_KRSC;
     default: return -1;
     }
 }
@@ -120,7 +131,9 @@ sn_status prepare_weights(Graph *g, int32_t li, int32_t r, int32_t v, sn_schema 
         *wt = it->second.ptr;
         return SN_OK;
     }
-    const int64_t elems = (fmt == k::W_WINO) ? 16 * K * Cg : K * Cg * R * S;
+    const int64_t elems = (fmt == k::W_WINO)         ? 16 * K * Cg
+                          : (fmt == k::W_KRSC_PAD64) ? K * ((Cg * R * S + 63) / 64 * 64)
+                                                     : K * Cg * R * S;
     Buffer src, dst;
     sn_status rc = dev_alloc(g, (size_t)K * Cg * R * S * sizeof(float), &src);
     if (rc != SN_OK) return rc;
@@ -146,7 +159,8 @@ sn_status prepare_weights(Graph *g, int32_t li, int32_t r, int32_t v, sn_schema 
 
 int32_t kernels_per_launch(int32_t r, int32_t v) {
     (void)v;
-    if (r == R_CONV_WINO) return 3;  // wgenc, wgconv, wgdec
+    if (r == R_CONV_WINO) return 3;       // wgenc, wgconv, wgdec
+    if (r == R_CONV_IM2COL_TC) return 2;  // im2col, GEMM
     return 1;
 }
 
@@ -162,6 +176,8 @@ sn_status launch_routine(const LaunchArgs &a) {
     case R_GAP: e = k::gap(a); break;
     case R_ADD: e = k::add(a); break;
     case R_DENSE: e = k::dense(a); break;
+    case R_CONV_IM2COL_TC: e = k::conv_im2col_tc(a); break;
+    case R_DENSE_TC: e = k::dense_tc(a); break;
     default: return fail(SN_EINVAL, "launch of a non-launchable routine");
     }
     if (e != cudaSuccess)

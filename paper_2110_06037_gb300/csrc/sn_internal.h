@@ -64,7 +64,9 @@ enum RoutineId : int32_t {
     R_ADD = 8,
     R_DENSE = 9,         // dense on CUDA cores
     R_ADAPT = 10,        // adapt layer (cast / layout change)
-    R_COUNT = 11
+    R_CONV_IM2COL_TC = 11,  // childnet: im2col -> tensor-core GEMM (any C, stride, dilation)
+    R_DENSE_TC = 12,     // childnet: reshape -> 1x1 conv2 on tensor cores -> reshape (section III-D)
+    R_COUNT = 13
 };
 
 // -------------------------------------------------------------------------
@@ -206,7 +208,7 @@ cudaError_t convert(const void *x, int dt_in, int lay_in, void *y, int dt_out, i
 cudaError_t fill_pattern(void *y, int dt, int64_t n, uint32_t seed, float scale,
                          cudaStream_t st);
 // weight re-layout / cast from fp32 KCRS (device) into a routine format
-enum WFormat { W_KCRS = 0, W_RSCK = 1, W_KRSC = 2, W_WINO = 3 };
+enum WFormat { W_KCRS = 0, W_RSCK = 1, W_KRSC = 2, W_WINO = 3, W_KRSC_PAD64 = 4 };
 cudaError_t weight_format(const float *w_kcrs, void *out, int fmt, int dt, int64_t K,
                           int64_t Cg, int64_t R, int64_t S, cudaStream_t st);
 
@@ -217,6 +219,12 @@ size_t conv_wino_ws(const Layer &l, const Shape &in, sn_schema s);
 cudaError_t conv_tc(const LaunchArgs &a);
 int32_t conv_tc_variants(const Layer &l, const Shape &in, sn_schema s);
 const char *conv_tc_variant_name(int32_t v);
+// im2col childnet and dense childnet on the tensor-core GEMM
+int32_t conv_im2col_tc_variants(const Layer &l, const Shape &in, sn_schema s);
+size_t conv_im2col_tc_ws(const Layer &l, const Shape &in, sn_schema s);
+cudaError_t conv_im2col_tc(const LaunchArgs &a);
+int32_t dense_tc_variants(const Layer &l, const Shape &in, sn_schema s);
+cudaError_t dense_tc(const LaunchArgs &a);
 cudaError_t dwconv(const LaunchArgs &a);
 cudaError_t maxpool(const LaunchArgs &a);
 cudaError_t gap(const LaunchArgs &a);

@@ -55,7 +55,8 @@ CONV_CASES = [
     (1, 130, 5, 5, 66, 3, 1, 1, 1, 1),     # channels past a tile edge
     (1, 16, 1, 1, 8, 3, 1, 1, 1, 1),       # 1x1 image, 3x3 kernel (padding only)
 ]
-ROUTINES = [("conv2/direct", 0), ("conv2/igemm_simt", 0), ("conv2/igemm_simt", 1), ("conv2/wino_f2x2_3x3", 0)]
+ROUTINES = ([("conv2/direct", 0), ("conv2/igemm_simt", 0), ("conv2/igemm_simt", 1), ("conv2/wino_f2x2_3x3", 0)]
+            + [("conv2/igemm_tc", v) for v in range(6)] + [("conv2/im2col_tc", v) for v in range(3)])
 
 
 @pytest.mark.parametrize("case", CONV_CASES)
@@ -112,6 +113,17 @@ def test_pool_gap_add_dense(schema):
     de["weight"] = (rng.standard_normal((33, 70)) * 0.2).astype(np.float32)
     de["bias"] = (rng.standard_normal(33) * 0.1).astype(np.float32)
     assert maxrel(run_one(de, xd, schema, "dense/simt", 0), ref_one(de, xd, schema[0])) <= TOL[schema[0]]
+    # dense childnet on the tensor-core GEMM (fp16/bf16 only)
+    xd = rng.standard_normal((5, 64, 1, 1)).astype(np.float32)
+    de = synth.dense(64, 40)
+    de["weight"] = (rng.standard_normal((40, 64)) * 0.2).astype(np.float32)
+    de["bias"] = (rng.standard_normal(40) * 0.1).astype(np.float32)
+    ref = ref_one(de, xd, schema[0])
+    for v in range(3):
+        got = run_one(de, xd, schema, "dense/gemm_tc", v)
+        if got is not None:
+            assert schema[0] != "f32"
+            assert maxrel(got, ref) <= TOL[schema[0]], v
 
 
 CONVERT_SHAPES = [(2, 5, 7, 9), (1, 64, 56, 56), (3, 130, 1, 1), (1, 3, 65, 67)]
