@@ -390,7 +390,10 @@ sn_status sn_plan_stats(sn_graph *gg, int32_t *n_ops, int32_t *n_kernels, void *
                 kern += 1;
             } else {
                 const Candidate &c = g->cands[op.cand];
-                kern += kernels_per_launch(c.routine, c.variant);
+                const Layer &L = g->layers[op.layer];
+                std::vector<Shape> in;
+                for (int32_t j : L.inputs) in.push_back(g->layers[j].out);
+                kern += kernels_per_launch(c.routine, c.variant, L, in, g->schemas[c.schema]);
             }
         }
         if (n_ops) *n_ops = (int32_t)g->plan.size();

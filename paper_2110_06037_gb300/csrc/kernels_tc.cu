@@ -16,15 +16,17 @@
 // Both land in shared memory in the 128-byte-swizzled K-major layout that
 // tcgen05.mma reads directly.
 //
-// The kernel is persistent: one CTA per SM walks the tiles (A-sharing tiles
-// adjacent), with two TMEM accumulators so that the epilogue of one tile
-// overlaps the main loop of the next.  Warp roles (192 threads): warp 0 =
-// TMA producer (+ TMEM allocation), warp 1 = MMA issuer (one thread), warps
-// 2-5 = epilogue: TMEM -> registers -> bias + activation -> fp16/bf16 ->
-// 64-byte-swizzled staging in shared memory -> TMA tensor store (clipped at
-// the tensor edges).  Every mbarrier wait is bounded; on expiry the kernel
-// records an error code in the library's error word, waits (bounded) for its
-// own copies and MMAs, frees TMEM and exits.
+// The kernel is persistent: one CTA per SM walks the work units (a tile, or
+// one K-range of a tile when the layer is split along K because it has too
+// few tiles to fill the GPU), A-sharing tiles adjacent, with two TMEM
+// accumulators so that draining one overlaps the main loop of the next.
+// Warp roles (320 threads): warp 0 = TMA producer (+ TMEM allocation),
+// warp 1 = MMA issuer (one thread), warps 2-9 = epilogue, two warps per TMEM
+// lane group taking alternate 32-channel chunks: TMEM -> registers -> bias +
+// activation -> fp16/bf16 -> 16-byte stores (or fp32 partial sums for a
+// K split, summed by splitk_reduce_kernel).  Every mbarrier wait is bounded;
+// on expiry the kernel records an error code in the library's error word,
+// waits (bounded) for its own copies and MMAs, frees TMEM and exits.
 #include <cuda.h>
 
 #include <algorithm>
@@ -42,22 +44,26 @@ namespace tc {
 
 constexpr int BM = 128;
 constexpr int BK = 64;
-constexpr int THREADS = 192;
+constexpr int THREADS = 320;
+constexpr int EPI_WARPS = 8;
+constexpr int MAX_K = 65536;
+constexpr uint32_t STG_BYTES = 32 * 32 * 2;      // one epilogue staging buffer: 32 rows x 32 channels
 constexpr long long WAIT_LIMIT = 4000000000LL;  // SM cycles (~2 s)
-constexpr uint32_t STG_BYTES = 32 * 32 * 2;    // one epilogue staging buffer: 32 rows x 32 channels
 enum : int { ERR_TMA_WAIT = 0x10, ERR_MMA_WAIT = 0x20, ERR_ACC_WAIT = 0x40, ERR_EPI_WAIT = 0x80 };
 
 struct Params {
     int32_t N, H, W, C, K, P, Q, R, S;
     int32_t stride, ph, pw, dh, dw;
-    int32_t cblocks, kiters;
+    int32_t cblocks, kiters, ksplit;
     int32_t BW, BH, BNI, tq, tp;   // pixel-tile geometry (implicit mode)
-    int32_t sbw, sbh, sbn;         // 32-row sub-box of a tile written by one epilogue warp
     int32_t mtiles, ntiles;
-    int64_t M;
+    int64_t M;                     // plain mode: input rows (= output pixels)
+    int64_t Mout;                  // output pixels N * P * Q
     int32_t act;
     const float *bias;
-    int *err;  // the library's device error word
+    void *y;                       // output, NHWC, fp16/bf16
+    float *part;                   // K split: fp32 partial sums [ksplit][Mout][K]
+    int *err;                      // the library's device error word
 };
 
 // ---------------------------------------------------------------- PTX helpers
@@ -188,6 +194,7 @@ __device__ __forceinline__ uint32_t pack2<__nv_bfloat16>(float a, float b) {
 }
 
 
+
 __device__ __forceinline__ void mbar_arrive(uint64_t *b) {
     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(su32(b)) : "memory");
 }
@@ -209,31 +216,37 @@ __device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.comm
 __device__ __forceinline__ void bulk_wait_read_1() { asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory"); }
 __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 
-struct TileCoord {
+// one unit of work: a 128 x BN tile and the K-range [it0, it1) it accumulates
+struct Work {
     int n0;          // first output channel
     int64_t m0;      // plain mode: first pixel row
     int q0, p0, i0;  // implicit mode: box origin (q, p, image)
+    int sp, it0, it1;
 };
 
-__device__ __forceinline__ TileCoord tile_coord(const Params &p, int t, int bn, bool implicit) {
-    TileCoord c;
+__device__ __forceinline__ Work work_of(const Params &p, int u, int bn, bool implicit) {
+    Work w;
+    w.sp = u % p.ksplit;
+    const int t = u / p.ksplit;
     const int mt = t / p.ntiles, nt = t - mt * p.ntiles;  // A-sharing tiles are adjacent
-    c.n0 = nt * bn;
-    c.m0 = 0;
-    c.q0 = c.p0 = c.i0 = 0;
+    w.n0 = nt * bn;
+    w.m0 = 0;
+    w.q0 = w.p0 = w.i0 = 0;
     if (implicit) {
         int bx = mt;
         const int bq = bx % p.tq;
         bx /= p.tq;
         const int bp = bx % p.tp;
         bx /= p.tp;
-        c.q0 = bq * p.BW;
-        c.p0 = bp * p.BH;
-        c.i0 = bx * p.BNI;
+        w.q0 = bq * p.BW;
+        w.p0 = bp * p.BH;
+        w.i0 = bx * p.BNI;
     } else {
-        c.m0 = (int64_t)mt * BM;
+        w.m0 = (int64_t)mt * BM;
     }
-    return c;
+    w.it0 = (int)((int64_t)w.sp * p.kiters / p.ksplit);
+    w.it1 = (int)((int64_t)(w.sp + 1) * p.kiters / p.ksplit);
+    return w;
 }
 
 // --------------------------------------------------------------------- kernel
@@ -257,9 +270,9 @@ __global__ void __launch_bounds__(THREADS, 1)
     __shared__ int issued_sh, consumed_sh;
 
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    uint8_t *stg = smem + STAGES * STAGE_BYTES;  // 4 warps x 2 staging buffers, 1024-B aligned
+    uint8_t *stg = smem + STAGES * STAGE_BYTES;  // epilogue staging: 8 warps x 2 buffers, 1024-B aligned
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-    const int total = p.mtiles * p.ntiles;
+    const int total = p.mtiles * p.ntiles * p.ksplit;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
@@ -268,7 +281,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(&accf_bar[b], 1);
-            mbar_init(&acce_bar[b], 4);  // one arrival per epilogue warp
+            mbar_init(&acce_bar[b], EPI_WARPS);  // one arrival per epilogue warp
         }
         abort_sh = 0;
         issued_sh = 0;
@@ -285,9 +298,9 @@ __global__ void __launch_bounds__(THREADS, 1)
         if (lane == 0) {  // ---------------- TMA producer
             int g = 0;
             bool stop = false;
-            for (int t = blockIdx.x; t < total && !stop; t += gridDim.x) {
-                const TileCoord tc = tile_coord(p, t, BN, IMPLICIT);
-                for (int it = 0; it < p.kiters; ++it, ++g) {
+            for (int u = blockIdx.x; u < total && !stop; u += gridDim.x) {
+                const Work w = work_of(p, u, BN, IMPLICIT);
+                for (int it = w.it0; it < w.it1; ++it, ++g) {
                     const int s = g % STAGES;
                     const uint32_t ph = (uint32_t)(g / STAGES) & 1u;
                     if (!mbar_wait(&empty_bar[s], ph ^ 1u)) {
@@ -307,17 +320,17 @@ __global__ void __launch_bounds__(THREADS, 1)
                     if (IMPLICIT) {
                         const int oh = r * p.dh - p.ph, ow = ss * p.dw - p.pw;
                         if (p.stride == 1) {
-                            tma_4d(sa, &mA0, &full_bar[s], c0, tc.q0 + ow, tc.p0 + oh, tc.i0);
+                            tma_4d(sa, &mA0, &full_bar[s], c0, w.q0 + ow, w.p0 + oh, w.i0);
                         } else {  // stride 2: even/odd sub-lattice maps
                             const int bh = oh & 1, bw = ow & 1;
                             const int ah = (oh - bh) / 2, aw = (ow - bw) / 2;
                             const CUtensorMap *m = bh ? (bw ? &mA3 : &mA2) : (bw ? &mA1 : &mA0);
-                            tma_4d(sa, m, &full_bar[s], c0, tc.q0 + aw, tc.p0 + ah, tc.i0);
+                            tma_4d(sa, m, &full_bar[s], c0, w.q0 + aw, w.p0 + ah, w.i0);
                         }
                     } else {
-                        tma_2d(sa, &mA0, &full_bar[s], c0, (int)tc.m0);
+                        tma_2d(sa, &mA0, &full_bar[s], c0, (int)w.m0);
                     }
-                    tma_3d(sb, &mB, &full_bar[s], c0, tap, tc.n0);
+                    tma_3d(sb, &mB, &full_bar[s], c0, tap, w.n0);
                 }
             }
             issued_sh = g;
@@ -327,7 +340,8 @@ __global__ void __launch_bounds__(THREADS, 1)
             const uint32_t idesc = idesc_f16<T>(BM, BN);
             int g = 0, lt = 0;
             bool stop = false;
-            for (int t = blockIdx.x; t < total && !stop; t += gridDim.x, ++lt) {
+            for (int u = blockIdx.x; u < total && !stop; u += gridDim.x, ++lt) {
+                const Work w = work_of(p, u, BN, IMPLICIT);
                 const int b = lt & 1;
                 const uint32_t aph = (uint32_t)(lt >> 1) & 1u;
                 if (!mbar_wait(&acce_bar[b], aph ^ 1u)) {
@@ -337,7 +351,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                 }
                 tc_fence_after();
                 const uint32_t d = tmem + (uint32_t)(b * BN);
-                for (int it = 0; it < p.kiters; ++it, ++g) {
+                for (int it = w.it0; it < w.it1; ++it, ++g) {
                     const int s = g % STAGES;
                     const uint32_t ph = (uint32_t)(g / STAGES) & 1u;
                     if (!mbar_wait(&full_bar[s], ph)) {
@@ -350,23 +364,27 @@ __global__ void __launch_bounds__(THREADS, 1)
                     const uint32_t sa = su32(smem + s * STAGE_BYTES), sb = sa + A_BYTES;
 #pragma unroll
                     for (int k = 0; k < BK / 16; ++k)
-                        umma(d, sdesc_sw128(sa + k * 32), sdesc_sw128(sb + k * 32), idesc, (it | k) ? 1u : 0u);
+                        umma(d, sdesc_sw128(sa + k * 32), sdesc_sw128(sb + k * 32), idesc,
+                             (it > w.it0 || k > 0) ? 1u : 0u);
                     umma_commit(&empty_bar[s]);  // frees the stage once these MMAs have read it
                 }
                 if (!stop) umma_commit(&accf_bar[b]);
             }
             consumed_sh = g;
         }
-    } else {  // ---------------- epilogue: warps 2..5
-        const int g4 = warp & 3;  // TMEM lanes 32*g4 .. +31 belong to this warp
+    } else {  // ---------------- epilogue: warps 2..9, two per TMEM lane group
+        const int g4 = warp & 3;          // TMEM lanes 32*g4 .. +31 belong to this warp
+        const int half = (warp - 2) >> 2;  // this warp drains chunks half, half + 2, ...
+        const int row = g4 * 32 + lane;
         uint8_t *my_stg = stg + (warp - 2) * 2 * STG_BYTES;
-        const int r0 = g4 * 32;  // first tile row of this warp
-        // origin of this warp's 32-row sub-box inside the tile (implicit mode)
+        // origin of this warp's 32-row sub-box inside a tile (implicit mode)
+        const int r0 = g4 * 32;
         const int wq0 = IMPLICIT ? r0 % p.BW : 0;
         const int hp0 = IMPLICIT ? (r0 / p.BW) % p.BH : 0;
         const int ni0 = IMPLICIT ? r0 / (p.BW * p.BH) : 0;
-        int lt = 0, chunk = 0;
-        for (int t = blockIdx.x; t < total; t += gridDim.x, ++lt) {
+        int chunk = 0;
+        int lt = 0;
+        for (int u = blockIdx.x; u < total; u += gridDim.x, ++lt) {
             const int b = lt & 1;
             const uint32_t aph = (uint32_t)(lt >> 1) & 1u;
             if (!mbar_wait(&accf_bar[b], aph)) {
@@ -375,46 +393,77 @@ __global__ void __launch_bounds__(THREADS, 1)
                 break;
             }
             tc_fence_after();
-            const TileCoord tc = tile_coord(p, t, BN, IMPLICIT);
+            const Work w = work_of(p, u, BN, IMPLICIT);
+            bool valid;
+            int64_t pix;
+            if (IMPLICIT) {
+                const int wq = row % p.BW, hp = (row / p.BW) % p.BH, ni = row / (p.BW * p.BH);
+                const int q = w.q0 + wq, pp = w.p0 + hp, n = w.i0 + ni;
+                valid = q < p.Q && pp < p.P && n < p.N;
+                pix = ((int64_t)n * p.P + pp) * p.Q + q;
+            } else {
+                pix = w.m0 + row;
+                valid = pix < p.Mout;
+            }
 #pragma unroll 1
-            for (int c = 0; c < BN && tc.n0 + c < p.K; c += 32, ++chunk) {
+            for (int c = half * 32; c < BN && w.n0 + c < p.K; c += 64) {
+                const int k0 = w.n0 + c;
+                // bias of channel k0 + lane, fetched before the TMEM load so its latency overlaps
+                const float bl = (p.ksplit == 1 && k0 + lane < p.K) ? __ldg(p.bias + k0 + lane) : 0.f;
                 uint32_t v[32];
                 __syncwarp();
-                tmem_ld32(tmem + ((uint32_t)r0 << 16) + (uint32_t)(b * BN + c), v);
-                const float bl = (tc.n0 + c + lane < p.K) ? p.bias[tc.n0 + c + lane] : 0.f;
-                uint32_t w[16];
+                tmem_ld32(tmem + ((uint32_t)(g4 * 32) << 16) + (uint32_t)(b * BN + c), v);
+                if (p.ksplit == 1) {
+                    // bias + activation -> 16-bit, staged in 64-byte-swizzled shared
+                    // memory (row = lane, 16-byte chunk j at j ^ ((row >> 1) & 3)),
+                    // then one TMA tensor store of the warp's 32 x 32 block; the
+                    // store clips rows and channels outside the output tensor
+                    uint32_t wv[16];
 #pragma unroll
-                for (int j = 0; j < 16; ++j) {
-                    const float f0 = act_apply(__uint_as_float(v[2 * j]) + __shfl_sync(0xffffffffu, bl, 2 * j), p.act);
-                    const float f1 =
-                        act_apply(__uint_as_float(v[2 * j + 1]) + __shfl_sync(0xffffffffu, bl, 2 * j + 1), p.act);
-                    w[j] = pack2<T>(f0, f1);
-                }
-                uint8_t *buf = my_stg + (chunk & 1) * STG_BYTES;
-                if (lane == 0) bulk_wait_read_1();  // the store that used this buffer has read it
-                __syncwarp();
-                // row `lane` (64 B = four 16-B chunks), 64-byte swizzle: chunk j -> j ^ ((row >> 1) & 3)
+                    for (int j = 0; j < 16; ++j) {
+                        const float f0 =
+                            act_apply(__uint_as_float(v[2 * j]) + __shfl_sync(0xffffffffu, bl, 2 * j), p.act);
+                        const float f1 =
+                            act_apply(__uint_as_float(v[2 * j + 1]) + __shfl_sync(0xffffffffu, bl, 2 * j + 1), p.act);
+                        wv[j] = pack2<T>(f0, f1);
+                    }
+                    uint8_t *buf = my_stg + (chunk & 1) * STG_BYTES;
+                    if (lane == 0) bulk_wait_read_1();  // the store that last used this buffer has read it
+                    __syncwarp();
 #pragma unroll
-                for (int j = 0; j < 4; ++j) {
-                    uint4 q4 = make_uint4(w[4 * j], w[4 * j + 1], w[4 * j + 2], w[4 * j + 3]);
-                    *reinterpret_cast<uint4 *>(buf + lane * 64 + ((j ^ ((lane >> 1) & 3)) << 4)) = q4;
-                }
-                fence_proxy_async_smem();
-                __syncwarp();
-                if (lane == 0) {
-                    if (IMPLICIT)
-                        tma_store_4d(&mY, buf, tc.n0 + c, tc.q0 + wq0, tc.p0 + hp0, tc.i0 + ni0);
-                    else
-                        tma_store_2d(&mY, buf, tc.n0 + c, (int)(tc.m0 + r0));
-                    bulk_commit();
+                    for (int j = 0; j < 4; ++j)
+                        *reinterpret_cast<uint4 *>(buf + lane * 64 + ((j ^ ((lane >> 1) & 3)) << 4)) =
+                            make_uint4(wv[4 * j], wv[4 * j + 1], wv[4 * j + 2], wv[4 * j + 3]);
+                    fence_proxy_async_smem();
+                    __syncwarp();
+                    if (lane == 0) {
+                        if (IMPLICIT)
+                            tma_store_4d(&mY, buf, k0, w.q0 + wq0, w.p0 + hp0, w.i0 + ni0);
+                        else
+                            tma_store_2d(&mY, buf, k0, (int)(w.m0 + r0));
+                        bulk_commit();
+                    }
+                    ++chunk;
+                } else if (valid) {
+                    float *dst = p.part + ((int64_t)w.sp * p.Mout + pix) * p.K + k0;
+                    if (k0 + 32 <= p.K) {
+#pragma unroll
+                        for (int q4 = 0; q4 < 8; ++q4)
+                            reinterpret_cast<uint4 *>(dst)[q4] =
+                                make_uint4(v[4 * q4], v[4 * q4 + 1], v[4 * q4 + 2], v[4 * q4 + 3]);
+                    } else {
+#pragma unroll
+                        for (int j = 0; j < 32; ++j)
+                            if (k0 + j < p.K) dst[j] = __uint_as_float(v[j]);
+                    }
                 }
             }
-            // every TMEM read of accumulator b is done: hand it back to the MMA warp
+            // every TMEM read of accumulator b by this warp is done: hand it back
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(&acce_bar[b]);
         }
-        if (lane == 0) bulk_wait_all();
+        if (lane == 0) bulk_wait_all();  // stores done before the CTA's shared memory is released
         __syncwarp();
     }
 
@@ -433,6 +482,30 @@ __global__ void __launch_bounds__(THREADS, 1)
         __syncwarp();
         tc_fence_after();
         tmem_dealloc(tmem, TMEM_COLS);
+    }
+}
+
+// y[m][k] = act(bias[k] + sum_s part[s][m][k]), four channels per thread
+template <typename T>
+__global__ void splitk_reduce_kernel(const float *__restrict__ part, const float *__restrict__ bias,
+                                     T *__restrict__ y, int64_t M, int K, int ks, int act) {
+    const int K4 = K / 4;
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < M * K4;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t m = i / K4;
+        const int k = (int)(i - m * K4) * 4;
+        float4 acc = make_float4(bias[k], bias[k + 1], bias[k + 2], bias[k + 3]);
+        for (int s = 0; s < ks; ++s) {
+            const float4 v = *reinterpret_cast<const float4 *>(part + ((int64_t)s * M + m) * K + k);
+            acc.x += v.x;
+            acc.y += v.y;
+            acc.z += v.z;
+            acc.w += v.w;
+        }
+        uint2 o;
+        o.x = pack2<T>(act_apply(acc.x, act), act_apply(acc.y, act));
+        o.y = pack2<T>(act_apply(acc.z, act), act_apply(acc.w, act));
+        *reinterpret_cast<uint2 *>(y + m * K + k) = o;
     }
 }
 
@@ -473,11 +546,15 @@ static bool encode(CUtensorMap *m, int dt, int rank, const void *base, const uin
               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+
 struct Config {
     bool implicit;
     int BN;
     int BW, BH, BNI;
+    int ksplit;
 };
+
+constexpr int kSmCount = 152;  // GB300; only used to decide which K splits to offer
 
 // deterministic list of routine-parameter combinations for a layer
 static std::vector<Config> configs(const Layer &l, const Shape &in, sn_schema s) {
@@ -485,17 +562,29 @@ static std::vector<Config> configs(const Layer &l, const Shape &in, sn_schema s)
     const sn_conv_params &c = l.conv;
     if (l.type != SN_L_CONV2 || c.groups != 1) return out;
     if (s.dtype == SN_F32 || s.layout != SN_NHWC) return out;
-    if (c.c_in % 8 || c.c_out % 8) return out;
+    if (c.c_in % 8 || c.c_out % 8 || c.c_out > MAX_K) return out;
     if (c.sh != c.sw || (c.sh != 1 && c.sh != 2)) return out;
     if (c.sh == 2 && (in.h % 2 || in.w % 2 || in.h < 2 || in.w < 2)) return out;
     const int K = c.c_out;
+    const int kiters = c.kh * c.kw * ((c.c_in + BK - 1) / BK);
     std::vector<int> bns;
     if (K <= 64) bns = {64};
     else if (K <= 128) bns = {64, 128};
     else bns = {64, 128, 256};
     const bool plain = c.kh == 1 && c.kw == 1 && c.sh == 1 && c.ph == 0 && c.pw == 0;
+    const int64_t N = l.out.n, P = l.out.h, Q = l.out.w;
+    auto push_splits = [&](Config cf, int64_t mtiles) {
+        cf.ksplit = 1;
+        out.push_back(cf);
+        const int64_t tiles = mtiles * ((K + cf.BN - 1) / cf.BN);
+        for (int ks : {2, 4})
+            if (tiles * ks <= 2 * kSmCount && kiters >= 4 * ks) {
+                cf.ksplit = ks;
+                out.push_back(cf);
+            }
+    };
     if (plain) {
-        for (int bn : bns) out.push_back({false, bn, 0, 0, 0});
+        for (int bn : bns) push_splits({false, bn, 0, 0, 0, 1}, (N * P * Q + BM - 1) / BM);
         return out;
     }
     struct G {
@@ -503,7 +592,6 @@ static std::vector<Config> configs(const Layer &l, const Shape &in, sn_schema s)
         int bw, bh, bni;
     };
     std::vector<G> gs;
-    const int64_t N = l.out.n, P = l.out.h, Q = l.out.w;
     for (int bw = 1; bw <= 128; bw *= 2)
         for (int bh = 1; bw * bh <= 128; bh *= 2) {
             const int bni = 128 / (bw * bh);
@@ -516,8 +604,11 @@ static std::vector<Config> configs(const Layer &l, const Shape &in, sn_schema s)
         return a.bh > b.bh;
     });
     const int keep = std::min<int>(2, (int)gs.size());
-    for (int gi = 0; gi < keep; ++gi)
-        for (int bn : bns) out.push_back({true, bn, gs[gi].bw, gs[gi].bh, gs[gi].bni});
+    for (int gi = 0; gi < keep; ++gi) {
+        const G &gg = gs[gi];
+        const int64_t mtiles = ((Q + gg.bw - 1) / gg.bw) * ((P + gg.bh - 1) / gg.bh) * ((N + gg.bni - 1) / gg.bni);
+        for (int bn : bns) push_splits({true, bn, gg.bw, gg.bh, gg.bni, 1}, mtiles);
+    }
     return out;
 }
 
@@ -535,7 +626,7 @@ template <typename T, int BN, bool IMPLICIT>
 static cudaError_t launch(const CUtensorMap *mA, const CUtensorMap &mB, const CUtensorMap &mY, const Params &p,
                           cudaStream_t st) {
     constexpr int STAGES = BN == 256 ? 4 : (BN == 128 ? 6 : 8);
-    constexpr size_t smem = (size_t)STAGES * (BM * BK * 2 + BN * BK * 2) + 8 * STG_BYTES + 1024;
+    constexpr size_t smem = (size_t)STAGES * (BM * BK * 2 + BN * BK * 2) + EPI_WARPS * 2 * STG_BYTES + 1024;
     auto kern = conv_tc_kernel<T, BN, STAGES, IMPLICIT>;
     static bool attr = false;
     if (!attr) {
@@ -543,9 +634,14 @@ static cudaError_t launch(const CUtensorMap *mA, const CUtensorMap &mB, const CU
         if (e != cudaSuccess) return e;
         attr = true;
     }
-    const int total = p.mtiles * p.ntiles;
+    const int total = p.mtiles * p.ntiles * p.ksplit;
     const unsigned grid = (unsigned)std::min(total, num_sms());
     kern<<<grid, THREADS, smem, st>>>(mA[0], mA[1], mA[2], mA[3], mB, mY, p);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess || p.ksplit == 1) return e;
+    const int64_t n4 = p.Mout * (p.K / 4);
+    splitk_reduce_kernel<T><<<grid_for(n4, 256), 256, 0, st>>>(p.part, p.bias, static_cast<T *>(p.y), p.Mout, p.K,
+                                                               p.ksplit, p.act);
     return cudaGetLastError();
 }
 
@@ -553,6 +649,12 @@ static cudaError_t launch(const CUtensorMap *mA, const CUtensorMap &mB, const CU
 
 int32_t conv_tc_variants(const Layer &l, const Shape &in, sn_schema s) {
     return (int32_t)tc::configs(l, in, s).size();
+}
+
+size_t conv_tc_ws(const Layer &l, const Shape &in, sn_schema s, int32_t v) {
+    const std::vector<tc::Config> cfgs = tc::configs(l, in, s);
+    if (v < 0 || v >= (int)cfgs.size() || cfgs[v].ksplit == 1) return 0;
+    return (size_t)cfgs[v].ksplit * l.out.n * l.out.h * l.out.w * l.conv.c_out * sizeof(float);
 }
 
 const char *conv_tc_variant_name(int32_t v) {
@@ -575,11 +677,19 @@ cudaError_t conv_tc(const LaunchArgs &a) {
     p.stride = c.sh, p.ph = c.ph, p.pw = c.pw, p.dh = c.dh, p.dw = c.dw;
     p.cblocks = (p.C + BK - 1) / BK;
     p.kiters = p.R * p.S * p.cblocks;
+    p.ksplit = cf.ksplit;
     p.act = c.act;
     p.bias = a.bias;
+    p.y = a.out;
     p.err = device_error_word();
     p.M = in.n * (int64_t)in.h * in.w;
+    p.Mout = (int64_t)p.N * p.P * p.Q;
     p.ntiles = (p.K + cf.BN - 1) / cf.BN;
+    if (cf.ksplit > 1) {
+        const size_t need = (size_t)cf.ksplit * p.Mout * p.K * sizeof(float);
+        if (!a.ws || a.ws_bytes < need || (uintptr_t)a.ws % 16) return cudaErrorInvalidValue;
+        p.part = static_cast<float *>(a.ws);
+    }
     const int dt = a.schema.dtype;
     const uint64_t es = 2;
     CUtensorMap mA[4], mB, mY;
@@ -589,18 +699,18 @@ cudaError_t conv_tc(const LaunchArgs &a) {
         const uint32_t box[3] = {BK, 1, (uint32_t)cf.BN};
         if (!encode(&mB, dt, 3, a.wt, dims, str, box)) return cudaErrorInvalidValue;
     }
-    const int64_t Mout = (int64_t)p.N * p.P * p.Q;
     if (!cf.implicit) {
         const uint64_t dims[2] = {(uint64_t)p.C, (uint64_t)p.M};
         const uint64_t str[1] = {p.C * es};
         const uint32_t box[2] = {BK, BM};
         if (!encode(&mA[0], dt, 2, a.in[0], dims, str, box)) return cudaErrorInvalidValue;
         mA[1] = mA[2] = mA[3] = mA[0];
-        const uint64_t ydims[2] = {(uint64_t)p.K, (uint64_t)Mout};
+        p.mtiles = (int)((p.M + BM - 1) / BM);
+        // output [Mout][K], one 32-row x 32-channel box per epilogue-warp chunk
+        const uint64_t ydims[2] = {(uint64_t)p.K, (uint64_t)p.Mout};
         const uint64_t ystr[1] = {p.K * es};
         const uint32_t ybox[2] = {32, 32};
         if (!encode(&mY, dt, 2, a.out, ydims, ystr, ybox, CU_TENSOR_MAP_SWIZZLE_64B)) return cudaErrorInvalidValue;
-        p.mtiles = (int)((p.M + BM - 1) / BM);
     } else {
         p.BW = cf.BW, p.BH = cf.BH, p.BNI = cf.BNI;
         p.tq = (p.Q + cf.BW - 1) / cf.BW;
@@ -622,17 +732,18 @@ cudaError_t conv_tc(const LaunchArgs &a) {
                     if (!encode(&mA[bh * 2 + bw], dt, 4, base, dims, str, box)) return cudaErrorInvalidValue;
                 }
         }
-        // the 32-row sub-box each epilogue warp stores
-        p.sbw = std::min(cf.BW, 32);
-        p.sbh = std::min(cf.BH, 32 / p.sbw);
-        p.sbn = 32 / (p.sbw * p.sbh);
+        p.mtiles = p.tq * p.tp * tn;
+        // output [N][P][Q][K]; an epilogue warp's 32 tile rows form a sub-box
+        // of sbw x sbh x sbn pixels (all dimensions powers of two)
+        const uint32_t sbw = (uint32_t)std::min(cf.BW, 32);
+        const uint32_t sbh = (uint32_t)std::min<int>(cf.BH, 32 / sbw);
+        const uint32_t sbn = 32 / (sbw * sbh);
         const uint64_t ydims[4] = {(uint64_t)p.K, (uint64_t)p.Q, (uint64_t)p.P, (uint64_t)p.N};
         const uint64_t ystr[3] = {p.K * es, (uint64_t)p.Q * p.K * es, (uint64_t)p.P * p.Q * p.K * es};
-        const uint32_t ybox[4] = {32, (uint32_t)p.sbw, (uint32_t)p.sbh, (uint32_t)p.sbn};
+        const uint32_t ybox[4] = {32, sbw, sbh, sbn};
         if (!encode(&mY, dt, 4, a.out, ydims, ystr, ybox, CU_TENSOR_MAP_SWIZZLE_64B)) return cudaErrorInvalidValue;
-        p.mtiles = p.tq * p.tp * tn;
     }
-    if (p.mtiles <= 0 || (int64_t)p.mtiles * p.ntiles > INT32_MAX) return cudaErrorInvalidValue;
+    if (p.mtiles <= 0 || (int64_t)p.mtiles * p.ntiles * p.ksplit > INT32_MAX) return cudaErrorInvalidValue;
     const bool bf = dt == SN_BF16;
 #define SN_TC_LAUNCH(TT, BNV)                                                                     \
     return cf.implicit ? launch<TT, BNV, true>(mA, mB, mY, p, a.stream)                            \
@@ -679,9 +790,15 @@ int32_t conv_im2col_tc_variants(const Layer &l, const Shape &in, sn_schema s) {
     return (int32_t)tc::configs(gl, gin, s).size();
 }
 
-size_t conv_im2col_tc_ws(const Layer &l, const Shape &in, sn_schema s) {
+static size_t im2col_bytes(const Layer &l, sn_schema s) {
+    return ((size_t)l.out.n * l.out.h * l.out.w * im2col_kpad(l) * dtype_size(s.dtype) + 255) & ~size_t(255);
+}
+
+size_t conv_im2col_tc_ws(const Layer &l, const Shape &in, sn_schema s, int32_t v) {
     (void)in;
-    return (size_t)l.out.n * l.out.h * l.out.w * im2col_kpad(l) * dtype_size(s.dtype);
+    const Layer gl = gemm_layer((int)im2col_kpad(l), l.conv.c_out, l.conv.act, l.out);
+    const Shape gin{l.out.n, im2col_kpad(l), l.out.h, l.out.w};
+    return im2col_bytes(l, s) + conv_tc_ws(gl, gin, s, v);
 }
 
 // A[m][kk] = x[n, p*sh - ph + r*dh, q*sw - pw + s*dw, c], kk = (r*S + s)*C + c,
@@ -713,16 +830,70 @@ __global__ void im2col_nhwc_kernel(const T *__restrict__ x, T *__restrict__ A, C
     }
 }
 
+// One block per output row (n, p): the R input rows it reads (W x C each,
+// zeros outside the image) are staged in shared memory with coalesced loads,
+// then the block writes its Q rows of A as 16-byte stores.
+template <typename T>
+__global__ void __launch_bounds__(256) im2col_rows_kernel(const T *__restrict__ x, T *__restrict__ A, ConvDims d,
+                                                          int kpad) {
+    extern __shared__ uint8_t im2col_smem[];
+    // per tap kk: (offset of (r, w = -pw + s*dw, c) in the staged rows, w) --
+    // the divisions by C and S happen once per block, not per element
+    int2 *tab = reinterpret_cast<int2 *>(im2col_smem);
+    T *rows = reinterpret_cast<T *>(im2col_smem + (size_t)kpad * sizeof(int2));
+    const int p = blockIdx.x;
+    const int64_t n = blockIdx.y;
+    const int WC = d.W * d.C;
+    const int crs = d.C * d.R * d.S;
+    for (int kk = threadIdx.x; kk < kpad; kk += blockDim.x) {
+        if (kk < crs) {
+            const int c = kk % d.C, rs = kk / d.C, r = rs / d.S, s = rs - r * d.S;
+            const int w = s * d.dw - d.pw;
+            tab[kk] = make_int2(r * WC + w * d.C + c, w);
+        } else {
+            tab[kk] = make_int2(0, -(1 << 29));  // padding tap: always zero
+        }
+    }
+    for (int i = threadIdx.x; i < d.R * WC; i += blockDim.x) {
+        const int r = i / WC, rem = i - r * WC;
+        const int h = p * d.sh - d.ph + r * d.dh;
+        rows[i] = (h >= 0 && h < d.H) ? x[((n * d.H + h) * d.W) * d.C + rem] : cvt<T>(0.f);
+    }
+    __syncthreads();
+    const int g8 = kpad / 8;
+    uint4 *out = reinterpret_cast<uint4 *>(A + ((n * d.P + p) * (int64_t)d.Q) * kpad);
+    for (int i = threadIdx.x; i < d.Q * g8; i += blockDim.x) {
+        const int q = i / g8, k0 = (i - q * g8) * 8;
+        const int qs = q * d.sw;
+        uint4 o;
+        T *po = reinterpret_cast<T *>(&o);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            const int2 t = tab[k0 + e];
+            const int w = t.y + qs;
+            po[e] = (w >= 0 && w < d.W) ? rows[t.x + qs * d.C] : cvt<T>(0.f);
+        }
+        out[i] = o;
+    }
+}
+
 cudaError_t conv_im2col_tc(const LaunchArgs &a) {
     const Layer &l = *a.layer;
     const ConvDims d = conv_dims(a);
     const int64_t kpad = im2col_kpad(l);
     const int64_t M = (int64_t)d.N * d.P * d.Q;
-    const size_t need = (size_t)M * kpad * dtype_size(a.schema.dtype);
+    const size_t need = im2col_bytes(l, a.schema);
     if (!a.ws || a.ws_bytes < need || (uintptr_t)a.ws % 16) return cudaErrorInvalidValue;
-    SN_DT_SWITCH(a.schema.dtype, T,
-                 im2col_nhwc_kernel<T><<<grid_for(M * (kpad / 8), 256), 256, 0, a.stream>>>(
-                     (const T *)a.in[0], (T *)a.ws, d, (int)kpad, M));
+    const size_t rows_bytes = (size_t)kpad * sizeof(int2) + (size_t)d.R * d.W * d.C * dtype_size(a.schema.dtype);
+    if (rows_bytes <= 48 * 1024 && d.N <= 65535) {
+        SN_DT_SWITCH(a.schema.dtype, T,
+                     im2col_rows_kernel<T><<<dim3((unsigned)d.P, (unsigned)d.N), 256, rows_bytes, a.stream>>>(
+                         (const T *)a.in[0], (T *)a.ws, d, (int)kpad));
+    } else {
+        SN_DT_SWITCH(a.schema.dtype, T,
+                     im2col_nhwc_kernel<T><<<grid_for(M * (kpad / 8), 256), 256, 0, a.stream>>>(
+                         (const T *)a.in[0], (T *)a.ws, d, (int)kpad, M));
+    }
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     const Layer gl = gemm_layer((int)kpad, d.K, d.act, l.out);
@@ -731,8 +902,8 @@ cudaError_t conv_im2col_tc(const LaunchArgs &a) {
     g.routine = R_CONV_TC;
     g.in_shapes = {Shape{l.out.n, kpad, l.out.h, l.out.w}};
     g.in[0] = a.ws;
-    g.ws = nullptr;
-    g.ws_bytes = 0;
+    g.ws = static_cast<uint8_t *>(a.ws) + im2col_bytes(l, a.schema);
+    g.ws_bytes = a.ws_bytes - im2col_bytes(l, a.schema);
     return conv_tc(g);
 }
 
@@ -743,6 +914,11 @@ int32_t dense_tc_variants(const Layer &l, const Shape &in, sn_schema s) {
     const sn_schema nhwc{s.dtype, SN_NHWC};
     const Layer gl = gemm_layer(l.dense_in, l.dense_out, l.act, l.out);
     return (int32_t)tc::configs(gl, in, nhwc).size();
+}
+
+size_t dense_tc_ws(const Layer &l, const Shape &in, sn_schema s, int32_t v) {
+    const Layer gl = gemm_layer(l.dense_in, l.dense_out, l.act, l.out);
+    return conv_tc_ws(gl, in, sn_schema{s.dtype, SN_NHWC}, v);
 }
 
 cudaError_t dense_tc(const LaunchArgs &a) {

@@ -77,9 +77,10 @@ int32_t routine_variants(int32_t r, const Layer &l, const std::vector<Shape> &in
 
 size_t routine_workspace(int32_t r, int32_t v, const Layer &l, const std::vector<Shape> &in,
                          sn_schema s) {
-    (void)v;
     if (r == R_CONV_WINO) return k::conv_wino_ws(l, in[0], s);
-    if (r == R_CONV_IM2COL_TC) return k::conv_im2col_tc_ws(l, in[0], s);
+    if (r == R_CONV_TC) return k::conv_tc_ws(l, in[0], s, v);
+    if (r == R_CONV_IM2COL_TC) return k::conv_im2col_tc_ws(l, in[0], s, v);
+    if (r == R_DENSE_TC) return k::dense_tc_ws(l, in[0], s, v);
     return 0;
 }
 
@@ -157,11 +158,14 @@ sn_status prepare_weights(Graph *g, int32_t li, int32_t r, int32_t v, sn_schema 
     return SN_OK;
 }
 
-int32_t kernels_per_launch(int32_t r, int32_t v) {
-    (void)v;
-    if (r == R_CONV_WINO) return 3;       // wgenc, wgconv, wgdec
-    if (r == R_CONV_IM2COL_TC) return 2;  // im2col, GEMM
-    return 1;
+int32_t kernels_per_launch(int32_t r, int32_t v, const Layer &l, const std::vector<Shape> &in, sn_schema s) {
+    // a K-split tensor-core GEMM adds its reduction kernel (it is the only
+    // variant with a workspace)
+    const int split = (r == R_CONV_TC || r == R_CONV_IM2COL_TC || r == R_DENSE_TC) &&
+                      routine_workspace(r, v, l, in, s) > (r == R_CONV_IM2COL_TC ? k::conv_im2col_tc_ws(l, in[0], s, -1) : 0);
+    if (r == R_CONV_WINO) return 3;             // wgenc, wgconv, wgdec
+    if (r == R_CONV_IM2COL_TC) return 2 + split;  // im2col, GEMM (+ reduction)
+    return 1 + split;
 }
 
 sn_status launch_routine(const LaunchArgs &a) {

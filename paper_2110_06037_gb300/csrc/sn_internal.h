@@ -186,7 +186,8 @@ size_t routine_workspace(int32_t routine, int32_t variant, const Layer &layer,
 sn_status prepare_weights(Graph *g, int32_t li, int32_t routine, int32_t variant, sn_schema s,
                           const void **wt, const float **bias, cudaStream_t st);
 sn_status launch_routine(const LaunchArgs &a);
-int32_t kernels_per_launch(int32_t routine, int32_t variant);
+int32_t kernels_per_launch(int32_t routine, int32_t variant, const Layer &layer, const std::vector<Shape> &in,
+                           sn_schema s);
 
 // selection (section IV)
 sn_status select_dprs(const Graph &g, std::vector<int32_t> &schema_of, int64_t &total);
@@ -218,10 +219,12 @@ cudaError_t conv_wino(const LaunchArgs &a);
 size_t conv_wino_ws(const Layer &l, const Shape &in, sn_schema s);
 cudaError_t conv_tc(const LaunchArgs &a);
 int32_t conv_tc_variants(const Layer &l, const Shape &in, sn_schema s);
+size_t conv_tc_ws(const Layer &l, const Shape &in, sn_schema s, int32_t v);  // K-split partial sums
+size_t dense_tc_ws(const Layer &l, const Shape &in, sn_schema s, int32_t v);
 const char *conv_tc_variant_name(int32_t v);
 // im2col childnet and dense childnet on the tensor-core GEMM
 int32_t conv_im2col_tc_variants(const Layer &l, const Shape &in, sn_schema s);
-size_t conv_im2col_tc_ws(const Layer &l, const Shape &in, sn_schema s);
+size_t conv_im2col_tc_ws(const Layer &l, const Shape &in, sn_schema s, int32_t v);
 cudaError_t conv_im2col_tc(const LaunchArgs &a);
 int32_t dense_tc_variants(const Layer &l, const Shape &in, sn_schema s);
 cudaError_t dense_tc(const LaunchArgs &a);

@@ -27,6 +27,8 @@ CASES = [
     (1, 24, 10, 10, 40, 3, 1, 1),     # C and K not multiples of 64 / 32
     (1, 16, 6, 6, 8, 1, 1, 0),        # tiny
     (1, 96, 12, 12, 72, 5, 1, 2),     # 5x5
+    (2, 256, 7, 7, 256, 3, 1, 1),     # few tiles: K-split variants (2, 4) offered
+    (4, 512, 7, 7, 136, 1, 1, 0),     # plain GEMM K split, K not a multiple of 32
 ]
 
 
