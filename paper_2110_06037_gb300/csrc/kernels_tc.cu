@@ -21,10 +21,12 @@
 // few tiles to fill the GPU), A-sharing tiles adjacent, with two TMEM
 // accumulators so that draining one overlaps the main loop of the next.
 // Warp roles (320 threads): warp 0 = TMA producer (+ TMEM allocation),
-// warp 1 = MMA issuer (one thread), warps 2-9 = epilogue, two warps per TMEM
-// lane group taking alternate 32-channel chunks: TMEM -> registers -> bias +
-// activation -> fp16/bf16 -> 16-byte stores (or fp32 partial sums for a
-// K split, summed by splitk_reduce_kernel).  Every mbarrier wait is bounded;
+// warp 1 = MMA issuer (one thread), warps 2-9 = epilogue in two groups of
+// four, group g draining accumulator g (alternate work units): TMEM ->
+// registers -> bias + activation -> fp16/bf16 -> 128-byte-swizzled staging
+// in shared memory -> one TMA tensor store per 32 rows x 64 channels
+// (clipped at the tensor edges), or fp32 partial sums for a K split, summed
+// by splitk_reduce_kernel.  Every mbarrier wait is bounded;
 // on expiry the kernel records an error code in the library's error word,
 // waits (bounded) for its own copies and MMAs, frees TMEM and exits.
 #include <cuda.h>
@@ -47,7 +49,7 @@ constexpr int BK = 64;
 constexpr int THREADS = 320;
 constexpr int EPI_WARPS = 8;
 constexpr int MAX_K = 65536;
-constexpr uint32_t STG_BYTES = 32 * 32 * 2;      // one epilogue staging buffer: 32 rows x 32 channels
+constexpr uint32_t STG_BYTES = 32 * 64 * 2;      // one epilogue staging block: 32 rows x 64 channels
 constexpr long long WAIT_LIMIT = 4000000000LL;  // SM cycles (~2 s)
 enum : int { ERR_TMA_WAIT = 0x10, ERR_MMA_WAIT = 0x20, ERR_ACC_WAIT = 0x40, ERR_EPI_WAIT = 0x80 };
 
@@ -213,7 +215,7 @@ __device__ __forceinline__ void tma_store_4d(const CUtensorMap *m, const void *s
 }
 __device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
 // at most one store group may still be reading shared memory
-__device__ __forceinline__ void bulk_wait_read_1() { asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_read_0() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
 __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 
 // one unit of work: a 128 x BN tile and the K-range [it0, it1) it accumulates
@@ -281,7 +283,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(&accf_bar[b], 1);
-            mbar_init(&acce_bar[b], EPI_WARPS);  // one arrival per epilogue warp
+            mbar_init(&acce_bar[b], EPI_WARPS / 2);  // one arrival per warp of the group draining it
         }
         abort_sh = 0;
         issued_sh = 0;
@@ -372,28 +374,39 @@ __global__ void __launch_bounds__(THREADS, 1)
             }
             consumed_sh = g;
         }
-    } else {  // ---------------- epilogue: warps 2..9, two per TMEM lane group
-        const int g4 = warp & 3;          // TMEM lanes 32*g4 .. +31 belong to this warp
-        const int half = (warp - 2) >> 2;  // this warp drains chunks half, half + 2, ...
+    } else {  // ---------------- epilogue: warps 2..9
+        // two groups of four warps; group eg drains accumulator eg, i.e. the
+        // work units with lt % 2 == eg; within a group warp w reads TMEM lanes
+        // 32*(w%4) .. +31 (tile rows) and walks all channels in 64-wide chunks
+        const int eg = (warp - 2) >> 2;
+        const int g4 = warp & 3;
         const int row = g4 * 32 + lane;
-        uint8_t *my_stg = stg + (warp - 2) * 2 * STG_BYTES;
-        // origin of this warp's 32-row sub-box inside a tile (implicit mode)
+        uint8_t *buf = stg + (warp - 2) * STG_BYTES;  // one 32 x 64 staging block per warp
         const int r0 = g4 * 32;
         const int wq0 = IMPLICIT ? r0 % p.BW : 0;
         const int hp0 = IMPLICIT ? (r0 / p.BW) % p.BH : 0;
         const int ni0 = IMPLICIT ? r0 / (p.BW * p.BH) : 0;
-        int chunk = 0;
-        int lt = 0;
-        for (int u = blockIdx.x; u < total; u += gridDim.x, ++lt) {
-            const int b = lt & 1;
+        constexpr int NCH = BN / 64 > 0 ? BN / 64 : 1;  // 64-channel chunks per tile
+        int lt = eg;
+        for (int u = blockIdx.x + eg * gridDim.x; u < total; u += 2 * gridDim.x, lt += 2) {
             const uint32_t aph = (uint32_t)(lt >> 1) & 1u;
-            if (!mbar_wait(&accf_bar[b], aph)) {
+            const Work w = work_of(p, u, BN, IMPLICIT);
+            // bias of channels chunk + lane and chunk + 32 + lane, loaded before
+            // the accumulator wait so the latency is hidden
+            float bias_r[NCH][2];
+#pragma unroll
+            for (int i = 0; i < NCH; ++i)
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    const int kb = w.n0 + 64 * i + 32 * h + lane;
+                    bias_r[i][h] = (p.ksplit == 1 && kb < p.K) ? __ldg(p.bias + kb) : 0.f;
+                }
+            if (!mbar_wait(&accf_bar[eg], aph)) {
                 if (lane == 0) atomicOr(p.err, ERR_ACC_WAIT);
                 abort_sh = 1;
                 break;
             }
             tc_fence_after();
-            const Work w = work_of(p, u, BN, IMPLICIT);
             bool valid;
             int64_t pix;
             if (IMPLICIT) {
@@ -405,34 +418,36 @@ __global__ void __launch_bounds__(THREADS, 1)
                 pix = w.m0 + row;
                 valid = pix < p.Mout;
             }
-#pragma unroll 1
-            for (int c = half * 32; c < BN && w.n0 + c < p.K; c += 64) {
-                const int k0 = w.n0 + c;
-                // bias of channel k0 + lane, fetched before the TMEM load so its latency overlaps
-                const float bl = (p.ksplit == 1 && k0 + lane < p.K) ? __ldg(p.bias + k0 + lane) : 0.f;
-                uint32_t v[32];
-                __syncwarp();
-                tmem_ld32(tmem + ((uint32_t)(g4 * 32) << 16) + (uint32_t)(b * BN + c), v);
-                if (p.ksplit == 1) {
-                    // bias + activation -> 16-bit, staged in 64-byte-swizzled shared
-                    // memory (row = lane, 16-byte chunk j at j ^ ((row >> 1) & 3)),
-                    // then one TMA tensor store of the warp's 32 x 32 block; the
-                    // store clips rows and channels outside the output tensor
-                    uint32_t wv[16];
 #pragma unroll
-                    for (int j = 0; j < 16; ++j) {
-                        const float f0 =
-                            act_apply(__uint_as_float(v[2 * j]) + __shfl_sync(0xffffffffu, bl, 2 * j), p.act);
-                        const float f1 =
-                            act_apply(__uint_as_float(v[2 * j + 1]) + __shfl_sync(0xffffffffu, bl, 2 * j + 1), p.act);
-                        wv[j] = pack2<T>(f0, f1);
+            for (int ci = 0; ci < NCH; ++ci) {
+                const int k0 = w.n0 + 64 * ci;
+                if (k0 >= p.K) break;
+                const uint32_t taddr = tmem + ((uint32_t)(g4 * 32) << 16) + (uint32_t)(eg * BN + 64 * ci);
+                if (p.ksplit == 1) {
+                    // bias + activation -> 16-bit, staged with the 128-byte swizzle
+                    // (row = lane, 16-byte chunk j at j ^ (row & 7)), then one TMA
+                    // tensor store of the warp's 32 x 64 block, clipped at the edges
+                    uint32_t wv[32];
+#pragma unroll
+                    for (int h = 0; h < 2; ++h) {
+                        uint32_t v[32];
+                        __syncwarp();
+                        tmem_ld32(taddr + 32 * h, v);
+#pragma unroll
+                        for (int j = 0; j < 16; ++j) {
+                            const float f0 = act_apply(
+                                __uint_as_float(v[2 * j]) + __shfl_sync(0xffffffffu, bias_r[ci][h], 2 * j), p.act);
+                            const float f1 = act_apply(
+                                __uint_as_float(v[2 * j + 1]) + __shfl_sync(0xffffffffu, bias_r[ci][h], 2 * j + 1),
+                                p.act);
+                            wv[16 * h + j] = pack2<T>(f0, f1);
+                        }
                     }
-                    uint8_t *buf = my_stg + (chunk & 1) * STG_BYTES;
-                    if (lane == 0) bulk_wait_read_1();  // the store that last used this buffer has read it
+                    if (lane == 0) bulk_wait_read_0();  // the previous store has read the staging block
                     __syncwarp();
 #pragma unroll
-                    for (int j = 0; j < 4; ++j)
-                        *reinterpret_cast<uint4 *>(buf + lane * 64 + ((j ^ ((lane >> 1) & 3)) << 4)) =
+                    for (int j = 0; j < 8; ++j)
+                        *reinterpret_cast<uint4 *>(buf + lane * 128 + ((j ^ (lane & 7)) << 4)) =
                             make_uint4(wv[4 * j], wv[4 * j + 1], wv[4 * j + 2], wv[4 * j + 3]);
                     fence_proxy_async_smem();
                     __syncwarp();
@@ -443,25 +458,32 @@ __global__ void __launch_bounds__(THREADS, 1)
                             tma_store_2d(&mY, buf, k0, (int)(w.m0 + r0));
                         bulk_commit();
                     }
-                    ++chunk;
-                } else if (valid) {
-                    float *dst = p.part + ((int64_t)w.sp * p.Mout + pix) * p.K + k0;
-                    if (k0 + 32 <= p.K) {
+                } else {
 #pragma unroll
-                        for (int q4 = 0; q4 < 8; ++q4)
-                            reinterpret_cast<uint4 *>(dst)[q4] =
-                                make_uint4(v[4 * q4], v[4 * q4 + 1], v[4 * q4 + 2], v[4 * q4 + 3]);
-                    } else {
+                    for (int h = 0; h < 2; ++h) {
+                        uint32_t v[32];
+                        __syncwarp();
+                        tmem_ld32(taddr + 32 * h, v);
+                        const int kh = k0 + 32 * h;
+                        if (!valid || kh >= p.K) continue;
+                        float *dst = p.part + ((int64_t)w.sp * p.Mout + pix) * p.K + kh;
+                        if (kh + 32 <= p.K) {
 #pragma unroll
-                        for (int j = 0; j < 32; ++j)
-                            if (k0 + j < p.K) dst[j] = __uint_as_float(v[j]);
+                            for (int q4 = 0; q4 < 8; ++q4)
+                                reinterpret_cast<uint4 *>(dst)[q4] =
+                                    make_uint4(v[4 * q4], v[4 * q4 + 1], v[4 * q4 + 2], v[4 * q4 + 3]);
+                        } else {
+#pragma unroll
+                            for (int j = 0; j < 32; ++j)
+                                if (kh + j < p.K) dst[j] = __uint_as_float(v[j]);
+                        }
                     }
                 }
             }
-            // every TMEM read of accumulator b by this warp is done: hand it back
+            // every TMEM read of accumulator eg by this warp is done: hand it back
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive(&acce_bar[b]);
+            if (lane == 0) mbar_arrive(&acce_bar[eg]);
         }
         if (lane == 0) bulk_wait_all();  // stores done before the CTA's shared memory is released
         __syncwarp();
@@ -626,7 +648,7 @@ template <typename T, int BN, bool IMPLICIT>
 static cudaError_t launch(const CUtensorMap *mA, const CUtensorMap &mB, const CUtensorMap &mY, const Params &p,
                           cudaStream_t st) {
     constexpr int STAGES = BN == 256 ? 4 : (BN == 128 ? 6 : 8);
-    constexpr size_t smem = (size_t)STAGES * (BM * BK * 2 + BN * BK * 2) + EPI_WARPS * 2 * STG_BYTES + 1024;
+    constexpr size_t smem = (size_t)STAGES * (BM * BK * 2 + BN * BK * 2) + EPI_WARPS * STG_BYTES + 1024;
     auto kern = conv_tc_kernel<T, BN, STAGES, IMPLICIT>;
     static bool attr = false;
     if (!attr) {
@@ -706,11 +728,11 @@ cudaError_t conv_tc(const LaunchArgs &a) {
         if (!encode(&mA[0], dt, 2, a.in[0], dims, str, box)) return cudaErrorInvalidValue;
         mA[1] = mA[2] = mA[3] = mA[0];
         p.mtiles = (int)((p.M + BM - 1) / BM);
-        // output [Mout][K], one 32-row x 32-channel box per epilogue-warp chunk
+        // output [Mout][K], one 32-row x 64-channel box per epilogue-warp chunk
         const uint64_t ydims[2] = {(uint64_t)p.K, (uint64_t)p.Mout};
         const uint64_t ystr[1] = {p.K * es};
-        const uint32_t ybox[2] = {32, 32};
-        if (!encode(&mY, dt, 2, a.out, ydims, ystr, ybox, CU_TENSOR_MAP_SWIZZLE_64B)) return cudaErrorInvalidValue;
+        const uint32_t ybox[2] = {64, 32};
+        if (!encode(&mY, dt, 2, a.out, ydims, ystr, ybox, CU_TENSOR_MAP_SWIZZLE_128B)) return cudaErrorInvalidValue;
     } else {
         p.BW = cf.BW, p.BH = cf.BH, p.BNI = cf.BNI;
         p.tq = (p.Q + cf.BW - 1) / cf.BW;
@@ -740,8 +762,8 @@ cudaError_t conv_tc(const LaunchArgs &a) {
         const uint32_t sbn = 32 / (sbw * sbh);
         const uint64_t ydims[4] = {(uint64_t)p.K, (uint64_t)p.Q, (uint64_t)p.P, (uint64_t)p.N};
         const uint64_t ystr[3] = {p.K * es, (uint64_t)p.Q * p.K * es, (uint64_t)p.P * p.Q * p.K * es};
-        const uint32_t ybox[4] = {32, sbw, sbh, sbn};
-        if (!encode(&mY, dt, 4, a.out, ydims, ystr, ybox, CU_TENSOR_MAP_SWIZZLE_64B)) return cudaErrorInvalidValue;
+        const uint32_t ybox[4] = {64, sbw, sbh, sbn};
+        if (!encode(&mY, dt, 4, a.out, ydims, ystr, ybox, CU_TENSOR_MAP_SWIZZLE_128B)) return cudaErrorInvalidValue;
     }
     if (p.mtiles <= 0 || (int64_t)p.mtiles * p.ntiles * p.ksplit > INT32_MAX) return cudaErrorInvalidValue;
     const bool bf = dt == SN_BF16;
