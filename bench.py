@@ -189,11 +189,16 @@ def main():
     ap.add_argument("--batch", type=int, default=32)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-b1", action="store_true")
+    ap.add_argument("--config", default="r50_b32",
+                    choices=["r50_b32", "bandwidth", "sweep", "mbv2_b1", "r50_b1", "tiny"],
+                    help="r50_b32 is the benchmark line; the others print one extra JSON line each")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
     ws, rank, local = dist_env()
     if args.impl == "reference":
         return run_reference(args, ws, rank)
+    if args.config != "r50_b32":
+        return run_extra_config(args)
 
     import torch
     import synth
@@ -371,6 +376,152 @@ def main():
     if dist:
         dist.destroy_process_group()
 
+
+
+# ----------------------------------------------------------------------------
+# the other configurations (one JSON line each; not the benchmark line)
+# ----------------------------------------------------------------------------
+
+def _single_layer_graph(sn, layer, in_shape, schema):
+    return sn.build_graph([dict(layer, inputs=[-1])], in_shape, schema, schema, [schema])
+
+
+def _time_back_to_back(torch, fn, reps=50, warm=5):
+    """Mean device time of `reps` back-to-back launches (CUDA events resolve ~2 us on this GPU)."""
+    for _ in range(warm):
+        fn()
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(reps):
+        fn()
+    b.record()
+    torch.cuda.synchronize()
+    return a.elapsed_time(b) / reps
+
+
+def _forced(sn, g, routine, variant=0):
+    import numpy as _np
+    t = g.cost_table()
+    c = [i for i in range(len(t["cost"])) if t["layer"][i] == 1 and sn.routine_name(int(t["routine"][i])) == routine
+         and t["variant"][i] == variant][0]
+    g.set_path([int(_np.flatnonzero(t["layer"] == 0)[0]), c, int(_np.flatnonzero(t["layer"] == 2)[0])])
+
+
+def run_extra_config(args):
+    import torch
+    import synth
+    import paper_2110_06037_gb300 as sn
+    pk, pk_kind = peaks()
+    hbm = pk["hbm_gbs"]
+    torch.cuda.set_device(0)
+    out = {"config": args.config, "peaks": pk_kind}
+    if args.config == "bandwidth":
+        # depthwise 3x3 (MobileNetV2 shapes) at batch 128 and the adapt conversion on
+        # ResNet-50 b32 activations; every working set is several times the 129 MB L2
+        rows = []
+        for (N, C, H, s_) in [(128, 144, 56, 1), (128, 96, 112, 2), (128, 192, 28, 1), (128, 576, 14, 1),
+                              (128, 960, 7, 1)]:
+            for lay in ("nhwc", "nchw"):
+                for var in (0, 1):
+                    sch = ("f16", lay)
+                    layer = synth.dwconv(C, 3, s_, act="relu6")
+                    layer["weight"] = np.zeros((C, 1, 3, 3), np.float32)
+                    layer["bias"] = np.zeros(C, np.float32)
+                    g = _single_layer_graph(sn, layer, (N, C, H, H), sch)
+                    _forced(sn, g, "dwconv2/direct", var)
+                    x = torch.zeros(sn.storage_shape((N, C, H, H), lay), dtype=torch.float16, device="cuda")
+                    y = g.new_output()
+                    ms = _time_back_to_back(torch, lambda: g.run(x, y), reps=20)
+                    P = (H + 2 - 3) // s_ + 1
+                    by = 2 * (N * C * H * H + N * C * P * P) + 2 * 9 * C + 4 * C
+                    rows.append({"kernel": "dwconv2/direct", "variant": sn.variant_name(5, var), "layout": lay,
+                                 "shape": [N, C, H, H], "stride": s_, "us": ms * 1e3, "gbs": by / ms / 1e6,
+                                 "frac": by / ms / 1e6 / hbm})
+        for shp in [(32, 64, 112, 112), (32, 256, 56, 56), (32, 1024, 14, 14)]:
+            for (a_, b_) in [(("bf16", "nchw"), ("bf16", "nhwc")), (("bf16", "nhwc"), ("bf16", "nchw")),
+                             (("f32", "nchw"), ("bf16", "nhwc")), (("bf16", "nhwc"), ("f32", "nchw"))]:
+                dt = {"f32": torch.float32, "bf16": torch.bfloat16}
+                x = torch.zeros(sn.storage_shape(shp, a_[1]), dtype=dt[a_[0]], device="cuda")
+                y = torch.empty(sn.storage_shape(shp, b_[1]), dtype=dt[b_[0]], device="cuda")
+                ms = _time_back_to_back(torch, lambda: sn.convert(x, a_, b_, shp, out=y), reps=20)
+                by = x.numel() * x.element_size() + y.numel() * y.element_size()
+                rows.append({"kernel": "adapt/convert", "from": "%s.%s" % a_, "to": "%s.%s" % b_, "shape": list(shp),
+                             "us": ms * 1e3, "gbs": by / ms / 1e6, "frac": by / ms / 1e6 / hbm})
+        out.update({"metric": "achieved HBM GB/s (algorithmic bytes / event time)", "peak_gbs": hbm, "rows": rows})
+    elif args.config == "sweep":
+        rows = []
+        for N in (1, 8, 32):
+            for H in (7, 14, 28, 56):
+                for C in (64, 128, 256, 512):
+                    for k in (1, 3):
+                        for s_ in (1, 2):
+                            for lay in ("nhwc", "nchw"):
+                                sch = ("f16", lay)
+                                x, layers = synth.single_conv(N, H, C, C, k, s_)
+                                g = _single_layer_graph(sn, layers[0], x.shape, sch)
+                                g.profile(warmup=2, iters=5, topk=0, passes=1)
+                                total, schemas, cands = g.select_path(sn.SN_SELECT_DPRS)
+                                t = g.cost_table()
+                                c = int(cands[1])
+                                xd = torch.zeros(sn.storage_shape(x.shape, lay), dtype=torch.float16, device="cuda")
+                                y = g.new_output()
+                                ms = _time_back_to_back(torch, lambda: g.run(xd, y), reps=10, warm=2)
+                                P = (H + 2 * (k // 2) - k) // s_ + 1
+                                fl = 2 * N * C * P * P * C * k * k
+                                by = 2 * (N * C * H * H + N * C * P * P + C * C * k * k)
+                                rows.append({"N": N, "H": H, "C": C, "k": k, "s": s_, "layout": lay,
+                                             "routine": sn.routine_name(int(t["routine"][c])),
+                                             "variant": int(t["variant"][c]), "us": ms * 1e3,
+                                             "tflops": fl / ms / 1e9, "gbs": by / ms / 1e6})
+        out.update({"metric": "single-layer conv, fp16, best routine by profiling + DPRS", "rows": rows})
+    else:
+        name = args.config
+        if name == "tiny":
+            x, layers = synth.tiny_cnn()
+            sch, io, dt = [("f32", "nchw"), ("f32", "nhwc")], ("f32", "nchw"), torch.float32
+        elif name == "mbv2_b1":
+            x, layers = synth.mobilenet_v2(1)
+            sch, io, dt = [("f16", "nchw"), ("f16", "nhwc")], ("f16", "nchw"), torch.float16
+        else:
+            x, layers = synth.resnet50(1)
+            sch, io, dt = [("f16", "nchw"), ("f16", "nhwc")], ("f16", "nchw"), torch.float16
+        stream = torch.cuda.Stream()
+        t0 = time.perf_counter()
+        with torch.cuda.stream(stream):
+            g = sn.build_graph(layers, x.shape, io, io, sch)
+            g.profile(warmup=3, iters=10, topk=2, passes=3)
+            total, schemas, cands = g.select_path(sn.SN_SELECT_DPRS)
+        stream.synchronize()
+        tune = time.perf_counter() - t0
+        g.set_option(sn.SN_OPT_CUDA_GRAPH, 1)
+        xd = torch.from_numpy(x).to(dt).cuda()
+        y = g.new_output()
+        flush = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
+        with torch.cuda.stream(stream):
+            for _ in range(5):
+                g.run(xd, y)
+        stream.synchronize()
+        lat = []
+        for _ in range(20):
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            with torch.cuda.stream(stream):
+                flush.zero_()
+                a.record(stream)
+                g.run(xd, y)
+                b.record(stream)
+            stream.synchronize()
+            lat.append(a.elapsed_time(b))
+        t = g.cost_table()
+        path = {}
+        for i in range(1, t["n_layers"] - 1):
+            r = sn.routine_name(int(t["routine"][int(cands[i])]))
+            path[r] = path.get(r, 0) + 1
+        out.update({"metric": "latency (ms), CUDA-graph replay, L2 flushed", "mean_ms": statistics.mean(lat),
+                    "std_ms": statistics.pstdev(lat), "median_ms": statistics.median(lat), "tuning_s": tune,
+                    "path_cost_ns": total, "routines_on_path": path,
+                    "schemas_on_path": {str(s_): int((schemas == i).sum()) for i, s_ in enumerate(g.schema_universe())}})
+    print(json.dumps(out))
 
 if __name__ == "__main__":
     main()

@@ -1,5 +1,6 @@
 // Adapt conversion, weight formatting, direct convolution, depthwise
 // convolution, pooling, elementwise add and dense routines (CUDA cores).
+#include <algorithm>
 #include <type_traits>
 
 #include "kern_common.cuh"
@@ -60,6 +61,45 @@ __global__ void __launch_bounds__(256) transpose_kernel(const Ti *__restrict__ x
     }
 }
 
+// the same transpose with 16-byte loads and stores (EI input, EO output
+// elements per vector); needs Cc % EI == 0, R % EO == 0 and aligned bases
+template <typename Ti, typename To>
+__global__ void __launch_bounds__(256) transpose_vec_kernel(const Ti *__restrict__ x, To *__restrict__ y,
+                                                             int64_t R, int64_t Cc) {
+    constexpr int EI = 16 / sizeof(Ti), EO = 16 / sizeof(To);
+    __shared__ float tile[TT][TT + 1];
+    const int64_t b = blockIdx.z;
+    const int64_t r0 = (int64_t)blockIdx.y * TT, c0 = (int64_t)blockIdx.x * TT;
+    const Ti *xb = x + b * R * Cc;
+    To *yb = y + b * R * Cc;
+    constexpr int VI = TT / EI;  // input vectors per tile row
+#pragma unroll
+    for (int i = threadIdx.x; i < TT * VI; i += 256) {
+        const int row = i / VI, cv = i % VI;
+        const int64_t r = r0 + row, c = c0 + cv * EI;
+        if (r < R && c < Cc) {
+            const uint4 v = *reinterpret_cast<const uint4 *>(xb + r * Cc + c);
+            const Ti *pv = reinterpret_cast<const Ti *>(&v);
+#pragma unroll
+            for (int e = 0; e < EI; ++e) tile[row][cv * EI + e] = ldf<Ti>(pv + e);
+        }
+    }
+    __syncthreads();
+    constexpr int VO = TT / EO;  // output vectors per tile row (output row = input column)
+#pragma unroll
+    for (int i = threadIdx.x; i < TT * VO; i += 256) {
+        const int orow = i / VO, ov = i % VO;
+        const int64_t c = c0 + orow, r = r0 + ov * EO;
+        if (c < Cc && r < R) {
+            uint4 v;
+            To *pv = reinterpret_cast<To *>(&v);
+#pragma unroll
+            for (int e = 0; e < EO; ++e) pv[e] = cvt<To>(tile[ov * EO + e][orow]);
+            *reinterpret_cast<uint4 *>(yb + c * R + r) = v;
+        }
+    }
+}
+
 // few channels (C <= 16): one thread per pixel moves all of its channels;
 // the planar side is read/written coalesced across threads, the interleaved
 // side as C consecutive elements per thread (C * 32 contiguous per warp)
@@ -110,7 +150,11 @@ static cudaError_t convert_t(const void *x, int lay_in, void *y, int lay_out, Sh
     if (s.n > 65535) return cudaErrorInvalidValue;
     dim3 grid((unsigned)((Cc + TT - 1) / TT), (unsigned)((R + TT - 1) / TT), (unsigned)s.n);
     if (grid.y > 65535) return cudaErrorInvalidValue;
-    transpose_kernel<Ti, To><<<grid, 256, 0, st>>>((const Ti *)x, (To *)y, R, Cc);
+    constexpr int EI = 16 / sizeof(Ti), EO = 16 / sizeof(To);
+    if (Cc % EI == 0 && R % EO == 0 && (uintptr_t)x % 16 == 0 && (uintptr_t)y % 16 == 0)
+        transpose_vec_kernel<Ti, To><<<grid, 256, 0, st>>>((const Ti *)x, (To *)y, R, Cc);
+    else
+        transpose_kernel<Ti, To><<<grid, 256, 0, st>>>((const Ti *)x, (To *)y, R, Cc);
     return cudaGetLastError();
 }
 
@@ -281,31 +325,6 @@ cudaError_t conv_direct(const LaunchArgs &a) {
 // depthwise convolution
 // ===========================================================================
 template <typename T>
-__global__ void dw_nchw(const T *__restrict__ x, const T *__restrict__ w, const float *__restrict__ bias,
-                        T *__restrict__ y, ConvDims d) {
-    const int64_t total = (int64_t)d.N * d.K * d.P * d.Q;
-    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total;
-         i += (int64_t)gridDim.x * blockDim.x) {
-        const int q = (int)(i % d.Q), p = (int)((i / d.Q) % d.P);
-        const int64_t nc = i / ((int64_t)d.Q * d.P);
-        const int c = (int)(nc % d.C);
-        const T *xc = x + nc * d.H * (int64_t)d.W;
-        const T *wc = w + (int64_t)c * d.R * d.S;
-        float acc = 0.f;
-        for (int r = 0; r < d.R; ++r) {
-            const int h = p * d.sh - d.ph + r * d.dh;
-            if (h < 0 || h >= d.H) continue;
-            for (int s = 0; s < d.S; ++s) {
-                const int ww = q * d.sw - d.pw + s * d.dw;
-                if (ww < 0 || ww >= d.W) continue;
-                acc += ldf<T>(xc + (int64_t)h * d.W + ww) * ldf<T>(wc + r * d.S + s);
-            }
-        }
-        stf<T>(y + i, act_apply(acc + bias[c], d.act));
-    }
-}
-
-template <typename T>
 __global__ void dw_nhwc(const T *__restrict__ x, const T *__restrict__ w, const float *__restrict__ bias,
                         T *__restrict__ y, ConvDims d) {
     const int64_t total = (int64_t)d.N * d.K * d.P * d.Q;
@@ -330,16 +349,368 @@ __global__ void dw_nhwc(const T *__restrict__ x, const T *__restrict__ w, const 
     }
 }
 
+// NHWC, 16 bytes of channels (E lanes) per thread and QB consecutive output
+// columns: each input vector a thread needs for its QB outputs is loaded from
+// global once per (tap row, column) and reused through L1 by its neighbours;
+// weights are [R][S][C].
+template <typename T, int QB, int SW>  // SW = 1 or 2: 3x3 fast path for that stride; 0 = any
+__global__ void __launch_bounds__(256, QB >= 4 ? 2 : 3) dw_nhwc_vec(const T *__restrict__ x, const T *__restrict__ w,
+                                                   const float *__restrict__ bias, T *__restrict__ y, ConvDims d) {
+    constexpr int E = 16 / sizeof(T);
+    const int CV = d.C / E;
+    const int QBLK = (d.Q + QB - 1) / QB;
+    const int64_t total = (int64_t)d.N * d.P * QBLK * CV;
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const int cv = (int)(i % CV);
+        int64_t rest = i / CV;
+        const int qb = (int)(rest % QBLK);
+        rest /= QBLK;
+        const int p = (int)(rest % d.P);
+        const int64_t n = rest / d.P;
+        const int c0 = cv * E, q0 = qb * QB;
+        float acc[QB][E];
+        {
+            float b[E];
+#pragma unroll
+            for (int e = 0; e < E; ++e) b[e] = bias[c0 + e];
+#pragma unroll
+            for (int j = 0; j < QB; ++j)
+#pragma unroll
+                for (int e = 0; e < E; ++e) acc[j][e] = b[e];
+        }
+        if (SW > 0) {
+            // 3x3 fast path: the input window of each tap row (QB outputs need
+            // (QB-1)*SW + 3 columns) is loaded once and reused by the three taps
+            constexpr int WN = (QB - 1) * (SW > 0 ? SW : 1) + 3;
+            const int wbase = q0 * SW - d.pw;
+#pragma unroll
+            for (int r = 0; r < 3; ++r) {
+                const int h = p * d.sh - d.ph + r * d.dh;
+                if (h < 0 || h >= d.H) continue;
+                const T *xrow = x + ((n * d.H + h) * (int64_t)d.W) * d.C + c0;
+                uint4 win[WN];
+#pragma unroll
+                for (int t = 0; t < WN; ++t) {
+                    const int ww = wbase + t;
+                    win[t] = (ww >= 0 && ww < d.W) ? *reinterpret_cast<const uint4 *>(xrow + (int64_t)ww * d.C)
+                                                    : make_uint4(0u, 0u, 0u, 0u);
+                }
+#pragma unroll
+                for (int s = 0; s < 3; ++s) {
+                    const uint4 wq = *reinterpret_cast<const uint4 *>(w + (int64_t)(r * 3 + s) * d.C + c0);
+                    const T *wp = reinterpret_cast<const T *>(&wq);
+                    float wf[E];
+#pragma unroll
+                    for (int e = 0; e < E; ++e) wf[e] = ldf<T>(wp + e);
+#pragma unroll
+                    for (int j = 0; j < QB; ++j) {
+                        const T *xp = reinterpret_cast<const T *>(&win[j * (SW > 0 ? SW : 1) + s]);
+#pragma unroll
+                        for (int e = 0; e < E; ++e) acc[j][e] = fmaf(ldf<T>(xp + e), wf[e], acc[j][e]);
+                    }
+                }
+            }
+        } else {
+            for (int r = 0; r < d.R; ++r) {
+                const int h = p * d.sh - d.ph + r * d.dh;
+                if (h < 0 || h >= d.H) continue;
+                const T *xrow = x + ((n * d.H + h) * (int64_t)d.W) * d.C + c0;
+                for (int s = 0; s < d.S; ++s) {
+                    const uint4 wq = *reinterpret_cast<const uint4 *>(w + (int64_t)(r * d.S + s) * d.C + c0);
+                    const T *wp = reinterpret_cast<const T *>(&wq);
+                    float wf[E];
+#pragma unroll
+                    for (int e = 0; e < E; ++e) wf[e] = ldf<T>(wp + e);
+#pragma unroll
+                    for (int j = 0; j < QB; ++j) {
+                        const int ww = (q0 + j) * d.sw - d.pw + s * d.dw;
+                        if (q0 + j < d.Q && ww >= 0 && ww < d.W) {
+                            const uint4 xq = *reinterpret_cast<const uint4 *>(xrow + (int64_t)ww * d.C);
+                            const T *xp = reinterpret_cast<const T *>(&xq);
+#pragma unroll
+                            for (int e = 0; e < E; ++e) acc[j][e] = fmaf(ldf<T>(xp + e), wf[e], acc[j][e]);
+                        }
+                    }
+                }
+            }
+        }
+        T *yrow = y + ((n * d.P + p) * (int64_t)d.Q) * d.C + c0;
+#pragma unroll
+        for (int j = 0; j < QB; ++j) {
+            if (q0 + j >= d.Q) break;
+            uint4 o;
+            T *op = reinterpret_cast<T *>(&o);
+#pragma unroll
+            for (int e = 0; e < E; ++e) op[e] = cvt<T>(act_apply(acc[j][e], d.act));
+            *reinterpret_cast<uint4 *>(yrow + (int64_t)(q0 + j) * d.C) = o;
+        }
+    }
+}
+
+// NCHW: one thread per (n, c, p) and 8 consecutive output columns; consecutive
+// threads take consecutive column blocks, so every load and store is
+// coalesced across the warp; weights are [C][R][S].
+template <typename T>
+__global__ void __launch_bounds__(256) dw_nchw_row(const T *__restrict__ x, const T *__restrict__ w,
+                                                   const float *__restrict__ bias, T *__restrict__ y, ConvDims d) {
+    constexpr int QB = 8;
+    const int QBLK = (d.Q + QB - 1) / QB;
+    const int64_t total = (int64_t)d.N * d.C * d.P * QBLK;
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const int qb = (int)(i % QBLK);
+        int64_t rest = i / QBLK;
+        const int p = (int)(rest % d.P);
+        const int64_t nc = rest / d.P;
+        const int c = (int)(nc % d.C);
+        const int q0 = qb * QB;
+        const T *xc = x + nc * d.H * (int64_t)d.W;
+        const T *wc = w + (int64_t)c * d.R * d.S;
+        const float bv = bias[c];
+        float acc[QB];
+#pragma unroll
+        for (int j = 0; j < QB; ++j) acc[j] = bv;
+        for (int r = 0; r < d.R; ++r) {
+            const int h = p * d.sh - d.ph + r * d.dh;
+            if (h < 0 || h >= d.H) continue;
+            const T *xr = xc + (int64_t)h * d.W;
+            for (int s = 0; s < d.S; ++s) {
+                const float wv = ldf<T>(wc + r * d.S + s);
+#pragma unroll
+                for (int j = 0; j < QB; ++j) {
+                    const int ww = (q0 + j) * d.sw - d.pw + s * d.dw;
+                    if (q0 + j < d.Q && ww >= 0 && ww < d.W) acc[j] = fmaf(ldf<T>(xr + ww), wv, acc[j]);
+                }
+            }
+        }
+        T *yr = y + (nc * d.P + p) * (int64_t)d.Q;
+        if (sizeof(T) == 2 && q0 + QB <= d.Q && ((uintptr_t)(yr + q0) & 15) == 0) {
+            uint4 o;
+            T *op = reinterpret_cast<T *>(&o);
+#pragma unroll
+            for (int j = 0; j < QB; ++j) op[j] = cvt<T>(act_apply(acc[j], d.act));
+            *reinterpret_cast<uint4 *>(yr + q0) = o;
+        } else {
+#pragma unroll
+            for (int j = 0; j < QB; ++j)
+                if (q0 + j < d.Q) stf<T>(yr + q0 + j, act_apply(acc[j], d.act));
+        }
+    }
+}
+
+// NHWC 3x3 (dilation 1) with shared-memory halo staging.  A work unit is TP
+// x TQ output pixels of one image and a 128-byte slice of channels; its input
+// halo ((TP-1)*SW+3 rows x (TQ-1)*SW+3 columns x 128 bytes) is copied into
+// shared memory with cp.async (zero-filled outside the image, which is the
+// padding).  The CTA is persistent with a ring of STAGES halo buffers: the
+// halos of its next STAGES-1 units are in flight while the current one is
+// computed from shared memory.
+// Every input byte comes from DRAM once (plus the halo overlap) and the nine
+// taps are served by shared memory.
+constexpr int DW_TP = 8;
+template <int SW> struct DwTQ { static constexpr int v = SW == 1 ? 16 : 8; };  // output columns per unit
+
+__device__ __forceinline__ void cp_async16(void *smem, const void *gmem, bool valid) {
+    const uint32_t sa = (uint32_t)__cvta_generic_to_shared(smem);
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(sa), "l"(gmem), "r"(valid ? 16 : 0)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
+
+template <typename T, int SW, int STAGES>
+__global__ void __launch_bounds__(256, 2) dw3_nhwc_halo(const T *__restrict__ x, const T *__restrict__ w,
+                                                        const float *__restrict__ bias, T *__restrict__ y, ConvDims d) {
+    constexpr int DW_TQ = DwTQ<SW>::v;
+    constexpr int E = 16 / sizeof(T);          // elements per 16-byte vector
+    constexpr int VS = 8;                      // vectors per 128-byte channel slice
+    constexpr int IH = (DW_TP - 1) * SW + 3, IW = (DW_TQ - 1) * SW + 3;
+    constexpr int HALO = IH * IW * VS;         // 16-byte vectors per buffer
+    extern __shared__ uint4 halo_smem[];
+    const int slices = (d.C * (int)sizeof(T) + 127) / 128;
+    const int tpn = (d.P + DW_TP - 1) / DW_TP, tqn = (d.Q + DW_TQ - 1) / DW_TQ;
+    const int64_t units = (int64_t)d.N * tpn * tqn * slices;
+    const int CV = d.C / E;  // 16-byte vectors per pixel
+    auto issue = [&](int64_t u, uint4 *buf) {
+        const int cs = (int)(u % slices);
+        int64_t r = u / slices;
+        const int tq = (int)(r % tqn);
+        r /= tqn;
+        const int tp = (int)(r % tpn);
+        const int64_t n = r / tpn;
+        const int h0 = tp * DW_TP * SW - d.ph, w0 = tq * DW_TQ * SW - d.pw;
+        for (int i = threadIdx.x; i < HALO; i += blockDim.x) {
+            const int v = i % VS, px = i / VS, ih = px / IW, iw = px % IW;
+            const int h = h0 + ih, ww = w0 + iw, cv = cs * VS + v;
+            const bool ok = h >= 0 && h < d.H && ww >= 0 && ww < d.W && cv < CV;
+            const T *src = ok ? x + (((n * d.H + h) * d.W + ww) * (int64_t)d.C + (int64_t)cv * E) : x;
+            cp_async16(buf + i, src, ok);
+        }
+        cp_async_commit();
+    };
+    const int v = threadIdx.x % VS;  // this thread's vector within the slice
+    // prologue: the first STAGES-1 units of this CTA in flight
+    for (int k = 0; k < STAGES - 1; ++k) {
+        const int64_t uk = blockIdx.x + (int64_t)k * gridDim.x;
+        if (uk < units) issue(uk, halo_smem + k * HALO);
+        else cp_async_commit();  // keep the group count uniform
+    }
+    int buf = 0;
+    for (int64_t u = blockIdx.x; u < units; u += gridDim.x, buf = (buf + 1) % STAGES) {
+        const int64_t un = u + (int64_t)(STAGES - 1) * gridDim.x;
+        if (un < units) issue(un, halo_smem + ((buf + STAGES - 1) % STAGES) * HALO);
+        else cp_async_commit();
+        cp_async_wait<STAGES - 1>();  // the current unit's halo has landed
+        __syncthreads();
+        const uint4 *hb = halo_smem + buf * HALO;
+        const int cs = (int)(u % slices);
+        int64_t r = u / slices;
+        const int tq = (int)(r % tqn);
+        r /= tqn;
+        const int tp = (int)(r % tpn);
+        const int64_t n = r / tpn;
+        const int cv = cs * VS + v;
+        if (cv < CV) {
+            const int c0 = cv * E;
+            float wf[9][E], bv[E];
+#pragma unroll
+            for (int t = 0; t < 9; ++t) {
+                const uint4 wq = *reinterpret_cast<const uint4 *>(w + (int64_t)t * d.C + c0);
+                const T *wp = reinterpret_cast<const T *>(&wq);
+#pragma unroll
+                for (int e = 0; e < E; ++e) wf[t][e] = ldf<T>(wp + e);
+            }
+#pragma unroll
+            for (int e = 0; e < E; ++e) bv[e] = bias[c0 + e];
+            for (int px = threadIdx.x / VS; px < DW_TP * DW_TQ; px += blockDim.x / VS) {
+                const int op = px / DW_TQ, oq = px % DW_TQ;
+                const int p = tp * DW_TP + op, q = tq * DW_TQ + oq;
+                if (p >= d.P || q >= d.Q) continue;
+                float acc[E];
+#pragma unroll
+                for (int e = 0; e < E; ++e) acc[e] = bv[e];
+#pragma unroll
+                for (int rr = 0; rr < 3; ++rr)
+#pragma unroll
+                    for (int ss = 0; ss < 3; ++ss) {
+                        const uint4 xq = hb[((op * SW + rr) * IW + oq * SW + ss) * VS + v];
+                        const T *xp = reinterpret_cast<const T *>(&xq);
+#pragma unroll
+                        for (int e = 0; e < E; ++e) acc[e] = fmaf(ldf<T>(xp + e), wf[rr * 3 + ss][e], acc[e]);
+                    }
+                uint4 o;
+                T *opp = reinterpret_cast<T *>(&o);
+#pragma unroll
+                for (int e = 0; e < E; ++e) opp[e] = cvt<T>(act_apply(acc[e], d.act));
+                *reinterpret_cast<uint4 *>(y + ((n * d.P + p) * (int64_t)d.Q + q) * d.C + c0) = o;
+            }
+        }
+        __syncthreads();  // everyone is done with this buffer before it is refilled
+    }
+}
+
+// NCHW 3x3: a block owns TH output rows of one (n, c) plane.  The input rows
+// they need (contiguous in NCHW) are staged in shared memory with coalesced
+// loads, zero-padded left/right and outside the image; then consecutive
+// threads compute consecutive outputs of the tile, so the stores are
+// coalesced too.  Weights are [C][3][3].
+template <typename T>
+__global__ void __launch_bounds__(256) dw3_nchw_tile(const T *__restrict__ x, const T *__restrict__ w,
+                                                     const float *__restrict__ bias, T *__restrict__ y, ConvDims d,
+                                                     int TH) {
+    extern __shared__ float dw_tile[];
+    const int tiles = (d.P + TH - 1) / TH;
+    const int64_t nc = blockIdx.x / tiles;
+    const int p0 = (int)(blockIdx.x % tiles) * TH;
+    const int c = (int)(nc % d.C);
+    const int rows = (TH - 1) * d.sh + 1 + 2 * d.dh;  // input rows touched by TH output rows
+    const int WP = d.W + 2 * d.pw;                     // padded width
+    const int h0 = p0 * d.sh - d.ph;
+    const T *xc = x + nc * d.H * (int64_t)d.W;
+    for (int i = threadIdx.x; i < rows * WP; i += blockDim.x) {
+        const int rr = i / WP, cc = i - rr * WP;
+        const int h = h0 + rr, ww = cc - d.pw;
+        dw_tile[i] = (h >= 0 && h < d.H && ww >= 0 && ww < d.W) ? ldf<T>(xc + (int64_t)h * d.W + ww) : 0.f;
+    }
+    float wr[9];
+#pragma unroll
+    for (int t = 0; t < 9; ++t) wr[t] = ldf<T>(w + (int64_t)c * 9 + t);
+    const float bv = bias[c];
+    __syncthreads();
+    const int pend = min(TH, d.P - p0);
+    T *yc = y + nc * d.P * (int64_t)d.Q;
+    for (int i = threadIdx.x; i < pend * d.Q; i += blockDim.x) {
+        const int pr = i / d.Q, q = i - pr * d.Q;
+        const float *base = dw_tile + (pr * d.sh) * WP + q * d.sw;
+        float acc = bv;
+#pragma unroll
+        for (int r = 0; r < 3; ++r)
+#pragma unroll
+            for (int s = 0; s < 3; ++s) acc = fmaf(base[r * d.dh * WP + s * d.dw], wr[r * 3 + s], acc);
+        stf<T>(yc + (int64_t)(p0 + pr) * d.Q + q, act_apply(acc, d.act));
+    }
+}
+
 cudaError_t dwconv(const LaunchArgs &a) {
+    // routine parameter (variant): NHWC 0 = register window (4 columns per
+    // thread), 1 = shared-memory halo tiles; NCHW 0 = row kernel (8 columns
+    // per thread), 1 = shared-memory plane tile
     const ConvDims d = conv_dims(a);
     const int64_t total = (int64_t)d.N * d.K * d.P * d.Q;
+    const int es = dtype_size(a.schema.dtype);
+    const bool vec_ok = (d.C * es) % 16 == 0 && (uintptr_t)a.in[0] % 16 == 0 && (uintptr_t)a.out % 16 == 0 &&
+                        (uintptr_t)a.wt % 16 == 0;
+    const bool k3 = d.R == 3 && d.S == 3 && d.dw == 1;
     SN_DT_SWITCH(a.schema.dtype, T, {
-        if (a.schema.layout == SN_NCHW)
-            dw_nchw<T><<<grid_for(total, 256), 256, 0, a.stream>>>((const T *)a.in[0], (const T *)a.wt,
-                                                                    a.bias, (T *)a.out, d);
-        else
-            dw_nhwc<T><<<grid_for(total, 256), 256, 0, a.stream>>>((const T *)a.in[0], (const T *)a.wt,
-                                                                    a.bias, (T *)a.out, d);
+        const T *x = (const T *)a.in[0];
+        const T *w = (const T *)a.wt;
+        T *y = (T *)a.out;
+        if (a.schema.layout == SN_NHWC && vec_ok) {
+            const int64_t cvec = d.C * es / 16;
+            const bool halo = k3 && d.dh == 1 && (d.sw == 1 || d.sw == 2) && d.sh == d.sw;
+            if (a.variant == 1 && halo) {
+                const int slices = (int)((d.C * (int64_t)es + 127) / 128);
+                const int tq = d.sw == 1 ? DwTQ<1>::v : DwTQ<2>::v;
+                const int64_t units = (int64_t)d.N * ((d.P + DW_TP - 1) / DW_TP) * ((d.Q + tq - 1) / tq) * slices;
+                const unsigned gb = (unsigned)std::min<int64_t>(units, 152LL * 2);
+                static bool attr = false;
+                const size_t sm1 = 4 * (size_t)((DW_TP - 1) + 3) * ((DwTQ<1>::v - 1) + 3) * 8 * 16;
+                const size_t sm2 = 3 * (size_t)((DW_TP - 1) * 2 + 3) * ((DwTQ<2>::v - 1) * 2 + 3) * 8 * 16;
+                if (!attr) {
+                    cudaFuncSetAttribute(dw3_nhwc_halo<T, 1, 4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm1);
+                    cudaFuncSetAttribute(dw3_nhwc_halo<T, 2, 3>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm2);
+                    attr = true;
+                }
+                if (d.sw == 1) dw3_nhwc_halo<T, 1, 4><<<gb, 256, sm1, a.stream>>>(x, w, a.bias, y, d);
+                else dw3_nhwc_halo<T, 2, 3><<<gb, 256, sm2, a.stream>>>(x, w, a.bias, y, d);
+            } else {
+                const unsigned gb = grid_for((int64_t)d.N * d.P * ((d.Q + 3) / 4) * cvec, 256, 152LL * 16);
+                if (k3 && d.sw == 1) dw_nhwc_vec<T, 4, 1><<<gb, 256, 0, a.stream>>>(x, w, a.bias, y, d);
+                else if (k3 && d.sw == 2) dw_nhwc_vec<T, 4, 2><<<gb, 256, 0, a.stream>>>(x, w, a.bias, y, d);
+                else dw_nhwc_vec<T, 4, 0><<<gb, 256, 0, a.stream>>>(x, w, a.bias, y, d);
+            }
+        } else if (a.schema.layout == SN_NHWC) {
+            dw_nhwc<T><<<grid_for(total, 256), 256, 0, a.stream>>>(x, w, a.bias, y, d);
+        } else {
+            bool tiled = false;
+            if (a.variant == 1 && d.R == 3 && d.S == 3) {
+                int TH = (int)std::max<int64_t>(1, std::min<int64_t>(d.P, 512 / std::max(1, d.Q)));
+                auto tile_bytes = [&](int th) {
+                    return (size_t)((th - 1) * d.sh + 1 + 2 * d.dh) * (d.W + 2 * d.pw) * sizeof(float);
+                };
+                while (tile_bytes(TH) > 40 * 1024 && TH > 1) TH /= 2;
+                const int64_t blocks = (int64_t)d.N * d.C * ((d.P + TH - 1) / TH);
+                if (tile_bytes(TH) <= 40 * 1024 && blocks < ((int64_t)1 << 31)) {
+                    dw3_nchw_tile<T><<<(unsigned)blocks, 256, tile_bytes(TH), a.stream>>>(x, w, a.bias, y, d, TH);
+                    tiled = true;
+                }
+            }
+            if (!tiled)
+                dw_nchw_row<T><<<grid_for((int64_t)d.N * d.C * d.P * ((d.Q + 7) / 8), 256, 152LL * 16), 256, 0,
+                                 a.stream>>>(x, w, a.bias, y, d);
+        }
     });
     return cudaGetLastError();
 }

@@ -33,6 +33,7 @@ const char *variant_name(int32_t r, int32_t v) {
     switch (r) {
     case R_CONV_IGEMM: return v == 0 ? "tile=64x64" : "tile=128x64";
     case R_CONV_WINO: return v == 0 ? "gemm=simt" : "gemm=tc";
+    case R_DW_DIRECT: return v == 0 ? "nhwc:window|nchw:rows" : "nhwc:smem_halo|nchw:plane_tile";
     case R_CONV_TC:
     case R_CONV_IM2COL_TC:
     case R_DENSE_TC: return k::conv_tc_variant_name(v);
@@ -57,7 +58,7 @@ int32_t routine_variants(int32_t r, const Layer &l, const std::vector<Shape> &in
     case R_CONV_TC:
         return is_conv(l) ? k::conv_tc_variants(l, in[0], s) : 0;
     case R_DW_DIRECT:
-        return l.type == SN_L_DWCONV2 ? 1 : 0;
+        return l.type == SN_L_DWCONV2 ? 2 : 0;
     case R_MAXPOOL:
         return l.type == SN_L_MAXPOOL ? 1 : 0;
     case R_GAP:

@@ -92,8 +92,10 @@ def test_depthwise(case, schema):
     layer = synth.dwconv(C, 3, s, act="relu6")
     layer["weight"] = (rng.standard_normal((C, 1, 3, 3)) * np.sqrt(2 / 9)).astype(np.float32)
     layer["bias"] = (rng.standard_normal(C) * 0.1).astype(np.float32)
-    got = run_one(layer, x, schema, "dwconv2/direct", 0)
-    assert maxrel(got, ref_one(layer, x, schema[0])) <= TOL[schema[0]]
+    ref = ref_one(layer, x, schema[0])
+    for v in (0, 1):  # routine parameters: columns per thread / row vs plane-tile kernel
+        got = run_one(layer, x, schema, "dwconv2/direct", v)
+        assert maxrel(got, ref) <= TOL[schema[0]], v
 
 
 @pytest.mark.parametrize("schema", SCHEMAS)
