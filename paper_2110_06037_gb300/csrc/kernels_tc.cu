@@ -20,9 +20,10 @@
 // one K-range of a tile when the layer is split along K because it has too
 // few tiles to fill the GPU), A-sharing tiles adjacent, with two TMEM
 // accumulators so that draining one overlaps the main loop of the next.
-// Warp roles (320 threads): warp 0 = TMA producer (+ TMEM allocation),
-// warp 1 = MMA issuer (one thread), warps 2-9 = epilogue in two groups of
-// four, group g draining accumulator g (alternate work units): TMEM ->
+// Warp roles (416 threads): warps 0 and 10-12 = TMA producers, each filling
+// every NPROD-th stage (warp 0 also allocates TMEM), warp 1 = MMA issuer (one
+// thread), warps 2-9 = epilogue, all eight draining each accumulator (four
+// row quarters x two column halves): TMEM ->
 // registers -> bias + activation -> fp16/bf16 -> 128-byte-swizzled staging
 // in shared memory -> one TMA tensor store per 32 rows x 64 channels
 // (clipped at the tensor edges), or fp32 partial sums for a K split, summed
@@ -37,229 +38,33 @@
 #include <type_traits>
 #include <vector>
 
-#include "kern_common.cuh"
+#include "tc_common.cuh"
 
 namespace sn {
 namespace k {
 
 namespace tc {
 
-constexpr int BM = 128;
-constexpr int BK = 64;
-constexpr int THREADS = 320;
-constexpr int EPI_WARPS = 8;
-constexpr int MAX_K = 65536;
-constexpr uint32_t STG_BYTES = 32 * 64 * 2;      // one epilogue staging block: 32 rows x 64 channels
-constexpr long long WAIT_LIMIT = 4000000000LL;  // SM cycles (~2 s)
-enum : int { ERR_TMA_WAIT = 0x10, ERR_MMA_WAIT = 0x20, ERR_ACC_WAIT = 0x40, ERR_EPI_WAIT = 0x80 };
-
-struct Params {
-    int32_t N, H, W, C, K, P, Q, R, S;
-    int32_t stride, ph, pw, dh, dw;
-    int32_t cblocks, kiters, ksplit;
-    int32_t BW, BH, BNI, tq, tp;   // pixel-tile geometry (implicit mode)
-    int32_t mtiles, ntiles;
-    int64_t M;                     // plain mode: input rows (= output pixels)
-    int64_t Mout;                  // output pixels N * P * Q
-    int32_t act;
-    const float *bias;
-    void *y;                       // output, NHWC, fp16/bf16
-    float *part;                   // K split: fp32 partial sums [ksplit][Mout][K]
-    int *err;                      // the library's device error word
-};
-
-// ---------------------------------------------------------------- PTX helpers
-__device__ __forceinline__ uint32_t su32(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
-
-__device__ __forceinline__ void mbar_init(uint64_t *b, uint32_t cnt) {
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(su32(b)), "r"(cnt) : "memory");
-}
-__device__ __forceinline__ void fence_mbar_init() {
-    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-}
-__device__ __forceinline__ void mbar_expect_tx(uint64_t *b, uint32_t bytes) {
-    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(su32(b)), "r"(bytes) : "memory");
-}
-__device__ __forceinline__ bool mbar_try(uint64_t *b, uint32_t parity) {
-    uint32_t ok;
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-        "selp.u32 %0, 1, 0, p;\n\t}"
-        : "=r"(ok)
-        : "r"(su32(b)), "r"(parity)
-        : "memory");
-    return ok != 0;
-}
-// bounded wait for the phase with the given parity; false on expiry
-__device__ __forceinline__ bool mbar_wait(uint64_t *b, uint32_t parity) {
-    if (mbar_try(b, parity)) return true;
-    const long long t0 = clock64();
-    while (!mbar_try(b, parity))
-        if (clock64() - t0 > WAIT_LIMIT) return false;
-    return true;
-}
-
-__device__ __forceinline__ void tma_2d(void *dst, const CUtensorMap *m, uint64_t *bar, int c0, int c1) {
-    asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4}], [%2];"
-        ::"r"(su32(dst)), "l"(reinterpret_cast<uint64_t>(m)), "r"(su32(bar)), "r"(c0), "r"(c1)
-        : "memory");
-}
-__device__ __forceinline__ void tma_3d(void *dst, const CUtensorMap *m, uint64_t *bar, int c0, int c1, int c2) {
-    asm volatile(
-        "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4, %5}], [%2];"
-        ::"r"(su32(dst)), "l"(reinterpret_cast<uint64_t>(m)), "r"(su32(bar)), "r"(c0), "r"(c1), "r"(c2)
-        : "memory");
-}
-__device__ __forceinline__ void tma_4d(void *dst, const CUtensorMap *m, uint64_t *bar, int c0, int c1, int c2,
-                                       int c3) {
-    asm volatile(
-        "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4, %5, %6}], [%2];"
-        ::"r"(su32(dst)), "l"(reinterpret_cast<uint64_t>(m)), "r"(su32(bar)), "r"(c0), "r"(c1), "r"(c2), "r"(c3)
-        : "memory");
-}
-
-__device__ __forceinline__ void tmem_alloc(uint32_t *dst, uint32_t ncols) {
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(su32(dst)), "r"(ncols)
-                 : "memory");
-    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
-}
-__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
-}
-__device__ __forceinline__ void tc_fence_before() {
-    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-}
-__device__ __forceinline__ void tc_fence_after() {
-    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-}
-
-// D[tmem] (+)= A[smem] * B[smem]^T, both K-major, fp32 accumulate
-__device__ __forceinline__ void umma(uint32_t d, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "setp.ne.b32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}"
-        ::"r"(d), "l"(a), "l"(b), "r"(idesc), "r"(acc)
-        : "memory");
-}
-// arrive on `bar` once every previously issued MMA of this thread has completed
-__device__ __forceinline__ void umma_commit(uint64_t *bar) {
-    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(su32(bar))
-                 : "memory");
-}
-
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
-        "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
-        "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
-        : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]),
-          "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]), "=r"(v[15]),
-          "=r"(v[16]), "=r"(v[17]), "=r"(v[18]), "=r"(v[19]), "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]),
-          "=r"(v[24]), "=r"(v[25]), "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31])
-        : "r"(taddr));
-    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-}
-
-// shared-memory matrix descriptor: K-major, 128-byte swizzle, rows of 128 B,
-// 8-row groups 1024 B apart (SBO); LBO unused for this layout
-__device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr) {
-    uint64_t d = 0;
-    d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
-    d |= (uint64_t)1 << 16;
-    d |= (uint64_t)(1024 >> 4) << 32;
-    d |= (uint64_t)1 << 46;  // descriptor version for tcgen05
-    d |= (uint64_t)2 << 61;  // 128-byte swizzle
-    return d;
-}
-
-// instruction descriptor, kind::f16: fp32 accumulate, A/B fp16 (0) or bf16 (1), K-major
-template <typename T>
-__device__ __forceinline__ uint32_t idesc_f16(int M, int N) {
-    const uint32_t fmt = std::is_same<T, __half>::value ? 0u : 1u;
-    return (1u << 4) | (fmt << 7) | (fmt << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
-}
-
-template <typename T>
-__device__ __forceinline__ uint32_t pack2(float a, float b);
-template <>
-__device__ __forceinline__ uint32_t pack2<__half>(float a, float b) {
-    __half2 h = __floats2half2_rn(a, b);
-    return *reinterpret_cast<uint32_t *>(&h);
-}
-template <>
-__device__ __forceinline__ uint32_t pack2<__nv_bfloat16>(float a, float b) {
-    __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
-    return *reinterpret_cast<uint32_t *>(&h);
-}
-
-
-
-__device__ __forceinline__ void mbar_arrive(uint64_t *b) {
-    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(su32(b)) : "memory");
-}
-__device__ __forceinline__ void fence_proxy_async_smem() {
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-}
-__device__ __forceinline__ void tma_store_2d(const CUtensorMap *m, const void *src, int c0, int c1) {
-    asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.tile.bulk_group [%0, {%2, %3}], [%1];"
-                 ::"l"(reinterpret_cast<uint64_t>(m)), "r"(su32(src)), "r"(c0), "r"(c1)
-                 : "memory");
-}
-__device__ __forceinline__ void tma_store_4d(const CUtensorMap *m, const void *src, int c0, int c1, int c2, int c3) {
-    asm volatile("cp.async.bulk.tensor.4d.global.shared::cta.tile.bulk_group [%0, {%2, %3, %4, %5}], [%1];"
-                 ::"l"(reinterpret_cast<uint64_t>(m)), "r"(su32(src)), "r"(c0), "r"(c1), "r"(c2), "r"(c3)
-                 : "memory");
-}
-__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
-// at most one store group may still be reading shared memory
-__device__ __forceinline__ void bulk_wait_read_0() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
-__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
-
-// one unit of work: a 128 x BN tile and the K-range [it0, it1) it accumulates
-struct Work {
-    int n0;          // first output channel
-    int64_t m0;      // plain mode: first pixel row
-    int q0, p0, i0;  // implicit mode: box origin (q, p, image)
-    int sp, it0, it1;
-};
-
-__device__ __forceinline__ Work work_of(const Params &p, int u, int bn, bool implicit) {
-    Work w;
-    w.sp = u % p.ksplit;
-    const int t = u / p.ksplit;
-    const int mt = t / p.ntiles, nt = t - mt * p.ntiles;  // A-sharing tiles are adjacent
-    w.n0 = nt * bn;
-    w.m0 = 0;
-    w.q0 = w.p0 = w.i0 = 0;
-    if (implicit) {
-        int bx = mt;
-        const int bq = bx % p.tq;
-        bx /= p.tq;
-        const int bp = bx % p.tp;
-        bx /= p.tp;
-        w.q0 = bq * p.BW;
-        w.p0 = bp * p.BH;
-        w.i0 = bx * p.BNI;
-    } else {
-        w.m0 = (int64_t)mt * BM;
-    }
-    w.it0 = (int)((int64_t)w.sp * p.kiters / p.ksplit);
-    w.it1 = (int)((int64_t)(w.sp + 1) * p.kiters / p.ksplit);
-    return w;
-}
-
 // --------------------------------------------------------------------- kernel
-template <typename T, int BN, int STAGES, bool IMPLICIT>
+// G = 1: one CTA per tile of 128 pixels x BN channels.
+// G = 2: a CTA pair (cluster of two on one TPC) shares a 256 x BN tile: each
+// CTA stages its own 128 pixel rows and half of the BN weight rows, the
+// leader (cluster rank 0) issues cta_group::2 MMAs that read both CTAs'
+// shared memory, and each CTA's TMEM receives its own 128 rows, drained by
+// its own epilogue.  Per SM this halves the weight bytes staged and read per
+// MMA, the shared-memory bandwidth that limits a one-CTA tile.
+template <typename T, int BN, int STAGES, bool IMPLICIT, int G, int KB>
 __global__ void __launch_bounds__(THREADS, 1)
     conv_tc_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ CUtensorMap mA1,
                    const __grid_constant__ CUtensorMap mA2, const __grid_constant__ CUtensorMap mA3,
                    const __grid_constant__ CUtensorMap mB, const __grid_constant__ CUtensorMap mY,
                    const Params p) {
-    constexpr uint32_t A_BYTES = BM * BK * 2;
-    constexpr uint32_t B_BYTES = BN * BK * 2;
+    // a stage holds KB 64-channel blocks of one filter tap; a block of A is
+    // 128 rows x 128 B, of B (BN / G) rows x 128 B (this CTA's share)
+    constexpr uint32_t A_BLK = BM * BK * 2;
+    constexpr uint32_t B_BLK = (BN / G) * BK * 2;
+    constexpr uint32_t A_BYTES = KB * A_BLK;
+    constexpr uint32_t B_BYTES = KB * B_BLK;
     constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
     constexpr uint32_t TMEM_COLS = 2 * BN;  // two accumulators
     extern __shared__ uint8_t smem_raw[];
@@ -269,116 +74,175 @@ __global__ void __launch_bounds__(THREADS, 1)
     __shared__ __align__(8) uint64_t acce_bar[2];  // epilogue -> MMA: accumulator drained
     __shared__ uint32_t tmem_sh;
     __shared__ volatile int abort_sh;
-    __shared__ int issued_sh, consumed_sh;
+    __shared__ int issued_sh[4], consumed_sh;
 
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t *stg = smem + STAGES * STAGE_BYTES;  // epilogue staging: 8 warps x 2 buffers, 1024-B aligned
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-    const int total = p.mtiles * p.ntiles * p.ksplit;
+    const uint32_t rank = G == 2 ? cluster_rank() : 0u;
+    const bool leader = rank == 0;
+    const int cid = G == 2 ? (int)(blockIdx.x / 2) : (int)blockIdx.x;  // pair (or CTA) index
+    const int ncl = G == 2 ? (int)(gridDim.x / 2) : (int)gridDim.x;
+    const int total = (p.mtiles + G - 1) / G * p.ntiles * p.ksplit;
+    // stop this CTA's loops, and the peer's
+    auto set_abort = [&]() {
+        abort_sh = 1;
+        if (G == 2) st_cluster_u32(mapa(su32((const void *)&abort_sh), rank ^ 1u), 1u);
+    };
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
-            mbar_init(&full_bar[s], 1);
+            mbar_init(&full_bar[s], 1);  // the (leader's) producer of the stage
             mbar_init(&empty_bar[s], 1);
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(&accf_bar[b], 1);
-            mbar_init(&acce_bar[b], EPI_WARPS / 2);  // one arrival per warp of the group draining it
+            mbar_init(&acce_bar[b], G * EPI_WARPS);  // one arrival per epilogue warp (of both CTAs)
         }
         abort_sh = 0;
-        issued_sh = 0;
+        issued_sh[0] = issued_sh[1] = issued_sh[2] = issued_sh[3] = 0;
         consumed_sh = 0;
         fence_mbar_init();
     }
-    if (warp == 0) tmem_alloc(&tmem_sh, TMEM_COLS);
+    if (G == 2) cluster_sync_all();  // both CTAs' barriers exist before either signals the other
+    if (warp == 0) tmem_alloc<G>(&tmem_sh, TMEM_COLS);
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = tmem_sh;
 
-    if (warp == 0) {
-        if (lane == 0) {  // ---------------- TMA producer
-            int g = 0;
+    constexpr int NPROD = producers_for(STAGES);
+    const int prod = warp == 0 ? 0 : (warp >= 10 ? warp - 9 : -1);  // producer index of this warp
+    if (prod >= 0) {
+        if (lane == 0 && prod < NPROD) {  // ---------------- TMA producers
+            // Producer `prod` fills the stages s with s % NPROD == prod (A and B
+            // of every CTA's own rows); several issuing threads, because one
+            // thread's issue loop is slower than the MMAs of a stage.  The
+            // tap / channel-block position advances incrementally for every
+            // K step, with no division per step.
+            const int cblocks = p.cblocks, S = p.S, dh = p.dh, dw = p.dw, ph0 = p.ph, pw0 = p.pw;
+            const int brow = (int)rank * (BN / G);
+            int g = 0, s = prod, issued = 0;
+            uint32_t par = 0;
             bool stop = false;
-            for (int u = blockIdx.x; u < total && !stop; u += gridDim.x) {
-                const Work w = work_of(p, u, BN, IMPLICIT);
+            for (int u = cid; u < total && !stop; u += ncl) {
+                const Work w = work_of(p, u, BN, IMPLICIT, G, (int)rank);
+                const int steps_per_tap = cblocks / KB;
+                int cb = (w.it0 % steps_per_tap) * KB;
+                int tap = w.it0 / steps_per_tap;
+                int r = tap / S, ss = tap - r * S;
                 for (int it = w.it0; it < w.it1; ++it, ++g) {
-                    const int s = g % STAGES;
-                    const uint32_t ph = (uint32_t)(g / STAGES) & 1u;
-                    if (!mbar_wait(&empty_bar[s], ph ^ 1u)) {
-                        atomicOr(p.err, ERR_TMA_WAIT);
-                        abort_sh = 1;
-                    }
-                    if (abort_sh) {
-                        stop = true;
-                        break;
-                    }
-                    uint8_t *sa = smem + s * STAGE_BYTES;
-                    uint8_t *sb = sa + A_BYTES;
-                    const int tap = it / p.cblocks, cb = it - tap * p.cblocks;
-                    const int r = tap / p.S, ss = tap - r * p.S;
-                    const int c0 = cb * BK;
-                    mbar_expect_tx(&full_bar[s], STAGE_BYTES);
-                    if (IMPLICIT) {
-                        const int oh = r * p.dh - p.ph, ow = ss * p.dw - p.pw;
-                        if (p.stride == 1) {
-                            tma_4d(sa, &mA0, &full_bar[s], c0, w.q0 + ow, w.p0 + oh, w.i0);
-                        } else {  // stride 2: even/odd sub-lattice maps
-                            const int bh = oh & 1, bw = ow & 1;
-                            const int ah = (oh - bh) / 2, aw = (ow - bw) / 2;
-                            const CUtensorMap *m = bh ? (bw ? &mA3 : &mA2) : (bw ? &mA1 : &mA0);
-                            tma_4d(sa, m, &full_bar[s], c0, w.q0 + aw, w.p0 + ah, w.i0);
+                    if (g % NPROD == prod) {
+                        if (!mbar_wait(&empty_bar[s], par ^ 1u)) {
+                            atomicOr(p.err, ERR_TMA_WAIT);
+                            set_abort();
                         }
-                    } else {
-                        tma_2d(sa, &mA0, &full_bar[s], c0, (int)w.m0);
+                        if (abort_sh) {
+                            stop = true;
+                            break;
+                        }
+                        const uint32_t sa = su32(smem + s * STAGE_BYTES);
+                        // KB = 1: channel coordinate cb * 64 on the innermost axis;
+                        // KB > 1: the maps carry a block axis (stride 128 B) and one
+                        // box spans KB blocks
+                        const int c0 = cb * BK;
+                        // the leader's barrier counts the bytes of both CTAs
+                        if (leader) mbar_expect_tx(&full_bar[s], G * STAGE_BYTES);
+                        const uint32_t bar = G == 2 ? mapa(su32(&full_bar[s]), 0u) : su32(&full_bar[s]);
+                        if (IMPLICIT) {
+                            const int oh = r * dh - ph0, ow = ss * dw - pw0;
+                            const CUtensorMap *m = &mA0;
+                            int qa = w.q0 + ow, pa = w.p0 + oh;
+                            if (p.stride != 1) {  // stride 2: even/odd sub-lattice maps
+                                const int bh = oh & 1, bw = ow & 1;
+                                m = bh ? (bw ? &mA3 : &mA2) : (bw ? &mA1 : &mA0);
+                                qa = w.q0 + ((ow - bw) >> 1);
+                                pa = w.p0 + ((oh - bh) >> 1);
+                            }
+                            if (KB == 1)
+                                tma_4d<G>(sa, m, bar, c0, qa, pa, w.i0);
+                            else
+                                tma_5d<G>(sa, m, bar, 0, qa, pa, w.i0, cb);
+                        } else {
+                            if (KB == 1)
+                                tma_2d<G>(sa, &mA0, bar, c0, (int)w.m0);
+                            else
+                                tma_3d<G>(sa, &mA0, bar, 0, (int)w.m0, cb);
+                        }
+                        if (KB == 1)
+                            tma_3d<G>(sa + A_BYTES, &mB, bar, c0, tap, w.n0 + brow);
+                        else
+                            tma_4d<G>(sa + A_BYTES, &mB, bar, 0, tap, w.n0 + brow, cb);
+                        issued = g + 1;
+                        s += NPROD;
+                        if (s >= STAGES) {
+                            s -= STAGES;
+                            par ^= 1u;
+                        }
                     }
-                    tma_3d(sb, &mB, &full_bar[s], c0, tap, w.n0);
+                    if ((cb += KB) == cblocks) {
+                        cb = 0;
+                        ++tap;
+                        if (++ss == S) {
+                            ss = 0;
+                            ++r;
+                        }
+                    }
                 }
             }
-            issued_sh = g;
+            issued_sh[prod] = issued;
         }
     } else if (warp == 1) {
-        if (lane == 0) {  // ---------------- MMA issuer
-            const uint32_t idesc = idesc_f16<T>(BM, BN);
-            int g = 0, lt = 0;
+        if (lane == 0 && leader) {  // ---------------- MMA issuer (the pair's leader)
+            const uint32_t idesc = idesc_f16<T>(BM * G, BN);
+            const uint64_t desc0 = sdesc_sw128(su32(smem));  // stage 0, A; offsets add to the address field
+            int g = 0, lt = 0, s = 0;
+            uint32_t par = 0;
             bool stop = false;
-            for (int u = blockIdx.x; u < total && !stop; u += gridDim.x, ++lt) {
-                const Work w = work_of(p, u, BN, IMPLICIT);
+            for (int u = cid; u < total && !stop; u += ncl, ++lt) {
+                const Work w = work_of(p, u, BN, IMPLICIT, G, 0);
                 const int b = lt & 1;
                 const uint32_t aph = (uint32_t)(lt >> 1) & 1u;
-                if (!mbar_wait(&acce_bar[b], aph ^ 1u)) {
+                const bool drained = G == 2 ? mbar_wait_cluster(&acce_bar[b], aph ^ 1u) : mbar_wait(&acce_bar[b], aph ^ 1u);
+                if (!drained) {
                     atomicOr(p.err, ERR_EPI_WAIT);
-                    abort_sh = 1;
+                    set_abort();
                     break;
                 }
                 tc_fence_after();
                 const uint32_t d = tmem + (uint32_t)(b * BN);
                 for (int it = w.it0; it < w.it1; ++it, ++g) {
-                    const int s = g % STAGES;
-                    const uint32_t ph = (uint32_t)(g / STAGES) & 1u;
-                    if (!mbar_wait(&full_bar[s], ph)) {
+                    if (!mbar_wait(&full_bar[s], par)) {
                         atomicOr(p.err, ERR_MMA_WAIT);
-                        abort_sh = 1;
+                        set_abort();
                         stop = true;
                         break;
                     }
                     tc_fence_after();
-                    const uint32_t sa = su32(smem + s * STAGE_BYTES), sb = sa + A_BYTES;
+                    // descriptors of this stage; a K step of 16 is 32 bytes (2 units)
+                    const uint64_t da = desc0 + (uint64_t)((s * STAGE_BYTES) >> 4);
+                    const uint64_t db = da + (A_BYTES >> 4);
 #pragma unroll
-                    for (int k = 0; k < BK / 16; ++k)
-                        umma(d, sdesc_sw128(sa + k * 32), sdesc_sw128(sb + k * 32), idesc,
-                             (it > w.it0 || k > 0) ? 1u : 0u);
-                    umma_commit(&empty_bar[s]);  // frees the stage once these MMAs have read it
+                    for (int j = 0; j < KB; ++j)
+#pragma unroll
+                        for (int k = 0; k < BK / 16; ++k)
+                            umma<G>(d, da + j * (A_BLK >> 4) + 2 * k, db + j * (B_BLK >> 4) + 2 * k, idesc,
+                                    (it > w.it0 || j > 0 || k > 0) ? 1u : 0u);
+                    umma_commit<G>(&empty_bar[s]);  // frees the stage (in both CTAs) once read
+                    if (++s == STAGES) {
+                        s = 0;
+                        par ^= 1u;
+                    }
                 }
-                if (!stop) umma_commit(&accf_bar[b]);
+                if (!stop) umma_commit<G>(&accf_bar[b]);
             }
             consumed_sh = g;
         }
     } else {  // ---------------- epilogue: warps 2..9
-        // two groups of four warps; group eg drains accumulator eg, i.e. the
-        // work units with lt % 2 == eg; within a group warp w reads TMEM lanes
-        // 32*(w%4) .. +31 (tile rows) and walks all channels in 64-wide chunks
-        const int eg = (warp - 2) >> 2;
+        // Every unit is drained by all eight warps: warp w reads TMEM lanes
+        // 32*(w%4) .. +31 (tile rows) of the 64-channel chunks of its column
+        // half (w-2)/4 (both halves' chunks alternate when a tile has one).
+        const int half = (warp - 2) >> 2;
         const int g4 = warp & 3;
         const int row = g4 * 32 + lane;
         uint8_t *buf = stg + (warp - 2) * STG_BYTES;  // one 32 x 64 staging block per warp
@@ -387,23 +251,26 @@ __global__ void __launch_bounds__(THREADS, 1)
         const int hp0 = IMPLICIT ? (r0 / p.BW) % p.BH : 0;
         const int ni0 = IMPLICIT ? r0 / (p.BW * p.BH) : 0;
         constexpr int NCH = BN / 64 > 0 ? BN / 64 : 1;  // 64-channel chunks per tile
-        int lt = eg;
-        for (int u = blockIdx.x + eg * gridDim.x; u < total; u += 2 * gridDim.x, lt += 2) {
+        constexpr int CPH = NCH >= 2 ? NCH / 2 : 1;      // chunks per column half
+        int lt = 0;
+        for (int u = cid; u < total; u += ncl, ++lt) {
+            const int b = lt & 1;
             const uint32_t aph = (uint32_t)(lt >> 1) & 1u;
-            const Work w = work_of(p, u, BN, IMPLICIT);
-            // bias of channels chunk + lane and chunk + 32 + lane, loaded before
-            // the accumulator wait so the latency is hidden
-            float bias_r[NCH][2];
+            const Work w = work_of(p, u, BN, IMPLICIT, G, (int)rank);
+            // bias of this warp's channels (lane j holds channel chunk + 32h + j;
+            // the buffer is zero-padded to a multiple of 256 channels), loaded
+            // before the accumulator wait so that the latency is hidden
+            float bias_r[CPH][2];
 #pragma unroll
-            for (int i = 0; i < NCH; ++i)
+            for (int cj = 0; cj < CPH; ++cj)
 #pragma unroll
-                for (int h = 0; h < 2; ++h) {
-                    const int kb = w.n0 + 64 * i + 32 * h + lane;
-                    bias_r[i][h] = (p.ksplit == 1 && kb < p.K) ? __ldg(p.bias + kb) : 0.f;
-                }
-            if (!mbar_wait(&accf_bar[eg], aph)) {
+                for (int h = 0; h < 2; ++h)
+                    bias_r[cj][h] = (p.ksplit == 1 && half * CPH + cj < NCH)
+                                        ? __ldg(p.bias + w.n0 + 64 * (half * CPH + cj) + 32 * h + lane)
+                                        : 0.f;
+            if (!mbar_wait(&accf_bar[b], aph)) {
                 if (lane == 0) atomicOr(p.err, ERR_ACC_WAIT);
-                abort_sh = 1;
+                set_abort();
                 break;
             }
             tc_fence_after();
@@ -418,11 +285,14 @@ __global__ void __launch_bounds__(THREADS, 1)
                 pix = w.m0 + row;
                 valid = pix < p.Mout;
             }
+            // the idle CTA of a pair whose group has one tile stores nothing
+            const bool tile_live = w.mt < p.mtiles && (NCH >= 2 || half == 0);
 #pragma unroll
-            for (int ci = 0; ci < NCH; ++ci) {
+            for (int cj = 0; cj < CPH; ++cj) {
+                const int ci = half * CPH + cj;
                 const int k0 = w.n0 + 64 * ci;
-                if (k0 >= p.K) break;
-                const uint32_t taddr = tmem + ((uint32_t)(g4 * 32) << 16) + (uint32_t)(eg * BN + 64 * ci);
+                if (k0 >= p.K || !tile_live) break;
+                const uint32_t taddr = tmem + ((uint32_t)(g4 * 32) << 16) + (uint32_t)(b * BN + 64 * ci);
                 if (p.ksplit == 1) {
                     // bias + activation -> 16-bit, staged with the 128-byte swizzle
                     // (row = lane, 16-byte chunk j at j ^ (row & 7)), then one TMA
@@ -436,9 +306,9 @@ __global__ void __launch_bounds__(THREADS, 1)
 #pragma unroll
                         for (int j = 0; j < 16; ++j) {
                             const float f0 = act_apply(
-                                __uint_as_float(v[2 * j]) + __shfl_sync(0xffffffffu, bias_r[ci][h], 2 * j), p.act);
+                                __uint_as_float(v[2 * j]) + __shfl_sync(0xffffffffu, bias_r[cj][h], 2 * j), p.act);
                             const float f1 = act_apply(
-                                __uint_as_float(v[2 * j + 1]) + __shfl_sync(0xffffffffu, bias_r[ci][h], 2 * j + 1),
+                                __uint_as_float(v[2 * j + 1]) + __shfl_sync(0xffffffffu, bias_r[cj][h], 2 * j + 1),
                                 p.act);
                             wv[16 * h + j] = pack2<T>(f0, f1);
                         }
@@ -480,10 +350,15 @@ __global__ void __launch_bounds__(THREADS, 1)
                     }
                 }
             }
-            // every TMEM read of accumulator eg by this warp is done: hand it back
+            // every TMEM read of accumulator b by this warp is done: hand it back
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive(&acce_bar[eg]);
+            if (lane == 0) {
+                if (G == 2)
+                    mbar_arrive_cluster(mapa(su32(&acce_bar[b]), 0u));
+                else
+                    mbar_arrive(&acce_bar[b]);
+            }
         }
         if (lane == 0) bulk_wait_all();  // stores done before the CTA's shared memory is released
         __syncwarp();
@@ -492,18 +367,29 @@ __global__ void __launch_bounds__(THREADS, 1)
     tc_fence_before();
     __syncthreads();
     if (warp == 0) {
-        if (abort_sh && lane == 0) {
-            // let this CTA's own copies and MMAs land before its memory goes away
-            for (int g = consumed_sh; g < issued_sh; ++g)
-                mbar_wait(&full_bar[g % STAGES], (uint32_t)(g / STAGES) & 1u);
+        if (abort_sh && lane == 0 && leader) {
+            // let the copies and MMAs this CTA waited for land before its
+            // memory goes away (one deadline for the whole drain)
+            const long long t0 = clock64();
+            int issued = 0;
+            for (int i = 0; i < 4; ++i) issued = issued_sh[i] > issued ? issued_sh[i] : issued;
+            for (int g = consumed_sh; g < issued; ++g)
+                while (!mbar_try(&full_bar[g % STAGES], (uint32_t)(g / STAGES) & 1u) && clock64() - t0 < WAIT_LIMIT) {
+                }
             if (consumed_sh > 0) {
                 const int g = consumed_sh - 1;
-                mbar_wait(&empty_bar[g % STAGES], (uint32_t)(g / STAGES) & 1u);
+                while (!mbar_try(&empty_bar[g % STAGES], (uint32_t)(g / STAGES) & 1u) && clock64() - t0 < WAIT_LIMIT) {
+                }
             }
         }
         __syncwarp();
+    }
+    // neither CTA of a pair leaves while the other may still signal its
+    // barriers or the leader's MMAs may still write its TMEM
+    if (G == 2) cluster_sync_all();
+    if (warp == 0) {
         tc_fence_after();
-        tmem_dealloc(tmem, TMEM_COLS);
+        tmem_dealloc<G>(tmem, TMEM_COLS);
     }
 }
 
@@ -574,6 +460,8 @@ struct Config {
     int BN;
     int BW, BH, BNI;
     int ksplit;
+    int G;   // CTAs per tile: 1, or 2 (CTA pair, 256-pixel tile)
+    int KB;  // 64-channel blocks per pipeline stage (one TMA box spans them)
 };
 
 constexpr int kSmCount = 152;  // GB300; only used to decide which K splits to offer
@@ -595,41 +483,64 @@ static std::vector<Config> configs(const Layer &l, const Shape &in, sn_schema s)
     else bns = {64, 128, 256};
     const bool plain = c.kh == 1 && c.kw == 1 && c.sh == 1 && c.ph == 0 && c.pw == 0;
     const int64_t N = l.out.n, P = l.out.h, Q = l.out.w;
+    // one-CTA tiles (128 x BN) with K splits of {1, 2, 4}; CTA-pair tiles
+    // (256 x BN, BN >= 128) with K splits of {1, 2, 3, 4}; a split is offered
+    // while the units stay within two waves of the GPU and each part keeps
+    // at least four K steps
     auto push_splits = [&](Config cf, int64_t mtiles) {
+        const int64_t units = (mtiles + cf.G - 1) / cf.G * ((K + cf.BN - 1) / cf.BN);
+        const int64_t slots = 2 * kSmCount / cf.G;
         cf.ksplit = 1;
         out.push_back(cf);
-        const int64_t tiles = mtiles * ((K + cf.BN - 1) / cf.BN);
-        for (int ks : {2, 4})
-            if (tiles * ks <= 2 * kSmCount && kiters >= 4 * ks) {
+        for (int ks : {2, 3, 4}) {
+            if (ks == 3 && cf.G == 1) continue;
+            if (units * ks <= slots && kiters >= 4 * ks) {
                 cf.ksplit = ks;
                 out.push_back(cf);
             }
+        }
+    };
+    auto push_all = [&](Config cf, int64_t mtiles) {
+        for (int bn : bns) {
+            cf.BN = bn;
+            cf.G = 1;
+            push_splits(cf, mtiles);
+        }
+        for (int bn : bns)
+            if (bn >= 128) {
+                cf.BN = bn;
+                cf.G = 2;
+                // two channel blocks per stage when the channels split evenly
+                cf.KB = c.c_in % 128 == 0 ? 2 : 1;
+                push_splits(cf, mtiles);
+                cf.KB = 1;
+            }
     };
     if (plain) {
-        for (int bn : bns) push_splits({false, bn, 0, 0, 0, 1}, (N * P * Q + BM - 1) / BM);
+        push_all({false, 0, 0, 0, 0, 1, 1, 1}, (N * P * Q + BM - 1) / BM);
         return out;
     }
-    struct G {
+    struct Geo {
         double waste;
         int bw, bh, bni;
     };
-    std::vector<G> gs;
+    std::vector<Geo> gs;
     for (int bw = 1; bw <= 128; bw *= 2)
         for (int bh = 1; bw * bh <= 128; bh *= 2) {
             const int bni = 128 / (bw * bh);
             const double cover = (double)((Q + bw - 1) / bw * bw) * ((P + bh - 1) / bh * bh) * ((N + bni - 1) / bni * bni);
             gs.push_back({cover / (double)(N * P * Q), bw, bh, bni});
         }
-    std::sort(gs.begin(), gs.end(), [](const G &a, const G &b) {
+    std::sort(gs.begin(), gs.end(), [](const Geo &a, const Geo &b) {
         if (a.waste != b.waste) return a.waste < b.waste;
         if (a.bw != b.bw) return a.bw > b.bw;
         return a.bh > b.bh;
     });
     const int keep = std::min<int>(2, (int)gs.size());
     for (int gi = 0; gi < keep; ++gi) {
-        const G &gg = gs[gi];
+        const Geo &gg = gs[gi];
         const int64_t mtiles = ((Q + gg.bw - 1) / gg.bw) * ((P + gg.bh - 1) / gg.bh) * ((N + gg.bni - 1) / gg.bni);
-        for (int bn : bns) push_splits({true, bn, gg.bw, gg.bh, gg.bni, 1}, mtiles);
+        push_all({true, 0, gg.bw, gg.bh, gg.bni, 1, 1, 1}, mtiles);
     }
     return out;
 }
@@ -644,22 +555,44 @@ static int num_sms() {
     return n;
 }
 
-template <typename T, int BN, bool IMPLICIT>
+template <typename T, int BN, bool IMPLICIT, int G, int KB>
 static cudaError_t launch(const CUtensorMap *mA, const CUtensorMap &mB, const CUtensorMap &mY, const Params &p,
                           cudaStream_t st) {
-    constexpr int STAGES = BN == 256 ? 4 : (BN == 128 ? 6 : 8);
-    constexpr size_t smem = (size_t)STAGES * (BM * BK * 2 + BN * BK * 2) + EPI_WARPS * STG_BYTES + 1024;
-    auto kern = conv_tc_kernel<T, BN, STAGES, IMPLICIT>;
-    static bool attr = false;
-    if (!attr) {
+    constexpr int STAGES = stages_for(BN, G, KB);
+    constexpr size_t smem = (size_t)STAGES * KB * (BM * BK * 2 + (BN / G) * BK * 2) + EPI_WARPS * STG_BYTES + 1024;
+    static_assert(smem <= 227 * 1024, "shared memory per CTA");
+    auto kern = conv_tc_kernel<T, BN, STAGES, IMPLICIT, G, KB>;
+    static int max_groups = 0;  // co-resident CTAs (G = 1) or CTA pairs (G = 2)
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[1];
+    cfg.blockDim = dim3(THREADS);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    if (G == 2) {
+        attr[0].id = cudaLaunchAttributeClusterDimension;
+        attr[0].val.clusterDim.x = 2;
+        attr[0].val.clusterDim.y = 1;
+        attr[0].val.clusterDim.z = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+    }
+    if (!max_groups) {
         cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
-        attr = true;
+        if (G == 2) {
+            cfg.gridDim = dim3(2);
+            int n = 0;
+            e = cudaOccupancyMaxActiveClusters(&n, kern, &cfg);
+            if (e != cudaSuccess) return e;
+            if (n <= 0) return cudaErrorInvalidConfiguration;
+            max_groups = n;
+        } else {
+            max_groups = num_sms();
+        }
     }
-    const int total = p.mtiles * p.ntiles * p.ksplit;
-    const unsigned grid = (unsigned)std::min(total, num_sms());
-    kern<<<grid, THREADS, smem, st>>>(mA[0], mA[1], mA[2], mA[3], mB, mY, p);
-    cudaError_t e = cudaGetLastError();
+    const int total = (p.mtiles + G - 1) / G * p.ntiles * p.ksplit;
+    cfg.gridDim = dim3((unsigned)(G * std::min(total, max_groups)));
+    cudaError_t e = cudaLaunchKernelEx(&cfg, kern, mA[0], mA[1], mA[2], mA[3], mB, mY, p);
     if (e != cudaSuccess || p.ksplit == 1) return e;
     const int64_t n4 = p.Mout * (p.K / 4);
     splitk_reduce_kernel<T><<<grid_for(n4, 256), 256, 0, st>>>(p.part, p.bias, static_cast<T *>(p.y), p.Mout, p.K,
@@ -698,7 +631,8 @@ cudaError_t conv_tc(const LaunchArgs &a) {
     p.K = c.c_out, p.P = (int)l.out.h, p.Q = (int)l.out.w, p.R = c.kh, p.S = c.kw;
     p.stride = c.sh, p.ph = c.ph, p.pw = c.pw, p.dh = c.dh, p.dw = c.dw;
     p.cblocks = (p.C + BK - 1) / BK;
-    p.kiters = p.R * p.S * p.cblocks;
+    if (p.cblocks % cf.KB) return cudaErrorInvalidValue;
+    p.kiters = p.R * p.S * p.cblocks / cf.KB;  // K steps of KB channel blocks
     p.ksplit = cf.ksplit;
     p.act = c.act;
     p.bias = a.bias;
@@ -715,17 +649,22 @@ cudaError_t conv_tc(const LaunchArgs &a) {
     const int dt = a.schema.dtype;
     const uint64_t es = 2;
     CUtensorMap mA[4], mB, mY;
+    // KB > 1 (channels a multiple of 128): every map gets an outermost
+    // channel-block axis of stride 128 B over the 64-channel inner axis, so that
+    // one box lands KB consecutive 128-B-row blocks in shared memory
+    const bool blk = cf.KB > 1;
+    const uint64_t CB = (uint64_t)p.cblocks;
     {  // B: weights [K][R*S][C]
-        const uint64_t dims[3] = {(uint64_t)p.C, (uint64_t)(p.R * p.S), (uint64_t)p.K};
-        const uint64_t str[2] = {p.C * es, (uint64_t)p.R * p.S * p.C * es};
-        const uint32_t box[3] = {BK, 1, (uint32_t)cf.BN};
-        if (!encode(&mB, dt, 3, a.wt, dims, str, box)) return cudaErrorInvalidValue;
+        const uint64_t dims[4] = {blk ? 64 : (uint64_t)p.C, (uint64_t)(p.R * p.S), (uint64_t)p.K, CB};
+        const uint64_t str[3] = {p.C * es, (uint64_t)p.R * p.S * p.C * es, 128};
+        const uint32_t box[4] = {BK, 1, (uint32_t)(cf.BN / cf.G), (uint32_t)cf.KB};  // a CTA's share of the BN rows
+        if (!encode(&mB, dt, blk ? 4 : 3, a.wt, dims, str, box)) return cudaErrorInvalidValue;
     }
     if (!cf.implicit) {
-        const uint64_t dims[2] = {(uint64_t)p.C, (uint64_t)p.M};
-        const uint64_t str[1] = {p.C * es};
-        const uint32_t box[2] = {BK, BM};
-        if (!encode(&mA[0], dt, 2, a.in[0], dims, str, box)) return cudaErrorInvalidValue;
+        const uint64_t dims[3] = {blk ? 64 : (uint64_t)p.C, (uint64_t)p.M, CB};
+        const uint64_t str[2] = {p.C * es, 128};
+        const uint32_t box[3] = {BK, BM, (uint32_t)cf.KB};
+        if (!encode(&mA[0], dt, blk ? 3 : 2, a.in[0], dims, str, box)) return cudaErrorInvalidValue;
         mA[1] = mA[2] = mA[3] = mA[0];
         p.mtiles = (int)((p.M + BM - 1) / BM);
         // output [Mout][K], one 32-row x 64-channel box per epilogue-warp chunk
@@ -738,20 +677,22 @@ cudaError_t conv_tc(const LaunchArgs &a) {
         p.tq = (p.Q + cf.BW - 1) / cf.BW;
         p.tp = (p.P + cf.BH - 1) / cf.BH;
         const int tn = (p.N + cf.BNI - 1) / cf.BNI;
-        const uint32_t box[4] = {BK, (uint32_t)cf.BW, (uint32_t)cf.BH, (uint32_t)cf.BNI};
+        const uint32_t box[5] = {BK, (uint32_t)cf.BW, (uint32_t)cf.BH, (uint32_t)cf.BNI, (uint32_t)cf.KB};
+        const uint64_t c0dim = blk ? 64 : (uint64_t)p.C;
         if (p.stride == 1) {
-            const uint64_t dims[4] = {(uint64_t)p.C, (uint64_t)p.W, (uint64_t)p.H, (uint64_t)p.N};
-            const uint64_t str[3] = {p.C * es, (uint64_t)p.W * p.C * es, (uint64_t)p.H * p.W * p.C * es};
-            if (!encode(&mA[0], dt, 4, a.in[0], dims, str, box)) return cudaErrorInvalidValue;
+            const uint64_t dims[5] = {c0dim, (uint64_t)p.W, (uint64_t)p.H, (uint64_t)p.N, CB};
+            const uint64_t str[4] = {p.C * es, (uint64_t)p.W * p.C * es, (uint64_t)p.H * p.W * p.C * es, 128};
+            if (!encode(&mA[0], dt, blk ? 5 : 4, a.in[0], dims, str, box)) return cudaErrorInvalidValue;
             mA[1] = mA[2] = mA[3] = mA[0];
         } else {
             for (int bh = 0; bh < 2; ++bh)
                 for (int bw = 0; bw < 2; ++bw) {
                     const char *base = static_cast<const char *>(a.in[0]) + ((int64_t)bh * p.W + bw) * p.C * es;
-                    const uint64_t dims[4] = {(uint64_t)p.C, (uint64_t)(p.W / 2), (uint64_t)(p.H / 2), (uint64_t)p.N};
-                    const uint64_t str[3] = {2 * p.C * es, 2 * (uint64_t)p.W * p.C * es,
-                                             (uint64_t)p.H * p.W * p.C * es};
-                    if (!encode(&mA[bh * 2 + bw], dt, 4, base, dims, str, box)) return cudaErrorInvalidValue;
+                    const uint64_t dims[5] = {c0dim, (uint64_t)(p.W / 2), (uint64_t)(p.H / 2), (uint64_t)p.N, CB};
+                    const uint64_t str[4] = {2 * p.C * es, 2 * (uint64_t)p.W * p.C * es,
+                                             (uint64_t)p.H * p.W * p.C * es, 128};
+                    if (!encode(&mA[bh * 2 + bw], dt, blk ? 5 : 4, base, dims, str, box))
+                        return cudaErrorInvalidValue;
                 }
         }
         p.mtiles = p.tq * p.tp * tn;
@@ -767,18 +708,27 @@ cudaError_t conv_tc(const LaunchArgs &a) {
     }
     if (p.mtiles <= 0 || (int64_t)p.mtiles * p.ntiles * p.ksplit > INT32_MAX) return cudaErrorInvalidValue;
     const bool bf = dt == SN_BF16;
-#define SN_TC_LAUNCH(TT, BNV)                                                                     \
-    return cf.implicit ? launch<TT, BNV, true>(mA, mB, mY, p, a.stream)                            \
-                       : launch<TT, BNV, false>(mA, mB, mY, p, a.stream)
+#define SN_TC_LAUNCH(TT, BNV, GV, KBV)                                                            \
+    return cf.implicit ? launch<TT, BNV, true, GV, KBV>(mA, mB, mY, p, a.stream)                   \
+                       : launch<TT, BNV, false, GV, KBV>(mA, mB, mY, p, a.stream)
+#define SN_TC_LAUNCH_T(TT)                                                                          \
+    if (cf.G == 2) {                                                                                \
+        if (cf.KB == 2) {                                                                           \
+            if (cf.BN == 128) SN_TC_LAUNCH(TT, 128, 2, 2);                                          \
+            SN_TC_LAUNCH(TT, 256, 2, 2);                                                            \
+        }                                                                                           \
+        if (cf.BN == 128) SN_TC_LAUNCH(TT, 128, 2, 1);                                              \
+        SN_TC_LAUNCH(TT, 256, 2, 1);                                                                \
+    }                                                                                               \
+    if (cf.BN == 64) SN_TC_LAUNCH(TT, 64, 1, 1);                                                    \
+    if (cf.BN == 128) SN_TC_LAUNCH(TT, 128, 1, 1);                                                  \
+    SN_TC_LAUNCH(TT, 256, 1, 1)
     if (bf) {
-        if (cf.BN == 64) SN_TC_LAUNCH(__nv_bfloat16, 64);
-        if (cf.BN == 128) SN_TC_LAUNCH(__nv_bfloat16, 128);
-        SN_TC_LAUNCH(__nv_bfloat16, 256);
+        SN_TC_LAUNCH_T(__nv_bfloat16);
     } else {
-        if (cf.BN == 64) SN_TC_LAUNCH(__half, 64);
-        if (cf.BN == 128) SN_TC_LAUNCH(__half, 128);
-        SN_TC_LAUNCH(__half, 256);
+        SN_TC_LAUNCH_T(__half);
     }
+#undef SN_TC_LAUNCH_T
 #undef SN_TC_LAUNCH
 }
 

@@ -115,12 +115,16 @@ sn_status prepare_weights(Graph *g, int32_t li, int32_t r, int32_t v, sn_schema 
     } else {
         K = L.conv.c_out, Cg = L.conv.c_in / L.conv.groups, R = L.conv.kh, S = L.conv.kw;
     }
-    // bias: fp32 on the device, shared by every routine of the layer
+    // bias: fp32 on the device, shared by every routine of the layer, zero-
+    // padded to a multiple of 256 entries so that a tile's epilogue may read
+    // its whole channel range without a bounds check
     auto bit = g->bias_cache.find(li);
     if (bit == g->bias_cache.end()) {
         Buffer b;
-        sn_status rc = dev_alloc(g, L.bias.size() * sizeof(float), &b);
+        const size_t padded = (L.bias.size() + 255) / 256 * 256;
+        sn_status rc = dev_alloc(g, padded * sizeof(float), &b);
         if (rc != SN_OK) return rc;
+        SN_CUDA_TRY(cudaMemsetAsync(b.ptr, 0, padded * sizeof(float), st));
         SN_CUDA_TRY(cudaMemcpyAsync(b.ptr, L.bias.data(), L.bias.size() * sizeof(float),
                                     cudaMemcpyHostToDevice, st));
         bit = g->bias_cache.emplace(li, b).first;

@@ -2,7 +2,8 @@
 against the oracle, over every routine-parameter combination it offers:
 1x1 GEMM tiles, 3x3 stride-1 box tiles, stride-2 sub-lattice maps, channel
 counts that are not multiples of the 64-channel K block, output channels
-that end inside an epilogue chunk, ragged pixel tiles."""
+that end inside an epilogue chunk, ragged pixel tiles, CTA-pair tiles whose
+second CTA has no pixels, stages of one and of two 64-channel blocks."""
 import numpy as np
 import pytest
 
@@ -29,6 +30,8 @@ CASES = [
     (1, 96, 12, 12, 72, 5, 1, 2),     # 5x5
     (2, 256, 7, 7, 256, 3, 1, 1),     # few tiles: K-split variants (2, 4) offered
     (4, 512, 7, 7, 136, 1, 1, 0),     # plain GEMM K split, K not a multiple of 32
+    (2, 128, 16, 16, 128, 3, 2, 1),   # 3x3 s2 with two 64-channel blocks per pipeline stage
+    (2, 256, 14, 14, 512, 1, 2, 0),   # 1x1 s2 downsample, two blocks per stage
 ]
 
 
