@@ -15,6 +15,7 @@ replicas (one batch per rank, no collective on the data path).
 from __future__ import annotations
 
 import argparse
+import hashlib
 import json
 import os
 import statistics
@@ -57,21 +58,33 @@ class ClockSampler:
     def __init__(self, index):
         self.index = index
         self.proc = None
-        self.lines = []
+        self.lines = []  # (arrival time, csv line)
+        self.t0 = self.t1 = None
 
     def start(self):
+        """Start sampling and wait (up to 5 s) for the first sample, so that
+        the timed region that follows is covered."""
         try:
             self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.Q}",
-                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                          "--format=csv,noheader,nounits", "-lms", "50"],
                                          stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
             self.t = threading.Thread(target=self._read, daemon=True)
             self.t.start()
+            deadline = time.monotonic() + 5.0
+            while not self.lines and time.monotonic() < deadline:
+                time.sleep(0.01)
         except Exception:
             self.proc = None
 
     def _read(self):
         for line in self.proc.stdout:
-            self.lines.append(line.strip())
+            self.lines.append((time.monotonic(), line.strip()))
+
+    def begin(self):
+        self.t0 = time.monotonic()
+
+    def end(self):
+        self.t1 = time.monotonic()
 
     def stop(self):
         if not self.proc:
@@ -83,7 +96,11 @@ class ClockSampler:
             self.proc.kill()
         sm, mx, reasons = [], [], set()
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        for l in self.lines:
+        # samples that arrived while the timed region ran (plus the first one
+        # after it, which nvidia-smi took during its last interval)
+        inside = [l for (t, l) in self.lines if self.t0 is not None and self.t0 <= t <= (self.t1 or t)]
+        after = [l for (t, l) in self.lines if self.t1 is not None and t > self.t1][:1]
+        for l in inside + after:
             f = [x.strip() for x in l.split(",")]
             if len(f) < 7:
                 continue
@@ -97,6 +114,36 @@ class ClockSampler:
                     reasons.add(n)
         return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
                 "reasons": sorted(reasons), "samples": len(sm)}
+
+
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "conv_tc_r50_b32_bf16_traffic.md")
+
+
+def tc_sources_digest():
+    """sha256 over the tensor-core conv kernel sources: a DRAM-traffic figure
+    measured with ncu is reported only while these are unchanged."""
+    h = hashlib.sha256()
+    for f in ("kernels_tc.cu", "tc_common.cuh"):
+        with open(os.path.join(ROOT, "paper_2110_06037_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()
+
+
+def tc_traffic_per_step():
+    """DRAM bytes (read + write) of the step's conv2/igemm_tc launches from the
+    committed ncu summary, or None when it is missing or the kernel changed."""
+    try:
+        kv = {}
+        with open(TRAFFIC_FILE) as fh:
+            for line in fh:
+                if ":" in line:
+                    k, v = line.split(":", 1)
+                    kv[k.strip().strip("`- ")] = v.strip().strip("`")
+        if kv.get("kernel_sources_sha256") != tc_sources_digest():
+            return None
+        return float(kv["igemm_tc_dram_bytes_per_step"])
+    except (OSError, KeyError, ValueError):
+        return None
 
 
 def conv_work(layers, in_shape, elem=2):
@@ -183,15 +230,19 @@ def cpu_baseline_sample():
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--batch", type=int, default=32)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-b1", action="store_true")
     ap.add_argument("--config", default="r50_b32",
-                    choices=["r50_b32", "bandwidth", "sweep", "mbv2_b1", "r50_b1", "tiny"],
+                    choices=["r50_b32", "bandwidth", "sweep", "mbv2_b1", "r50_b1", "tiny", "layer"],
                     help="r50_b32 is the benchmark line; the others print one extra JSON line each")
+    ap.add_argument("--layer", default="32,512,56,512,3,1",
+                    help="--config layer: N,C,H,K,k,s of one bf16 NHWC conv (C -> K channels, HxH input)")
+    ap.add_argument("--variant", type=int, default=-1,
+                    help="--config layer: conv2/igemm_tc routine parameter index (-1: every one)")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
     ws, rank, local = dist_env()
@@ -241,6 +292,7 @@ def main():
         dist.barrier()
     torch.cuda.synchronize()
     clocks.start()
+    clocks.begin()
     torch.cuda.nvtx.range_push("sn_timed")
     with torch.cuda.stream(stream):
         for i in range(args.steps):
@@ -250,6 +302,7 @@ def main():
             ev[i][1].record(stream)
     torch.cuda.synchronize()
     torch.cuda.nvtx.range_pop()
+    clocks.end()
     if dist:
         dist.barrier()
     clk = clocks.stop()
@@ -317,7 +370,9 @@ def main():
     if dom == "conv2/igemm_tc":
         achieved = d["flop"] / (d["ms"] / 1e3) / 1e12
         roof = {"bound": "tensor", "achieved": achieved, "peak": sustained, "unit": "TFLOP/s",
-                "frac": achieved / sustained, "traffic": None}
+                "frac": achieved / sustained, "traffic": tc_traffic_per_step(),
+                "traffic_unit": "DRAM bytes per step over the igemm_tc launches (ncu, cold L2 per kernel)",
+                "algorithmic_bytes": d["bytes"]}
     elif dom in ("conv2/igemm_simt", "conv2/direct", "conv2/wino_f2x2_3x3"):
         ffma_peak = 2 * 128 * 152 * pk.get("sm_max_mhz", 2070.0) / 1e6  # TFLOP/s fp32 FFMA
         achieved = d["flop"] / (d["ms"] / 1e3) / 1e12
@@ -449,6 +504,31 @@ def run_extra_config(args):
                 rows.append({"kernel": "adapt/convert", "from": "%s.%s" % a_, "to": "%s.%s" % b_, "shape": list(shp),
                              "us": ms * 1e3, "gbs": by / ms / 1e6, "frac": by / ms / 1e6 / hbm})
         out.update({"metric": "achieved HBM GB/s (algorithmic bytes / event time)", "peak_gbs": hbm, "rows": rows})
+    elif args.config == "layer":
+        # one bf16 NHWC conv layer on the tensor-core routine: every routine-parameter
+        # combination (or the one given), timed back to back
+        N, C, H, K, k, s_ = map(int, args.layer.split(","))
+        sch = ("bf16", "nhwc")
+        x, layers = synth.single_conv(N, H, C, K, k, s_)
+        g = _single_layer_graph(sn, layers[0], x.shape, sch)
+        t = g.cost_table()
+        xd = torch.from_numpy(x).to(torch.bfloat16).cuda().permute(0, 2, 3, 1).contiguous()
+        y = g.new_output()
+        P = (H + 2 * (k // 2) - k) // s_ + 1
+        fl = 2 * N * K * P * P * C * k * k
+        by = 2 * (N * C * H * H + N * K * P * P + K * C * k * k)
+        sustained = pk.get("bf16_tflops_sustained", pk["bf16_tflops"])
+        rows = []
+        nvar = sum(1 for c in range(len(t["cost"])) if t["layer"][c] == 1 and
+                   sn.routine_name(int(t["routine"][c])) == "conv2/igemm_tc")
+        for var in ([args.variant] if args.variant >= 0 else range(nvar)):
+            _forced(sn, g, "conv2/igemm_tc", var)
+            ms = _time_back_to_back(torch, lambda: g.run(xd, y), reps=max(3, min(args.steps, 20)))
+            rows.append({"variant": var, "us": ms * 1e3, "tflops": fl / ms / 1e9, "gbs": by / ms / 1e6,
+                         "frac_tensor": fl / ms / 1e9 / sustained, "frac_hbm": by / ms / 1e6 / hbm})
+        best = min(rows, key=lambda r: r["us"])
+        out.update({"metric": "single-layer conv2/igemm_tc, bf16 NHWC, back-to-back event time",
+                    "layer": [N, C, H, K, k, s_], "gflop": fl / 1e9, "bytes": by, "best": best, "rows": rows})
     elif args.config == "sweep":
         rows = []
         for N in (1, 8, 32):
@@ -503,6 +583,7 @@ def run_extra_config(args):
                 g.run(xd, y)
         stream.synchronize()
         lat = []
+        torch.cuda.nvtx.range_push("sn_timed")
         for _ in range(20):
             a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             with torch.cuda.stream(stream):
@@ -512,6 +593,7 @@ def run_extra_config(args):
                 b.record(stream)
             stream.synchronize()
             lat.append(a.elapsed_time(b))
+        torch.cuda.nvtx.range_pop()
         t = g.cost_table()
         path = {}
         for i in range(1, t["n_layers"] - 1):

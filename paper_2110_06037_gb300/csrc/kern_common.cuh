@@ -48,6 +48,31 @@ inline unsigned grid_for(int64_t n, int block, int64_t cap = 152LL * 64) {
 }
 
 // dispatch a runtime dtype to a C++ type
+// Programmatic dependent launch.  Every kernel of the library is launched
+// with launch_pdl, which lets it start (set up, fetch descriptors) while the
+// previous kernel on the stream drains; the kernel calls griddep_wait()
+// before its first global-memory access, which returns once the previous
+// grid has completed and its writes are visible, and griddep_launch() to let
+// its own successor start early.  Both are no-ops for a plain launch.
+__device__ __forceinline__ void griddep_launch() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                              Args... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, args...);
+}
+
 #define SN_DT_SWITCH(dt, T, ...)                          \
     switch (dt) {                                         \
     case SN_F32: { using T = float; __VA_ARGS__; break; } \

@@ -23,6 +23,8 @@ int *device_error_word() {
 // same layout: elementwise cast (or copy)
 template <typename Ti, typename To>
 __global__ void cast_kernel(const Ti *__restrict__ x, To *__restrict__ y, int64_t n) {
+    griddep_launch();
+    griddep_wait();
     for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
          i += (int64_t)gridDim.x * blockDim.x)
         stf<To>(y + i, ldf<Ti>(x + i));
@@ -30,6 +32,8 @@ __global__ void cast_kernel(const Ti *__restrict__ x, To *__restrict__ y, int64_
 
 // 16-byte vectorised copy when dtypes match
 __global__ void copy16_kernel(const uint4 *__restrict__ x, uint4 *__restrict__ y, int64_t n16) {
+    griddep_launch();
+    griddep_wait();
     for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n16;
          i += (int64_t)gridDim.x * blockDim.x)
         y[i] = x[i];
@@ -42,6 +46,8 @@ constexpr int TT = 64;
 template <typename Ti, typename To>
 __global__ void __launch_bounds__(256) transpose_kernel(const Ti *__restrict__ x, To *__restrict__ y,
                                                          int64_t R, int64_t Cc) {
+    griddep_launch();
+    griddep_wait();
     __shared__ float tile[TT][TT + 1];
     const int64_t b = blockIdx.z;
     const int64_t r0 = (int64_t)blockIdx.y * TT, c0 = (int64_t)blockIdx.x * TT;
@@ -66,6 +72,8 @@ __global__ void __launch_bounds__(256) transpose_kernel(const Ti *__restrict__ x
 template <typename Ti, typename To>
 __global__ void __launch_bounds__(256) transpose_vec_kernel(const Ti *__restrict__ x, To *__restrict__ y,
                                                              int64_t R, int64_t Cc) {
+    griddep_launch();
+    griddep_wait();
     constexpr int EI = 16 / sizeof(Ti), EO = 16 / sizeof(To);
     __shared__ float tile[TT][TT + 1];
     const int64_t b = blockIdx.z;
@@ -105,6 +113,8 @@ __global__ void __launch_bounds__(256) transpose_vec_kernel(const Ti *__restrict
 // side as C consecutive elements per thread (C * 32 contiguous per warp)
 template <typename Ti, typename To, bool TO_NHWC>
 __global__ void permute_small_c_kernel(const Ti *__restrict__ x, To *__restrict__ y, int64_t N, int C, int64_t HW) {
+    griddep_launch();
+    griddep_wait();
     for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < N * HW;
          i += (int64_t)gridDim.x * blockDim.x) {
         const int64_t n = i / HW, hw = i % HW;
@@ -125,22 +135,22 @@ static cudaError_t convert_t(const void *x, int lay_in, void *y, int lay_out, Sh
         if (std::is_same<Ti, To>::value) {
             const int64_t bytes = n * (int64_t)sizeof(Ti);
             if (bytes % 16 == 0 && ((uintptr_t)x % 16) == 0 && ((uintptr_t)y % 16) == 0) {
-                copy16_kernel<<<grid_for(bytes / 16, 256), 256, 0, st>>>((const uint4 *)x, (uint4 *)y,
+                launch_pdl(copy16_kernel, grid_for(bytes / 16, 256), 256, 0, st, (const uint4 *)x, (uint4 *)y,
                                                                           bytes / 16);
                 return cudaGetLastError();
             }
             return cudaMemcpyAsync(y, x, bytes, cudaMemcpyDeviceToDevice, st);
         }
-        cast_kernel<Ti, To><<<grid_for(n, 256), 256, 0, st>>>((const Ti *)x, (To *)y, n);
+        launch_pdl(cast_kernel<Ti, To>, grid_for(n, 256), 256, 0, st, (const Ti *)x, (To *)y, n);
         return cudaGetLastError();
     }
     if (s.c <= 16) {
         const int64_t px = s.n * s.h * s.w;
         if (lay_in == SN_NCHW)
-            permute_small_c_kernel<Ti, To, true><<<grid_for(px, 256), 256, 0, st>>>((const Ti *)x, (To *)y, s.n,
+            launch_pdl(permute_small_c_kernel<Ti, To, true>, grid_for(px, 256), 256, 0, st, (const Ti *)x, (To *)y, s.n,
                                                                                      (int)s.c, s.h * s.w);
         else
-            permute_small_c_kernel<Ti, To, false><<<grid_for(px, 256), 256, 0, st>>>((const Ti *)x, (To *)y, s.n,
+            launch_pdl(permute_small_c_kernel<Ti, To, false>, grid_for(px, 256), 256, 0, st, (const Ti *)x, (To *)y, s.n,
                                                                                       (int)s.c, s.h * s.w);
         return cudaGetLastError();
     }
@@ -152,9 +162,9 @@ static cudaError_t convert_t(const void *x, int lay_in, void *y, int lay_out, Sh
     if (grid.y > 65535) return cudaErrorInvalidValue;
     constexpr int EI = 16 / sizeof(Ti), EO = 16 / sizeof(To);
     if (Cc % EI == 0 && R % EO == 0 && (uintptr_t)x % 16 == 0 && (uintptr_t)y % 16 == 0)
-        transpose_vec_kernel<Ti, To><<<grid, 256, 0, st>>>((const Ti *)x, (To *)y, R, Cc);
+        launch_pdl(transpose_vec_kernel<Ti, To>, grid, 256, 0, st, (const Ti *)x, (To *)y, R, Cc);
     else
-        transpose_kernel<Ti, To><<<grid, 256, 0, st>>>((const Ti *)x, (To *)y, R, Cc);
+        launch_pdl(transpose_kernel<Ti, To>, grid, 256, 0, st, (const Ti *)x, (To *)y, R, Cc);
     return cudaGetLastError();
 }
 
@@ -167,6 +177,8 @@ cudaError_t convert(const void *x, int dt_in, int lay_in, void *y, int dt_out, i
 // deterministic pseudo-random fill in [-scale, scale)
 template <typename T>
 __global__ void fill_kernel(T *y, int64_t n, uint32_t seed, float scale) {
+    griddep_launch();
+    griddep_wait();
     for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
          i += (int64_t)gridDim.x * blockDim.x) {
         uint32_t h = (uint32_t)i * 2654435761u ^ seed;
@@ -182,7 +194,7 @@ __global__ void fill_kernel(T *y, int64_t n, uint32_t seed, float scale) {
 
 cudaError_t fill_pattern(void *y, int dt, int64_t n, uint32_t seed, float scale, cudaStream_t st) {
     if (n == 0) return cudaSuccess;
-    SN_DT_SWITCH(dt, T, fill_kernel<T><<<grid_for(n, 256), 256, 0, st>>>((T *)y, n, seed, scale));
+    SN_DT_SWITCH(dt, T, launch_pdl(fill_kernel<T>, grid_for(n, 256), 256, 0, st, (T *)y, n, seed, scale));
     return cudaGetLastError();
 }
 
@@ -192,6 +204,8 @@ cudaError_t fill_pattern(void *y, int dt, int64_t n, uint32_t seed, float scale,
 template <typename T>
 __global__ void weight_perm_kernel(const float *__restrict__ w, T *__restrict__ out, int fmt,
                                    int64_t K, int64_t Cg, int64_t R, int64_t S) {
+    griddep_launch();
+    griddep_wait();
     const int64_t total = K * Cg * R * S;
     for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total;
          i += (int64_t)gridDim.x * blockDim.x) {
@@ -211,6 +225,8 @@ __global__ void weight_perm_kernel(const float *__restrict__ w, T *__restrict__ 
 template <typename T>
 __global__ void weight_wino_kernel(const float *__restrict__ w, T *__restrict__ out, int64_t K,
                                    int64_t C) {
+    griddep_launch();
+    griddep_wait();
     for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < K * C;
          i += (int64_t)gridDim.x * blockDim.x) {
         const float *g = w + i * 9;  // [3][3] for (k, c) = (i / C, i % C)
@@ -234,7 +250,7 @@ cudaError_t weight_format(const float *w, void *out, int fmt, int dt, int64_t K,
                           int64_t R, int64_t S, cudaStream_t st) {
     if (fmt == W_WINO) {
         if (R != 3 || S != 3) return cudaErrorInvalidValue;
-        SN_DT_SWITCH(dt, T, weight_wino_kernel<T><<<grid_for(K * Cg, 256), 256, 0, st>>>(w, (T *)out, K, Cg));
+        SN_DT_SWITCH(dt, T, launch_pdl(weight_wino_kernel<T>, grid_for(K * Cg, 256), 256, 0, st, w, (T *)out, K, Cg));
         return cudaGetLastError();
     }
     if (fmt == W_KRSC_PAD64) {  // rows padded with zeros to a multiple of 64 taps
@@ -243,7 +259,7 @@ cudaError_t weight_format(const float *w, void *out, int fmt, int dt, int64_t K,
         if (e != cudaSuccess) return e;
     }
     SN_DT_SWITCH(dt, T,
-                 weight_perm_kernel<T><<<grid_for(K * Cg * R * S, 256), 256, 0, st>>>(w, (T *)out, fmt, K, Cg, R, S));
+                 launch_pdl(weight_perm_kernel<T>, grid_for(K * Cg * R * S, 256), 256, 0, st, w, (T *)out, fmt, K, Cg, R, S));
     return cudaGetLastError();
 }
 
@@ -253,6 +269,8 @@ cudaError_t weight_format(const float *w, void *out, int fmt, int dt, int64_t K,
 template <typename T>
 __global__ void conv_direct_nchw(const T *__restrict__ x, const T *__restrict__ w,
                                  const float *__restrict__ bias, T *__restrict__ y, ConvDims d) {
+    griddep_launch();
+    griddep_wait();
     const int64_t total = (int64_t)d.N * d.K * d.P * d.Q;
     const int Cg = d.C / d.groups, Kg = d.K / d.groups;
     for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total;
@@ -282,6 +300,8 @@ __global__ void conv_direct_nchw(const T *__restrict__ x, const T *__restrict__ 
 template <typename T>
 __global__ void conv_direct_nhwc(const T *__restrict__ x, const T *__restrict__ w,
                                  const float *__restrict__ bias, T *__restrict__ y, ConvDims d) {
+    griddep_launch();
+    griddep_wait();
     const int64_t total = (int64_t)d.N * d.K * d.P * d.Q;
     const int Cg = d.C / d.groups, Kg = d.K / d.groups;
     for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total;
@@ -312,10 +332,10 @@ cudaError_t conv_direct(const LaunchArgs &a) {
     const int64_t total = (int64_t)d.N * d.K * d.P * d.Q;
     SN_DT_SWITCH(a.schema.dtype, T, {
         if (a.schema.layout == SN_NCHW)
-            conv_direct_nchw<T><<<grid_for(total, 256), 256, 0, a.stream>>>(
+            launch_pdl(conv_direct_nchw<T>, grid_for(total, 256), 256, 0, a.stream, 
                 (const T *)a.in[0], (const T *)a.wt, a.bias, (T *)a.out, d);
         else
-            conv_direct_nhwc<T><<<grid_for(total, 256), 256, 0, a.stream>>>(
+            launch_pdl(conv_direct_nhwc<T>, grid_for(total, 256), 256, 0, a.stream, 
                 (const T *)a.in[0], (const T *)a.wt, a.bias, (T *)a.out, d);
     });
     return cudaGetLastError();
@@ -327,6 +347,8 @@ cudaError_t conv_direct(const LaunchArgs &a) {
 template <typename T>
 __global__ void dw_nhwc(const T *__restrict__ x, const T *__restrict__ w, const float *__restrict__ bias,
                         T *__restrict__ y, ConvDims d) {
+    griddep_launch();
+    griddep_wait();
     const int64_t total = (int64_t)d.N * d.K * d.P * d.Q;
     for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total;
          i += (int64_t)gridDim.x * blockDim.x) {
@@ -356,6 +378,8 @@ __global__ void dw_nhwc(const T *__restrict__ x, const T *__restrict__ w, const 
 template <typename T, int QB, int SW>  // SW = 1 or 2: 3x3 fast path for that stride; 0 = any
 __global__ void __launch_bounds__(256, QB >= 4 ? 2 : 3) dw_nhwc_vec(const T *__restrict__ x, const T *__restrict__ w,
                                                    const float *__restrict__ bias, T *__restrict__ y, ConvDims d) {
+    griddep_launch();
+    griddep_wait();
     constexpr int E = 16 / sizeof(T);
     const int CV = d.C / E;
     const int QBLK = (d.Q + QB - 1) / QB;
@@ -454,6 +478,8 @@ __global__ void __launch_bounds__(256, QB >= 4 ? 2 : 3) dw_nhwc_vec(const T *__r
 template <typename T>
 __global__ void __launch_bounds__(256) dw_nchw_row(const T *__restrict__ x, const T *__restrict__ w,
                                                    const float *__restrict__ bias, T *__restrict__ y, ConvDims d) {
+    griddep_launch();
+    griddep_wait();
     constexpr int QB = 8;
     const int QBLK = (d.Q + QB - 1) / QB;
     const int64_t total = (int64_t)d.N * d.C * d.P * QBLK;
@@ -523,6 +549,8 @@ __device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_gr
 template <typename T, int SW, int STAGES>
 __global__ void __launch_bounds__(256, 2) dw3_nhwc_halo(const T *__restrict__ x, const T *__restrict__ w,
                                                         const float *__restrict__ bias, T *__restrict__ y, ConvDims d) {
+    griddep_launch();
+    griddep_wait();
     constexpr int DW_TQ = DwTQ<SW>::v;
     constexpr int E = 16 / sizeof(T);          // elements per 16-byte vector
     constexpr int VS = 8;                      // vectors per 128-byte channel slice
@@ -620,6 +648,8 @@ template <typename T>
 __global__ void __launch_bounds__(256) dw3_nchw_tile(const T *__restrict__ x, const T *__restrict__ w,
                                                      const float *__restrict__ bias, T *__restrict__ y, ConvDims d,
                                                      int TH) {
+    griddep_launch();
+    griddep_wait();
     extern __shared__ float dw_tile[];
     const int tiles = (d.P + TH - 1) / TH;
     const int64_t nc = blockIdx.x / tiles;
@@ -683,16 +713,16 @@ cudaError_t dwconv(const LaunchArgs &a) {
                     cudaFuncSetAttribute(dw3_nhwc_halo<T, 2, 3>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm2);
                     attr = true;
                 }
-                if (d.sw == 1) dw3_nhwc_halo<T, 1, 4><<<gb, 256, sm1, a.stream>>>(x, w, a.bias, y, d);
-                else dw3_nhwc_halo<T, 2, 3><<<gb, 256, sm2, a.stream>>>(x, w, a.bias, y, d);
+                if (d.sw == 1) launch_pdl(dw3_nhwc_halo<T, 1, 4>, gb, 256, sm1, a.stream, x, w, a.bias, y, d);
+                else launch_pdl(dw3_nhwc_halo<T, 2, 3>, gb, 256, sm2, a.stream, x, w, a.bias, y, d);
             } else {
                 const unsigned gb = grid_for((int64_t)d.N * d.P * ((d.Q + 3) / 4) * cvec, 256, 152LL * 16);
-                if (k3 && d.sw == 1) dw_nhwc_vec<T, 4, 1><<<gb, 256, 0, a.stream>>>(x, w, a.bias, y, d);
-                else if (k3 && d.sw == 2) dw_nhwc_vec<T, 4, 2><<<gb, 256, 0, a.stream>>>(x, w, a.bias, y, d);
-                else dw_nhwc_vec<T, 4, 0><<<gb, 256, 0, a.stream>>>(x, w, a.bias, y, d);
+                if (k3 && d.sw == 1) launch_pdl(dw_nhwc_vec<T, 4, 1>, gb, 256, 0, a.stream, x, w, a.bias, y, d);
+                else if (k3 && d.sw == 2) launch_pdl(dw_nhwc_vec<T, 4, 2>, gb, 256, 0, a.stream, x, w, a.bias, y, d);
+                else launch_pdl(dw_nhwc_vec<T, 4, 0>, gb, 256, 0, a.stream, x, w, a.bias, y, d);
             }
         } else if (a.schema.layout == SN_NHWC) {
-            dw_nhwc<T><<<grid_for(total, 256), 256, 0, a.stream>>>(x, w, a.bias, y, d);
+            launch_pdl(dw_nhwc<T>, grid_for(total, 256), 256, 0, a.stream, x, w, a.bias, y, d);
         } else {
             bool tiled = false;
             if (a.variant == 1 && d.R == 3 && d.S == 3) {
@@ -703,13 +733,12 @@ cudaError_t dwconv(const LaunchArgs &a) {
                 while (tile_bytes(TH) > 40 * 1024 && TH > 1) TH /= 2;
                 const int64_t blocks = (int64_t)d.N * d.C * ((d.P + TH - 1) / TH);
                 if (tile_bytes(TH) <= 40 * 1024 && blocks < ((int64_t)1 << 31)) {
-                    dw3_nchw_tile<T><<<(unsigned)blocks, 256, tile_bytes(TH), a.stream>>>(x, w, a.bias, y, d, TH);
+                    launch_pdl(dw3_nchw_tile<T>, (unsigned)blocks, 256, tile_bytes(TH), a.stream, x, w, a.bias, y, d, TH);
                     tiled = true;
                 }
             }
             if (!tiled)
-                dw_nchw_row<T><<<grid_for((int64_t)d.N * d.C * d.P * ((d.Q + 7) / 8), 256, 152LL * 16), 256, 0,
-                                 a.stream>>>(x, w, a.bias, y, d);
+                launch_pdl(dw_nchw_row<T>, grid_for((int64_t)d.N * d.C * d.P * ((d.Q + 7) / 8), 256, 152LL * 16), 256, 0, a.stream, x, w, a.bias, y, d);
         }
     });
     return cudaGetLastError();
@@ -721,6 +750,8 @@ cudaError_t dwconv(const LaunchArgs &a) {
 template <typename T, bool NHWC>
 __global__ void maxpool_kernel(const T *__restrict__ x, T *__restrict__ y, int N, int C, int H, int W,
                                int P, int Q, int kh, int kw, int sh, int sw, int ph, int pw) {
+    griddep_launch();
+    griddep_wait();
     const int64_t total = (int64_t)N * C * P * Q;
     for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total;
          i += (int64_t)gridDim.x * blockDim.x) {
@@ -757,6 +788,8 @@ __global__ void maxpool_kernel(const T *__restrict__ x, T *__restrict__ y, int N
 template <typename T>
 __global__ void maxpool_nhwc_vec(const uint4 *__restrict__ x, uint4 *__restrict__ y, int N, int C16, int H, int W,
                                  int P, int Q, int kh, int kw, int sh, int sw, int ph, int pw) {
+    griddep_launch();
+    griddep_wait();
     constexpr int E = 16 / sizeof(T);
     const int64_t total = (int64_t)N * P * Q * C16;
     for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total;
@@ -797,15 +830,15 @@ cudaError_t maxpool(const LaunchArgs &a) {
         if (a.schema.layout == SN_NHWC && cb % 16 == 0 && (uintptr_t)a.in[0] % 16 == 0 &&
             (uintptr_t)a.out % 16 == 0) {
             const int c16 = (int)(cb / 16);
-            maxpool_nhwc_vec<T><<<grid_for(o.n * o.h * o.w * c16, 256), 256, 0, a.stream>>>(
+            launch_pdl(maxpool_nhwc_vec<T>, grid_for(o.n * o.h * o.w * c16, 256), 256, 0, a.stream, 
                 (const uint4 *)a.in[0], (uint4 *)a.out, (int)i.n, c16, (int)i.h, (int)i.w, (int)o.h, (int)o.w,
                 p.kh, p.kw, p.sh, p.sw, p.ph, p.pw);
         } else if (a.schema.layout == SN_NHWC)
-            maxpool_kernel<T, true><<<grid_for(total, 256), 256, 0, a.stream>>>(
+            launch_pdl(maxpool_kernel<T, true>, grid_for(total, 256), 256, 0, a.stream, 
                 (const T *)a.in[0], (T *)a.out, (int)i.n, (int)i.c, (int)i.h, (int)i.w, (int)o.h, (int)o.w,
                 p.kh, p.kw, p.sh, p.sw, p.ph, p.pw);
         else
-            maxpool_kernel<T, false><<<grid_for(total, 256), 256, 0, a.stream>>>(
+            launch_pdl(maxpool_kernel<T, false>, grid_for(total, 256), 256, 0, a.stream, 
                 (const T *)a.in[0], (T *)a.out, (int)i.n, (int)i.c, (int)i.h, (int)i.w, (int)o.h, (int)o.w,
                 p.kh, p.kw, p.sh, p.sw, p.ph, p.pw);
     });
@@ -815,6 +848,8 @@ cudaError_t maxpool(const LaunchArgs &a) {
 // NCHW: one warp per (n, c) sums HW contiguous values
 template <typename T>
 __global__ void gap_nchw(const T *__restrict__ x, T *__restrict__ y, int64_t NC, int64_t HW) {
+    griddep_launch();
+    griddep_wait();
     const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) / 32;
     const int lane = threadIdx.x % 32;
     for (int64_t nc = warp; nc < NC; nc += (int64_t)gridDim.x * blockDim.x / 32) {
@@ -828,6 +863,8 @@ __global__ void gap_nchw(const T *__restrict__ x, T *__restrict__ y, int64_t NC,
 // NHWC: one thread per (n, c); consecutive threads read consecutive channels
 template <typename T>
 __global__ void gap_nhwc(const T *__restrict__ x, T *__restrict__ y, int64_t N, int64_t C, int64_t HW) {
+    griddep_launch();
+    griddep_wait();
     for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < N * C;
          i += (int64_t)gridDim.x * blockDim.x) {
         const int64_t n = i / C, c = i % C;
@@ -841,10 +878,10 @@ cudaError_t gap(const LaunchArgs &a) {
     const Shape &i = a.in_shapes[0];
     SN_DT_SWITCH(a.schema.dtype, T, {
         if (a.schema.layout == SN_NCHW)
-            gap_nchw<T><<<grid_for(i.n * i.c * 32, 256), 256, 0, a.stream>>>((const T *)a.in[0], (T *)a.out,
+            launch_pdl(gap_nchw<T>, grid_for(i.n * i.c * 32, 256), 256, 0, a.stream, (const T *)a.in[0], (T *)a.out,
                                                                                i.n * i.c, i.h * i.w);
         else
-            gap_nhwc<T><<<grid_for(i.n * i.c, 256), 256, 0, a.stream>>>((const T *)a.in[0], (T *)a.out, i.n,
+            launch_pdl(gap_nhwc<T>, grid_for(i.n * i.c, 256), 256, 0, a.stream, (const T *)a.in[0], (T *)a.out, i.n,
                                                                          i.c, i.h * i.w);
     });
     return cudaGetLastError();
@@ -853,6 +890,8 @@ cudaError_t gap(const LaunchArgs &a) {
 template <typename T>
 __global__ void add_kernel(const T *__restrict__ a, const T *__restrict__ b, T *__restrict__ y, int64_t n,
                            int act) {
+    griddep_launch();
+    griddep_wait();
     for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
          i += (int64_t)gridDim.x * blockDim.x)
         stf<T>(y + i, act_apply(ldf<T>(a + i) + ldf<T>(b + i), act));
@@ -862,6 +901,8 @@ __global__ void add_kernel(const T *__restrict__ a, const T *__restrict__ b, T *
 template <typename T>
 __global__ void add16_kernel(const uint4 *__restrict__ a, const uint4 *__restrict__ b, uint4 *__restrict__ y,
                              int64_t n16, int act) {
+    griddep_launch();
+    griddep_wait();
     constexpr int E = 16 / sizeof(T);
     for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n16;
          i += (int64_t)gridDim.x * blockDim.x) {
@@ -881,10 +922,10 @@ cudaError_t add(const LaunchArgs &a) {
         const int64_t bytes = n * (int64_t)sizeof(T);
         if (bytes % 16 == 0 && (uintptr_t)a.in[0] % 16 == 0 && (uintptr_t)a.in[1] % 16 == 0 &&
             (uintptr_t)a.out % 16 == 0)
-            add16_kernel<T><<<grid_for(bytes / 16, 256), 256, 0, a.stream>>>(
+            launch_pdl(add16_kernel<T>, grid_for(bytes / 16, 256), 256, 0, a.stream, 
                 (const uint4 *)a.in[0], (const uint4 *)a.in[1], (uint4 *)a.out, bytes / 16, a.layer->act);
         else
-            add_kernel<T><<<grid_for(n, 256), 256, 0, a.stream>>>((const T *)a.in[0], (const T *)a.in[1],
+            launch_pdl(add_kernel<T>, grid_for(n, 256), 256, 0, a.stream, (const T *)a.in[0], (const T *)a.in[1],
                                                                    (T *)a.out, n, a.layer->act);
     });
     return cudaGetLastError();
@@ -894,6 +935,8 @@ cudaError_t add(const LaunchArgs &a) {
 template <typename T>
 __global__ void dense_kernel(const T *__restrict__ x, const T *__restrict__ w, const float *__restrict__ bias,
                              T *__restrict__ y, int64_t N, int64_t IN, int64_t OUT, int act) {
+    griddep_launch();
+    griddep_wait();
     const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) / 32;
     const int lane = threadIdx.x % 32;
     for (int64_t no = warp; no < N * OUT; no += (int64_t)gridDim.x * blockDim.x / 32) {
@@ -909,7 +952,7 @@ cudaError_t dense(const LaunchArgs &a) {
     const Shape &i = a.in_shapes[0];
     const int64_t N = i.n, IN = a.layer->dense_in, OUT = a.layer->dense_out;
     SN_DT_SWITCH(a.schema.dtype, T,
-                 dense_kernel<T><<<grid_for(N * OUT * 32, 256), 256, 0, a.stream>>>(
+                 launch_pdl(dense_kernel<T>, grid_for(N * OUT * 32, 256), 256, 0, a.stream, 
                      (const T *)a.in[0], (const T *)a.wt, a.bias, (T *)a.out, N, IN, OUT, a.layer->act));
     return cudaGetLastError();
 }

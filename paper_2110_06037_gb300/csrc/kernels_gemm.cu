@@ -19,6 +19,8 @@ template <typename T, bool NHWC, int BM>
 __global__ void __launch_bounds__(256) igemm_simt_kernel(const T *__restrict__ x, const T *__restrict__ w,
                                                          const float *__restrict__ bias, T *__restrict__ y,
                                                          ConvDims d) {
+    griddep_launch();
+    griddep_wait();
     constexpr int BN = 64, BK = 16, TM = BM / 16, TN = 4;
     constexpr int A_PER = BK * BM / 256, B_PER = BK * BN / 256;
     __shared__ float As[BK][BM + 4];
@@ -164,11 +166,11 @@ cudaError_t conv_igemm(const LaunchArgs &a) {
         const T *w = (const T *)a.wt;
         T *y = (T *)a.out;
         if (a.schema.layout == SN_NHWC) {
-            if (BM == 64) igemm_simt_kernel<T, true, 64><<<grid, 256, 0, a.stream>>>(x, w, a.bias, y, d);
-            else igemm_simt_kernel<T, true, 128><<<grid, 256, 0, a.stream>>>(x, w, a.bias, y, d);
+            if (BM == 64) launch_pdl(igemm_simt_kernel<T, true, 64>, grid, 256, 0, a.stream, x, w, a.bias, y, d);
+            else launch_pdl(igemm_simt_kernel<T, true, 128>, grid, 256, 0, a.stream, x, w, a.bias, y, d);
         } else {
-            if (BM == 64) igemm_simt_kernel<T, false, 64><<<grid, 256, 0, a.stream>>>(x, w, a.bias, y, d);
-            else igemm_simt_kernel<T, false, 128><<<grid, 256, 0, a.stream>>>(x, w, a.bias, y, d);
+            if (BM == 64) launch_pdl(igemm_simt_kernel<T, false, 64>, grid, 256, 0, a.stream, x, w, a.bias, y, d);
+            else launch_pdl(igemm_simt_kernel<T, false, 128>, grid, 256, 0, a.stream, x, w, a.bias, y, d);
         }
     });
     return cudaGetLastError();
@@ -201,6 +203,8 @@ size_t conv_wino_ws(const Layer &l, const Shape &in, sn_schema s) {
 // wgenc: V[xi][t][c] = (B^T d B)[xi] for the 4x4 input tile of output tile t
 template <typename T, bool NHWC>
 __global__ void wino_input_kernel(const T *__restrict__ x, float *__restrict__ V, WinoDims wd) {
+    griddep_launch();
+    griddep_wait();
     const ConvDims &d = wd.d;
     const int64_t total = wd.T * d.C;
     for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total;
@@ -246,6 +250,8 @@ __global__ void wino_input_kernel(const T *__restrict__ x, float *__restrict__ V
 template <typename TB>
 __global__ void __launch_bounds__(256) gemm_nt_simt(const float *__restrict__ A, const TB *__restrict__ B,
                                                     float *__restrict__ Cm, int64_t M, int N, int Kd) {
+    griddep_launch();
+    griddep_wait();
     constexpr int BM = 64, BN = 64, BK = 16, TM = 4, TN = 4;
     __shared__ float As[BK][BM + 4];
     __shared__ float Bs[BK][BN + 4];
@@ -297,6 +303,8 @@ __global__ void __launch_bounds__(256) gemm_nt_simt(const float *__restrict__ A,
 template <typename T, bool NHWC>
 __global__ void wino_output_kernel(const float *__restrict__ Mx, const float *__restrict__ bias,
                                    T *__restrict__ y, WinoDims wd) {
+    griddep_launch();
+    griddep_wait();
     const ConvDims &d = wd.d;
     const int64_t total = wd.T * d.K;
     for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total;
@@ -345,14 +353,14 @@ cudaError_t conv_wino(const LaunchArgs &a) {
     if (ggrid.y > 65535) return cudaErrorInvalidValue;
     SN_DT_SWITCH(a.schema.dtype, T, {
         if (a.schema.layout == SN_NHWC)
-            wino_input_kernel<T, true><<<grid_for(wd.T * d.C, 256), 256, 0, a.stream>>>((const T *)a.in[0], V, wd);
+            launch_pdl(wino_input_kernel<T, true>, grid_for(wd.T * d.C, 256), 256, 0, a.stream, (const T *)a.in[0], V, wd);
         else
-            wino_input_kernel<T, false><<<grid_for(wd.T * d.C, 256), 256, 0, a.stream>>>((const T *)a.in[0], V, wd);
-        gemm_nt_simt<T><<<ggrid, 256, 0, a.stream>>>(V, (const T *)a.wt, Mx, wd.T, d.K, d.C);
+            launch_pdl(wino_input_kernel<T, false>, grid_for(wd.T * d.C, 256), 256, 0, a.stream, (const T *)a.in[0], V, wd);
+        launch_pdl(gemm_nt_simt<T>, ggrid, 256, 0, a.stream, V, (const T *)a.wt, Mx, wd.T, d.K, d.C);
         if (a.schema.layout == SN_NHWC)
-            wino_output_kernel<T, true><<<grid_for(wd.T * d.K, 256), 256, 0, a.stream>>>(Mx, a.bias, (T *)a.out, wd);
+            launch_pdl(wino_output_kernel<T, true>, grid_for(wd.T * d.K, 256), 256, 0, a.stream, Mx, a.bias, (T *)a.out, wd);
         else
-            wino_output_kernel<T, false><<<grid_for(wd.T * d.K, 256), 256, 0, a.stream>>>(Mx, a.bias, (T *)a.out, wd);
+            launch_pdl(wino_output_kernel<T, false>, grid_for(wd.T * d.K, 256), 256, 0, a.stream, Mx, a.bias, (T *)a.out, wd);
     });
     return cudaGetLastError();
 }
@@ -366,14 +374,14 @@ cudaError_t conv_wino_buffers(const ConvDims &d, sn_schema s, const void *x, con
     if (ggrid.y > 65535) return cudaErrorInvalidValue;
     SN_DT_SWITCH(s.dtype, T, {
         if (s.layout == SN_NHWC)
-            wino_input_kernel<T, true><<<grid_for(wd.T * d.C, 256), 256, 0, st>>>((const T *)x, V, wd);
+            launch_pdl(wino_input_kernel<T, true>, grid_for(wd.T * d.C, 256), 256, 0, st, (const T *)x, V, wd);
         else
-            wino_input_kernel<T, false><<<grid_for(wd.T * d.C, 256), 256, 0, st>>>((const T *)x, V, wd);
-        gemm_nt_simt<T><<<ggrid, 256, 0, st>>>(V, (const T *)u, Mx, wd.T, d.K, d.C);
+            launch_pdl(wino_input_kernel<T, false>, grid_for(wd.T * d.C, 256), 256, 0, st, (const T *)x, V, wd);
+        launch_pdl(gemm_nt_simt<T>, ggrid, 256, 0, st, V, (const T *)u, Mx, wd.T, d.K, d.C);
         if (s.layout == SN_NHWC)
-            wino_output_kernel<T, true><<<grid_for(wd.T * d.K, 256), 256, 0, st>>>(Mx, bias, (T *)y, wd);
+            launch_pdl(wino_output_kernel<T, true>, grid_for(wd.T * d.K, 256), 256, 0, st, Mx, bias, (T *)y, wd);
         else
-            wino_output_kernel<T, false><<<grid_for(wd.T * d.K, 256), 256, 0, st>>>(Mx, bias, (T *)y, wd);
+            launch_pdl(wino_output_kernel<T, false>, grid_for(wd.T * d.K, 256), 256, 0, st, Mx, bias, (T *)y, wd);
     });
     return cudaGetLastError();
 }

@@ -76,6 +76,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     __shared__ volatile int abort_sh;
     __shared__ int issued_sh[4], consumed_sh;
 
+    griddep_launch();
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t *stg = smem + STAGES * STAGE_BYTES;  // epilogue staging: 8 warps x 2 buffers, 1024-B aligned
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
@@ -91,6 +92,9 @@ __global__ void __launch_bounds__(THREADS, 1)
     };
 
     if (threadIdx.x == 0) {
+        // the tensor maps are kernel parameters, not data of the previous kernel
+        const CUtensorMap *maps[6] = {&mA0, &mA1, &mA2, &mA3, &mB, &mY};
+        for (int i = 0; i < 6; ++i) asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(maps[i])) : "memory");
         for (int s = 0; s < STAGES; ++s) {
             mbar_init(&full_bar[s], 1);  // the (leader's) producer of the stage
             mbar_init(&empty_bar[s], 1);
@@ -110,6 +114,9 @@ __global__ void __launch_bounds__(THREADS, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = tmem_sh;
+    // everything above overlaps the previous kernel's tail; global memory is
+    // touched only from here on
+    griddep_wait();
 
     constexpr int NPROD = producers_for(STAGES);
     const int prod = warp == 0 ? 0 : (warp >= 10 ? warp - 9 : -1);  // producer index of this warp
@@ -397,6 +404,8 @@ __global__ void __launch_bounds__(THREADS, 1)
 template <typename T>
 __global__ void splitk_reduce_kernel(const float *__restrict__ part, const float *__restrict__ bias,
                                      T *__restrict__ y, int64_t M, int K, int ks, int act) {
+    griddep_launch();
+    griddep_wait();
     const int K4 = K / 4;
     for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < M * K4;
          i += (int64_t)gridDim.x * blockDim.x) {
@@ -564,25 +573,31 @@ static cudaError_t launch(const CUtensorMap *mA, const CUtensorMap &mB, const CU
     auto kern = conv_tc_kernel<T, BN, STAGES, IMPLICIT, G, KB>;
     static int max_groups = 0;  // co-resident CTAs (G = 1) or CTA pairs (G = 2)
     cudaLaunchConfig_t cfg = {};
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     cfg.blockDim = dim3(THREADS);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = st;
+    cfg.attrs = attr;
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;  // see launch_pdl
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.numAttrs = 1;
     if (G == 2) {
-        attr[0].id = cudaLaunchAttributeClusterDimension;
-        attr[0].val.clusterDim.x = 2;
-        attr[0].val.clusterDim.y = 1;
-        attr[0].val.clusterDim.z = 1;
-        cfg.attrs = attr;
-        cfg.numAttrs = 1;
+        attr[1].id = cudaLaunchAttributeClusterDimension;
+        attr[1].val.clusterDim.x = 2;
+        attr[1].val.clusterDim.y = 1;
+        attr[1].val.clusterDim.z = 1;
+        cfg.numAttrs = 2;
     }
     if (!max_groups) {
         cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
         if (G == 2) {
-            cfg.gridDim = dim3(2);
+            cudaLaunchConfig_t q = cfg;  // the cluster shape alone
+            q.gridDim = dim3(2);
+            q.attrs = attr + 1;
+            q.numAttrs = 1;
             int n = 0;
-            e = cudaOccupancyMaxActiveClusters(&n, kern, &cfg);
+            e = cudaOccupancyMaxActiveClusters(&n, kern, &q);
             if (e != cudaSuccess) return e;
             if (n <= 0) return cudaErrorInvalidConfiguration;
             max_groups = n;
@@ -595,7 +610,7 @@ static cudaError_t launch(const CUtensorMap *mA, const CUtensorMap &mB, const CU
     cudaError_t e = cudaLaunchKernelEx(&cfg, kern, mA[0], mA[1], mA[2], mA[3], mB, mY, p);
     if (e != cudaSuccess || p.ksplit == 1) return e;
     const int64_t n4 = p.Mout * (p.K / 4);
-    splitk_reduce_kernel<T><<<grid_for(n4, 256), 256, 0, st>>>(p.part, p.bias, static_cast<T *>(p.y), p.Mout, p.K,
+    launch_pdl(splitk_reduce_kernel<T>, grid_for(n4, 256), 256, 0, st, p.part, p.bias, static_cast<T *>(p.y), p.Mout, p.K,
                                                                p.ksplit, p.act);
     return cudaGetLastError();
 }
@@ -777,6 +792,8 @@ size_t conv_im2col_tc_ws(const Layer &l, const Shape &in, sn_schema s, int32_t v
 // zero outside the image and for kk >= C*R*S; 8 taps (16 bytes) per thread
 template <typename T>
 __global__ void im2col_nhwc_kernel(const T *__restrict__ x, T *__restrict__ A, ConvDims d, int kpad, int64_t M) {
+    griddep_launch();
+    griddep_wait();
     const int g8 = kpad / 8;
     const int crs = d.C * d.R * d.S;
     for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < M * g8;
@@ -808,6 +825,8 @@ __global__ void im2col_nhwc_kernel(const T *__restrict__ x, T *__restrict__ A, C
 template <typename T>
 __global__ void __launch_bounds__(256) im2col_rows_kernel(const T *__restrict__ x, T *__restrict__ A, ConvDims d,
                                                           int kpad) {
+    griddep_launch();
+    griddep_wait();
     extern __shared__ uint8_t im2col_smem[];
     // per tap kk: (offset of (r, w = -pw + s*dw, c) in the staged rows, w) --
     // the divisions by C and S happen once per block, not per element
@@ -859,11 +878,11 @@ cudaError_t conv_im2col_tc(const LaunchArgs &a) {
     const size_t rows_bytes = (size_t)kpad * sizeof(int2) + (size_t)d.R * d.W * d.C * dtype_size(a.schema.dtype);
     if (rows_bytes <= 48 * 1024 && d.N <= 65535) {
         SN_DT_SWITCH(a.schema.dtype, T,
-                     im2col_rows_kernel<T><<<dim3((unsigned)d.P, (unsigned)d.N), 256, rows_bytes, a.stream>>>(
+                     launch_pdl(im2col_rows_kernel<T>, dim3((unsigned)d.P, (unsigned)d.N), 256, rows_bytes, a.stream, 
                          (const T *)a.in[0], (T *)a.ws, d, (int)kpad));
     } else {
         SN_DT_SWITCH(a.schema.dtype, T,
-                     im2col_nhwc_kernel<T><<<grid_for(M * (kpad / 8), 256), 256, 0, a.stream>>>(
+                     launch_pdl(im2col_nhwc_kernel<T>, grid_for(M * (kpad / 8), 256), 256, 0, a.stream, 
                          (const T *)a.in[0], (T *)a.ws, d, (int)kpad, M));
     }
     cudaError_t e = cudaGetLastError();
