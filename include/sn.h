@@ -72,7 +72,8 @@ typedef struct { int32_t dtype; int32_t layout; } sn_schema;
 /* Layer types (section III-B); activations are fused layer attributes (the
  * importer's ReLU fusion, section III-A). */
 typedef enum {
-    SN_L_CONV2 = 0,   /* 2-D convolution (cross-correlation) + bias + act      */
+    SN_L_CONV2 = 0,   /* 2-D convolution (cross-correlation) + bias + act;
+                       * optionally + a residual blob before the act (fused add) */
     SN_L_DWCONV2 = 1, /* depthwise conv2: groups = c_in = c_out                */
     SN_L_MAXPOOL = 2, /* max pooling, -inf padding                             */
     SN_L_GAP = 3,     /* global average pooling -> N x C x 1 x 1               */
@@ -113,6 +114,11 @@ SN_API sn_status sn_graph_create(const int64_t in_nchw[4], sn_schema in_schema, 
  * (sn_conv_params for CONV2/DWCONV2, sn_pool_params, sn_add_params,
  * sn_dense_params; NULL for GAP).  inputs[0..n_inputs) are ids returned by
  * earlier calls, -1 = the net input (ADD takes two, the others one).
+ * CONV2 may take a second input, a residual of exactly the output's shape:
+ * y = act(conv(x) + bias + residual), the residual add of a ResNet block fused
+ * into the convolution that feeds it (the paper's graph optimiser fuses
+ * layers before tuning, section III-A); the direct and the tensor-core
+ * routines serve such a layer.
  * weights: host fp32, conv [c_out][c_in/groups][kh][kw], dense [out][in];
  * bias: host fp32 [c_out] or NULL (zeros).  Both are copied.  The last layer
  * added is the net output.  *out_layer_id receives the new layer's id.

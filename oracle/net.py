@@ -30,6 +30,12 @@ def run_layer(layer: dict, inputs: list, dtype: str = "f32") -> np.ndarray:
         w = round_to(layer["weight"], dtype)
         b = layer.get("bias")
         groups = p.get("groups", 1) if t == "conv2" else p["c_in"]
+        if len(inputs) == 2:
+            # conv2 with a residual input: the activation applies to
+            # conv + bias + residual, with no rounding in between
+            y = conv2d(inputs[0], w, b, stride=(p["sh"], p["sw"]), pad=(p["ph"], p["pw"]),
+                       dil=(p.get("dh", 1), p.get("dw", 1)), groups=groups, act="none")
+            return add(y, inputs[1], act=p.get("act", "none"))
         return conv2d(inputs[0], w, b, stride=(p["sh"], p["sw"]), pad=(p["ph"], p["pw"]),
                       dil=(p.get("dh", 1), p.get("dw", 1)), groups=groups,
                       act=p.get("act", "none"))

@@ -9,7 +9,7 @@ thin binding over it.
 from ._sn import (SN_SELECT_BRUTE, SN_SELECT_DPRS, SN_OPT_CHECK, SN_OPT_CUDA_GRAPH, SnError, lib,
                   routine_name, variant_name)
 from .api import Graph, convert, storage_shape
-from .netbuild import build_graph
+from .netbuild import build_graph, fuse_residual
 
-__all__ = ["Graph", "convert", "build_graph", "storage_shape", "SnError", "lib", "routine_name",
+__all__ = ["Graph", "convert", "build_graph", "fuse_residual", "storage_shape", "SnError", "lib", "routine_name",
            "variant_name", "SN_SELECT_DPRS", "SN_SELECT_BRUTE", "SN_OPT_CHECK", "SN_OPT_CUDA_GRAPH"]

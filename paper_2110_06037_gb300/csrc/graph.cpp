@@ -87,7 +87,10 @@ static sn_status infer_shape(Layer &L, const std::vector<Shape> &in) {
     case SN_L_CONV2:
     case SN_L_DWCONV2: {
         const sn_conv_params &p = L.conv;
-        if (in.size() != 1) return fail(SN_EINVAL, "conv2 takes one input");
+        // conv2 may take a second input: a residual of the output's shape,
+        // added after the bias and before the activation (a fused add)
+        if (in.size() != 1 && !(L.type == SN_L_CONV2 && in.size() == 2))
+            return fail(SN_EINVAL, "conv2 takes one input (or two: input, residual); dwconv2 takes one");
         if (p.kh < 1 || p.kw < 1 || p.sh < 1 || p.sw < 1 || p.ph < 0 || p.pw < 0 || p.dh < 1 ||
             p.dw < 1 || p.groups < 1 || p.c_in < 1 || p.c_out < 1)
             return fail(SN_EINVAL, "conv2: invalid parameter");
@@ -102,6 +105,8 @@ static sn_status infer_shape(Layer &L, const std::vector<Shape> &in) {
         if (P < 1 || Q < 1) return fail(SN_EINVAL, "conv2: empty output");
         L.out = {in[0].n, p.c_out, P, Q};
         L.act = p.act;
+        if (in.size() == 2 && !(in[1] == L.out))
+            return fail(SN_EINVAL, "conv2: the residual input must have the output's shape");
         return SN_OK;
     }
     case SN_L_MAXPOOL: {

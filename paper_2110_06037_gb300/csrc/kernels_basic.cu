@@ -268,7 +268,8 @@ cudaError_t weight_format(const float *w, void *out, int fmt, int dt, int64_t K,
 // ===========================================================================
 template <typename T>
 __global__ void conv_direct_nchw(const T *__restrict__ x, const T *__restrict__ w,
-                                 const float *__restrict__ bias, T *__restrict__ y, ConvDims d) {
+                                 const float *__restrict__ bias, const T *__restrict__ res, T *__restrict__ y,
+                                 ConvDims d) {
     griddep_launch();
     griddep_wait();
     const int64_t total = (int64_t)d.N * d.K * d.P * d.Q;
@@ -293,13 +294,15 @@ __global__ void conv_direct_nchw(const T *__restrict__ x, const T *__restrict__ 
                 }
             }
         }
+        if (res) acc += ldf<T>(res + i);  // residual: same layout and index as the output
         stf<T>(y + i, act_apply(acc + bias[kk], d.act));
     }
 }
 
 template <typename T>
 __global__ void conv_direct_nhwc(const T *__restrict__ x, const T *__restrict__ w,
-                                 const float *__restrict__ bias, T *__restrict__ y, ConvDims d) {
+                                 const float *__restrict__ bias, const T *__restrict__ res, T *__restrict__ y,
+                                 ConvDims d) {
     griddep_launch();
     griddep_wait();
     const int64_t total = (int64_t)d.N * d.K * d.P * d.Q;
@@ -323,6 +326,7 @@ __global__ void conv_direct_nhwc(const T *__restrict__ x, const T *__restrict__ 
                 for (int c = 0; c < Cg; ++c) acc += ldf<T>(xp + c) * ldf<T>(wp + (int64_t)c * d.K);
             }
         }
+        if (res) acc += ldf<T>(res + i);  // residual: same layout and index as the output
         stf<T>(y + i, act_apply(acc + bias[kk], d.act));
     }
 }
@@ -333,10 +337,10 @@ cudaError_t conv_direct(const LaunchArgs &a) {
     SN_DT_SWITCH(a.schema.dtype, T, {
         if (a.schema.layout == SN_NCHW)
             launch_pdl(conv_direct_nchw<T>, grid_for(total, 256), 256, 0, a.stream, 
-                (const T *)a.in[0], (const T *)a.wt, a.bias, (T *)a.out, d);
+                (const T *)a.in[0], (const T *)a.wt, a.bias, (const T *)a.in[1], (T *)a.out, d);
         else
             launch_pdl(conv_direct_nhwc<T>, grid_for(total, 256), 256, 0, a.stream, 
-                (const T *)a.in[0], (const T *)a.wt, a.bias, (T *)a.out, d);
+                (const T *)a.in[0], (const T *)a.wt, a.bias, (const T *)a.in[1], (T *)a.out, d);
     });
     return cudaGetLastError();
 }

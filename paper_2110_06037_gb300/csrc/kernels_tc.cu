@@ -101,7 +101,8 @@ __global__ void __launch_bounds__(THREADS, 1)
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(&accf_bar[b], 1);
-            mbar_init(&acce_bar[b], G * EPI_WARPS);  // one arrival per epilogue warp (of both CTAs)
+            // one arrival per epilogue warp draining it, in both CTAs of a pair
+            mbar_init(&acce_bar[b], G * (BN >= 128 ? EPI_WARPS : EPI_WARPS / 2));
         }
         abort_sh = 0;
         issued_sh[0] = issued_sh[1] = issued_sh[2] = issued_sh[3] = 0;
@@ -246,9 +247,10 @@ __global__ void __launch_bounds__(THREADS, 1)
             consumed_sh = g;
         }
     } else {  // ---------------- epilogue: warps 2..9
-        // Every unit is drained by all eight warps: warp w reads TMEM lanes
-        // 32*(w%4) .. +31 (tile rows) of the 64-channel chunks of its column
-        // half (w-2)/4 (both halves' chunks alternate when a tile has one).
+        // Warp w reads TMEM lanes 32*(w%4) .. +31 (tile rows).  Tiles of two or
+        // more 64-channel chunks: all eight warps drain every unit, warp w the
+        // chunks of column half (w-2)/4.  One-chunk tiles (BN = 64): the two
+        // groups of four take alternate units, i.e. one accumulator each.
         const int half = (warp - 2) >> 2;
         const int g4 = warp & 3;
         const int row = g4 * 32 + lane;
@@ -259,8 +261,10 @@ __global__ void __launch_bounds__(THREADS, 1)
         const int ni0 = IMPLICIT ? r0 / (p.BW * p.BH) : 0;
         constexpr int NCH = BN / 64 > 0 ? BN / 64 : 1;  // 64-channel chunks per tile
         constexpr int CPH = NCH >= 2 ? NCH / 2 : 1;      // chunks per column half
-        int lt = 0;
-        for (int u = cid; u < total; u += ncl, ++lt) {
+        constexpr bool ALT = NCH == 1;                   // alternate units between the groups
+        const int cbase = ALT ? 0 : half * CPH;          // first chunk of this warp
+        int lt = ALT ? half : 0;
+        for (int u = cid + (ALT ? half * ncl : 0); u < total; u += (ALT ? 2 : 1) * ncl, lt += ALT ? 2 : 1) {
             const int b = lt & 1;
             const uint32_t aph = (uint32_t)(lt >> 1) & 1u;
             const Work w = work_of(p, u, BN, IMPLICIT, G, (int)rank);
@@ -272,15 +276,9 @@ __global__ void __launch_bounds__(THREADS, 1)
             for (int cj = 0; cj < CPH; ++cj)
 #pragma unroll
                 for (int h = 0; h < 2; ++h)
-                    bias_r[cj][h] = (p.ksplit == 1 && half * CPH + cj < NCH)
-                                        ? __ldg(p.bias + w.n0 + 64 * (half * CPH + cj) + 32 * h + lane)
+                    bias_r[cj][h] = (p.ksplit == 1 && cbase + cj < NCH)
+                                        ? __ldg(p.bias + w.n0 + 64 * (cbase + cj) + 32 * h + lane)
                                         : 0.f;
-            if (!mbar_wait(&accf_bar[b], aph)) {
-                if (lane == 0) atomicOr(p.err, ERR_ACC_WAIT);
-                set_abort();
-                break;
-            }
-            tc_fence_after();
             bool valid;
             int64_t pix;
             if (IMPLICIT) {
@@ -293,10 +291,45 @@ __global__ void __launch_bounds__(THREADS, 1)
                 valid = pix < p.Mout;
             }
             // the idle CTA of a pair whose group has one tile stores nothing
-            const bool tile_live = w.mt < p.mtiles && (NCH >= 2 || half == 0);
+            const bool tile_live = w.mt < p.mtiles;
+            // residual (fused add) of this row's 64 channels of a chunk, zero past
+            // K or outside the output; the first chunk's is loaded before the
+            // accumulator wait, the next one's while the current one is stored
+            uint32_t rv[2][16];
+            auto load_res = [&](int k0) {
+#pragma unroll
+                for (int h = 0; h < 2; ++h)
+#pragma unroll
+                    for (int j = 0; j < 16; ++j) rv[h][j] = 0u;
+                if (!p.res || p.ksplit != 1 || !valid || !tile_live || k0 >= p.K) return;
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    const int kh = k0 + 32 * h;
+                    const T *rp = static_cast<const T *>(p.res) + pix * p.K + kh;
+                    if (kh + 32 <= p.K) {
+#pragma unroll
+                        for (int q4 = 0; q4 < 4; ++q4) {
+                            const uint4 u = __ldg(reinterpret_cast<const uint4 *>(rp) + q4);
+                            rv[h][4 * q4] = u.x, rv[h][4 * q4 + 1] = u.y, rv[h][4 * q4 + 2] = u.z,
+                            rv[h][4 * q4 + 3] = u.w;
+                        }
+                    } else {
+#pragma unroll
+                        for (int j = 0; j < 16; ++j)  // K % 8 == 0: pairs never straddle K
+                            if (kh + 2 * j < p.K) rv[h][j] = __ldg(reinterpret_cast<const unsigned int *>(rp) + j);
+                    }
+                }
+            };
+            load_res(w.n0 + 64 * cbase);
+            if (!mbar_wait(&accf_bar[b], aph)) {
+                if (lane == 0) atomicOr(p.err, ERR_ACC_WAIT);
+                set_abort();
+                break;
+            }
+            tc_fence_after();
 #pragma unroll
             for (int cj = 0; cj < CPH; ++cj) {
-                const int ci = half * CPH + cj;
+                const int ci = cbase + cj;
                 const int k0 = w.n0 + 64 * ci;
                 if (k0 >= p.K || !tile_live) break;
                 const uint32_t taddr = tmem + ((uint32_t)(g4 * 32) << 16) + (uint32_t)(b * BN + 64 * ci);
@@ -312,14 +345,17 @@ __global__ void __launch_bounds__(THREADS, 1)
                         tmem_ld32(taddr + 32 * h, v);
 #pragma unroll
                         for (int j = 0; j < 16; ++j) {
+                            const float2 r2 = unpack2<T>(rv[h][j]);
                             const float f0 = act_apply(
-                                __uint_as_float(v[2 * j]) + __shfl_sync(0xffffffffu, bias_r[cj][h], 2 * j), p.act);
-                            const float f1 = act_apply(
-                                __uint_as_float(v[2 * j + 1]) + __shfl_sync(0xffffffffu, bias_r[cj][h], 2 * j + 1),
+                                __uint_as_float(v[2 * j]) + __shfl_sync(0xffffffffu, bias_r[cj][h], 2 * j) + r2.x,
                                 p.act);
+                            const float f1 = act_apply(__uint_as_float(v[2 * j + 1]) +
+                                                           __shfl_sync(0xffffffffu, bias_r[cj][h], 2 * j + 1) + r2.y,
+                                                       p.act);
                             wv[16 * h + j] = pack2<T>(f0, f1);
                         }
                     }
+                    if (cj + 1 < CPH) load_res(k0 + 64);
                     if (lane == 0) bulk_wait_read_0();  // the previous store has read the staging block
                     __syncwarp();
 #pragma unroll
@@ -400,10 +436,11 @@ __global__ void __launch_bounds__(THREADS, 1)
     }
 }
 
-// y[m][k] = act(bias[k] + sum_s part[s][m][k]), four channels per thread
+// y[m][k] = act(bias[k] + sum_s part[s][m][k] (+ res[m][k])), four channels per thread
 template <typename T>
 __global__ void splitk_reduce_kernel(const float *__restrict__ part, const float *__restrict__ bias,
-                                     T *__restrict__ y, int64_t M, int K, int ks, int act) {
+                                     const T *__restrict__ res, T *__restrict__ y, int64_t M, int K, int ks,
+                                     int act) {
     griddep_launch();
     griddep_wait();
     const int K4 = K / 4;
@@ -418,6 +455,14 @@ __global__ void splitk_reduce_kernel(const float *__restrict__ part, const float
             acc.y += v.y;
             acc.z += v.z;
             acc.w += v.w;
+        }
+        if (res) {
+            const uint2 r = *reinterpret_cast<const uint2 *>(res + m * K + k);
+            const float2 r0 = unpack2<T>(r.x), r1 = unpack2<T>(r.y);
+            acc.x += r0.x;
+            acc.y += r0.y;
+            acc.z += r1.x;
+            acc.w += r1.y;
         }
         uint2 o;
         o.x = pack2<T>(act_apply(acc.x, act), act_apply(acc.y, act));
@@ -610,7 +655,8 @@ static cudaError_t launch(const CUtensorMap *mA, const CUtensorMap &mB, const CU
     cudaError_t e = cudaLaunchKernelEx(&cfg, kern, mA[0], mA[1], mA[2], mA[3], mB, mY, p);
     if (e != cudaSuccess || p.ksplit == 1) return e;
     const int64_t n4 = p.Mout * (p.K / 4);
-    launch_pdl(splitk_reduce_kernel<T>, grid_for(n4, 256), 256, 0, st, p.part, p.bias, static_cast<T *>(p.y), p.Mout, p.K,
+    launch_pdl(splitk_reduce_kernel<T>, grid_for(n4, 256), 256, 0, st, p.part, p.bias, static_cast<const T *>(p.res),
+               static_cast<T *>(p.y), p.Mout, p.K,
                                                                p.ksplit, p.act);
     return cudaGetLastError();
 }
@@ -652,6 +698,8 @@ cudaError_t conv_tc(const LaunchArgs &a) {
     p.act = c.act;
     p.bias = a.bias;
     p.y = a.out;
+    p.res = a.in[1];  // residual input of a fused add (null when the layer has one input)
+    if (p.res && (uintptr_t)p.res % 16) return cudaErrorInvalidValue;  // read as 16-byte vectors
     p.err = device_error_word();
     p.M = in.n * (int64_t)in.h * in.w;
     p.Mout = (int64_t)p.N * p.P * p.Q;

@@ -45,6 +45,9 @@ static bool is_conv(const Layer &l) { return l.type == SN_L_CONV2; }
 
 int32_t routine_variants(int32_t r, const Layer &l, const std::vector<Shape> &in, sn_schema s) {
     const sn_conv_params &p = l.conv;
+    // a conv2 with a residual input is served by the routines whose epilogue
+    // adds it: direct and the tensor-core implicit GEMM
+    if (is_conv(l) && in.size() == 2 && r != R_CONV_DIRECT && r != R_CONV_TC) return 0;
     switch (r) {
     case R_CONV_DIRECT:
         return is_conv(l) ? 1 : 0;

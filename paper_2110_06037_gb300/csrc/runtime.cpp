@@ -279,7 +279,7 @@ sn_status profile_graph(Graph *g, const sn_profile_opts &o, cudaStream_t st) {
             a.schema = s;
             a.in_shapes = in;
             a.in[0] = sc.in0.ptr;
-            a.in[1] = sc.in1.ptr;
+            a.in[1] = in.size() > 1 ? sc.in1.ptr : nullptr;  // a residual only where the layer has one
             a.out = sc.out.ptr;
             a.stream = st;
             if (k::fill_pattern(sc.in0.ptr, s.dtype, in[0].numel(), 1234u + i, 1.0f, st) != cudaSuccess ||

@@ -39,6 +39,7 @@ struct Params {
     int32_t act;
     const float *bias;             // fp32 [K], zero-padded to a multiple of 256 entries
     void *y;                       // output, NHWC, fp16/bf16
+    const void *res;               // residual added before the activation (output's layout), or null
     float *part;                   // K split: fp32 partial sums [ksplit][Mout][K]
     int *err;                      // the library's device error word
 };
@@ -261,6 +262,17 @@ template <>
 __device__ __forceinline__ uint32_t pack2<__nv_bfloat16>(float a, float b) {
     __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
     return *reinterpret_cast<uint32_t *>(&h);
+}
+// the two 16-bit values of a packed pair, widened exactly
+template <typename T>
+__device__ __forceinline__ float2 unpack2(uint32_t v);
+template <>
+__device__ __forceinline__ float2 unpack2<__half>(uint32_t v) {
+    return __half22float2(*reinterpret_cast<const __half2 *>(&v));
+}
+template <>
+__device__ __forceinline__ float2 unpack2<__nv_bfloat16>(uint32_t v) {
+    return __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&v));
 }
 
 

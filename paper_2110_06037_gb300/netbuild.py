@@ -21,3 +21,49 @@ def build_graph(layers, in_shape, in_schema, out_schema, schemas, torch_alloc=Tr
                           l.get("bias"))
         assert lid == i
     return g
+
+
+def fuse_residual(layers):
+    """Fuse every residual add into the convolution that feeds it.
+
+    A graph-optimiser pass over the plain-data description, run before the
+    net is built and tuned (the paper fuses layers ahead of tuning, section
+    III-A): an 'add' whose input is a 'conv2' with no activation, read by
+    nothing else, becomes that conv2 with the add's other input as a
+    residual and the add's activation, y = act(conv(x) + b + residual).  The
+    fused layer takes the add's place in the list (after both of its inputs)
+    and the conv2 is dropped; indices are renumbered.  Returns a new list.
+    """
+    consumers = {}
+    for i, l in enumerate(layers):
+        for j in l["inputs"]:
+            consumers.setdefault(j, []).append(i)
+    fold = {}  # add index -> (conv index, residual index)
+    for i, l in enumerate(layers):
+        if l["type"] != "add":
+            continue
+        for pos in (0, 1):
+            j, other = l["inputs"][pos], l["inputs"][1 - pos]
+            if j < 0 or layers[j]["type"] != "conv2" or len(layers[j]["inputs"]) != 1:
+                continue
+            if layers[j]["params"].get("act", "none") != "none" or consumers.get(j) != [i]:
+                continue
+            fold[i] = (j, other)
+            break
+    dropped = {j for (j, _) in fold.values()}
+    new_index, out = {}, []
+    for i, l in enumerate(layers):
+        if i in dropped:
+            continue
+        new_index[i] = len(out)
+        if i in fold:
+            j, other = fold[i]
+            conv = layers[j]
+            params = dict(conv["params"], act=l["params"].get("act", "none"))
+            out.append(dict(conv, name=conv.get("name", "conv") + "+" + l.get("name", "add"), params=params,
+                            inputs=[conv["inputs"][0], other]))
+        else:
+            out.append(dict(l))
+    for l in out:
+        l["inputs"] = [j if j < 0 else new_index[j] for j in l["inputs"]]
+    return out

@@ -7,6 +7,8 @@
   * MobileNetV2 b1 fp16, ResNet-50 b1 fp16: DPRS equals the oracle's exact
     block-wise search on the profiled table; output within 2e-2.
   * ResNet-50 b32 bf16: sampled images of the batch against the oracle.
+  * The same nets with every residual add fused into its conv2: DPRS equals
+    the block-wise search, outputs within 2e-2 of the (unfused) oracle.
 """
 import numpy as np
 import pytest
@@ -15,7 +17,7 @@ import oracle
 import synth
 from oracle.net import run_net
 from oracle.paths import blockwise_search
-from paper_2110_06037_gb300 import SN_OPT_CUDA_GRAPH, SN_SELECT_BRUTE, SN_SELECT_DPRS, build_graph
+from paper_2110_06037_gb300 import SN_OPT_CUDA_GRAPH, SN_SELECT_BRUTE, SN_SELECT_DPRS, build_graph, fuse_residual
 
 from gpu_helpers import TOL, from_device, maxrel, to_device
 from test_dprs import oracle_layer_cost
@@ -131,5 +133,38 @@ def test_resnet50_b32_bf16_sampled():
     torch.cuda.synchronize()
     got = from_device(y, ("bf16", "nchw"))
     for n in (0, 31):
+        ref = run_net(layers, x[n:n + 1], "bf16")
+        assert maxrel(got[n:n + 1], ref) <= TOL["bf16"]
+
+
+def test_fused_mobilenet_v2_b1_fp16():
+    x, layers = synth.mobilenet_v2(1)
+    fused = fuse_residual(layers)
+    g, got = _profile_select_run(fused, x, ("f16", "nchw"), ("f16", "nchw"), F16, exhaustive=False)
+    assert maxrel(got, run_net(layers, x, "f16")) <= TOL["f16"]
+
+
+def test_fused_resnet50_b1_fp16():
+    x, layers = synth.resnet50(1)
+    fused = fuse_residual(layers)
+    g, got = _profile_select_run(fused, x, ("f16", "nchw"), ("f16", "nchw"), F16, exhaustive=False)
+    assert maxrel(got, run_net(layers, x, "f16")) <= TOL["f16"]
+
+
+def test_fused_resnet50_b32_bf16_sampled():
+    import torch
+    x, layers = synth.resnet50(32)
+    fused = fuse_residual(layers)
+    g = build_graph(fused, x.shape, ("bf16", "nchw"), ("bf16", "nchw"), BF16)
+    g.profile(warmup=1, iters=3, topk=1, passes=2)
+    t = g.cost_table()
+    lc = oracle_layer_cost(t)
+    ref_total, _ = blockwise_search(lc, t["edges"], t["adapt"])
+    total, sch, _ = g.select_path(SN_SELECT_DPRS)
+    assert total == ref_total
+    y = g.run(to_device(x, ("bf16", "nchw")))
+    torch.cuda.synchronize()
+    got = from_device(y, ("bf16", "nchw"))
+    for n in (0, 17):
         ref = run_net(layers, x[n:n + 1], "bf16")
         assert maxrel(got[n:n + 1], ref) <= TOL["bf16"]

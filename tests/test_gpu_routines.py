@@ -157,3 +157,52 @@ def test_convert_empty_is_noop():
     import torch
     x = torch.zeros(4, device="cuda")
     convert(x, ("f32", "nchw"), ("f16", "nhwc"), (0, 3, 4, 4), out=torch.zeros(1, device="cuda", dtype=torch.float16))
+
+
+RES_CASES = [
+    # N, C, H, W, k, p  (C -> C channels, stride 1, "same" padding: the output has the input's shape)
+    (2, 24, 9, 11, 3, 1),     # C not a multiple of 64
+    (1, 64, 14, 14, 1, 0),    # plain GEMM tile
+    (2, 128, 8, 8, 3, 1),     # CTA pairs, two channel blocks per stage
+    (2, 256, 7, 7, 3, 1),     # K-split variants: the residual is added by the reduction
+    (4, 512, 7, 7, 1, 0),     # plain GEMM K split
+]
+
+
+@pytest.mark.parametrize("case", RES_CASES)
+@pytest.mark.parametrize("schema", SCHEMAS)
+def test_conv_residual(case, schema):
+    """conv2 with a residual input (a fused add): y = relu(conv(x) + b + r),
+    r = the 3x3 stride-1 max pool of x (a blob distinct from the conv input),
+    for every direct and tensor-core routine parameter the layer offers."""
+    import torch
+    N, C, H, W, k, p = case
+    rng = np.random.default_rng(abs(hash((case, schema, "res"))) % 2**32)
+    x = rng.standard_normal((N, C, H, W)).astype(np.float32)
+    pool = {"type": "maxpool", "name": "pool", "inputs": [-1],
+            "params": dict(kh=3, kw=3, sh=1, sw=1, ph=1, pw=1)}
+    conv = synth.conv(C, C, k, 1, p, act="relu")
+    conv["weight"] = (rng.standard_normal((C, C, k, k)) * np.sqrt(2.0 / (C * k * k))).astype(np.float32)
+    conv["bias"] = (rng.standard_normal(C) * 0.1).astype(np.float32)
+    conv["inputs"] = [-1, 0]
+    net = [pool, conv]
+    dt = schema[0]
+    xs = stored_values(x, dt)
+    r = run_layer(pool, [xs], dt)
+    ref = run_layer(conv, [xs, r], dt)
+    g = build_graph(net, x.shape, schema, schema, [schema])
+    t = g.cost_table()
+    io_in = int(np.flatnonzero(t["layer"] == 0)[0])
+    io_out = int(np.flatnonzero(t["layer"] == 3)[0])
+    pc = find_candidate(t, 1, "maxpool/direct", 0, 0)
+    ran = 0
+    for c in range(len(t["cost"])):
+        if t["layer"][c] != 2:
+            continue
+        g.set_path([io_in, pc, c, io_out])
+        y = g.run(to_device(x, schema))
+        torch.cuda.synchronize()
+        err = maxrel(from_device(y, schema), ref)
+        assert err <= TOL[dt], (int(t["routine"][c]), int(t["variant"][c]), err)
+        ran += 1
+    assert ran >= 1
