@@ -58,7 +58,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     conv_tc_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ CUtensorMap mA1,
                    const __grid_constant__ CUtensorMap mA2, const __grid_constant__ CUtensorMap mA3,
                    const __grid_constant__ CUtensorMap mB, const __grid_constant__ CUtensorMap mY,
-                   const Params p) {
+                   const __grid_constant__ CUtensorMap mR, const Params p) {
     // a stage holds KB 64-channel blocks of one filter tap; a block of A is
     // 128 rows x 128 B, of B (BN / G) rows x 128 B (this CTA's share)
     constexpr uint32_t A_BLK = BM * BK * 2;
@@ -72,6 +72,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     __shared__ __align__(8) uint64_t empty_bar[STAGES];
     __shared__ __align__(8) uint64_t accf_bar[2];  // MMA -> epilogue: accumulator ready
     __shared__ __align__(8) uint64_t acce_bar[2];  // epilogue -> MMA: accumulator drained
+    __shared__ __align__(8) uint64_t res_bar[EPI_WARPS];  // residual tile landed in a warp's staging block
     __shared__ uint32_t tmem_sh;
     __shared__ volatile int abort_sh;
     __shared__ int issued_sh[4], consumed_sh;
@@ -93,8 +94,8 @@ __global__ void __launch_bounds__(THREADS, 1)
 
     if (threadIdx.x == 0) {
         // the tensor maps are kernel parameters, not data of the previous kernel
-        const CUtensorMap *maps[6] = {&mA0, &mA1, &mA2, &mA3, &mB, &mY};
-        for (int i = 0; i < 6; ++i) asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(maps[i])) : "memory");
+        const CUtensorMap *maps[7] = {&mA0, &mA1, &mA2, &mA3, &mB, &mY, &mR};
+        for (int i = 0; i < 7; ++i) asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(maps[i])) : "memory");
         for (int s = 0; s < STAGES; ++s) {
             mbar_init(&full_bar[s], 1);  // the (leader's) producer of the stage
             mbar_init(&empty_bar[s], 1);
@@ -103,6 +104,9 @@ __global__ void __launch_bounds__(THREADS, 1)
             mbar_init(&accf_bar[b], 1);
             // one arrival per epilogue warp draining it, in both CTAs of a pair
             mbar_init(&acce_bar[b], G * (BN >= 128 ? EPI_WARPS : EPI_WARPS / 2));
+        }
+        for (int i = 0; i < EPI_WARPS; ++i) {
+            mbar_init(&res_bar[i], 1);
         }
         abort_sh = 0;
         issued_sh[0] = issued_sh[1] = issued_sh[2] = issued_sh[3] = 0;
@@ -264,6 +268,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         constexpr bool ALT = NCH == 1;                   // alternate units between the groups
         const int cbase = ALT ? 0 : half * CPH;          // first chunk of this warp
         int lt = ALT ? half : 0;
+        uint32_t rpar = 0;  // phase parity of this warp's residual barrier
         for (int u = cid + (ALT ? half * ncl : 0); u < total; u += (ALT ? 2 : 1) * ncl, lt += ALT ? 2 : 1) {
             const int b = lt & 1;
             const uint32_t aph = (uint32_t)(lt >> 1) & 1u;
@@ -292,35 +297,24 @@ __global__ void __launch_bounds__(THREADS, 1)
             }
             // the idle CTA of a pair whose group has one tile stores nothing
             const bool tile_live = w.mt < p.mtiles;
-            // residual (fused add) of this row's 64 channels of a chunk, zero past
-            // K or outside the output; the first chunk's is loaded before the
-            // accumulator wait, the next one's while the current one is stored
-            uint32_t rv[2][16];
-            auto load_res = [&](int k0) {
-#pragma unroll
-                for (int h = 0; h < 2; ++h)
-#pragma unroll
-                    for (int j = 0; j < 16; ++j) rv[h][j] = 0u;
-                if (!p.res || p.ksplit != 1 || !valid || !tile_live || k0 >= p.K) return;
-#pragma unroll
-                for (int h = 0; h < 2; ++h) {
-                    const int kh = k0 + 32 * h;
-                    const T *rp = static_cast<const T *>(p.res) + pix * p.K + kh;
-                    if (kh + 32 <= p.K) {
-#pragma unroll
-                        for (int q4 = 0; q4 < 4; ++q4) {
-                            const uint4 u = __ldg(reinterpret_cast<const uint4 *>(rp) + q4);
-                            rv[h][4 * q4] = u.x, rv[h][4 * q4 + 1] = u.y, rv[h][4 * q4 + 2] = u.z,
-                            rv[h][4 * q4 + 3] = u.w;
-                        }
-                    } else {
-#pragma unroll
-                        for (int j = 0; j < 16; ++j)  // K % 8 == 0: pairs never straddle K
-                            if (kh + 2 * j < p.K) rv[h][j] = __ldg(reinterpret_cast<const unsigned int *>(rp) + j);
-                    }
+            // residual (fused add): the warp's 32 x 64 block of it is loaded by
+            // TMA into the warp's staging block (the box and coordinates of the
+            // output store; zero outside the tensor) once the previous store has
+            // read that block; the first chunk's load is issued before the
+            // accumulator wait, the next one's after the current chunk's store
+            const bool has_res = p.res != nullptr && p.ksplit == 1;
+            auto issue_res = [&](int k0) {
+                if (!has_res || !tile_live || k0 >= p.K) return;
+                if (lane == 0) {
+                    bulk_wait_read_0();
+                    mbar_expect_tx(&res_bar[warp - 2], STG_BYTES);
+                    if (IMPLICIT)
+                        tma_4d<1>(su32(buf), &mR, su32(&res_bar[warp - 2]), k0, w.q0 + wq0, w.p0 + hp0, w.i0 + ni0);
+                    else
+                        tma_2d<1>(su32(buf), &mR, su32(&res_bar[warp - 2]), k0, (int)(w.m0 + r0));
                 }
             };
-            load_res(w.n0 + 64 * cbase);
+            issue_res(w.n0 + 64 * cbase);
             if (!mbar_wait(&accf_bar[b], aph)) {
                 if (lane == 0) atomicOr(p.err, ERR_ACC_WAIT);
                 set_abort();
@@ -338,6 +332,27 @@ __global__ void __launch_bounds__(THREADS, 1)
                     // (row = lane, 16-byte chunk j at j ^ (row & 7)), then one TMA
                     // tensor store of the warp's 32 x 64 block, clipped at the edges
                     uint32_t wv[32];
+                    // this row's residual: 16-byte piece j of the row at j ^ (row & 7)
+                    uint32_t rv[2][16];
+#pragma unroll
+                    for (int h = 0; h < 2; ++h)
+#pragma unroll
+                        for (int j = 0; j < 16; ++j) rv[h][j] = 0u;
+                    if (has_res) {
+                        if (!mbar_wait(&res_bar[warp - 2], rpar)) {
+                            if (lane == 0) atomicOr(p.err, ERR_EPI_WAIT);
+                            set_abort();
+                        }
+                        rpar ^= 1u;
+#pragma unroll
+                        for (int j = 0; j < 8; ++j) {
+                            const uint4 u = *reinterpret_cast<const uint4 *>(buf + lane * 128 + ((j ^ (lane & 7)) << 4));
+                            rv[j >> 2][4 * (j & 3)] = u.x;
+                            rv[j >> 2][4 * (j & 3) + 1] = u.y;
+                            rv[j >> 2][4 * (j & 3) + 2] = u.z;
+                            rv[j >> 2][4 * (j & 3) + 3] = u.w;
+                        }
+                    }
 #pragma unroll
                     for (int h = 0; h < 2; ++h) {
                         uint32_t v[32];
@@ -355,7 +370,6 @@ __global__ void __launch_bounds__(THREADS, 1)
                             wv[16 * h + j] = pack2<T>(f0, f1);
                         }
                     }
-                    if (cj + 1 < CPH) load_res(k0 + 64);
                     if (lane == 0) bulk_wait_read_0();  // the previous store has read the staging block
                     __syncwarp();
 #pragma unroll
@@ -371,6 +385,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                             tma_store_2d(&mY, buf, k0, (int)(w.m0 + r0));
                         bulk_commit();
                     }
+                    if (cj + 1 < CPH) issue_res(k0 + 64);
                 } else {
 #pragma unroll
                     for (int h = 0; h < 2; ++h) {
@@ -610,7 +625,8 @@ static int num_sms() {
 }
 
 template <typename T, int BN, bool IMPLICIT, int G, int KB>
-static cudaError_t launch(const CUtensorMap *mA, const CUtensorMap &mB, const CUtensorMap &mY, const Params &p,
+static cudaError_t launch(const CUtensorMap *mA, const CUtensorMap &mB, const CUtensorMap &mY, const CUtensorMap &mR,
+                          const Params &p,
                           cudaStream_t st) {
     constexpr int STAGES = stages_for(BN, G, KB);
     constexpr size_t smem = (size_t)STAGES * KB * (BM * BK * 2 + (BN / G) * BK * 2) + EPI_WARPS * STG_BYTES + 1024;
@@ -652,7 +668,7 @@ static cudaError_t launch(const CUtensorMap *mA, const CUtensorMap &mB, const CU
     }
     const int total = (p.mtiles + G - 1) / G * p.ntiles * p.ksplit;
     cfg.gridDim = dim3((unsigned)(G * std::min(total, max_groups)));
-    cudaError_t e = cudaLaunchKernelEx(&cfg, kern, mA[0], mA[1], mA[2], mA[3], mB, mY, p);
+    cudaError_t e = cudaLaunchKernelEx(&cfg, kern, mA[0], mA[1], mA[2], mA[3], mB, mY, mR, p);
     if (e != cudaSuccess || p.ksplit == 1) return e;
     const int64_t n4 = p.Mout * (p.K / 4);
     launch_pdl(splitk_reduce_kernel<T>, grid_for(n4, 256), 256, 0, st, p.part, p.bias, static_cast<const T *>(p.res),
@@ -711,7 +727,7 @@ cudaError_t conv_tc(const LaunchArgs &a) {
     }
     const int dt = a.schema.dtype;
     const uint64_t es = 2;
-    CUtensorMap mA[4], mB, mY;
+    CUtensorMap mA[4], mB, mY, mR;
     // KB > 1 (channels a multiple of 128): every map gets an outermost
     // channel-block axis of stride 128 B over the 64-channel inner axis, so that
     // one box lands KB consecutive 128-B-row blocks in shared memory
@@ -735,6 +751,9 @@ cudaError_t conv_tc(const LaunchArgs &a) {
         const uint64_t ystr[1] = {p.K * es};
         const uint32_t ybox[2] = {64, 32};
         if (!encode(&mY, dt, 2, a.out, ydims, ystr, ybox, CU_TENSOR_MAP_SWIZZLE_128B)) return cudaErrorInvalidValue;
+        mR = mY;  // the residual has the output's layout
+        if (p.res && !encode(&mR, dt, 2, p.res, ydims, ystr, ybox, CU_TENSOR_MAP_SWIZZLE_128B))
+            return cudaErrorInvalidValue;
     } else {
         p.BW = cf.BW, p.BH = cf.BH, p.BNI = cf.BNI;
         p.tq = (p.Q + cf.BW - 1) / cf.BW;
@@ -768,12 +787,15 @@ cudaError_t conv_tc(const LaunchArgs &a) {
         const uint64_t ystr[3] = {p.K * es, (uint64_t)p.Q * p.K * es, (uint64_t)p.P * p.Q * p.K * es};
         const uint32_t ybox[4] = {64, sbw, sbh, sbn};
         if (!encode(&mY, dt, 4, a.out, ydims, ystr, ybox, CU_TENSOR_MAP_SWIZZLE_128B)) return cudaErrorInvalidValue;
+        mR = mY;
+        if (p.res && !encode(&mR, dt, 4, p.res, ydims, ystr, ybox, CU_TENSOR_MAP_SWIZZLE_128B))
+            return cudaErrorInvalidValue;
     }
     if (p.mtiles <= 0 || (int64_t)p.mtiles * p.ntiles * p.ksplit > INT32_MAX) return cudaErrorInvalidValue;
     const bool bf = dt == SN_BF16;
 #define SN_TC_LAUNCH(TT, BNV, GV, KBV)                                                            \
-    return cf.implicit ? launch<TT, BNV, true, GV, KBV>(mA, mB, mY, p, a.stream)                   \
-                       : launch<TT, BNV, false, GV, KBV>(mA, mB, mY, p, a.stream)
+    return cf.implicit ? launch<TT, BNV, true, GV, KBV>(mA, mB, mY, mR, p, a.stream)               \
+                       : launch<TT, BNV, false, GV, KBV>(mA, mB, mY, mR, p, a.stream)
 #define SN_TC_LAUNCH_T(TT)                                                                          \
     if (cf.G == 2) {                                                                                \
         if (cf.KB == 2) {                                                                           \
