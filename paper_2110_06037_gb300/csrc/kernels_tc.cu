@@ -763,7 +763,11 @@ cudaError_t conv_tc(const LaunchArgs &a) {
         const uint64_t c0dim = blk ? 64 : (uint64_t)p.C;
         if (p.stride == 1) {
             const uint64_t dims[5] = {c0dim, (uint64_t)p.W, (uint64_t)p.H, (uint64_t)p.N, CB};
-            const uint64_t str[4] = {p.C * es, (uint64_t)p.W * p.C * es, (uint64_t)p.H * p.W * p.C * es, 128};
+            uint64_t str[4] = {p.C * es, (uint64_t)p.W * p.C * es, (uint64_t)p.H * p.W * p.C * es, 128};
+            if (a.a_strides[0] > 0) {  // a caller-laid-out A (overlapping pixel rows)
+                if (blk) return cudaErrorInvalidValue;
+                for (int i = 0; i < 3; ++i) str[i] = (uint64_t)a.a_strides[i];
+            }
             if (!encode(&mA[0], dt, blk ? 5 : 4, a.in[0], dims, str, box)) return cudaErrorInvalidValue;
             mA[1] = mA[2] = mA[3] = mA[0];
         } else {
@@ -965,6 +969,116 @@ cudaError_t conv_im2col_tc(const LaunchArgs &a) {
     g.in[0] = a.ws;
     g.ws = static_cast<uint8_t *>(a.ws) + im2col_bytes(l, a.schema);
     g.ws_bytes = a.ws_bytes - im2col_bytes(l, a.schema);
+    return conv_tc(g);
+}
+
+// ---------------------------------------------------------------------------
+// space-to-depth childnet: stride-2 convolutions of at most 4 input channels
+// (the RGB stem) as a stride-1 tensor-core convolution, with no im2col matrix.
+//
+// With xp the input zero-padded by (ph, pw) and taps r = 2a + i, s = 2b + j,
+//   y[p][q] = sum_{a, b, i, j, c} X[p + a][q + b][(2i + j) C + c] * W[a][b][(2i + j) C + c]
+//   X[u][v][(2i + j) C + c] = xp[2u + i][2v + j][c],   W[a][b][..] = w[2a + i][2b + j][c]
+// (W zero where 2a + i >= kh or 2b + j >= kw): ceil(kh/2) x ceil(kw/2) taps
+// over an image of 4C channels.  X stores 16 channels per pixel (4C <= 16,
+// the rest zero) and b runs over 4 pixels (kw <= 8), so the 64 values that
+// one row of taps a multiplies for output pixel (p, q) are X[p + a][q .. q+3],
+// contiguous: the GEMM's A row is one 128-byte window of X whose start moves
+// by one 32-byte pixel per output pixel.  The tensor map over X says exactly
+// that (pixel stride 32 B, rows of 64 values), so the implicit-GEMM kernel
+// runs unchanged with ceil(kh/2) K steps of 64.
+// ---------------------------------------------------------------------------
+namespace {
+struct S2dDims {
+    int32_t N, H, W, C, ph, pw, Pp, Qp;  // input; X extent Pp x Qp
+};
+}  // namespace
+
+static bool s2d_applies(const Layer &l, sn_schema s) {
+    const sn_conv_params &c = l.conv;
+    return l.type == SN_L_CONV2 && c.groups == 1 && c.sh == 2 && c.sw == 2 && c.dh == 1 && c.dw == 1 &&
+           4 * c.c_in <= 16 && c.kh >= 3 && c.kh <= 8 && c.kw <= 8 && c.c_out % 8 == 0 && s.dtype != SN_F32 &&
+           s.layout == SN_NHWC;
+}
+
+// the stride-1 layer the GEMM computes, and its input (X: Pp x Qp pixels of 64
+// "channels", the window)
+static Layer s2d_gemm_layer(const Layer &l) {
+    Layer g;
+    g.type = SN_L_CONV2;
+    g.conv = sn_conv_params{64, l.conv.c_out, (l.conv.kh + 1) / 2, 1, 1, 1, 0, 0, 1, 1, 1, l.conv.act};
+    g.act = l.conv.act;
+    g.out = l.out;
+    return g;
+}
+static Shape s2d_gemm_in(const Layer &l) { return Shape{l.out.n, 64, l.out.h + (l.conv.kh + 1) / 2 - 1, l.out.w}; }
+
+static size_t s2d_bytes(const Layer &l, sn_schema s) {
+    const int64_t Pp = l.out.h + (l.conv.kh + 1) / 2 - 1, Qp = l.out.w + 3;
+    return ((size_t)l.out.n * Pp * Qp * 16 * dtype_size(s.dtype) + 255) & ~size_t(255);
+}
+
+int32_t conv_s2d_tc_variants(const Layer &l, const Shape &in, sn_schema s) {
+    (void)in;
+    if (!s2d_applies(l, s)) return 0;
+    return (int32_t)tc::configs(s2d_gemm_layer(l), s2d_gemm_in(l), s).size();
+}
+
+size_t conv_s2d_tc_ws(const Layer &l, const Shape &in, sn_schema s, int32_t v) {
+    (void)in;
+    return s2d_bytes(l, s) + conv_tc_ws(s2d_gemm_layer(l), s2d_gemm_in(l), s, v);
+}
+
+// X[n][u][v][16]: one thread per X pixel, two 16-byte stores
+template <typename T>
+__global__ void __launch_bounds__(256) s2d_kernel(const T *__restrict__ x, T *__restrict__ X, S2dDims d) {
+    griddep_launch();
+    griddep_wait();
+    const int64_t total = (int64_t)d.N * d.Pp * d.Qp;
+    for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < total; t += (int64_t)gridDim.x * blockDim.x) {
+        const int v = (int)(t % d.Qp), u = (int)((t / d.Qp) % d.Pp);
+        const int64_t n = t / ((int64_t)d.Qp * d.Pp);
+        uint4 o[2] = {make_uint4(0, 0, 0, 0), make_uint4(0, 0, 0, 0)};
+        T *po = reinterpret_cast<T *>(o);
+#pragma unroll
+        for (int ij = 0; ij < 4; ++ij) {
+            const int h = 2 * u + (ij >> 1) - d.ph, w = 2 * v + (ij & 1) - d.pw;
+            if (h < 0 || h >= d.H || w < 0 || w >= d.W) continue;
+            const T *xp = x + ((n * d.H + h) * d.W + w) * d.C;
+            for (int c = 0; c < d.C; ++c) po[ij * d.C + c] = xp[c];
+        }
+        uint4 *dst = reinterpret_cast<uint4 *>(X + t * 16);
+        dst[0] = o[0];
+        dst[1] = o[1];
+    }
+}
+
+cudaError_t conv_s2d_tc(const LaunchArgs &a) {
+    const Layer &l = *a.layer;
+    if (!s2d_applies(l, a.schema)) return cudaErrorInvalidValue;
+    const Shape &in = a.in_shapes[0];
+    const Shape gin = s2d_gemm_in(l);
+    S2dDims d{(int32_t)in.n, (int32_t)in.h, (int32_t)in.w, (int32_t)in.c, l.conv.ph, l.conv.pw,
+              (int32_t)gin.h, (int32_t)(l.out.w + 3)};
+    const size_t xb = s2d_bytes(l, a.schema);
+    if (!a.ws || a.ws_bytes < xb || (uintptr_t)a.ws % 256) return cudaErrorInvalidValue;
+    const int64_t total = (int64_t)d.N * d.Pp * d.Qp;
+    SN_DT_SWITCH(a.schema.dtype, T,
+                 launch_pdl(s2d_kernel<T>, grid_for(total, 256), 256, 0, a.stream, (const T *)a.in[0], (T *)a.ws, d));
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    const Layer gl = s2d_gemm_layer(l);
+    LaunchArgs g = a;
+    g.layer = &gl;
+    g.routine = R_CONV_TC;
+    g.in_shapes = {gin};
+    g.in[0] = a.ws;
+    const int64_t pix = 16 * (int64_t)dtype_size(a.schema.dtype);  // 32 bytes: one X pixel
+    g.a_strides[0] = pix;
+    g.a_strides[1] = pix * d.Qp;
+    g.a_strides[2] = pix * d.Qp * d.Pp;
+    g.ws = static_cast<uint8_t *>(a.ws) + xb;
+    g.ws_bytes = a.ws_bytes - xb;
     return conv_tc(g);
 }
 

@@ -25,6 +25,7 @@ const char *routine_name(int32_t r) {
     case R_ADAPT: return "adapt/convert";
     case R_CONV_IM2COL_TC: return "conv2/im2col_tc";
     case R_DENSE_TC: return "dense/gemm_tc";
+    case R_CONV_S2D_TC: return "conv2/s2d_tc";
     default: return nullptr;
     }
 }
@@ -36,6 +37,7 @@ const char *variant_name(int32_t r, int32_t v) {
     case R_DW_DIRECT: return v == 0 ? "nhwc:window|nchw:rows" : "nhwc:smem_halo|nchw:plane_tile";
     case R_CONV_TC:
     case R_CONV_IM2COL_TC:
+    case R_CONV_S2D_TC:
     case R_DENSE_TC: return k::conv_tc_variant_name(v);
     default: return v == 0 ? "" : "?";
     }
@@ -74,6 +76,8 @@ int32_t routine_variants(int32_t r, const Layer &l, const std::vector<Shape> &in
         return is_conv(l) ? k::conv_im2col_tc_variants(l, in[0], s) : 0;
     case R_DENSE_TC:
         return l.type == SN_L_DENSE ? k::dense_tc_variants(l, in[0], s) : 0;
+    case R_CONV_S2D_TC:
+        return is_conv(l) ? k::conv_s2d_tc_variants(l, in[0], s) : 0;
     default:
         return 0;
     }
@@ -85,6 +89,7 @@ size_t routine_workspace(int32_t r, int32_t v, const Layer &l, const std::vector
     if (r == R_CONV_TC) return k::conv_tc_ws(l, in[0], s, v);
     if (r == R_CONV_IM2COL_TC) return k::conv_im2col_tc_ws(l, in[0], s, v);
     if (r == R_DENSE_TC) return k::dense_tc_ws(l, in[0], s, v);
+    if (r == R_CONV_S2D_TC) return k::conv_s2d_tc_ws(l, in[0], s, v);
     return 0;
 }
 
@@ -99,6 +104,7 @@ static int weight_format_of(int32_t r, sn_schema s) {
     case R_DENSE: return k::W_KCRS;
     case R_CONV_IM2COL_TC: return k::W_KRSC_PAD64;
     case R_DENSE_TC: return k::W_KRSC;
+    case R_CONV_S2D_TC: return k::W_S2D;
     default: return -1;
     }
 }
@@ -142,6 +148,7 @@ sn_status prepare_weights(Graph *g, int32_t li, int32_t r, int32_t v, sn_schema 
     }
     const int64_t elems = (fmt == k::W_WINO)         ? 16 * K * Cg
                           : (fmt == k::W_KRSC_PAD64) ? K * ((Cg * R * S + 63) / 64 * 64)
+                          : (fmt == k::W_S2D)        ? K * ((R + 1) / 2) * 64
                                                      : K * Cg * R * S;
     Buffer src, dst;
     sn_status rc = dev_alloc(g, (size_t)K * Cg * R * S * sizeof(float), &src);
@@ -169,10 +176,13 @@ sn_status prepare_weights(Graph *g, int32_t li, int32_t r, int32_t v, sn_schema 
 int32_t kernels_per_launch(int32_t r, int32_t v, const Layer &l, const std::vector<Shape> &in, sn_schema s) {
     // a K-split tensor-core GEMM adds its reduction kernel (it is the only
     // variant with a workspace)
-    const int split = (r == R_CONV_TC || r == R_CONV_IM2COL_TC || r == R_DENSE_TC) &&
-                      routine_workspace(r, v, l, in, s) > (r == R_CONV_IM2COL_TC ? k::conv_im2col_tc_ws(l, in[0], s, -1) : 0);
+    const int split = (r == R_CONV_TC || r == R_CONV_IM2COL_TC || r == R_DENSE_TC || r == R_CONV_S2D_TC) &&
+                      routine_workspace(r, v, l, in, s) >
+                          (r == R_CONV_IM2COL_TC ? k::conv_im2col_tc_ws(l, in[0], s, -1)
+                           : r == R_CONV_S2D_TC  ? k::conv_s2d_tc_ws(l, in[0], s, -1)
+                                                 : 0);
     if (r == R_CONV_WINO) return 3;             // wgenc, wgconv, wgdec
-    if (r == R_CONV_IM2COL_TC) return 2 + split;  // im2col, GEMM (+ reduction)
+    if (r == R_CONV_IM2COL_TC || r == R_CONV_S2D_TC) return 2 + split;  // re-layout, GEMM (+ reduction)
     return 1 + split;
 }
 
@@ -190,6 +200,7 @@ sn_status launch_routine(const LaunchArgs &a) {
     case R_DENSE: e = k::dense(a); break;
     case R_CONV_IM2COL_TC: e = k::conv_im2col_tc(a); break;
     case R_DENSE_TC: e = k::dense_tc(a); break;
+    case R_CONV_S2D_TC: e = k::conv_s2d_tc(a); break;
     default: return fail(SN_EINVAL, "launch of a non-launchable routine");
     }
     if (e != cudaSuccess)

@@ -66,7 +66,8 @@ enum RoutineId : int32_t {
     R_ADAPT = 10,        // adapt layer (cast / layout change)
     R_CONV_IM2COL_TC = 11,  // childnet: im2col -> tensor-core GEMM (any C, stride, dilation)
     R_DENSE_TC = 12,     // childnet: reshape -> 1x1 conv2 on tensor cores -> reshape (section III-D)
-    R_COUNT = 13
+    R_CONV_S2D_TC = 13,  // childnet: space-to-depth -> stride-1 tensor-core conv (stride 2, <= 4 channels)
+    R_COUNT = 14
 };
 
 // -------------------------------------------------------------------------
@@ -119,6 +120,10 @@ struct LaunchArgs {
     const float *bias = nullptr;
     void *ws = nullptr;         // workspace
     size_t ws_bytes = 0;
+    // tensor-core implicit GEMM only: byte strides of the A tensor's pixel,
+    // row and image axes when they differ from dense NHWC (0 = dense); a pixel
+    // stride below the 128-byte row makes consecutive pixels' rows overlap
+    int64_t a_strides[3] = {0, 0, 0};
     cudaStream_t stream = nullptr;
 };
 
@@ -209,7 +214,7 @@ cudaError_t convert(const void *x, int dt_in, int lay_in, void *y, int dt_out, i
 cudaError_t fill_pattern(void *y, int dt, int64_t n, uint32_t seed, float scale,
                          cudaStream_t st);
 // weight re-layout / cast from fp32 KCRS (device) into a routine format
-enum WFormat { W_KCRS = 0, W_RSCK = 1, W_KRSC = 2, W_WINO = 3, W_KRSC_PAD64 = 4 };
+enum WFormat { W_KCRS = 0, W_RSCK = 1, W_KRSC = 2, W_WINO = 3, W_KRSC_PAD64 = 4, W_S2D = 5 };
 cudaError_t weight_format(const float *w_kcrs, void *out, int fmt, int dt, int64_t K,
                           int64_t Cg, int64_t R, int64_t S, cudaStream_t st);
 
@@ -227,6 +232,10 @@ int32_t conv_im2col_tc_variants(const Layer &l, const Shape &in, sn_schema s);
 size_t conv_im2col_tc_ws(const Layer &l, const Shape &in, sn_schema s, int32_t v);
 cudaError_t conv_im2col_tc(const LaunchArgs &a);
 int32_t dense_tc_variants(const Layer &l, const Shape &in, sn_schema s);
+// space-to-depth childnet for stride-2 convolutions of few input channels
+int32_t conv_s2d_tc_variants(const Layer &l, const Shape &in, sn_schema s);
+size_t conv_s2d_tc_ws(const Layer &l, const Shape &in, sn_schema s, int32_t v);
+cudaError_t conv_s2d_tc(const LaunchArgs &a);
 cudaError_t dense_tc(const LaunchArgs &a);
 cudaError_t dwconv(const LaunchArgs &a);
 cudaError_t maxpool(const LaunchArgs &a);

@@ -54,9 +54,13 @@ CONV_CASES = [
     (1, 8, 12, 12, 8, 3, 1, 2, 2, 1),      # dilation
     (1, 130, 5, 5, 66, 3, 1, 1, 1, 1),     # channels past a tile edge
     (1, 16, 1, 1, 8, 3, 1, 1, 1, 1),       # 1x1 image, 3x3 kernel (padding only)
+    (2, 3, 30, 30, 64, 7, 2, 3, 1, 1),     # the ResNet stem's shape class (space-to-depth routine)
+    (1, 4, 17, 19, 24, 3, 2, 1, 1, 1),     # space-to-depth: 4 channels, odd extents
+    (1, 2, 16, 16, 8, 5, 2, 2, 1, 1),      # space-to-depth: 5x5 kernel
 ]
 ROUTINES = ([("conv2/direct", 0), ("conv2/igemm_simt", 0), ("conv2/igemm_simt", 1), ("conv2/wino_f2x2_3x3", 0)]
-            + [("conv2/igemm_tc", v) for v in range(6)] + [("conv2/im2col_tc", v) for v in range(3)])
+            + [("conv2/igemm_tc", v) for v in range(6)] + [("conv2/im2col_tc", v) for v in range(3)]
+            + [("conv2/s2d_tc", v) for v in range(4)])
 
 
 @pytest.mark.parametrize("case", CONV_CASES)
