@@ -350,26 +350,18 @@ sn_status sn_run_timed(sn_graph *gg, const void *in_dev, void *out_dev, void *st
             sn_status rc = build_plan(g, st);
             if (rc != SN_OK) return rc;
         }
-        std::vector<cudaEvent_t> evs(2 * g->plan.size());
-        for (auto &e : evs) SN_CUDA_TRY(cudaEventCreate(&e));
-        sn_status rc = run_plan(g, in_dev, out_dev, st, &evs);
-        cudaError_t ce = cudaStreamSynchronize(st);
-        if (rc == SN_OK && ce == cudaSuccess) {
-            if (layer_ms)
-                for (int32_t i = 0; i < g->n_layers(); ++i) layer_ms[i] = 0.f;
-            if (edge_ms)
-                for (size_t e = 0; e < g->edges.size(); ++e) edge_ms[e] = 0.f;
-            for (size_t q = 0; q < g->plan.size(); ++q) {
-                float t = 0;
-                cudaEventElapsedTime(&t, evs[2 * q], evs[2 * q + 1]);
-                const PlanOp &op = g->plan[q];
-                if (op.kind == PlanOp::LAYER && layer_ms) layer_ms[op.layer] += t;
-                if (op.kind == PlanOp::ADAPT && edge_ms && op.edge >= 0) edge_ms[op.edge] += t;
-            }
-        }
-        for (auto &e : evs) cudaEventDestroy(e);
+        std::vector<float> op_ms;
+        sn_status rc = run_plan_timed(g, in_dev, out_dev, st, &op_ms);
         if (rc != SN_OK) return rc;
-        if (ce != cudaSuccess) return fail(SN_ECUDA, std::string("sn_run_timed: ") + cudaGetErrorString(ce));
+        if (layer_ms)
+            for (int32_t i = 0; i < g->n_layers(); ++i) layer_ms[i] = 0.f;
+        if (edge_ms)
+            for (size_t e = 0; e < g->edges.size(); ++e) edge_ms[e] = 0.f;
+        for (size_t q = 0; q < g->plan.size(); ++q) {
+            const PlanOp &op = g->plan[q];
+            if (op.kind == PlanOp::LAYER && layer_ms) layer_ms[op.layer] += op_ms[q];
+            if (op.kind == PlanOp::ADAPT && edge_ms && op.edge >= 0) edge_ms[op.edge] += op_ms[q];
+        }
         if (g->opt_check) return check_device(g, st);
         return SN_OK;
     })

@@ -165,10 +165,11 @@ sn_status run_plan(Graph *g, const void *in, void *out, cudaStream_t st,
         if (rc != SN_OK) return rc;
     }
     for (size_t i = 0; i < g->plan.size(); ++i) {
-        if (evs) SN_CUDA_TRY(cudaEventRecord((*evs)[2 * i], st));
+        // external records: timing nodes when the stream is being captured
+        if (evs) SN_CUDA_TRY(cudaEventRecordWithFlags((*evs)[2 * i], st, cudaEventRecordExternal));
         sn_status rc = launch_op(g, g->plan[i], in, out, st);
         if (rc != SN_OK) return rc;
-        if (evs) SN_CUDA_TRY(cudaEventRecord((*evs)[2 * i + 1], st));
+        if (evs) SN_CUDA_TRY(cudaEventRecordWithFlags((*evs)[2 * i + 1], st, cudaEventRecordExternal));
     }
     return SN_OK;
 }
@@ -188,34 +189,68 @@ sn_status ensure(Graph *g, Buffer &b, size_t bytes) {
     return dev_alloc(g, bytes, &b);
 }
 
+// Capture the stream work `body` issues into a CUDA graph and instantiate it.
+template <class F>
+sn_status capture_graph(cudaStream_t st, F body, cudaGraphExec_t *exec) {
+    cudaGraph_t graph = nullptr;
+    SN_CUDA_TRY(cudaStreamBeginCapture(st, cudaStreamCaptureModeThreadLocal));
+    sn_status rc = body();
+    cudaError_t ce = cudaStreamEndCapture(st, &graph);
+    if (rc != SN_OK) {
+        if (graph) cudaGraphDestroy(graph);
+        return rc;
+    }
+    if (ce != cudaSuccess) return fail(SN_ECUDA, std::string("profiling capture: ") + cudaGetErrorString(ce));
+    ce = cudaGraphInstantiate(exec, graph, 0);
+    cudaGraphDestroy(graph);
+    if (ce != cudaSuccess) return fail(SN_ECUDA, std::string("profiling instantiate: ") + cudaGetErrorString(ce));
+    return SN_OK;
+}
+
+// Device time of one launch: `warm` eager launches (first-use set-up), then
+// `iters` back-to-back launches captured into a CUDA graph, replayed three
+// times; the median replay over iters.  Timing a replay rather than each
+// eager launch keeps the host's launch cost out of the figure (for a small
+// kernel it exceeds the kernel) and averages over the ~2 us resolution of
+// events; the launches overlap as they do in a replayed net.
 template <class F>
 sn_status time_median(int warm, int iters, cudaStream_t st, F launch, int64_t *ns_out) {
-    for (int i = 0; i < warm; ++i) {
+    for (int i = 0; i < std::max(warm, 1); ++i) {
         sn_status rc = launch();
         if (rc != SN_OK) return rc;
     }
-    std::vector<cudaEvent_t> ev(2 * iters);
-    for (auto &e : ev) SN_CUDA_TRY(cudaEventCreate(&e));
-    sn_status rc = SN_OK;
-    for (int i = 0; i < iters && rc == SN_OK; ++i) {
-        cudaEventRecord(ev[2 * i], st);
-        rc = launch();
-        cudaEventRecord(ev[2 * i + 1], st);
-    }
-    cudaError_t e = cudaStreamSynchronize(st);
-    std::vector<float> ms;
-    if (rc == SN_OK && e == cudaSuccess)
+    iters = std::max(iters, 1);
+    cudaGraphExec_t exec = nullptr;
+    sn_status rc = capture_graph(st, [&]() -> sn_status {
         for (int i = 0; i < iters; ++i) {
+            sn_status r = launch();
+            if (r != SN_OK) return r;
+        }
+        return SN_OK;
+    }, &exec);
+    if (rc != SN_OK) return rc;
+    constexpr int REPS = 3;
+    cudaEvent_t ev[REPS + 1];
+    for (auto &e : ev) SN_CUDA_TRY(cudaEventCreate(&e));
+    cudaError_t e = cudaGraphLaunch(exec, st);  // warm replay
+    for (int r = 0; r < REPS && e == cudaSuccess; ++r) {
+        if (r == 0) e = cudaEventRecord(ev[0], st);
+        if (e == cudaSuccess) e = cudaGraphLaunch(exec, st);
+        if (e == cudaSuccess) e = cudaEventRecord(ev[r + 1], st);
+    }
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    std::vector<float> ms;
+    if (e == cudaSuccess)
+        for (int r = 0; r < REPS; ++r) {
             float t = 0;
-            cudaEventElapsedTime(&t, ev[2 * i], ev[2 * i + 1]);
+            cudaEventElapsedTime(&t, ev[r], ev[r + 1]);
             ms.push_back(t);
         }
     for (auto &x : ev) cudaEventDestroy(x);
-    if (rc != SN_OK) return rc;
+    cudaGraphExecDestroy(exec);
     if (e != cudaSuccess) return fail(SN_ECUDA, std::string("profiling: ") + cudaGetErrorString(e));
     std::sort(ms.begin(), ms.end());
-    const double med = iters % 2 ? ms[iters / 2] : 0.5 * (ms[iters / 2 - 1] + ms[iters / 2]);
-    *ns_out = std::max<int64_t>(1, (int64_t)(med * 1e6 + 0.5));
+    *ns_out = std::max<int64_t>(1, (int64_t)(ms[REPS / 2] / iters * 1e6 + 0.5));
     return SN_OK;
 }
 
@@ -237,7 +272,47 @@ std::string signature(const Graph *g, int32_t i, const Candidate &c) {
 
 }  // namespace
 
-sn_status profile_graph(Graph *g, const sn_profile_opts &o, cudaStream_t st) {
+sn_status run_plan_timed(Graph *g, const void *in, void *out, cudaStream_t user, std::vector<float> *op_ms) {
+    if (!g->plan_valid) {
+        sn_status rc = build_plan(g, user);
+        if (rc != SN_OK) return rc;
+    }
+    SN_CUDA_TRY(cudaStreamSynchronize(user));
+    cudaStream_t st = nullptr;
+    SN_CUDA_TRY(cudaStreamCreateWithFlags(&st, cudaStreamNonBlocking));
+    std::vector<cudaEvent_t> evs(2 * g->plan.size());
+    for (auto &e : evs) cudaEventCreate(&e);
+    cudaGraphExec_t exec = nullptr;
+    sn_status rc = run_plan(g, in, out, st, nullptr);  // first-use set-up outside the capture
+    if (rc == SN_OK) rc = capture_graph(st, [&]() { return run_plan(g, in, out, st, &evs); }, &exec);
+    if (rc == SN_OK && cudaGraphLaunch(exec, st) != cudaSuccess) rc = fail(SN_ECUDA, "timed run: replay failed");
+    if (cudaStreamSynchronize(st) != cudaSuccess && rc == SN_OK) rc = fail(SN_ECUDA, "timed run: stream failed");
+    if (rc == SN_OK) {
+        op_ms->assign(g->plan.size(), 0.f);
+        for (size_t q = 0; q < g->plan.size(); ++q) cudaEventElapsedTime(&(*op_ms)[q], evs[2 * q], evs[2 * q + 1]);
+    }
+    if (exec) cudaGraphExecDestroy(exec);
+    for (auto &e : evs) cudaEventDestroy(e);
+    cudaStreamDestroy(st);
+    return rc;
+}
+
+static sn_status profile_graph_on(Graph *g, const sn_profile_opts &o, cudaStream_t st);
+
+// Profiling runs on a private stream (a CUDA graph cannot be captured on the
+// legacy default stream), after the caller's stream has drained.
+sn_status profile_graph(Graph *g, const sn_profile_opts &o, cudaStream_t user) {
+    SN_CUDA_TRY(cudaStreamSynchronize(user));
+    cudaStream_t st = nullptr;
+    SN_CUDA_TRY(cudaStreamCreateWithFlags(&st, cudaStreamNonBlocking));
+    const sn_status rc = profile_graph_on(g, o, st);
+    const cudaError_t e = cudaStreamSynchronize(st);
+    cudaStreamDestroy(st);
+    if (rc == SN_OK && e != cudaSuccess) return fail(SN_ECUDA, std::string("profiling: ") + cudaGetErrorString(e));
+    return rc;
+}
+
+static sn_status profile_graph_on(Graph *g, const sn_profile_opts &o, cudaStream_t st) {
     const int32_t n = g->n_layers(), ns = g->n_schemas();
     size_t max_bytes = 0;
     for (int32_t i = 0; i < n; ++i)
@@ -394,11 +469,17 @@ sn_status profile_graph(Graph *g, const sn_profile_opts &o, cudaStream_t st) {
             std::vector<cudaEvent_t> evs(2 * g->plan.size());
             for (auto &e : evs) cudaEventCreate(&e);
             std::vector<std::vector<float>> per_op(g->plan.size());
-            for (int32_t w = 0; w < o.warmup && rc == SN_OK; ++w)
+            for (int32_t w = 0; w < std::max(o.warmup, 1) && rc == SN_OK; ++w)
                 rc = run_plan(g, xin.ptr, xout.ptr, st, nullptr);
+            // the whole net with a timing node around every op, replayed
+            cudaGraphExec_t exec = nullptr;
+            if (rc == SN_OK)
+                rc = capture_graph(st, [&]() { return run_plan(g, xin.ptr, xout.ptr, st, &evs); }, &exec);
             for (int32_t p = 0; p < o.passes && rc == SN_OK; ++p) {
-                rc = run_plan(g, xin.ptr, xout.ptr, st, &evs);
-                if (rc != SN_OK) break;
+                if (cudaGraphLaunch(exec, st) != cudaSuccess) {
+                    rc = fail(SN_ECUDA, "integrated profiling: replay failed");
+                    break;
+                }
                 if (cudaStreamSynchronize(st) != cudaSuccess) {
                     rc = fail(SN_ECUDA, "integrated profiling: stream failed");
                     break;
@@ -409,6 +490,7 @@ sn_status profile_graph(Graph *g, const sn_profile_opts &o, cudaStream_t st) {
                     per_op[q].push_back(t);
                 }
             }
+            if (exec) cudaGraphExecDestroy(exec);
             for (auto &e : evs) cudaEventDestroy(e);
             if (rc != SN_OK) break;
             for (size_t q = 0; q < g->plan.size(); ++q) {
@@ -422,12 +504,28 @@ sn_status profile_graph(Graph *g, const sn_profile_opts &o, cudaStream_t st) {
     }
     dev_free(g, &xin);
     dev_free(g, &xout);
+    // in-situ medians replace the unit times of the re-timed candidates; the
+    // candidates of the same (layer, schema) that were not re-timed keep their
+    // unit ranking, moved to the in-situ scale by the best candidate's ratio
+    // (in-situ times carry the op's whole latency, unit times its share of a
+    // back-to-back replay, so mixing the two unscaled would favour the
+    // candidates that were not re-timed)
+    const std::vector<Candidate> unit = g->cands;
     for (size_t c = 0; c < insitu.size(); ++c) {
         if (insitu[c].empty()) continue;
         auto v = insitu[c];
         std::sort(v.begin(), v.end());
         g->cands[c].cost = std::max<int64_t>(1, (int64_t)(v[v.size() / 2] * 1e6 + 0.5));
     }
+    for (int32_t i = 1; i < n - 1; ++i)
+        for (int32_t lam = 0; lam < ns; ++lam) {
+            const auto &v = ranked[i][lam];
+            if (v.empty() || insitu[v[0]].empty() || unit[v[0]].cost <= 0 || unit[v[0]].cost == kInf) continue;
+            const double ratio = (double)g->cands[v[0]].cost / (double)unit[v[0]].cost;
+            for (int32_t c : v)
+                if (insitu[c].empty() && unit[c].cost != kInf)
+                    g->cands[c].cost = std::max<int64_t>(1, (int64_t)(unit[c].cost * ratio + 0.5));
+        }
     g->has_path = had_path;
     g->path_cand = saved_path;
     g->path_total = saved_total;

@@ -203,6 +203,9 @@ void fastest_per_schema(const Graph &g, std::vector<int64_t> &F, std::vector<int
 sn_status build_plan(Graph *g, cudaStream_t st);
 sn_status run_plan(Graph *g, const void *in, void *out, cudaStream_t st,
                    std::vector<cudaEvent_t> *evs);
+// one run of the plan replayed from a CUDA graph with a timing node around
+// every op (device time of each op, no host launch cost); op_ms[q] in ms
+sn_status run_plan_timed(Graph *g, const void *in, void *out, cudaStream_t st, std::vector<float> *op_ms);
 sn_status profile_graph(Graph *g, const sn_profile_opts &o, cudaStream_t st);
 
 // -------------------------------------------------------------------------
