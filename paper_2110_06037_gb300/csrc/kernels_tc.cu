@@ -20,7 +20,7 @@
 // one K-range of a tile when the layer is split along K because it has too
 // few tiles to fill the GPU), A-sharing tiles adjacent, with two TMEM
 // accumulators so that draining one overlaps the main loop of the next.
-// Warp roles (416 threads): warps 0 and 10-12 = TMA producers, each filling
+// Warp roles (384 threads): warps 0, 10 and 11 = TMA producers, each filling
 // every NPROD-th stage (warp 0 also allocates TMEM), warp 1 = MMA issuer (one
 // thread), warps 2-9 = epilogue, all eight draining each accumulator (four
 // row quarters x two column halves): TMEM ->
@@ -119,9 +119,11 @@ __global__ void __launch_bounds__(THREADS, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = tmem_sh;
-    // everything above overlaps the previous kernel's tail; global memory is
-    // touched only from here on
-    griddep_wait();
+    // Everything up to each role's griddep_wait() overlaps the previous
+    // kernel's tail: the producers wait before their first TMA load, the
+    // epilogue warps before their first residual load or store (the MMA warp
+    // touches no global memory); kernel parameters, bias and weights are not
+    // written by the previous kernel.
 
     constexpr int NPROD = producers_for(STAGES);
     const int prod = warp == 0 ? 0 : (warp >= 10 ? warp - 9 : -1);  // producer index of this warp
@@ -136,7 +138,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             const int brow = (int)rank * (BN / G);
             int g = 0, s = prod, issued = 0;
             uint32_t par = 0;
-            bool stop = false;
+            bool stop = false, waited = false;
             for (int u = cid; u < total && !stop; u += ncl) {
                 const Work w = work_of(p, u, BN, IMPLICIT, G, (int)rank);
                 const int steps_per_tap = cblocks / KB;
@@ -152,6 +154,10 @@ __global__ void __launch_bounds__(THREADS, 1)
                         if (abort_sh) {
                             stop = true;
                             break;
+                        }
+                        if (!waited) {
+                            griddep_wait();
+                            waited = true;
                         }
                         const uint32_t sa = su32(smem + s * STAGE_BYTES);
                         // KB = 1: channel coordinate cb * 64 on the innermost axis;
@@ -269,6 +275,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         const int cbase = ALT ? 0 : half * CPH;          // first chunk of this warp
         int lt = ALT ? half : 0;
         uint32_t rpar = 0;  // phase parity of this warp's residual barrier
+        bool waited = false;
         for (int u = cid + (ALT ? half * ncl : 0); u < total; u += (ALT ? 2 : 1) * ncl, lt += ALT ? 2 : 1) {
             const int b = lt & 1;
             const uint32_t aph = (uint32_t)(lt >> 1) & 1u;
@@ -302,6 +309,10 @@ __global__ void __launch_bounds__(THREADS, 1)
             // output store; zero outside the tensor) once the previous store has
             // read that block; the first chunk's load is issued before the
             // accumulator wait, the next one's after the current chunk's store
+            if (!waited) {
+                griddep_wait();
+                waited = true;
+            }
             const bool has_res = p.res != nullptr && p.ksplit == 1;
             auto issue_res = [&](int k0) {
                 if (!has_res || !tile_live || k0 >= p.K) return;
@@ -331,13 +342,13 @@ __global__ void __launch_bounds__(THREADS, 1)
                     // bias + activation -> 16-bit, staged with the 128-byte swizzle
                     // (row = lane, 16-byte chunk j at j ^ (row & 7)), then one TMA
                     // tensor store of the warp's 32 x 64 block, clipped at the edges
-                    uint32_t wv[32];
                     // this row's residual: 16-byte piece j of the row at j ^ (row & 7)
                     uint32_t rv[2][16];
 #pragma unroll
                     for (int h = 0; h < 2; ++h)
 #pragma unroll
                         for (int j = 0; j < 16; ++j) rv[h][j] = 0u;
+                    if (!has_res && lane == 0) bulk_wait_read_0();  // the previous store has read the block
                     if (has_res) {
                         if (!mbar_wait(&res_bar[warp - 2], rpar)) {
                             if (lane == 0) atomicOr(p.err, ERR_EPI_WAIT);
@@ -353,29 +364,30 @@ __global__ void __launch_bounds__(THREADS, 1)
                             rv[j >> 2][4 * (j & 3) + 3] = u.w;
                         }
                     }
+                    uint32_t v[64];
+                    __syncwarp();
+                    tmem_ld64(taddr, v);
+                    // every 4 packed pairs (8 channels) go to their 16-byte piece
+                    // of the row as soon as they are computed
 #pragma unroll
-                    for (int h = 0; h < 2; ++h) {
-                        uint32_t v[32];
-                        __syncwarp();
-                        tmem_ld32(taddr + 32 * h, v);
+                    for (int q = 0; q < 8; ++q) {
+                        const int h = q >> 2;
+                        uint32_t wq[4];
 #pragma unroll
-                        for (int j = 0; j < 16; ++j) {
+                        for (int e = 0; e < 4; ++e) {
+                            const int j = 4 * (q & 3) + e;  // pair index within the half
                             const float2 r2 = unpack2<T>(rv[h][j]);
-                            const float f0 = act_apply(
-                                __uint_as_float(v[2 * j]) + __shfl_sync(0xffffffffu, bias_r[cj][h], 2 * j) + r2.x,
-                                p.act);
-                            const float f1 = act_apply(__uint_as_float(v[2 * j + 1]) +
+                            const float f0 = act_apply(__uint_as_float(v[32 * h + 2 * j]) +
+                                                           __shfl_sync(0xffffffffu, bias_r[cj][h], 2 * j) + r2.x,
+                                                       p.act);
+                            const float f1 = act_apply(__uint_as_float(v[32 * h + 2 * j + 1]) +
                                                            __shfl_sync(0xffffffffu, bias_r[cj][h], 2 * j + 1) + r2.y,
                                                        p.act);
-                            wv[16 * h + j] = pack2<T>(f0, f1);
+                            wq[e] = pack2<T>(f0, f1);
                         }
+                        *reinterpret_cast<uint4 *>(buf + lane * 128 + ((q ^ (lane & 7)) << 4)) =
+                            make_uint4(wq[0], wq[1], wq[2], wq[3]);
                     }
-                    if (lane == 0) bulk_wait_read_0();  // the previous store has read the staging block
-                    __syncwarp();
-#pragma unroll
-                    for (int j = 0; j < 8; ++j)
-                        *reinterpret_cast<uint4 *>(buf + lane * 128 + ((j ^ (lane & 7)) << 4)) =
-                            make_uint4(wv[4 * j], wv[4 * j + 1], wv[4 * j + 2], wv[4 * j + 3]);
                     fence_proxy_async_smem();
                     __syncwarp();
                     if (lane == 0) {
@@ -418,7 +430,9 @@ __global__ void __launch_bounds__(THREADS, 1)
                     mbar_arrive(&acce_bar[b]);
             }
         }
-        if (lane == 0) bulk_wait_all();  // stores done before the CTA's shared memory is released
+        // the last stores have read their staging blocks before the CTA's shared
+        // memory is released (their global writes complete with the grid)
+        if (lane == 0) bulk_wait_read_0();
         __syncwarp();
     }
 
@@ -430,7 +444,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             // memory goes away (one deadline for the whole drain)
             const long long t0 = clock64();
             int issued = 0;
-            for (int i = 0; i < 4; ++i) issued = issued_sh[i] > issued ? issued_sh[i] : issued;
+            for (int i = 0; i < 3; ++i) issued = issued_sh[i] > issued ? issued_sh[i] : issued;
             for (int g = consumed_sh; g < issued; ++g)
                 while (!mbar_try(&full_bar[g % STAGES], (uint32_t)(g / STAGES) & 1u) && clock64() - t0 < WAIT_LIMIT) {
                 }

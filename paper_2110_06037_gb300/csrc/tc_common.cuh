@@ -13,10 +13,12 @@ namespace tc {
 
 constexpr int BM = 128;
 constexpr int BK = 64;
-constexpr int THREADS = 416;  // 13 warps: producer 0, MMA, 8 epilogue, producers 1-3
+// 12 warps: producer 0, MMA, 8 epilogue, producers 1-2.  Three warps per SM
+// sub-partition leave the epilogue up to 168 registers a thread.
+constexpr int THREADS = 384;
 // TMA producer threads for a ring of `stages` stages: one issuing thread
 // walks the stages s with s % n == its index, so n must divide the depth
-constexpr int producers_for(int stages) { return stages % 4 == 0 ? 4 : (stages % 3 == 0 ? 3 : 2); }
+constexpr int producers_for(int stages) { return stages % 3 == 0 ? 3 : 2; }
 // pipeline depth: as many stages of KB 64-channel blocks as fit beside the
 // epilogue staging (227 KB - 32 KB staging - 1 KB alignment slack)
 constexpr int stages_for(int bn, int g, int kb) {
@@ -229,6 +231,25 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
           "=r"(v[16]), "=r"(v[17]), "=r"(v[18]), "=r"(v[19]), "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]),
           "=r"(v[24]), "=r"(v[25]), "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31])
         : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+// 64 consecutive columns of the warp's 32 lanes, one wait for both halves
+__device__ __forceinline__ void tmem_ld64(uint32_t taddr, uint32_t (&v)[64]) {
+#define SN_LD32(OFF, B)                                                                                        \
+    asm volatile(                                                                                              \
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "                                                              \
+        "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "                              \
+        "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"              \
+        : "=r"(v[B + 0]), "=r"(v[B + 1]), "=r"(v[B + 2]), "=r"(v[B + 3]), "=r"(v[B + 4]), "=r"(v[B + 5]),      \
+          "=r"(v[B + 6]), "=r"(v[B + 7]), "=r"(v[B + 8]), "=r"(v[B + 9]), "=r"(v[B + 10]), "=r"(v[B + 11]),    \
+          "=r"(v[B + 12]), "=r"(v[B + 13]), "=r"(v[B + 14]), "=r"(v[B + 15]), "=r"(v[B + 16]), "=r"(v[B + 17]), \
+          "=r"(v[B + 18]), "=r"(v[B + 19]), "=r"(v[B + 20]), "=r"(v[B + 21]), "=r"(v[B + 22]), "=r"(v[B + 23]), \
+          "=r"(v[B + 24]), "=r"(v[B + 25]), "=r"(v[B + 26]), "=r"(v[B + 27]), "=r"(v[B + 28]), "=r"(v[B + 29]), \
+          "=r"(v[B + 30]), "=r"(v[B + 31])                                                                     \
+        : "r"(taddr + OFF))
+    SN_LD32(0, 0);
+    SN_LD32(32, 32);
+#undef SN_LD32
     asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
