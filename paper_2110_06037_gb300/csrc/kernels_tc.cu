@@ -141,10 +141,9 @@ __global__ void __launch_bounds__(THREADS, 1)
             bool stop = false, waited = false;
             for (int u = cid; u < total && !stop; u += ncl) {
                 const Work w = work_of(p, u, BN, IMPLICIT, G, (int)rank);
-                const int steps_per_tap = cblocks / KB;
-                int cb = (w.it0 % steps_per_tap) * KB;
-                int tap = w.it0 / steps_per_tap;
-                int r = tap / S, ss = tap - r * S;
+                int tap = (int)fdiv((uint32_t)w.it0, p.fd_spt);
+                int cb = (w.it0 - tap * p.fd_spt.d) * KB;
+                int r = (int)fdiv((uint32_t)tap, p.fd_S), ss = tap - r * S;
                 for (int it = w.it0; it < w.it1; ++it, ++g) {
                     if (g % NPROD == prod) {
                         if (!mbar_wait(&empty_bar[s], par ^ 1u)) {
@@ -266,9 +265,9 @@ __global__ void __launch_bounds__(THREADS, 1)
         const int row = g4 * 32 + lane;
         uint8_t *buf = stg + (warp - 2) * STG_BYTES;  // one 32 x 64 staging block per warp
         const int r0 = g4 * 32;
-        const int wq0 = IMPLICIT ? r0 % p.BW : 0;
-        const int hp0 = IMPLICIT ? (r0 / p.BW) % p.BH : 0;
-        const int ni0 = IMPLICIT ? r0 / (p.BW * p.BH) : 0;
+        const int wq0 = IMPLICIT ? r0 & (p.BW - 1) : 0;
+        const int hp0 = IMPLICIT ? (r0 >> p.lbw) & (p.BH - 1) : 0;
+        const int ni0 = IMPLICIT ? r0 >> p.lbwh : 0;
         constexpr int NCH = BN / 64 > 0 ? BN / 64 : 1;  // 64-channel chunks per tile
         constexpr int CPH = NCH >= 2 ? NCH / 2 : 1;      // chunks per column half
         constexpr bool ALT = NCH == 1;                   // alternate units between the groups
@@ -294,7 +293,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             bool valid;
             int64_t pix;
             if (IMPLICIT) {
-                const int wq = row % p.BW, hp = (row / p.BW) % p.BH, ni = row / (p.BW * p.BH);
+                const int wq = row & (p.BW - 1), hp = (row >> p.lbw) & (p.BH - 1), ni = row >> p.lbwh;
                 const int q = w.q0 + wq, pp = w.p0 + hp, n = w.i0 + ni;
                 valid = q < p.Q && pp < p.P && n < p.N;
                 pix = ((int64_t)n * p.P + pp) * p.Q + q;
@@ -810,6 +809,18 @@ cudaError_t conv_tc(const LaunchArgs &a) {
             return cudaErrorInvalidValue;
     }
     if (p.mtiles <= 0 || (int64_t)p.mtiles * p.ntiles * p.ksplit > INT32_MAX) return cudaErrorInvalidValue;
+    if ((int64_t)(p.ksplit + 1) * p.kiters > INT32_MAX) return cudaErrorInvalidValue;
+    p.fd_ksplit = make_fastdiv((uint32_t)p.ksplit);
+    p.fd_ntiles = make_fastdiv((uint32_t)p.ntiles);
+    p.fd_tq = make_fastdiv((uint32_t)std::max(p.tq, 1));
+    p.fd_tp = make_fastdiv((uint32_t)std::max(p.tp, 1));
+    p.fd_spt = make_fastdiv((uint32_t)(p.cblocks / cf.KB));
+    p.fd_S = make_fastdiv((uint32_t)p.S);
+    p.lbw = p.lbwh = 0;
+    if (cf.implicit) {
+        while ((1 << p.lbw) < cf.BW) ++p.lbw;
+        while ((1 << p.lbwh) < cf.BW * cf.BH) ++p.lbwh;
+    }
     const bool bf = dt == SN_BF16;
 #define SN_TC_LAUNCH(TT, BNV, GV, KBV)                                                            \
     return cf.implicit ? launch<TT, BNV, true, GV, KBV>(mA, mB, mY, mR, p, a.stream)               \

@@ -30,12 +30,32 @@ constexpr uint32_t STG_BYTES = 32 * 64 * 2;      // one epilogue staging block: 
 constexpr long long WAIT_LIMIT = 4000000000LL;  // SM cycles (~2 s)
 enum : int { ERR_TMA_WAIT = 0x10, ERR_MMA_WAIT = 0x20, ERR_ACC_WAIT = 0x40, ERR_EPI_WAIT = 0x80 };
 
+// Division by a divisor fixed at launch, for numerators below 2^31:
+// q = (umulhi(n, m) + n) >> l with l = ceil(log2 d), m = floor(2^32 (2^l - d) / d) + 1
+// (the round-up multiplier method of Granlund and Montgomery).  A single
+// issuing thread's prologue runs a few of these; the generic 32-bit division
+// is a dependent chain of ~20 instructions, 64-bit division a library call.
+struct FastDiv {
+    uint32_t d, m, l;
+};
+inline FastDiv make_fastdiv(uint32_t d) {
+    uint32_t l = 0;
+    while ((1ull << l) < d) ++l;
+    const uint64_t m = ((1ull << 32) * ((1ull << l) - d)) / d + 1;
+    return FastDiv{d, (uint32_t)m, l};
+}
+__device__ __forceinline__ uint32_t fdiv(uint32_t n, const FastDiv &f) {
+    return (uint32_t)(((uint64_t)__umulhi(n, f.m) + n) >> f.l);
+}
+
 struct Params {
     int32_t N, H, W, C, K, P, Q, R, S;
     int32_t stride, ph, pw, dh, dw;
     int32_t cblocks, kiters, ksplit;  // 64-channel blocks; K steps (of KB blocks) per tile; K split
     int32_t BW, BH, BNI, tq, tp;   // pixel-tile geometry (implicit mode)
     int32_t mtiles, ntiles;
+    FastDiv fd_ksplit, fd_ntiles, fd_tq, fd_tp, fd_spt, fd_S;  // spt: K steps per filter tap
+    int32_t lbw, lbwh;             // log2 BW, log2 (BW * BH): the tile geometry is powers of two
     int64_t M;                     // plain mode: input rows (= output pixels)
     int64_t Mout;                  // output pixels N * P * Q
     int32_t act;
@@ -334,9 +354,9 @@ struct Work {
 __device__ __forceinline__ Work work_of(const Params &p, int u, int bn, bool implicit, int ctas = 1,
                                         int rank = 0) {
     Work w;
-    w.sp = u % p.ksplit;
-    const int t = u / p.ksplit;
-    const int mg = t / p.ntiles, nt = t - mg * p.ntiles;
+    const int t = (int)fdiv((uint32_t)u, p.fd_ksplit);
+    w.sp = u - t * p.ksplit;
+    const int mg = (int)fdiv((uint32_t)t, p.fd_ntiles), nt = t - mg * p.ntiles;
     const int mt = mg * ctas + rank;
     w.mt = mt;
     w.n0 = nt * bn;
@@ -344,18 +364,20 @@ __device__ __forceinline__ Work work_of(const Params &p, int u, int bn, bool imp
     w.q0 = w.p0 = w.i0 = 0;
     if (implicit) {
         int bx = mt;
-        const int bq = bx % p.tq;
-        bx /= p.tq;
-        const int bp = bx % p.tp;
-        bx /= p.tp;
+        int nb = (int)fdiv((uint32_t)bx, p.fd_tq);
+        const int bq = bx - nb * p.tq;
+        bx = nb;
+        nb = (int)fdiv((uint32_t)bx, p.fd_tp);
+        const int bp = bx - nb * p.tp;
+        bx = nb;
         w.q0 = bq * p.BW;
         w.p0 = bp * p.BH;
         w.i0 = bx * p.BNI;
     } else {
         w.m0 = (int64_t)mt * BM;
     }
-    w.it0 = (int)((int64_t)w.sp * p.kiters / p.ksplit);
-    w.it1 = (int)((int64_t)(w.sp + 1) * p.kiters / p.ksplit);
+    w.it0 = (int)fdiv((uint32_t)(w.sp * p.kiters), p.fd_ksplit);
+    w.it1 = (int)fdiv((uint32_t)((w.sp + 1) * p.kiters), p.fd_ksplit);
     return w;
 }
 
