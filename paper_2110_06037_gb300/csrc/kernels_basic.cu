@@ -215,8 +215,9 @@ __global__ void weight_perm_kernel(const float *__restrict__ w, T *__restrict__ 
         if (fmt == W_KCRS) o = i;
         else if (fmt == W_RSCK) o = ((r * S + s) * Cg + c) * K + kk;
         else if (fmt == W_KRSC_PAD64) o = kk * ((Cg * R * S + 63) / 64 * 64) + (r * S + s) * Cg + c;
-        else if (fmt == W_S2D)  // [K][ceil(R/2)][4 pixels][16]: tap (r, s) -> row r/2, pixel s/2, slot (2(r%2)+s%2)Cg+c
-            o = (kk * ((R + 1) / 2) + r / 2) * 64 + (s / 2) * 16 + ((r % 2) * 2 + s % 2) * Cg + c;
+        else if (fmt == W_S2D)  // [K][A][4 pixels][16], A = 2 (R <= 4) or 4 tap rows (the rest zero):
+            // tap (r, s) -> row r/2, pixel s/2, slot (2(r%2)+s%2)Cg+c
+            o = (kk * (R <= 4 ? 2 : 4) + r / 2) * 64 + (s / 2) * 16 + ((r % 2) * 2 + s % 2) * Cg + c;
         else o = ((kk * R + r) * S + s) * Cg + c;  // W_KRSC
         stf<T>(out + o, w[i]);
     }
@@ -262,7 +263,7 @@ cudaError_t weight_format(const float *w, void *out, int fmt, int dt, int64_t K,
     }
     if (fmt == W_S2D) {  // taps outside the kernel and channels past 4 Cg are zero
         if (R > 8 || S > 8 || 4 * Cg > 16) return cudaErrorInvalidValue;
-        cudaError_t e = cudaMemsetAsync(out, 0, (size_t)K * ((R + 1) / 2) * 64 * dtype_size(dt), st);
+        cudaError_t e = cudaMemsetAsync(out, 0, (size_t)K * (R <= 4 ? 2 : 4) * 64 * dtype_size(dt), st);
         if (e != cudaSuccess) return e;
     }
     SN_DT_SWITCH(dt, T,

@@ -549,7 +549,10 @@ struct Config {
 constexpr int kSmCount = 152;  // GB300; only used to decide which K splits to offer
 
 // deterministic list of routine-parameter combinations for a layer
-static std::vector<Config> configs(const Layer &l, const Shape &in, sn_schema s) {
+// a_blocks > 0: the space-to-depth formulation (a 1x1 layer of a_blocks x 64
+// "channels" over a caller-laid-out A): implicit tiles only, BN = 64, one
+// CTA per tile, all a_blocks blocks in one stage
+static std::vector<Config> configs(const Layer &l, const Shape &in, sn_schema s, int a_blocks = 0) {
     std::vector<Config> out;
     const sn_conv_params &c = l.conv;
     if (l.type != SN_L_CONV2 || c.groups != 1) return out;
@@ -598,7 +601,7 @@ static std::vector<Config> configs(const Layer &l, const Shape &in, sn_schema s)
                 cf.KB = 1;
             }
     };
-    if (plain) {
+    if (plain && a_blocks == 0) {
         push_all({false, 0, 0, 0, 0, 1, 1, 1}, (N * P * Q + BM - 1) / BM);
         return out;
     }
@@ -622,7 +625,10 @@ static std::vector<Config> configs(const Layer &l, const Shape &in, sn_schema s)
     for (int gi = 0; gi < keep; ++gi) {
         const Geo &gg = gs[gi];
         const int64_t mtiles = ((Q + gg.bw - 1) / gg.bw) * ((P + gg.bh - 1) / gg.bh) * ((N + gg.bni - 1) / gg.bni);
-        push_all({true, 0, gg.bw, gg.bh, gg.bni, 1, 1, 1}, mtiles);
+        if (a_blocks > 0)
+            out.push_back({true, 64, gg.bw, gg.bh, gg.bni, 1, 1, a_blocks});
+        else
+            push_all({true, 0, gg.bw, gg.bh, gg.bni, 1, 1, 1}, mtiles);
     }
     return out;
 }
@@ -696,8 +702,8 @@ int32_t conv_tc_variants(const Layer &l, const Shape &in, sn_schema s) {
     return (int32_t)tc::configs(l, in, s).size();
 }
 
-size_t conv_tc_ws(const Layer &l, const Shape &in, sn_schema s, int32_t v) {
-    const std::vector<tc::Config> cfgs = tc::configs(l, in, s);
+size_t conv_tc_ws(const Layer &l, const Shape &in, sn_schema s, int32_t v, int32_t a_blocks) {
+    const std::vector<tc::Config> cfgs = tc::configs(l, in, s, a_blocks);
     if (v < 0 || v >= (int)cfgs.size() || cfgs[v].ksplit == 1) return 0;
     return (size_t)cfgs[v].ksplit * l.out.n * l.out.h * l.out.w * l.conv.c_out * sizeof(float);
 }
@@ -712,7 +718,7 @@ cudaError_t conv_tc(const LaunchArgs &a) {
     using namespace tc;
     const Layer &l = *a.layer;
     const Shape &in = a.in_shapes[0];
-    const std::vector<Config> cfgs = configs(l, in, a.schema);
+    const std::vector<Config> cfgs = configs(l, in, a.schema, a.a_blocks);
     if (a.variant < 0 || a.variant >= (int)cfgs.size()) return cudaErrorInvalidValue;
     const Config cf = cfgs[a.variant];
     const sn_conv_params &c = l.conv;
@@ -777,10 +783,8 @@ cudaError_t conv_tc(const LaunchArgs &a) {
         if (p.stride == 1) {
             const uint64_t dims[5] = {c0dim, (uint64_t)p.W, (uint64_t)p.H, (uint64_t)p.N, CB};
             uint64_t str[4] = {p.C * es, (uint64_t)p.W * p.C * es, (uint64_t)p.H * p.W * p.C * es, 128};
-            if (a.a_strides[0] > 0) {  // a caller-laid-out A (overlapping pixel rows)
-                if (blk) return cudaErrorInvalidValue;
-                for (int i = 0; i < 3; ++i) str[i] = (uint64_t)a.a_strides[i];
-            }
+            if (a.a_strides[0] > 0)  // a caller-laid-out A (overlapping pixel rows)
+                for (int i = 0; i < 4; ++i) str[i] = (uint64_t)a.a_strides[i];
             if (!encode(&mA[0], dt, blk ? 5 : 4, a.in[0], dims, str, box)) return cudaErrorInvalidValue;
             mA[1] = mA[2] = mA[3] = mA[0];
         } else {
@@ -826,6 +830,12 @@ cudaError_t conv_tc(const LaunchArgs &a) {
     return cf.implicit ? launch<TT, BNV, true, GV, KBV>(mA, mB, mY, mR, p, a.stream)               \
                        : launch<TT, BNV, false, GV, KBV>(mA, mB, mY, mR, p, a.stream)
 #define SN_TC_LAUNCH_T(TT)                                                                          \
+    if (cf.G == 1 && cf.KB > 1) {                                                                   \
+        if (!cf.implicit || cf.BN != 64) return cudaErrorInvalidValue;                              \
+        if (cf.KB == 2) return launch<TT, 64, true, 1, 2>(mA, mB, mY, mR, p, a.stream);            \
+        if (cf.KB == 4) return launch<TT, 64, true, 1, 4>(mA, mB, mY, mR, p, a.stream);            \
+        return cudaErrorInvalidValue;                                                               \
+    }                                                                                               \
     if (cf.G == 2) {                                                                                \
         if (cf.KB == 2) {                                                                           \
             if (cf.BN == 128) SN_TC_LAUNCH(TT, 128, 2, 2);                                          \
@@ -1010,8 +1020,11 @@ cudaError_t conv_im2col_tc(const LaunchArgs &a) {
 // one row of taps a multiplies for output pixel (p, q) are X[p + a][q .. q+3],
 // contiguous: the GEMM's A row is one 128-byte window of X whose start moves
 // by one 32-byte pixel per output pixel.  The tensor map over X says exactly
-// that (pixel stride 32 B, rows of 64 values), so the implicit-GEMM kernel
-// runs unchanged with ceil(kh/2) K steps of 64.
+// that (pixel stride 32 B, rows of 64 values), with a fifth axis over the
+// rows of taps (stride one X row), so one TMA box brings all A = 2 or 4 rows
+// of taps of a 128-pixel tile (A x 16 KB) and the implicit-GEMM kernel runs
+// one pipeline stage per tile: a TMA box costs about the same whatever its
+// size, so few large boxes keep the tensor cores fed.
 // ---------------------------------------------------------------------------
 namespace {
 struct S2dDims {
@@ -1026,32 +1039,36 @@ static bool s2d_applies(const Layer &l, sn_schema s) {
            s.layout == SN_NHWC;
 }
 
-// the stride-1 layer the GEMM computes, and its input (X: Pp x Qp pixels of 64
-// "channels", the window)
+// rows of taps A = ceil(kh/2) rounded up to 2 or 4 (zero weights beyond kh);
+// all A rows, 64 values each, are one TMA box and one pipeline stage
+static int s2d_rows(const Layer &l) { return l.conv.kh <= 4 ? 2 : 4; }
+
+// the GEMM as a 1x1 layer of A x 64 "channels" over the P x Q output pixels:
+// "channel" block a of pixel (p, q) is X[p + a][q .. q + 3]
 static Layer s2d_gemm_layer(const Layer &l) {
     Layer g;
     g.type = SN_L_CONV2;
-    g.conv = sn_conv_params{64, l.conv.c_out, (l.conv.kh + 1) / 2, 1, 1, 1, 0, 0, 1, 1, 1, l.conv.act};
+    g.conv = sn_conv_params{64 * s2d_rows(l), l.conv.c_out, 1, 1, 1, 1, 0, 0, 1, 1, 1, l.conv.act};
     g.act = l.conv.act;
     g.out = l.out;
     return g;
 }
-static Shape s2d_gemm_in(const Layer &l) { return Shape{l.out.n, 64, l.out.h + (l.conv.kh + 1) / 2 - 1, l.out.w}; }
+static Shape s2d_gemm_in(const Layer &l) { return Shape{l.out.n, 64 * s2d_rows(l), l.out.h, l.out.w}; }
 
 static size_t s2d_bytes(const Layer &l, sn_schema s) {
-    const int64_t Pp = l.out.h + (l.conv.kh + 1) / 2 - 1, Qp = l.out.w + 3;
+    const int64_t Pp = l.out.h + s2d_rows(l) - 1, Qp = l.out.w + 3;
     return ((size_t)l.out.n * Pp * Qp * 16 * dtype_size(s.dtype) + 255) & ~size_t(255);
 }
 
 int32_t conv_s2d_tc_variants(const Layer &l, const Shape &in, sn_schema s) {
     (void)in;
     if (!s2d_applies(l, s)) return 0;
-    return (int32_t)tc::configs(s2d_gemm_layer(l), s2d_gemm_in(l), s).size();
+    return (int32_t)tc::configs(s2d_gemm_layer(l), s2d_gemm_in(l), s, s2d_rows(l)).size();
 }
 
 size_t conv_s2d_tc_ws(const Layer &l, const Shape &in, sn_schema s, int32_t v) {
     (void)in;
-    return s2d_bytes(l, s) + conv_tc_ws(s2d_gemm_layer(l), s2d_gemm_in(l), s, v);
+    return s2d_bytes(l, s) + conv_tc_ws(s2d_gemm_layer(l), s2d_gemm_in(l), s, v, s2d_rows(l));
 }
 
 // X[n][u][v][16]: one thread per X pixel, two 16-byte stores
@@ -1084,7 +1101,7 @@ cudaError_t conv_s2d_tc(const LaunchArgs &a) {
     const Shape &in = a.in_shapes[0];
     const Shape gin = s2d_gemm_in(l);
     S2dDims d{(int32_t)in.n, (int32_t)in.h, (int32_t)in.w, (int32_t)in.c, l.conv.ph, l.conv.pw,
-              (int32_t)gin.h, (int32_t)(l.out.w + 3)};
+              (int32_t)(l.out.h + s2d_rows(l) - 1), (int32_t)(l.out.w + 3)};
     const size_t xb = s2d_bytes(l, a.schema);
     if (!a.ws || a.ws_bytes < xb || (uintptr_t)a.ws % 256) return cudaErrorInvalidValue;
     const int64_t total = (int64_t)d.N * d.Pp * d.Qp;
@@ -1099,9 +1116,11 @@ cudaError_t conv_s2d_tc(const LaunchArgs &a) {
     g.in_shapes = {gin};
     g.in[0] = a.ws;
     const int64_t pix = 16 * (int64_t)dtype_size(a.schema.dtype);  // 32 bytes: one X pixel
-    g.a_strides[0] = pix;
-    g.a_strides[1] = pix * d.Qp;
-    g.a_strides[2] = pix * d.Qp * d.Pp;
+    g.a_strides[0] = pix;                   // next output column: next window
+    g.a_strides[1] = pix * d.Qp;            // next output row
+    g.a_strides[2] = pix * d.Qp * d.Pp;     // next image
+    g.a_strides[3] = pix * d.Qp;            // next row of taps: one X row down
+    g.a_blocks = s2d_rows(l);
     g.ws = static_cast<uint8_t *>(a.ws) + xb;
     g.ws_bytes = a.ws_bytes - xb;
     return conv_tc(g);

@@ -148,7 +148,7 @@ sn_status prepare_weights(Graph *g, int32_t li, int32_t r, int32_t v, sn_schema 
     }
     const int64_t elems = (fmt == k::W_WINO)         ? 16 * K * Cg
                           : (fmt == k::W_KRSC_PAD64) ? K * ((Cg * R * S + 63) / 64 * 64)
-                          : (fmt == k::W_S2D)        ? K * ((R + 1) / 2) * 64
+                          : (fmt == k::W_S2D)        ? K * (R <= 4 ? 2 : 4) * 64
                                                      : K * Cg * R * S;
     Buffer src, dst;
     sn_status rc = dev_alloc(g, (size_t)K * Cg * R * S * sizeof(float), &src);

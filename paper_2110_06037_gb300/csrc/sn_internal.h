@@ -121,9 +121,13 @@ struct LaunchArgs {
     void *ws = nullptr;         // workspace
     size_t ws_bytes = 0;
     // tensor-core implicit GEMM only: byte strides of the A tensor's pixel,
-    // row and image axes when they differ from dense NHWC (0 = dense); a pixel
-    // stride below the 128-byte row makes consecutive pixels' rows overlap
-    int64_t a_strides[3] = {0, 0, 0};
+    // row, image and 64-value-block axes when they differ from dense NHWC
+    // (0 = dense); a pixel stride below the 128-byte row makes consecutive
+    // pixels' rows overlap
+    int64_t a_strides[4] = {0, 0, 0, 0};
+    // tensor-core implicit GEMM only: > 0 when the layer's "channels" are
+    // a_blocks blocks of 64 read as one box (the space-to-depth stem's taps)
+    int32_t a_blocks = 0;
     cudaStream_t stream = nullptr;
 };
 
@@ -227,7 +231,7 @@ cudaError_t conv_wino(const LaunchArgs &a);
 size_t conv_wino_ws(const Layer &l, const Shape &in, sn_schema s);
 cudaError_t conv_tc(const LaunchArgs &a);
 int32_t conv_tc_variants(const Layer &l, const Shape &in, sn_schema s);
-size_t conv_tc_ws(const Layer &l, const Shape &in, sn_schema s, int32_t v);  // K-split partial sums
+size_t conv_tc_ws(const Layer &l, const Shape &in, sn_schema s, int32_t v, int32_t a_blocks = 0);  // K-split partials
 size_t dense_tc_ws(const Layer &l, const Shape &in, sn_schema s, int32_t v);
 const char *conv_tc_variant_name(int32_t v);
 // im2col childnet and dense childnet on the tensor-core GEMM
