@@ -73,6 +73,24 @@ inline cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, siz
     return cudaLaunchKernelEx(&cfg, kern, args...);
 }
 
+// Division by a divisor fixed at launch, for numerators below 2^31:
+// q = (umulhi(n, m) + n) >> l with l = ceil(log2 d), m = floor(2^32 (2^l - d) / d) + 1
+// (the round-up multiplier method of Granlund and Montgomery).  The generic
+// 32-bit division is a dependent chain of ~20 instructions, 64-bit division a
+// library call.
+struct FastDiv {
+    uint32_t d, m, l;
+};
+inline FastDiv make_fastdiv(uint32_t d) {
+    uint32_t l = 0;
+    while ((1ull << l) < d) ++l;
+    const uint64_t m = ((1ull << 32) * ((1ull << l) - d)) / d + 1;
+    return FastDiv{d, (uint32_t)m, l};
+}
+__device__ __forceinline__ uint32_t fdiv(uint32_t n, const FastDiv &f) {
+    return (uint32_t)(((uint64_t)__umulhi(n, f.m) + n) >> f.l);
+}
+
 #define SN_DT_SWITCH(dt, T, ...)                          \
     switch (dt) {                                         \
     case SN_F32: { using T = float; __VA_ARGS__; break; } \

@@ -387,34 +387,38 @@ __global__ void dw_nhwc(const T *__restrict__ x, const T *__restrict__ w, const 
 // columns: each input vector a thread needs for its QB outputs is loaded from
 // global once per (tap row, column) and reused through L1 by its neighbours;
 // weights are [R][S][C].
+// One thread: QB consecutive output columns x E channels (16 bytes) of one
+// output row.  The grid's y axis walks the N x P output rows, its x axis the
+// (column block, channel vector) pairs of a row with the channel vector
+// fastest (coalesced 16-byte accesses); all index math is 32-bit, one
+// division per thread (64-bit division and modulo by runtime values cost
+// more than the arithmetic of the taps).
 template <typename T, int QB, int SW>  // SW = 1 or 2: 3x3 fast path for that stride; 0 = any
-__global__ void __launch_bounds__(256, QB >= 4 ? 2 : 3) dw_nhwc_vec(const T *__restrict__ x, const T *__restrict__ w,
-                                                   const float *__restrict__ bias, T *__restrict__ y, ConvDims d) {
+__global__ void __launch_bounds__(256, 2) dw_nhwc_vec(const T *__restrict__ x, const T *__restrict__ w,
+                                                      const float *__restrict__ bias, T *__restrict__ y, ConvDims d,
+                                                      int CV, int QBLK) {
     griddep_launch();
     griddep_wait();
     constexpr int E = 16 / sizeof(T);
-    const int CV = d.C / E;
-    const int QBLK = (d.Q + QB - 1) / QB;
-    const int64_t total = (int64_t)d.N * d.P * QBLK * CV;
-    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total;
-         i += (int64_t)gridDim.x * blockDim.x) {
-        const int cv = (int)(i % CV);
-        int64_t rest = i / CV;
-        const int qb = (int)(rest % QBLK);
-        rest /= QBLK;
-        const int p = (int)(rest % d.P);
-        const int64_t n = rest / d.P;
-        const int c0 = cv * E, q0 = qb * QB;
+    const int t = blockIdx.x * blockDim.x + threadIdx.x;
+    if (t >= QBLK * CV) return;
+    const int qb = t / CV, cv = t - qb * CV;
+    const int c0 = cv * E, q0 = qb * QB;
+    float b[E];
+    {
+        const float4 b0 = *reinterpret_cast<const float4 *>(bias + c0);
+        const float4 b1 = *reinterpret_cast<const float4 *>(bias + c0 + 4);
+        const float bb[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
+#pragma unroll
+        for (int e = 0; e < E; ++e) b[e] = bb[e];
+    }
+    for (int rowi = blockIdx.y; rowi < d.N * d.P; rowi += gridDim.y) {
+        const int n = rowi / d.P, p = rowi - n * d.P;
         float acc[QB][E];
-        {
-            float b[E];
 #pragma unroll
-            for (int e = 0; e < E; ++e) b[e] = bias[c0 + e];
+        for (int j = 0; j < QB; ++j)
 #pragma unroll
-            for (int j = 0; j < QB; ++j)
-#pragma unroll
-                for (int e = 0; e < E; ++e) acc[j][e] = b[e];
-        }
+            for (int e = 0; e < E; ++e) acc[j][e] = b[e];
         if (SW > 0) {
             // 3x3 fast path: the input window of each tap row (QB outputs need
             // (QB-1)*SW + 3 columns) is loaded once and reused by the three taps
@@ -424,7 +428,7 @@ __global__ void __launch_bounds__(256, QB >= 4 ? 2 : 3) dw_nhwc_vec(const T *__r
             for (int r = 0; r < 3; ++r) {
                 const int h = p * d.sh - d.ph + r * d.dh;
                 if (h < 0 || h >= d.H) continue;
-                const T *xrow = x + ((n * d.H + h) * (int64_t)d.W) * d.C + c0;
+                const T *xrow = x + (((int64_t)n * d.H + h) * d.W) * d.C + c0;
                 uint4 win[WN];
 #pragma unroll
                 for (int t = 0; t < WN; ++t) {
@@ -451,7 +455,7 @@ __global__ void __launch_bounds__(256, QB >= 4 ? 2 : 3) dw_nhwc_vec(const T *__r
             for (int r = 0; r < d.R; ++r) {
                 const int h = p * d.sh - d.ph + r * d.dh;
                 if (h < 0 || h >= d.H) continue;
-                const T *xrow = x + ((n * d.H + h) * (int64_t)d.W) * d.C + c0;
+                const T *xrow = x + (((int64_t)n * d.H + h) * d.W) * d.C + c0;
                 for (int s = 0; s < d.S; ++s) {
                     const uint4 wq = *reinterpret_cast<const uint4 *>(w + (int64_t)(r * d.S + s) * d.C + c0);
                     const T *wp = reinterpret_cast<const T *>(&wq);
@@ -471,7 +475,7 @@ __global__ void __launch_bounds__(256, QB >= 4 ? 2 : 3) dw_nhwc_vec(const T *__r
                 }
             }
         }
-        T *yrow = y + ((n * d.P + p) * (int64_t)d.Q) * d.C + c0;
+        T *yrow = y + ((int64_t)rowi * d.Q) * d.C + c0;
 #pragma unroll
         for (int j = 0; j < QB; ++j) {
             if (q0 + j >= d.Q) break;
@@ -728,10 +732,11 @@ cudaError_t dwconv(const LaunchArgs &a) {
                 if (d.sw == 1) launch_pdl(dw3_nhwc_halo<T, 1, 4>, gb, 256, sm1, a.stream, x, w, a.bias, y, d);
                 else launch_pdl(dw3_nhwc_halo<T, 2, 3>, gb, 256, sm2, a.stream, x, w, a.bias, y, d);
             } else {
-                const unsigned gb = grid_for((int64_t)d.N * d.P * ((d.Q + 3) / 4) * cvec, 256, 152LL * 16);
-                if (k3 && d.sw == 1) launch_pdl(dw_nhwc_vec<T, 4, 1>, gb, 256, 0, a.stream, x, w, a.bias, y, d);
-                else if (k3 && d.sw == 2) launch_pdl(dw_nhwc_vec<T, 4, 2>, gb, 256, 0, a.stream, x, w, a.bias, y, d);
-                else launch_pdl(dw_nhwc_vec<T, 4, 0>, gb, 256, 0, a.stream, x, w, a.bias, y, d);
+                const int QBLK = (d.Q + 3) / 4, CV = (int)cvec;
+                const dim3 gb((unsigned)((QBLK * CV + 255) / 256), (unsigned)std::min<int64_t>((int64_t)d.N * d.P, 65535));
+                if (k3 && d.sw == 1) launch_pdl(dw_nhwc_vec<T, 4, 1>, gb, 256, 0, a.stream, x, w, a.bias, y, d, CV, QBLK);
+                else if (k3 && d.sw == 2) launch_pdl(dw_nhwc_vec<T, 4, 2>, gb, 256, 0, a.stream, x, w, a.bias, y, d, CV, QBLK);
+                else launch_pdl(dw_nhwc_vec<T, 4, 0>, gb, 256, 0, a.stream, x, w, a.bias, y, d, CV, QBLK);
             }
         } else if (a.schema.layout == SN_NHWC) {
             launch_pdl(dw_nhwc<T>, grid_for(total, 256), 256, 0, a.stream, x, w, a.bias, y, d);

@@ -30,24 +30,6 @@ constexpr uint32_t STG_BYTES = 32 * 64 * 2;      // one epilogue staging block: 
 constexpr long long WAIT_LIMIT = 4000000000LL;  // SM cycles (~2 s)
 enum : int { ERR_TMA_WAIT = 0x10, ERR_MMA_WAIT = 0x20, ERR_ACC_WAIT = 0x40, ERR_EPI_WAIT = 0x80 };
 
-// Division by a divisor fixed at launch, for numerators below 2^31:
-// q = (umulhi(n, m) + n) >> l with l = ceil(log2 d), m = floor(2^32 (2^l - d) / d) + 1
-// (the round-up multiplier method of Granlund and Montgomery).  A single
-// issuing thread's prologue runs a few of these; the generic 32-bit division
-// is a dependent chain of ~20 instructions, 64-bit division a library call.
-struct FastDiv {
-    uint32_t d, m, l;
-};
-inline FastDiv make_fastdiv(uint32_t d) {
-    uint32_t l = 0;
-    while ((1ull << l) < d) ++l;
-    const uint64_t m = ((1ull << 32) * ((1ull << l) - d)) / d + 1;
-    return FastDiv{d, (uint32_t)m, l};
-}
-__device__ __forceinline__ uint32_t fdiv(uint32_t n, const FastDiv &f) {
-    return (uint32_t)(((uint64_t)__umulhi(n, f.m) + n) >> f.l);
-}
-
 struct Params {
     int32_t N, H, W, C, K, P, Q, R, S;
     int32_t stride, ph, pw, dh, dw;
