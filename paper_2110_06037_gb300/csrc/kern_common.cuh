@@ -40,6 +40,17 @@ __device__ __forceinline__ float act_apply(float v, int act) {
     return v;
 }
 
+// streaming multiprocessors of the current device (host)
+inline int num_sms() {
+    static int n = 0;
+    if (!n) {
+        int dev = 0;
+        cudaGetDevice(&dev);
+        if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 1;
+    }
+    return n;
+}
+
 inline unsigned grid_for(int64_t n, int block, int64_t cap = 152LL * 64) {
     int64_t g = (n + block - 1) / block;
     if (g > cap) g = cap;
@@ -73,6 +84,27 @@ inline cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, siz
     return cudaLaunchKernelEx(&cfg, kern, args...);
 }
 
+// acc += x * w on the two 16-bit lanes of x2 and w2, accumulating in f32 with
+// the sm_100 mixed-precision FMA (fp32 destination, f16/bf16 factors).  The
+// product of two f16 or two bf16 values is exact in f32, so each lane equals
+// fmaf(float(x), float(w), acc) bit for bit, without the two conversions.
+template <typename T>
+__device__ __forceinline__ void mac2(float &a0, float &a1, uint32_t x2, uint32_t w2);
+template <>
+__device__ __forceinline__ void mac2<__half>(float &a0, float &a1, uint32_t x2, uint32_t w2) {
+    asm("{\n\t.reg .b16 xl, xh, wl, wh;\n\tmov.b32 {xl, xh}, %2;\n\tmov.b32 {wl, wh}, %3;\n\t"
+        "fma.rn.f32.f16 %0, xl, wl, %0;\n\tfma.rn.f32.f16 %1, xh, wh, %1;\n\t}"
+        : "+f"(a0), "+f"(a1)
+        : "r"(x2), "r"(w2));
+}
+template <>
+__device__ __forceinline__ void mac2<__nv_bfloat16>(float &a0, float &a1, uint32_t x2, uint32_t w2) {
+    asm("{\n\t.reg .b16 xl, xh, wl, wh;\n\tmov.b32 {xl, xh}, %2;\n\tmov.b32 {wl, wh}, %3;\n\t"
+        "fma.rn.f32.bf16 %0, xl, wl, %0;\n\tfma.rn.f32.bf16 %1, xh, wh, %1;\n\t}"
+        : "+f"(a0), "+f"(a1)
+        : "r"(x2), "r"(w2));
+}
+
 // Division by a divisor fixed at launch, for numerators below 2^31:
 // q = (umulhi(n, m) + n) >> l with l = ceil(log2 d), m = floor(2^32 (2^l - d) / d) + 1
 // (the round-up multiplier method of Granlund and Montgomery).  The generic
@@ -101,6 +133,10 @@ __device__ __forceinline__ uint32_t fdiv(uint32_t n, const FastDiv &f) {
 struct ConvDims {
     int32_t N, C, H, W, K, P, Q, R, S, sh, sw, ph, pw, dh, dw, groups, act;
 };
+
+// NHWC 3x3 depthwise through a TMA-fed shared-memory ring of input rows
+bool dw3_ring_applies(const LaunchArgs &a, const ConvDims &d);
+cudaError_t dw3_nhwc_ring(const LaunchArgs &a, const ConvDims &d);
 
 cudaError_t conv_wino_buffers(const ConvDims &d, sn_schema s, const void *x, const void *u, const float *bias,
                               void *y, float *V, float *Mx, cudaStream_t st);

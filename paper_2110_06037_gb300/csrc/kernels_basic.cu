@@ -30,6 +30,56 @@ __global__ void cast_kernel(const Ti *__restrict__ x, To *__restrict__ y, int64_
         stf<To>(y + i, ldf<Ti>(x + i));
 }
 
+// VB-byte vector access to VB / sizeof(T) consecutive elements, as floats
+template <typename T, int VB>
+struct VecIO {
+    static constexpr int E = VB / (int)sizeof(T);
+    using V = typename std::conditional<
+        VB == 16, uint4,
+        typename std::conditional<VB == 8, uint2,
+                                  typename std::conditional<VB == 4, uint32_t, uint16_t>::type>::type>::type;
+    __device__ __forceinline__ static void load(const T *p, float (&f)[E]) {
+        const V v = *reinterpret_cast<const V *>(p);
+        const T *t = reinterpret_cast<const T *>(&v);
+#pragma unroll
+        for (int e = 0; e < E; ++e) f[e] = ldf<T>(t + e);
+    }
+    __device__ __forceinline__ static void store(T *p, const float (&f)[E]) {
+        V v;
+        T *t = reinterpret_cast<T *>(&v);
+#pragma unroll
+        for (int e = 0; e < E; ++e) t[e] = cvt<T>(f[e]);
+        *reinterpret_cast<V *>(p) = v;
+    }
+};
+
+// same layout, 8 elements per thread and iteration with 16-byte accesses
+// (n % 8 == 0, 16-byte aligned bases)
+template <typename Ti, typename To>
+__global__ void cast_vec8_kernel(const Ti *__restrict__ x, To *__restrict__ y, int64_t n8) {
+    griddep_launch();
+    griddep_wait();
+    constexpr int EI = VecIO<Ti, 16>::E, EO = VecIO<To, 16>::E;
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n8;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        float f[8];
+#pragma unroll
+        for (int j = 0; j < 8; j += EI) {
+            float g[EI];
+            VecIO<Ti, 16>::load(x + i * 8 + j, g);
+#pragma unroll
+            for (int e = 0; e < EI; ++e) f[j + e] = g[e];
+        }
+#pragma unroll
+        for (int j = 0; j < 8; j += EO) {
+            float g[EO];
+#pragma unroll
+            for (int e = 0; e < EO; ++e) g[e] = f[j + e];
+            VecIO<To, 16>::store(y + i * 8 + j, g);
+        }
+    }
+}
+
 // 16-byte vectorised copy when dtypes match
 __global__ void copy16_kernel(const uint4 *__restrict__ x, uint4 *__restrict__ y, int64_t n16) {
     griddep_launch();
@@ -40,72 +90,56 @@ __global__ void copy16_kernel(const uint4 *__restrict__ x, uint4 *__restrict__ y
 }
 
 // batched transpose y[b][c][r] = x[b][r][c] with a cast, through a 64x64
-// shared-memory tile (256 threads, 16 elements each); rows of 64 contiguous
-// elements are read and written by consecutive threads.
+// shared-memory tile: VBI-byte vectors along the input rows, VBO-byte vectors
+// along the output rows (the widest the row lengths and bases allow: a
+// 14 x 14 plane is 392 bytes of bf16, so its rows take 8-byte vectors)
 constexpr int TT = 64;
-template <typename Ti, typename To>
-__global__ void __launch_bounds__(256) transpose_kernel(const Ti *__restrict__ x, To *__restrict__ y,
-                                                         int64_t R, int64_t Cc) {
-    griddep_launch();
-    griddep_wait();
-    __shared__ float tile[TT][TT + 1];
-    const int64_t b = blockIdx.z;
-    const int64_t r0 = (int64_t)blockIdx.y * TT, c0 = (int64_t)blockIdx.x * TT;
-    const Ti *xb = x + b * R * Cc;
-    To *yb = y + b * R * Cc;
-    const int tx = threadIdx.x % TT, ty = threadIdx.x / TT;  // 64 x 4
-#pragma unroll
-    for (int i = 0; i < TT; i += 4) {
-        const int64_t r = r0 + ty + i, c = c0 + tx;
-        if (r < R && c < Cc) tile[ty + i][tx] = ldf<Ti>(xb + r * Cc + c);
-    }
-    __syncthreads();
-#pragma unroll
-    for (int i = 0; i < TT; i += 4) {
-        const int64_t c = c0 + ty + i, r = r0 + tx;
-        if (r < R && c < Cc) stf<To>(yb + c * R + r, tile[tx][ty + i]);
-    }
-}
-
-// the same transpose with 16-byte loads and stores (EI input, EO output
-// elements per vector); needs Cc % EI == 0, R % EO == 0 and aligned bases
-template <typename Ti, typename To>
+template <typename Ti, typename To, int VBI, int VBO>
 __global__ void __launch_bounds__(256) transpose_vec_kernel(const Ti *__restrict__ x, To *__restrict__ y,
                                                              int64_t R, int64_t Cc) {
     griddep_launch();
     griddep_wait();
-    constexpr int EI = 16 / sizeof(Ti), EO = 16 / sizeof(To);
+    using LI = VecIO<Ti, VBI>;
+    using LO = VecIO<To, VBO>;
+    constexpr int EI = LI::E, EO = LO::E;
     __shared__ float tile[TT][TT + 1];
     const int64_t b = blockIdx.z;
     const int64_t r0 = (int64_t)blockIdx.y * TT, c0 = (int64_t)blockIdx.x * TT;
     const Ti *xb = x + b * R * Cc;
     To *yb = y + b * R * Cc;
     constexpr int VI = TT / EI;  // input vectors per tile row
-#pragma unroll
+#pragma unroll 4
     for (int i = threadIdx.x; i < TT * VI; i += 256) {
         const int row = i / VI, cv = i % VI;
         const int64_t r = r0 + row, c = c0 + cv * EI;
         if (r < R && c < Cc) {
-            const uint4 v = *reinterpret_cast<const uint4 *>(xb + r * Cc + c);
-            const Ti *pv = reinterpret_cast<const Ti *>(&v);
+            float f[EI];
+            LI::load(xb + r * Cc + c, f);
 #pragma unroll
-            for (int e = 0; e < EI; ++e) tile[row][cv * EI + e] = ldf<Ti>(pv + e);
+            for (int e = 0; e < EI; ++e) tile[row][cv * EI + e] = f[e];
         }
     }
     __syncthreads();
     constexpr int VO = TT / EO;  // output vectors per tile row (output row = input column)
-#pragma unroll
+#pragma unroll 4
     for (int i = threadIdx.x; i < TT * VO; i += 256) {
         const int orow = i / VO, ov = i % VO;
         const int64_t c = c0 + orow, r = r0 + ov * EO;
         if (c < Cc && r < R) {
-            uint4 v;
-            To *pv = reinterpret_cast<To *>(&v);
+            float f[EO];
 #pragma unroll
-            for (int e = 0; e < EO; ++e) pv[e] = cvt<To>(tile[ov * EO + e][orow]);
-            *reinterpret_cast<uint4 *>(yb + c * R + r) = v;
+            for (int e = 0; e < EO; ++e) f[e] = tile[ov * EO + e][orow];
+            LO::store(yb + c * R + r, f);
         }
     }
+}
+
+// widest vector (16, 8 or element bytes) that a row of n elements of es bytes
+// starting at every row of an aligned base admits
+static int row_vec_bytes(int64_t n, int es, const void *base) {
+    for (int vb : {16, 8})
+        if ((n * es) % vb == 0 && (uintptr_t)base % vb == 0) return vb;
+    return es;
 }
 
 // few channels (C <= 16): one thread per pixel moves all of its channels;
@@ -141,7 +175,10 @@ static cudaError_t convert_t(const void *x, int lay_in, void *y, int lay_out, Sh
             }
             return cudaMemcpyAsync(y, x, bytes, cudaMemcpyDeviceToDevice, st);
         }
-        launch_pdl(cast_kernel<Ti, To>, grid_for(n, 256), 256, 0, st, (const Ti *)x, (To *)y, n);
+        if (n % 8 == 0 && ((uintptr_t)x % 16) == 0 && ((uintptr_t)y % 16) == 0)
+            launch_pdl(cast_vec8_kernel<Ti, To>, grid_for(n / 8, 256), 256, 0, st, (const Ti *)x, (To *)y, n / 8);
+        else
+            launch_pdl(cast_kernel<Ti, To>, grid_for(n, 256), 256, 0, st, (const Ti *)x, (To *)y, n);
         return cudaGetLastError();
     }
     if (s.c <= 16) {
@@ -160,11 +197,18 @@ static cudaError_t convert_t(const void *x, int lay_in, void *y, int lay_out, Sh
     if (s.n > 65535) return cudaErrorInvalidValue;
     dim3 grid((unsigned)((Cc + TT - 1) / TT), (unsigned)((R + TT - 1) / TT), (unsigned)s.n);
     if (grid.y > 65535) return cudaErrorInvalidValue;
-    constexpr int EI = 16 / sizeof(Ti), EO = 16 / sizeof(To);
-    if (Cc % EI == 0 && R % EO == 0 && (uintptr_t)x % 16 == 0 && (uintptr_t)y % 16 == 0)
-        launch_pdl(transpose_vec_kernel<Ti, To>, grid, 256, 0, st, (const Ti *)x, (To *)y, R, Cc);
-    else
-        launch_pdl(transpose_kernel<Ti, To>, grid, 256, 0, st, (const Ti *)x, (To *)y, R, Cc);
+    constexpr int SI = (int)sizeof(Ti), SO = (int)sizeof(To);
+    const int vi = row_vec_bytes(Cc, SI, x), vo = row_vec_bytes(R, SO, y);
+    const Ti *xi = (const Ti *)x;
+    To *yo = (To *)y;
+#define SN_TRANSPOSE(A, B) launch_pdl(transpose_vec_kernel<Ti, To, A, B>, grid, 256, 0, st, xi, yo, R, Cc)
+    if (vi == 16 && vo == 16) SN_TRANSPOSE(16, 16);
+    else if (vi == 16 && vo == 8) SN_TRANSPOSE(16, 8);
+    else if (vi == 8 && vo == 16) SN_TRANSPOSE(8, 16);
+    else if (vi == 16) SN_TRANSPOSE(16, SO);
+    else if (vo == 16) SN_TRANSPOSE(SI, 16);
+    else SN_TRANSPOSE(SI, SO);
+#undef SN_TRANSPOSE
     return cudaGetLastError();
 }
 
@@ -387,6 +431,24 @@ __global__ void dw_nhwc(const T *__restrict__ x, const T *__restrict__ w, const 
 // columns: each input vector a thread needs for its QB outputs is loaded from
 // global once per (tap row, column) and reused through L1 by its neighbours;
 // weights are [R][S][C].
+// acc[e] += x[e] * w[e] over the 16 bytes of x and w (E = 16 / sizeof(T)
+// lanes); 16-bit types use the mixed-precision FMA, which equals converting
+// both factors to f32 first
+template <typename T, int E>
+__device__ __forceinline__ void fma16(float (&acc)[E], const uint4 &x, const uint4 &w) {
+    if constexpr (sizeof(T) == 2) {
+        mac2<T>(acc[0], acc[1], x.x, w.x);
+        mac2<T>(acc[2], acc[3], x.y, w.y);
+        mac2<T>(acc[4], acc[5], x.z, w.z);
+        mac2<T>(acc[6], acc[7], x.w, w.w);
+    } else {
+        const T *xp = reinterpret_cast<const T *>(&x);
+        const T *wp = reinterpret_cast<const T *>(&w);
+#pragma unroll
+        for (int e = 0; e < E; ++e) acc[e] = fmaf(ldf<T>(xp + e), ldf<T>(wp + e), acc[e]);
+    }
+}
+
 // One thread: QB consecutive output columns x E channels (16 bytes) of one
 // output row.  The grid's y axis walks the N x P output rows, its x axis the
 // (column block, channel vector) pairs of a row with the channel vector
@@ -439,16 +501,8 @@ __global__ void __launch_bounds__(256, 2) dw_nhwc_vec(const T *__restrict__ x, c
 #pragma unroll
                 for (int s = 0; s < 3; ++s) {
                     const uint4 wq = *reinterpret_cast<const uint4 *>(w + (int64_t)(r * 3 + s) * d.C + c0);
-                    const T *wp = reinterpret_cast<const T *>(&wq);
-                    float wf[E];
 #pragma unroll
-                    for (int e = 0; e < E; ++e) wf[e] = ldf<T>(wp + e);
-#pragma unroll
-                    for (int j = 0; j < QB; ++j) {
-                        const T *xp = reinterpret_cast<const T *>(&win[j * (SW > 0 ? SW : 1) + s]);
-#pragma unroll
-                        for (int e = 0; e < E; ++e) acc[j][e] = fmaf(ldf<T>(xp + e), wf[e], acc[j][e]);
-                    }
+                    for (int j = 0; j < QB; ++j) fma16<T>(acc[j], win[j * (SW > 0 ? SW : 1) + s], wq);
                 }
             }
         } else {
@@ -458,19 +512,11 @@ __global__ void __launch_bounds__(256, 2) dw_nhwc_vec(const T *__restrict__ x, c
                 const T *xrow = x + (((int64_t)n * d.H + h) * d.W) * d.C + c0;
                 for (int s = 0; s < d.S; ++s) {
                     const uint4 wq = *reinterpret_cast<const uint4 *>(w + (int64_t)(r * d.S + s) * d.C + c0);
-                    const T *wp = reinterpret_cast<const T *>(&wq);
-                    float wf[E];
-#pragma unroll
-                    for (int e = 0; e < E; ++e) wf[e] = ldf<T>(wp + e);
 #pragma unroll
                     for (int j = 0; j < QB; ++j) {
                         const int ww = (q0 + j) * d.sw - d.pw + s * d.dw;
-                        if (q0 + j < d.Q && ww >= 0 && ww < d.W) {
-                            const uint4 xq = *reinterpret_cast<const uint4 *>(xrow + (int64_t)ww * d.C);
-                            const T *xp = reinterpret_cast<const T *>(&xq);
-#pragma unroll
-                            for (int e = 0; e < E; ++e) acc[j][e] = fmaf(ldf<T>(xp + e), wf[e], acc[j][e]);
-                        }
+                        if (q0 + j < d.Q && ww >= 0 && ww < d.W)
+                            fma16<T>(acc[j], *reinterpret_cast<const uint4 *>(xrow + (int64_t)ww * d.C), wq);
                     }
                 }
             }
@@ -701,9 +747,11 @@ __global__ void __launch_bounds__(256) dw3_nchw_tile(const T *__restrict__ x, co
 
 cudaError_t dwconv(const LaunchArgs &a) {
     // routine parameter (variant): NHWC 0 = register window (4 columns per
-    // thread), 1 = shared-memory halo tiles; NCHW 0 = row kernel (8 columns
-    // per thread), 1 = shared-memory plane tile
+    // thread), 1 = input rows staged by TMA in a shared-memory ring (3x3,
+    // 16-bit; shared-memory halo tiles otherwise); NCHW 0 = row kernel (8
+    // columns per thread), 1 = shared-memory plane tile
     const ConvDims d = conv_dims(a);
+    if (a.variant == 1 && dw3_ring_applies(a, d)) return dw3_nhwc_ring(a, d);
     const int64_t total = (int64_t)d.N * d.K * d.P * d.Q;
     const int es = dtype_size(a.schema.dtype);
     const bool vec_ok = (d.C * es) % 16 == 0 && (uintptr_t)a.in[0] % 16 == 0 && (uintptr_t)a.out % 16 == 0 &&

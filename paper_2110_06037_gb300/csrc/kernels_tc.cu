@@ -536,6 +536,10 @@ static bool encode(CUtensorMap *m, int dt, int rank, const void *base, const uin
               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+bool tma_encode(CUtensorMap *m, int dt, int rank, const void *base, const uint64_t *dims,
+                const uint64_t *strides_bytes, const uint32_t *box, CUtensorMapSwizzle sw) {
+    return encode(m, dt, rank, base, dims, strides_bytes, box, sw);
+}
 
 struct Config {
     bool implicit;
@@ -631,16 +635,6 @@ static std::vector<Config> configs(const Layer &l, const Shape &in, sn_schema s,
             push_all({true, 0, gg.bw, gg.bh, gg.bni, 1, 1, 1}, mtiles);
     }
     return out;
-}
-
-static int num_sms() {
-    static int n = 0;
-    if (!n) {
-        int dev = 0;
-        cudaGetDevice(&dev);
-        if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 1;
-    }
-    return n;
 }
 
 template <typename T, int BN, bool IMPLICIT, int G, int KB>

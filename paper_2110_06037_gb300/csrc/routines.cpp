@@ -34,7 +34,7 @@ const char *variant_name(int32_t r, int32_t v) {
     switch (r) {
     case R_CONV_IGEMM: return v == 0 ? "tile=64x64" : "tile=128x64";
     case R_CONV_WINO: return v == 0 ? "gemm=simt" : "gemm=tc";
-    case R_DW_DIRECT: return v == 0 ? "nhwc:window|nchw:rows" : "nhwc:smem_halo|nchw:plane_tile";
+    case R_DW_DIRECT: return v == 0 ? "nhwc:window|nchw:rows" : "nhwc:tma_rows|nchw:plane_tile";
     case R_CONV_TC:
     case R_CONV_IM2COL_TC:
     case R_CONV_S2D_TC:

@@ -363,6 +363,11 @@ __device__ __forceinline__ Work work_of(const Params &p, int u, int bn, bool imp
     return w;
 }
 
+// host: encode a tiled tensor map over an f16/bf16 tensor (dims innermost
+// first, byte strides of the outer dims); false if the driver refuses it
+bool tma_encode(CUtensorMap *m, int dt, int rank, const void *base, const uint64_t *dims,
+                const uint64_t *strides_bytes, const uint32_t *box, CUtensorMapSwizzle sw);
+
 }  // namespace tc
 }  // namespace k
 }  // namespace sn

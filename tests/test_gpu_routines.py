@@ -1,6 +1,8 @@
 """Per-routine parity on the GPU through the C ABI: every routine of every
 layer type, in every schema it serves, against the oracle on the same stored
 inputs.  Adapt conversions are checked bit for bit."""
+import zlib
+
 import numpy as np
 import pytest
 
@@ -67,7 +69,7 @@ ROUTINES = ([("conv2/direct", 0), ("conv2/igemm_simt", 0), ("conv2/igemm_simt", 
 @pytest.mark.parametrize("schema", SCHEMAS)
 def test_conv_routines(case, schema):
     N, C, H, W, K, k, s, p, d, g = case
-    rng = np.random.default_rng(abs(hash((case, schema))) % 2**32)
+    rng = np.random.default_rng(zlib.crc32(repr((case, schema)).encode()))
     x = rng.standard_normal((N, C, H, W)).astype(np.float32)
     layer = synth.conv(C, K, k, s, p, act="relu", groups=g, d=d)
     layer["weight"] = (rng.standard_normal((K, C // g, k, k)) * np.sqrt(2.0 / (C // g * k * k))).astype(np.float32)
@@ -84,22 +86,33 @@ def test_conv_routines(case, schema):
     assert ran >= 1
 
 
-DW_CASES = [(1, 32, 16, 16, 1), (2, 24, 9, 9, 2), (1, 144, 28, 28, 1), (1, 40, 7, 7, 2), (1, 8, 1, 1, 1)]
+DW_CASES = [(1, 32, 16, 16, 1), (2, 24, 9, 9, 2), (1, 144, 28, 28, 1), (1, 40, 7, 7, 2), (1, 8, 1, 1, 1),
+            (2, 576, 14, 14, 1),    # channel slices of 192 (TMA box limit 256)
+            (4, 320, 9, 9, 1),      # two slices of 160, ragged column blocks
+            (3, 96, 30, 30, 2),
+            (16, 64, 57, 57, 2),    # odd extent, stride 2, ranges spanning images
+            (48, 128, 48, 48, 1)]   # ranges longer than the row ring (slots reused)
 
 
 @pytest.mark.parametrize("case", DW_CASES)
 @pytest.mark.parametrize("schema", SCHEMAS)
 def test_depthwise(case, schema):
     N, C, H, W, s = case
-    rng = np.random.default_rng(abs(hash((case, schema))) % 2**32)
+    rng = np.random.default_rng(zlib.crc32(repr((case, schema)).encode()))
     x = rng.standard_normal((N, C, H, W)).astype(np.float32)
     layer = synth.dwconv(C, 3, s, act="relu6")
     layer["weight"] = (rng.standard_normal((C, 1, 3, 3)) * np.sqrt(2 / 9)).astype(np.float32)
     layer["bias"] = (rng.standard_normal(C) * 0.1).astype(np.float32)
     ref = ref_one(layer, x, schema[0])
-    for v in (0, 1):  # routine parameters: columns per thread / row vs plane-tile kernel
+    outs = []
+    for v in (0, 1):  # routine parameters: register window / rows in shared memory (NHWC), row / plane tile (NCHW)
         got = run_one(layer, x, schema, "dwconv2/direct", v)
         assert maxrel(got, ref) <= TOL[schema[0]], v
+        outs.append(got)
+    if schema[1] == "nhwc" and schema[0] != "f32":
+        # both NHWC kernels accumulate the nine taps in f32 in the same order
+        # (bias, then rows, then columns) with exact products: equal results
+        assert np.array_equal(outs[0], outs[1])
 
 
 @pytest.mark.parametrize("schema", SCHEMAS)
@@ -132,7 +145,10 @@ def test_pool_gap_add_dense(schema):
             assert maxrel(got, ref) <= TOL[schema[0]], v
 
 
-CONVERT_SHAPES = [(2, 5, 7, 9), (1, 64, 56, 56), (3, 130, 1, 1), (1, 3, 65, 67)]
+# planes of 196 (8-byte bf16 rows, 16-byte f32 rows), 49 (element-wide rows)
+# and 130 channels (ragged tiles on both axes, element-wide channel rows)
+CONVERT_SHAPES = [(2, 5, 7, 9), (1, 64, 56, 56), (3, 130, 1, 1), (1, 3, 65, 67), (2, 24, 14, 14),
+                  (2, 40, 7, 7), (2, 130, 14, 14), (1, 1024, 14, 14)]
 
 
 @pytest.mark.parametrize("shape", CONVERT_SHAPES)
@@ -181,7 +197,7 @@ def test_conv_residual(case, schema):
     for every direct and tensor-core routine parameter the layer offers."""
     import torch
     N, C, H, W, k, p = case
-    rng = np.random.default_rng(abs(hash((case, schema, "res"))) % 2**32)
+    rng = np.random.default_rng(zlib.crc32(repr((case, schema, "res")).encode()))
     x = rng.standard_normal((N, C, H, W)).astype(np.float32)
     pool = {"type": "maxpool", "name": "pool", "inputs": [-1],
             "params": dict(kh=3, kw=3, sh=1, sw=1, ph=1, pw=1)}

@@ -4,6 +4,8 @@ against the oracle, over every routine-parameter combination it offers:
 counts that are not multiples of the 64-channel K block, output channels
 that end inside an epilogue chunk, ragged pixel tiles, CTA-pair tiles whose
 second CTA has no pixels, stages of one and of two 64-channel blocks."""
+import zlib
+
 import numpy as np
 import pytest
 
@@ -41,7 +43,7 @@ def test_tc_routine_all_variants(case, dt):
     import torch
     N, C, H, W, K, k, s, pd = case
     schema = (dt, "nhwc")
-    rng = np.random.default_rng(abs(hash((case, dt))) % 2**32)
+    rng = np.random.default_rng(zlib.crc32(repr((case, dt)).encode()))
     x = rng.standard_normal((N, C, H, W)).astype(np.float32)
     layer = synth.conv(C, K, k, s, pd, act="relu")
     layer["weight"] = (rng.standard_normal((K, C, k, k)) * np.sqrt(2.0 / (C * k * k))).astype(np.float32)
