@@ -53,7 +53,7 @@ namespace tc {
 // shared memory, and each CTA's TMEM receives its own 128 rows, drained by
 // its own epilogue.  Per SM this halves the weight bytes staged and read per
 // MMA, the shared-memory bandwidth that limits a one-CTA tile.
-template <typename T, int BN, int STAGES, bool IMPLICIT, int G, int KB>
+template <typename T, int BN, int STAGES, bool IMPLICIT, int G, int KB, bool BST>
 __global__ void __launch_bounds__(THREADS, 1)
     conv_tc_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ CUtensorMap mA1,
                    const __grid_constant__ CUtensorMap mA2, const __grid_constant__ CUtensorMap mA3,
@@ -65,7 +65,9 @@ __global__ void __launch_bounds__(THREADS, 1)
     constexpr uint32_t B_BLK = (BN / G) * BK * 2;
     constexpr uint32_t A_BYTES = KB * A_BLK;
     constexpr uint32_t B_BYTES = KB * B_BLK;
-    constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
+    // BST (weight-stationary, G = 1, one N tile, no K split): a stage holds A
+    // only; B of every K step sits after the stages for the whole kernel
+    constexpr uint32_t STAGE_BYTES = BST ? A_BYTES : A_BYTES + B_BYTES;
     constexpr uint32_t TMEM_COLS = 2 * BN;  // two accumulators
     extern __shared__ uint8_t smem_raw[];
     __shared__ __align__(8) uint64_t full_bar[STAGES];
@@ -73,13 +75,15 @@ __global__ void __launch_bounds__(THREADS, 1)
     __shared__ __align__(8) uint64_t accf_bar[2];  // MMA -> epilogue: accumulator ready
     __shared__ __align__(8) uint64_t acce_bar[2];  // epilogue -> MMA: accumulator drained
     __shared__ __align__(8) uint64_t res_bar[EPI_WARPS];  // residual tile landed in a warp's staging block
+    __shared__ __align__(8) uint64_t bst_bar;              // weight-stationary B landed
     __shared__ uint32_t tmem_sh;
     __shared__ volatile int abort_sh;
     __shared__ int issued_sh[4], consumed_sh;
 
     griddep_launch();
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    uint8_t *stg = smem + STAGES * STAGE_BYTES;  // epilogue staging: 8 warps x 2 buffers, 1024-B aligned
+    uint8_t *bst = smem + STAGES * STAGE_BYTES;  // weight-stationary B (BST), 1024-B aligned
+    uint8_t *stg = bst + (BST ? p.bst_bytes : 0);  // epilogue staging: one block per warp, 1024-B aligned
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
     const uint32_t rank = G == 2 ? cluster_rank() : 0u;
     const bool leader = rank == 0;
@@ -108,6 +112,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         for (int i = 0; i < EPI_WARPS; ++i) {
             mbar_init(&res_bar[i], 1);
         }
+        mbar_init(&bst_bar, 1);
         abort_sh = 0;
         issued_sh[0] = issued_sh[1] = issued_sh[2] = issued_sh[3] = 0;
         consumed_sh = 0;
@@ -126,8 +131,45 @@ __global__ void __launch_bounds__(THREADS, 1)
     // written by the previous kernel.
 
     constexpr int NPROD = producers_for(STAGES);
+    constexpr bool WAITER = waits_for_mma(STAGES);
     const int prod = warp == 0 ? 0 : (warp >= 10 ? warp - 9 : -1);  // producer index of this warp
-    if (prod >= 0) {
+    if (WAITER && warp == 11) {
+        if (leader) {  // ---------------- the MMA warp's barrier waits (whole warp)
+            // the same sequence as the MMA warp: per unit, accumulator b
+            // drained, then every K step's stage full; one bar_red_or each
+            int lt = 0, s = 0;
+            uint32_t par = 0;
+            bool stop = false;
+            for (int u = cid; u < total && !stop; u += ncl, ++lt) {
+                const Work w = work_of(p, u, BN, IMPLICIT, G, 0);
+                const int b = lt & 1;
+                const uint32_t aph = (uint32_t)(lt >> 1) & 1u;
+                bool ok = G == 2 ? mbar_wait_cluster(&acce_bar[b], aph ^ 1u) : mbar_wait(&acce_bar[b], aph ^ 1u);
+                if (!ok) {
+                    if (lane == 0) atomicOr(p.err, ERR_EPI_WAIT);
+                    set_abort();
+                }
+                __syncwarp();  // bar.red is warp-aligned: reconverge after the polling loops
+                if (bar_red_or(BAR_MMA, 64, !ok || abort_sh)) break;
+                for (int it = w.it0; it < w.it1; ++it) {
+                    ok = mbar_wait(&full_bar[s], par);
+                    if (!ok) {
+                        if (lane == 0) atomicOr(p.err, ERR_MMA_WAIT);
+                        set_abort();
+                    }
+                    __syncwarp();
+                    if (bar_red_or(BAR_MMA, 64, !ok || abort_sh)) {
+                        stop = true;
+                        break;
+                    }
+                    if (++s == STAGES) {
+                        s = 0;
+                        par ^= 1u;
+                    }
+                }
+            }
+        }
+    } else if (prod >= 0) {
         if (lane == 0 && prod < NPROD) {  // ---------------- TMA producers
             // Producer `prod` fills the stages s with s % NPROD == prod (A and B
             // of every CTA's own rows); several issuing threads, because one
@@ -139,6 +181,19 @@ __global__ void __launch_bounds__(THREADS, 1)
             int g = 0, s = prod, issued = 0;
             uint32_t par = 0;
             bool stop = false, waited = false;
+            if (BST && prod == 0) {
+                // the weights are not written by the previous kernel: loaded
+                // before the dependency wait, one box per K step
+                mbar_expect_tx(&bst_bar, (uint32_t)p.bst_bytes);
+                int tap = 0, cb = 0;
+                for (int it = 0; it < p.kiters; ++it) {
+                    tma_3d<1>(su32(bst + it * B_BYTES), &mB, su32(&bst_bar), cb * BK, tap, 0);
+                    if (++cb == cblocks) {
+                        cb = 0;
+                        ++tap;
+                    }
+                }
+            }
             for (int u = cid; u < total && !stop; u += ncl) {
                 const Work w = work_of(p, u, BN, IMPLICIT, G, (int)rank);
                 int tap = (int)fdiv((uint32_t)w.it0, p.fd_spt);
@@ -164,7 +219,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                         // box spans KB blocks
                         const int c0 = cb * BK;
                         // the leader's barrier counts the bytes of both CTAs
-                        if (leader) mbar_expect_tx(&full_bar[s], G * STAGE_BYTES);
+                        if (leader) mbar_expect_tx(&full_bar[s], G * STAGE_BYTES);  // A only when BST
                         const uint32_t bar = G == 2 ? mapa(su32(&full_bar[s]), 0u) : su32(&full_bar[s]);
                         if (IMPLICIT) {
                             const int oh = r * dh - ph0, ow = ss * dw - pw0;
@@ -186,10 +241,12 @@ __global__ void __launch_bounds__(THREADS, 1)
                             else
                                 tma_3d<G>(sa, &mA0, bar, 0, (int)w.m0, cb);
                         }
-                        if (KB == 1)
-                            tma_3d<G>(sa + A_BYTES, &mB, bar, c0, tap, w.n0 + brow);
-                        else
-                            tma_4d<G>(sa + A_BYTES, &mB, bar, 0, tap, w.n0 + brow, cb);
+                        if (!BST) {  // weight-stationary B is already resident
+                            if (KB == 1)
+                                tma_3d<G>(sa + A_BYTES, &mB, bar, c0, tap, w.n0 + brow);
+                            else
+                                tma_4d<G>(sa + A_BYTES, &mB, bar, 0, tap, w.n0 + brow, cb);
+                        }
                         issued = g + 1;
                         s += NPROD;
                         if (s >= STAGES) {
@@ -209,13 +266,64 @@ __global__ void __launch_bounds__(THREADS, 1)
             }
             issued_sh[prod] = issued;
         }
+    } else if (warp == 1 && WAITER) {
+        if (leader) {  // ---------------- MMA issuer (lane 0; the whole warp meets the waiter)
+            const uint32_t idesc = idesc_f16<T>(BM * G, BN);
+            const uint64_t desc0 = sdesc_sw128(su32(smem));  // stage 0, A; offsets add to the address field
+            const uint64_t descb = sdesc_sw128(su32(bst));   // weight-stationary B, K step 0
+            int g = 0, lt = 0, s = 0;
+            bool stop = false;
+            if (BST && lane == 0 && !mbar_wait(&bst_bar, 0u)) {
+                atomicOr(p.err, ERR_MMA_WAIT);
+                set_abort();
+            }
+            __syncwarp();
+            for (int u = cid; u < total && !stop; u += ncl, ++lt) {
+                const Work w = work_of(p, u, BN, IMPLICIT, G, 0);
+                const int b = lt & 1;
+                if (bar_red_or(BAR_MMA, 64, false)) break;  // accumulator b drained
+                tc_fence_after();
+                const uint32_t d = tmem + (uint32_t)(b * BN);
+                for (int it = w.it0; it < w.it1; ++it, ++g) {
+                    if (bar_red_or(BAR_MMA, 64, false)) {  // stage s full
+                        stop = true;
+                        break;
+                    }
+                    tc_fence_after();
+                    if (lane == 0) {
+                        // descriptors of this stage; a K step of 16 is 32 bytes (2 units)
+                        const uint64_t da = desc0 + (uint64_t)((s * STAGE_BYTES) >> 4);
+                        const uint64_t db =
+                            BST ? descb + (uint64_t)(((uint32_t)it * B_BYTES) >> 4) : da + (A_BYTES >> 4);
+#pragma unroll
+                        for (int j = 0; j < KB; ++j)
+#pragma unroll
+                            for (int k = 0; k < BK / 16; ++k)
+                                umma<G>(d, da + j * (A_BLK >> 4) + 2 * k, db + j * (B_BLK >> 4) + 2 * k, idesc,
+                                        (it > w.it0 || j > 0 || k > 0) ? 1u : 0u);
+                        umma_commit<G>(&empty_bar[s]);  // frees the stage (in both CTAs) once read
+                    }
+                    __syncwarp();
+                    if (++s == STAGES) s = 0;
+                }
+                if (!stop && lane == 0) umma_commit<G>(&accf_bar[b]);
+                __syncwarp();
+            }
+            if (lane == 0) consumed_sh = g;
+        }
     } else if (warp == 1) {
         if (lane == 0 && leader) {  // ---------------- MMA issuer (the pair's leader)
             const uint32_t idesc = idesc_f16<T>(BM * G, BN);
             const uint64_t desc0 = sdesc_sw128(su32(smem));  // stage 0, A; offsets add to the address field
+            const uint64_t descb = sdesc_sw128(su32(bst));   // weight-stationary B, K step 0
             int g = 0, lt = 0, s = 0;
             uint32_t par = 0;
             bool stop = false;
+            if (BST && !mbar_wait(&bst_bar, 0u)) {
+                atomicOr(p.err, ERR_MMA_WAIT);
+                set_abort();
+                stop = true;
+            }
             for (int u = cid; u < total && !stop; u += ncl, ++lt) {
                 const Work w = work_of(p, u, BN, IMPLICIT, G, 0);
                 const int b = lt & 1;
@@ -238,7 +346,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                     tc_fence_after();
                     // descriptors of this stage; a K step of 16 is 32 bytes (2 units)
                     const uint64_t da = desc0 + (uint64_t)((s * STAGE_BYTES) >> 4);
-                    const uint64_t db = da + (A_BYTES >> 4);
+                    const uint64_t db = BST ? descb + (uint64_t)(((uint32_t)it * B_BYTES) >> 4) : da + (A_BYTES >> 4);
 #pragma unroll
                     for (int j = 0; j < KB; ++j)
 #pragma unroll
@@ -452,6 +560,9 @@ __global__ void __launch_bounds__(THREADS, 1)
                 while (!mbar_try(&empty_bar[g % STAGES], (uint32_t)(g / STAGES) & 1u) && clock64() - t0 < WAIT_LIMIT) {
                 }
             }
+            if (BST)
+                while (!mbar_try(&bst_bar, 0u) && clock64() - t0 < WAIT_LIMIT) {
+                }
         }
         __syncwarp();
     }
@@ -548,6 +659,7 @@ struct Config {
     int ksplit;
     int G;   // CTAs per tile: 1, or 2 (CTA pair, 256-pixel tile)
     int KB;  // 64-channel blocks per pipeline stage (one TMA box spans them)
+    bool bst = false;  // weight-stationary: B loaded once per CTA (one N tile, G = 1, no split)
 };
 
 constexpr int kSmCount = 152;  // GB300; only used to decide which K splits to offer
@@ -605,8 +717,24 @@ static std::vector<Config> configs(const Layer &l, const Shape &in, sn_schema s,
                 cf.KB = 1;
             }
     };
+    // weight-stationary variant: the whole B of a one-N-tile layer fits in
+    // shared memory beside BST_STAGES A stages and the epilogue staging
+    auto push_bst = [&](Config cf) {
+        for (int bn : bns)
+            if (K <= bn) {
+                const int64_t bytes = (int64_t)kiters * bn * BK * 2;
+                // 227 KB less the alignment slack, the static barriers and the A stages and staging
+                const int64_t room = 227 * 1024 - 2048 - (int64_t)BST_STAGES * BM * BK * 2 - EPI_WARPS * STG_BYTES;
+                if (bytes <= room) {
+                    cf.BN = bn, cf.G = 1, cf.KB = 1, cf.ksplit = 1, cf.bst = true;
+                    out.push_back(cf);
+                }
+                break;
+            }
+    };
     if (plain && a_blocks == 0) {
         push_all({false, 0, 0, 0, 0, 1, 1, 1}, (N * P * Q + BM - 1) / BM);
+        push_bst({false, 0, 0, 0, 0, 1, 1, 1});
         return out;
     }
     struct Geo {
@@ -629,22 +757,30 @@ static std::vector<Config> configs(const Layer &l, const Shape &in, sn_schema s,
     for (int gi = 0; gi < keep; ++gi) {
         const Geo &gg = gs[gi];
         const int64_t mtiles = ((Q + gg.bw - 1) / gg.bw) * ((P + gg.bh - 1) / gg.bh) * ((N + gg.bni - 1) / gg.bni);
-        if (a_blocks > 0)
+        if (a_blocks > 0) {
             out.push_back({true, 64, gg.bw, gg.bh, gg.bni, 1, 1, a_blocks});
-        else
+        } else {
             push_all({true, 0, gg.bw, gg.bh, gg.bni, 1, 1, 1}, mtiles);
+            push_bst({true, 0, gg.bw, gg.bh, gg.bni, 1, 1, 1});
+        }
     }
     return out;
 }
 
-template <typename T, int BN, bool IMPLICIT, int G, int KB>
+template <typename T, int BN, bool IMPLICIT, int G, int KB, bool BST = false>
 static cudaError_t launch(const CUtensorMap *mA, const CUtensorMap &mB, const CUtensorMap &mY, const CUtensorMap &mR,
                           const Params &p,
                           cudaStream_t st) {
-    constexpr int STAGES = stages_for(BN, G, KB);
-    constexpr size_t smem = (size_t)STAGES * KB * (BM * BK * 2 + (BN / G) * BK * 2) + EPI_WARPS * STG_BYTES + 1024;
-    static_assert(smem <= 227 * 1024, "shared memory per CTA");
-    auto kern = conv_tc_kernel<T, BN, STAGES, IMPLICIT, G, KB>;
+    constexpr int STAGES = BST ? BST_STAGES : stages_for(BN, G, KB);
+    constexpr size_t smem_max = 227 * 1024;
+    const size_t smem = BST ? (size_t)STAGES * BM * BK * 2 + p.bst_bytes + EPI_WARPS * STG_BYTES + 1024
+                            : (size_t)STAGES * KB * (BM * BK * 2 + (BN / G) * BK * 2) + EPI_WARPS * STG_BYTES + 1024;
+    static_assert(BST || (size_t)STAGES * KB * (BM * BK * 2 + (BN / G) * BK * 2) + EPI_WARPS * STG_BYTES + 1024 <=
+                             smem_max,
+                  "shared memory per CTA");
+    static_assert(!BST || (G == 1 && KB == 1), "weight-stationary tiles are one-CTA, one block per stage");
+    if (smem > smem_max) return cudaErrorInvalidValue;
+    auto kern = conv_tc_kernel<T, BN, STAGES, IMPLICIT, G, KB, BST>;
     static int max_groups = 0;  // co-resident CTAs (G = 1) or CTA pairs (G = 2)
     cudaLaunchConfig_t cfg = {};
     cudaLaunchAttribute attr[2];
@@ -662,9 +798,14 @@ static cudaError_t launch(const CUtensorMap *mA, const CUtensorMap &mB, const CU
         attr[1].val.clusterDim.z = 1;
         cfg.numAttrs = 2;
     }
-    if (!max_groups) {
+    static size_t smem_set = 0;  // dynamic shared memory the kernel is currently allowed
+    if (smem > smem_set) {
         cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
+        smem_set = smem;
+    }
+    if (!max_groups) {
+        cudaError_t e = cudaSuccess;
         if (G == 2) {
             cudaLaunchConfig_t q = cfg;  // the cluster shape alone
             q.gridDim = dim3(2);
@@ -733,6 +874,10 @@ cudaError_t conv_tc(const LaunchArgs &a) {
     p.M = in.n * (int64_t)in.h * in.w;
     p.Mout = (int64_t)p.N * p.P * p.Q;
     p.ntiles = (p.K + cf.BN - 1) / cf.BN;
+    if (cf.bst) {
+        if (p.ntiles != 1 || cf.ksplit != 1 || cf.G != 1 || cf.KB != 1) return cudaErrorInvalidValue;
+        p.bst_bytes = p.kiters * cf.BN * BK * 2;
+    }
     if (cf.ksplit > 1) {
         const size_t need = (size_t)cf.ksplit * p.Mout * p.K * sizeof(float);
         if (!a.ws || a.ws_bytes < need || (uintptr_t)a.ws % 16) return cudaErrorInvalidValue;
@@ -824,6 +969,16 @@ cudaError_t conv_tc(const LaunchArgs &a) {
     return cf.implicit ? launch<TT, BNV, true, GV, KBV>(mA, mB, mY, mR, p, a.stream)               \
                        : launch<TT, BNV, false, GV, KBV>(mA, mB, mY, mR, p, a.stream)
 #define SN_TC_LAUNCH_T(TT)                                                                          \
+    if (cf.bst) {                                                                                   \
+        if (cf.implicit) {                                                                          \
+            if (cf.BN == 64) return launch<TT, 64, true, 1, 1, true>(mA, mB, mY, mR, p, a.stream);  \
+            if (cf.BN == 128) return launch<TT, 128, true, 1, 1, true>(mA, mB, mY, mR, p, a.stream);\
+            return launch<TT, 256, true, 1, 1, true>(mA, mB, mY, mR, p, a.stream);                  \
+        }                                                                                           \
+        if (cf.BN == 64) return launch<TT, 64, false, 1, 1, true>(mA, mB, mY, mR, p, a.stream);     \
+        if (cf.BN == 128) return launch<TT, 128, false, 1, 1, true>(mA, mB, mY, mR, p, a.stream);   \
+        return launch<TT, 256, false, 1, 1, true>(mA, mB, mY, mR, p, a.stream);                     \
+    }                                                                                               \
     if (cf.G == 1 && cf.KB > 1) {                                                                   \
         if (!cf.implicit || cf.BN != 64) return cudaErrorInvalidValue;                              \
         if (cf.KB == 2) return launch<TT, 64, true, 1, 2>(mA, mB, mY, mR, p, a.stream);            \

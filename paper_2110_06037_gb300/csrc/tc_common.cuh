@@ -17,13 +17,26 @@ constexpr int BK = 64;
 // sub-partition leave the epilogue up to 168 registers a thread.
 constexpr int THREADS = 384;
 // TMA producer threads for a ring of `stages` stages: one issuing thread
-// walks the stages s with s % n == its index, so n must divide the depth
-constexpr int producers_for(int stages) { return stages % 3 == 0 ? 3 : 2; }
+// walks the stages s with s % n == its index, so n must divide the depth.
+// Two for an even depth; the third producer warp then waits on the MMA
+// issuer's barriers for it (see waits_for_mma).
+constexpr int producers_for(int stages) { return stages % 2 == 0 ? 2 : 3; }
+// A shared-memory access by the MMA-issuing thread (an mbarrier wait included)
+// queues behind the tensor core's operand reads and costs ~250 cycles, as much
+// as four MMAs: with an even ring depth, warp 11 waits on the stage-full and
+// accumulator-drained barriers instead and hands each result to the MMA warp
+// through a hardware named barrier (bar.red.or: both warps pass it together,
+// and the OR of their predicates tells both whether to stop).
+constexpr bool waits_for_mma(int stages) { return producers_for(stages) == 2; }
+constexpr uint32_t BAR_MMA = 1;  // named barrier of the MMA warp and its waiter (0 is __syncthreads)
 // pipeline depth: as many stages of KB 64-channel blocks as fit beside the
 // epilogue staging (227 KB - 32 KB staging - 1 KB alignment slack)
 constexpr int stages_for(int bn, int g, int kb) {
     return 198656 / (kb * (16384 + bn / g * 128)) < 8 ? 198656 / (kb * (16384 + bn / g * 128)) : 8;
 }
+// weight-stationary tiles: the layer's whole B (K steps x BN rows x 128 B) is
+// loaded once per CTA and stays in shared memory beside this many A stages
+constexpr int BST_STAGES = 4;
 constexpr int EPI_WARPS = 8;
 constexpr int MAX_K = 65536;
 constexpr uint32_t STG_BYTES = 32 * 64 * 2;      // one epilogue staging block: 32 rows x 64 channels
@@ -41,6 +54,7 @@ struct Params {
     int64_t M;                     // plain mode: input rows (= output pixels)
     int64_t Mout;                  // output pixels N * P * Q
     int32_t act;
+    int32_t bst_bytes;             // weight-stationary: bytes of the resident B (0 otherwise)
     const float *bias;             // fp32 [K], zero-padded to a multiple of 256 entries
     void *y;                       // output, NHWC, fp16/bf16
     const void *res;               // residual added before the activation (output's layout), or null
@@ -300,6 +314,20 @@ __device__ __forceinline__ float2 unpack2<__nv_bfloat16>(uint32_t v) {
 
 
 
+// named barrier `id` over `count` threads (whole warps) that also ORs a
+// predicate across them; every participant gets the result
+__device__ __forceinline__ bool bar_red_or(uint32_t id, uint32_t count, bool pred) {
+    uint32_t r;
+    asm volatile(
+        "{\n\t.reg .pred pi, po;\n\t"
+        "setp.ne.u32 pi, %1, 0;\n\t"
+        "bar.red.or.pred po, %2, %3, pi;\n\t"
+        "selp.u32 %0, 1, 0, po;\n\t}"
+        : "=r"(r)
+        : "r"((uint32_t)pred), "r"(id), "r"(count)
+        : "memory");
+    return r != 0;
+}
 __device__ __forceinline__ void mbar_arrive(uint64_t *b) {
     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(su32(b)) : "memory");
 }
