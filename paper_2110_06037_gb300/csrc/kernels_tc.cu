@@ -685,7 +685,7 @@ static std::vector<Config> configs(const Layer &l, const Shape &in, sn_schema s,
     const bool plain = c.kh == 1 && c.kw == 1 && c.sh == 1 && c.ph == 0 && c.pw == 0;
     const int64_t N = l.out.n, P = l.out.h, Q = l.out.w;
     // one-CTA tiles (128 x BN) with K splits of {1, 2, 4}; CTA-pair tiles
-    // (256 x BN, BN >= 128) with K splits of {1, 2, 3, 4}; a split is offered
+    // (256 x BN) with K splits of {1, 2, 3, 4}; a split is offered
     // while the units stay within two waves of the GPU and each part keeps
     // at least four K steps
     auto push_splits = [&](Config cf, int64_t mtiles) {
@@ -707,15 +707,16 @@ static std::vector<Config> configs(const Layer &l, const Shape &in, sn_schema s,
             cf.G = 1;
             push_splits(cf, mtiles);
         }
-        for (int bn : bns)
-            if (bn >= 128) {
-                cf.BN = bn;
-                cf.G = 2;
-                // two channel blocks per stage when the channels split evenly
-                cf.KB = c.c_in % 128 == 0 ? 2 : 1;
-                push_splits(cf, mtiles);
-                cf.KB = 1;
-            }
+        for (int bn : bns) {
+            // a pair issues one MMA for both SMs: twice the work per issued
+            // instruction, half the B rows staged per SM
+            cf.BN = bn;
+            cf.G = 2;
+            // two channel blocks per stage when the channels split evenly
+            cf.KB = c.c_in % 128 == 0 ? 2 : 1;
+            push_splits(cf, mtiles);
+            cf.KB = 1;
+        }
     };
     // weight-stationary variant: the whole B of a one-N-tile layer fits in
     // shared memory beside BST_STAGES A stages and the epilogue staging
@@ -987,9 +988,11 @@ cudaError_t conv_tc(const LaunchArgs &a) {
     }                                                                                               \
     if (cf.G == 2) {                                                                                \
         if (cf.KB == 2) {                                                                           \
+            if (cf.BN == 64) SN_TC_LAUNCH(TT, 64, 2, 2);                                            \
             if (cf.BN == 128) SN_TC_LAUNCH(TT, 128, 2, 2);                                          \
             SN_TC_LAUNCH(TT, 256, 2, 2);                                                            \
         }                                                                                           \
+        if (cf.BN == 64) SN_TC_LAUNCH(TT, 64, 2, 1);                                                \
         if (cf.BN == 128) SN_TC_LAUNCH(TT, 128, 2, 1);                                              \
         SN_TC_LAUNCH(TT, 256, 2, 1);                                                                \
     }                                                                                               \
