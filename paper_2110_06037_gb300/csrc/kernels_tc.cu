@@ -706,6 +706,13 @@ static std::vector<Config> configs(const Layer &l, const Shape &in, sn_schema s,
             cf.BN = bn;
             cf.G = 1;
             push_splits(cf, mtiles);
+            // two channel blocks per box: a TMA box costs the SM ~400 cycles
+            // whatever its size (up to 32 KB), so fewer, larger boxes
+            if (bn <= 128 && c.c_in % 128 == 0) {
+                cf.KB = 2;
+                push_splits(cf, mtiles);
+                cf.KB = 1;
+            }
         }
         for (int bn : bns) {
             // a pair issues one MMA for both SMs: twice the work per issued
@@ -981,9 +988,13 @@ cudaError_t conv_tc(const LaunchArgs &a) {
         return launch<TT, 256, false, 1, 1, true>(mA, mB, mY, mR, p, a.stream);                     \
     }                                                                                               \
     if (cf.G == 1 && cf.KB > 1) {                                                                   \
-        if (!cf.implicit || cf.BN != 64) return cudaErrorInvalidValue;                              \
-        if (cf.KB == 2) return launch<TT, 64, true, 1, 2>(mA, mB, mY, mR, p, a.stream);            \
-        if (cf.KB == 4) return launch<TT, 64, true, 1, 4>(mA, mB, mY, mR, p, a.stream);            \
+        if (cf.KB == 4) {                                                                           \
+            if (!cf.implicit || cf.BN != 64) return cudaErrorInvalidValue;                          \
+            return launch<TT, 64, true, 1, 4>(mA, mB, mY, mR, p, a.stream);                         \
+        }                                                                                           \
+        if (cf.KB != 2) return cudaErrorInvalidValue;                                               \
+        if (cf.BN == 64) SN_TC_LAUNCH(TT, 64, 1, 2);                                                \
+        if (cf.BN == 128) SN_TC_LAUNCH(TT, 128, 1, 2);                                              \
         return cudaErrorInvalidValue;                                                               \
     }                                                                                               \
     if (cf.G == 2) {                                                                                \
