@@ -53,7 +53,7 @@ namespace tc {
 // shared memory, and each CTA's TMEM receives its own 128 rows, drained by
 // its own epilogue.  Per SM this halves the weight bytes staged and read per
 // MMA, the shared-memory bandwidth that limits a one-CTA tile.
-template <typename T, int BN, int STAGES, bool IMPLICIT, int G, int KB, bool BST>
+template <typename T, int BN, int STAGES, bool IMPLICIT, int G, int KB, bool BST, int MS>
 __global__ void __launch_bounds__(THREADS, 1)
     conv_tc_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ CUtensorMap mA1,
                    const __grid_constant__ CUtensorMap mA2, const __grid_constant__ CUtensorMap mA3,
@@ -61,14 +61,17 @@ __global__ void __launch_bounds__(THREADS, 1)
                    const __grid_constant__ CUtensorMap mR, const Params p) {
     // a stage holds KB 64-channel blocks of one filter tap; a block of A is
     // 128 rows x 128 B, of B (BN / G) rows x 128 B (this CTA's share)
-    constexpr uint32_t A_BLK = BM * BK * 2;
+    // MS = 2: a one-CTA tile of 256 rows, one TMA box of A for both 128-row
+    // halves and two MMAs (one per half, one TMEM accumulator each) sharing B
+    constexpr uint32_t A_SUB = BM * BK * 2;  // one 128-row half
+    constexpr uint32_t A_BLK = MS * A_SUB;
     constexpr uint32_t B_BLK = (BN / G) * BK * 2;
     constexpr uint32_t A_BYTES = KB * A_BLK;
     constexpr uint32_t B_BYTES = KB * B_BLK;
     // BST (weight-stationary, G = 1, one N tile, no K split): a stage holds A
     // only; B of every K step sits after the stages for the whole kernel
     constexpr uint32_t STAGE_BYTES = BST ? A_BYTES : A_BYTES + B_BYTES;
-    constexpr uint32_t TMEM_COLS = 2 * BN;  // two accumulators
+    constexpr uint32_t TMEM_COLS = 2 * MS * BN;  // two accumulators (of MS halves each)
     extern __shared__ uint8_t smem_raw[];
     __shared__ __align__(8) uint64_t full_bar[STAGES];
     __shared__ __align__(8) uint64_t empty_bar[STAGES];
@@ -107,7 +110,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         for (int b = 0; b < 2; ++b) {
             mbar_init(&accf_bar[b], 1);
             // one arrival per epilogue warp draining it, in both CTAs of a pair
-            mbar_init(&acce_bar[b], G * (BN >= 128 ? EPI_WARPS : EPI_WARPS / 2));
+            mbar_init(&acce_bar[b], G * (BN >= 128 || MS == 2 ? EPI_WARPS : EPI_WARPS / 2));
         }
         for (int i = 0; i < EPI_WARPS; ++i) {
             mbar_init(&res_bar[i], 1);
@@ -141,7 +144,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             uint32_t par = 0;
             bool stop = false;
             for (int u = cid; u < total && !stop; u += ncl, ++lt) {
-                const Work w = work_of(p, u, BN, IMPLICIT, G, 0);
+                const Work w = work_of(p, u, BN, IMPLICIT, G, MS, 0);
                 const int b = lt & 1;
                 const uint32_t aph = (uint32_t)(lt >> 1) & 1u;
                 bool ok = G == 2 ? mbar_wait_cluster(&acce_bar[b], aph ^ 1u) : mbar_wait(&acce_bar[b], aph ^ 1u);
@@ -195,7 +198,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                 }
             }
             for (int u = cid; u < total && !stop; u += ncl) {
-                const Work w = work_of(p, u, BN, IMPLICIT, G, (int)rank);
+                const Work w = work_of(p, u, BN, IMPLICIT, G, MS, (int)rank);
                 int tap = (int)fdiv((uint32_t)w.it0, p.fd_spt);
                 int cb = (w.it0 - tap * p.fd_spt.d) * KB;
                 int r = (int)fdiv((uint32_t)tap, p.fd_S), ss = tap - r * S;
@@ -279,11 +282,11 @@ __global__ void __launch_bounds__(THREADS, 1)
             }
             __syncwarp();
             for (int u = cid; u < total && !stop; u += ncl, ++lt) {
-                const Work w = work_of(p, u, BN, IMPLICIT, G, 0);
+                const Work w = work_of(p, u, BN, IMPLICIT, G, MS, 0);
                 const int b = lt & 1;
                 if (bar_red_or(BAR_MMA, 64, false)) break;  // accumulator b drained
                 tc_fence_after();
-                const uint32_t d = tmem + (uint32_t)(b * BN);
+                const uint32_t d = tmem + (uint32_t)(b * MS * BN);
                 for (int it = w.it0; it < w.it1; ++it, ++g) {
                     if (bar_red_or(BAR_MMA, 64, false)) {  // stage s full
                         stop = true;
@@ -299,8 +302,11 @@ __global__ void __launch_bounds__(THREADS, 1)
                         for (int j = 0; j < KB; ++j)
 #pragma unroll
                             for (int k = 0; k < BK / 16; ++k)
-                                umma<G>(d, da + j * (A_BLK >> 4) + 2 * k, db + j * (B_BLK >> 4) + 2 * k, idesc,
-                                        (it > w.it0 || j > 0 || k > 0) ? 1u : 0u);
+#pragma unroll
+                                for (int m = 0; m < MS; ++m)
+                                    umma<G>(d + (uint32_t)(m * BN), da + j * (A_BLK >> 4) + m * (A_SUB >> 4) + 2 * k,
+                                            db + j * (B_BLK >> 4) + 2 * k, idesc,
+                                            (it > w.it0 || j > 0 || k > 0) ? 1u : 0u);
                         umma_commit<G>(&empty_bar[s]);  // frees the stage (in both CTAs) once read
                     }
                     __syncwarp();
@@ -325,7 +331,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                 stop = true;
             }
             for (int u = cid; u < total && !stop; u += ncl, ++lt) {
-                const Work w = work_of(p, u, BN, IMPLICIT, G, 0);
+                const Work w = work_of(p, u, BN, IMPLICIT, G, MS, 0);
                 const int b = lt & 1;
                 const uint32_t aph = (uint32_t)(lt >> 1) & 1u;
                 const bool drained = G == 2 ? mbar_wait_cluster(&acce_bar[b], aph ^ 1u) : mbar_wait(&acce_bar[b], aph ^ 1u);
@@ -335,7 +341,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                     break;
                 }
                 tc_fence_after();
-                const uint32_t d = tmem + (uint32_t)(b * BN);
+                const uint32_t d = tmem + (uint32_t)(b * MS * BN);
                 for (int it = w.it0; it < w.it1; ++it, ++g) {
                     if (!mbar_wait(&full_bar[s], par)) {
                         atomicOr(p.err, ERR_MMA_WAIT);
@@ -351,8 +357,11 @@ __global__ void __launch_bounds__(THREADS, 1)
                     for (int j = 0; j < KB; ++j)
 #pragma unroll
                         for (int k = 0; k < BK / 16; ++k)
-                            umma<G>(d, da + j * (A_BLK >> 4) + 2 * k, db + j * (B_BLK >> 4) + 2 * k, idesc,
-                                    (it > w.it0 || j > 0 || k > 0) ? 1u : 0u);
+#pragma unroll
+                            for (int m = 0; m < MS; ++m)
+                                umma<G>(d + (uint32_t)(m * BN), da + j * (A_BLK >> 4) + m * (A_SUB >> 4) + 2 * k,
+                                        db + j * (B_BLK >> 4) + 2 * k, idesc,
+                                        (it > w.it0 || j > 0 || k > 0) ? 1u : 0u);
                     umma_commit<G>(&empty_bar[s]);  // frees the stage (in both CTAs) once read
                     if (++s == STAGES) {
                         s = 0;
@@ -368,25 +377,27 @@ __global__ void __launch_bounds__(THREADS, 1)
         // more 64-channel chunks: all eight warps drain every unit, warp w the
         // chunks of column half (w-2)/4.  One-chunk tiles (BN = 64): the two
         // groups of four take alternate units, i.e. one accumulator each.
+        // Two-half tiles (MS = 2): group (w-2)/4 drains half (w-2)/4, all chunks.
         const int half = (warp - 2) >> 2;
         const int g4 = warp & 3;
-        const int row = g4 * 32 + lane;
+        const int msub = MS == 2 ? half : 0;          // the 128-row half this warp drains
+        const int row = msub * BM + g4 * 32 + lane;    // row within the unit's tile
         uint8_t *buf = stg + (warp - 2) * STG_BYTES;  // one 32 x 64 staging block per warp
-        const int r0 = g4 * 32;
+        const int r0 = msub * BM + g4 * 32;
         const int wq0 = IMPLICIT ? r0 & (p.BW - 1) : 0;
         const int hp0 = IMPLICIT ? (r0 >> p.lbw) & (p.BH - 1) : 0;
         const int ni0 = IMPLICIT ? r0 >> p.lbwh : 0;
         constexpr int NCH = BN / 64 > 0 ? BN / 64 : 1;  // 64-channel chunks per tile
-        constexpr int CPH = NCH >= 2 ? NCH / 2 : 1;      // chunks per column half
-        constexpr bool ALT = NCH == 1;                   // alternate units between the groups
-        const int cbase = ALT ? 0 : half * CPH;          // first chunk of this warp
+        constexpr int CPH = MS == 2 ? NCH : (NCH >= 2 ? NCH / 2 : 1);  // chunks this warp drains
+        constexpr bool ALT = NCH == 1 && MS == 1;        // alternate units between the groups
+        const int cbase = (ALT || MS == 2) ? 0 : half * CPH;  // first chunk of this warp
         int lt = ALT ? half : 0;
         uint32_t rpar = 0;  // phase parity of this warp's residual barrier
         bool waited = false;
         for (int u = cid + (ALT ? half * ncl : 0); u < total; u += (ALT ? 2 : 1) * ncl, lt += ALT ? 2 : 1) {
             const int b = lt & 1;
             const uint32_t aph = (uint32_t)(lt >> 1) & 1u;
-            const Work w = work_of(p, u, BN, IMPLICIT, G, (int)rank);
+            const Work w = work_of(p, u, BN, IMPLICIT, G, MS, (int)rank);
             // bias of this warp's channels (lane j holds channel chunk + 32h + j;
             // the buffer is zero-padded to a multiple of 256 channels), loaded
             // before the accumulator wait so that the latency is hidden
@@ -444,7 +455,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                 const int ci = cbase + cj;
                 const int k0 = w.n0 + 64 * ci;
                 if (k0 >= p.K || !tile_live) break;
-                const uint32_t taddr = tmem + ((uint32_t)(g4 * 32) << 16) + (uint32_t)(b * BN + 64 * ci);
+                const uint32_t taddr = tmem + ((uint32_t)(g4 * 32) << 16) + (uint32_t)((b * MS + msub) * BN + 64 * ci);
                 if (p.ksplit == 1) {
                     // bias + activation -> 16-bit, staged with the 128-byte swizzle
                     // (row = lane, 16-byte chunk j at j ^ (row & 7)), then one TMA
@@ -660,6 +671,7 @@ struct Config {
     int G;   // CTAs per tile: 1, or 2 (CTA pair, 256-pixel tile)
     int KB;  // 64-channel blocks per pipeline stage (one TMA box spans them)
     bool bst = false;  // weight-stationary: B loaded once per CTA (one N tile, G = 1, no split)
+    int ms = 1;        // 128-row halves per one-CTA tile (2: 256 x BN, one A box, B shared)
 };
 
 constexpr int kSmCount = 152;  // GB300; only used to decide which K splits to offer
@@ -740,55 +752,77 @@ static std::vector<Config> configs(const Layer &l, const Shape &in, sn_schema s,
                 break;
             }
     };
+    // 256-row one-CTA tiles for 64- and 128-channel N tiles: one 32 KB A box
+    // per stage for two MMAs that share B (the SM's TMA issue, not bytes, is
+    // what small tiles run out of)
+    auto push_ms2 = [&](Config cf, int64_t mtiles256) {
+        for (int bn : bns)
+            if (bn <= 128) {
+                cf.BN = bn, cf.G = 1, cf.KB = 1, cf.ms = 2;
+                push_splits(cf, mtiles256);
+            }
+    };
     if (plain && a_blocks == 0) {
         push_all({false, 0, 0, 0, 0, 1, 1, 1}, (N * P * Q + BM - 1) / BM);
         push_bst({false, 0, 0, 0, 0, 1, 1, 1});
+        push_ms2({false, 0, 0, 0, 0, 1, 1, 1}, (N * P * Q + 2 * BM - 1) / (2 * BM));
         return out;
     }
     struct Geo {
         double waste;
         int bw, bh, bni;
     };
-    std::vector<Geo> gs;
-    for (int bw = 1; bw <= 128; bw *= 2)
-        for (int bh = 1; bw * bh <= 128; bh *= 2) {
-            const int bni = 128 / (bw * bh);
-            const double cover = (double)((Q + bw - 1) / bw * bw) * ((P + bh - 1) / bh * bh) * ((N + bni - 1) / bni * bni);
-            gs.push_back({cover / (double)(N * P * Q), bw, bh, bni});
-        }
-    std::sort(gs.begin(), gs.end(), [](const Geo &a, const Geo &b) {
-        if (a.waste != b.waste) return a.waste < b.waste;
-        if (a.bw != b.bw) return a.bw > b.bw;
-        return a.bh > b.bh;
-    });
-    const int keep = std::min<int>(2, (int)gs.size());
-    for (int gi = 0; gi < keep; ++gi) {
-        const Geo &gg = gs[gi];
-        const int64_t mtiles = ((Q + gg.bw - 1) / gg.bw) * ((P + gg.bh - 1) / gg.bh) * ((N + gg.bni - 1) / gg.bni);
+    // box geometries of `tm` pixels (powers of two), least padding first
+    auto geos = [&](int tm) {
+        std::vector<Geo> gs;
+        for (int bw = 1; bw <= tm && bw <= 256; bw *= 2)
+            for (int bh = 1; bw * bh <= tm && bh <= 256; bh *= 2) {
+                const int bni = tm / (bw * bh);
+                if (bni > 256) continue;
+                const double cover =
+                    (double)((Q + bw - 1) / bw * bw) * ((P + bh - 1) / bh * bh) * ((N + bni - 1) / bni * bni);
+                gs.push_back({cover / (double)(N * P * Q), bw, bh, bni});
+            }
+        std::sort(gs.begin(), gs.end(), [](const Geo &a, const Geo &b) {
+            if (a.waste != b.waste) return a.waste < b.waste;
+            if (a.bw != b.bw) return a.bw > b.bw;
+            return a.bh > b.bh;
+        });
+        if (gs.size() > 2) gs.resize(2);
+        return gs;
+    };
+    auto tiles_of = [&](const Geo &gg) {
+        return ((Q + gg.bw - 1) / gg.bw) * ((P + gg.bh - 1) / gg.bh) * ((N + gg.bni - 1) / gg.bni);
+    };
+    for (const Geo &gg : geos(BM)) {
         if (a_blocks > 0) {
             out.push_back({true, 64, gg.bw, gg.bh, gg.bni, 1, 1, a_blocks});
         } else {
-            push_all({true, 0, gg.bw, gg.bh, gg.bni, 1, 1, 1}, mtiles);
+            push_all({true, 0, gg.bw, gg.bh, gg.bni, 1, 1, 1}, tiles_of(gg));
             push_bst({true, 0, gg.bw, gg.bh, gg.bni, 1, 1, 1});
         }
     }
+    if (a_blocks == 0)
+        for (const Geo &gg : geos(2 * BM)) push_ms2({true, 0, gg.bw, gg.bh, gg.bni, 1, 1, 1}, tiles_of(gg));
     return out;
 }
 
-template <typename T, int BN, bool IMPLICIT, int G, int KB, bool BST = false>
+template <typename T, int BN, bool IMPLICIT, int G, int KB, bool BST = false, int MS = 1>
 static cudaError_t launch(const CUtensorMap *mA, const CUtensorMap &mB, const CUtensorMap &mY, const CUtensorMap &mR,
                           const Params &p,
                           cudaStream_t st) {
-    constexpr int STAGES = BST ? BST_STAGES : stages_for(BN, G, KB);
+    constexpr int STAGES = BST ? BST_STAGES : stages_for(BN, G, KB, MS);
     constexpr size_t smem_max = 227 * 1024;
     const size_t smem = BST ? (size_t)STAGES * BM * BK * 2 + p.bst_bytes + EPI_WARPS * STG_BYTES + 1024
-                            : (size_t)STAGES * KB * (BM * BK * 2 + (BN / G) * BK * 2) + EPI_WARPS * STG_BYTES + 1024;
-    static_assert(BST || (size_t)STAGES * KB * (BM * BK * 2 + (BN / G) * BK * 2) + EPI_WARPS * STG_BYTES + 1024 <=
-                             smem_max,
+                            : (size_t)STAGES * KB * (MS * BM * BK * 2 + (BN / G) * BK * 2) + EPI_WARPS * STG_BYTES + 1024;
+    static_assert(BST ||
+                      (size_t)STAGES * KB * (MS * BM * BK * 2 + (BN / G) * BK * 2) + EPI_WARPS * STG_BYTES + 1024 <=
+                          smem_max,
                   "shared memory per CTA");
-    static_assert(!BST || (G == 1 && KB == 1), "weight-stationary tiles are one-CTA, one block per stage");
+    static_assert(!BST || (G == 1 && KB == 1 && MS == 1), "weight-stationary tiles are one-CTA, one block per stage");
+    static_assert(MS == 1 || (G == 1 && KB == 1 && !BST && 2 * MS * BN <= 512), "two-half tiles: one CTA, TMEM");
     if (smem > smem_max) return cudaErrorInvalidValue;
-    auto kern = conv_tc_kernel<T, BN, STAGES, IMPLICIT, G, KB, BST>;
+    auto kern = conv_tc_kernel<T, BN, STAGES, IMPLICIT, G, KB, BST, MS>;
     static int max_groups = 0;  // co-resident CTAs (G = 1) or CTA pairs (G = 2)
     cudaLaunchConfig_t cfg = {};
     cudaLaunchAttribute attr[2];
@@ -908,10 +942,10 @@ cudaError_t conv_tc(const LaunchArgs &a) {
     if (!cf.implicit) {
         const uint64_t dims[3] = {blk ? 64 : (uint64_t)p.C, (uint64_t)p.M, CB};
         const uint64_t str[2] = {p.C * es, 128};
-        const uint32_t box[3] = {BK, BM, (uint32_t)cf.KB};
+        const uint32_t box[3] = {BK, (uint32_t)(BM * cf.ms), (uint32_t)cf.KB};
         if (!encode(&mA[0], dt, blk ? 3 : 2, a.in[0], dims, str, box)) return cudaErrorInvalidValue;
         mA[1] = mA[2] = mA[3] = mA[0];
-        p.mtiles = (int)((p.M + BM - 1) / BM);
+        p.mtiles = (int)((p.M + BM * cf.ms - 1) / (BM * cf.ms));
         // output [Mout][K], one 32-row x 64-channel box per epilogue-warp chunk
         const uint64_t ydims[2] = {(uint64_t)p.K, (uint64_t)p.Mout};
         const uint64_t ystr[1] = {p.K * es};
@@ -977,6 +1011,17 @@ cudaError_t conv_tc(const LaunchArgs &a) {
     return cf.implicit ? launch<TT, BNV, true, GV, KBV>(mA, mB, mY, mR, p, a.stream)               \
                        : launch<TT, BNV, false, GV, KBV>(mA, mB, mY, mR, p, a.stream)
 #define SN_TC_LAUNCH_T(TT)                                                                          \
+    if (cf.ms == 2) {                                                                               \
+        if (cf.G != 1 || cf.KB != 1 || cf.bst) return cudaErrorInvalidValue;                        \
+        if (cf.implicit) {                                                                          \
+            if (cf.BN == 64) return launch<TT, 64, true, 1, 1, false, 2>(mA, mB, mY, mR, p, a.stream); \
+            if (cf.BN == 128) return launch<TT, 128, true, 1, 1, false, 2>(mA, mB, mY, mR, p, a.stream); \
+            return cudaErrorInvalidValue;                                                           \
+        }                                                                                           \
+        if (cf.BN == 64) return launch<TT, 64, false, 1, 1, false, 2>(mA, mB, mY, mR, p, a.stream); \
+        if (cf.BN == 128) return launch<TT, 128, false, 1, 1, false, 2>(mA, mB, mY, mR, p, a.stream); \
+        return cudaErrorInvalidValue;                                                               \
+    }                                                                                               \
     if (cf.bst) {                                                                                   \
         if (cf.implicit) {                                                                          \
             if (cf.BN == 64) return launch<TT, 64, true, 1, 1, true>(mA, mB, mY, mR, p, a.stream);  \

@@ -31,8 +31,8 @@ constexpr bool waits_for_mma(int stages) { return producers_for(stages) == 2; }
 constexpr uint32_t BAR_MMA = 1;  // named barrier of the MMA warp and its waiter (0 is __syncthreads)
 // pipeline depth: as many stages of KB 64-channel blocks as fit beside the
 // epilogue staging (227 KB - 32 KB staging - 1 KB alignment slack)
-constexpr int stages_for(int bn, int g, int kb) {
-    return 198656 / (kb * (16384 + bn / g * 128)) < 8 ? 198656 / (kb * (16384 + bn / g * 128)) : 8;
+constexpr int stages_for(int bn, int g, int kb, int ms = 1) {
+    return 198656 / (kb * (16384 * ms + bn / g * 128)) < 8 ? 198656 / (kb * (16384 * ms + bn / g * 128)) : 8;
 }
 // weight-stationary tiles: the layer's whole B (K steps x BN rows x 128 B) is
 // loaded once per CTA and stays in shared memory beside this many A stages
@@ -361,7 +361,7 @@ struct Work {
 // work unit u: K-split part sp of output-channel tile nt of pixel-tile group
 // mg; a group is `ctas` consecutive pixel tiles (one per CTA of a pair), and
 // units sharing a group are adjacent so that their A tiles are reused in L2
-__device__ __forceinline__ Work work_of(const Params &p, int u, int bn, bool implicit, int ctas = 1,
+__device__ __forceinline__ Work work_of(const Params &p, int u, int bn, bool implicit, int ctas, int ms,
                                         int rank = 0) {
     Work w;
     const int t = (int)fdiv((uint32_t)u, p.fd_ksplit);
@@ -384,7 +384,7 @@ __device__ __forceinline__ Work work_of(const Params &p, int u, int bn, bool imp
         w.p0 = bp * p.BH;
         w.i0 = bx * p.BNI;
     } else {
-        w.m0 = (int64_t)mt * BM;
+        w.m0 = (int64_t)mt * BM * ms;
     }
     w.it0 = (int)fdiv((uint32_t)(w.sp * p.kiters), p.fd_ksplit);
     w.it1 = (int)fdiv((uint32_t)((w.sp + 1) * p.kiters), p.fd_ksplit);
