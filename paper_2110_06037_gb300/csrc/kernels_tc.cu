@@ -53,7 +53,7 @@ namespace tc {
 // shared memory, and each CTA's TMEM receives its own 128 rows, drained by
 // its own epilogue.  Per SM this halves the weight bytes staged and read per
 // MMA, the shared-memory bandwidth that limits a one-CTA tile.
-template <typename T, int BN, int STAGES, bool IMPLICIT, int G, int KB, bool BST, int MS>
+template <typename T, int BN, int STAGES, bool IMPLICIT, int G, int KB, bool BST, int MS, int CSK>
 __global__ void __launch_bounds__(THREADS, 1)
     conv_tc_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ CUtensorMap mA1,
                    const __grid_constant__ CUtensorMap mA2, const __grid_constant__ CUtensorMap mA3,
@@ -79,6 +79,11 @@ __global__ void __launch_bounds__(THREADS, 1)
     __shared__ __align__(8) uint64_t acce_bar[2];  // epilogue -> MMA: accumulator drained
     __shared__ __align__(8) uint64_t res_bar[EPI_WARPS];  // residual tile landed in a warp's staging block
     __shared__ __align__(8) uint64_t bst_bar;              // weight-stationary B landed
+    // CSK = 2 (cluster K split): the two CTAs of a cluster take the two halves
+    // of a tile's K steps; CTA 1's epilogue warps write their fp32 partial
+    // rows into CTA 0's exchange blocks (distributed shared memory)
+    __shared__ __align__(8) uint64_t xfull_bar[EPI_WARPS];  // CTA 0: a partial block landed
+    __shared__ __align__(8) uint64_t xfree_bar[EPI_WARPS];  // CTA 1: CTA 0 has read the block
     __shared__ uint32_t tmem_sh;
     __shared__ volatile int abort_sh;
     __shared__ int issued_sh[4], consumed_sh;
@@ -87,16 +92,28 @@ __global__ void __launch_bounds__(THREADS, 1)
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t *bst = smem + STAGES * STAGE_BYTES;  // weight-stationary B (BST), 1024-B aligned
     uint8_t *stg = bst + (BST ? p.bst_bytes : 0);  // epilogue staging: one block per warp, 1024-B aligned
+    uint8_t *xbuf = stg + EPI_WARPS * STG_BYTES;   // CSK: 32 x 64 fp32 exchange block per warp (XBLK_BYTES)
+    constexpr bool CLUSTER = G == 2 || CSK == 2;
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-    const uint32_t rank = G == 2 ? cluster_rank() : 0u;
+    const uint32_t crank = CLUSTER ? cluster_rank() : 0u;
+    const uint32_t rank = G == 2 ? crank : 0u;    // rank within a CTA pair (B rows, MMA issue)
+    const uint32_t krank = CSK == 2 ? crank : 0u;  // half of the K steps (cluster K split)
     const bool leader = rank == 0;
-    const int cid = G == 2 ? (int)(blockIdx.x / 2) : (int)blockIdx.x;  // pair (or CTA) index
-    const int ncl = G == 2 ? (int)(gridDim.x / 2) : (int)gridDim.x;
+    const int cid = CLUSTER ? (int)(blockIdx.x / 2) : (int)blockIdx.x;  // pair / cluster (or CTA) index
+    const int ncl = CLUSTER ? (int)(gridDim.x / 2) : (int)gridDim.x;
     const int total = (p.mtiles + G - 1) / G * p.ntiles * p.ksplit;
+    // this CTA's K steps of a unit: all, or one half under the cluster split
+    auto krange = [&](Work &w) {
+        if (CSK == 2) {
+            const int mid = p.kiters >> 1;
+            w.it0 = krank ? mid : 0;
+            w.it1 = krank ? p.kiters : mid;
+        }
+    };
     // stop this CTA's loops, and the peer's
     auto set_abort = [&]() {
         abort_sh = 1;
-        if (G == 2) st_cluster_u32(mapa(su32((const void *)&abort_sh), rank ^ 1u), 1u);
+        if (CLUSTER) st_cluster_u32(mapa(su32((const void *)&abort_sh), crank ^ 1u), 1u);
     };
 
     if (threadIdx.x == 0) {
@@ -116,12 +133,16 @@ __global__ void __launch_bounds__(THREADS, 1)
             mbar_init(&res_bar[i], 1);
         }
         mbar_init(&bst_bar, 1);
+        for (int i = 0; i < EPI_WARPS; ++i) {
+            mbar_init(&xfull_bar[i], 32);  // every lane of the peer warp arrives after its stores
+            mbar_init(&xfree_bar[i], 32);
+        }
         abort_sh = 0;
         issued_sh[0] = issued_sh[1] = issued_sh[2] = issued_sh[3] = 0;
         consumed_sh = 0;
         fence_mbar_init();
     }
-    if (G == 2) cluster_sync_all();  // both CTAs' barriers exist before either signals the other
+    if (CLUSTER) cluster_sync_all();  // both CTAs' barriers exist before either signals the other
     if (warp == 0) tmem_alloc<G>(&tmem_sh, TMEM_COLS);
     tc_fence_before();
     __syncthreads();
@@ -144,7 +165,8 @@ __global__ void __launch_bounds__(THREADS, 1)
             uint32_t par = 0;
             bool stop = false;
             for (int u = cid; u < total && !stop; u += ncl, ++lt) {
-                const Work w = work_of(p, u, BN, IMPLICIT, G, MS, 0);
+                Work w = work_of(p, u, BN, IMPLICIT, G, MS, 0);
+                krange(w);
                 const int b = lt & 1;
                 const uint32_t aph = (uint32_t)(lt >> 1) & 1u;
                 bool ok = G == 2 ? mbar_wait_cluster(&acce_bar[b], aph ^ 1u) : mbar_wait(&acce_bar[b], aph ^ 1u);
@@ -198,7 +220,8 @@ __global__ void __launch_bounds__(THREADS, 1)
                 }
             }
             for (int u = cid; u < total && !stop; u += ncl) {
-                const Work w = work_of(p, u, BN, IMPLICIT, G, MS, (int)rank);
+                Work w = work_of(p, u, BN, IMPLICIT, G, MS, (int)rank);
+                krange(w);
                 int tap = (int)fdiv((uint32_t)w.it0, p.fd_spt);
                 int cb = (w.it0 - tap * p.fd_spt.d) * KB;
                 int r = (int)fdiv((uint32_t)tap, p.fd_S), ss = tap - r * S;
@@ -282,7 +305,8 @@ __global__ void __launch_bounds__(THREADS, 1)
             }
             __syncwarp();
             for (int u = cid; u < total && !stop; u += ncl, ++lt) {
-                const Work w = work_of(p, u, BN, IMPLICIT, G, MS, 0);
+                Work w = work_of(p, u, BN, IMPLICIT, G, MS, 0);
+                krange(w);
                 const int b = lt & 1;
                 if (bar_red_or(BAR_MMA, 64, false)) break;  // accumulator b drained
                 tc_fence_after();
@@ -331,7 +355,8 @@ __global__ void __launch_bounds__(THREADS, 1)
                 stop = true;
             }
             for (int u = cid; u < total && !stop; u += ncl, ++lt) {
-                const Work w = work_of(p, u, BN, IMPLICIT, G, MS, 0);
+                Work w = work_of(p, u, BN, IMPLICIT, G, MS, 0);
+                krange(w);
                 const int b = lt & 1;
                 const uint32_t aph = (uint32_t)(lt >> 1) & 1u;
                 const bool drained = G == 2 ? mbar_wait_cluster(&acce_bar[b], aph ^ 1u) : mbar_wait(&acce_bar[b], aph ^ 1u);
@@ -372,6 +397,56 @@ __global__ void __launch_bounds__(THREADS, 1)
             }
             consumed_sh = g;
         }
+    } else if (CSK == 2 && krank == 1) {  // ---------------- cluster K split, CTA 1: send partials
+        // the same units and chunks as CTA 0's warp of the same index; each
+        // lane's row of 64 fp32 goes to the peer's exchange block, 16-byte
+        // piece j at slot j ^ (lane & 15) (fewer bank conflicts there)
+        constexpr int NCH = BN / 64;
+        constexpr int CPH = NCH / 2;
+        const int half = (warp - 2) >> 2;
+        const int g4 = warp & 3;
+        const int cbase = half * CPH;
+        const uint32_t peer_row = mapa(su32(xbuf + (warp - 2) * XBLK_BYTES + lane * 256), 0u);
+        const uint32_t peer_full = mapa(su32(&xfull_bar[warp - 2]), 0u);
+        uint32_t xph = 0;
+        int lt = 0;
+        bool stop = false;
+        for (int u = cid; u < total && !stop; u += ncl, ++lt) {
+            const int b = lt & 1;
+            const uint32_t aph = (uint32_t)(lt >> 1) & 1u;
+            const Work w = work_of(p, u, BN, IMPLICIT, G, MS, 0);
+            const bool tile_live = w.mt < p.mtiles;
+            if (!mbar_wait(&accf_bar[b], aph)) {
+                if (lane == 0) atomicOr(p.err, ERR_ACC_WAIT);
+                set_abort();
+                break;
+            }
+            tc_fence_after();
+#pragma unroll
+            for (int cj = 0; cj < CPH; ++cj) {
+                const int k0 = w.n0 + 64 * (cbase + cj);
+                if (k0 >= p.K || !tile_live) break;
+                const uint32_t taddr = tmem + ((uint32_t)(g4 * 32) << 16) + (uint32_t)(b * BN + 64 * (cbase + cj));
+                uint32_t v[64];
+                __syncwarp();
+                tmem_ld64(taddr, v);
+                if (!mbar_wait_cluster(&xfree_bar[warp - 2], xph ^ 1u)) {
+                    if (lane == 0) atomicOr(p.err, ERR_EPI_WAIT);
+                    set_abort();
+                    stop = true;
+                    break;
+                }
+#pragma unroll
+                for (int j = 0; j < 16; ++j)
+                    st_cluster_v4(peer_row + ((uint32_t)(j ^ (lane & 15)) << 4), v[4 * j], v[4 * j + 1], v[4 * j + 2],
+                                  v[4 * j + 3]);
+                mbar_arrive_cluster(peer_full);
+                xph ^= 1u;
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&acce_bar[b]);
+        }
     } else {  // ---------------- epilogue: warps 2..9
         // Warp w reads TMEM lanes 32*(w%4) .. +31 (tile rows).  Tiles of two or
         // more 64-channel chunks: all eight warps drain every unit, warp w the
@@ -393,6 +468,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         const int cbase = (ALT || MS == 2) ? 0 : half * CPH;  // first chunk of this warp
         int lt = ALT ? half : 0;
         uint32_t rpar = 0;  // phase parity of this warp's residual barrier
+        uint32_t xph = 0;   // cluster K split: phase parity of this warp's exchange block
         bool waited = false;
         for (int u = cid + (ALT ? half * ncl : 0); u < total; u += (ALT ? 2 : 1) * ncl, lt += ALT ? 2 : 1) {
             const int b = lt & 1;
@@ -485,6 +561,25 @@ __global__ void __launch_bounds__(THREADS, 1)
                     uint32_t v[64];
                     __syncwarp();
                     tmem_ld64(taddr, v);
+                    if (CSK == 2) {
+                        // add CTA 1's partial of the same rows and channels, then
+                        // hand its exchange block back
+                        if (!mbar_wait_cluster(&xfull_bar[warp - 2], xph)) {
+                            if (lane == 0) atomicOr(p.err, ERR_EPI_WAIT);
+                            set_abort();
+                        }
+                        const uint8_t *xr = xbuf + (warp - 2) * XBLK_BYTES + lane * 256;
+#pragma unroll
+                        for (int j = 0; j < 16; ++j) {
+                            const uint4 x = *reinterpret_cast<const uint4 *>(xr + ((j ^ (lane & 15)) << 4));
+                            v[4 * j] = __float_as_uint(__uint_as_float(v[4 * j]) + __uint_as_float(x.x));
+                            v[4 * j + 1] = __float_as_uint(__uint_as_float(v[4 * j + 1]) + __uint_as_float(x.y));
+                            v[4 * j + 2] = __float_as_uint(__uint_as_float(v[4 * j + 2]) + __uint_as_float(x.z));
+                            v[4 * j + 3] = __float_as_uint(__uint_as_float(v[4 * j + 3]) + __uint_as_float(x.w));
+                        }
+                        mbar_arrive_cluster(mapa(su32(&xfree_bar[warp - 2]), 1u));
+                        xph ^= 1u;
+                    }
                     // every 4 packed pairs (8 channels) go to their 16-byte piece
                     // of the row as soon as they are computed
 #pragma unroll
@@ -579,7 +674,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     }
     // neither CTA of a pair leaves while the other may still signal its
     // barriers or the leader's MMAs may still write its TMEM
-    if (G == 2) cluster_sync_all();
+    if (CLUSTER) cluster_sync_all();
     if (warp == 0) {
         tc_fence_after();
         tmem_dealloc<G>(tmem, TMEM_COLS);
@@ -672,6 +767,7 @@ struct Config {
     int KB;  // 64-channel blocks per pipeline stage (one TMA box spans them)
     bool bst = false;  // weight-stationary: B loaded once per CTA (one N tile, G = 1, no split)
     int ms = 1;        // 128-row halves per one-CTA tile (2: 256 x BN, one A box, B shared)
+    int csk = 1;       // 2: a cluster of two CTAs splits each tile's K steps, reducing on chip
 };
 
 constexpr int kSmCount = 152;  // GB300; only used to decide which K splits to offer
@@ -762,10 +858,21 @@ static std::vector<Config> configs(const Layer &l, const Shape &in, sn_schema s,
                 push_splits(cf, mtiles256);
             }
     };
+    // cluster K split for layers whose tiles do not fill the GPU: two CTAs per
+    // tile, each half the K steps, partials summed through distributed
+    // shared memory (no fp32 round trip through HBM, no reduction kernel)
+    auto push_csk = [&](Config cf, int64_t mtiles) {
+        for (int bn : bns)
+            if (bn >= 128 && kiters >= 4 && mtiles * ((K + bn - 1) / bn) < kSmCount) {
+                cf.BN = bn, cf.G = 1, cf.KB = 1, cf.ksplit = 1, cf.csk = 2;
+                out.push_back(cf);
+            }
+    };
     if (plain && a_blocks == 0) {
         push_all({false, 0, 0, 0, 0, 1, 1, 1}, (N * P * Q + BM - 1) / BM);
         push_bst({false, 0, 0, 0, 0, 1, 1, 1});
         push_ms2({false, 0, 0, 0, 0, 1, 1, 1}, (N * P * Q + 2 * BM - 1) / (2 * BM));
+        push_csk({false, 0, 0, 0, 0, 1, 1, 1}, (N * P * Q + BM - 1) / BM);
         return out;
     }
     struct Geo {
@@ -800,6 +907,7 @@ static std::vector<Config> configs(const Layer &l, const Shape &in, sn_schema s,
         } else {
             push_all({true, 0, gg.bw, gg.bh, gg.bni, 1, 1, 1}, tiles_of(gg));
             push_bst({true, 0, gg.bw, gg.bh, gg.bni, 1, 1, 1});
+            push_csk({true, 0, gg.bw, gg.bh, gg.bni, 1, 1, 1}, tiles_of(gg));
         }
     }
     if (a_blocks == 0)
@@ -807,23 +915,28 @@ static std::vector<Config> configs(const Layer &l, const Shape &in, sn_schema s,
     return out;
 }
 
-template <typename T, int BN, bool IMPLICIT, int G, int KB, bool BST = false, int MS = 1>
+template <typename T, int BN, bool IMPLICIT, int G, int KB, bool BST = false, int MS = 1, int CSK = 1>
 static cudaError_t launch(const CUtensorMap *mA, const CUtensorMap &mB, const CUtensorMap &mY, const CUtensorMap &mR,
                           const Params &p,
                           cudaStream_t st) {
-    constexpr int STAGES = BST ? BST_STAGES : stages_for(BN, G, KB, MS);
+    constexpr int XB = CSK == 2 ? EPI_WARPS * XBLK_BYTES : 0;  // cluster K split exchange blocks
+    constexpr int STAGES = BST ? BST_STAGES : stages_for(BN, G, KB, MS, XB);
     constexpr size_t smem_max = 227 * 1024;
     const size_t smem = BST ? (size_t)STAGES * BM * BK * 2 + p.bst_bytes + EPI_WARPS * STG_BYTES + 1024
-                            : (size_t)STAGES * KB * (MS * BM * BK * 2 + (BN / G) * BK * 2) + EPI_WARPS * STG_BYTES + 1024;
+                            : (size_t)STAGES * KB * (MS * BM * BK * 2 + (BN / G) * BK * 2) + EPI_WARPS * STG_BYTES + XB +
+                                  1024;
     static_assert(BST ||
                       (size_t)STAGES * KB * (MS * BM * BK * 2 + (BN / G) * BK * 2) + EPI_WARPS * STG_BYTES + 1024 <=
                           smem_max,
                   "shared memory per CTA");
     static_assert(!BST || (G == 1 && KB == 1 && MS == 1), "weight-stationary tiles are one-CTA, one block per stage");
     static_assert(MS == 1 || (G == 1 && KB == 1 && !BST && 2 * MS * BN <= 512), "two-half tiles: one CTA, TMEM");
+    static_assert(CSK == 1 || (G == 1 && MS == 1 && !BST && BN >= 128), "cluster K split: one-CTA tiles of >= 2 chunks");
+    static_assert(STAGES >= 2, "pipeline depth");
     if (smem > smem_max) return cudaErrorInvalidValue;
-    auto kern = conv_tc_kernel<T, BN, STAGES, IMPLICIT, G, KB, BST, MS>;
-    static int max_groups = 0;  // co-resident CTAs (G = 1) or CTA pairs (G = 2)
+    auto kern = conv_tc_kernel<T, BN, STAGES, IMPLICIT, G, KB, BST, MS, CSK>;
+    constexpr bool CLUSTER = G == 2 || CSK == 2;
+    static int max_groups = 0;  // co-resident CTAs (G = 1) or clusters of two (pairs, K split)
     cudaLaunchConfig_t cfg = {};
     cudaLaunchAttribute attr[2];
     cfg.blockDim = dim3(THREADS);
@@ -833,7 +946,7 @@ static cudaError_t launch(const CUtensorMap *mA, const CUtensorMap &mB, const CU
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;  // see launch_pdl
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.numAttrs = 1;
-    if (G == 2) {
+    if (CLUSTER) {
         attr[1].id = cudaLaunchAttributeClusterDimension;
         attr[1].val.clusterDim.x = 2;
         attr[1].val.clusterDim.y = 1;
@@ -848,7 +961,7 @@ static cudaError_t launch(const CUtensorMap *mA, const CUtensorMap &mB, const CU
     }
     if (!max_groups) {
         cudaError_t e = cudaSuccess;
-        if (G == 2) {
+        if (CLUSTER) {
             cudaLaunchConfig_t q = cfg;  // the cluster shape alone
             q.gridDim = dim3(2);
             q.attrs = attr + 1;
@@ -863,7 +976,7 @@ static cudaError_t launch(const CUtensorMap *mA, const CUtensorMap &mB, const CU
         }
     }
     const int total = (p.mtiles + G - 1) / G * p.ntiles * p.ksplit;
-    cfg.gridDim = dim3((unsigned)(G * std::min(total, max_groups)));
+    cfg.gridDim = dim3((unsigned)((CLUSTER ? 2 : 1) * std::min(total, max_groups)));
     cudaError_t e = cudaLaunchKernelEx(&cfg, kern, mA[0], mA[1], mA[2], mA[3], mB, mY, mR, p);
     if (e != cudaSuccess || p.ksplit == 1) return e;
     const int64_t n4 = p.Mout * (p.K / 4);
@@ -1011,6 +1124,17 @@ cudaError_t conv_tc(const LaunchArgs &a) {
     return cf.implicit ? launch<TT, BNV, true, GV, KBV>(mA, mB, mY, mR, p, a.stream)               \
                        : launch<TT, BNV, false, GV, KBV>(mA, mB, mY, mR, p, a.stream)
 #define SN_TC_LAUNCH_T(TT)                                                                          \
+    if (cf.csk == 2) {                                                                              \
+        if (cf.G != 1 || cf.KB != 1 || cf.ms != 1 || cf.bst || cf.ksplit != 1) return cudaErrorInvalidValue; \
+        if (cf.implicit) {                                                                          \
+            if (cf.BN == 128) return launch<TT, 128, true, 1, 1, false, 1, 2>(mA, mB, mY, mR, p, a.stream); \
+            if (cf.BN == 256) return launch<TT, 256, true, 1, 1, false, 1, 2>(mA, mB, mY, mR, p, a.stream); \
+            return cudaErrorInvalidValue;                                                           \
+        }                                                                                           \
+        if (cf.BN == 128) return launch<TT, 128, false, 1, 1, false, 1, 2>(mA, mB, mY, mR, p, a.stream); \
+        if (cf.BN == 256) return launch<TT, 256, false, 1, 1, false, 1, 2>(mA, mB, mY, mR, p, a.stream); \
+        return cudaErrorInvalidValue;                                                               \
+    }                                                                                               \
     if (cf.ms == 2) {                                                                               \
         if (cf.G != 1 || cf.KB != 1 || cf.bst) return cudaErrorInvalidValue;                        \
         if (cf.implicit) {                                                                          \

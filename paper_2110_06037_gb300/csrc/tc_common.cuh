@@ -31,8 +31,10 @@ constexpr bool waits_for_mma(int stages) { return producers_for(stages) == 2; }
 constexpr uint32_t BAR_MMA = 1;  // named barrier of the MMA warp and its waiter (0 is __syncthreads)
 // pipeline depth: as many stages of KB 64-channel blocks as fit beside the
 // epilogue staging (227 KB - 32 KB staging - 1 KB alignment slack)
-constexpr int stages_for(int bn, int g, int kb, int ms = 1) {
-    return 198656 / (kb * (16384 * ms + bn / g * 128)) < 8 ? 198656 / (kb * (16384 * ms + bn / g * 128)) : 8;
+constexpr int stages_for(int bn, int g, int kb, int ms = 1, int extra = 0) {
+    return (198656 - extra) / (kb * (16384 * ms + bn / g * 128)) < 8
+               ? (198656 - extra) / (kb * (16384 * ms + bn / g * 128))
+               : 8;
 }
 // weight-stationary tiles: the layer's whole B (K steps x BN rows x 128 B) is
 // loaded once per CTA and stays in shared memory beside this many A stages
@@ -40,6 +42,7 @@ constexpr int BST_STAGES = 4;
 constexpr int EPI_WARPS = 8;
 constexpr int MAX_K = 65536;
 constexpr uint32_t STG_BYTES = 32 * 64 * 2;      // one epilogue staging block: 32 rows x 64 channels
+constexpr uint32_t XBLK_BYTES = 32 * 64 * 4;     // cluster K split: one warp's fp32 partial block
 constexpr long long WAIT_LIMIT = 4000000000LL;  // SM cycles (~2 s)
 enum : int { ERR_TMA_WAIT = 0x10, ERR_MMA_WAIT = 0x20, ERR_ACC_WAIT = 0x40, ERR_EPI_WAIT = 0x80 };
 
@@ -232,6 +235,10 @@ __device__ __forceinline__ bool mbar_wait_cluster(uint64_t *b, uint32_t parity) 
     while (!mbar_try_cluster(b, parity))
         if (clock64() - t0 > WAIT_LIMIT) return false;
     return true;
+}
+__device__ __forceinline__ void st_cluster_v4(uint32_t caddr, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
+    asm volatile("st.shared::cluster.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(caddr), "r"(a), "r"(b), "r"(c), "r"(d)
+                 : "memory");
 }
 __device__ __forceinline__ void st_cluster_u32(uint32_t caddr, uint32_t v) {
     asm volatile("st.shared::cluster.u32 [%0], %1;" ::"r"(caddr), "r"(v) : "memory");
