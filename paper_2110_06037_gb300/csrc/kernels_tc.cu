@@ -863,7 +863,7 @@ static std::vector<Config> configs(const Layer &l, const Shape &in, sn_schema s,
     // shared memory (no fp32 round trip through HBM, no reduction kernel)
     auto push_csk = [&](Config cf, int64_t mtiles) {
         for (int bn : bns)
-            if (bn >= 128 && kiters >= 4 && mtiles * ((K + bn - 1) / bn) < kSmCount) {
+            if (bn >= 128 && kiters >= 4 && 2 * mtiles * ((K + bn - 1) / bn) <= kSmCount) {  // one wave of pairs
                 cf.BN = bn, cf.G = 1, cf.KB = 1, cf.ksplit = 1, cf.csk = 2;
                 out.push_back(cf);
             }
