@@ -751,7 +751,10 @@ cudaError_t dwconv(const LaunchArgs &a) {
     // 16-bit; shared-memory halo tiles otherwise); NCHW 0 = row kernel (8
     // columns per thread), 1 = shared-memory plane tile
     const ConvDims d = conv_dims(a);
-    if (a.variant == 1 && dw3_ring_applies(a, d)) return dw3_nhwc_ring(a, d);
+    if (a.variant == 1 && dw3_ring_applies(a, d)) {
+        const cudaError_t e = dw3_nhwc_ring(a, d);
+        if (e != cudaErrorNotSupported) return e;  // else the shared-memory halo kernel below
+    }
     const int64_t total = (int64_t)d.N * d.K * d.P * d.Q;
     const int es = dtype_size(a.schema.dtype);
     const bool vec_ok = (d.C * es) % 16 == 0 && (uintptr_t)a.in[0] % 16 == 0 && (uintptr_t)a.out % 16 == 0 &&

@@ -81,7 +81,8 @@ __global__ void __launch_bounds__(THREADS, 1)
     __shared__ __align__(8) uint64_t bst_bar;              // weight-stationary B landed
     // CSK = 2 (cluster K split): the two CTAs of a cluster take the two halves
     // of a tile's K steps; CTA 1's epilogue warps write their fp32 partial
-    // rows into CTA 0's exchange blocks (distributed shared memory)
+    // rows into CTA 0's exchange blocks (distributed shared memory), each
+    // block handed to CTA 1 once CTA 0's stages are done with (xfree)
     __shared__ __align__(8) uint64_t xfull_bar[EPI_WARPS];  // CTA 0: a partial block landed
     __shared__ __align__(8) uint64_t xfree_bar[EPI_WARPS];  // CTA 1: CTA 0 has read the block
     __shared__ uint32_t tmem_sh;
@@ -92,7 +93,10 @@ __global__ void __launch_bounds__(THREADS, 1)
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t *bst = smem + STAGES * STAGE_BYTES;  // weight-stationary B (BST), 1024-B aligned
     uint8_t *stg = bst + (BST ? p.bst_bytes : 0);  // epilogue staging: one block per warp, 1024-B aligned
-    uint8_t *xbuf = stg + EPI_WARPS * STG_BYTES;   // CSK: 32 x 64 fp32 exchange block per warp (XBLK_BYTES)
+    // CSK: the exchange blocks (32 x 64 fp32 per warp) reuse the pipeline
+    // stages, free once this CTA's only unit has been accumulated (the host
+    // launches the split only when every cluster gets one unit)
+    uint8_t *xbuf = smem;
     constexpr bool CLUSTER = G == 2 || CSK == 2;
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
     const uint32_t crank = CLUSTER ? cluster_rank() : 0u;
@@ -430,7 +434,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                 uint32_t v[64];
                 __syncwarp();
                 tmem_ld64(taddr, v);
-                if (!mbar_wait_cluster(&xfree_bar[warp - 2], xph ^ 1u)) {
+                if (!mbar_wait_cluster(&xfree_bar[warp - 2], xph)) {
                     if (lane == 0) atomicOr(p.err, ERR_EPI_WAIT);
                     set_abort();
                     stop = true;
@@ -526,6 +530,9 @@ __global__ void __launch_bounds__(THREADS, 1)
                 break;
             }
             tc_fence_after();
+            // cluster K split: this CTA's MMAs have read their last stage, so
+            // the stage memory may now take CTA 1's partials
+            if (CSK == 2) mbar_arrive_cluster(mapa(su32(&xfree_bar[warp - 2]), 1u));
 #pragma unroll
             for (int cj = 0; cj < CPH; ++cj) {
                 const int ci = cbase + cj;
@@ -919,12 +926,12 @@ template <typename T, int BN, bool IMPLICIT, int G, int KB, bool BST = false, in
 static cudaError_t launch(const CUtensorMap *mA, const CUtensorMap &mB, const CUtensorMap &mY, const CUtensorMap &mR,
                           const Params &p,
                           cudaStream_t st) {
-    constexpr int XB = CSK == 2 ? EPI_WARPS * XBLK_BYTES : 0;  // cluster K split exchange blocks
-    constexpr int STAGES = BST ? BST_STAGES : stages_for(BN, G, KB, MS, XB);
+    constexpr int STAGES = BST ? BST_STAGES : stages_for(BN, G, KB, MS);
+    static_assert(CSK == 1 || (size_t)STAGES * KB * (BM * BK * 2 + BN * BK * 2) >= EPI_WARPS * XBLK_BYTES,
+                  "cluster K split: the exchange blocks live in the stage memory");
     constexpr size_t smem_max = 227 * 1024;
     const size_t smem = BST ? (size_t)STAGES * BM * BK * 2 + p.bst_bytes + EPI_WARPS * STG_BYTES + 1024
-                            : (size_t)STAGES * KB * (MS * BM * BK * 2 + (BN / G) * BK * 2) + EPI_WARPS * STG_BYTES + XB +
-                                  1024;
+                            : (size_t)STAGES * KB * (MS * BM * BK * 2 + (BN / G) * BK * 2) + EPI_WARPS * STG_BYTES + 1024;
     static_assert(BST ||
                       (size_t)STAGES * KB * (MS * BM * BK * 2 + (BN / G) * BK * 2) + EPI_WARPS * STG_BYTES + 1024 <=
                           smem_max,
@@ -976,6 +983,8 @@ static cudaError_t launch(const CUtensorMap *mA, const CUtensorMap &mB, const CU
         }
     }
     const int total = (p.mtiles + G - 1) / G * p.ntiles * p.ksplit;
+    // the cluster K split reuses stage memory for its exchange: one unit per cluster
+    if (CSK == 2 && total > max_groups) return cudaErrorNotSupported;
     cfg.gridDim = dim3((unsigned)((CLUSTER ? 2 : 1) * std::min(total, max_groups)));
     cudaError_t e = cudaLaunchKernelEx(&cfg, kern, mA[0], mA[1], mA[2], mA[3], mB, mY, mR, p);
     if (e != cudaSuccess || p.ksplit == 1) return e;

@@ -203,6 +203,8 @@ sn_status launch_routine(const LaunchArgs &a) {
     case R_CONV_S2D_TC: e = k::conv_s2d_tc(a); break;
     default: return fail(SN_EINVAL, "launch of a non-launchable routine");
     }
+    if (e == cudaErrorNotSupported)  // a routine parameter this device cannot run (e.g. too few co-resident clusters)
+        return fail(SN_EUNSUPPORTED, std::string(routine_name(a.routine)) + ": not supported here");
     if (e != cudaSuccess)
         return fail(SN_ECUDA, std::string(routine_name(a.routine)) + ": " + cudaGetErrorString(e));
     return SN_OK;

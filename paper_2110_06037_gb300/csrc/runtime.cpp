@@ -375,6 +375,10 @@ static sn_status profile_graph_on(Graph *g, const sn_profile_opts &o, cudaStream
             a.ws_bytes = g->workspace.bytes;
             int64_t t = kInf;
             rc = time_median(o.warmup, o.iters, st, [&]() { return launch_routine(a); }, &t);
+            if (rc == SN_EUNSUPPORTED) {  // a routine parameter this device cannot run: infeasible
+                rc = SN_OK;
+                t = kInf;
+            }
             if (rc != SN_OK) break;
             cd.cost = t;
             seen.emplace(sig, t);
