@@ -241,7 +241,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-b1", action="store_true")
     ap.add_argument("--config", default="r50_b32",
-                    choices=["r50_b32", "bandwidth", "sweep", "mbv2_b1", "r50_b1", "tiny", "layer"],
+                    choices=["r50_b32", "bandwidth", "sweep", "mbv2_b1", "r50_b1", "tiny", "layer", "vgg16_b32",
+                             "vgg16_b1"],
                     help="r50_b32 is the benchmark line; the others print one extra JSON line each")
     ap.add_argument("--layer", default="32,512,56,512,3,1",
                     help="--config layer: N,C,H,K,k,s of one bf16 NHWC conv (C -> K channels, HxH input)")
@@ -627,6 +628,12 @@ def run_extra_config(args):
             x, layers = synth.mobilenet_v2(1)
             layers = sn.fuse_residual(layers)
             sch, io, dt = [("f16", "nchw"), ("f16", "nhwc")], ("f16", "nchw"), torch.float16
+        elif name == "vgg16_b32":
+            x, layers = synth.vgg16(32)
+            sch, io, dt = [("bf16", "nchw"), ("bf16", "nhwc")], ("bf16", "nchw"), torch.bfloat16
+        elif name == "vgg16_b1":
+            x, layers = synth.vgg16(1)
+            sch, io, dt = [("f16", "nchw"), ("f16", "nhwc")], ("f16", "nchw"), torch.float16
         else:
             x, layers = synth.resnet50(1)
             layers = sn.fuse_residual(layers)
@@ -664,6 +671,10 @@ def run_extra_config(args):
         for i in range(1, t["n_layers"] - 1):
             r = sn.routine_name(int(t["routine"][int(cands[i])]))
             path[r] = path.get(r, 0) + 1
+        work, _ = conv_work(layers, x.shape)
+        fl = sum(w[0] for w in work)
+        out.update({"batch": int(x.shape[0]), "images_per_s": x.shape[0] / statistics.median(lat) * 1e3,
+                    "gflop": fl / 1e9, "tflops": fl / statistics.median(lat) / 1e9})
         out.update({"metric": "latency (ms), CUDA-graph replay, L2 flushed", "mean_ms": statistics.mean(lat),
                     "std_ms": statistics.pstdev(lat), "median_ms": statistics.median(lat), "tuning_s": tune,
                     "path_cost_ns": total, "routines_on_path": path,

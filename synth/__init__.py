@@ -198,6 +198,31 @@ def resnet50(batch=1, seed=0, res=224):
     return materialise(b.layers, (batch, 3, res, res), seed, weight_gain=gains)
 
 
+def vgg16(batch=1, seed=0, res=224):
+    """VGG16 (configuration D): thirteen 3x3 convs with ReLU in five groups,
+    each followed by a 2x2 stride-2 max pool, then three fully connected
+    layers.  The first of them runs as a convolution whose kernel covers the
+    whole final feature map (res/32 square, valid padding): it is the dense
+    layer over the flattened map, independent of the activation layout.
+    He-normal weights keep the ReLU activations' variance level without BN.
+    """
+    if res % 32:
+        raise ValueError("vgg16: the input side must be a multiple of 32")
+    b = _Builder()
+    l, c = -1, 3
+    groups = [(64, 2), (128, 2), (256, 3), (512, 3), (512, 3)]
+    for gi, (width, n) in enumerate(groups):
+        for i in range(n):
+            l = b.push(conv(c, width, 3, 1, 1, act="relu", name=f"conv{gi + 1}_{i + 1}"), [l])
+            c = width
+        l = b.push(maxpool(2, 2, 0, name=f"pool{gi + 1}"), [l])
+    f = res // 32
+    l = b.push(conv(512, 4096, f, 1, 0, act="relu", name="fc6"), [l])
+    l = b.push(dense(4096, 4096, act="relu", name="fc7"), [l])
+    b.push(dense(4096, 1000, name="fc8"), [l])
+    return materialise(b.layers, (batch, 3, res, res), seed)
+
+
 def single_conv(N, H, C, K, k, s, seed=0, act="relu"):
     """One conv layer of the single-layer sweep: NxCxHxH N(0,1), He-normal."""
     b = _Builder()

@@ -7,6 +7,8 @@
   * MobileNetV2 b1 fp16, ResNet-50 b1 fp16: DPRS equals the oracle's exact
     block-wise search on the profiled table; output within 2e-2.
   * ResNet-50 b32 bf16: sampled images of the batch against the oracle.
+  * VGG16 bf16 (64x64 input, batch 2): DPRS equals the block-wise search;
+    output within 2e-2.
   * The same nets with every residual add fused into its conv2: DPRS equals
     the block-wise search, outputs within 2e-2 of the (unfused) oracle.
 """
@@ -99,6 +101,14 @@ def test_mobilenet_v2_b1_fp16():
     g, got = _profile_select_run(layers, x, ("f16", "nchw"), ("f16", "nchw"), F16, exhaustive=False)
     ref = run_net(layers, x, "f16")
     assert maxrel(got, ref) <= TOL["f16"]
+
+
+def test_vgg16_bf16():
+    """VGG16 (fc6 as a whole-map convolution) at a 64x64 input, batch 2."""
+    x, layers = synth.vgg16(2, res=64)
+    g, got = _profile_select_run(layers, x, ("bf16", "nchw"), ("bf16", "nchw"), BF16, exhaustive=False)
+    ref = run_net(layers, x, "bf16")
+    assert maxrel(got, ref) <= TOL["bf16"]
 
 
 def test_resnet50_b1_fp16_and_graph_replay():
