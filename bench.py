@@ -177,6 +177,9 @@ def conv_work(layers, in_shape, elem=2):
         elif l["type"] == "add":
             out = ins[0]
             fl, by = n * c * h * w, 3 * elem * n * c * h * w
+        elif l["type"] == "mul":  # per-channel scale: the blob in and out, one scale per (n, c)
+            out = ins[0]
+            fl, by = n * c * h * w, elem * (2 * n * c * h * w + n * c)
         else:  # dense
             out = (n, p["out_features"], 1, 1)
             fl = 2 * n * p["in_features"] * p["out_features"]
@@ -242,7 +245,7 @@ def main():
     ap.add_argument("--no-b1", action="store_true")
     ap.add_argument("--config", default="r50_b32",
                     choices=["r50_b32", "bandwidth", "sweep", "mbv2_b1", "r50_b1", "tiny", "layer", "vgg16_b32",
-                             "vgg16_b1"],
+                             "vgg16_b1", "mbv3_b1"],
                     help="r50_b32 is the benchmark line; the others print one extra JSON line each")
     ap.add_argument("--layer", default="32,512,56,512,3,1",
                     help="--config layer: N,C,H,K,k,s of one bf16 NHWC conv (C -> K channels, HxH input)")
@@ -626,6 +629,10 @@ def run_extra_config(args):
             sch, io, dt = [("f32", "nchw"), ("f32", "nhwc")], ("f32", "nchw"), torch.float32
         elif name == "mbv2_b1":
             x, layers = synth.mobilenet_v2(1)
+            layers = sn.fuse_residual(layers)
+            sch, io, dt = [("f16", "nchw"), ("f16", "nhwc")], ("f16", "nchw"), torch.float16
+        elif name == "mbv3_b1":
+            x, layers = synth.mobilenet_v3(1)
             layers = sn.fuse_residual(layers)
             sch, io, dt = [("f16", "nchw"), ("f16", "nhwc")], ("f16", "nchw"), torch.float16
         elif name == "vgg16_b32":

@@ -78,10 +78,21 @@ typedef enum {
     SN_L_MAXPOOL = 2, /* max pooling, -inf padding                             */
     SN_L_GAP = 3,     /* global average pooling -> N x C x 1 x 1               */
     SN_L_ADD = 4,     /* elementwise sum of two blobs + act                    */
-    SN_L_DENSE = 5    /* y = W x + b on an N x C x 1 x 1 blob                  */
+    SN_L_DENSE = 5,   /* y = W x + b on an N x C x 1 x 1 blob                  */
+    SN_L_MUL = 6      /* y[n,c,h,w] = x[n,c,h,w] * s[n,c] + act: the scale of
+                       * a squeeze-and-excite block; inputs (x, s), s is
+                       * N x C x 1 x 1; params sn_add_params                   */
 } sn_layer_type;
 
-typedef enum { SN_ACT_NONE = 0, SN_ACT_RELU = 1, SN_ACT_RELU6 = 2 } sn_act;
+/* Activations: max(0,x); min(max(0,x),6); hard swish x * relu6(x+3) / 6 and
+ * hard sigmoid relu6(x+3) / 6 (MobileNetV3's piecewise-linear forms). */
+typedef enum {
+    SN_ACT_NONE = 0,
+    SN_ACT_RELU = 1,
+    SN_ACT_RELU6 = 2,
+    SN_ACT_HSWISH = 3,
+    SN_ACT_HSIGMOID = 4
+} sn_act;
 
 /* conv2 / dwconv2 parameters: output extent P = floor((H + 2ph - dh(kh-1) - 1)/sh) + 1. */
 typedef struct {

@@ -24,7 +24,7 @@ _LIB_PATH = os.path.join(_HERE, "liboracle.so")
 GCC_CMD = ["gcc", "-O2", "-std=c11", "-fopenmp", "-ffp-contract=off", "-fPIC", "-shared",
            _SRC, "-o", _LIB_PATH, "-lm"]
 
-ACT = {"none": 0, "relu": 1, "relu6": 2, None: 0}
+ACT = {"none": 0, "relu": 1, "relu6": 2, "hswish": 3, "hsigmoid": 4, None: 0}
 INF = np.iinfo(np.int64).max
 
 _lib = None
@@ -57,6 +57,8 @@ def lib():
         L.or_add.argtypes = [dp, dp, i64, ctypes.c_int, dp]
         L.or_dense.restype = None
         L.or_dense.argtypes = [dp, dp, dp, i64, i64, i64, ctypes.c_int, dp]
+        L.or_mul.restype = None
+        L.or_mul.argtypes = [dp, dp, i64, i64, i64, ctypes.c_int, dp]
         for name in ("or_cast_f32_to_f16", "or_cast_f32_to_bf16",
                      "or_cast_f16_to_f32", "or_cast_bf16_to_f32"):
             getattr(L, name).restype = None
@@ -133,6 +135,18 @@ def add(a, b, act="none"):
         raise ValueError("add operands differ in shape")
     y = np.empty_like(a)
     lib().or_add(_p(a), _p(b), a.size, ACT[act], _p(y))
+    return y
+
+
+def mul(x, s, act="none"):
+    """y[n,c,h,w] = act(x[n,c,h,w] * s[n,c]): the scale of a squeeze-and-excite
+    block (MobileNetV3); s is [N, C] or [N, C, 1, 1]."""
+    x, s = _f64(x), _f64(s)
+    N, C, H, W = x.shape
+    if s.size != N * C:
+        raise ValueError("mul: the scale must hold one value per (image, channel)")
+    y = np.empty_like(x)
+    lib().or_mul(_p(x), _p(np.ascontiguousarray(s.reshape(N, C))), N, C, H * W, ACT[act], _p(y))
     return y
 
 

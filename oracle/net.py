@@ -5,7 +5,7 @@ TEST INFRASTRUCTURE ONLY (see the package docstring).
 A net is the plain-data description used throughout the tests: a list of
 layers in topological order (section IV-A numbers them L_1..L_n the same way),
 each a dict with keys
-    type    'conv2' | 'dwconv2' | 'maxpool' | 'gap' | 'add' | 'dense'
+    type    'conv2' | 'dwconv2' | 'maxpool' | 'gap' | 'add' | 'dense' | 'mul'
     inputs  list of earlier layer indices, -1 = the net input
     params  dict of layer parameters (section III-B)
     weight, bias   fp32 arrays (conv: [K, C/groups, R, S]; dense: [out, in])
@@ -20,7 +20,7 @@ from __future__ import annotations
 
 import numpy as np
 
-from . import add, conv2d, dense, gap, maxpool2d, round_to
+from . import add, conv2d, dense, gap, maxpool2d, mul, round_to
 
 
 def run_layer(layer: dict, inputs: list, dtype: str = "f32") -> np.ndarray:
@@ -46,6 +46,8 @@ def run_layer(layer: dict, inputs: list, dtype: str = "f32") -> np.ndarray:
         return gap(inputs[0])
     if t == "add":
         return add(inputs[0], inputs[1], act=p.get("act", "none"))
+    if t == "mul":
+        return mul(inputs[0], inputs[1], act=p.get("act", "none"))
     if t == "dense":
         w = round_to(layer["weight"], dtype)
         return dense(inputs[0], w, layer.get("bias"), act=p.get("act", "none"))

@@ -43,11 +43,17 @@
 
 #define OR_INF INT64_MAX
 
-enum { OR_ACT_NONE = 0, OR_ACT_RELU = 1, OR_ACT_RELU6 = 2 };
+enum { OR_ACT_NONE = 0, OR_ACT_RELU = 1, OR_ACT_RELU6 = 2, OR_ACT_HSWISH = 3, OR_ACT_HSIGMOID = 4 };
 
+static double or_relu6(double v) { return v < 0.0 ? 0.0 : (v > 6.0 ? 6.0 : v); }
+
+/* ReLU, ReLU6, and MobileNetV3's hard swish x * ReLU6(x + 3) / 6 and hard
+ * sigmoid ReLU6(x + 3) / 6 */
 static double or_act(double v, int act) {
     if (act == OR_ACT_RELU) return v > 0.0 ? v : 0.0;
-    if (act == OR_ACT_RELU6) return v < 0.0 ? 0.0 : (v > 6.0 ? 6.0 : v);
+    if (act == OR_ACT_RELU6) return or_relu6(v);
+    if (act == OR_ACT_HSWISH) return v * or_relu6(v + 3.0) / 6.0;
+    if (act == OR_ACT_HSIGMOID) return or_relu6(v + 3.0) / 6.0;
     return v;
 }
 
@@ -146,6 +152,12 @@ void or_gap(const double *x, int64_t N, int64_t C, int64_t H, int64_t W, double 
 /* Elementwise y = act(a + b). */
 void or_add(const double *a, const double *b, int64_t n, int act, double *y) {
     for (int64_t i = 0; i < n; ++i) y[i] = or_act(a[i] + b[i], act);
+}
+
+/* Per-channel scale (squeeze-and-excite): y[n,c,h,w] = act(x[n,c,h,w] * s[n,c]), NCHW. */
+void or_mul(const double *x, const double *s, int64_t N, int64_t C, int64_t HW, int act, double *y) {
+    for (int64_t nc = 0; nc < N * C; ++nc)
+        for (int64_t i = 0; i < HW; ++i) y[nc * HW + i] = or_act(x[nc * HW + i] * s[nc], act);
 }
 
 /* Dense: y[n,o] = act(b[o] + sum_i W[o,i] x[n,i]); W is [out, in]. */

@@ -19,8 +19,8 @@ STATUS_NAMES = ["SN_OK", "SN_EINVAL", "SN_ENOMEM", "SN_ECUDA", "SN_EUNSUPPORTED"
                 "SN_ETIMEOUT", "SN_EINFEASIBLE"]
 SN_F32, SN_F16, SN_BF16 = 0, 1, 2
 SN_NCHW, SN_NHWC = 0, 1
-SN_L_CONV2, SN_L_DWCONV2, SN_L_MAXPOOL, SN_L_GAP, SN_L_ADD, SN_L_DENSE = range(6)
-SN_ACT = {"none": 0, None: 0, "relu": 1, "relu6": 2}
+SN_L_CONV2, SN_L_DWCONV2, SN_L_MAXPOOL, SN_L_GAP, SN_L_ADD, SN_L_DENSE, SN_L_MUL = range(7)
+SN_ACT = {"none": 0, None: 0, "relu": 1, "relu6": 2, "hswish": 3, "hsigmoid": 4}
 SN_SELECT_DPRS, SN_SELECT_BRUTE = 0, 1
 SN_OPT_CUDA_GRAPH, SN_OPT_CHECK = 0, 1
 COST_INF = np.iinfo(np.int64).max

@@ -94,7 +94,7 @@ class Graph:
         elif type_ == _sn.SN_L_MAXPOOL:
             p = _sn.sn_pool_params(params["kh"], params["kw"], params["sh"], params["sw"], params["ph"],
                                    params["pw"])
-        elif type_ == _sn.SN_L_ADD:
+        elif type_ in (_sn.SN_L_ADD, _sn.SN_L_MUL):
             p = _sn.sn_add_params(_sn.SN_ACT[(params or {}).get("act", "none")])
         elif type_ == _sn.SN_L_DENSE:
             p = _sn.sn_dense_params(params["in_features"], params["out_features"],

@@ -94,7 +94,7 @@ static sn_status infer_shape(Layer &L, const std::vector<Shape> &in) {
         if (p.kh < 1 || p.kw < 1 || p.sh < 1 || p.sw < 1 || p.ph < 0 || p.pw < 0 || p.dh < 1 ||
             p.dw < 1 || p.groups < 1 || p.c_in < 1 || p.c_out < 1)
             return fail(SN_EINVAL, "conv2: invalid parameter");
-        if (p.act < SN_ACT_NONE || p.act > SN_ACT_RELU6) return fail(SN_EINVAL, "conv2: bad act");
+        if (p.act < SN_ACT_NONE || p.act > SN_ACT_HSIGMOID) return fail(SN_EINVAL, "conv2: bad act");
         if (in[0].c != p.c_in) return fail(SN_EINVAL, "conv2: input channels != c_in");
         if (p.c_in % p.groups || p.c_out % p.groups)
             return fail(SN_EINVAL, "conv2: groups must divide c_in and c_out");
@@ -128,14 +128,21 @@ static sn_status infer_shape(Layer &L, const std::vector<Shape> &in) {
     case SN_L_ADD:
         if (in.size() != 2) return fail(SN_EINVAL, "add takes two inputs");
         if (!(in[0] == in[1])) return fail(SN_EINVAL, "add: input shapes differ");
-        if (L.act < SN_ACT_NONE || L.act > SN_ACT_RELU6) return fail(SN_EINVAL, "add: bad act");
+        if (L.act < SN_ACT_NONE || L.act > SN_ACT_HSIGMOID) return fail(SN_EINVAL, "add: bad act");
+        L.out = in[0];
+        return SN_OK;
+    case SN_L_MUL:
+        if (in.size() != 2) return fail(SN_EINVAL, "mul takes two inputs (blob, per-channel scale)");
+        if (!(in[1] == Shape{in[0].n, in[0].c, 1, 1}))
+            return fail(SN_EINVAL, "mul: the scale must be N x C x 1 x 1 of the blob's N and C");
+        if (L.act < SN_ACT_NONE || L.act > SN_ACT_HSIGMOID) return fail(SN_EINVAL, "mul: bad act");
         L.out = in[0];
         return SN_OK;
     case SN_L_DENSE:
         if (in.size() != 1) return fail(SN_EINVAL, "dense takes one input");
         if (in[0].h != 1 || in[0].w != 1 || in[0].c != L.dense_in || L.dense_out < 1)
             return fail(SN_EINVAL, "dense: input must be N x in_features x 1 x 1");
-        if (L.act < SN_ACT_NONE || L.act > SN_ACT_RELU6) return fail(SN_EINVAL, "dense: bad act");
+        if (L.act < SN_ACT_NONE || L.act > SN_ACT_HSIGMOID) return fail(SN_EINVAL, "dense: bad act");
         L.out = {in[0].n, L.dense_out, 1, 1};
         return SN_OK;
     default:
@@ -173,6 +180,7 @@ sn_status add_layer(Graph *g, int32_t type, const void *params, const int32_t *i
     case SN_L_GAP:
         break;
     case SN_L_ADD:
+    case SN_L_MUL:
         L.act = params ? static_cast<const sn_add_params *>(params)->act : SN_ACT_NONE;
         break;
     case SN_L_DENSE: {

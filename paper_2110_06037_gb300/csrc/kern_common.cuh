@@ -37,6 +37,8 @@ template <> __device__ __forceinline__ __nv_bfloat16 cvt<__nv_bfloat16>(float v)
 __device__ __forceinline__ float act_apply(float v, int act) {
     if (act == SN_ACT_RELU) return fmaxf(v, 0.0f);
     if (act == SN_ACT_RELU6) return fminf(fmaxf(v, 0.0f), 6.0f);
+    if (act == SN_ACT_HSWISH) return v * fminf(fmaxf(v + 3.0f, 0.0f), 6.0f) / 6.0f;
+    if (act == SN_ACT_HSIGMOID) return fminf(fmaxf(v + 3.0f, 0.0f), 6.0f) / 6.0f;
     return v;
 }
 

@@ -999,6 +999,64 @@ cudaError_t add(const LaunchArgs &a) {
     return cudaGetLastError();
 }
 
+// per-channel scale: y[n,c,h,w] = act(x[n,c,h,w] * s[n,c]).  NHWC, 16-byte
+// vectors when C allows: one thread per 8 (16-bit) or 4 (fp32) channels of a
+// pixel; otherwise one thread per element, (n, c) from the layout.
+template <typename T>
+__global__ void mul_nhwc_vec(const uint4 *__restrict__ x, const T *__restrict__ s, uint4 *__restrict__ y,
+                             int64_t pixels, int64_t HW, int CV, int act) {
+    griddep_launch();
+    griddep_wait();
+    constexpr int E = 16 / sizeof(T);
+    const int64_t total = pixels * CV;
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t pix = i / CV;
+        const int cv = (int)(i - pix * CV);
+        const int64_t n = pix / HW;
+        const uint4 xv = x[i];
+        const uint4 sv = reinterpret_cast<const uint4 *>(s + n * (int64_t)CV * E)[cv];
+        uint4 o;
+        const T *px = reinterpret_cast<const T *>(&xv), *ps = reinterpret_cast<const T *>(&sv);
+        T *po = reinterpret_cast<T *>(&o);
+#pragma unroll
+        for (int e = 0; e < E; ++e) po[e] = cvt<T>(act_apply(ldf<T>(px + e) * ldf<T>(ps + e), act));
+        y[i] = o;
+    }
+}
+
+template <typename T, bool NHWC>
+__global__ void mul_kernel(const T *__restrict__ x, const T *__restrict__ s, T *__restrict__ y, int64_t n,
+                           int64_t C, int64_t HW, int act) {
+    griddep_launch();
+    griddep_wait();
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t nc = NHWC ? (i / (HW * C)) * C + i % C : i / HW;  // index of (n, c) in s
+        stf<T>(y + i, act_apply(ldf<T>(x + i) * ldf<T>(s + nc), act));
+    }
+}
+
+cudaError_t mul(const LaunchArgs &a) {
+    const Shape &o = a.layer->out;
+    const int64_t n = o.numel(), HW = o.h * o.w;
+    SN_DT_SWITCH(a.schema.dtype, T, {
+        const int64_t cb = o.c * (int64_t)sizeof(T);
+        if (a.schema.layout == SN_NHWC && cb % 16 == 0 && (uintptr_t)a.in[0] % 16 == 0 &&
+            (uintptr_t)a.in[1] % 16 == 0 && (uintptr_t)a.out % 16 == 0)
+            launch_pdl(mul_nhwc_vec<T>, grid_for(n * (int64_t)sizeof(T) / 16, 256), 256, 0, a.stream,
+                       (const uint4 *)a.in[0], (const T *)a.in[1], (uint4 *)a.out, o.n * HW, HW, (int)(cb / 16),
+                       a.layer->act);
+        else if (a.schema.layout == SN_NHWC)
+            launch_pdl(mul_kernel<T, true>, grid_for(n, 256), 256, 0, a.stream, (const T *)a.in[0],
+                       (const T *)a.in[1], (T *)a.out, n, o.c, HW, a.layer->act);
+        else
+            launch_pdl(mul_kernel<T, false>, grid_for(n, 256), 256, 0, a.stream, (const T *)a.in[0],
+                       (const T *)a.in[1], (T *)a.out, n, o.c, HW, a.layer->act);
+    });
+    return cudaGetLastError();
+}
+
 // dense: one warp per (n, o), dot product over the input features
 template <typename T>
 __global__ void dense_kernel(const T *__restrict__ x, const T *__restrict__ w, const float *__restrict__ bias,

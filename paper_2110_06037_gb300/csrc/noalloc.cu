@@ -52,7 +52,7 @@ extern "C" sn_status sn_conv2d_wino_noalloc(const void *x_dev, sn_schema schema,
             return fail(SN_EINVAL, "sn_conv2d_wino_noalloc: NULL argument");
         if (!schema_valid(schema)) return fail(SN_EINVAL, "sn_conv2d_wino_noalloc: invalid schema");
         if (pad < 0 || pad > 2) return fail(SN_EINVAL, "sn_conv2d_wino_noalloc: pad must be 0, 1 or 2");
-        if (act < SN_ACT_NONE || act > SN_ACT_RELU6) return fail(SN_EINVAL, "sn_conv2d_wino_noalloc: bad act");
+        if (act < SN_ACT_NONE || act > SN_ACT_HSIGMOID) return fail(SN_EINVAL, "sn_conv2d_wino_noalloc: bad act");
         for (int i = 0; i < 4; ++i)
             if (in_nchw[i] < 1 || in_nchw[i] > (1 << 30))
                 return fail(SN_EINVAL, "sn_conv2d_wino_noalloc: extents must be in [1, 2^30]");

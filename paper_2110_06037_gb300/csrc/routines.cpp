@@ -21,6 +21,7 @@ const char *routine_name(int32_t r) {
     case R_MAXPOOL: return "maxpool/direct";
     case R_GAP: return "gap/reduce";
     case R_ADD: return "add/eltwise";
+    case R_MUL: return "mul/eltwise";
     case R_DENSE: return "dense/simt";
     case R_ADAPT: return "adapt/convert";
     case R_CONV_IM2COL_TC: return "conv2/im2col_tc";
@@ -70,6 +71,8 @@ int32_t routine_variants(int32_t r, const Layer &l, const std::vector<Shape> &in
         return l.type == SN_L_GAP ? 1 : 0;
     case R_ADD:
         return l.type == SN_L_ADD ? 1 : 0;
+    case R_MUL:
+        return l.type == SN_L_MUL ? 1 : 0;
     case R_DENSE:
         return l.type == SN_L_DENSE ? 1 : 0;
     case R_CONV_IM2COL_TC:
@@ -197,6 +200,7 @@ sn_status launch_routine(const LaunchArgs &a) {
     case R_MAXPOOL: e = k::maxpool(a); break;
     case R_GAP: e = k::gap(a); break;
     case R_ADD: e = k::add(a); break;
+    case R_MUL: e = k::mul(a); break;
     case R_DENSE: e = k::dense(a); break;
     case R_CONV_IM2COL_TC: e = k::conv_im2col_tc(a); break;
     case R_DENSE_TC: e = k::dense_tc(a); break;

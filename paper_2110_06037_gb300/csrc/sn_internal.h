@@ -67,7 +67,8 @@ enum RoutineId : int32_t {
     R_CONV_IM2COL_TC = 11,  // childnet: im2col -> tensor-core GEMM (any C, stride, dilation)
     R_DENSE_TC = 12,     // childnet: reshape -> 1x1 conv2 on tensor cores -> reshape (section III-D)
     R_CONV_S2D_TC = 13,  // childnet: space-to-depth -> stride-1 tensor-core conv (stride 2, <= 4 channels)
-    R_COUNT = 14
+    R_MUL = 14,          // per-channel scale (squeeze-and-excite)
+    R_COUNT = 15
 };
 
 // -------------------------------------------------------------------------
@@ -248,6 +249,7 @@ cudaError_t dwconv(const LaunchArgs &a);
 cudaError_t maxpool(const LaunchArgs &a);
 cudaError_t gap(const LaunchArgs &a);
 cudaError_t add(const LaunchArgs &a);
+cudaError_t mul(const LaunchArgs &a);
 cudaError_t dense(const LaunchArgs &a);
 int *device_error_word();  // device address of the library's error word
 }  // namespace k

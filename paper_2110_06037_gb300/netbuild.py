@@ -11,7 +11,7 @@ from . import _sn
 from .api import Graph
 
 TYPES = {"conv2": _sn.SN_L_CONV2, "dwconv2": _sn.SN_L_DWCONV2, "maxpool": _sn.SN_L_MAXPOOL,
-         "gap": _sn.SN_L_GAP, "add": _sn.SN_L_ADD, "dense": _sn.SN_L_DENSE}
+         "gap": _sn.SN_L_GAP, "add": _sn.SN_L_ADD, "dense": _sn.SN_L_DENSE, "mul": _sn.SN_L_MUL}
 
 
 def build_graph(layers, in_shape, in_schema, out_schema, schemas, torch_alloc=True) -> Graph:

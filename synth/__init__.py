@@ -50,6 +50,11 @@ def add(act="none", name=""):
     return {"name": name, "type": "add", "params": dict(act=act)}
 
 
+def mul(act="none", name=""):
+    """Per-channel scale: inputs (blob, N x C x 1 x 1 scale)."""
+    return {"name": name, "type": "mul", "params": dict(act=act)}
+
+
 def dense(fin, fout, act="none", name=""):
     return {"name": name, "type": "dense", "params": dict(in_features=fin, out_features=fout,
                                                           act=act)}
@@ -157,6 +162,52 @@ def mobilenet_v2(batch=1, seed=0, res=224):
     l = b.push(conv(c_in, 1280, 1, 1, act="relu6", name="head"), [l])
     l = b.push(gap(name="gap"), [l])
     b.push(dense(1280, 1000, name="fc"), [l])
+    return materialise(b.layers, (batch, 3, res, res), seed)
+
+
+def _make_divisible(v, d=8):
+    """Round v to the nearest multiple of d, not below 90 % of v (MobileNet rule)."""
+    r = max(d, int(v + d / 2) // d * d)
+    return r + d if r < 0.9 * v else r
+
+
+def mobilenet_v3(batch=1, seed=0, res=224):
+    """MobileNetV3-Large, width 1.0, BN folded: hard-swish stem; fifteen
+    bottlenecks (kernel, expansion, output, squeeze-excite, activation,
+    stride); a 1x1 conv to 960 channels; GAP; a 960 -> 1280 hard-swish layer
+    (the 1x1 conv on the pooled map, i.e. dense) and the 1280 -> 1000
+    classifier.  Squeeze-excite: GAP -> dense to make_divisible(exp/4) + ReLU
+    -> dense back to exp + hard sigmoid -> per-channel scale of the depthwise
+    output."""
+    spec = [(3, 16, 16, False, "relu", 1), (3, 64, 24, False, "relu", 2), (3, 72, 24, False, "relu", 1),
+            (5, 72, 40, True, "relu", 2), (5, 120, 40, True, "relu", 1), (5, 120, 40, True, "relu", 1),
+            (3, 240, 80, False, "hswish", 2), (3, 200, 80, False, "hswish", 1),
+            (3, 184, 80, False, "hswish", 1), (3, 184, 80, False, "hswish", 1),
+            (3, 480, 112, True, "hswish", 1), (3, 672, 112, True, "hswish", 1),
+            (5, 672, 160, True, "hswish", 2), (5, 960, 160, True, "hswish", 1),
+            (5, 960, 160, True, "hswish", 1)]
+    b = _Builder()
+    l = b.push(conv(3, 16, 3, 2, act="hswish", name="stem"), [-1])
+    c_in = 16
+    for blk, (k, exp, out, se, nl, s) in enumerate(spec):
+        x_in = l
+        if exp != c_in:
+            l = b.push(conv(c_in, exp, 1, 1, act=nl, name=f"b{blk}.expand"), [l])
+        l = b.push(dwconv(exp, k, s, act=nl, name=f"b{blk}.dw"), [l])
+        if se:
+            red = _make_divisible(exp // 4)
+            g = b.push(gap(name=f"b{blk}.se.gap"), [l])
+            g = b.push(dense(exp, red, act="relu", name=f"b{blk}.se.fc1"), [g])
+            g = b.push(dense(red, exp, act="hsigmoid", name=f"b{blk}.se.fc2"), [g])
+            l = b.push(mul(name=f"b{blk}.se.scale"), [l, g])
+        l = b.push(conv(exp, out, 1, 1, act="none", name=f"b{blk}.project"), [l])
+        if s == 1 and c_in == out:
+            l = b.push(add(name=f"b{blk}.add"), [x_in, l])
+        c_in = out
+    l = b.push(conv(c_in, 960, 1, 1, act="hswish", name="head"), [l])
+    l = b.push(gap(name="gap"), [l])
+    l = b.push(dense(960, 1280, act="hswish", name="fc1"), [l])
+    b.push(dense(1280, 1000, name="fc2"), [l])
     return materialise(b.layers, (batch, 3, res, res), seed)
 
 

@@ -244,10 +244,11 @@ def test_golden_net_c_through_abi():
     assert tot == gold["expect_cost"] and list(sch) == gold["expect_assign"]
 
 
-@pytest.mark.parametrize("net", ["resnet50", "mobilenet_v2", "vgg16"])
+@pytest.mark.parametrize("net", ["resnet50", "mobilenet_v2", "vgg16", "mobilenet_v3"])
 def test_dprs_equals_blockwise_search_on_real_nets(net):
     """Nets too large to enumerate: the oracle's block-wise exact search."""
-    build = {"resnet50": synth.resnet50, "mobilenet_v2": synth.mobilenet_v2, "vgg16": synth.vgg16}[net]
+    build = {"resnet50": synth.resnet50, "mobilenet_v2": synth.mobilenet_v2, "vgg16": synth.vgg16,
+             "mobilenet_v3": synth.mobilenet_v3}[net]
     _, layers = build(1, res=32)
     sch = [("f16", "nchw"), ("f16", "nhwc")]
     g = build_graph(layers, (1, 3, 32, 32), ("f32", "nchw"), ("f32", "nchw"), sch, torch_alloc=False)

@@ -7,8 +7,8 @@
   * MobileNetV2 b1 fp16, ResNet-50 b1 fp16: DPRS equals the oracle's exact
     block-wise search on the profiled table; output within 2e-2.
   * ResNet-50 b32 bf16: sampled images of the batch against the oracle.
-  * VGG16 bf16 (64x64 input, batch 2): DPRS equals the block-wise search;
-    output within 2e-2.
+  * VGG16 bf16 (64x64 input, batch 2) and MobileNetV3-Large b1 fp16: DPRS
+    equals the block-wise search; output within 2e-2.
   * The same nets with every residual add fused into its conv2: DPRS equals
     the block-wise search, outputs within 2e-2 of the (unfused) oracle.
 """
@@ -98,6 +98,14 @@ def test_mixed_precision_schemas_tiny():
 
 def test_mobilenet_v2_b1_fp16():
     x, layers = synth.mobilenet_v2(1)
+    g, got = _profile_select_run(layers, x, ("f16", "nchw"), ("f16", "nchw"), F16, exhaustive=False)
+    ref = run_net(layers, x, "f16")
+    assert maxrel(got, ref) <= TOL["f16"]
+
+
+def test_mobilenet_v3_b1_fp16():
+    """MobileNetV3-Large: hard swish / hard sigmoid, squeeze-excite scales."""
+    x, layers = synth.mobilenet_v3(1)
     g, got = _profile_select_run(layers, x, ("f16", "nchw"), ("f16", "nchw"), F16, exhaustive=False)
     ref = run_net(layers, x, "f16")
     assert maxrel(got, ref) <= TOL["f16"]

@@ -8,7 +8,7 @@ import pytest
 
 import oracle
 import synth
-from oracle.net import run_layer
+from oracle.net import run_layer, run_net
 from paper_2110_06037_gb300 import build_graph, convert
 
 from gpu_helpers import TOL, find_candidate, from_device, maxrel, raw_bits, stored_values, to_device
@@ -143,6 +143,51 @@ def test_pool_gap_add_dense(schema):
         if got is not None:
             assert schema[0] != "f32"
             assert maxrel(got, ref) <= TOL[schema[0]], v
+
+
+@pytest.mark.parametrize("shape", [(2, 16, 13, 11), (1, 40, 7, 7), (3, 12, 5, 5)])
+@pytest.mark.parametrize("schema", SCHEMAS)
+def test_mul_squeeze_excite_scale(shape, schema):
+    """gap -> per-channel scale of the same blob (+ hard swish): the vector NHWC
+    kernel (C * elem a multiple of 16 bytes), the element kernel otherwise."""
+    import torch
+    rng = np.random.default_rng(zlib.crc32(repr((shape, schema, "mul")).encode()))
+    x = (rng.standard_normal(shape) * 2).astype(np.float32)
+    net = [dict(synth.gap(), inputs=[-1]), dict(synth.mul(act="hswish"), inputs=[-1, 0])]
+    ref = run_net(net, x, schema[0])
+    g = build_graph(net, x.shape, schema, schema, [schema])
+    t = g.cost_table()
+    pc = [int(np.flatnonzero(t["layer"] == 0)[0]), find_candidate(t, 1, "gap/reduce", 0, 0),
+          find_candidate(t, 2, "mul/eltwise", 0, 0), int(np.flatnonzero(t["layer"] == 3)[0])]
+    g.set_path(pc)
+    y = g.run(to_device(x, schema))
+    torch.cuda.synchronize()
+    assert maxrel(from_device(y, schema), ref) <= TOL[schema[0]]
+
+
+@pytest.mark.parametrize("act", ["hswish", "hsigmoid"])
+@pytest.mark.parametrize("schema", [("f32", "nchw"), ("f16", "nhwc"), ("bf16", "nhwc")])
+def test_conv_hard_activations(act, schema):
+    """MobileNetV3's activations in the epilogues of every conv routine the
+    layer offers (direct, SIMT GEMM, Winograd, tensor cores)."""
+    import torch
+    rng = np.random.default_rng(zlib.crc32(repr((act, schema)).encode()))
+    x = (rng.standard_normal((2, 32, 9, 9)) * 2).astype(np.float32)
+    layer = synth.conv(32, 64, 3, 1, 1, act=act)
+    layer["weight"] = (rng.standard_normal((64, 32, 3, 3)) * np.sqrt(2 / 288)).astype(np.float32)
+    layer["bias"] = (rng.standard_normal(64) * 0.5).astype(np.float32)
+    ref = ref_one(layer, x, schema[0])
+    g = build_graph([dict(layer, inputs=[-1])], x.shape, schema, schema, [schema])
+    t = g.cost_table()
+    io = [int(np.flatnonzero(t["layer"] == 0)[0]), int(np.flatnonzero(t["layer"] == 2)[0])]
+    ran = 0
+    for c in np.flatnonzero(t["layer"] == 1):
+        g.set_path([io[0], int(c), io[1]])
+        y = g.run(to_device(x, schema))
+        torch.cuda.synchronize()
+        assert maxrel(from_device(y, schema), ref) <= TOL[schema[0]], int(t["routine"][c])
+        ran += 1
+    assert ran >= 2
 
 
 # planes of 196 (8-byte bf16 rows, 16-byte f32 rows), 49 (element-wide rows)

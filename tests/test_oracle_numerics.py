@@ -102,6 +102,30 @@ def test_bias_and_activations():
                                   np.clip(x[0, 0, 0] + 0.5, 0, 6))
 
 
+def test_hard_swish_and_hard_sigmoid_closed_forms():
+    """MobileNetV3's piecewise-linear activations at their knots and in each
+    piece: hswish(x) = x relu6(x + 3) / 6, hsigmoid(x) = relu6(x + 3) / 6."""
+    x = np.array([-10.0, -4.0, -3.0, -1.5, 0.0, 1.0, 1.5, 3.0, 4.0, 10.0])
+    z = np.zeros_like(x)
+    hsw = oracle.add(x, z, act="hswish")
+    hsg = oracle.add(x, z, act="hsigmoid")
+    np.testing.assert_allclose(hsw, [0.0, 0.0, 0.0, -0.375, 0.0, 2.0 / 3.0, 1.125, 3.0, 4.0, 10.0], rtol=0, atol=1e-15)
+    np.testing.assert_allclose(hsg, [0.0, 0.0, 0.0, 0.25, 0.5, 2.0 / 3.0, 0.75, 1.0, 1.0, 1.0], rtol=0, atol=1e-15)
+    # the two are consistent: hswish = x * hsigmoid
+    np.testing.assert_allclose(hsw, x * hsg, rtol=0, atol=1e-15)
+
+
+def test_mul_scales_each_channel():
+    """Per-channel scale: a hand case, then the identity and zero scales."""
+    x = np.arange(2 * 3 * 2 * 2, dtype=np.float64).reshape(2, 3, 2, 2)
+    s = np.array([[1.0, -2.0, 0.5], [0.0, 3.0, -1.0]])
+    y = oracle.mul(x, s)
+    assert y[0, 1, 1, 0] == x[0, 1, 1, 0] * -2.0 and y[1, 0, 0, 1] == 0.0 and y[1, 2, 1, 1] == -x[1, 2, 1, 1]
+    np.testing.assert_array_equal(oracle.mul(x, np.ones((2, 3, 1, 1))), x)
+    np.testing.assert_array_equal(oracle.mul(x, np.zeros((2, 3))), np.zeros_like(x))
+    np.testing.assert_array_equal(oracle.mul(x, np.full((2, 3), 2.0), act="relu6"), np.clip(2 * x, 0, 6))
+
+
 @pytest.mark.parametrize("case", [
     # N, C, H, W, K, R, S, stride, pad, dil, groups
     (1, 3, 11, 13, 4, 3, 3, (1, 1), (1, 1), (1, 1), 1),

@@ -34,3 +34,21 @@ def test_vgg16_fc6_equals_dense_over_the_flattened_map():
     ref = np.maximum(w @ feat.reshape(-1) + fc6["bias"], 0.0)
     got = run_net(layers[: i6 + 1], x, "f32").reshape(-1)
     assert np.max(np.abs(got - ref)) <= 1e-9 * max(1.0, np.max(np.abs(ref)))
+
+
+def test_mobilenet_v3_large_structure():
+    x, layers = synth.mobilenet_v3(1, res=64)
+    kinds = [l["type"] for l in layers]
+    assert kinds.count("dwconv2") == 15 and kinds.count("mul") == 8 and kinds.count("add") == 10
+    dws = [l["params"]["kh"] for l in layers if l["type"] == "dwconv2"]
+    assert dws == [3, 3, 3, 5, 5, 5, 3, 3, 3, 3, 3, 3, 5, 5, 5]
+    # squeeze-excite widths: make_divisible(exp / 4, 8)
+    red = [l["params"]["out_features"] for l in layers if l.get("name", "").endswith(".se.fc1")]
+    assert red == [24, 32, 32, 120, 168, 168, 240, 240]
+    acts = {l["params"].get("act") for l in layers if l["type"] in ("conv2", "dwconv2", "dense")}
+    assert {"hswish", "hsigmoid", "relu", "none"} <= acts
+    for l in layers:
+        if l["type"] == "mul":
+            assert layers[l["inputs"][1]].get("name", "").endswith(".se.fc2")
+    y = run_net(layers, x, "f32")
+    assert y.shape == (1, 1000, 1, 1) and np.all(np.isfinite(y))
