@@ -293,8 +293,43 @@ __global__ void weight_wino_kernel(const float *__restrict__ w, T *__restrict__ 
     }
 }
 
+// Winograd F(4x4,3x3) filter transform U = G g G^T with Lavin & Gray's 6x3
+// G (points 0, +-1, +-2, infinity), fp32 [36][K][C]
+__device__ __forceinline__ void wino4_g(float g0, float g1, float g2, float (&u)[6]) {
+    u[0] = 0.25f * g0;
+    u[1] = -(g0 + g1 + g2) / 6.f;
+    u[2] = -(g0 - g1 + g2) / 6.f;
+    u[3] = g0 / 24.f + g1 / 12.f + g2 / 6.f;
+    u[4] = g0 / 24.f - g1 / 12.f + g2 / 6.f;
+    u[5] = g2;
+}
+__global__ void weight_wino4_kernel(const float *__restrict__ w, float *__restrict__ out, int64_t K, int64_t C) {
+    griddep_launch();
+    griddep_wait();
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < K * C;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const float *g = w + i * 9;  // [3][3] for (k, c) = (i / C, i % C)
+        float t[6][3];               // G g, column by column
+        for (int j = 0; j < 3; ++j) {
+            float u[6];
+            wino4_g(g[0 * 3 + j], g[1 * 3 + j], g[2 * 3 + j], u);
+            for (int a = 0; a < 6; ++a) t[a][j] = u[a];
+        }
+        for (int a = 0; a < 6; ++a) {  // (G g) G^T
+            float u[6];
+            wino4_g(t[a][0], t[a][1], t[a][2], u);
+            for (int b = 0; b < 6; ++b) out[(int64_t)(a * 6 + b) * K * C + i] = u[b];
+        }
+    }
+}
+
 cudaError_t weight_format(const float *w, void *out, int fmt, int dt, int64_t K, int64_t Cg,
                           int64_t R, int64_t S, cudaStream_t st) {
+    if (fmt == W_WINO4) {  // fp32 whatever the schema's dtype
+        if (R != 3 || S != 3) return cudaErrorInvalidValue;
+        launch_pdl(weight_wino4_kernel, grid_for(K * Cg, 256), 256, 0, st, w, (float *)out, K, Cg);
+        return cudaGetLastError();
+    }
     if (fmt == W_WINO) {
         if (R != 3 || S != 3) return cudaErrorInvalidValue;
         SN_DT_SWITCH(dt, T, launch_pdl(weight_wino_kernel<T>, grid_for(K * Cg, 256), 256, 0, st, w, (T *)out, K, Cg));

@@ -365,6 +365,162 @@ cudaError_t conv_wino(const LaunchArgs &a) {
     return cudaGetLastError();
 }
 
+// ---------------------------------------------------------------------------
+// Winograd F(4x4, 3x3): 6x6 input tiles, 36 element-wise GEMMs, 4x4 outputs
+// (Lavin & Gray's interpolation points 0, +-1, +-2 and infinity).  The
+// transformed filters are kept in fp32 whatever the schema (the larger
+// transform coefficients would amplify a 16-bit rounding of U).
+// ---------------------------------------------------------------------------
+static WinoDims wino4_dims(const ConvDims &d) {
+    WinoDims w;
+    w.d = d;
+    w.tP = (d.P + 3) / 4;
+    w.tQ = (d.Q + 3) / 4;
+    w.T = (int64_t)d.N * w.tP * w.tQ;
+    return w;
+}
+
+size_t conv_wino4_ws(const Layer &l, const Shape &in, sn_schema s) {
+    (void)s;
+    const int64_t tiles = in.n * ((l.out.h + 3) / 4) * ((l.out.w + 3) / 4);
+    return (size_t)36 * tiles * (in.c + l.out.c) * sizeof(float);
+}
+
+// r = B^T d for one column d of the 6x6 tile
+__device__ __forceinline__ void wino4_bt(const float (&d)[6], float (&r)[6]) {
+    r[0] = 4.f * d[0] - 5.f * d[2] + d[4];
+    r[1] = -4.f * d[1] - 4.f * d[2] + d[3] + d[4];
+    r[2] = 4.f * d[1] - 4.f * d[2] - d[3] + d[4];
+    r[3] = -2.f * d[1] - d[2] + 2.f * d[3] + d[4];
+    r[4] = 2.f * d[1] - d[2] - 2.f * d[3] + d[4];
+    r[5] = 4.f * d[1] - 5.f * d[3] + d[5];
+}
+// o = A^T m for one column m
+__device__ __forceinline__ void wino4_at(const float (&m)[6], float (&o)[4]) {
+    o[0] = m[0] + m[1] + m[2] + m[3] + m[4];
+    o[1] = m[1] - m[2] + 2.f * (m[3] - m[4]);
+    o[2] = m[1] + m[2] + 4.f * (m[3] + m[4]);
+    o[3] = m[1] - m[2] + 8.f * (m[3] - m[4]) + m[5];
+}
+
+// wgenc: V[xi][t][c] = (B^T d B)[xi] for the 6x6 input tile of output tile t
+template <typename T, bool NHWC>
+__global__ void wino4_input_kernel(const T *__restrict__ x, float *__restrict__ V, WinoDims wd) {
+    griddep_launch();
+    griddep_wait();
+    const ConvDims &d = wd.d;
+    const int64_t total = wd.T * d.C;
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const int c = (int)(i % d.C);
+        const int64_t t = i / d.C;
+        const int tq = (int)(t % wd.tQ), tp = (int)((t / wd.tQ) % wd.tP);
+        const int64_t n = t / ((int64_t)wd.tQ * wd.tP);
+        const int h0 = 4 * tp - d.ph, w0 = 4 * tq - d.pw;
+        float v[6][6];
+#pragma unroll
+        for (int a = 0; a < 6; ++a)
+#pragma unroll
+            for (int b = 0; b < 6; ++b) {
+                const int h = h0 + a, ww = w0 + b;
+                float val = 0.f;
+                if (h >= 0 && h < d.H && ww >= 0 && ww < d.W) {
+                    const int64_t idx = NHWC ? ((n * d.H + h) * d.W + ww) * d.C + c
+                                             : ((n * d.C + c) * d.H + h) * (int64_t)d.W + ww;
+                    val = ldf<T>(x + idx);
+                }
+                v[a][b] = val;
+            }
+        float t6[6][6];  // B^T d, column by column
+#pragma unroll
+        for (int b = 0; b < 6; ++b) {
+            const float col[6] = {v[0][b], v[1][b], v[2][b], v[3][b], v[4][b], v[5][b]};
+            float r[6];
+            wino4_bt(col, r);
+#pragma unroll
+            for (int a = 0; a < 6; ++a) t6[a][b] = r[a];
+        }
+#pragma unroll
+        for (int a = 0; a < 6; ++a) {  // (B^T d) B: B^T applied to each row
+            float r[6];
+            wino4_bt(t6[a], r);
+#pragma unroll
+            for (int b = 0; b < 6; ++b) V[((int64_t)(a * 6 + b) * wd.T + t) * d.C + c] = r[b];
+        }
+    }
+}
+
+// wgdec: Y = A^T M A for each output tile, + bias, activation, store
+template <typename T, bool NHWC>
+__global__ void wino4_output_kernel(const float *__restrict__ Mx, const float *__restrict__ bias,
+                                    T *__restrict__ y, WinoDims wd) {
+    griddep_launch();
+    griddep_wait();
+    const ConvDims &d = wd.d;
+    const int64_t total = wd.T * d.K;
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const int kk = (int)(i % d.K);
+        const int64_t t = i / d.K;
+        const int tq = (int)(t % wd.tQ), tp = (int)((t / wd.tQ) % wd.tP);
+        const int64_t n = t / ((int64_t)wd.tQ * wd.tP);
+        float u[4][6];  // A^T M, column by column
+#pragma unroll
+        for (int b = 0; b < 6; ++b) {
+            float col[6];
+#pragma unroll
+            for (int a = 0; a < 6; ++a) col[a] = Mx[((int64_t)(a * 6 + b) * wd.T + t) * d.K + kk];
+            float o[4];
+            wino4_at(col, o);
+#pragma unroll
+            for (int a = 0; a < 4; ++a) u[a][b] = o[a];
+        }
+        const float bv = bias[kk];
+#pragma unroll
+        for (int a = 0; a < 4; ++a) {
+            const int p = 4 * tp + a;
+            if (p >= d.P) continue;
+            float yy[4];
+            wino4_at(u[a], yy);
+#pragma unroll
+            for (int b = 0; b < 4; ++b) {
+                const int q = 4 * tq + b;
+                if (q >= d.Q) continue;
+                const int64_t o = NHWC ? ((n * d.P + p) * d.Q + q) * d.K + kk
+                                       : ((n * d.K + kk) * d.P + p) * (int64_t)d.Q + q;
+                stf<T>(y + o, act_apply(yy[b] + bv, d.act));
+            }
+        }
+    }
+}
+
+cudaError_t conv_wino4(const LaunchArgs &a) {
+    const ConvDims d = conv_dims(a);
+    const WinoDims wd = wino4_dims(d);
+    const size_t need = (size_t)36 * wd.T * (d.C + d.K) * sizeof(float);
+    if (!a.ws || a.ws_bytes < need) return cudaErrorInvalidValue;
+    float *V = static_cast<float *>(a.ws);
+    float *Mx = V + (size_t)36 * wd.T * d.C;
+    dim3 ggrid((unsigned)((wd.T + 63) / 64), (unsigned)((d.K + 63) / 64), 36);
+    if (ggrid.y > 65535) return cudaErrorInvalidValue;
+    SN_DT_SWITCH(a.schema.dtype, T, {
+        if (a.schema.layout == SN_NHWC)
+            launch_pdl(wino4_input_kernel<T, true>, grid_for(wd.T * d.C, 256), 256, 0, a.stream, (const T *)a.in[0],
+                       V, wd);
+        else
+            launch_pdl(wino4_input_kernel<T, false>, grid_for(wd.T * d.C, 256), 256, 0, a.stream,
+                       (const T *)a.in[0], V, wd);
+        launch_pdl(gemm_nt_simt<float>, ggrid, 256, 0, a.stream, V, (const float *)a.wt, Mx, wd.T, d.K, d.C);
+        if (a.schema.layout == SN_NHWC)
+            launch_pdl(wino4_output_kernel<T, true>, grid_for(wd.T * d.K, 256), 256, 0, a.stream, Mx, a.bias,
+                       (T *)a.out, wd);
+        else
+            launch_pdl(wino4_output_kernel<T, false>, grid_for(wd.T * d.K, 256), 256, 0, a.stream, Mx, a.bias,
+                       (T *)a.out, wd);
+    });
+    return cudaGetLastError();
+}
+
 // The three Winograd stages on caller-provided buffers (used by the
 // allocation-free entry point): U [16][K][C] in the schema dtype, V and Mx fp32.
 cudaError_t conv_wino_buffers(const ConvDims &d, sn_schema s, const void *x, const void *u, const float *bias,
