@@ -34,12 +34,14 @@ template <> __device__ __forceinline__ __nv_bfloat16 cvt<__nv_bfloat16>(float v)
     return __float2bfloat16_rn(v);
 }
 
+// The common activations first, as before the hard-swish pair was added: in
+// an unrolled epilogue every extra test of `act` is paid per element.
 __device__ __forceinline__ float act_apply(float v, int act) {
     if (act == SN_ACT_RELU) return fmaxf(v, 0.0f);
+    if (act == SN_ACT_NONE) return v;
     if (act == SN_ACT_RELU6) return fminf(fmaxf(v, 0.0f), 6.0f);
-    if (act == SN_ACT_HSWISH) return v * fminf(fmaxf(v + 3.0f, 0.0f), 6.0f) / 6.0f;
-    if (act == SN_ACT_HSIGMOID) return fminf(fmaxf(v + 3.0f, 0.0f), 6.0f) / 6.0f;
-    return v;
+    const float t = fminf(fmaxf(v + 3.0f, 0.0f), 6.0f) / 6.0f;  // hard sigmoid
+    return act == SN_ACT_HSWISH ? v * t : t;
 }
 
 // streaming multiprocessors of the current device (host)

@@ -144,20 +144,21 @@ static int row_vec_bytes(int64_t n, int es, const void *base) {
 
 // few channels (C <= 16): one thread per pixel moves all of its channels;
 // the planar side is read/written coalesced across threads, the interleaved
-// side as C consecutive elements per thread (C * 32 contiguous per warp)
+// side as C consecutive elements per thread (C * 32 contiguous per warp).
+// Grid: y = image, x = pixels of the image (no index division).
 template <typename Ti, typename To, bool TO_NHWC>
-__global__ void permute_small_c_kernel(const Ti *__restrict__ x, To *__restrict__ y, int64_t N, int C, int64_t HW) {
+__global__ void permute_small_c_kernel(const Ti *__restrict__ x, To *__restrict__ y, int N, int C, int HW) {
     griddep_launch();
     griddep_wait();
-    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < N * HW;
-         i += (int64_t)gridDim.x * blockDim.x) {
-        const int64_t n = i / HW, hw = i % HW;
-        for (int c = 0; c < C; ++c) {
-            const int64_t planar = (n * C + c) * HW + hw, inter = i * C + c;
-            if (TO_NHWC) stf<To>(y + inter, ldf<Ti>(x + planar));
-            else stf<To>(y + planar, ldf<Ti>(x + inter));
+    for (int n = blockIdx.y; n < N; n += gridDim.y)
+        for (int hw = blockIdx.x * blockDim.x + threadIdx.x; hw < HW; hw += gridDim.x * blockDim.x) {
+            const size_t planar0 = (size_t)n * C * HW + hw, inter0 = ((size_t)n * HW + hw) * C;
+            for (int c = 0; c < C; ++c) {
+                const size_t planar = planar0 + (size_t)c * HW, inter = inter0 + c;
+                if (TO_NHWC) stf<To>(y + inter, ldf<Ti>(x + planar));
+                else stf<To>(y + planar, ldf<Ti>(x + inter));
+            }
         }
-    }
 }
 
 template <typename Ti, typename To>
@@ -182,13 +183,15 @@ static cudaError_t convert_t(const void *x, int lay_in, void *y, int lay_out, Sh
         return cudaGetLastError();
     }
     if (s.c <= 16) {
-        const int64_t px = s.n * s.h * s.w;
+        const int64_t HW = s.h * s.w;
+        if (HW >= ((int64_t)1 << 31) || s.n >= ((int64_t)1 << 31)) return cudaErrorInvalidValue;
+        const dim3 g((unsigned)std::min<int64_t>((HW + 255) / 256, 1024), (unsigned)std::min<int64_t>(s.n, 65535));
         if (lay_in == SN_NCHW)
-            launch_pdl(permute_small_c_kernel<Ti, To, true>, grid_for(px, 256), 256, 0, st, (const Ti *)x, (To *)y, s.n,
-                                                                                     (int)s.c, s.h * s.w);
+            launch_pdl(permute_small_c_kernel<Ti, To, true>, g, 256, 0, st, (const Ti *)x, (To *)y, (int)s.n, (int)s.c,
+                       (int)HW);
         else
-            launch_pdl(permute_small_c_kernel<Ti, To, false>, grid_for(px, 256), 256, 0, st, (const Ti *)x, (To *)y, s.n,
-                                                                                      (int)s.c, s.h * s.w);
+            launch_pdl(permute_small_c_kernel<Ti, To, false>, g, 256, 0, st, (const Ti *)x, (To *)y, (int)s.n,
+                       (int)s.c, (int)HW);
         return cudaGetLastError();
     }
     // NCHW -> NHWC: per image [C][HW] -> [HW][C]; NHWC -> NCHW: [HW][C] -> [C][HW]
@@ -888,39 +891,57 @@ __global__ void maxpool_kernel(const T *__restrict__ x, T *__restrict__ y, int N
 }
 
 // NHWC, 16 bytes of channels per thread (8 x 16-bit or 4 x fp32 lanes)
+// NHWC, 16-byte channel vectors: the grid's y axis walks the N x P output
+// rows, its x axis the (column, channel vector) pairs of a row, channel vector
+// fastest (coalesced); 32-bit index math, one division per thread.  Packed
+// 16-bit max (exact: the result is one of the stored values).
 template <typename T>
-__global__ void maxpool_nhwc_vec(const uint4 *__restrict__ x, uint4 *__restrict__ y, int N, int C16, int H, int W,
-                                 int P, int Q, int kh, int kw, int sh, int sw, int ph, int pw) {
+__device__ __forceinline__ uint32_t max2(uint32_t a, uint32_t b);
+template <>
+__device__ __forceinline__ uint32_t max2<__half>(uint32_t a, uint32_t b) {
+    const __half2 r = __hmax2(*reinterpret_cast<const __half2 *>(&a), *reinterpret_cast<const __half2 *>(&b));
+    return *reinterpret_cast<const uint32_t *>(&r);
+}
+template <>
+__device__ __forceinline__ uint32_t max2<__nv_bfloat16>(uint32_t a, uint32_t b) {
+    const __nv_bfloat162 r =
+        __hmax2(*reinterpret_cast<const __nv_bfloat162 *>(&a), *reinterpret_cast<const __nv_bfloat162 *>(&b));
+    return *reinterpret_cast<const uint32_t *>(&r);
+}
+template <>
+__device__ __forceinline__ uint32_t max2<float>(uint32_t a, uint32_t b) {
+    return __float_as_uint(fmaxf(__uint_as_float(a), __uint_as_float(b)));
+}
+
+template <typename T>
+__global__ void __launch_bounds__(256) maxpool_nhwc_vec(const uint4 *__restrict__ x, uint4 *__restrict__ y, int N,
+                                                       int C16, int H, int W, int P, int Q, int kh, int kw, int sh,
+                                                       int sw, int ph, int pw) {
     griddep_launch();
     griddep_wait();
-    constexpr int E = 16 / sizeof(T);
-    const int64_t total = (int64_t)N * P * Q * C16;
-    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total;
-         i += (int64_t)gridDim.x * blockDim.x) {
-        const int cv = (int)(i % C16);
-        const int64_t pix = i / C16;
-        const int q = (int)(pix % Q), p = (int)((pix / Q) % P);
-        const int64_t n = pix / ((int64_t)Q * P);
-        float m[E];
-#pragma unroll
-        for (int e = 0; e < E; ++e) m[e] = -INFINITY;
+    const int t = blockIdx.x * blockDim.x + threadIdx.x;
+    if (t >= Q * C16) return;
+    const int q = t / C16, cv = t - q * C16;
+    // -inf in every lane (16-bit: 0xfc00 half, 0xff80 bfloat16; fp32: 0xff800000)
+    const uint32_t ninf = sizeof(T) == 4 ? 0xff800000u : (std::is_same<T, __half>::value ? 0xfc00fc00u : 0xff80ff80u);
+    for (int row = blockIdx.y; row < N * P; row += gridDim.y) {
+        const int n = row / P, p = row - n * P;
+        uint4 m = make_uint4(ninf, ninf, ninf, ninf);
         for (int r = 0; r < kh; ++r) {
             const int h = p * sh - ph + r;
             if (h < 0 || h >= H) continue;
-            for (int s = 0; s < kw; ++s) {
-                const int ww = q * sw - pw + s;
+            const uint4 *xr = x + ((size_t)(n * H + h) * W) * C16 + cv;
+            for (int s2 = 0; s2 < kw; ++s2) {
+                const int ww = q * sw - pw + s2;
                 if (ww < 0 || ww >= W) continue;
-                const uint4 v = x[((n * H + h) * W + ww) * C16 + cv];
-                const T *pv = reinterpret_cast<const T *>(&v);
-#pragma unroll
-                for (int e = 0; e < E; ++e) m[e] = fmaxf(m[e], ldf<T>(pv + e));
+                const uint4 v = xr[(size_t)ww * C16];
+                m.x = max2<T>(m.x, v.x);
+                m.y = max2<T>(m.y, v.y);
+                m.z = max2<T>(m.z, v.z);
+                m.w = max2<T>(m.w, v.w);
             }
         }
-        uint4 o;
-        T *po = reinterpret_cast<T *>(&o);
-#pragma unroll
-        for (int e = 0; e < E; ++e) po[e] = cvt<T>(m[e]);  // exact: m is one of the stored values
-        y[i] = o;
+        y[((size_t)row * Q + q) * C16 + cv] = m;
     }
 }
 
@@ -933,9 +954,9 @@ cudaError_t maxpool(const LaunchArgs &a) {
         if (a.schema.layout == SN_NHWC && cb % 16 == 0 && (uintptr_t)a.in[0] % 16 == 0 &&
             (uintptr_t)a.out % 16 == 0) {
             const int c16 = (int)(cb / 16);
-            launch_pdl(maxpool_nhwc_vec<T>, grid_for(o.n * o.h * o.w * c16, 256), 256, 0, a.stream, 
-                (const uint4 *)a.in[0], (uint4 *)a.out, (int)i.n, c16, (int)i.h, (int)i.w, (int)o.h, (int)o.w,
-                p.kh, p.kw, p.sh, p.sw, p.ph, p.pw);
+            const dim3 g((unsigned)((o.w * c16 + 255) / 256), (unsigned)std::min<int64_t>(o.n * o.h, 65535));
+            launch_pdl(maxpool_nhwc_vec<T>, g, 256, 0, a.stream, (const uint4 *)a.in[0], (uint4 *)a.out, (int)i.n,
+                       c16, (int)i.h, (int)i.w, (int)o.h, (int)o.w, p.kh, p.kw, p.sh, p.sw, p.ph, p.pw);
         } else if (a.schema.layout == SN_NHWC)
             launch_pdl(maxpool_kernel<T, true>, grid_for(total, 256), 256, 0, a.stream, 
                 (const T *)a.in[0], (T *)a.out, (int)i.n, (int)i.c, (int)i.h, (int)i.w, (int)o.h, (int)o.w,
@@ -963,6 +984,47 @@ __global__ void gap_nchw(const T *__restrict__ x, T *__restrict__ y, int64_t NC,
     }
 }
 
+// NHWC, 16-byte channel vectors: a block of 32 channel vectors x 8 pixel
+// slices per (image, 32-vector group); each thread sums its slice's pixels in
+// f32, the block adds the 8 slices in order through shared memory
+template <typename T>
+__global__ void __launch_bounds__(256) gap_nhwc_vec(const T *__restrict__ x, T *__restrict__ y, int C, int HW) {
+    griddep_launch();
+    griddep_wait();
+    constexpr int E = 16 / sizeof(T);
+    __shared__ float part[8][32][E + 1];
+    const int cvl = threadIdx.x & 31, sl = threadIdx.x >> 5;
+    const int n = blockIdx.y;
+    const int CV = C / E;
+    const int cv = blockIdx.x * 32 + cvl;
+    float s[E];
+#pragma unroll
+    for (int e = 0; e < E; ++e) s[e] = 0.f;
+    if (cv < CV) {
+        const T *xn = x + (size_t)n * HW * C + (size_t)cv * E;
+        for (int p = sl; p < HW; p += 8) {
+            const uint4 v = *reinterpret_cast<const uint4 *>(xn + (size_t)p * C);
+            const T *pv = reinterpret_cast<const T *>(&v);
+#pragma unroll
+            for (int e = 0; e < E; ++e) s[e] += ldf<T>(pv + e);
+        }
+    }
+#pragma unroll
+    for (int e = 0; e < E; ++e) part[sl][cvl][e] = s[e];
+    __syncthreads();
+    if (sl == 0 && cv < CV) {
+        uint4 o;
+        T *po = reinterpret_cast<T *>(&o);
+#pragma unroll
+        for (int e = 0; e < E; ++e) {
+            float t = 0.f;
+            for (int k = 0; k < 8; ++k) t += part[k][cvl][e];
+            po[e] = cvt<T>(t / (float)HW);
+        }
+        *reinterpret_cast<uint4 *>(y + (size_t)n * C + (size_t)cv * E) = o;
+    }
+}
+
 // NHWC: one thread per (n, c); consecutive threads read consecutive channels
 template <typename T>
 __global__ void gap_nhwc(const T *__restrict__ x, T *__restrict__ y, int64_t N, int64_t C, int64_t HW) {
@@ -983,7 +1045,12 @@ cudaError_t gap(const LaunchArgs &a) {
         if (a.schema.layout == SN_NCHW)
             launch_pdl(gap_nchw<T>, grid_for(i.n * i.c * 32, 256), 256, 0, a.stream, (const T *)a.in[0], (T *)a.out,
                                                                                i.n * i.c, i.h * i.w);
-        else
+        else if ((i.c * (int64_t)sizeof(T)) % 16 == 0 && (uintptr_t)a.in[0] % 16 == 0 && (uintptr_t)a.out % 16 == 0 &&
+                 i.n <= 65535 && i.h * i.w * i.c < ((int64_t)1 << 31)) {
+            const int CV = (int)(i.c * (int64_t)sizeof(T) / 16);
+            launch_pdl(gap_nhwc_vec<T>, dim3((unsigned)((CV + 31) / 32), (unsigned)i.n), 256, 0, a.stream,
+                       (const T *)a.in[0], (T *)a.out, (int)i.c, (int)(i.h * i.w));
+        } else
             launch_pdl(gap_nhwc<T>, grid_for(i.n * i.c, 256), 256, 0, a.stream, (const T *)a.in[0], (T *)a.out, i.n,
                                                                          i.c, i.h * i.w);
     });

@@ -588,26 +588,33 @@ __global__ void __launch_bounds__(THREADS, 1)
                         xph ^= 1u;
                     }
                     // every 4 packed pairs (8 channels) go to their 16-byte piece
-                    // of the row as soon as they are computed
+                    // of the row as soon as they are computed; the activation is
+                    // chosen once per chunk, so the unrolled body carries only its own
+                    auto stage_rows = [&](auto act) {
 #pragma unroll
-                    for (int q = 0; q < 8; ++q) {
-                        const int h = q >> 2;
-                        uint32_t wq[4];
+                        for (int q = 0; q < 8; ++q) {
+                            const int h = q >> 2;
+                            uint32_t wq[4];
 #pragma unroll
-                        for (int e = 0; e < 4; ++e) {
-                            const int j = 4 * (q & 3) + e;  // pair index within the half
-                            const float2 r2 = unpack2<T>(rv[h][j]);
-                            const float f0 = act_apply(__uint_as_float(v[32 * h + 2 * j]) +
-                                                           __shfl_sync(0xffffffffu, bias_r[cj][h], 2 * j) + r2.x,
-                                                       p.act);
-                            const float f1 = act_apply(__uint_as_float(v[32 * h + 2 * j + 1]) +
-                                                           __shfl_sync(0xffffffffu, bias_r[cj][h], 2 * j + 1) + r2.y,
-                                                       p.act);
-                            wq[e] = pack2<T>(f0, f1);
+                            for (int e = 0; e < 4; ++e) {
+                                const int j = 4 * (q & 3) + e;  // pair index within the half
+                                const float2 r2 = unpack2<T>(rv[h][j]);
+                                const float f0 = act(__uint_as_float(v[32 * h + 2 * j]) +
+                                                     __shfl_sync(0xffffffffu, bias_r[cj][h], 2 * j) + r2.x);
+                                const float f1 = act(__uint_as_float(v[32 * h + 2 * j + 1]) +
+                                                     __shfl_sync(0xffffffffu, bias_r[cj][h], 2 * j + 1) + r2.y);
+                                wq[e] = pack2<T>(f0, f1);
+                            }
+                            *reinterpret_cast<uint4 *>(buf + lane * 128 + ((q ^ (lane & 7)) << 4)) =
+                                make_uint4(wq[0], wq[1], wq[2], wq[3]);
                         }
-                        *reinterpret_cast<uint4 *>(buf + lane * 128 + ((q ^ (lane & 7)) << 4)) =
-                            make_uint4(wq[0], wq[1], wq[2], wq[3]);
-                    }
+                    };
+                    if (p.act == SN_ACT_RELU)
+                        stage_rows([](float x) { return fmaxf(x, 0.0f); });
+                    else if (p.act == SN_ACT_NONE)
+                        stage_rows([](float x) { return x; });
+                    else
+                        stage_rows([act = p.act](float x) { return act_apply(x, act); });
                     fence_proxy_async_smem();
                     __syncwarp();
                     if (lane == 0) {
