@@ -64,8 +64,18 @@ typedef enum {
 /* Routine schema (section III-C): the platform is always this GPU, so a
  * schema is the pair (data type, layout).  Two adjacent layers whose routines
  * have different schemas are joined by an adapt routine that casts and/or
- * permutes the blob. */
-typedef enum { SN_F32 = 0, SN_F16 = 1, SN_BF16 = 2 } sn_dtype;
+ * permutes the blob.
+ *
+ * SN_QI8 is the quantised schema of section II-C in its symmetric form
+ * (offset 0): a blob holds int8 codes q in [-127, 127] and one fp32 scale s
+ * per blob (set by sn_set_qscale or sn_calibrate), standing for the values
+ * q * s.  Quantising a float blob gives q = clamp(rint(x * (1/s)), -127, 127)
+ * (1/s rounded to fp32; round half to even); dequantising gives the fp32
+ * value q * s.  qint8 routines keep one scale per weight output channel,
+ * s_w[k] = max |W[k, .]| / 127, sum code products exactly and requantise
+ * y = act(float(acc) * (s_x * s_w[k]) + bias[k] (+ residual value)) to the
+ * output blob's scale, every fp32 operation rounded on its own. */
+typedef enum { SN_F32 = 0, SN_F16 = 1, SN_BF16 = 2, SN_QI8 = 3 } sn_dtype;
 typedef enum { SN_NCHW = 0, SN_NHWC = 1 } sn_layout;
 typedef struct { int32_t dtype; int32_t layout; } sn_schema;
 
@@ -260,6 +270,32 @@ SN_API const char *sn_variant_name(int32_t routine, int32_t variant);
  * Errors: SN_EINVAL, SN_ECUDA. */
 SN_API sn_status sn_convert(const void *x_dev, sn_schema from, void *y_dev, sn_schema to,
                      const int64_t nchw[4], void *stream);
+/* sn_convert where either side may be SN_QI8: qscale > 0 is the blob's
+ * scale (quantise: float -> codes; dequantise: codes -> float; codes ->
+ * codes: layout permutation only).  Errors: SN_EINVAL (bad schema, no qint8
+ * side, qscale not finite and positive), SN_ECUDA. */
+SN_API sn_status sn_convert_q(const void *x_dev, sn_schema from, void *y_dev, sn_schema to,
+                              const int64_t nchw[4], float qscale, void *stream);
+
+/* ---------------- qint8 scales (section II-C, hybrid tuning of section V-C)
+ * Every blob that a selected path keeps in SN_QI8 needs a scale: the net
+ * input (layer id -1) and the output of each layer (ids from sn_add_layer).
+ * Profiling does not need them (it times on scratch codes); building the plan
+ * of a path that quantises a blob without a scale fails with SN_ESTATE.
+ * sn_set_qscale: scale finite and > 0.  Invalidates the plan.
+ * sn_get_qscale: *scale = the blob's scale, 0 when none is set.
+ * Errors: SN_EINVAL (bad id or scale). */
+SN_API sn_status sn_set_qscale(sn_graph *g, int32_t layer_id, float scale);
+SN_API sn_status sn_get_qscale(sn_graph *g, int32_t layer_id, float *scale);
+/* Calibration (post-training, symmetric, per tensor): run the net once on
+ * in_dev (in in_schema, caller-owned) along the cheapest path that keeps every
+ * layer in a float schema of Lambda (DPRS over the current cost table with the
+ * qint8 candidates left out), and set the scale of the net input and of every
+ * layer's output to max |x| / 127 of the blob as that path stores it (1 for an
+ * all-zero blob).  The selected path, if any, is kept.  Synchronises stream.
+ * Errors: SN_ESTATE (costs not profiled or set: no finite float path),
+ * SN_EUNSUPPORTED (in_schema or out_schema is SN_QI8), SN_ECUDA, SN_ENOMEM. */
+SN_API sn_status sn_calibrate(sn_graph *g, const void *in_dev, void *stream);
 
 /* ---------------- allocation-free Winograd convolution --------------------
  * The paper has no counterpart to this call; it exists for callers that

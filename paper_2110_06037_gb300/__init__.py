@@ -8,8 +8,8 @@ thin binding over it.
 """
 from ._sn import (SN_SELECT_BRUTE, SN_SELECT_DPRS, SN_OPT_CHECK, SN_OPT_CUDA_GRAPH, SnError, lib,
                   routine_name, variant_name)
-from .api import Graph, convert, storage_shape
+from .api import Graph, convert, convert_q, storage_shape
 from .netbuild import build_graph, fuse_residual
 
-__all__ = ["Graph", "convert", "build_graph", "fuse_residual", "storage_shape", "SnError", "lib", "routine_name",
+__all__ = ["Graph", "convert", "convert_q", "build_graph", "fuse_residual", "storage_shape", "SnError", "lib", "routine_name",
            "variant_name", "SN_SELECT_DPRS", "SN_SELECT_BRUTE", "SN_OPT_CHECK", "SN_OPT_CUDA_GRAPH"]

@@ -17,7 +17,7 @@ LIB_PATH = os.path.join(_HERE, "libsn.so")
 SN_OK, SN_EINVAL, SN_ENOMEM, SN_ECUDA, SN_EUNSUPPORTED, SN_ESTATE, SN_ETIMEOUT, SN_EINFEASIBLE = range(8)
 STATUS_NAMES = ["SN_OK", "SN_EINVAL", "SN_ENOMEM", "SN_ECUDA", "SN_EUNSUPPORTED", "SN_ESTATE",
                 "SN_ETIMEOUT", "SN_EINFEASIBLE"]
-SN_F32, SN_F16, SN_BF16 = 0, 1, 2
+SN_F32, SN_F16, SN_BF16, SN_QI8 = 0, 1, 2, 3
 SN_NCHW, SN_NHWC = 0, 1
 SN_L_CONV2, SN_L_DWCONV2, SN_L_MAXPOOL, SN_L_GAP, SN_L_ADD, SN_L_DENSE, SN_L_MUL = range(7)
 SN_ACT = {"none": 0, None: 0, "relu": 1, "relu6": 2, "hswish": 3, "hsigmoid": 4}
@@ -25,7 +25,7 @@ SN_SELECT_DPRS, SN_SELECT_BRUTE = 0, 1
 SN_OPT_CUDA_GRAPH, SN_OPT_CHECK = 0, 1
 COST_INF = np.iinfo(np.int64).max
 
-DTYPES = {"f32": SN_F32, "f16": SN_F16, "bf16": SN_BF16}
+DTYPES = {"f32": SN_F32, "f16": SN_F16, "bf16": SN_BF16, "qi8": SN_QI8}
 LAYOUTS = {"nchw": SN_NCHW, "nhwc": SN_NHWC}
 
 
@@ -97,6 +97,11 @@ SIGNATURES = {
     "sn_routine_name": (C.c_char_p, [C.c_int32]),
     "sn_variant_name": (C.c_char_p, [C.c_int32, C.c_int32]),
     "sn_convert": (C.c_int, [C.c_void_p, sn_schema, C.c_void_p, sn_schema, C.POINTER(C.c_int64), C.c_void_p]),
+    "sn_convert_q": (C.c_int, [C.c_void_p, sn_schema, C.c_void_p, sn_schema, C.POINTER(C.c_int64), C.c_float,
+                               C.c_void_p]),
+    "sn_set_qscale": (C.c_int, [C.c_void_p, C.c_int32, C.c_float]),
+    "sn_get_qscale": (C.c_int, [C.c_void_p, C.c_int32, C.POINTER(C.c_float)]),
+    "sn_calibrate": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p]),
     "sn_conv2d_wino_noalloc": (C.c_int, [C.c_void_p, sn_schema, C.POINTER(C.c_int64), C.c_int32, C.c_int32,
                                          C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p]),
     "sn_last_error": (C.c_char_p, []),

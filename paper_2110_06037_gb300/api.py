@@ -14,7 +14,7 @@ import numpy as np
 from . import _sn
 from ._sn import check, lib
 
-TORCH_DTYPES = {"f32": "float32", "f16": "float16", "bf16": "bfloat16"}
+TORCH_DTYPES = {"f32": "float32", "f16": "float16", "bf16": "bfloat16", "qi8": "int8"}
 
 
 def _torch():
@@ -187,6 +187,20 @@ class Graph:
     def load_plan(self, path):
         check(lib().sn_load_plan(self.h, str(path).encode()))
 
+    # ------------------------------------------------------ qint8 scales
+    def set_qscale(self, layer_id, scale):
+        """Scale of a blob kept in qi8: layer_id from add_layer, -1 = net input."""
+        check(lib().sn_set_qscale(self.h, int(layer_id), float(scale)))
+
+    def get_qscale(self, layer_id):
+        v = C.c_float(0.0)
+        check(lib().sn_get_qscale(self.h, int(layer_id), C.byref(v)))
+        return v.value
+
+    def calibrate(self, x, stream=None):
+        """Set every blob's qi8 scale from one float-path run on x (max |x| / 127)."""
+        check(lib().sn_calibrate(self.h, C.c_void_p(x.data_ptr()), _stream_ptr(stream)))
+
     # --------------------------------------------------------------- running
     def output_shape(self):
         t = self.cost_table()
@@ -224,4 +238,16 @@ def convert(x, from_schema, to_schema, shape_nchw, out=None, stream=None):
     shp = (C.c_int64 * 4)(*shape_nchw)
     check(lib().sn_convert(C.c_void_p(x.data_ptr()), _sn.schema(from_schema), C.c_void_p(out.data_ptr()),
                            _sn.schema(to_schema), shp, _stream_ptr(stream)))
+    return out
+
+
+def convert_q(x, from_schema, to_schema, shape_nchw, qscale, out=None, stream=None):
+    """The adapt routine with a qi8 side: quantise, dequantise or permute codes."""
+    torch = _torch()
+    if out is None:
+        out = torch.empty(storage_shape(shape_nchw, to_schema[1]),
+                          dtype=getattr(torch, TORCH_DTYPES[to_schema[0]]), device="cuda")
+    shp = (C.c_int64 * 4)(*shape_nchw)
+    check(lib().sn_convert_q(C.c_void_p(x.data_ptr()), _sn.schema(from_schema), C.c_void_p(out.data_ptr()),
+                             _sn.schema(to_schema), shp, C.c_float(qscale), _stream_ptr(stream)))
     return out

@@ -1,6 +1,7 @@
 // extern "C" boundary of the library (declared in include/sn.h).  Every entry
 // point catches C++ exceptions and turns them into a status, so nothing but
 // an sn_status crosses the ABI.
+#include <cmath>
 #include <cstdio>
 #include <cstring>
 #include <fstream>
@@ -531,10 +532,77 @@ sn_status sn_convert(const void *x_dev, sn_schema from, void *y_dev, sn_schema t
         if (!schema_valid(from) || !schema_valid(to)) return fail(SN_EINVAL, "sn_convert: invalid schema");
         for (int k = 0; k < 4; ++k)
             if (nchw[k] < 0) return fail(SN_EINVAL, "sn_convert: negative extent");
+        if (from.dtype == SN_QI8 || to.dtype == SN_QI8)
+            return fail(SN_EINVAL, "sn_convert: a qint8 side needs its scale (sn_convert_q)");
         const Shape s{nchw[0], nchw[1], nchw[2], nchw[3]};
         if (s.numel() == 0) return SN_OK;
         SN_CUDA_TRY(k::convert(x_dev, from.dtype, from.layout, y_dev, to.dtype, to.layout, s,
                                static_cast<cudaStream_t>(stream)));
+        return SN_OK;
+    })
+}
+
+sn_status sn_convert_q(const void *x_dev, sn_schema from, void *y_dev, sn_schema to, const int64_t nchw[4],
+                       float qscale, void *stream) {
+    SN_GUARD({
+        if (!x_dev || !y_dev || !nchw) return fail(SN_EINVAL, "sn_convert_q: NULL argument");
+        if (!schema_valid(from) || !schema_valid(to)) return fail(SN_EINVAL, "sn_convert_q: invalid schema");
+        if (from.dtype != SN_QI8 && to.dtype != SN_QI8) return fail(SN_EINVAL, "sn_convert_q: no qint8 side");
+        if (!(qscale > 0.0f) || !std::isfinite(qscale)) return fail(SN_EINVAL, "sn_convert_q: bad scale");
+        for (int k = 0; k < 4; ++k)
+            if (nchw[k] < 0) return fail(SN_EINVAL, "sn_convert_q: negative extent");
+        const Shape s{nchw[0], nchw[1], nchw[2], nchw[3]};
+        if (s.numel() == 0) return SN_OK;
+        SN_CUDA_TRY(k::convert_q8(x_dev, from.dtype, from.layout, y_dev, to.dtype, to.layout, s, qscale,
+                                  static_cast<cudaStream_t>(stream)));
+        return SN_OK;
+    })
+}
+
+static float *qscale_ref(Graph *g, int32_t id, bool internal) {
+    if (id == -1) return internal ? &g->layers[0].qscale : &g->in_qscale;
+    if (id < 0 || id >= (int32_t)g->user.size()) return nullptr;
+    return internal ? &g->layers[id + 1].qscale : &g->user[id].qscale;
+}
+
+sn_status sn_set_qscale(sn_graph *gg, int32_t layer_id, float scale) {
+    SN_GUARD({
+        if (!gg) return fail(SN_EINVAL, "sn_set_qscale: NULL graph");
+        Graph *g = G(gg);
+        if (!(scale > 0.0f) || !std::isfinite(scale)) return fail(SN_EINVAL, "sn_set_qscale: bad scale");
+        float *u = qscale_ref(g, layer_id, false);
+        if (!u) return fail(SN_EINVAL, "sn_set_qscale: bad layer id");
+        *u = scale;
+        if (g->finalized) *qscale_ref(g, layer_id, true) = scale;
+        invalidate_plan(g);
+        return SN_OK;
+    })
+}
+
+sn_status sn_get_qscale(sn_graph *gg, int32_t layer_id, float *scale) {
+    SN_GUARD({
+        if (!gg || !scale) return fail(SN_EINVAL, "sn_get_qscale: NULL argument");
+        Graph *g = G(gg);
+        const float *u = qscale_ref(g, layer_id, false);
+        if (!u) return fail(SN_EINVAL, "sn_get_qscale: bad layer id");
+        *scale = *u;
+        return SN_OK;
+    })
+}
+
+sn_status sn_calibrate(sn_graph *gg, const void *in_dev, void *stream) {
+    SN_GUARD({
+        if (!gg || !in_dev) return fail(SN_EINVAL, "sn_calibrate: NULL argument");
+        Graph *g = G(gg);
+        sn_status rc = graph_finalize(g);
+        if (rc != SN_OK) return rc;
+        if (g->in_schema.dtype == SN_QI8 || g->out_schema.dtype == SN_QI8)
+            return fail(SN_EUNSUPPORTED, "sn_calibrate: the net input and output must be float");
+        rc = calibrate(g, in_dev, static_cast<cudaStream_t>(stream));
+        if (rc != SN_OK) return rc;
+        // mirror into the layers as added
+        g->in_qscale = g->layers[0].qscale;
+        for (size_t u = 0; u < g->user.size(); ++u) g->user[u].qscale = g->layers[u + 1].qscale;
         return SN_OK;
     })
 }

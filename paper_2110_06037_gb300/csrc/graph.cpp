@@ -18,7 +18,7 @@ sn_status fail(sn_status s, const std::string &msg) {
 const char *last_error() { return g_last_error.c_str(); }
 
 std::string schema_str(sn_schema s) {
-    static const char *dt[] = {"f32", "f16", "bf16"};
+    static const char *dt[] = {"f32", "f16", "bf16", "qi8"};
     static const char *ly[] = {"nchw", "nhwc"};
     if (!schema_valid(s)) return "invalid";
     return std::string(dt[s.dtype]) + "." + ly[s.layout];
@@ -219,6 +219,7 @@ sn_status graph_finalize(Graph *g) {
     Layer in_l;
     in_l.type = -1;
     in_l.out = g->in_shape;
+    in_l.qscale = g->in_qscale;
     L.push_back(in_l);
     for (auto &u : g->user) L.push_back(u);
     Layer out_l;

@@ -217,6 +217,7 @@ static cudaError_t convert_t(const void *x, int lay_in, void *y, int lay_out, Sh
 
 cudaError_t convert(const void *x, int dt_in, int lay_in, void *y, int dt_out, int lay_out, Shape s,
                     cudaStream_t st) {
+    if (dt_in == SN_QI8 || dt_out == SN_QI8) return cudaErrorInvalidValue;  // needs a scale: convert_q8
     SN_DT_SWITCH(dt_in, Ti, SN_DT_SWITCH(dt_out, To, return convert_t<Ti, To>(x, lay_in, y, lay_out, s, st)));
     return cudaErrorInvalidValue;
 }
@@ -241,6 +242,7 @@ __global__ void fill_kernel(T *y, int64_t n, uint32_t seed, float scale) {
 
 cudaError_t fill_pattern(void *y, int dt, int64_t n, uint32_t seed, float scale, cudaStream_t st) {
     if (n == 0) return cudaSuccess;
+    if (dt == SN_QI8) return fill_q8(y, n, seed, st);
     SN_DT_SWITCH(dt, T, launch_pdl(fill_kernel<T>, grid_for(n, 256), 256, 0, st, (T *)y, n, seed, scale));
     return cudaGetLastError();
 }
@@ -328,6 +330,7 @@ __global__ void weight_wino4_kernel(const float *__restrict__ w, float *__restri
 
 cudaError_t weight_format(const float *w, void *out, int fmt, int dt, int64_t K, int64_t Cg,
                           int64_t R, int64_t S, cudaStream_t st) {
+    if (dt == SN_QI8) return cudaErrorInvalidValue;  // codes and scales: weight_format_q8
     if (fmt == W_WINO4) {  // fp32 whatever the schema's dtype
         if (R != 3 || S != 3) return cudaErrorInvalidValue;
         launch_pdl(weight_wino4_kernel, grid_for(K * Cg, 256), 256, 0, st, w, (float *)out, K, Cg);

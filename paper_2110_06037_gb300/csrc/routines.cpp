@@ -28,6 +28,7 @@ const char *routine_name(int32_t r) {
     case R_CONV_IM2COL_TC: return "conv2/im2col_tc";
     case R_DENSE_TC: return "dense/gemm_tc";
     case R_CONV_S2D_TC: return "conv2/s2d_tc";
+    case R_CONV_DP4A: return "conv2/igemm_dp4a";
     default: return nullptr;
     }
 }
@@ -47,7 +48,24 @@ const char *variant_name(int32_t r, int32_t v) {
 
 static bool is_conv(const Layer &l) { return l.type == SN_L_CONV2; }
 
+// qint8 schema: the routines that have an int8 kernel (one variant each)
+static int32_t q8_variants(int32_t r, const Layer &l, const std::vector<Shape> &in, sn_schema s) {
+    switch (r) {
+    case R_CONV_DIRECT: return is_conv(l) ? 1 : 0;
+    case R_CONV_DP4A: return k::q8_conv_dp4a_applies(l, in[0], s) ? 1 : 0;
+    case R_DW_DIRECT: return l.type == SN_L_DWCONV2 ? 1 : 0;
+    case R_MAXPOOL: return l.type == SN_L_MAXPOOL ? 1 : 0;
+    case R_GAP: return l.type == SN_L_GAP ? 1 : 0;
+    case R_ADD: return l.type == SN_L_ADD ? 1 : 0;
+    case R_MUL: return l.type == SN_L_MUL ? 1 : 0;
+    case R_DENSE: return (l.type == SN_L_DENSE && in[0].h == 1 && in[0].w == 1) ? 1 : 0;
+    default: return 0;
+    }
+}
+
 int32_t routine_variants(int32_t r, const Layer &l, const std::vector<Shape> &in, sn_schema s) {
+    if (s.dtype == SN_QI8) return q8_variants(r, l, in, s);
+    if (r == R_CONV_DP4A) return 0;
     const sn_conv_params &p = l.conv;
     // a conv2 with a residual input is served by the routines whose epilogue
     // adds it: direct and the tensor-core implicit GEMM
@@ -101,6 +119,15 @@ size_t routine_workspace(int32_t r, int32_t v, const Layer &l, const std::vector
 
 // weight format of (routine, layout)
 static int weight_format_of(int32_t r, sn_schema s) {
+    if (s.dtype == SN_QI8) {
+        switch (r) {
+        case R_CONV_DIRECT:
+        case R_DW_DIRECT: return s.layout == SN_NCHW ? k::W_KCRS : k::W_RSCK;
+        case R_CONV_DP4A: return k::W_KRSC;
+        case R_DENSE: return k::W_KCRS;
+        default: return -1;
+        }
+    }
     switch (r) {
     case R_CONV_DIRECT: return s.layout == SN_NCHW ? k::W_KCRS : k::W_RSCK;
     case R_CONV_IGEMM: return s.layout == SN_NCHW ? k::W_KCRS : k::W_KRSC;
@@ -161,7 +188,9 @@ sn_status prepare_weights(Graph *g, int32_t li, int32_t r, int32_t v, sn_schema 
     Buffer src, dst;
     sn_status rc = dev_alloc(g, (size_t)K * Cg * R * S * sizeof(float), &src);
     if (rc != SN_OK) return rc;
-    rc = dev_alloc(g, (size_t)elems * (fmt == k::W_WINO4 ? sizeof(float) : dtype_size(s.dtype)), &dst);
+    const size_t dst_bytes = s.dtype == SN_QI8 ? k::q8_weight_bytes(K, elems)  // codes + per-channel scales
+                             : (size_t)elems * (fmt == k::W_WINO4 ? sizeof(float) : dtype_size(s.dtype));
+    rc = dev_alloc(g, dst_bytes, &dst);
     if (rc != SN_OK) {
         dev_free(g, &src);
         return rc;
@@ -169,7 +198,9 @@ sn_status prepare_weights(Graph *g, int32_t li, int32_t r, int32_t v, sn_schema 
     cudaError_t e = cudaMemcpyAsync(src.ptr, L.weight.data(), L.weight.size() * sizeof(float),
                                     cudaMemcpyHostToDevice, st);
     if (e == cudaSuccess)
-        e = k::weight_format(static_cast<const float *>(src.ptr), dst.ptr, fmt, s.dtype, K, Cg, R, S, st);
+        e = s.dtype == SN_QI8
+                ? k::weight_format_q8(static_cast<const float *>(src.ptr), dst.ptr, fmt, K, Cg, R, S, st)
+                : k::weight_format(static_cast<const float *>(src.ptr), dst.ptr, fmt, s.dtype, K, Cg, R, S, st);
     if (e == cudaSuccess) e = cudaStreamSynchronize(st);  // src is freed next
     dev_free(g, &src);
     if (e != cudaSuccess) {
@@ -182,6 +213,7 @@ sn_status prepare_weights(Graph *g, int32_t li, int32_t r, int32_t v, sn_schema 
 }
 
 int32_t kernels_per_launch(int32_t r, int32_t v, const Layer &l, const std::vector<Shape> &in, sn_schema s) {
+    if (s.dtype == SN_QI8) return 1;
     // a K-split tensor-core GEMM adds its reduction kernel (it is the only
     // variant with a workspace)
     const int split = (r == R_CONV_TC || r == R_CONV_IM2COL_TC || r == R_DENSE_TC || r == R_CONV_S2D_TC) &&
@@ -194,8 +226,28 @@ int32_t kernels_per_launch(int32_t r, int32_t v, const Layer &l, const std::vect
     return 1 + split;
 }
 
+static cudaError_t launch_q8(const LaunchArgs &a) {
+    switch (a.routine) {
+    case R_CONV_DIRECT:
+    case R_DW_DIRECT: return k::q8_conv_direct(a);
+    case R_CONV_DP4A: return k::q8_conv_dp4a(a);
+    case R_MAXPOOL: return k::q8_maxpool(a);
+    case R_GAP: return k::q8_gap(a);
+    case R_ADD: return k::q8_add(a);
+    case R_MUL: return k::q8_mul(a);
+    case R_DENSE: return k::q8_dense(a);
+    default: return cudaErrorInvalidValue;
+    }
+}
+
 sn_status launch_routine(const LaunchArgs &a) {
     cudaError_t e = cudaSuccess;
+    if (a.schema.dtype == SN_QI8) {
+        e = launch_q8(a);
+        if (e != cudaSuccess)
+            return fail(SN_ECUDA, std::string(routine_name(a.routine)) + " (qi8): " + cudaGetErrorString(e));
+        return SN_OK;
+    }
     switch (a.routine) {
     case R_CONV_DIRECT: e = k::conv_direct(a); break;
     case R_CONV_IGEMM: e = k::conv_igemm(a); break;

@@ -19,12 +19,24 @@
 
 namespace sn {
 
-static sn_status schema_slot(Graph *g, Shape s, sn_schema sc) {
+static sn_status schema_slot(Graph *g, Shape s, sn_schema sc, float qscale) {
     g->slots.push_back({});
     g->slot_shape.push_back(s);
     g->slot_schema.push_back(sc);
+    g->slot_qscale.push_back(qscale);
     return SN_OK;
 }
+
+// an adapt between two schemas; a qint8 side uses the blob's scale
+static cudaError_t convert_blob(const void *x, sn_schema a, void *y, sn_schema b, Shape s, float qscale,
+                                cudaStream_t st) {
+    if (a.dtype == SN_QI8 || b.dtype == SN_QI8)
+        return k::convert_q8(x, a.dtype, a.layout, y, b.dtype, b.layout, s, qscale, st);
+    return k::convert(x, a.dtype, a.layout, y, b.dtype, b.layout, s, st);
+}
+
+// stand-in scale of qint8 blobs while profiling (timing does not depend on it)
+constexpr float kProfileQScale = 1.0f / 64.0f;
 
 sn_status build_plan(Graph *g, cudaStream_t st) {
     if (!g->has_path) return fail(SN_ESTATE, "no routine path selected");
@@ -33,11 +45,13 @@ sn_status build_plan(Graph *g, cudaStream_t st) {
     g->slots.clear();
     g->slot_shape.clear();
     g->slot_schema.clear();
+    g->slot_qscale.clear();
     const int32_t n = g->n_layers();
     std::vector<sn_schema> sch(n);
     for (int32_t i = 0; i < n; ++i) sch[i] = g->schemas[g->cands[g->path_cand[i]].schema];
-    schema_slot(g, g->in_shape, g->in_schema);              // slot 0: caller's input
-    schema_slot(g, g->layers[n - 1].out, g->out_schema);    // slot 1: caller's output
+    schema_slot(g, g->in_shape, g->in_schema, g->layers[0].qscale);  // slot 0: caller's input
+    schema_slot(g, g->layers[n - 1].out, g->out_schema,
+                g->layers[g->layers[n - 1].inputs[0]].qscale);         // slot 1: caller's output
     std::vector<int32_t> out_slot(n, -1);
     out_slot[0] = 0;
     const int32_t last = n - 2;  // last user layer (0 if none)
@@ -80,7 +94,7 @@ sn_status build_plan(Graph *g, cudaStream_t st) {
                 continue;
             }
             if (!same) {
-                schema_slot(g, g->layers[j].out, sch[i]);
+                schema_slot(g, g->layers[j].out, sch[i], g->layers[j].qscale);
                 PlanOp a;
                 a.kind = PlanOp::ADAPT;
                 a.layer = i;
@@ -96,7 +110,7 @@ sn_status build_plan(Graph *g, cudaStream_t st) {
         if (i == last && schema_eq(sch[i], g->out_schema)) {
             op.out_slot = 1;
         } else {
-            schema_slot(g, L.out, sch[i]);
+            schema_slot(g, L.out, sch[i], L.qscale);
             op.out_slot = (int32_t)g->slots.size() - 1;
         }
         out_slot[i] = op.out_slot;
@@ -107,6 +121,15 @@ sn_status build_plan(Graph *g, cudaStream_t st) {
         sn_status rc = prepare_weights(g, i, c.routine, c.variant, sch[i], &op.wt, &op.bias, st);
         if (rc != SN_OK) return rc;
         g->plan.push_back(op);
+    }
+    // every blob the path keeps in qint8 needs its scale
+    for (size_t s = 0; s < g->slots.size(); ++s) {
+        if (g->slot_qscale[s] > 0.0f) continue;
+        if (g->profiling) {
+            g->slot_qscale[s] = kProfileQScale;  // both sides of a timed adapt
+        } else if (g->slot_schema[s].dtype == SN_QI8) {
+            return fail(SN_ESTATE, "the path keeps a blob in qi8 without a scale (sn_set_qscale or sn_calibrate)");
+        }
     }
     for (size_t s = 2; s < g->slots.size(); ++s) {
         const size_t bytes = (size_t)g->slot_shape[s].numel() * dtype_size(g->slot_schema[s].dtype);
@@ -132,8 +155,8 @@ static sn_status launch_op(Graph *g, const PlanOp &op, const void *in, void *out
     if (op.kind == PlanOp::ADAPT) {
         const int32_t si = op.in_slots[0], so = op.out_slot;
         const sn_schema a = g->slot_schema[si], b = g->slot_schema[so];
-        cudaError_t e = k::convert(ptr(si), a.dtype, a.layout, ptr(so), b.dtype, b.layout,
-                                   g->slot_shape[si], st);
+        const float qs = a.dtype == SN_QI8 ? g->slot_qscale[si] : g->slot_qscale[so];  // the qi8 side's
+        cudaError_t e = convert_blob(ptr(si), a, ptr(so), b, g->slot_shape[si], qs, st);
         if (e != cudaSuccess) return fail(SN_ECUDA, std::string("adapt: ") + cudaGetErrorString(e));
         return SN_OK;
     }
@@ -148,8 +171,10 @@ static sn_status launch_op(Graph *g, const PlanOp &op, const void *in, void *out
     for (size_t k = 0; k < op.in_slots.size(); ++k) {
         a.in[k] = ptr(op.in_slots[k]);
         a.in_shapes.push_back(g->layers[L.inputs[k]].out);
+        a.qs_in[k] = g->slot_qscale[op.in_slots[k]];
     }
     a.out = ptr(op.out_slot);
+    a.qs_out = g->slot_qscale[op.out_slot];
     a.wt = op.wt;
     a.bias = op.bias;
     a.ws = g->workspace.ptr;
@@ -305,7 +330,9 @@ sn_status profile_graph(Graph *g, const sn_profile_opts &o, cudaStream_t user) {
     SN_CUDA_TRY(cudaStreamSynchronize(user));
     cudaStream_t st = nullptr;
     SN_CUDA_TRY(cudaStreamCreateWithFlags(&st, cudaStreamNonBlocking));
+    g->profiling = true;
     const sn_status rc = profile_graph_on(g, o, st);
+    g->profiling = false;
     const cudaError_t e = cudaStreamSynchronize(st);
     cudaStreamDestroy(st);
     if (rc == SN_OK && e != cudaSuccess) return fail(SN_ECUDA, std::string("profiling: ") + cudaGetErrorString(e));
@@ -357,6 +384,7 @@ static sn_status profile_graph_on(Graph *g, const sn_profile_opts &o, cudaStream
             a.in[1] = in.size() > 1 ? sc.in1.ptr : nullptr;  // a residual only where the layer has one
             a.out = sc.out.ptr;
             a.stream = st;
+            a.qs_in[0] = a.qs_in[1] = a.qs_out = kProfileQScale;
             if (k::fill_pattern(sc.in0.ptr, s.dtype, in[0].numel(), 1234u + i, 1.0f, st) != cudaSuccess ||
                 (in.size() > 1 &&
                  k::fill_pattern(sc.in1.ptr, s.dtype, in[1].numel(), 99u + i, 1.0f, st) != cudaSuccess)) {
@@ -410,8 +438,7 @@ static sn_status profile_graph_on(Graph *g, const sn_profile_opts &o, cudaStream
                 }
                 int64_t t = kInf;
                 rc = time_median(o.warmup, o.iters, st, [&]() -> sn_status {
-                    cudaError_t ce = k::convert(sc.in0.ptr, A.dtype, A.layout, sc.out.ptr, B.dtype,
-                                                B.layout, s, st);
+                    cudaError_t ce = convert_blob(sc.in0.ptr, A, sc.out.ptr, B, s, kProfileQScale, st);
                     return ce == cudaSuccess ? SN_OK : fail(SN_ECUDA, cudaGetErrorString(ce));
                 }, &t);
                 if (rc != SN_OK) break;
@@ -535,6 +562,71 @@ static sn_status profile_graph_on(Graph *g, const sn_profile_opts &o, cudaStream
     g->path_total = saved_total;
     invalidate_plan(g);
     return rc;
+}
+
+// ---------------------------------------------------------------------------
+// qint8 calibration (post-training, symmetric, one scale per blob)
+// ---------------------------------------------------------------------------
+sn_status calibrate(Graph *g, const void *in, cudaStream_t st) {
+    const int32_t n = g->n_layers(), ns = g->n_schemas();
+    // the cheapest float path: DPRS over the current costs without the qint8
+    // candidates
+    const std::vector<Candidate> saved_costs = g->cands;
+    for (auto &c : g->cands)
+        if (g->schemas[c.schema].dtype == SN_QI8) c.cost = kInf;
+    std::vector<int32_t> schema_of;
+    int64_t total = kInf;
+    sn_status rc = select_dprs(*g, schema_of, total);
+    std::vector<int64_t> F;
+    std::vector<int32_t> argF;
+    if (rc == SN_OK) fastest_per_schema(*g, F, argF);
+    g->cands = saved_costs;
+    if (rc != SN_OK || total == kInf)
+        return fail(SN_ESTATE, "sn_calibrate: no float path of finite cost (profile or set the costs first)");
+    std::vector<int32_t> pc(n);
+    for (int32_t i = 0; i < n; ++i) pc[i] = argF[(size_t)i * ns + schema_of[i]];
+
+    const bool had_path = g->has_path;
+    const std::vector<int32_t> saved_path = g->path_cand;
+    const int64_t saved_total = g->path_total;
+    g->path_cand = pc;
+    g->has_path = true;
+    Buffer out, dmax;
+    auto finish = [&](sn_status r) {
+        dev_free(g, &out);
+        dev_free(g, &dmax);
+        g->has_path = had_path;
+        g->path_cand = saved_path;
+        g->path_total = saved_total;
+        invalidate_plan(g);
+        return r;
+    };
+    if ((rc = build_plan(g, st)) != SN_OK) return finish(rc);
+    if ((rc = dev_alloc(g, (size_t)g->layers[n - 1].out.numel() * dtype_size(g->out_schema.dtype), &out)) != SN_OK)
+        return finish(rc);
+    if ((rc = dev_alloc(g, (size_t)n * sizeof(unsigned), &dmax)) != SN_OK) return finish(rc);
+    unsigned *dm = static_cast<unsigned *>(dmax.ptr);
+    if (cudaMemsetAsync(dm, 0, (size_t)n * sizeof(unsigned), st) != cudaSuccess ||
+        k::absmax(in, g->in_schema.dtype, g->in_shape.numel(), dm, st) != cudaSuccess)
+        return finish(fail(SN_ECUDA, "sn_calibrate: input reduction failed"));
+    for (const PlanOp &op : g->plan) {
+        if ((rc = launch_op(g, op, in, out.ptr, st)) != SN_OK) return finish(rc);
+        if (op.kind != PlanOp::LAYER) continue;
+        const int32_t so = op.out_slot;
+        const void *y = so == 1 ? out.ptr : g->slots[so].ptr;
+        if (k::absmax(y, g->slot_schema[so].dtype, g->slot_shape[so].numel(), dm + op.layer, st) != cudaSuccess)
+            return finish(fail(SN_ECUDA, "sn_calibrate: reduction failed"));
+    }
+    std::vector<unsigned> hm(n);
+    if (cudaMemcpyAsync(hm.data(), dm, (size_t)n * sizeof(unsigned), cudaMemcpyDeviceToHost, st) != cudaSuccess ||
+        cudaStreamSynchronize(st) != cudaSuccess)
+        return finish(fail(SN_ECUDA, "sn_calibrate: read-back failed"));
+    for (int32_t i = 0; i < n - 1; ++i) {
+        float m;
+        std::memcpy(&m, &hm[i], sizeof(float));
+        g->layers[i].qscale = m > 0.0f ? m / 127.0f : 1.0f;
+    }
+    return finish(SN_OK);
 }
 
 }  // namespace sn

@@ -42,10 +42,10 @@ struct Shape {
     bool operator==(const Shape &o) const { return n == o.n && c == o.c && h == o.h && w == o.w; }
 };
 
-inline int dtype_size(int dt) { return dt == SN_F32 ? 4 : 2; }
+inline int dtype_size(int dt) { return dt == SN_F32 ? 4 : dt == SN_QI8 ? 1 : 2; }
 inline bool schema_eq(sn_schema a, sn_schema b) { return a.dtype == b.dtype && a.layout == b.layout; }
 inline bool schema_valid(sn_schema s) {
-    return s.dtype >= SN_F32 && s.dtype <= SN_BF16 && s.layout >= SN_NCHW && s.layout <= SN_NHWC;
+    return s.dtype >= SN_F32 && s.dtype <= SN_QI8 && s.layout >= SN_NCHW && s.layout <= SN_NHWC;
 }
 std::string schema_str(sn_schema s);
 
@@ -69,7 +69,8 @@ enum RoutineId : int32_t {
     R_CONV_S2D_TC = 13,  // childnet: space-to-depth -> stride-1 tensor-core conv (stride 2, <= 4 channels)
     R_MUL = 14,          // per-channel scale (squeeze-and-excite)
     R_CONV_WINO4 = 15,   // Winograd F(4x4,3x3) childnet (fp32 transformed filters)
-    R_COUNT = 16
+    R_CONV_DP4A = 16,    // qint8 implicit GEMM with dp4a (NHWC)
+    R_COUNT = 17
 };
 
 // -------------------------------------------------------------------------
@@ -84,6 +85,7 @@ struct Layer {
     std::vector<int32_t> inputs;  // internal layer indices
     Shape out;
     std::vector<float> weight, bias;  // host fp32 copies
+    float qscale = 0.0f;              // qint8 scale of the output blob (0 = not set)
 };
 
 struct Candidate {
@@ -130,6 +132,9 @@ struct LaunchArgs {
     // tensor-core implicit GEMM only: > 0 when the layer's "channels" are
     // a_blocks blocks of 64 read as one box (the space-to-depth stem's taps)
     int32_t a_blocks = 0;
+    // qint8 routines: scales of the input blobs and of the output blob
+    float qs_in[2] = {0.0f, 0.0f};
+    float qs_out = 0.0f;
     cudaStream_t stream = nullptr;
 };
 
@@ -143,6 +148,7 @@ struct Graph {
     sn_free_fn free_fn = nullptr;
     void *alloc_ctx = nullptr;
 
+    float in_qscale = 0.0f;           // qint8 scale of the net input (0 = not set)
     std::vector<Layer> user;          // as added
     bool finalized = false;
     std::vector<Layer> layers;        // internal: [input, user..., output]
@@ -161,10 +167,12 @@ struct Graph {
     std::vector<Buffer> slots;        // activation buffers; slot 0 = in, 1 = out (external)
     std::vector<Shape> slot_shape;
     std::vector<sn_schema> slot_schema;
+    std::vector<float> slot_qscale;   // qint8 scale of the blob a slot holds
     std::map<std::string, Buffer> weight_cache;  // key: layer/format/dtype
     std::map<int32_t, Buffer> bias_cache;        // per layer fp32 bias
     Buffer workspace;
     int opt_graph = 0, opt_check = 0;
+    bool profiling = false;           // plans built while profiling may lack qint8 scales
     cudaGraphExec_t gexec = nullptr;
     const void *gexec_in = nullptr;
     void *gexec_out = nullptr;
@@ -213,6 +221,9 @@ sn_status run_plan(Graph *g, const void *in, void *out, cudaStream_t st,
 // every op (device time of each op, no host launch cost); op_ms[q] in ms
 sn_status run_plan_timed(Graph *g, const void *in, void *out, cudaStream_t st, std::vector<float> *op_ms);
 sn_status profile_graph(Graph *g, const sn_profile_opts &o, cudaStream_t st);
+// qint8 calibration: run the fastest float-schema path, set every blob's scale
+// to max |x| / 127
+sn_status calibrate(Graph *g, const void *in, cudaStream_t st);
 
 // -------------------------------------------------------------------------
 // kernels (launchers; all asynchronous on `st`)
@@ -255,6 +266,23 @@ cudaError_t add(const LaunchArgs &a);
 cudaError_t mul(const LaunchArgs &a);
 cudaError_t dense(const LaunchArgs &a);
 int *device_error_word();  // device address of the library's error word
+// qint8 schema (symmetric codes, one scale per blob, per-channel weight scales)
+cudaError_t convert_q8(const void *x, int dt_in, int lay_in, void *y, int dt_out, int lay_out, Shape s,
+                       float qscale, cudaStream_t st);
+cudaError_t fill_q8(void *y, int64_t n, uint32_t seed, cudaStream_t st);
+size_t q8_weight_bytes(int64_t K, int64_t elems);  // codes, then fp32 scales [K]
+cudaError_t weight_format_q8(const float *w_kcrs, void *out, int fmt, int64_t K, int64_t Cg, int64_t R,
+                             int64_t S, cudaStream_t st);
+cudaError_t q8_conv_direct(const LaunchArgs &a);
+bool q8_conv_dp4a_applies(const Layer &l, const Shape &in, sn_schema s);
+cudaError_t q8_conv_dp4a(const LaunchArgs &a);
+cudaError_t q8_dense(const LaunchArgs &a);
+cudaError_t q8_maxpool(const LaunchArgs &a);
+cudaError_t q8_gap(const LaunchArgs &a);
+cudaError_t q8_add(const LaunchArgs &a);
+cudaError_t q8_mul(const LaunchArgs &a);
+// running max |x| of a float blob into *out (fp32 bits; zero it first)
+cudaError_t absmax(const void *x, int dt, int64_t n, unsigned *out, cudaStream_t st);
 }  // namespace k
 
 }  // namespace sn

@@ -123,3 +123,45 @@ def test_tc_not_offered_where_it_cannot_run():
                         torch_alloc=False)
         t = g.cost_table()
         assert not any(_sn.routine_name(int(r)) == "conv2/igemm_tc" for r in t["routine"])
+
+
+def test_qint8_candidates_and_scales():
+    """The qint8 schema offers exactly the routines with an int8 kernel, and
+    blob scales are validated and kept across finalisation."""
+    x, layers = synth.tiny_cnn()
+    g = build_graph(layers, x.shape, ("f32", "nchw"), ("f32", "nchw"), [("f32", "nhwc"), ("qi8", "nhwc")],
+                    torch_alloc=False)
+    g.set_qscale(-1, 0.5)
+    t = g.cost_table()  # finalises
+    q8_names = {_sn.routine_name(int(t["routine"][c])) for c in range(len(t["cost"]))
+                if t["schema"][c] == 1}
+    assert q8_names <= {"io", "conv2/direct", "conv2/igemm_dp4a", "dwconv2/direct", "maxpool/direct", "gap/reduce",
+                        "add/eltwise", "mul/eltwise", "dense/simt"}
+    assert "conv2/direct" in q8_names
+    f_names = {_sn.routine_name(int(t["routine"][c])) for c in range(len(t["cost"])) if t["schema"][c] == 0}
+    assert "conv2/igemm_dp4a" not in f_names
+    assert g.get_qscale(-1) == 0.5 and g.get_qscale(0) == 0.0
+    g.set_qscale(2, 0.125)
+    assert g.get_qscale(2) == 0.125
+    for bad in (0.0, -1.0, float("inf"), float("nan")):
+        with pytest.raises(SnError) as e:
+            g.set_qscale(0, bad)
+        assert e.value.status == _sn.SN_EINVAL
+    with pytest.raises(SnError):
+        g.set_qscale(len(layers), 1.0)
+    with pytest.raises(SnError):
+        g.get_qscale(-2)
+
+
+def test_convert_needs_a_scale_for_qint8():
+    import ctypes as C
+    shp = (C.c_int64 * 4)(1, 2, 3, 4)
+    fake = C.c_void_p(256)  # validation fails before any device access
+    st = _sn.lib().sn_convert(fake, _sn.schema(("f16", "nchw")), fake, _sn.schema(("qi8", "nchw")), shp, None)
+    assert st == _sn.SN_EINVAL
+    st = _sn.lib().sn_convert_q(fake, _sn.schema(("f16", "nchw")), fake, _sn.schema(("f16", "nhwc")), shp,
+                                C.c_float(1.0), None)
+    assert st == _sn.SN_EINVAL  # no qint8 side
+    st = _sn.lib().sn_convert_q(fake, _sn.schema(("f16", "nchw")), fake, _sn.schema(("qi8", "nchw")), shp,
+                                C.c_float(0.0), None)
+    assert st == _sn.SN_EINVAL  # bad scale
