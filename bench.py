@@ -245,7 +245,7 @@ def main():
     ap.add_argument("--no-b1", action="store_true")
     ap.add_argument("--config", default="r50_b32",
                     choices=["r50_b32", "bandwidth", "sweep", "mbv2_b1", "r50_b1", "tiny", "layer", "vgg16_b32",
-                             "vgg16_b1", "mbv3_b1"],
+                             "vgg16_b1", "mbv3_b1", "hybrid"],
                     help="r50_b32 is the benchmark line; the others print one extra JSON line each")
     ap.add_argument("--layer", default="32,512,56,512,3,1",
                     help="--config layer: N,C,H,K,k,s of one bf16 NHWC conv (C -> K channels, HxH input)")
@@ -256,6 +256,8 @@ def main():
     ws, rank, local = dist_env()
     if args.impl == "reference":
         return run_reference(args, ws, rank)
+    if args.config == "hybrid":
+        return run_hybrid(args)
     if args.config != "r50_b32":
         return run_extra_config(args)
 
@@ -522,6 +524,97 @@ def _forced(sn, g, routine, variant=0):
     c = [i for i in range(len(t["cost"])) if t["layer"][i] == 1 and sn.routine_name(int(t["routine"][i])) == routine
          and t["variant"][i] == variant][0]
     g.set_path([int(_np.flatnonzero(t["layer"] == 0)[0]), c, int(_np.flatnonzero(t["layer"] == 2)[0])])
+
+
+def _latency_ms(torch, g, xd, y, stream, flush, reps=20):
+    """Median CUDA-event latency of one CUDA-graph replay of the net, L2 flushed before each."""
+    with torch.cuda.stream(stream):
+        for _ in range(3):
+            g.run(xd, y)
+    stream.synchronize()
+    lat = []
+    for _ in range(reps):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(stream):
+            flush.zero_()
+            a.record(stream)
+            g.run(xd, y)
+            b.record(stream)
+        stream.synchronize()
+        lat.append(a.elapsed_time(b))
+    return statistics.median(lat)
+
+
+def run_hybrid(args):
+    """Hybrid float/qint8 tuning (section V-C, Table I) on the paper's four nets
+    at batch 1: (1) no tuning: every layer's first routine in fp16 NCHW;
+    (2) tuning over the fp16 schemas; (3) over the qint8 schemas; (4) over both
+    (hybrid).  Scales come from calibration on the synthetic input."""
+    import torch
+    import synth
+    import paper_2110_06037_gb300 as sn
+    torch.cuda.set_device(0)
+    F16 = [("f16", "nchw"), ("f16", "nhwc")]
+    Q8 = [("qi8", "nchw"), ("qi8", "nhwc")]
+    io = ("f16", "nchw")
+    stream = torch.cuda.Stream()
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
+    nets = {"vgg16": lambda: synth.vgg16(1), "resnet50": lambda: synth.resnet50(1),
+            "mobilenet_v2": lambda: synth.mobilenet_v2(1), "mobilenet_v3": lambda: synth.mobilenet_v3(1)}
+    rows = {}
+    for name, make in nets.items():
+        x, layers = make()
+        if name != "vgg16":
+            layers = sn.fuse_residual(layers)
+        xd = torch.from_numpy(x).to(torch.float16).cuda()
+        row = {}
+        outs = {}
+
+        def tuned(schemas, scales_from=None):
+            with torch.cuda.stream(stream):
+                g = sn.build_graph(layers, x.shape, io, io, schemas)
+                if scales_from is not None:
+                    for i in range(-1, len(layers)):
+                        g.set_qscale(i, scales_from.get_qscale(i))
+                g.profile(warmup=2, iters=5, topk=1, passes=2)
+                if scales_from is None and any(d == "qi8" for d, _ in schemas):
+                    g.calibrate(xd)
+                total, sch, cands = g.select_path(sn.SN_SELECT_DPRS)
+            stream.synchronize()
+            g.set_option(sn.SN_OPT_CUDA_GRAPH, 1)
+            return g, total, sch, cands
+
+        # (1) no tuning
+        g0 = sn.build_graph(layers, x.shape, io, io, [F16[0]])
+        t = g0.cost_table()
+        g0.set_path([int(np.flatnonzero(t["layer"] == i)[0]) for i in range(t["n_layers"])])
+        g0.set_option(sn.SN_OPT_CUDA_GRAPH, 1)
+        y = g0.new_output()
+        row["untuned_ms"] = _latency_ms(torch, g0, xd, y, stream, flush, reps=5)
+        del g0
+        # (4) hybrid first: its calibration gives the scales for (3)
+        gh, th, sch_h, cand_h = tuned(F16 + Q8)
+        gf, tf, _, _ = tuned(F16)
+        gq, tq, _, _ = tuned(Q8, scales_from=gh)
+        for key, g in (("float_ms", gf), ("qint8_ms", gq), ("hybrid_ms", gh)):
+            y = g.new_output()
+            row[key] = _latency_ms(torch, g, xd, y, stream, flush)
+            outs[key] = y.float().cpu().numpy().ravel()
+        uni = gh.schema_universe()
+        t = gh.cost_table()
+        row["qint8_layers"] = [[i - 1, layers[i - 1]["type"], sn.routine_name(int(t["routine"][int(cand_h[i])]))]
+                               for i in range(1, t["n_layers"] - 1) if uni[int(sch_h[i])][0] == "qi8"]
+        row["path_cost_ns"] = {"float": int(tf), "qint8": int(tq), "hybrid": int(th)}
+        ref = outs["float_ms"]
+        den = max(float(np.abs(ref).max()), 1e-30)
+        row["out_maxrel_vs_float"] = {k: float(np.abs(outs[k] - ref).max()) / den for k in ("qint8_ms", "hybrid_ms")}
+        row["hybrid_vs_float"] = row["float_ms"] / row["hybrid_ms"]
+        rows[name] = row
+        del gh, gf, gq
+        torch.cuda.empty_cache()
+    print(json.dumps({"config": "hybrid", "metric": "batch-1 latency (ms) by tuning case, CUDA-graph replay, "
+                      "L2 flushed: untuned / fp16-tuned / qint8-tuned / hybrid (section V-C, Table I)",
+                      "data": "synthetic inputs and random weights", "nets": rows}))
 
 
 def run_extra_config(args):
