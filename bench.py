@@ -245,7 +245,7 @@ def main():
     ap.add_argument("--no-b1", action="store_true")
     ap.add_argument("--config", default="r50_b32",
                     choices=["r50_b32", "bandwidth", "sweep", "mbv2_b1", "r50_b1", "tiny", "layer", "vgg16_b32",
-                             "vgg16_b1", "mbv3_b1", "hybrid"],
+                             "vgg16_b1", "mbv3_b1", "hybrid", "q8_dense"],
                     help="r50_b32 is the benchmark line; the others print one extra JSON line each")
     ap.add_argument("--layer", default="32,512,56,512,3,1",
                     help="--config layer: N,C,H,K,k,s of one bf16 NHWC conv (C -> K channels, HxH input)")
@@ -663,7 +663,59 @@ def run_extra_config(args):
                 by = x.numel() * x.element_size() + y.numel() * y.element_size()
                 rows.append({"kernel": "adapt/convert", "from": "%s.%s" % a_, "to": "%s.%s" % b_, "shape": list(shp),
                              "us": ms * 1e3, "gbs": by / ms / 1e6, "frac": by / ms / 1e6 / hbm})
+        # qint8 schema: the quantise / dequantise adapts on ResNet-50 b32 activations
+        # and the int8 dense routine at batch 1 (VGG16's fully connected shapes),
+        # where the weight codes are the bytes that matter
+        for shp in [(32, 256, 56, 56), (32, 1024, 14, 14)]:
+            for (a_, b_) in [(("f16", "nchw"), ("qi8", "nhwc")), (("f16", "nhwc"), ("qi8", "nhwc")),
+                             (("qi8", "nhwc"), ("f16", "nhwc"))]:
+                dt = {"f16": torch.float16, "qi8": torch.int8}
+                x = torch.zeros(sn.storage_shape(shp, a_[1]), dtype=dt[a_[0]], device="cuda")
+                y = torch.empty(sn.storage_shape(shp, b_[1]), dtype=dt[b_[0]], device="cuda")
+                bufs = [(x, y)] + [(torch.zeros_like(x), torch.empty_like(y))
+                                   for _ in range(_sets_for(x.nbytes + y.nbytes) - 1)]
+                ms = _time_cold(torch, [(lambda xb=xb, yb=yb: sn.convert_q(xb, a_, b_, shp, 0.05, out=yb))
+                                        for xb, yb in bufs])
+                del bufs
+                by = x.numel() * x.element_size() + y.numel() * y.element_size()
+                rows.append({"kernel": "adapt/convert (qi8)", "from": "%s.%s" % a_, "to": "%s.%s" % b_,
+                             "shape": list(shp), "us": ms * 1e3, "gbs": by / ms / 1e6, "frac": by / ms / 1e6 / hbm})
+        for (fi, fo) in [(25088, 4096), (4096, 4096)]:
+            layer = {"type": "dense", "params": dict(in_features=fi, out_features=fo, act="relu"),
+                     "weight": np.zeros((fo, fi), np.float32), "bias": np.zeros(fo, np.float32)}
+            sets = _sets_for(fi * fo)
+            gs = []
+            for _ in range(sets):
+                g = _single_layer_graph(sn, layer, (1, fi, 1, 1), ("qi8", "nhwc"))
+                g.set_qscale(-1, 0.05)
+                g.set_qscale(0, 0.05)
+                _forced(sn, g, "dense/simt")
+                gs.append((g, torch.zeros((1, 1, 1, fi), dtype=torch.int8, device="cuda"), g.new_output()))
+                gs[-1][0].run(gs[-1][1], gs[-1][2])  # plan and weights built before the capture
+            torch.cuda.synchronize()
+            ms = _time_cold(torch, [(lambda g=g, xb=xb, yb=yb: g.run(xb, yb)) for g, xb, yb in gs])
+            del gs
+            by = fi * fo + fi + fo + 8 * fo  # codes, input, output, weight scales + bias
+            rows.append({"kernel": "dense/simt (qi8)", "shape": [1, fi, fo], "us": ms * 1e3, "gbs": by / ms / 1e6,
+                         "frac": by / ms / 1e6 / hbm})
         out.update({"metric": "achieved HBM GB/s (algorithmic bytes / event time)", "peak_gbs": hbm, "rows": rows})
+    elif args.config == "q8_dense":
+        # the int8 dense routine on VGG16's first fully connected shape at batch 1
+        # (102.8 MB of weight codes, read once per launch): a small case for ncu
+        fi, fo = 25088, 4096
+        layer = {"type": "dense", "params": dict(in_features=fi, out_features=fo, act="relu"),
+                 "weight": np.zeros((fo, fi), np.float32), "bias": np.zeros(fo, np.float32)}
+        g = _single_layer_graph(sn, layer, (1, fi, 1, 1), ("qi8", "nhwc"))
+        g.set_qscale(-1, 0.05)
+        g.set_qscale(0, 0.05)
+        _forced(sn, g, "dense/simt")
+        xb = torch.zeros((1, 1, 1, fi), dtype=torch.int8, device="cuda")
+        yb = g.new_output()
+        ms = _time_back_to_back(torch, lambda: g.run(xb, yb), reps=20, warm=3)
+        by = fi * fo + fi + fo + 8 * fo
+        out.update({"metric": "dense/simt (qi8), batch 1, back-to-back launches of one weight set (102.8 MB, "
+                              "within L2; --config bandwidth gives the cold-L2 figure)",
+                    "shape": [1, fi, fo], "us": ms * 1e3, "gbs": by / ms / 1e6, "frac": by / ms / 1e6 / hbm})
     elif args.config == "layer":
         # one bf16 NHWC conv layer on the tensor-core routine: every routine-parameter
         # combination (or the one given), timed back to back

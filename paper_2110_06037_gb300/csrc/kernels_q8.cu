@@ -103,26 +103,130 @@ __global__ void q8_cast4_kernel(const Vec<Ti, 4> *__restrict__ x, Vec<To, 4> *__
     }
 }
 
-// y[b][c][r] = f(x[b][r][c]) through a 32 x 32 shared-memory tile
+// the value a conversion stores, as a float: a code (exact) when the output is
+// qint8, the fp32 value q * s when the input is
 template <typename Ti, typename To>
-__global__ void __launch_bounds__(256) q8_transpose_kernel(const Ti *__restrict__ x, To *__restrict__ y, int R,
-                                                           int C, float s, float inv) {
+__device__ __forceinline__ float q8_pre(float v, float s, float inv) {
+    if constexpr (std::is_same<Ti, int8_t>::value && std::is_same<To, int8_t>::value) return v;
+    else if constexpr (std::is_same<Ti, int8_t>::value) return __fmul_rn(v, s);
+    else return (float)q8_code(v, inv);
+}
+
+template <typename T> __device__ __forceinline__ float q8_ld(const T *p) { return ldf<T>(p); }
+template <> __device__ __forceinline__ float q8_ld<int8_t>(const int8_t *p) { return (float)*p; }
+template <typename T> __device__ __forceinline__ T q8_cv(float v) { return cvt<T>(v); }
+template <> __device__ __forceinline__ int8_t q8_cv<int8_t>(float v) { return (int8_t)(int)v; }
+
+template <typename T, int VB>
+struct QVec {
+    static constexpr int E = VB / (int)sizeof(T);
+    using V = typename std::conditional<
+        VB == 16, uint4,
+        typename std::conditional<VB == 8, uint2,
+                                  typename std::conditional<VB == 4, uint32_t,
+                                                            typename std::conditional<VB == 2, uint16_t,
+                                                                                      uint8_t>::type>::type>::type>::type;
+    __device__ __forceinline__ static void load(const T *p, float (&f)[E]) {
+        const V v = *reinterpret_cast<const V *>(p);
+        const T *t = reinterpret_cast<const T *>(&v);
+#pragma unroll
+        for (int e = 0; e < E; ++e) f[e] = q8_ld<T>(t + e);
+    }
+    __device__ __forceinline__ static void store(T *p, const float (&f)[E]) {
+        V v;
+        T *t = reinterpret_cast<T *>(&v);
+#pragma unroll
+        for (int e = 0; e < E; ++e) t[e] = q8_cv<T>(f[e]);
+        *reinterpret_cast<V *>(p) = v;
+    }
+};
+
+// same layout, 16 elements per thread (n % 16 == 0, 16-byte aligned bases)
+template <typename Ti, typename To>
+__global__ void q8_cast16_kernel(const Ti *__restrict__ x, To *__restrict__ y, int64_t n16, float s, float inv) {
     griddep_launch();
     griddep_wait();
-    __shared__ Ti tile[32][33];
+    constexpr int EI = 16 / (int)sizeof(Ti), EO = 16 / (int)sizeof(To);
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n16;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        float f[16];
+#pragma unroll
+        for (int k = 0; k < 16 / EI; ++k) {
+            float g[EI];
+            QVec<Ti, 16>::load(x + i * 16 + k * EI, g);
+#pragma unroll
+            for (int e = 0; e < EI; ++e) f[k * EI + e] = q8_pre<Ti, To>(g[e], s, inv);
+        }
+#pragma unroll
+        for (int k = 0; k < 16 / EO; ++k) {
+            float g[EO];
+#pragma unroll
+            for (int e = 0; e < EO; ++e) g[e] = f[k * EO + e];
+            QVec<To, 16>::store(y + i * 16 + k * EO, g);
+        }
+    }
+}
+
+// y[b][c][r] = f(x[b][r][c]) through a 64 x 64 shared-memory tile, VBI-byte
+// vectors along the input rows and VBO-byte vectors along the output rows
+constexpr int QT = 64;
+template <typename Ti, typename To, int VBI, int VBO>
+__global__ void __launch_bounds__(256) q8_transpose_vec_kernel(const Ti *__restrict__ x, To *__restrict__ y,
+                                                               int64_t R, int64_t Cc, float s, float inv) {
+    griddep_launch();
+    griddep_wait();
+    using LI = QVec<Ti, VBI>;
+    using LO = QVec<To, VBO>;
+    constexpr int EI = LI::E, EO = LO::E;
+    __shared__ float tile[QT][QT + 1];
     const int64_t b = blockIdx.z;
-    const int r0 = blockIdx.y * 32, c0 = blockIdx.x * 32;
-    const Ti *xb = x + b * (int64_t)R * C;
-    To *yb = y + b * (int64_t)R * C;
-    for (int i = threadIdx.y; i < 32; i += 8) {
-        const int r = r0 + i, c = c0 + threadIdx.x;
-        if (r < R && c < C) tile[i][threadIdx.x] = xb[(int64_t)r * C + c];
+    const int64_t r0 = (int64_t)blockIdx.y * QT, c0 = (int64_t)blockIdx.x * QT;
+    const Ti *xb = x + b * R * Cc;
+    To *yb = y + b * R * Cc;
+    constexpr int VI = QT / EI;
+#pragma unroll 4
+    for (int i = threadIdx.x; i < QT * VI; i += 256) {
+        const int row = i / VI, cv = i % VI;
+        const int64_t r = r0 + row, c = c0 + cv * EI;
+        if (r < R && c < Cc) {
+            float f[EI];
+            LI::load(xb + r * Cc + c, f);
+#pragma unroll
+            for (int e = 0; e < EI; ++e) tile[row][cv * EI + e] = q8_pre<Ti, To>(f[e], s, inv);
+        }
     }
     __syncthreads();
-    for (int i = threadIdx.y; i < 32; i += 8) {
-        const int c = c0 + i, r = r0 + threadIdx.x;
-        if (r < R && c < C) yb[(int64_t)c * R + r] = q8_xform<Ti, To>(tile[threadIdx.x][i], s, inv);
+    constexpr int VO = QT / EO;
+#pragma unroll 4
+    for (int i = threadIdx.x; i < QT * VO; i += 256) {
+        const int orow = i / VO, ov = i % VO;
+        const int64_t c = c0 + orow, r = r0 + ov * EO;
+        if (c < Cc && r < R) {
+            float f[EO];
+#pragma unroll
+            for (int e = 0; e < EO; ++e) f[e] = tile[ov * EO + e][orow];
+            LO::store(yb + c * R + r, f);
+        }
     }
+}
+
+// widest vector (16, 8 or 4 bytes, else one element) that every row of n
+// elements of es bytes from an aligned base admits, and at most 64 elements
+static int q8_row_vec(int64_t n, int es, const void *base) {
+    for (int vb : {16, 8, 4})
+        if (vb / es <= QT && vb >= es && (n * es) % vb == 0 && (uintptr_t)base % vb == 0) return vb;
+    return es;
+}
+
+template <typename Ti, typename To, int VBI>
+static void launch_q8_transpose(int vo, dim3 grid, cudaStream_t st, const Ti *x, To *y, int64_t R, int64_t Cc,
+                                float s, float inv) {
+    constexpr int SO = (int)sizeof(To);
+    if (vo == 16) launch_pdl(q8_transpose_vec_kernel<Ti, To, VBI, 16>, grid, 256, 0, st, x, y, R, Cc, s, inv);
+    else if (vo == 8) launch_pdl(q8_transpose_vec_kernel<Ti, To, VBI, 8>, grid, 256, 0, st, x, y, R, Cc, s, inv);
+    else if (vo == 4) launch_pdl(q8_transpose_vec_kernel<Ti, To, VBI, (SO <= 4 ? 4 : SO)>, grid, 256, 0, st, x, y, R,
+                                 Cc, s, inv);
+    else launch_pdl(q8_transpose_vec_kernel<Ti, To, VBI, SO>, grid, 256, 0, st, x, y, R, Cc, s, inv);
 }
 
 template <typename Ti, typename To>
@@ -131,6 +235,11 @@ static cudaError_t convert_q8_t(const void *x, int lay_in, void *y, int lay_out,
     const int64_t n = sh.numel();
     if (n == 0) return cudaSuccess;
     if (lay_in == lay_out || sh.c == 1 || sh.h * sh.w == 1) {
+        if (n % 16 == 0 && (uintptr_t)x % 16 == 0 && (uintptr_t)y % 16 == 0) {
+            launch_pdl(q8_cast16_kernel<Ti, To>, grid_for(n / 16, 256), 256, 0, st, (const Ti *)x, (To *)y, n / 16, s,
+                       inv);
+            return cudaGetLastError();
+        }
         const bool vec = n % 4 == 0 && (uintptr_t)x % (4 * sizeof(Ti)) == 0 && (uintptr_t)y % (4 * sizeof(To)) == 0;
         if (vec)
             launch_pdl(q8_cast4_kernel<Ti, To>, grid_for(n / 4, 256), 256, 0, st, (const Vec<Ti, 4> *)x,
@@ -143,8 +252,15 @@ static cudaError_t convert_q8_t(const void *x, int lay_in, void *y, int lay_out,
     const int64_t hw = sh.h * sh.w;
     const int R = (int)(lay_in == SN_NCHW ? sh.c : hw), C = (int)(lay_in == SN_NCHW ? hw : sh.c);
     if (sh.n > 65535) return cudaErrorInvalidValue;
-    const dim3 grid((unsigned)((C + 31) / 32), (unsigned)((R + 31) / 32), (unsigned)sh.n);
-    launch_pdl(q8_transpose_kernel<Ti, To>, grid, dim3(32, 8), 0, st, (const Ti *)x, (To *)y, R, C, s, inv);
+    const dim3 grid((unsigned)((C + QT - 1) / QT), (unsigned)((R + QT - 1) / QT), (unsigned)sh.n);
+    constexpr int SI = (int)sizeof(Ti);
+    const int vi = q8_row_vec(C, SI, x), vo = q8_row_vec(R, (int)sizeof(To), y);
+    const Ti *xi = (const Ti *)x;
+    To *yo = (To *)y;
+    if (vi == 16) launch_q8_transpose<Ti, To, 16>(vo, grid, st, xi, yo, R, C, s, inv);
+    else if (vi == 8) launch_q8_transpose<Ti, To, 8>(vo, grid, st, xi, yo, R, C, s, inv);
+    else if (vi == 4) launch_q8_transpose<Ti, To, (SI <= 4 ? 4 : SI)>(vo, grid, st, xi, yo, R, C, s, inv);
+    else launch_q8_transpose<Ti, To, SI>(vo, grid, st, xi, yo, R, C, s, inv);
     return cudaGetLastError();
 }
 
@@ -463,7 +579,8 @@ __global__ void __launch_bounds__(256) q8_dense_kernel(const int8_t *__restrict_
     for (int n0 = 0; n0 < N; n0 += NB) {
         int acc[NB] = {};
         if (V16) {
-            for (int i = lane * 16; i < I; i += 32 * 16) {
+            int i = lane * 16;
+            for (; i < I; i += 512) {
                 const int4 wv = *reinterpret_cast<const int4 *>(wr + i);
 #pragma unroll
                 for (int b = 0; b < NB; ++b) {
