@@ -328,12 +328,49 @@ __global__ void weight_wino4_kernel(const float *__restrict__ w, float *__restri
     }
 }
 
+// Winograd F(6x6,3x3) filter transform U = G g G^T with the 8x3 G of the
+// points 0, +-1, +-2, +-1/2 and infinity, fp32 [64][K][C]
+__device__ __forceinline__ void wino6_g(float g0, float g1, float g2, float (&u)[8]) {
+    u[0] = g0;
+    u[1] = -2.f * (g0 + g1 + g2) / 9.f;
+    u[2] = -2.f * (g0 - g1 + g2) / 9.f;
+    u[3] = g0 / 90.f + g1 / 45.f + 2.f * g2 / 45.f;
+    u[4] = g0 / 90.f - g1 / 45.f + 2.f * g2 / 45.f;
+    u[5] = 32.f * g0 / 45.f + 16.f * g1 / 45.f + 8.f * g2 / 45.f;
+    u[6] = 32.f * g0 / 45.f - 16.f * g1 / 45.f + 8.f * g2 / 45.f;
+    u[7] = g2;
+}
+__global__ void weight_wino6_kernel(const float *__restrict__ w, float *__restrict__ out, int64_t K, int64_t C) {
+    griddep_launch();
+    griddep_wait();
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < K * C;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const float *g = w + i * 9;  // [3][3] for (k, c) = (i / C, i % C)
+        float t[8][3];               // G g, column by column
+        for (int j = 0; j < 3; ++j) {
+            float u[8];
+            wino6_g(g[0 * 3 + j], g[1 * 3 + j], g[2 * 3 + j], u);
+            for (int a = 0; a < 8; ++a) t[a][j] = u[a];
+        }
+        for (int a = 0; a < 8; ++a) {  // (G g) G^T
+            float u[8];
+            wino6_g(t[a][0], t[a][1], t[a][2], u);
+            for (int b = 0; b < 8; ++b) out[(int64_t)(a * 8 + b) * K * C + i] = u[b];
+        }
+    }
+}
+
 cudaError_t weight_format(const float *w, void *out, int fmt, int dt, int64_t K, int64_t Cg,
                           int64_t R, int64_t S, cudaStream_t st) {
     if (dt == SN_QI8) return cudaErrorInvalidValue;  // codes and scales: weight_format_q8
     if (fmt == W_WINO4) {  // fp32 whatever the schema's dtype
         if (R != 3 || S != 3) return cudaErrorInvalidValue;
         launch_pdl(weight_wino4_kernel, grid_for(K * Cg, 256), 256, 0, st, w, (float *)out, K, Cg);
+        return cudaGetLastError();
+    }
+    if (fmt == W_WINO6) {  // fp32 whatever the schema's dtype
+        if (R != 3 || S != 3) return cudaErrorInvalidValue;
+        launch_pdl(weight_wino6_kernel, grid_for(K * Cg, 256), 256, 0, st, w, (float *)out, K, Cg);
         return cudaGetLastError();
     }
     if (fmt == W_WINO) {

@@ -521,6 +521,165 @@ cudaError_t conv_wino4(const LaunchArgs &a) {
     return cudaGetLastError();
 }
 
+// ---------------------------------------------------------------------------
+// Winograd F(6x6, 3x3): 8x8 input tiles, 64 element-wise GEMMs, 6x6 outputs
+// (Toom-Cook interpolation points 0, +-1, +-2, +-1/2 and infinity; the
+// paper's tile_size 8).  Transformed filters and the GEMM stay fp32.
+// ---------------------------------------------------------------------------
+static WinoDims wino6_dims(const ConvDims &d) {
+    WinoDims w;
+    w.d = d;
+    w.tP = (d.P + 5) / 6;
+    w.tQ = (d.Q + 5) / 6;
+    w.T = (int64_t)d.N * w.tP * w.tQ;
+    return w;
+}
+
+size_t conv_wino6_ws(const Layer &l, const Shape &in, sn_schema s) {
+    (void)s;
+    const int64_t tiles = in.n * ((l.out.h + 5) / 6) * ((l.out.w + 5) / 6);
+    return (size_t)64 * tiles * (in.c + l.out.c) * sizeof(float);
+}
+
+// r = B^T d for one column d of the 8x8 tile
+__device__ __forceinline__ void wino6_bt(const float (&d)[8], float (&r)[8]) {
+    r[0] = d[0] - 5.25f * d[2] + 5.25f * d[4] - d[6];
+    r[1] = d[1] + d[2] - 4.25f * d[3] - 4.25f * d[4] + d[5] + d[6];
+    r[2] = -d[1] + d[2] + 4.25f * d[3] - 4.25f * d[4] - d[5] + d[6];
+    r[3] = 0.5f * d[1] + 0.25f * d[2] - 2.5f * d[3] - 1.25f * d[4] + 2.f * d[5] + d[6];
+    r[4] = -0.5f * d[1] + 0.25f * d[2] + 2.5f * d[3] - 1.25f * d[4] - 2.f * d[5] + d[6];
+    r[5] = 2.f * d[1] + 4.f * d[2] - 2.5f * d[3] - 5.f * d[4] + 0.5f * d[5] + d[6];
+    r[6] = -2.f * d[1] + 4.f * d[2] + 2.5f * d[3] - 5.f * d[4] - 0.5f * d[5] + d[6];
+    r[7] = -d[1] + 5.25f * d[3] - 5.25f * d[5] + d[7];
+}
+// o = A^T m for one column m
+__device__ __forceinline__ void wino6_at(const float (&m)[8], float (&o)[6]) {
+    const float p12 = m[1] + m[2], m12 = m[1] - m[2];
+    const float p34 = m[3] + m[4], m34 = m[3] - m[4];
+    const float p56 = m[5] + m[6], m56 = m[5] - m[6];
+    o[0] = m[0] + p12 + p34 + p56;
+    o[1] = m12 + 2.f * m34 + 0.5f * m56;
+    o[2] = p12 + 4.f * p34 + 0.25f * p56;
+    o[3] = m12 + 8.f * m34 + 0.125f * m56;
+    o[4] = p12 + 16.f * p34 + 0.0625f * p56;
+    o[5] = m12 + 32.f * m34 + 0.03125f * m56 + m[7];
+}
+
+// wgenc: V[xi][t][c] = (B^T d B)[xi] for the 8x8 input tile of output tile t
+template <typename T, bool NHWC>
+__global__ void wino6_input_kernel(const T *__restrict__ x, float *__restrict__ V, WinoDims wd) {
+    griddep_launch();
+    griddep_wait();
+    const ConvDims &d = wd.d;
+    const int64_t total = wd.T * d.C;
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const int c = (int)(i % d.C);
+        const int64_t t = i / d.C;
+        const int tq = (int)(t % wd.tQ), tp = (int)((t / wd.tQ) % wd.tP);
+        const int64_t n = t / ((int64_t)wd.tQ * wd.tP);
+        const int h0 = 6 * tp - d.ph, w0 = 6 * tq - d.pw;
+        float t8[8][8];  // B^T d, column by column
+#pragma unroll
+        for (int b = 0; b < 8; ++b) {
+            float col[8];
+#pragma unroll
+            for (int a = 0; a < 8; ++a) {
+                const int h = h0 + a, ww = w0 + b;
+                float val = 0.f;
+                if (h >= 0 && h < d.H && ww >= 0 && ww < d.W) {
+                    const int64_t idx = NHWC ? ((n * d.H + h) * d.W + ww) * d.C + c
+                                             : ((n * d.C + c) * d.H + h) * (int64_t)d.W + ww;
+                    val = ldf<T>(x + idx);
+                }
+                col[a] = val;
+            }
+            float r[8];
+            wino6_bt(col, r);
+#pragma unroll
+            for (int a = 0; a < 8; ++a) t8[a][b] = r[a];
+        }
+#pragma unroll
+        for (int a = 0; a < 8; ++a) {  // (B^T d) B: B^T applied to each row
+            float r[8];
+            wino6_bt(t8[a], r);
+#pragma unroll
+            for (int b = 0; b < 8; ++b) V[((int64_t)(a * 8 + b) * wd.T + t) * d.C + c] = r[b];
+        }
+    }
+}
+
+// wgdec: Y = A^T M A for each output tile, + bias, activation, store
+template <typename T, bool NHWC>
+__global__ void wino6_output_kernel(const float *__restrict__ Mx, const float *__restrict__ bias,
+                                    T *__restrict__ y, WinoDims wd) {
+    griddep_launch();
+    griddep_wait();
+    const ConvDims &d = wd.d;
+    const int64_t total = wd.T * d.K;
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const int kk = (int)(i % d.K);
+        const int64_t t = i / d.K;
+        const int tq = (int)(t % wd.tQ), tp = (int)((t / wd.tQ) % wd.tP);
+        const int64_t n = t / ((int64_t)wd.tQ * wd.tP);
+        float u[6][8];  // A^T M, column by column
+#pragma unroll
+        for (int b = 0; b < 8; ++b) {
+            float col[8];
+#pragma unroll
+            for (int a = 0; a < 8; ++a) col[a] = Mx[((int64_t)(a * 8 + b) * wd.T + t) * d.K + kk];
+            float o[6];
+            wino6_at(col, o);
+#pragma unroll
+            for (int a = 0; a < 6; ++a) u[a][b] = o[a];
+        }
+        const float bv = bias[kk];
+#pragma unroll
+        for (int a = 0; a < 6; ++a) {
+            const int p = 6 * tp + a;
+            if (p >= d.P) continue;
+            float yy[6];
+            wino6_at(u[a], yy);
+#pragma unroll
+            for (int b = 0; b < 6; ++b) {
+                const int q = 6 * tq + b;
+                if (q >= d.Q) continue;
+                const int64_t o = NHWC ? ((n * d.P + p) * d.Q + q) * d.K + kk
+                                       : ((n * d.K + kk) * d.P + p) * (int64_t)d.Q + q;
+                stf<T>(y + o, act_apply(yy[b] + bv, d.act));
+            }
+        }
+    }
+}
+
+cudaError_t conv_wino6(const LaunchArgs &a) {
+    const ConvDims d = conv_dims(a);
+    const WinoDims wd = wino6_dims(d);
+    const size_t need = (size_t)64 * wd.T * (d.C + d.K) * sizeof(float);
+    if (!a.ws || a.ws_bytes < need) return cudaErrorInvalidValue;
+    float *V = static_cast<float *>(a.ws);
+    float *Mx = V + (size_t)64 * wd.T * d.C;
+    dim3 ggrid((unsigned)((wd.T + 63) / 64), (unsigned)((d.K + 63) / 64), 64);
+    if (ggrid.y > 65535) return cudaErrorInvalidValue;
+    SN_DT_SWITCH(a.schema.dtype, T, {
+        if (a.schema.layout == SN_NHWC)
+            launch_pdl(wino6_input_kernel<T, true>, grid_for(wd.T * d.C, 256), 256, 0, a.stream, (const T *)a.in[0],
+                       V, wd);
+        else
+            launch_pdl(wino6_input_kernel<T, false>, grid_for(wd.T * d.C, 256), 256, 0, a.stream,
+                       (const T *)a.in[0], V, wd);
+        launch_pdl(gemm_nt_simt<float>, ggrid, 256, 0, a.stream, V, (const float *)a.wt, Mx, wd.T, d.K, d.C);
+        if (a.schema.layout == SN_NHWC)
+            launch_pdl(wino6_output_kernel<T, true>, grid_for(wd.T * d.K, 256), 256, 0, a.stream, Mx, a.bias,
+                       (T *)a.out, wd);
+        else
+            launch_pdl(wino6_output_kernel<T, false>, grid_for(wd.T * d.K, 256), 256, 0, a.stream, Mx, a.bias,
+                       (T *)a.out, wd);
+    });
+    return cudaGetLastError();
+}
+
 // The three Winograd stages on caller-provided buffers (used by the
 // allocation-free entry point): U [16][K][C] in the schema dtype, V and Mx fp32.
 cudaError_t conv_wino_buffers(const ConvDims &d, sn_schema s, const void *x, const void *u, const float *bias,

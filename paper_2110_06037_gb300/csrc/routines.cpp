@@ -17,6 +17,7 @@ const char *routine_name(int32_t r) {
     case R_CONV_IGEMM: return "conv2/igemm_simt";
     case R_CONV_WINO: return "conv2/wino_f2x2_3x3";
     case R_CONV_WINO4: return "conv2/wino_f4x4_3x3";
+    case R_CONV_WINO6: return "conv2/wino_f6x6_3x3";
     case R_CONV_TC: return "conv2/igemm_tc";
     case R_DW_DIRECT: return "dwconv2/direct";
     case R_MAXPOOL: return "maxpool/direct";
@@ -77,6 +78,7 @@ int32_t routine_variants(int32_t r, const Layer &l, const std::vector<Shape> &in
         return (is_conv(l) && p.groups == 1) ? 2 : 0;
     case R_CONV_WINO:
     case R_CONV_WINO4:
+    case R_CONV_WINO6:
         return (is_conv(l) && p.groups == 1 && p.kh == 3 && p.kw == 3 && p.sh == 1 && p.sw == 1 &&
                 p.dh == 1 && p.dw == 1 && p.ph <= 2 && p.pw <= 2)
                    ? 1
@@ -110,6 +112,7 @@ size_t routine_workspace(int32_t r, int32_t v, const Layer &l, const std::vector
                          sn_schema s) {
     if (r == R_CONV_WINO) return k::conv_wino_ws(l, in[0], s);
     if (r == R_CONV_WINO4) return k::conv_wino4_ws(l, in[0], s);
+    if (r == R_CONV_WINO6) return k::conv_wino6_ws(l, in[0], s);
     if (r == R_CONV_TC) return k::conv_tc_ws(l, in[0], s, v);
     if (r == R_CONV_IM2COL_TC) return k::conv_im2col_tc_ws(l, in[0], s, v);
     if (r == R_DENSE_TC) return k::dense_tc_ws(l, in[0], s, v);
@@ -133,6 +136,7 @@ static int weight_format_of(int32_t r, sn_schema s) {
     case R_CONV_IGEMM: return s.layout == SN_NCHW ? k::W_KCRS : k::W_KRSC;
     case R_CONV_WINO: return k::W_WINO;
     case R_CONV_WINO4: return k::W_WINO4;
+    case R_CONV_WINO6: return k::W_WINO6;
     case R_CONV_TC: return k::W_KRSC;
     case R_DW_DIRECT: return s.layout == SN_NCHW ? k::W_KCRS : k::W_RSCK;
     case R_DENSE: return k::W_KCRS;
@@ -182,6 +186,7 @@ sn_status prepare_weights(Graph *g, int32_t li, int32_t r, int32_t v, sn_schema 
     }
     const int64_t elems = (fmt == k::W_WINO)         ? 16 * K * Cg
                           : (fmt == k::W_WINO4)      ? 36 * K * Cg
+                          : (fmt == k::W_WINO6)      ? 64 * K * Cg
                           : (fmt == k::W_KRSC_PAD64) ? K * ((Cg * R * S + 63) / 64 * 64)
                           : (fmt == k::W_S2D)        ? K * (R <= 4 ? 2 : 4) * 64
                                                      : K * Cg * R * S;
@@ -189,7 +194,7 @@ sn_status prepare_weights(Graph *g, int32_t li, int32_t r, int32_t v, sn_schema 
     sn_status rc = dev_alloc(g, (size_t)K * Cg * R * S * sizeof(float), &src);
     if (rc != SN_OK) return rc;
     const size_t dst_bytes = s.dtype == SN_QI8 ? k::q8_weight_bytes(K, elems)  // codes + per-channel scales
-                             : (size_t)elems * (fmt == k::W_WINO4 ? sizeof(float) : dtype_size(s.dtype));
+                             : (size_t)elems * ((fmt == k::W_WINO4 || fmt == k::W_WINO6) ? sizeof(float) : dtype_size(s.dtype));
     rc = dev_alloc(g, dst_bytes, &dst);
     if (rc != SN_OK) {
         dev_free(g, &src);
@@ -221,7 +226,7 @@ int32_t kernels_per_launch(int32_t r, int32_t v, const Layer &l, const std::vect
                           (r == R_CONV_IM2COL_TC ? k::conv_im2col_tc_ws(l, in[0], s, -1)
                            : r == R_CONV_S2D_TC  ? k::conv_s2d_tc_ws(l, in[0], s, -1)
                                                  : 0);
-    if (r == R_CONV_WINO || r == R_CONV_WINO4) return 3;  // wgenc, wgconv, wgdec
+    if (r == R_CONV_WINO || r == R_CONV_WINO4 || r == R_CONV_WINO6) return 3;  // wgenc, wgconv, wgdec
     if (r == R_CONV_IM2COL_TC || r == R_CONV_S2D_TC) return 2 + split;  // re-layout, GEMM (+ reduction)
     return 1 + split;
 }
@@ -253,6 +258,7 @@ sn_status launch_routine(const LaunchArgs &a) {
     case R_CONV_IGEMM: e = k::conv_igemm(a); break;
     case R_CONV_WINO: e = k::conv_wino(a); break;
     case R_CONV_WINO4: e = k::conv_wino4(a); break;
+    case R_CONV_WINO6: e = k::conv_wino6(a); break;
     case R_CONV_TC: e = k::conv_tc(a); break;
     case R_DW_DIRECT: e = k::dwconv(a); break;
     case R_MAXPOOL: e = k::maxpool(a); break;

@@ -70,7 +70,8 @@ enum RoutineId : int32_t {
     R_MUL = 14,          // per-channel scale (squeeze-and-excite)
     R_CONV_WINO4 = 15,   // Winograd F(4x4,3x3) childnet (fp32 transformed filters)
     R_CONV_DP4A = 16,    // qint8 implicit GEMM with dp4a (NHWC)
-    R_COUNT = 17
+    R_CONV_WINO6 = 17,   // Winograd F(6x6,3x3) childnet (fp32 transformed filters)
+    R_COUNT = 18
 };
 
 // -------------------------------------------------------------------------
@@ -234,7 +235,7 @@ cudaError_t convert(const void *x, int dt_in, int lay_in, void *y, int dt_out, i
 cudaError_t fill_pattern(void *y, int dt, int64_t n, uint32_t seed, float scale,
                          cudaStream_t st);
 // weight re-layout / cast from fp32 KCRS (device) into a routine format
-enum WFormat { W_KCRS = 0, W_RSCK = 1, W_KRSC = 2, W_WINO = 3, W_KRSC_PAD64 = 4, W_S2D = 5, W_WINO4 = 6 };
+enum WFormat { W_KCRS = 0, W_RSCK = 1, W_KRSC = 2, W_WINO = 3, W_KRSC_PAD64 = 4, W_S2D = 5, W_WINO4 = 6, W_WINO6 = 7 };
 cudaError_t weight_format(const float *w_kcrs, void *out, int fmt, int dt, int64_t K,
                           int64_t Cg, int64_t R, int64_t S, cudaStream_t st);
 
@@ -244,6 +245,8 @@ cudaError_t conv_wino(const LaunchArgs &a);
 size_t conv_wino_ws(const Layer &l, const Shape &in, sn_schema s);
 cudaError_t conv_wino4(const LaunchArgs &a);
 size_t conv_wino4_ws(const Layer &l, const Shape &in, sn_schema s);
+cudaError_t conv_wino6(const LaunchArgs &a);
+size_t conv_wino6_ws(const Layer &l, const Shape &in, sn_schema s);
 cudaError_t conv_tc(const LaunchArgs &a);
 int32_t conv_tc_variants(const Layer &l, const Shape &in, sn_schema s);
 size_t conv_tc_ws(const Layer &l, const Shape &in, sn_schema s, int32_t v, int32_t a_blocks = 0);  // K-split partials

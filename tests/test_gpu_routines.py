@@ -61,7 +61,7 @@ CONV_CASES = [
     (1, 2, 16, 16, 8, 5, 2, 2, 1, 1),      # space-to-depth: 5x5 kernel
 ]
 ROUTINES = ([("conv2/direct", 0), ("conv2/igemm_simt", 0), ("conv2/igemm_simt", 1), ("conv2/wino_f2x2_3x3", 0),
-             ("conv2/wino_f4x4_3x3", 0)]
+             ("conv2/wino_f4x4_3x3", 0), ("conv2/wino_f6x6_3x3", 0)]
             + [("conv2/igemm_tc", v) for v in range(6)] + [("conv2/im2col_tc", v) for v in range(3)]
             + [("conv2/s2d_tc", v) for v in range(4)])
 
