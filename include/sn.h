@@ -134,7 +134,8 @@ SN_API sn_status sn_graph_create(const int64_t in_nchw[4], sn_schema in_schema, 
  * Append a layer (section III-B).  params points to the struct for the type
  * (sn_conv_params for CONV2/DWCONV2, sn_pool_params, sn_add_params,
  * sn_dense_params; NULL for GAP).  inputs[0..n_inputs) are ids returned by
- * earlier calls, -1 = the net input (ADD takes two, the others one).
+ * earlier calls, -1 = the net input, -2, -3, ... = the inputs declared by
+ * sn_add_input (ADD takes two, the others one).
  * CONV2 may take a second input, a residual of exactly the output's shape:
  * y = act(conv(x) + bias + residual), the residual add of a ResNet block fused
  * into the convolution that feeds it (the paper's graph optimiser fuses
@@ -142,7 +143,8 @@ SN_API sn_status sn_graph_create(const int64_t in_nchw[4], sn_schema in_schema, 
  * routines serve such a layer.
  * weights: host fp32, conv [c_out][c_in/groups][kh][kw], dense [out][in];
  * bias: host fp32 [c_out] or NULL (zeros).  Both are copied.  The last layer
- * added is the net output.  *out_layer_id receives the new layer's id.
+ * added is the net output unless sn_set_outputs names others.
+ * *out_layer_id receives the new layer's id.
  * Errors: SN_EINVAL (shape mismatch, bad parameter), SN_ESTATE (after the
  * net was finalised by sn_profile/sn_get_cost_table/sn_select_path/...).
  */
@@ -150,10 +152,30 @@ SN_API sn_status sn_add_layer(sn_graph *g, int32_t type, const void *params, con
                        int32_t n_inputs, const float *weights, const float *bias,
                        int32_t *out_layer_id);
 
+/* ---------------- several inputs and outputs (section IV-E) ---------------
+ * A net may read several input blobs and produce several output blobs; the
+ * auxiliary input layer feeds every input layer and the auxiliary output layer
+ * merges every output, so the tuning problem stays 1-in-1-out.
+ * sn_add_input: declare another net input of logical shape in_nchw, stored in
+ *   in_schema; *input_id receives its id for sn_add_layer's inputs (-2 for the
+ *   second input, -3 for the third, ...; the first, from sn_graph_create, is
+ *   -1).  Every input must be declared before the first sn_add_layer, and
+ *   every input must feed some layer.
+ * sn_set_outputs: the net outputs, in order (distinct layer ids); each is
+ *   delivered in out_schema.  Default: the last layer added.
+ * sn_get_io: the number of net inputs and outputs.
+ * Errors: SN_EINVAL (bad extent or id), SN_ESTATE (after finalisation, or
+ * sn_add_input after a layer). */
+SN_API sn_status sn_add_input(sn_graph *g, const int64_t in_nchw[4], int32_t *input_id);
+SN_API sn_status sn_set_outputs(sn_graph *g, const int32_t *layer_ids, int32_t n);
+SN_API sn_status sn_get_io(sn_graph *g, int32_t *n_inputs, int32_t *n_outputs);
+
 /* ---------------- the cost table (profiling data, section III-C) ----------
- * After finalisation the net has n_layers = (layers added) + 2 internal
- * layers in topological order: 0 is the input layer, n_layers-1 the output
- * layer and layer id u returned by sn_add_layer is internal layer u+1.
+ * After finalisation the net has n_layers = (net inputs) + (layers added) + 1
+ * internal layers in topological order: 0 is the auxiliary input layer (it
+ * holds the first net input), 1 .. n_inputs-1 hold the other net inputs,
+ * layer id u returned by sn_add_layer is internal layer u + n_inputs, and
+ * n_layers-1 is the auxiliary output layer.
  * Each layer has candidate routines (routine id, routine-parameter
  * combination "variant", schema index); each edge (src, dst) has an adapt
  * cost for every ordered schema pair (void adapt = 0 on the diagonal).
@@ -233,11 +255,18 @@ SN_API sn_status sn_set_option(sn_graph *g, int32_t option, int64_t value);
  * builds the plan (adapt insertion, buffers, weight copies per schema).
  * Errors: SN_ESTATE (no path), SN_ENOMEM, SN_ECUDA, SN_ETIMEOUT. */
 SN_API sn_status sn_run(sn_graph *g, const void *in_dev, void *out_dev, void *stream);
+/* sn_run for a net with several inputs or outputs: in_devs[0..n_in) in the
+ * order of their ids (-1, -2, ...), out_devs[0..n_out) in the order given to
+ * sn_set_outputs.  n_in and n_out must match the net (SN_EINVAL otherwise);
+ * sn_run is this call with one of each. */
+SN_API sn_status sn_run_multi(sn_graph *g, const void *const *in_devs, int32_t n_in, void *const *out_devs,
+                              int32_t n_out, void *stream);
 
 /* sn_run with a CUDA event pair around every launch of the plan; after the
  * stream has finished (this call synchronises it) layer_ms[i] holds the time
  * of layer i's routine and edge_ms[e] that of edge e's adapt (0 if void).
- * Either array may be NULL.  Sizes: n_layers and n_edges. */
+ * Either array may be NULL.  Sizes: n_layers and n_edges.  Nets with one
+ * input and one output only (SN_EINVAL otherwise). */
 SN_API sn_status sn_run_timed(sn_graph *g, const void *in_dev, void *out_dev, void *stream,
                        float *layer_ms, float *edge_ms);
 
@@ -294,7 +323,9 @@ SN_API sn_status sn_get_qscale(sn_graph *g, int32_t layer_id, float *scale);
  * layer's output to max |x| / 127 of the blob as that path stores it (1 for an
  * all-zero blob).  The selected path, if any, is kept.  Synchronises stream.
  * Errors: SN_ESTATE (costs not profiled or set: no finite float path),
- * SN_EUNSUPPORTED (in_schema or out_schema is SN_QI8), SN_ECUDA, SN_ENOMEM. */
+ * SN_EUNSUPPORTED (in_schema or out_schema is SN_QI8, or the net has several
+ * inputs: set their scales with sn_set_qscale), SN_ECUDA, SN_ENOMEM.
+ * sn_set_qscale / sn_get_qscale take the ids of sn_add_input too. */
 SN_API sn_status sn_calibrate(sn_graph *g, const void *in_dev, void *stream);
 
 /* ---------------- allocation-free Winograd convolution --------------------

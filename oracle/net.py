@@ -54,15 +54,18 @@ def run_layer(layer: dict, inputs: list, dtype: str = "f32") -> np.ndarray:
     raise ValueError(f"unknown layer type {t}")
 
 
-def run_net(layers: list, x: np.ndarray, dtype: str = "f32", keep: bool = False):
+def run_net(layers: list, x, dtype: str = "f32", keep: bool = False):
     """Whole net from the input as stored in `dtype`.
 
-    Returns the output (fp64 NCHW), or (output, [every layer's output]) when
+    x is the net input, or a list of net inputs for ids -1, -2, ... (several
+    input layers under the auxiliary input layer, section IV-E).  Returns the
+    last layer's output (fp64 NCHW), or (output, [every layer's output]) when
     keep=True.
     """
-    x0 = round_to(np.asarray(x, np.float32), dtype).astype(np.float64)
+    xs = list(x) if isinstance(x, (list, tuple)) else [x]
+    x0s = [round_to(np.asarray(v, np.float32), dtype).astype(np.float64) for v in xs]
     outs = []
     for layer in layers:
-        ins = [x0 if j < 0 else outs[j] for j in layer["inputs"]]
+        ins = [x0s[-1 - j] if j < 0 else outs[j] for j in layer["inputs"]]
         outs.append(run_layer(layer, ins, dtype))
     return (outs[-1], outs) if keep else outs[-1]

@@ -102,6 +102,11 @@ SIGNATURES = {
     "sn_set_qscale": (C.c_int, [C.c_void_p, C.c_int32, C.c_float]),
     "sn_get_qscale": (C.c_int, [C.c_void_p, C.c_int32, C.POINTER(C.c_float)]),
     "sn_calibrate": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p]),
+    "sn_add_input": (C.c_int, [C.c_void_p, C.POINTER(C.c_int64), C.POINTER(C.c_int32)]),
+    "sn_set_outputs": (C.c_int, [C.c_void_p, C.POINTER(C.c_int32), C.c_int32]),
+    "sn_get_io": (C.c_int, [C.c_void_p, C.POINTER(C.c_int32), C.POINTER(C.c_int32)]),
+    "sn_run_multi": (C.c_int, [C.c_void_p, C.POINTER(C.c_void_p), C.c_int32, C.POINTER(C.c_void_p), C.c_int32,
+                               C.c_void_p]),
     "sn_conv2d_wino_noalloc": (C.c_int, [C.c_void_p, sn_schema, C.POINTER(C.c_int64), C.c_int32, C.c_int32,
                                          C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p]),
     "sn_last_error": (C.c_char_p, []),

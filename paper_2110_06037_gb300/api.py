@@ -83,6 +83,23 @@ class Graph:
             self.h = None
 
     # ------------------------------------------------------------- building
+    def add_input(self, shape):
+        """Another net input (before any layer); returns its id (-2, -3, ...)."""
+        shp = (C.c_int64 * 4)(*[int(v) for v in shape])
+        i = C.c_int32(0)
+        check(lib().sn_add_input(self.h, shp, C.byref(i)))
+        return i.value
+
+    def set_outputs(self, ids):
+        """The net outputs, in order (default: the last layer added)."""
+        arr = (C.c_int32 * len(ids))(*[int(v) for v in ids])
+        check(lib().sn_set_outputs(self.h, arr, len(ids)))
+
+    def io_counts(self):
+        a, b = C.c_int32(0), C.c_int32(0)
+        check(lib().sn_get_io(self.h, C.byref(a), C.byref(b)))
+        return a.value, b.value
+
     def add_layer(self, type_, params=None, inputs=(-1,), weight=None, bias=None) -> int:
         ins = (C.c_int32 * len(inputs))(*inputs)
         p = None
@@ -216,6 +233,25 @@ class Graph:
             out = self.new_output()
         check(lib().sn_run(self.h, C.c_void_p(x.data_ptr()), C.c_void_p(out.data_ptr()), _stream_ptr(stream)))
         return out
+
+    def output_shapes(self):
+        """Logical shapes of the net outputs (in order)."""
+        t = self.cost_table()
+        n = t["n_layers"]
+        srcs = [int(t["edges"][e][0]) for e in range(len(t["edges"])) if int(t["edges"][e][1]) == n - 1]
+        return [self.layer_shape(j) for j in srcs]
+
+    def run_multi(self, xs, outs=None, stream=None):
+        """Run a net with several inputs / outputs; returns the output tensors."""
+        torch = _torch()
+        if outs is None:
+            outs = [torch.empty(storage_shape(sh, self.out_schema[1]),
+                                dtype=getattr(torch, TORCH_DTYPES[self.out_schema[0]]), device="cuda")
+                    for sh in self.output_shapes()]
+        ins = (C.c_void_p * len(xs))(*[x.data_ptr() for x in xs])
+        os_ = (C.c_void_p * len(outs))(*[o.data_ptr() for o in outs])
+        check(lib().sn_run_multi(self.h, ins, len(xs), os_, len(outs), _stream_ptr(stream)))
+        return outs
 
     def run_timed(self, x, out=None, stream=None):
         if out is None:

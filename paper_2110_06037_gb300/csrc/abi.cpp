@@ -294,48 +294,95 @@ static sn_status check_device(Graph *g, cudaStream_t st) {
     return SN_OK;
 }
 
+static sn_status run_io(Graph *g, const IoPtrs &io, cudaStream_t st) {
+    if (!g->has_path) return fail(SN_ESTATE, "sn_run: select or set a routine path first");
+    if ((int32_t)io.in.size() != g->n_in() || (int32_t)io.out.size() != g->n_out())
+        return fail(SN_EINVAL, "sn_run: the net has " + std::to_string(g->n_in()) + " input(s) and " +
+                                   std::to_string(g->n_out()) + " output(s) (sn_run_multi)");
+    for (const void *p : io.in)
+        if (!p) return fail(SN_EINVAL, "sn_run: NULL input buffer");
+    for (void *p : io.out)
+        if (!p) return fail(SN_EINVAL, "sn_run: NULL output buffer");
+    if (!g->plan_valid) {
+        sn_status rc = build_plan(g, st);
+        if (rc != SN_OK) return rc;
+    }
+    sn_status rc = SN_OK;
+    if (g->opt_graph && st != nullptr) {
+        if (!g->gexec || g->gexec_in != io.in || g->gexec_out != io.out || g->gexec_stream != st) {
+            if (g->gexec) {
+                cudaGraphExecDestroy(g->gexec);
+                g->gexec = nullptr;
+            }
+            cudaGraph_t graph = nullptr;
+            SN_CUDA_TRY(cudaStreamBeginCapture(st, cudaStreamCaptureModeThreadLocal));
+            rc = run_plan(g, io, st, nullptr);
+            cudaError_t ce = cudaStreamEndCapture(st, &graph);
+            if (rc != SN_OK) {
+                if (graph) cudaGraphDestroy(graph);
+                return rc;
+            }
+            if (ce != cudaSuccess) return fail(SN_ECUDA, std::string("graph capture: ") + cudaGetErrorString(ce));
+            ce = cudaGraphInstantiate(&g->gexec, graph, 0);
+            cudaGraphDestroy(graph);
+            if (ce != cudaSuccess) {
+                g->gexec = nullptr;
+                return fail(SN_ECUDA, std::string("graph instantiate: ") + cudaGetErrorString(ce));
+            }
+            g->gexec_in = io.in;
+            g->gexec_out = io.out;
+            g->gexec_stream = st;
+        }
+        SN_CUDA_TRY(cudaGraphLaunch(g->gexec, st));
+    } else {
+        rc = run_plan(g, io, st, nullptr);
+        if (rc != SN_OK) return rc;
+    }
+    if (g->opt_check) return check_device(g, st);
+    return SN_OK;
+}
+
 sn_status sn_run(sn_graph *gg, const void *in_dev, void *out_dev, void *stream) {
     SN_GUARD({
         if (!gg || !in_dev || !out_dev) return fail(SN_EINVAL, "sn_run: NULL argument");
+        IoPtrs io;
+        io.in = {in_dev};
+        io.out = {out_dev};
+        return run_io(G(gg), io, static_cast<cudaStream_t>(stream));
+    })
+}
+
+sn_status sn_run_multi(sn_graph *gg, const void *const *in_devs, int32_t n_in, void *const *out_devs, int32_t n_out,
+                       void *stream) {
+    SN_GUARD({
+        if (!gg || !in_devs || !out_devs || n_in < 1 || n_out < 1) return fail(SN_EINVAL, "sn_run_multi: bad argument");
+        IoPtrs io;
+        io.in.assign(in_devs, in_devs + n_in);
+        io.out.assign(out_devs, out_devs + n_out);
+        return run_io(G(gg), io, static_cast<cudaStream_t>(stream));
+    })
+}
+
+sn_status sn_add_input(sn_graph *gg, const int64_t in_nchw[4], int32_t *input_id) {
+    SN_GUARD({
+        if (!gg || !in_nchw || !input_id) return fail(SN_EINVAL, "sn_add_input: NULL argument");
+        return add_input(G(gg), in_nchw, input_id);
+    })
+}
+
+sn_status sn_set_outputs(sn_graph *gg, const int32_t *layer_ids, int32_t n) {
+    SN_GUARD({
+        if (!gg) return fail(SN_EINVAL, "sn_set_outputs: NULL graph");
+        return set_outputs(G(gg), layer_ids, n);
+    })
+}
+
+sn_status sn_get_io(sn_graph *gg, int32_t *n_inputs, int32_t *n_outputs) {
+    SN_GUARD({
+        if (!gg) return fail(SN_EINVAL, "sn_get_io: NULL graph");
         Graph *g = G(gg);
-        if (!g->has_path) return fail(SN_ESTATE, "sn_run: select or set a routine path first");
-        cudaStream_t st = static_cast<cudaStream_t>(stream);
-        if (!g->plan_valid) {
-            sn_status rc = build_plan(g, st);
-            if (rc != SN_OK) return rc;
-        }
-        sn_status rc = SN_OK;
-        if (g->opt_graph && st != nullptr) {
-            if (!g->gexec || g->gexec_in != in_dev || g->gexec_out != out_dev || g->gexec_stream != st) {
-                if (g->gexec) {
-                    cudaGraphExecDestroy(g->gexec);
-                    g->gexec = nullptr;
-                }
-                cudaGraph_t graph = nullptr;
-                SN_CUDA_TRY(cudaStreamBeginCapture(st, cudaStreamCaptureModeThreadLocal));
-                rc = run_plan(g, in_dev, out_dev, st, nullptr);
-                cudaError_t ce = cudaStreamEndCapture(st, &graph);
-                if (rc != SN_OK) {
-                    if (graph) cudaGraphDestroy(graph);
-                    return rc;
-                }
-                if (ce != cudaSuccess) return fail(SN_ECUDA, std::string("graph capture: ") + cudaGetErrorString(ce));
-                ce = cudaGraphInstantiate(&g->gexec, graph, 0);
-                cudaGraphDestroy(graph);
-                if (ce != cudaSuccess) {
-                    g->gexec = nullptr;
-                    return fail(SN_ECUDA, std::string("graph instantiate: ") + cudaGetErrorString(ce));
-                }
-                g->gexec_in = in_dev;
-                g->gexec_out = out_dev;
-                g->gexec_stream = st;
-            }
-            SN_CUDA_TRY(cudaGraphLaunch(g->gexec, st));
-        } else {
-            rc = run_plan(g, in_dev, out_dev, st, nullptr);
-            if (rc != SN_OK) return rc;
-        }
-        if (g->opt_check) return check_device(g, st);
+        if (n_inputs) *n_inputs = g->n_in();
+        if (n_outputs) *n_outputs = g->n_out();
         return SN_OK;
     })
 }
@@ -351,8 +398,13 @@ sn_status sn_run_timed(sn_graph *gg, const void *in_dev, void *out_dev, void *st
             sn_status rc = build_plan(g, st);
             if (rc != SN_OK) return rc;
         }
+        if (g->n_in() != 1 || g->n_out() != 1)
+            return fail(SN_EINVAL, "sn_run_timed: the net has several inputs or outputs");
+        IoPtrs io;
+        io.in = {in_dev};
+        io.out = {out_dev};
         std::vector<float> op_ms;
-        sn_status rc = run_plan_timed(g, in_dev, out_dev, st, &op_ms);
+        sn_status rc = run_plan_timed(g, io, st, &op_ms);
         if (rc != SN_OK) return rc;
         if (layer_ms)
             for (int32_t i = 0; i < g->n_layers(); ++i) layer_ms[i] = 0.f;
@@ -560,9 +612,14 @@ sn_status sn_convert_q(const void *x_dev, sn_schema from, void *y_dev, sn_schema
 }
 
 static float *qscale_ref(Graph *g, int32_t id, bool internal) {
+    const int32_t m_in = g->n_in();
     if (id == -1) return internal ? &g->layers[0].qscale : &g->in_qscale;
+    if (id < -1 && id >= -m_in) {  // another net input
+        const int32_t k = -1 - id;
+        return internal ? &g->layers[k].qscale : &g->extra_in_qscale[k - 1];
+    }
     if (id < 0 || id >= (int32_t)g->user.size()) return nullptr;
-    return internal ? &g->layers[id + 1].qscale : &g->user[id].qscale;
+    return internal ? &g->layers[id + m_in].qscale : &g->user[id].qscale;
 }
 
 sn_status sn_set_qscale(sn_graph *gg, int32_t layer_id, float scale) {
@@ -598,11 +655,13 @@ sn_status sn_calibrate(sn_graph *gg, const void *in_dev, void *stream) {
         if (rc != SN_OK) return rc;
         if (g->in_schema.dtype == SN_QI8 || g->out_schema.dtype == SN_QI8)
             return fail(SN_EUNSUPPORTED, "sn_calibrate: the net input and output must be float");
+        if (g->n_in() != 1)
+            return fail(SN_EUNSUPPORTED, "sn_calibrate: nets with several inputs take their scales from sn_set_qscale");
         rc = calibrate(g, in_dev, static_cast<cudaStream_t>(stream));
         if (rc != SN_OK) return rc;
         // mirror into the layers as added
         g->in_qscale = g->layers[0].qscale;
-        for (size_t u = 0; u < g->user.size(); ++u) g->user[u].qscale = g->layers[u + 1].qscale;
+        for (size_t u = 0; u < g->user.size(); ++u) g->user[u].qscale = g->layers[u + g->n_in()].qscale;
         return SN_OK;
     })
 }

@@ -157,11 +157,20 @@ sn_status add_layer(Graph *g, int32_t type, const void *params, const int32_t *i
     Layer L;
     L.type = type;
     std::vector<Shape> in;
+    // internal indices: net input k (id -1 - k) is layer k, user layer u is
+    // layer u + (number of net inputs)
+    const int32_t m_in = 1 + (int32_t)g->extra_in.size();
     for (int32_t i = 0; i < n_inputs; ++i) {
         const int32_t id = inputs[i];
-        if (id < -1 || id >= (int32_t)g->user.size()) return fail(SN_EINVAL, "input id out of range");
-        L.inputs.push_back(id + 1);  // internal index
-        in.push_back(id < 0 ? g->in_shape : g->user[id].out);
+        if (id < -m_in || id >= (int32_t)g->user.size()) return fail(SN_EINVAL, "input id out of range");
+        if (id < 0) {
+            const int32_t k = -1 - id;
+            L.inputs.push_back(k);
+            in.push_back(k == 0 ? g->in_shape : g->extra_in[k - 1]);
+        } else {
+            L.inputs.push_back(id + m_in);
+            in.push_back(g->user[id].out);
+        }
     }
     int64_t wn = 0, bn = 0;
     switch (type) {
@@ -212,20 +221,63 @@ sn_status add_layer(Graph *g, int32_t type, const void *params, const int32_t *i
 // ---------------------------------------------------------------------------
 // finalisation: internal layers, edges, candidates
 // ---------------------------------------------------------------------------
+sn_status add_input(Graph *g, const int64_t nchw[4], int32_t *id) {
+    if (g->finalized) return fail(SN_ESTATE, "net already finalised");
+    if (!g->user.empty()) return fail(SN_ESTATE, "declare every net input before the first layer");
+    for (int k = 0; k < 4; ++k)
+        if (nchw[k] < 1) return fail(SN_EINVAL, "input extents must be >= 1");
+    g->extra_in.push_back(Shape{nchw[0], nchw[1], nchw[2], nchw[3]});
+    g->extra_in_qscale.push_back(0.0f);
+    *id = -1 - (int32_t)g->extra_in.size();
+    return SN_OK;
+}
+
+sn_status set_outputs(Graph *g, const int32_t *ids, int32_t n) {
+    if (g->finalized) return fail(SN_ESTATE, "net already finalised");
+    if (n < 1 || !ids) return fail(SN_EINVAL, "at least one output");
+    std::vector<int32_t> v;
+    for (int32_t i = 0; i < n; ++i) {
+        if (ids[i] < 0 || ids[i] >= (int32_t)g->user.size()) return fail(SN_EINVAL, "output id out of range");
+        for (int32_t u : v)
+            if (u == ids[i]) return fail(SN_EINVAL, "duplicate output id");
+        v.push_back(ids[i]);
+    }
+    g->outputs = v;
+    return SN_OK;
+}
+
 sn_status graph_finalize(Graph *g) {
     if (g->finalized) return SN_OK;
     const int32_t m = (int32_t)g->user.size();
+    const int32_t m_in = g->n_in();
+    if (g->outputs.empty() && m > 0) g->outputs = {m - 1};
     std::vector<Layer> L;
     Layer in_l;
     in_l.type = -1;
     in_l.out = g->in_shape;
     in_l.qscale = g->in_qscale;
     L.push_back(in_l);
+    // the other net inputs: input layers fed by the auxiliary input layer 0
+    // (section IV-E), one zero-cost routine each
+    for (size_t k = 0; k < g->extra_in.size(); ++k) {
+        Layer x;
+        x.type = -3;
+        x.inputs = {0};
+        x.out = g->extra_in[k];
+        x.qscale = g->extra_in_qscale[k];
+        L.push_back(x);
+    }
     for (auto &u : g->user) L.push_back(u);
+    // the auxiliary output layer merges every net output
     Layer out_l;
     out_l.type = -2;
-    out_l.inputs = {m};  // last user layer (internal index m), or the input when m == 0
-    out_l.out = m ? g->user[m - 1].out : g->in_shape;
+    if (m == 0) {
+        out_l.inputs = {0};
+        out_l.out = g->in_shape;
+    } else {
+        for (int32_t u : g->outputs) out_l.inputs.push_back(u + m_in);
+        out_l.out = g->user[g->outputs[0]].out;
+    }
     L.push_back(out_l);
     const int32_t n = (int32_t)L.size();
 
@@ -237,8 +289,9 @@ sn_status graph_finalize(Graph *g) {
             for (int32_t j : L[i].inputs) reach[j] = 1;
     for (int32_t i = 0; i < n; ++i)
         if (!reach[i])
-            return fail(SN_EINVAL, "layer " + std::to_string(i - 1) +
-                                       " does not reach the net output (net must be 1-in-1-out)");
+            return fail(SN_EINVAL, (L[i].type == -3 ? "net input " + std::to_string(i) + " feeds no layer"
+                                                    : "layer " + std::to_string(i - m_in) +
+                                                          " does not reach a net output (every layer must feed one)"));
 
     std::vector<std::pair<int32_t, int32_t>> edges;
     for (int32_t i = 0; i < n; ++i)
@@ -248,8 +301,8 @@ sn_status graph_finalize(Graph *g) {
     std::vector<int32_t> begin(n + 1, 0);
     for (int32_t i = 0; i < n; ++i) {
         begin[i] = (int32_t)cands.size();
-        if (i == 0) {
-            cands.push_back({R_IO, 0, g->in_schema_idx, 0, 0});
+        if (i == 0 || L[i].type == -3) {  // net inputs: the caller's buffers, in in_schema
+            cands.push_back({R_IO, 0, g->in_schema_idx, i, 0});
             continue;
         }
         if (i == n - 1) {
@@ -266,7 +319,7 @@ sn_status graph_finalize(Graph *g) {
             }
         }
         if ((int32_t)cands.size() == begin[i])
-            return fail(SN_EINFEASIBLE, "layer " + std::to_string(i - 1) +
+            return fail(SN_EINFEASIBLE, "layer " + std::to_string(i - m_in) +
                                             " has no routine in any schema of Lambda");
     }
     begin[n] = (int32_t)cands.size();

@@ -47,16 +47,27 @@ sn_status build_plan(Graph *g, cudaStream_t st) {
     g->slot_schema.clear();
     g->slot_qscale.clear();
     const int32_t n = g->n_layers();
+    const int32_t m_in = g->n_in();
+    const Layer &OL = g->layers[n - 1];  // auxiliary output layer: its inputs are the net outputs
+    const int32_t m_out = (int32_t)OL.inputs.size();
     std::vector<sn_schema> sch(n);
     for (int32_t i = 0; i < n; ++i) sch[i] = g->schemas[g->cands[g->path_cand[i]].schema];
-    schema_slot(g, g->in_shape, g->in_schema, g->layers[0].qscale);  // slot 0: caller's input
-    schema_slot(g, g->layers[n - 1].out, g->out_schema,
-                g->layers[g->layers[n - 1].inputs[0]].qscale);         // slot 1: caller's output
+    // external slots: the caller's input buffers 0..m_in-1, then its output
+    // buffers m_in..m_in+m_out-1
+    for (int32_t k = 0; k < m_in; ++k) schema_slot(g, g->layers[k].out, g->in_schema, g->layers[k].qscale);
+    for (int32_t q = 0; q < m_out; ++q) {
+        const Layer &src = g->layers[OL.inputs[q]];
+        schema_slot(g, src.out, g->out_schema, src.qscale);
+    }
+    g->n_ext = m_in + m_out;
     std::vector<int32_t> out_slot(n, -1);
-    out_slot[0] = 0;
-    const int32_t last = n - 2;  // last user layer (0 if none)
+    for (int32_t k = 0; k < m_in; ++k) out_slot[k] = k;
+    // output index of each layer that is a net output (-1 otherwise)
+    std::vector<int32_t> out_index(n, -1);
+    for (int32_t q = 0; q < m_out; ++q)
+        if (OL.inputs[q] >= m_in) out_index[OL.inputs[q]] = q;
     size_t ws = 0;
-    for (int32_t i = 1; i < n; ++i) {
+    for (int32_t i = m_in; i < n; ++i) {
         const Layer &L = g->layers[i];
         PlanOp op;
         op.kind = PlanOp::LAYER;
@@ -80,15 +91,15 @@ sn_status build_plan(Graph *g, cudaStream_t st) {
             int32_t src = out_slot[j];
             const bool same = schema_eq(sch[j], sch[i]);
             if (i == n - 1) {
-                // output layer: adapt into the caller's buffer unless the last
-                // layer already wrote there
-                if (!same || j == 0) {
+                // output layer: adapt into the caller's buffer unless the
+                // producer already wrote there
+                if (!same || out_slot[j] != m_in + (int32_t)k) {
                     PlanOp a;
                     a.kind = PlanOp::ADAPT;
                     a.layer = i;
                     a.edge = e;
                     a.in_slots = {src};
-                    a.out_slot = 1;
+                    a.out_slot = m_in + (int32_t)k;
                     g->plan.push_back(a);
                 }
                 continue;
@@ -107,8 +118,8 @@ sn_status build_plan(Graph *g, cudaStream_t st) {
             op.in_slots.push_back(src);
         }
         if (i == n - 1) break;
-        if (i == last && schema_eq(sch[i], g->out_schema)) {
-            op.out_slot = 1;
+        if (out_index[i] >= 0 && schema_eq(sch[i], g->out_schema)) {
+            op.out_slot = m_in + out_index[i];  // a net output written in place
         } else {
             schema_slot(g, L.out, sch[i], L.qscale);
             op.out_slot = (int32_t)g->slots.size() - 1;
@@ -131,7 +142,7 @@ sn_status build_plan(Graph *g, cudaStream_t st) {
             return fail(SN_ESTATE, "the path keeps a blob in qi8 without a scale (sn_set_qscale or sn_calibrate)");
         }
     }
-    for (size_t s = 2; s < g->slots.size(); ++s) {
+    for (size_t s = g->n_ext; s < g->slots.size(); ++s) {
         const size_t bytes = (size_t)g->slot_shape[s].numel() * dtype_size(g->slot_schema[s].dtype);
         sn_status rc = dev_alloc(g, bytes, &g->slots[s]);
         if (rc != SN_OK) return rc;
@@ -145,11 +156,11 @@ sn_status build_plan(Graph *g, cudaStream_t st) {
     return SN_OK;
 }
 
-static sn_status launch_op(Graph *g, const PlanOp &op, const void *in, void *out,
-                           cudaStream_t st) {
+static sn_status launch_op(Graph *g, const PlanOp &op, const IoPtrs &io, cudaStream_t st) {
+    const int32_t m_in = (int32_t)io.in.size();
     auto ptr = [&](int32_t s) -> void * {
-        if (s == 0) return const_cast<void *>(in);
-        if (s == 1) return out;
+        if (s < m_in) return const_cast<void *>(io.in[s]);
+        if (s < g->n_ext) return io.out[s - m_in];
         return g->slots[s].ptr;
     };
     if (op.kind == PlanOp::ADAPT) {
@@ -183,16 +194,17 @@ static sn_status launch_op(Graph *g, const PlanOp &op, const void *in, void *out
     return launch_routine(a);
 }
 
-sn_status run_plan(Graph *g, const void *in, void *out, cudaStream_t st,
-                   std::vector<cudaEvent_t> *evs) {
+sn_status run_plan(Graph *g, const IoPtrs &io, cudaStream_t st, std::vector<cudaEvent_t> *evs) {
     if (!g->plan_valid) {
         sn_status rc = build_plan(g, st);
         if (rc != SN_OK) return rc;
     }
+    if ((int32_t)(io.in.size() + io.out.size()) != g->n_ext || (int32_t)io.in.size() != g->n_in())
+        return fail(SN_EINVAL, "run: wrong number of input or output buffers");
     for (size_t i = 0; i < g->plan.size(); ++i) {
         // external records: timing nodes when the stream is being captured
         if (evs) SN_CUDA_TRY(cudaEventRecordWithFlags((*evs)[2 * i], st, cudaEventRecordExternal));
-        sn_status rc = launch_op(g, g->plan[i], in, out, st);
+        sn_status rc = launch_op(g, g->plan[i], io, st);
         if (rc != SN_OK) return rc;
         if (evs) SN_CUDA_TRY(cudaEventRecordWithFlags((*evs)[2 * i + 1], st, cudaEventRecordExternal));
     }
@@ -297,7 +309,7 @@ std::string signature(const Graph *g, int32_t i, const Candidate &c) {
 
 }  // namespace
 
-sn_status run_plan_timed(Graph *g, const void *in, void *out, cudaStream_t user, std::vector<float> *op_ms) {
+sn_status run_plan_timed(Graph *g, const IoPtrs &io, cudaStream_t user, std::vector<float> *op_ms) {
     if (!g->plan_valid) {
         sn_status rc = build_plan(g, user);
         if (rc != SN_OK) return rc;
@@ -308,8 +320,8 @@ sn_status run_plan_timed(Graph *g, const void *in, void *out, cudaStream_t user,
     std::vector<cudaEvent_t> evs(2 * g->plan.size());
     for (auto &e : evs) cudaEventCreate(&e);
     cudaGraphExec_t exec = nullptr;
-    sn_status rc = run_plan(g, in, out, st, nullptr);  // first-use set-up outside the capture
-    if (rc == SN_OK) rc = capture_graph(st, [&]() { return run_plan(g, in, out, st, &evs); }, &exec);
+    sn_status rc = run_plan(g, io, st, nullptr);  // first-use set-up outside the capture
+    if (rc == SN_OK) rc = capture_graph(st, [&]() { return run_plan(g, io, st, &evs); }, &exec);
     if (rc == SN_OK && cudaGraphLaunch(exec, st) != cudaSuccess) rc = fail(SN_ECUDA, "timed run: replay failed");
     if (cudaStreamSynchronize(st) != cudaSuccess && rc == SN_OK) rc = fail(SN_ECUDA, "timed run: stream failed");
     if (rc == SN_OK) {
@@ -362,6 +374,7 @@ static sn_status profile_graph_on(Graph *g, const sn_profile_opts &o, cudaStream
     // --- unit profiling of layer routines ---
     for (int32_t i = 1; i < n - 1 && rc == SN_OK; ++i) {
         const Layer &L = g->layers[i];
+        if (L.type < 0) continue;  // a net input layer: its one routine is the caller's buffer
         std::vector<Shape> in;
         for (int32_t j : L.inputs) in.push_back(g->layers[j].out);
         for (int32_t c = g->cand_begin[i]; c < g->cand_begin[i + 1] && rc == SN_OK; ++c) {
@@ -465,15 +478,32 @@ static sn_status profile_graph_on(Graph *g, const sn_profile_opts &o, cudaStream
                 return g->cands[x].cost < g->cands[y].cost;
             });
     }
-    Buffer xin, xout;
-    if ((rc = dev_alloc(g, (size_t)g->in_shape.numel() * dtype_size(g->in_schema.dtype), &xin)) != SN_OK)
-        return rc;
-    if ((rc = dev_alloc(g, (size_t)g->layers[n - 1].out.numel() * dtype_size(g->out_schema.dtype), &xout)) !=
-        SN_OK) {
-        dev_free(g, &xin);
+    // scratch net inputs (filled) and outputs
+    std::vector<Buffer> xbufs;
+    IoPtrs io;
+    auto free_io = [&]() {
+        for (auto &b : xbufs) dev_free(g, &b);
+    };
+    for (int32_t k = 0; k < g->n_in() && rc == SN_OK; ++k) {
+        Buffer b;
+        const Shape &sh = g->layers[k].out;
+        if ((rc = dev_alloc(g, (size_t)sh.numel() * dtype_size(g->in_schema.dtype), &b)) != SN_OK) break;
+        xbufs.push_back(b);
+        io.in.push_back(b.ptr);
+        k::fill_pattern(b.ptr, g->in_schema.dtype, sh.numel(), 5u + k, 1.0f, st);
+    }
+    for (int32_t j : g->layers[n - 1].inputs) {
+        if (rc != SN_OK) break;
+        Buffer b;
+        if ((rc = dev_alloc(g, (size_t)g->layers[j].out.numel() * dtype_size(g->out_schema.dtype), &b)) != SN_OK)
+            break;
+        xbufs.push_back(b);
+        io.out.push_back(b.ptr);
+    }
+    if (rc != SN_OK) {
+        free_io();
         return rc;
     }
-    k::fill_pattern(xin.ptr, g->in_schema.dtype, g->in_shape.numel(), 5u, 1.0f, st);
     std::vector<std::vector<float>> insitu(g->cands.size());
     for (int32_t lam = 0; lam < g->n_lambda && rc == SN_OK; ++lam) {
         for (int32_t r = 0; r < o.topk && rc == SN_OK; ++r) {
@@ -501,11 +531,11 @@ static sn_status profile_graph_on(Graph *g, const sn_profile_opts &o, cudaStream
             for (auto &e : evs) cudaEventCreate(&e);
             std::vector<std::vector<float>> per_op(g->plan.size());
             for (int32_t w = 0; w < std::max(o.warmup, 1) && rc == SN_OK; ++w)
-                rc = run_plan(g, xin.ptr, xout.ptr, st, nullptr);
+                rc = run_plan(g, io, st, nullptr);
             // the whole net with a timing node around every op, replayed
             cudaGraphExec_t exec = nullptr;
             if (rc == SN_OK)
-                rc = capture_graph(st, [&]() { return run_plan(g, xin.ptr, xout.ptr, st, &evs); }, &exec);
+                rc = capture_graph(st, [&]() { return run_plan(g, io, st, &evs); }, &exec);
             for (int32_t p = 0; p < o.passes && rc == SN_OK; ++p) {
                 if (cudaGraphLaunch(exec, st) != cudaSuccess) {
                     rc = fail(SN_ECUDA, "integrated profiling: replay failed");
@@ -533,8 +563,7 @@ static sn_status profile_graph_on(Graph *g, const sn_profile_opts &o, cudaStream
             }
         }
     }
-    dev_free(g, &xin);
-    dev_free(g, &xout);
+    free_io();
     // in-situ medians replace the unit times of the re-timed candidates; the
     // candidates of the same (layer, schema) that were not re-timed keep their
     // unit ranking, moved to the in-situ scale by the best candidate's ratio
@@ -591,9 +620,10 @@ sn_status calibrate(Graph *g, const void *in, cudaStream_t st) {
     const int64_t saved_total = g->path_total;
     g->path_cand = pc;
     g->has_path = true;
-    Buffer out, dmax;
+    std::vector<Buffer> outs;
+    Buffer dmax;
     auto finish = [&](sn_status r) {
-        dev_free(g, &out);
+        for (auto &b : outs) dev_free(g, &b);
         dev_free(g, &dmax);
         g->has_path = had_path;
         g->path_cand = saved_path;
@@ -602,18 +632,25 @@ sn_status calibrate(Graph *g, const void *in, cudaStream_t st) {
         return r;
     };
     if ((rc = build_plan(g, st)) != SN_OK) return finish(rc);
-    if ((rc = dev_alloc(g, (size_t)g->layers[n - 1].out.numel() * dtype_size(g->out_schema.dtype), &out)) != SN_OK)
-        return finish(rc);
+    IoPtrs io;
+    io.in.push_back(in);
+    for (int32_t j : g->layers[n - 1].inputs) {
+        Buffer b;
+        if ((rc = dev_alloc(g, (size_t)g->layers[j].out.numel() * dtype_size(g->out_schema.dtype), &b)) != SN_OK)
+            return finish(rc);
+        outs.push_back(b);
+        io.out.push_back(b.ptr);
+    }
     if ((rc = dev_alloc(g, (size_t)n * sizeof(unsigned), &dmax)) != SN_OK) return finish(rc);
     unsigned *dm = static_cast<unsigned *>(dmax.ptr);
     if (cudaMemsetAsync(dm, 0, (size_t)n * sizeof(unsigned), st) != cudaSuccess ||
         k::absmax(in, g->in_schema.dtype, g->in_shape.numel(), dm, st) != cudaSuccess)
         return finish(fail(SN_ECUDA, "sn_calibrate: input reduction failed"));
     for (const PlanOp &op : g->plan) {
-        if ((rc = launch_op(g, op, in, out.ptr, st)) != SN_OK) return finish(rc);
+        if ((rc = launch_op(g, op, io, st)) != SN_OK) return finish(rc);
         if (op.kind != PlanOp::LAYER) continue;
         const int32_t so = op.out_slot;
-        const void *y = so == 1 ? out.ptr : g->slots[so].ptr;
+        const void *y = so < 1 ? in : so < g->n_ext ? io.out[so - 1] : g->slots[so].ptr;
         if (k::absmax(y, g->slot_schema[so].dtype, g->slot_shape[so].numel(), dm + op.layer, st) != cudaSuccess)
             return finish(fail(SN_ECUDA, "sn_calibrate: reduction failed"));
     }

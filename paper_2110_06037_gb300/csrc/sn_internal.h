@@ -150,6 +150,9 @@ struct Graph {
     void *alloc_ctx = nullptr;
 
     float in_qscale = 0.0f;           // qint8 scale of the net input (0 = not set)
+    std::vector<Shape> extra_in;      // net inputs 1.. (section IV-E: several input layers)
+    std::vector<float> extra_in_qscale;
+    std::vector<int32_t> outputs;     // user ids of the net outputs (default: the last layer)
     std::vector<Layer> user;          // as added
     bool finalized = false;
     std::vector<Layer> layers;        // internal: [input, user..., output]
@@ -169,18 +172,21 @@ struct Graph {
     std::vector<Shape> slot_shape;
     std::vector<sn_schema> slot_schema;
     std::vector<float> slot_qscale;   // qint8 scale of the blob a slot holds
+    int32_t n_ext = 2;                // slots [0, n_ext) are the caller's: inputs, then outputs
     std::map<std::string, Buffer> weight_cache;  // key: layer/format/dtype
     std::map<int32_t, Buffer> bias_cache;        // per layer fp32 bias
     Buffer workspace;
     int opt_graph = 0, opt_check = 0;
     bool profiling = false;           // plans built while profiling may lack qint8 scales
     cudaGraphExec_t gexec = nullptr;
-    const void *gexec_in = nullptr;
-    void *gexec_out = nullptr;
+    std::vector<const void *> gexec_in;
+    std::vector<void *> gexec_out;
     cudaStream_t gexec_stream = nullptr;
 
     ~Graph();
     int32_t n_layers() const { return (int32_t)layers.size(); }
+    int32_t n_in() const { return 1 + (int32_t)extra_in.size(); }
+    int32_t n_out() const { return outputs.empty() ? 1 : (int32_t)outputs.size(); }
     int32_t n_schemas() const { return (int32_t)schemas.size(); }
     int64_t &adapt(int32_t e, int32_t a, int32_t b) {
         return adapt_cost[((size_t)e * schemas.size() + a) * schemas.size() + b];
@@ -191,6 +197,14 @@ struct Graph {
 };
 
 sn_status graph_finalize(Graph *g);
+sn_status add_input(Graph *g, const int64_t nchw[4], int32_t *id);
+sn_status set_outputs(Graph *g, const int32_t *ids, int32_t n);
+
+// the caller's buffers of one run: net inputs in in_schema, outputs in out_schema
+struct IoPtrs {
+    std::vector<const void *> in;
+    std::vector<void *> out;
+};
 sn_status dev_alloc(Graph *g, size_t bytes, Buffer *b);
 void dev_free(Graph *g, Buffer *b);
 void invalidate_plan(Graph *g);
@@ -216,11 +230,11 @@ void fastest_per_schema(const Graph &g, std::vector<int64_t> &F, std::vector<int
 
 // plan + run
 sn_status build_plan(Graph *g, cudaStream_t st);
-sn_status run_plan(Graph *g, const void *in, void *out, cudaStream_t st,
+sn_status run_plan(Graph *g, const IoPtrs &io, cudaStream_t st,
                    std::vector<cudaEvent_t> *evs);
 // one run of the plan replayed from a CUDA graph with a timing node around
 // every op (device time of each op, no host launch cost); op_ms[q] in ms
-sn_status run_plan_timed(Graph *g, const void *in, void *out, cudaStream_t st, std::vector<float> *op_ms);
+sn_status run_plan_timed(Graph *g, const IoPtrs &io, cudaStream_t st, std::vector<float> *op_ms);
 sn_status profile_graph(Graph *g, const sn_profile_opts &o, cudaStream_t st);
 // qint8 calibration: run the fastest float-schema path, set every blob's scale
 // to max |x| / 127

@@ -1,7 +1,7 @@
 """Build a Graph from the plain-data net description (list of layer dicts).
 
 Each dict has 'type' (conv2 | dwconv2 | maxpool | gap | add | dense),
-'inputs' (earlier layer indices, -1 = net input), 'params', and for conv and
+'inputs' (earlier layer indices; -1, -2, ... = net inputs), 'params', and for conv and
 dense layers 'weight' (fp32, conv [K][C/groups][R][S], dense [out][in]) and
 'bias'.  Layer i of the list becomes layer id i of the graph.
 """
@@ -14,12 +14,19 @@ TYPES = {"conv2": _sn.SN_L_CONV2, "dwconv2": _sn.SN_L_DWCONV2, "maxpool": _sn.SN
          "gap": _sn.SN_L_GAP, "add": _sn.SN_L_ADD, "dense": _sn.SN_L_DENSE, "mul": _sn.SN_L_MUL}
 
 
-def build_graph(layers, in_shape, in_schema, out_schema, schemas, torch_alloc=True) -> Graph:
+def build_graph(layers, in_shape, in_schema, out_schema, schemas, torch_alloc=True, extra_inputs=(),
+                outputs=None) -> Graph:
+    """extra_inputs: shapes of net inputs -2, -3, ...; outputs: layer indices
+    of the net outputs (default: the last layer)."""
     g = Graph(in_shape, in_schema, out_schema, schemas, torch_alloc=torch_alloc)
+    for k, shp in enumerate(extra_inputs):
+        assert g.add_input(shp) == -2 - k
     for i, l in enumerate(layers):
         lid = g.add_layer(TYPES[l["type"]], l.get("params"), tuple(l["inputs"]), l.get("weight"),
                           l.get("bias"))
         assert lid == i
+    if outputs is not None:
+        g.set_outputs(list(outputs))
     return g
 
 
