@@ -554,6 +554,64 @@ __global__ void __launch_bounds__(256, 2) dw_nhwc_vec(const T *__restrict__ x, c
     }
     for (int rowi = blockIdx.y; rowi < d.N * d.P; rowi += gridDim.y) {
         const int n = rowi / d.P, p = rowi - n * d.P;
+        if constexpr (std::is_same<T, __half>::value && SW > 0) {
+            // fp16 3x3: packed half2 multiply-adds accumulating in fp16, in the
+            // same order as the ring kernel (bias, rows, columns)
+            __half2 hacc[QB][4];
+#pragma unroll
+            for (int j = 0; j < QB; ++j)
+#pragma unroll
+                for (int k = 0; k < 4; ++k) hacc[j][k] = __floats2half2_rn(b[2 * k], b[2 * k + 1]);
+            constexpr int WN = (QB - 1) * SW + 3;
+            const int wbase = q0 * SW - d.pw;
+#pragma unroll
+            for (int r = 0; r < 3; ++r) {
+                const int h = p * d.sh - d.ph + r * d.dh;
+                if (h < 0 || h >= d.H) continue;
+                const T *xrow = x + (((int64_t)n * d.H + h) * d.W) * d.C + c0;
+                uint4 win[WN];
+#pragma unroll
+                for (int t = 0; t < WN; ++t) {
+                    const int ww = wbase + t;
+                    win[t] = (ww >= 0 && ww < d.W) ? *reinterpret_cast<const uint4 *>(xrow + (int64_t)ww * d.C)
+                                                    : make_uint4(0u, 0u, 0u, 0u);
+                }
+#pragma unroll
+                for (int s = 0; s < 3; ++s) {
+                    const uint4 wq4 = *reinterpret_cast<const uint4 *>(w + (int64_t)(r * 3 + s) * d.C + c0);
+                    const __half2 *wq = reinterpret_cast<const __half2 *>(&wq4);
+#pragma unroll
+                    for (int j = 0; j < QB; ++j) {
+                        const __half2 *xv = reinterpret_cast<const __half2 *>(&win[j * SW + s]);
+#pragma unroll
+                        for (int k = 0; k < 4; ++k) hacc[j][k] = __hfma2(xv[k], wq[k], hacc[j][k]);
+                    }
+                }
+            }
+            T *yrow = y + ((int64_t)rowi * d.Q) * d.C + c0;
+            const __half2 z2 = __float2half2_rn(0.0f), six2 = __float2half2_rn(6.0f);
+#pragma unroll
+            for (int j = 0; j < QB; ++j) {
+                if (q0 + j >= d.Q) break;
+                uint4 o;
+                __half2 *oh = reinterpret_cast<__half2 *>(&o);
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    __half2 v = hacc[j][k];
+                    if (d.act == SN_ACT_RELU) {
+                        v = __hmax2(v, z2);
+                    } else if (d.act == SN_ACT_RELU6) {
+                        v = __hmin2(__hmax2(v, z2), six2);
+                    } else if (d.act != SN_ACT_NONE) {
+                        const float2 f = __half22float2(v);
+                        v = __floats2half2_rn(act_apply(f.x, d.act), act_apply(f.y, d.act));
+                    }
+                    oh[k] = v;
+                }
+                *reinterpret_cast<uint4 *>(yrow + (int64_t)(q0 + j) * d.C) = o;
+            }
+            continue;
+        }
         float acc[QB][E];
 #pragma unroll
         for (int j = 0; j < QB; ++j)

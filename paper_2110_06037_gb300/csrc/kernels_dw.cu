@@ -13,6 +13,7 @@
 // so the kernel reads the input about once and writes the output once: the
 // HBM floor of the operation.
 #include <algorithm>
+#include <type_traits>
 
 #include "tc_common.cuh"
 
@@ -154,6 +155,68 @@ __global__ void __launch_bounds__(DW_THREADS, 1)
                 const int cl = (rem - qb * p.CVS) * E;  // channel within the slice
                 const int c0 = s.sl * p.CS + cl;
                 const int pp = s.pA + j, q0 = qb * QB;
+                uint4 wt[9];  // the item's nine taps, fetched together
+#pragma unroll
+                for (int t = 0; t < 9; ++t) wt[t] = *reinterpret_cast<const uint4 *>(w + t * p.C + c0);
+                T *yrow = y + ((int64_t)(s.n * p.P + pp) * p.Q) * p.C + c0;
+                if constexpr (std::is_same<T, __half>::value) {
+                    // fp16: packed half2 multiply-adds (two channels per
+                    // instruction) accumulating in fp16, half the issue slots
+                    // of the widening fp32 path
+                    const float4 b0 = *reinterpret_cast<const float4 *>(p.bias + c0);
+                    const float4 b1 = *reinterpret_cast<const float4 *>(p.bias + c0 + 4);
+                    const __half2 hb[4] = {__floats2half2_rn(b0.x, b0.y), __floats2half2_rn(b0.z, b0.w),
+                                           __floats2half2_rn(b1.x, b1.y), __floats2half2_rn(b1.z, b1.w)};
+                    __half2 hacc[QB][4];
+#pragma unroll
+                    for (int q = 0; q < QB; ++q)
+#pragma unroll
+                        for (int k = 0; k < 4; ++k) hacc[q][k] = hb[k];
+#pragma unroll
+                    for (int r = 0; r < 3; ++r) {
+                        const int h = pp * SW - p.ph + r;
+                        if (h < s.hlo || h >= s.hhi) continue;  // zero padding
+                        const T *row = ringT + slot_of(L + (h - s.hlo), p) * slot_elems + cl;
+                        uint4 win[WN];
+#pragma unroll
+                        for (int t = 0; t < WN; ++t) {
+                            const int col = q0 * SW + t;
+                            win[t] = col < p.WB ? *reinterpret_cast<const uint4 *>(row + col * p.CS)
+                                                : make_uint4(0u, 0u, 0u, 0u);
+                        }
+#pragma unroll
+                        for (int sx = 0; sx < 3; ++sx) {
+                            const __half2 *wq = reinterpret_cast<const __half2 *>(&wt[r * 3 + sx]);
+#pragma unroll
+                            for (int q = 0; q < QB; ++q) {
+                                const __half2 *xv = reinterpret_cast<const __half2 *>(&win[q * SW + sx]);
+#pragma unroll
+                                for (int k = 0; k < 4; ++k) hacc[q][k] = __hfma2(xv[k], wq[k], hacc[q][k]);
+                            }
+                        }
+                    }
+                    const __half2 z2 = __float2half2_rn(0.0f), six2 = __float2half2_rn(6.0f);
+#pragma unroll
+                    for (int q = 0; q < QB; ++q) {
+                        if (q0 + q >= p.Q) break;
+                        uint4 o;
+                        __half2 *oh = reinterpret_cast<__half2 *>(&o);
+#pragma unroll
+                        for (int k = 0; k < 4; ++k) {
+                            __half2 v = hacc[q][k];
+                            if (p.act == SN_ACT_RELU) {
+                                v = __hmax2(v, z2);
+                            } else if (p.act == SN_ACT_RELU6) {
+                                v = __hmin2(__hmax2(v, z2), six2);
+                            } else if (p.act != SN_ACT_NONE) {
+                                const float2 f = __half22float2(v);
+                                v = __floats2half2_rn(act_apply(f.x, p.act), act_apply(f.y, p.act));
+                            }
+                            oh[k] = v;
+                        }
+                        *reinterpret_cast<uint4 *>(yrow + (int64_t)(q0 + q) * p.C) = o;
+                    }
+                } else {
                 float acc[QB][E];
                 {
                     const float4 b0 = *reinterpret_cast<const float4 *>(p.bias + c0);
@@ -164,9 +227,6 @@ __global__ void __launch_bounds__(DW_THREADS, 1)
 #pragma unroll
                         for (int e = 0; e < E; ++e) acc[q][e] = bb[e];
                 }
-                uint4 wt[9];  // the item's nine taps, fetched together
-#pragma unroll
-                for (int t = 0; t < 9; ++t) wt[t] = *reinterpret_cast<const uint4 *>(w + t * p.C + c0);
 #pragma unroll
                 for (int r = 0; r < 3; ++r) {
                     const int h = pp * SW - p.ph + r;
@@ -192,7 +252,6 @@ __global__ void __launch_bounds__(DW_THREADS, 1)
                         }
                     }
                 }
-                T *yrow = y + ((int64_t)(s.n * p.P + pp) * p.Q) * p.C + c0;
 #pragma unroll
                 for (int q = 0; q < QB; ++q) {
                     if (q0 + q >= p.Q) break;
@@ -203,6 +262,7 @@ __global__ void __launch_bounds__(DW_THREADS, 1)
                     o.w = tc::pack2<T>(act_apply(acc[q][6], p.act), act_apply(acc[q][7], p.act));
                     *reinterpret_cast<uint4 *>(yrow + (int64_t)(q0 + q) * p.C) = o;
                 }
+                }  // fp32-accumulating path
             }
             // rows below the next round's first input row are done with
             const int nrow = base + DW_CONSUMERS < total

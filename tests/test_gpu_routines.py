@@ -111,8 +111,9 @@ def test_depthwise(case, schema):
         assert maxrel(got, ref) <= TOL[schema[0]], v
         outs.append(got)
     if schema[1] == "nhwc" and schema[0] != "f32":
-        # both NHWC kernels accumulate the nine taps in f32 in the same order
-        # (bias, then rows, then columns) with exact products: equal results
+        # both NHWC kernels accumulate the nine taps in the same order (bias,
+        # then rows, then columns): in f32 with exact products for bf16, in
+        # packed half2 for f16: equal results
         assert np.array_equal(outs[0], outs[1])
 
 
