@@ -342,7 +342,11 @@ __global__ void wino_output_kernel(const float *__restrict__ Mx, const float *__
     }
 }
 
-cudaError_t conv_wino(const LaunchArgs &a) {
+cudaError_t conv_wino(const LaunchArgs &a) { return conv_wino_stage(a, -1); }
+
+// stage 0: input transform (wgenc); 1: element-wise GEMMs (wgconv); 2: output
+// transform (wgdec); -1: all three
+cudaError_t conv_wino_stage(const LaunchArgs &a, int stage) {
     const ConvDims d = conv_dims(a);
     const WinoDims wd = wino_dims(d);
     const size_t need = (size_t)16 * wd.T * (d.C + d.K) * sizeof(float);
@@ -352,15 +356,21 @@ cudaError_t conv_wino(const LaunchArgs &a) {
     dim3 ggrid((unsigned)((wd.T + 63) / 64), (unsigned)((d.K + 63) / 64), 16);
     if (ggrid.y > 65535) return cudaErrorInvalidValue;
     SN_DT_SWITCH(a.schema.dtype, T, {
-        if (a.schema.layout == SN_NHWC)
-            launch_pdl(wino_input_kernel<T, true>, grid_for(wd.T * d.C, 256), 256, 0, a.stream, (const T *)a.in[0], V, wd);
-        else
-            launch_pdl(wino_input_kernel<T, false>, grid_for(wd.T * d.C, 256), 256, 0, a.stream, (const T *)a.in[0], V, wd);
-        launch_pdl(gemm_nt_simt<T>, ggrid, 256, 0, a.stream, V, (const T *)a.wt, Mx, wd.T, d.K, d.C);
-        if (a.schema.layout == SN_NHWC)
-            launch_pdl(wino_output_kernel<T, true>, grid_for(wd.T * d.K, 256), 256, 0, a.stream, Mx, a.bias, (T *)a.out, wd);
-        else
-            launch_pdl(wino_output_kernel<T, false>, grid_for(wd.T * d.K, 256), 256, 0, a.stream, Mx, a.bias, (T *)a.out, wd);
+        if (stage < 0 || stage == 0) {
+            if (a.schema.layout == SN_NHWC)
+                launch_pdl(wino_input_kernel<T, true>, grid_for(wd.T * d.C, 256), 256, 0, a.stream, (const T *)a.in[0], V, wd);
+            else
+                launch_pdl(wino_input_kernel<T, false>, grid_for(wd.T * d.C, 256), 256, 0, a.stream, (const T *)a.in[0], V, wd);
+        }
+        if (stage < 0 || stage == 1) {
+            launch_pdl(gemm_nt_simt<T>, ggrid, 256, 0, a.stream, V, (const T *)a.wt, Mx, wd.T, d.K, d.C);
+        }
+        if (stage < 0 || stage == 2) {
+            if (a.schema.layout == SN_NHWC)
+                launch_pdl(wino_output_kernel<T, true>, grid_for(wd.T * d.K, 256), 256, 0, a.stream, Mx, a.bias, (T *)a.out, wd);
+            else
+                launch_pdl(wino_output_kernel<T, false>, grid_for(wd.T * d.K, 256), 256, 0, a.stream, Mx, a.bias, (T *)a.out, wd);
+        }
     });
     return cudaGetLastError();
 }
@@ -494,7 +504,11 @@ __global__ void wino4_output_kernel(const float *__restrict__ Mx, const float *_
     }
 }
 
-cudaError_t conv_wino4(const LaunchArgs &a) {
+cudaError_t conv_wino4(const LaunchArgs &a) { return conv_wino4_stage(a, -1); }
+
+// stage 0: input transform (wgenc); 1: element-wise GEMMs (wgconv); 2: output
+// transform (wgdec); -1: all three
+cudaError_t conv_wino4_stage(const LaunchArgs &a, int stage) {
     const ConvDims d = conv_dims(a);
     const WinoDims wd = wino4_dims(d);
     const size_t need = (size_t)36 * wd.T * (d.C + d.K) * sizeof(float);
@@ -504,19 +518,25 @@ cudaError_t conv_wino4(const LaunchArgs &a) {
     dim3 ggrid((unsigned)((wd.T + 63) / 64), (unsigned)((d.K + 63) / 64), 36);
     if (ggrid.y > 65535) return cudaErrorInvalidValue;
     SN_DT_SWITCH(a.schema.dtype, T, {
-        if (a.schema.layout == SN_NHWC)
-            launch_pdl(wino4_input_kernel<T, true>, grid_for(wd.T * d.C, 256), 256, 0, a.stream, (const T *)a.in[0],
-                       V, wd);
-        else
-            launch_pdl(wino4_input_kernel<T, false>, grid_for(wd.T * d.C, 256), 256, 0, a.stream,
-                       (const T *)a.in[0], V, wd);
-        launch_pdl(gemm_nt_simt<float>, ggrid, 256, 0, a.stream, V, (const float *)a.wt, Mx, wd.T, d.K, d.C);
-        if (a.schema.layout == SN_NHWC)
-            launch_pdl(wino4_output_kernel<T, true>, grid_for(wd.T * d.K, 256), 256, 0, a.stream, Mx, a.bias,
-                       (T *)a.out, wd);
-        else
-            launch_pdl(wino4_output_kernel<T, false>, grid_for(wd.T * d.K, 256), 256, 0, a.stream, Mx, a.bias,
-                       (T *)a.out, wd);
+        if (stage < 0 || stage == 0) {
+            if (a.schema.layout == SN_NHWC)
+                launch_pdl(wino4_input_kernel<T, true>, grid_for(wd.T * d.C, 256), 256, 0, a.stream, (const T *)a.in[0],
+                           V, wd);
+            else
+                launch_pdl(wino4_input_kernel<T, false>, grid_for(wd.T * d.C, 256), 256, 0, a.stream,
+                           (const T *)a.in[0], V, wd);
+        }
+        if (stage < 0 || stage == 1) {
+            launch_pdl(gemm_nt_simt<float>, ggrid, 256, 0, a.stream, V, (const float *)a.wt, Mx, wd.T, d.K, d.C);
+        }
+        if (stage < 0 || stage == 2) {
+            if (a.schema.layout == SN_NHWC)
+                launch_pdl(wino4_output_kernel<T, true>, grid_for(wd.T * d.K, 256), 256, 0, a.stream, Mx, a.bias,
+                           (T *)a.out, wd);
+            else
+                launch_pdl(wino4_output_kernel<T, false>, grid_for(wd.T * d.K, 256), 256, 0, a.stream, Mx, a.bias,
+                           (T *)a.out, wd);
+        }
     });
     return cudaGetLastError();
 }
@@ -653,7 +673,11 @@ __global__ void wino6_output_kernel(const float *__restrict__ Mx, const float *_
     }
 }
 
-cudaError_t conv_wino6(const LaunchArgs &a) {
+cudaError_t conv_wino6(const LaunchArgs &a) { return conv_wino6_stage(a, -1); }
+
+// stage 0: input transform (wgenc); 1: element-wise GEMMs (wgconv); 2: output
+// transform (wgdec); -1: all three
+cudaError_t conv_wino6_stage(const LaunchArgs &a, int stage) {
     const ConvDims d = conv_dims(a);
     const WinoDims wd = wino6_dims(d);
     const size_t need = (size_t)64 * wd.T * (d.C + d.K) * sizeof(float);
@@ -663,19 +687,25 @@ cudaError_t conv_wino6(const LaunchArgs &a) {
     dim3 ggrid((unsigned)((wd.T + 63) / 64), (unsigned)((d.K + 63) / 64), 64);
     if (ggrid.y > 65535) return cudaErrorInvalidValue;
     SN_DT_SWITCH(a.schema.dtype, T, {
-        if (a.schema.layout == SN_NHWC)
-            launch_pdl(wino6_input_kernel<T, true>, grid_for(wd.T * d.C, 256), 256, 0, a.stream, (const T *)a.in[0],
-                       V, wd);
-        else
-            launch_pdl(wino6_input_kernel<T, false>, grid_for(wd.T * d.C, 256), 256, 0, a.stream,
-                       (const T *)a.in[0], V, wd);
-        launch_pdl(gemm_nt_simt<float>, ggrid, 256, 0, a.stream, V, (const float *)a.wt, Mx, wd.T, d.K, d.C);
-        if (a.schema.layout == SN_NHWC)
-            launch_pdl(wino6_output_kernel<T, true>, grid_for(wd.T * d.K, 256), 256, 0, a.stream, Mx, a.bias,
-                       (T *)a.out, wd);
-        else
-            launch_pdl(wino6_output_kernel<T, false>, grid_for(wd.T * d.K, 256), 256, 0, a.stream, Mx, a.bias,
-                       (T *)a.out, wd);
+        if (stage < 0 || stage == 0) {
+            if (a.schema.layout == SN_NHWC)
+                launch_pdl(wino6_input_kernel<T, true>, grid_for(wd.T * d.C, 256), 256, 0, a.stream, (const T *)a.in[0],
+                           V, wd);
+            else
+                launch_pdl(wino6_input_kernel<T, false>, grid_for(wd.T * d.C, 256), 256, 0, a.stream,
+                           (const T *)a.in[0], V, wd);
+        }
+        if (stage < 0 || stage == 1) {
+            launch_pdl(gemm_nt_simt<float>, ggrid, 256, 0, a.stream, V, (const float *)a.wt, Mx, wd.T, d.K, d.C);
+        }
+        if (stage < 0 || stage == 2) {
+            if (a.schema.layout == SN_NHWC)
+                launch_pdl(wino6_output_kernel<T, true>, grid_for(wd.T * d.K, 256), 256, 0, a.stream, Mx, a.bias,
+                           (T *)a.out, wd);
+            else
+                launch_pdl(wino6_output_kernel<T, false>, grid_for(wd.T * d.K, 256), 256, 0, a.stream, Mx, a.bias,
+                           (T *)a.out, wd);
+        }
     });
     return cudaGetLastError();
 }

@@ -1325,7 +1325,10 @@ __global__ void __launch_bounds__(256) im2col_rows_kernel(const T *__restrict__ 
     }
 }
 
-cudaError_t conv_im2col_tc(const LaunchArgs &a) {
+cudaError_t conv_im2col_tc(const LaunchArgs &a) { return conv_im2col_tc_stage(a, -1); }
+
+// stage 0: im2col; stage 1: the tensor-core GEMM; -1: both
+cudaError_t conv_im2col_tc_stage(const LaunchArgs &a, int stage) {
     const Layer &l = *a.layer;
     const ConvDims d = conv_dims(a);
     const int64_t kpad = im2col_kpad(l);
@@ -1333,7 +1336,8 @@ cudaError_t conv_im2col_tc(const LaunchArgs &a) {
     const size_t need = im2col_bytes(l, a.schema);
     if (!a.ws || a.ws_bytes < need || (uintptr_t)a.ws % 16) return cudaErrorInvalidValue;
     const size_t rows_bytes = (size_t)kpad * sizeof(int2) + (size_t)d.R * d.W * d.C * dtype_size(a.schema.dtype);
-    if (rows_bytes <= 48 * 1024 && d.N <= 65535) {
+    if (stage == 1) {
+    } else if (rows_bytes <= 48 * 1024 && d.N <= 65535) {
         SN_DT_SWITCH(a.schema.dtype, T,
                      launch_pdl(im2col_rows_kernel<T>, dim3((unsigned)d.P, (unsigned)d.N), 256, rows_bytes, a.stream, 
                          (const T *)a.in[0], (T *)a.ws, d, (int)kpad));
@@ -1343,7 +1347,7 @@ cudaError_t conv_im2col_tc(const LaunchArgs &a) {
                          (const T *)a.in[0], (T *)a.ws, d, (int)kpad, M));
     }
     cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
+    if (e != cudaSuccess || stage == 0) return e;
     const Layer gl = gemm_layer((int)kpad, d.K, d.act, l.out);
     LaunchArgs g = a;
     g.layer = &gl;
@@ -1443,7 +1447,10 @@ __global__ void __launch_bounds__(256) s2d_kernel(const T *__restrict__ x, T *__
     }
 }
 
-cudaError_t conv_s2d_tc(const LaunchArgs &a) {
+cudaError_t conv_s2d_tc(const LaunchArgs &a) { return conv_s2d_tc_stage(a, -1); }
+
+// stage 0: space-to-depth re-layout; stage 1: the tensor-core GEMM; -1: both
+cudaError_t conv_s2d_tc_stage(const LaunchArgs &a, int stage) {
     const Layer &l = *a.layer;
     if (!s2d_applies(l, a.schema)) return cudaErrorInvalidValue;
     const Shape &in = a.in_shapes[0];
@@ -1453,10 +1460,13 @@ cudaError_t conv_s2d_tc(const LaunchArgs &a) {
     const size_t xb = s2d_bytes(l, a.schema);
     if (!a.ws || a.ws_bytes < xb || (uintptr_t)a.ws % 256) return cudaErrorInvalidValue;
     const int64_t total = (int64_t)d.N * d.Pp * d.Qp;
-    SN_DT_SWITCH(a.schema.dtype, T,
-                 launch_pdl(s2d_kernel<T>, grid_for(total, 256), 256, 0, a.stream, (const T *)a.in[0], (T *)a.ws, d));
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
+    if (stage != 1) {
+        SN_DT_SWITCH(a.schema.dtype, T,
+                     launch_pdl(s2d_kernel<T>, grid_for(total, 256), 256, 0, a.stream, (const T *)a.in[0], (T *)a.ws,
+                                d));
+        cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess || stage == 0) return e;
+    }
     const Layer gl = s2d_gemm_layer(l);
     LaunchArgs g = a;
     g.layer = &gl;

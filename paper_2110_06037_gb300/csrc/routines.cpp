@@ -231,6 +231,41 @@ int32_t kernels_per_launch(int32_t r, int32_t v, const Layer &l, const std::vect
     return 1 + split;
 }
 
+int32_t childnet_stages(int32_t r, sn_schema s) {
+    if (s.dtype == SN_QI8) return 1;
+    switch (r) {
+    case R_CONV_IM2COL_TC:
+    case R_CONV_S2D_TC: return 2;  // re-layout, GEMM
+    case R_CONV_WINO:
+    case R_CONV_WINO4:
+    case R_CONV_WINO6: return 3;   // wgenc, wgconv, wgdec
+    default: return 1;
+    }
+}
+
+bool stage_uses_variant(int32_t r, int32_t stage) {
+    // the GEMM of the im2col / space-to-depth childnets carries the tile
+    // parameters; their re-layout and the Winograd stages have none
+    return (r == R_CONV_IM2COL_TC || r == R_CONV_S2D_TC) && stage == 1;
+}
+
+sn_status launch_routine_stage(const LaunchArgs &a, int32_t stage) {
+    cudaError_t e = cudaSuccess;
+    switch (a.routine) {
+    case R_CONV_IM2COL_TC: e = k::conv_im2col_tc_stage(a, stage); break;
+    case R_CONV_S2D_TC: e = k::conv_s2d_tc_stage(a, stage); break;
+    case R_CONV_WINO: e = k::conv_wino_stage(a, stage); break;
+    case R_CONV_WINO4: e = k::conv_wino4_stage(a, stage); break;
+    case R_CONV_WINO6: e = k::conv_wino6_stage(a, stage); break;
+    default: return launch_routine(a);
+    }
+    if (e == cudaErrorNotSupported)
+        return fail(SN_EUNSUPPORTED, std::string(routine_name(a.routine)) + ": not supported here");
+    if (e != cudaSuccess)
+        return fail(SN_ECUDA, std::string(routine_name(a.routine)) + " (stage): " + cudaGetErrorString(e));
+    return SN_OK;
+}
+
 static cudaError_t launch_q8(const LaunchArgs &a) {
     switch (a.routine) {
     case R_CONV_DIRECT:

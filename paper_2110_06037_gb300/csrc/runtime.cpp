@@ -370,7 +370,7 @@ static sn_status profile_graph_on(Graph *g, const sn_profile_opts &o, cudaStream
     }
     // scratch inputs: small deterministic values (fp32 patterns reinterpreted
     // per dtype are not needed: fill each dtype's worth of elements)
-    std::map<std::string, int64_t> seen;
+    std::map<std::string, int64_t> seen, seen_stage;
     // --- unit profiling of layer routines ---
     for (int32_t i = 1; i < n - 1 && rc == SN_OK; ++i) {
         const Layer &L = g->layers[i];
@@ -415,7 +415,31 @@ static sn_status profile_graph_on(Graph *g, const sn_profile_opts &o, cudaStream
             a.ws = g->workspace.ptr;
             a.ws_bytes = g->workspace.bytes;
             int64_t t = kInf;
-            rc = time_median(o.warmup, o.iters, st, [&]() { return launch_routine(a); }, &t);
+            const int32_t nst = childnet_stages(cd.routine, s);
+            if (nst == 1) {
+                rc = time_median(o.warmup, o.iters, st, [&]() { return launch_routine(a); }, &t);
+            } else {
+                // a childnet (section III-D): each sub-layer is timed on its
+                // own, once for every routine parameter it depends on, and
+                // the childnet's cost is the sum along its chain (DPRS on a
+                // chain whose sub-layer schemas the parent routine fixes)
+                t = 0;
+                for (int32_t stg = 0; stg < nst && rc == SN_OK && t != kInf; ++stg) {
+                    std::ostringstream sk;
+                    sk << signature(g, i, Candidate{cd.routine, stage_uses_variant(cd.routine, stg) ? cd.variant : -1,
+                                                    cd.schema, cd.layer, 0})
+                       << "#stage" << stg;
+                    auto hit = seen_stage.find(sk.str());
+                    int64_t ts = kInf;
+                    if (hit != seen_stage.end()) {
+                        ts = hit->second;
+                    } else {
+                        rc = time_median(o.warmup, o.iters, st, [&]() { return launch_routine_stage(a, stg); }, &ts);
+                        if (rc == SN_OK) seen_stage.emplace(sk.str(), ts);
+                    }
+                    t = sat_add(t, ts);
+                }
+            }
             if (rc == SN_EUNSUPPORTED) {  // a routine parameter this device cannot run: infeasible
                 rc = SN_OK;
                 t = kInf;

@@ -220,6 +220,13 @@ size_t routine_workspace(int32_t routine, int32_t variant, const Layer &layer,
 sn_status prepare_weights(Graph *g, int32_t li, int32_t routine, int32_t variant, sn_schema s,
                           const void **wt, const float **bias, cudaStream_t st);
 sn_status launch_routine(const LaunchArgs &a);
+// childnets (section III-D): routines made of sub-layers that the profiler
+// times one by one.  childnet_stages = number of sub-layers (1 = a plain
+// routine); stage_uses_variant = whether a sub-layer's time depends on the
+// parent routine's parameter (otherwise it is timed once for all of them).
+int32_t childnet_stages(int32_t routine, sn_schema s);
+bool stage_uses_variant(int32_t routine, int32_t stage);
+sn_status launch_routine_stage(const LaunchArgs &a, int32_t stage);
 int32_t kernels_per_launch(int32_t routine, int32_t variant, const Layer &layer, const std::vector<Shape> &in,
                            sn_schema s);
 
@@ -260,6 +267,12 @@ size_t conv_wino_ws(const Layer &l, const Shape &in, sn_schema s);
 cudaError_t conv_wino4(const LaunchArgs &a);
 size_t conv_wino4_ws(const Layer &l, const Shape &in, sn_schema s);
 cudaError_t conv_wino6(const LaunchArgs &a);
+// childnet stages, launched on their own (stage -1 = the whole routine)
+cudaError_t conv_wino_stage(const LaunchArgs &a, int stage);
+cudaError_t conv_wino4_stage(const LaunchArgs &a, int stage);
+cudaError_t conv_wino6_stage(const LaunchArgs &a, int stage);
+cudaError_t conv_im2col_tc_stage(const LaunchArgs &a, int stage);
+cudaError_t conv_s2d_tc_stage(const LaunchArgs &a, int stage);
 size_t conv_wino6_ws(const Layer &l, const Shape &in, sn_schema s);
 cudaError_t conv_tc(const LaunchArgs &a);
 int32_t conv_tc_variants(const Layer &l, const Shape &in, sn_schema s);
