@@ -182,11 +182,18 @@ SN_API sn_status sn_get_io(sn_graph *g, int32_t *n_inputs, int32_t *n_outputs);
  * Schema indices run over the graph's schema universe: Lambda in the order
  * given, then in_schema and out_schema if they are not in Lambda. */
 typedef struct {
-    int32_t routine;  /* routine id, see sn_routine_name()                */
-    int32_t variant;  /* routine-parameter combination index              */
-    int32_t schema;   /* schema index                                      */
-    int32_t layer;    /* internal layer index                              */
-    int64_t cost_ns;  /* T(r); SN_COST_INF until profiled or set           */
+    int32_t routine;    /* routine id, see sn_routine_name()                */
+    int32_t variant;    /* routine-parameter combination index              */
+    int32_t schema;     /* schema index the routine reads its inputs in     */
+    int32_t layer;      /* internal layer index                              */
+    int64_t cost_ns;    /* T(r); SN_COST_INF until profiled or set           */
+    int32_t out_schema; /* schema index it writes its output in: = schema,
+                           except for fused-boundary routines (a qint8
+                           routine leaving its result in a float schema).
+                           When any candidate has out_schema != schema, the
+                           selection runs over (schema, out_schema) pairs and
+                           an edge's adapt goes from the producer's
+                           out_schema to the consumer's schema. */
 } sn_candidate;
 
 typedef struct {

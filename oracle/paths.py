@@ -175,3 +175,37 @@ def full_routine_product(cands, edges, adapt_cost, ns):
                 t = INF if (t == INF or c == INF) else t + c
         best = min(best, t)
     return best
+
+
+def brute_force_candidates(cands, edges, adapt_cost):
+    """Exact optimum when a routine may write a schema other than the one it
+    reads (a fused boundary): enumerate one candidate per layer, with
+    T = sum of candidate times + sum over edges (u, v) of the adapt from u's
+    written schema to v's read schema (0 when they agree).
+
+    cands: per layer a list of (cost, read_schema, written_schema); adapt_cost
+    [n_edges, ns, ns].  Returns (T*, [chosen index per layer]) — the first
+    minimum in lexicographic order of the choices; INF when none is finite.
+    """
+    n = len(cands)
+    best, best_pick = INF, None
+    for pick in itertools.product(*[range(len(c)) for c in cands]):
+        t = 0
+        for i, k in enumerate(pick):
+            t = INF if cands[i][k][0] >= INF else t + int(cands[i][k][0])
+            if t >= INF:
+                break
+        if t >= INF:
+            continue
+        for e, (u, v) in enumerate(edges):
+            w, r = cands[u][pick[u]][2], cands[v][pick[v]][1]
+            if w != r:
+                a = int(adapt_cost[e][w][r])
+                if a >= INF:
+                    t = INF
+                    break
+                t += a
+        if t < best:
+            best, best_pick = t, list(pick)
+    return best, best_pick
+

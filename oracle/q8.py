@@ -85,7 +85,18 @@ def act_f32(y, act: str):
     raise ValueError(act)
 
 
-def _epilogue(acc, m, bias, act, s_out, resid=None):
+def finish(y, s_out, out_dtype=None):
+    """The output of a qint8 routine from its fp32 result y: codes of scale
+    s_out, or, for a routine that writes a float schema (dequantisation fused
+    into its epilogue), y rounded to nearest even in that dtype (returned as
+    fp32 values)."""
+    if out_dtype in (None, "qi8"):
+        return requantize(y, s_out)
+    from . import round_to
+    return round_to(np.asarray(y, dtype=F32), out_dtype)
+
+
+def _epilogue(acc, m, bias, act, s_out, resid=None, out_dtype=None):
     """acc: int64 [N, K, ...]; m: fp32 [K] multipliers s_x * s_w[k]."""
     shape = (1, -1) + (1,) * (acc.ndim - 2)
     y = acc.astype(F32) * m.reshape(shape)
@@ -94,7 +105,7 @@ def _epilogue(acc, m, bias, act, s_out, resid=None):
     if resid is not None:
         qr, sr = resid
         y = y + dequantize(qr, sr)
-    return requantize(act_f32(y, act), s_out)
+    return finish(act_f32(y, act), s_out, out_dtype)
 
 
 def conv_acc(qx, qw, stride=(1, 1), pad=(0, 0), dil=(1, 1), groups=1) -> np.ndarray:
@@ -124,26 +135,26 @@ def conv_acc(qx, qw, stride=(1, 1), pad=(0, 0), dil=(1, 1), groups=1) -> np.ndar
 
 
 def conv2d(qx, s_x, qw, s_w, bias, s_out, stride=(1, 1), pad=(0, 0), dil=(1, 1), groups=1,
-           act="none", resid=None) -> np.ndarray:
+           act="none", resid=None, out_dtype=None) -> np.ndarray:
     """qint8 conv2 / dwconv2 (groups = C): codes of y = act(conv + bias [+ residual]).
     resid = (codes, scale) of a residual blob shaped like the output."""
     acc = conv_acc(qx, qw, stride, pad, dil, groups)
     m = F32(s_x) * np.asarray(s_w, dtype=F32)
-    return _epilogue(acc, m, bias, act, s_out, resid)
+    return _epilogue(acc, m, bias, act, s_out, resid, out_dtype)
 
 
-def dense(qx, s_x, qw, s_w, bias, s_out, act="none") -> np.ndarray:
+def dense(qx, s_x, qw, s_w, bias, s_out, act="none", out_dtype=None) -> np.ndarray:
     """qint8 dense on an N x C (x 1 x 1) blob: y = act(W x + b)."""
     qx = np.asarray(qx)
     shp = qx.shape
     x2 = qx.reshape(shp[0], -1).astype(np.int64)
     acc = x2 @ np.asarray(qw).astype(np.int64).T
     m = F32(s_x) * np.asarray(s_w, dtype=F32)
-    y = _epilogue(acc, m, bias, act, s_out)
+    y = _epilogue(acc, m, bias, act, s_out, out_dtype=out_dtype)
     return y.reshape((shp[0], -1) + shp[2:]) if len(shp) == 4 else y
 
 
-def maxpool2d(qx, s_x, s_out, k=(3, 3), stride=(2, 2), pad=(1, 1)) -> np.ndarray:
+def maxpool2d(qx, s_x, s_out, k=(3, 3), stride=(2, 2), pad=(1, 1), out_dtype=None) -> np.ndarray:
     """Max over the window's in-image codes (padding never wins), then the
     maximum's value q * s_x requantised to s_out."""
     qx = np.asarray(qx).astype(np.int64)
@@ -159,30 +170,30 @@ def maxpool2d(qx, s_x, s_out, k=(3, 3), stride=(2, 2), pad=(1, 1)) -> np.ndarray
     for i in range(kh):
         for j in range(kw):
             out = np.maximum(out, xp[:, :, i:i + sh * (p - 1) + 1:sh, j:j + sw * (q - 1) + 1:sw])
-    return requantize(dequantize(out, s_x), s_out)
+    return finish(dequantize(out, s_x), s_out, out_dtype)
 
 
-def gap(qx, s_x, s_out) -> np.ndarray:
+def gap(qx, s_x, s_out, out_dtype=None) -> np.ndarray:
     """Global average pool: the exact code sum over H x W, times s_x, divided
     by H*W (two fp32 roundings), requantised.  Output N x C x 1 x 1."""
     qx = np.asarray(qx).astype(np.int64)
     n, c, h, w = qx.shape
     tot = qx.sum(axis=(2, 3)).astype(F32) * F32(s_x)
     y = tot / F32(h * w)
-    return requantize(y, s_out).reshape(n, c, 1, 1)
+    return finish(y, s_out, out_dtype).reshape(n, c, 1, 1)
 
 
-def add(qa, s_a, qb, s_b, s_out, act="none") -> np.ndarray:
+def add(qa, s_a, qb, s_b, s_out, act="none", out_dtype=None) -> np.ndarray:
     """y = act(a + b) with a, b dequantised (one rounding each), one rounded add."""
     y = dequantize(qa, s_a) + dequantize(qb, s_b)
-    return requantize(act_f32(y, act), s_out)
+    return finish(act_f32(y, act), s_out, out_dtype)
 
 
-def mul(qx, s_x, qs, s_s, s_out, act="none") -> np.ndarray:
+def mul(qx, s_x, qs, s_s, s_out, act="none", out_dtype=None) -> np.ndarray:
     """Squeeze-and-excite scale y[n,c,h,w] = act(x[n,c,h,w] * s[n,c])."""
     x = dequantize(qx, s_x)
     sc = dequantize(np.asarray(qs).reshape(qx.shape[0], qx.shape[1], 1, 1), s_s)
-    return requantize(act_f32(x * sc, act), s_out)
+    return finish(act_f32(x * sc, act), s_out, out_dtype)
 
 
 def absmax_scale(x) -> np.float32:
@@ -191,9 +202,11 @@ def absmax_scale(x) -> np.float32:
     return a / F32(QMAX) if a > 0 else F32(1.0)
 
 
-def run_layer(layer: dict, ins: list, s_ins: list, s_out) -> np.ndarray:
+def run_layer(layer: dict, ins: list, s_ins: list, s_out, out_dtype=None) -> np.ndarray:
     """One layer of a net (the dict format of oracle.net) in the qint8 schema:
-    ins are int8 NCHW codes with scales s_ins; returns the output codes."""
+    ins are int8 NCHW codes with scales s_ins; returns the output codes (or,
+    with out_dtype a float dtype, the fused-dequantisation output values)."""
+    o = dict(out_dtype=out_dtype)
     t, p = layer["type"], layer.get("params", {})
     act = p.get("act", "none")
     if t in ("conv2", "dwconv2"):
@@ -202,19 +215,19 @@ def run_layer(layer: dict, ins: list, s_ins: list, s_out) -> np.ndarray:
         resid = (ins[1], s_ins[1]) if len(ins) == 2 else None
         return conv2d(ins[0], s_ins[0], qw, s_w, layer.get("bias"), s_out, stride=(p["sh"], p["sw"]),
                       pad=(p["ph"], p["pw"]), dil=(p.get("dh", 1), p.get("dw", 1)), groups=groups,
-                      act=act, resid=resid)
+                      act=act, resid=resid, **o)
     if t == "dense":
         qw, s_w = quantize_weights(layer["weight"])
-        return dense(ins[0], s_ins[0], qw, s_w, layer.get("bias"), s_out, act=act)
+        return dense(ins[0], s_ins[0], qw, s_w, layer.get("bias"), s_out, act=act, **o)
     if t == "maxpool":
         return maxpool2d(ins[0], s_ins[0], s_out, k=(p["kh"], p["kw"]), stride=(p["sh"], p["sw"]),
-                         pad=(p["ph"], p["pw"]))
+                         pad=(p["ph"], p["pw"]), **o)
     if t == "gap":
-        return gap(ins[0], s_ins[0], s_out)
+        return gap(ins[0], s_ins[0], s_out, **o)
     if t == "add":
-        return add(ins[0], s_ins[0], ins[1], s_ins[1], s_out, act=act)
+        return add(ins[0], s_ins[0], ins[1], s_ins[1], s_out, act=act, **o)
     if t == "mul":
-        return mul(ins[0], s_ins[0], ins[1], s_ins[1], s_out, act=act)
+        return mul(ins[0], s_ins[0], ins[1], s_ins[1], s_out, act=act, **o)
     raise ValueError(f"unknown layer type {t}")
 
 

@@ -52,7 +52,7 @@ class sn_dense_params(C.Structure):
 
 class sn_candidate(C.Structure):
     _fields_ = [("routine", C.c_int32), ("variant", C.c_int32), ("schema", C.c_int32),
-                ("layer", C.c_int32), ("cost_ns", C.c_int64)]
+                ("layer", C.c_int32), ("cost_ns", C.c_int64), ("out_schema", C.c_int32)]
 
 
 class sn_cost_table(C.Structure):

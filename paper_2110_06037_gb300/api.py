@@ -136,19 +136,21 @@ class Graph:
         t.edges = edges.ctypes.data_as(C.POINTER(C.c_int32))
         t.adapt_cost = adapt.ctypes.data_as(C.POINTER(C.c_int64))
         check(lib().sn_get_cost_table(self.h, C.byref(t)))
-        arr = np.array([(c.routine, c.variant, c.schema, c.layer, c.cost_ns) for c in cands],
-                       dtype=np.int64).reshape(-1, 5)
+        arr = np.array([(c.routine, c.variant, c.schema, c.layer, c.cost_ns, c.out_schema) for c in cands],
+                       dtype=np.int64).reshape(-1, 6)
         return {"n_layers": t.n_layers, "n_schemas": t.n_schemas,
                 "routine": arr[:, 0].astype(np.int32), "variant": arr[:, 1].astype(np.int32),
                 "schema": arr[:, 2].astype(np.int32), "layer": arr[:, 3].astype(np.int32),
-                "cost": arr[:, 4].copy(), "edges": edges.reshape(-1, 2),
+                "cost": arr[:, 4].copy(), "out_schema": arr[:, 5].astype(np.int32), "edges": edges.reshape(-1, 2),
                 "adapt": adapt.reshape(t.n_edges, t.n_schemas, t.n_schemas)}
 
     def set_cost_table(self, table):
         n = len(table["cost"])
         cands = (_sn.sn_candidate * n)(*[
             _sn.sn_candidate(int(table["routine"][i]), int(table["variant"][i]), int(table["schema"][i]),
-                             int(table["layer"][i]), int(table["cost"][i])) for i in range(n)])
+                             int(table["layer"][i]), int(table["cost"][i]),
+                             int(table["out_schema"][i] if "out_schema" in table else table["schema"][i]))
+            for i in range(n)])
         adapt = np.ascontiguousarray(table["adapt"], dtype=np.int64).ravel()
         t = _sn.sn_cost_table(table["n_layers"], table["n_schemas"], len(table["edges"]), n, cands, None,
                               adapt.ctypes.data_as(C.POINTER(C.c_int64)))

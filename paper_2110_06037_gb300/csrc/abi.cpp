@@ -111,7 +111,7 @@ sn_status sn_get_cost_table(sn_graph *gg, sn_cost_table *t) {
             if (t->candidates)
                 for (size_t c = 0; c < g->cands.size(); ++c) {
                     const Candidate &k = g->cands[c];
-                    t->candidates[c] = {k.routine, k.variant, k.schema, k.layer, k.cost};
+                    t->candidates[c] = {k.routine, k.variant, k.schema, k.layer, k.cost, cand_out(k)};
                 }
             if (t->edges)
                 for (size_t e = 0; e < g->edges.size(); ++e) {
@@ -142,7 +142,8 @@ sn_status sn_set_cost_table(sn_graph *gg, const sn_cost_table *t) {
         for (size_t c = 0; c < g->cands.size(); ++c) {
             const Candidate &k = g->cands[c];
             const sn_candidate &x = t->candidates[c];
-            if (x.routine != k.routine || x.variant != k.variant || x.schema != k.schema || x.layer != k.layer)
+            if (x.routine != k.routine || x.variant != k.variant || x.schema != k.schema || x.layer != k.layer ||
+                x.out_schema != cand_out(k))
                 return fail(SN_EINVAL, "sn_set_cost_table: candidate " + std::to_string(c) + " differs");
             if (x.cost_ns < 0) return fail(SN_EINVAL, "sn_set_cost_table: negative cost");
         }
@@ -188,16 +189,10 @@ sn_status sn_profile(sn_graph *gg, const sn_profile_opts *opts, void *stream) {
     })
 }
 
-static sn_status fill_path(Graph *g, const std::vector<int32_t> &schema_of, int64_t total, sn_path *out) {
-    std::vector<int64_t> F;
-    std::vector<int32_t> argF;
-    fastest_per_schema(*g, F, argF);
-    const int32_t n = g->n_layers(), ns = g->n_schemas();
-    std::vector<int32_t> pc(n);
-    for (int32_t i = 0; i < n; ++i) {
-        pc[i] = argF[(size_t)i * ns + schema_of[i]];
-        if (pc[i] < 0) return fail(SN_EINFEASIBLE, "selected schema has no routine");
-    }
+static sn_status fill_path(Graph *g, const std::vector<int32_t> &pc, int64_t total, sn_path *out) {
+    const int32_t n = g->n_layers();
+    std::vector<int32_t> schema_of(n);
+    for (int32_t i = 0; i < n; ++i) schema_of[i] = g->cands[pc[i]].schema;
     g->path_cand = pc;
     g->path_total = total;
     g->has_path = true;
@@ -221,13 +216,12 @@ sn_status sn_select_path(sn_graph *gg, int32_t method, sn_path *out) {
         Graph *g = G(gg);
         sn_status rc = graph_finalize(g);
         if (rc != SN_OK) return rc;
-        std::vector<int32_t> schema_of;
+        if (method != SN_SELECT_DPRS && method != SN_SELECT_BRUTE) return fail(SN_EINVAL, "sn_select_path: unknown method");
+        std::vector<int32_t> cand_of;
         int64_t total = kInf;
-        if (method == SN_SELECT_DPRS) rc = select_dprs(*g, schema_of, total);
-        else if (method == SN_SELECT_BRUTE) rc = select_brute(*g, schema_of, total);
-        else return fail(SN_EINVAL, "sn_select_path: unknown method");
+        rc = select_path(*g, method, cand_of, total);
         if (rc != SN_OK) return rc;
-        return fill_path(g, schema_of, total, out);
+        return fill_path(g, cand_of, total, out);
     })
 }
 

@@ -102,7 +102,7 @@ struct Ctx {
             if (t == kInf) return kInf;
             for (int32_t e : in_edges[v]) {
                 const int32_t u = g.edges[e].first;
-                if (asg[u] != asg[v]) t = sat_add(t, g.adapt(e, asg[u], asg[v]));
+                t = sat_add(t, g.adapt(e, asg[u], asg[v]));  // 0 for a void adapt
                 if (t == kInf) return kInf;
             }
         }
@@ -294,6 +294,56 @@ sn_status select_brute(const Graph &g, std::vector<int32_t> &schema_of, int64_t 
     if (best == kInf) return fail(SN_EINFEASIBLE, "no routine path with finite cost");
     schema_of.assign(best_asg.begin(), best_asg.end());
     total = best;
+    return SN_OK;
+}
+
+// ---------------------------------------------------------------------------
+// fused boundaries: the same algorithm over (read, written) schema pairs
+// ---------------------------------------------------------------------------
+// The pair problem has |Lambda|^2 schemas p = read * ns + written; candidate c
+// of layer i sits at its pair, and edge (u, v) costs the adapt from u's
+// written schema to v's read one (void when they agree).  Pairs no routine
+// has keep F = INF, so DPRS never enters them.
+static void expand_pairs(const Graph &g, Graph &x) {
+    const int32_t ns = g.n_schemas(), np = ns * ns;
+    x.layers.resize(g.layers.size());
+    x.schemas.assign((size_t)np, sn_schema{SN_F32, SN_NCHW});
+    x.edges = g.edges;
+    x.cand_begin = g.cand_begin;
+    x.cands = g.cands;
+    for (auto &c : x.cands) {
+        c.schema = c.schema * ns + cand_out(c);
+        c.out_schema = -1;
+    }
+    x.adapt_cost.assign(g.edges.size() * (size_t)np * np, kInf);
+    for (size_t e = 0; e < g.edges.size(); ++e)
+        for (int32_t p = 0; p < np; ++p)
+            for (int32_t q = 0; q < np; ++q)
+                x.adapt((int32_t)e, p, q) = g.adapt((int32_t)e, p % ns, q / ns);
+    x.finalized = true;
+}
+
+sn_status select_path(const Graph &g, int32_t method, std::vector<int32_t> &cand_of, int64_t &total) {
+    bool fused = false;
+    for (const auto &c : g.cands) fused = fused || cand_out(c) != c.schema;
+    Graph xg;
+    const Graph *pg = &g;
+    if (fused) {
+        expand_pairs(g, xg);
+        pg = &xg;
+    }
+    std::vector<int32_t> schema_of;
+    sn_status rc = method == SN_SELECT_BRUTE ? select_brute(*pg, schema_of, total) : select_dprs(*pg, schema_of, total);
+    if (rc != SN_OK) return rc;
+    std::vector<int64_t> F;
+    std::vector<int32_t> argF;
+    fastest_per_schema(*pg, F, argF);
+    const int32_t n = pg->n_layers(), ns = pg->n_schemas();
+    cand_of.assign(n, -1);
+    for (int32_t i = 0; i < n; ++i) {
+        cand_of[i] = argF[(size_t)i * ns + schema_of[i]];
+        if (cand_of[i] < 0) return fail(SN_EINFEASIBLE, "selected schema has no routine");
+    }
     return SN_OK;
 }
 

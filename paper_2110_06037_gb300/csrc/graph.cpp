@@ -316,6 +316,16 @@ sn_status graph_finalize(Graph *g) {
             for (int32_t s = 0; s < g->n_lambda; ++s) {
                 const int32_t nv = routine_variants(r, L[i], in, g->schemas[s]);
                 for (int32_t v = 0; v < nv; ++v) cands.push_back({r, v, s, i, kInf});
+                if (nv == 0) continue;
+                // the same routine writing another schema of Lambda (fused boundary)
+                for (const sn_schema &o : fused_outputs(r, L[i], g->schemas[s]))
+                    for (int32_t so = 0; so < g->n_lambda; ++so)
+                        if (so != s && schema_eq(g->schemas[so], o))
+                            for (int32_t v = 0; v < nv; ++v) {
+                                Candidate c{r, v, s, i, kInf};
+                                c.out_schema = so;
+                                cands.push_back(c);
+                            }
             }
         }
         if ((int32_t)cands.size() == begin[i])

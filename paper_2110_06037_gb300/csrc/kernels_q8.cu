@@ -38,12 +38,20 @@ __device__ __forceinline__ float q8_act(float v, int act) {
     return act == SN_ACT_HSWISH ? __fmul_rn(v, t) : t;
 }
 
-// float(acc) * (s_x * s_w) + bias [+ residual value], act, code
-__device__ __forceinline__ int8_t q8_epilogue(int acc, float s_x, float s_w, float bias, float resid, int act,
-                                              float inv) {
+// act(float(acc) * (s_x * s_w) + bias [+ residual value]) in fp32
+__device__ __forceinline__ float q8_value(int acc, float s_x, float s_w, float bias, float resid, int act) {
     float y = __fadd_rn(__fmul_rn(__int2float_rn(acc), __fmul_rn(s_x, s_w)), bias);
     y = __fadd_rn(y, resid);
-    return q8_code(q8_act(y, act), inv);
+    return q8_act(y, act);
+}
+
+// the output element: a code of the output blob's scale, or, when the routine
+// writes a float schema (dequantisation fused into the epilogue), the fp32
+// value rounded to that type
+template <typename TO>
+__device__ __forceinline__ TO q8_out(float y, float inv) {
+    if constexpr (std::is_same<TO, int8_t>::value) return q8_code(y, inv);
+    else return cvt<TO>(y);
 }
 
 __device__ __forceinline__ int dp4a(int a, int b, int c) { return __dp4a(a, b, c); }
@@ -373,10 +381,10 @@ struct Q8Scales {
     float s_x, s_r, inv_out;
 };
 
-template <bool NHWC>
+template <bool NHWC, typename TO>
 __global__ void q8_conv_direct_kernel(const int8_t *__restrict__ x, const int8_t *__restrict__ w,
                                       const float *__restrict__ ws, const float *__restrict__ bias,
-                                      const int8_t *__restrict__ res, int8_t *__restrict__ y, ConvDims d, Q8Scales q) {
+                                      const int8_t *__restrict__ res, TO *__restrict__ y, ConvDims d, Q8Scales q) {
     griddep_launch();
     griddep_wait();
     const int64_t total = (int64_t)d.N * d.K * d.P * d.Q;
@@ -417,18 +425,32 @@ __global__ void q8_conv_direct_kernel(const int8_t *__restrict__ x, const int8_t
             }
         }
         const float rv = res ? __fmul_rn((float)res[i], q.s_r) : 0.0f;  // residual: the output's index
-        y[i] = q8_epilogue(acc, q.s_x, ws[kk], bias[kk], rv, d.act, q.inv_out);
+        y[i] = q8_out<TO>(q8_value(acc, q.s_x, ws[kk], bias[kk], rv, d.act), q.inv_out);
     }
 }
 
+// the schema dtype the routine writes: qint8, or a float type when the
+// dequantisation is fused into its epilogue
+static int out_dtype(const LaunchArgs &a) { return a.out_schema.dtype < 0 ? a.schema.dtype : a.out_schema.dtype; }
+
+#define SN_Q8_OUT_SWITCH(dt, TO, ...)                               \
+    switch (dt) {                                                   \
+    case SN_QI8: { using TO = int8_t; __VA_ARGS__; break; }         \
+    case SN_F16: { using TO = __half; __VA_ARGS__; break; }         \
+    case SN_BF16: { using TO = __nv_bfloat16; __VA_ARGS__; break; } \
+    case SN_F32: { using TO = float; __VA_ARGS__; break; }          \
+    default: return cudaErrorInvalidValue;                          \
+    }
+
 static Q8Scales scales_of(const LaunchArgs &a) {
-    return Q8Scales{a.qs_in[0], a.qs_in[1], 1.0f / a.qs_out};
+    return Q8Scales{a.qs_in[0], a.qs_in[1], a.qs_out > 0.0f ? 1.0f / a.qs_out : 0.0f};
 }
 
+// the input scales, and the output scale when the output is qint8
 static bool scales_ok(const LaunchArgs &a, int n_in) {
     for (int i = 0; i < n_in; ++i)
         if (!(a.qs_in[i] > 0.0f) || !std::isfinite(a.qs_in[i])) return false;
-    return a.qs_out > 0.0f && std::isfinite(a.qs_out);
+    return out_dtype(a) != SN_QI8 || (a.qs_out > 0.0f && std::isfinite(a.qs_out));
 }
 
 cudaError_t q8_conv_direct(const LaunchArgs &a) {
@@ -437,12 +459,16 @@ cudaError_t q8_conv_direct(const LaunchArgs &a) {
     const int64_t total = (int64_t)d.N * d.K * d.P * d.Q;
     const int64_t elems = (int64_t)d.K * (d.C / d.groups) * d.R * d.S;
     const float *ws = wscales(a.wt, elems);
-    if (a.schema.layout == SN_NHWC)
-        launch_pdl(q8_conv_direct_kernel<true>, grid_for(total, 256), 256, 0, a.stream, (const int8_t *)a.in[0],
-                   (const int8_t *)a.wt, ws, a.bias, (const int8_t *)a.in[1], (int8_t *)a.out, d, scales_of(a));
-    else
-        launch_pdl(q8_conv_direct_kernel<false>, grid_for(total, 256), 256, 0, a.stream, (const int8_t *)a.in[0],
-                   (const int8_t *)a.wt, ws, a.bias, (const int8_t *)a.in[1], (int8_t *)a.out, d, scales_of(a));
+    SN_Q8_OUT_SWITCH(out_dtype(a), TO, {
+        if (a.schema.layout == SN_NHWC)
+            launch_pdl(q8_conv_direct_kernel<true, TO>, grid_for(total, 256), 256, 0, a.stream,
+                       (const int8_t *)a.in[0], (const int8_t *)a.wt, ws, a.bias, (const int8_t *)a.in[1], (TO *)a.out,
+                       d, scales_of(a));
+        else
+            launch_pdl(q8_conv_direct_kernel<false, TO>, grid_for(total, 256), 256, 0, a.stream,
+                       (const int8_t *)a.in[0], (const int8_t *)a.wt, ws, a.bias, (const int8_t *)a.in[1], (TO *)a.out,
+                       d, scales_of(a));
+    });
     return cudaGetLastError();
 }
 
@@ -456,10 +482,11 @@ cudaError_t q8_conv_direct(const LaunchArgs &a) {
 // Weights are [K][R][S][C].
 constexpr int DP_BM = 64, DP_BN = 64, DP_WORDS = 8;
 
+template <typename TO>
 __global__ void __launch_bounds__(256) q8_conv_dp4a_kernel(const int8_t *__restrict__ x, const int8_t *__restrict__ w,
                                                            const float *__restrict__ ws,
                                                            const float *__restrict__ bias,
-                                                           const int8_t *__restrict__ res, int8_t *__restrict__ y,
+                                                           const int8_t *__restrict__ res, TO *__restrict__ y,
                                                            ConvDims d, Q8Scales q) {
     griddep_launch();
     __shared__ __align__(16) int As[2][DP_WORDS][DP_BM];
@@ -532,13 +559,18 @@ __global__ void __launch_bounds__(256) q8_conv_dp4a_kernel(const int8_t *__restr
         char4 rr = make_char4(0, 0, 0, 0);
         if (res) rr = *reinterpret_cast<const char4 *>(res + m * d.K + kb);
         const int8_t r4[4] = {rr.x, rr.y, rr.z, rr.w};
-        int8_t o[4];
+        TO o[4];
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
             const float rv = res ? __fmul_rn((float)r4[j], q.s_r) : 0.0f;
-            o[j] = q8_epilogue(acc[i][j], q.s_x, sw[j], bs[j], rv, d.act, q.inv_out);
+            o[j] = q8_out<TO>(q8_value(acc[i][j], q.s_x, sw[j], bs[j], rv, d.act), q.inv_out);
         }
-        *reinterpret_cast<char4 *>(y + m * d.K + kb) = make_char4(o[0], o[1], o[2], o[3]);
+        if constexpr (std::is_same<TO, int8_t>::value) {
+            *reinterpret_cast<char4 *>(y + m * d.K + kb) = make_char4(o[0], o[1], o[2], o[3]);
+        } else {
+#pragma unroll
+            for (int j = 0; j < 4; ++j) y[m * d.K + kb + j] = o[j];
+        }
     }
 }
 
@@ -556,8 +588,10 @@ cudaError_t q8_conv_dp4a(const LaunchArgs &a) {
     const int64_t elems = (int64_t)d.K * d.C * d.R * d.S;
     const dim3 grid((unsigned)((M + DP_BM - 1) / DP_BM), (unsigned)((d.K + DP_BN - 1) / DP_BN));
     if (grid.y > 65535) return cudaErrorInvalidValue;
-    launch_pdl(q8_conv_dp4a_kernel, grid, 256, 0, a.stream, (const int8_t *)a.in[0], (const int8_t *)a.wt,
-               wscales(a.wt, elems), a.bias, (const int8_t *)a.in[1], (int8_t *)a.out, d, scales_of(a));
+    SN_Q8_OUT_SWITCH(out_dtype(a), TO,
+                     launch_pdl(q8_conv_dp4a_kernel<TO>, grid, 256, 0, a.stream, (const int8_t *)a.in[0],
+                                (const int8_t *)a.wt, wscales(a.wt, elems), a.bias, (const int8_t *)a.in[1],
+                                (TO *)a.out, d, scales_of(a)));
     return cudaGetLastError();
 }
 
@@ -565,10 +599,10 @@ cudaError_t q8_conv_dp4a(const LaunchArgs &a) {
 // dense: one warp per output feature, NB images per pass over its weight row
 // (16-byte loads and dp4a when in_features % 16 == 0)
 // ===========================================================================
-template <int NB, bool V16>
+template <int NB, bool V16, typename TO>
 __global__ void __launch_bounds__(256) q8_dense_kernel(const int8_t *__restrict__ x, const int8_t *__restrict__ w,
                                                        const float *__restrict__ ws, const float *__restrict__ bias,
-                                                       int8_t *__restrict__ y, int N, int I, int O, int act,
+                                                       TO *__restrict__ y, int N, int I, int O, int act,
                                                        Q8Scales q) {
     griddep_launch();
     griddep_wait();
@@ -608,7 +642,7 @@ __global__ void __launch_bounds__(256) q8_dense_kernel(const int8_t *__restrict_
 #pragma unroll
             for (int b = 1; b < NB; ++b)
                 if (lane == b) v = acc[b];
-            y[(int64_t)(n0 + lane) * O + o] = q8_epilogue(v, q.s_x, ws[o], bias[o], 0.0f, act, q.inv_out);
+            y[(int64_t)(n0 + lane) * O + o] = q8_out<TO>(q8_value(v, q.s_x, ws[o], bias[o], 0.0f, act), q.inv_out);
         }
     }
 }
@@ -621,18 +655,22 @@ cudaError_t q8_dense(const LaunchArgs &a) {
     const dim3 grid((unsigned)((O + 7) / 8));
     const bool v16 = I % 16 == 0 && (uintptr_t)a.in[0] % 16 == 0 && (uintptr_t)a.wt % 16 == 0;
 #define SN_Q8_DENSE(NB)                                                                                        \
-    (v16 ? launch_pdl(q8_dense_kernel<NB, true>, grid, 256, 0, a.stream, (const int8_t *)a.in[0],             \
-                      (const int8_t *)a.wt, ws, a.bias, (int8_t *)a.out, N, I, O, l.act, scales_of(a))        \
-         : launch_pdl(q8_dense_kernel<NB, false>, grid, 256, 0, a.stream, (const int8_t *)a.in[0],            \
-                      (const int8_t *)a.wt, ws, a.bias, (int8_t *)a.out, N, I, O, l.act, scales_of(a)))
-    if (N <= 1)
+    SN_Q8_OUT_SWITCH(out_dtype(a), TO,                                                                         \
+                     (v16 ? launch_pdl(q8_dense_kernel<NB, true, TO>, grid, 256, 0, a.stream,                  \
+                                       (const int8_t *)a.in[0], (const int8_t *)a.wt, ws, a.bias, (TO *)a.out, \
+                                       N, I, O, l.act, scales_of(a))                                           \
+                          : launch_pdl(q8_dense_kernel<NB, false, TO>, grid, 256, 0, a.stream,                 \
+                                       (const int8_t *)a.in[0], (const int8_t *)a.wt, ws, a.bias, (TO *)a.out, \
+                                       N, I, O, l.act, scales_of(a))))
+    if (N <= 1) {
         SN_Q8_DENSE(1);
-    else if (N <= 2)
+    } else if (N <= 2) {
         SN_Q8_DENSE(2);
-    else if (N <= 4)
+    } else if (N <= 4) {
         SN_Q8_DENSE(4);
-    else
+    } else {
         SN_Q8_DENSE(8);
+    }
 #undef SN_Q8_DENSE
     return cudaGetLastError();
 }
@@ -640,8 +678,8 @@ cudaError_t q8_dense(const LaunchArgs &a) {
 // ===========================================================================
 // max pool, global average pool, add, squeeze-and-excite scale
 // ===========================================================================
-template <bool NHWC>
-__global__ void q8_maxpool_kernel(const int8_t *__restrict__ x, int8_t *__restrict__ y, int N, int C, int H, int W,
+template <bool NHWC, typename TO>
+__global__ void q8_maxpool_kernel(const int8_t *__restrict__ x, TO *__restrict__ y, int N, int C, int H, int W,
                                   int P, int Q, sn_pool_params pp, float s_x, float inv) {
     griddep_launch();
     griddep_wait();
@@ -672,7 +710,7 @@ __global__ void q8_maxpool_kernel(const int8_t *__restrict__ x, int8_t *__restri
                 m = max(m, (int)x[xi]);
             }
         }
-        y[i] = q8_code(__fmul_rn((float)m, s_x), inv);
+        y[i] = q8_out<TO>(__fmul_rn((float)m, s_x), inv);
     }
 }
 
@@ -680,23 +718,25 @@ cudaError_t q8_maxpool(const LaunchArgs &a) {
     if (!scales_ok(a, 1)) return cudaErrorInvalidValue;
     const Shape &i = a.in_shapes[0], &o = a.layer->out;
     const int64_t total = o.numel();
-    const float inv = 1.0f / a.qs_out;
-    if (a.schema.layout == SN_NHWC)
-        launch_pdl(q8_maxpool_kernel<true>, grid_for(total, 256), 256, 0, a.stream, (const int8_t *)a.in[0],
-                   (int8_t *)a.out, (int)i.n, (int)i.c, (int)i.h, (int)i.w, (int)o.h, (int)o.w, a.layer->pool,
-                   a.qs_in[0], inv);
-    else
-        launch_pdl(q8_maxpool_kernel<false>, grid_for(total, 256), 256, 0, a.stream, (const int8_t *)a.in[0],
-                   (int8_t *)a.out, (int)i.n, (int)i.c, (int)i.h, (int)i.w, (int)o.h, (int)o.w, a.layer->pool,
-                   a.qs_in[0], inv);
+    const float inv = scales_of(a).inv_out;
+    SN_Q8_OUT_SWITCH(out_dtype(a), TO, {
+        if (a.schema.layout == SN_NHWC)
+            launch_pdl(q8_maxpool_kernel<true, TO>, grid_for(total, 256), 256, 0, a.stream, (const int8_t *)a.in[0],
+                       (TO *)a.out, (int)i.n, (int)i.c, (int)i.h, (int)i.w, (int)o.h, (int)o.w, a.layer->pool,
+                       a.qs_in[0], inv);
+        else
+            launch_pdl(q8_maxpool_kernel<false, TO>, grid_for(total, 256), 256, 0, a.stream,
+                       (const int8_t *)a.in[0], (TO *)a.out, (int)i.n, (int)i.c, (int)i.h, (int)i.w, (int)o.h,
+                       (int)o.w, a.layer->pool, a.qs_in[0], inv);
+    });
     return cudaGetLastError();
 }
 
 // NCHW: one warp per (n, c) plane; NHWC: one thread per (n, c), consecutive
 // threads on consecutive channels.  The code sum is exact; its value is
 // (float(sum) * s_x) / (H*W), two roundings.
-template <bool NHWC>
-__global__ void q8_gap_kernel(const int8_t *__restrict__ x, int8_t *__restrict__ y, int N, int C, int HW, float s_x,
+template <bool NHWC, typename TO>
+__global__ void q8_gap_kernel(const int8_t *__restrict__ x, TO *__restrict__ y, int N, int C, int HW, float s_x,
                               float inv) {
     griddep_launch();
     griddep_wait();
@@ -707,7 +747,7 @@ __global__ void q8_gap_kernel(const int8_t *__restrict__ x, int8_t *__restrict__
             const int c = (int)(t % C);
             int sum = 0;
             for (int j = 0; j < HW; ++j) sum += x[(n * HW + j) * C + c];
-            y[t] = q8_code(__fdiv_rn(__fmul_rn(__int2float_rn(sum), s_x), (float)HW), inv);
+            y[t] = q8_out<TO>(__fdiv_rn(__fmul_rn(__int2float_rn(sum), s_x), (float)HW), inv);
         }
     } else {
         const int lane = threadIdx.x & 31;
@@ -717,7 +757,7 @@ __global__ void q8_gap_kernel(const int8_t *__restrict__ x, int8_t *__restrict__
             int sum = 0;
             for (int j = lane; j < HW; j += 32) sum += x[t * HW + j];
             for (int off = 16; off; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
-            if (lane == 0) y[t] = q8_code(__fdiv_rn(__fmul_rn(__int2float_rn(sum), s_x), (float)HW), inv);
+            if (lane == 0) y[t] = q8_out<TO>(__fdiv_rn(__fmul_rn(__int2float_rn(sum), s_x), (float)HW), inv);
         }
     }
 }
@@ -725,22 +765,24 @@ __global__ void q8_gap_kernel(const int8_t *__restrict__ x, int8_t *__restrict__
 cudaError_t q8_gap(const LaunchArgs &a) {
     if (!scales_ok(a, 1)) return cudaErrorInvalidValue;
     const Shape &i = a.in_shapes[0];
-    const float inv = 1.0f / a.qs_out;
+    const float inv = scales_of(a).inv_out;
     const int64_t nc = i.n * i.c;
     if (i.h * i.w >= (1 << 23)) return cudaErrorInvalidValue;  // int32 sums stay exact
-    if (a.schema.layout == SN_NHWC)
-        launch_pdl(q8_gap_kernel<true>, grid_for(nc, 256), 256, 0, a.stream, (const int8_t *)a.in[0],
-                   (int8_t *)a.out, (int)i.n, (int)i.c, (int)(i.h * i.w), a.qs_in[0], inv);
-    else
-        launch_pdl(q8_gap_kernel<false>, grid_for(nc * 32, 256), 256, 0, a.stream, (const int8_t *)a.in[0],
-                   (int8_t *)a.out, (int)i.n, (int)i.c, (int)(i.h * i.w), a.qs_in[0], inv);
+    SN_Q8_OUT_SWITCH(out_dtype(a), TO, {
+        if (a.schema.layout == SN_NHWC)
+            launch_pdl(q8_gap_kernel<true, TO>, grid_for(nc, 256), 256, 0, a.stream, (const int8_t *)a.in[0],
+                       (TO *)a.out, (int)i.n, (int)i.c, (int)(i.h * i.w), a.qs_in[0], inv);
+        else
+            launch_pdl(q8_gap_kernel<false, TO>, grid_for(nc * 32, 256), 256, 0, a.stream, (const int8_t *)a.in[0],
+                       (TO *)a.out, (int)i.n, (int)i.c, (int)(i.h * i.w), a.qs_in[0], inv);
+    });
     return cudaGetLastError();
 }
 
 // MUL = false: y = act(a * s_a + b * s_b); MUL = true: y = act((a * s_a) *
 // (b[n, c] * s_b)), b an N x C blob
-template <bool MUL, bool NHWC>
-__global__ void q8_binary_kernel(const int8_t *__restrict__ a, const int8_t *__restrict__ b, int8_t *__restrict__ y,
+template <bool MUL, bool NHWC, typename TO>
+__global__ void q8_binary_kernel(const int8_t *__restrict__ a, const int8_t *__restrict__ b, TO *__restrict__ y,
                                  int64_t total, int C, int64_t HW, float s_a, float s_b, int act, float inv) {
     griddep_launch();
     griddep_wait();
@@ -755,7 +797,7 @@ __global__ void q8_binary_kernel(const int8_t *__restrict__ a, const int8_t *__r
         } else {
             v = __fadd_rn(va, __fmul_rn((float)b[i], s_b));
         }
-        y[i] = q8_code(q8_act(v, act), inv);
+        y[i] = q8_out<TO>(q8_act(v, act), inv);
     }
 }
 
@@ -764,16 +806,18 @@ static cudaError_t q8_binary(const LaunchArgs &a) {
     if (!scales_ok(a, 2)) return cudaErrorInvalidValue;
     const Shape &o = a.layer->out;
     const int64_t total = o.numel();
-    const float inv = 1.0f / a.qs_out;
+    const float inv = scales_of(a).inv_out;
     const int act = a.layer->act;
-    if (a.schema.layout == SN_NHWC)
-        launch_pdl(q8_binary_kernel<MUL, true>, grid_for(total, 256), 256, 0, a.stream, (const int8_t *)a.in[0],
-                   (const int8_t *)a.in[1], (int8_t *)a.out, total, (int)o.c, o.h * o.w, a.qs_in[0], a.qs_in[1],
-                   act, inv);
-    else
-        launch_pdl(q8_binary_kernel<MUL, false>, grid_for(total, 256), 256, 0, a.stream, (const int8_t *)a.in[0],
-                   (const int8_t *)a.in[1], (int8_t *)a.out, total, (int)o.c, o.h * o.w, a.qs_in[0], a.qs_in[1],
-                   act, inv);
+    SN_Q8_OUT_SWITCH(out_dtype(a), TO, {
+        if (a.schema.layout == SN_NHWC)
+            launch_pdl(q8_binary_kernel<MUL, true, TO>, grid_for(total, 256), 256, 0, a.stream,
+                       (const int8_t *)a.in[0], (const int8_t *)a.in[1], (TO *)a.out, total, (int)o.c, o.h * o.w,
+                       a.qs_in[0], a.qs_in[1], act, inv);
+        else
+            launch_pdl(q8_binary_kernel<MUL, false, TO>, grid_for(total, 256), 256, 0, a.stream,
+                       (const int8_t *)a.in[0], (const int8_t *)a.in[1], (TO *)a.out, total, (int)o.c, o.h * o.w,
+                       a.qs_in[0], a.qs_in[1], act, inv);
+    });
     return cudaGetLastError();
 }
 

@@ -231,6 +231,25 @@ int32_t kernels_per_launch(int32_t r, int32_t v, const Layer &l, const std::vect
     return 1 + split;
 }
 
+std::vector<sn_schema> fused_outputs(int32_t r, const Layer &l, sn_schema s) {
+    // qint8 routines can leave their fp32 result in a float schema of the
+    // same layout instead of requantising it (dequantisation fused into the
+    // epilogue)
+    if (s.dtype != SN_QI8) return {};
+    (void)l;
+    switch (r) {
+    case R_CONV_DIRECT:
+    case R_CONV_DP4A:
+    case R_DW_DIRECT:
+    case R_MAXPOOL:
+    case R_GAP:
+    case R_ADD:
+    case R_MUL:
+    case R_DENSE: return {{SN_F16, s.layout}, {SN_BF16, s.layout}, {SN_F32, s.layout}};
+    default: return {};
+    }
+}
+
 int32_t childnet_stages(int32_t r, sn_schema s) {
     if (s.dtype == SN_QI8) return 1;
     switch (r) {

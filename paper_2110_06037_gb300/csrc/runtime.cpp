@@ -50,8 +50,12 @@ sn_status build_plan(Graph *g, cudaStream_t st) {
     const int32_t m_in = g->n_in();
     const Layer &OL = g->layers[n - 1];  // auxiliary output layer: its inputs are the net outputs
     const int32_t m_out = (int32_t)OL.inputs.size();
-    std::vector<sn_schema> sch(n);
-    for (int32_t i = 0; i < n; ++i) sch[i] = g->schemas[g->cands[g->path_cand[i]].schema];
+    // the schema each layer's routine reads its inputs in and writes its output in
+    std::vector<sn_schema> sch(n), sch_out(n);
+    for (int32_t i = 0; i < n; ++i) {
+        sch[i] = g->schemas[g->cands[g->path_cand[i]].schema];
+        sch_out[i] = g->schemas[cand_out(g->cands[g->path_cand[i]])];
+    }
     // external slots: the caller's input buffers 0..m_in-1, then its output
     // buffers m_in..m_in+m_out-1
     for (int32_t k = 0; k < m_in; ++k) schema_slot(g, g->layers[k].out, g->in_schema, g->layers[k].qscale);
@@ -89,7 +93,7 @@ sn_status build_plan(Graph *g, cudaStream_t st) {
                     break;
                 }
             int32_t src = out_slot[j];
-            const bool same = schema_eq(sch[j], sch[i]);
+            const bool same = schema_eq(sch_out[j], sch[i]);
             if (i == n - 1) {
                 // output layer: adapt into the caller's buffer unless the
                 // producer already wrote there
@@ -118,10 +122,10 @@ sn_status build_plan(Graph *g, cudaStream_t st) {
             op.in_slots.push_back(src);
         }
         if (i == n - 1) break;
-        if (out_index[i] >= 0 && schema_eq(sch[i], g->out_schema)) {
+        if (out_index[i] >= 0 && schema_eq(sch_out[i], g->out_schema)) {
             op.out_slot = m_in + out_index[i];  // a net output written in place
         } else {
-            schema_slot(g, L.out, sch[i], L.qscale);
+            schema_slot(g, L.out, sch_out[i], L.qscale);
             op.out_slot = (int32_t)g->slots.size() - 1;
         }
         out_slot[i] = op.out_slot;
@@ -179,6 +183,7 @@ static sn_status launch_op(Graph *g, const PlanOp &op, const IoPtrs &io, cudaStr
     a.routine = c.routine;
     a.variant = c.variant;
     a.schema = g->schemas[c.schema];
+    a.out_schema = g->schemas[cand_out(c)];
     for (size_t k = 0; k < op.in_slots.size(); ++k) {
         a.in[k] = ptr(op.in_slots[k]);
         a.in_shapes.push_back(g->layers[L.inputs[k]].out);
@@ -303,7 +308,7 @@ std::string signature(const Graph *g, int32_t i, const Candidate &c) {
     o << p.c_in << ',' << p.c_out << ',' << p.kh << ',' << p.kw << ',' << p.sh << ',' << p.sw << ','
       << p.ph << ',' << p.pw << ',' << p.dh << ',' << p.dw << ',' << p.groups << ',' << L.act << ','
       << L.pool.kh << ',' << L.pool.sh << ',' << L.pool.ph << ',' << L.dense_in << ',' << L.dense_out
-      << '|' << c.routine << '/' << c.variant << '/' << c.schema;
+      << '|' << c.routine << '/' << c.variant << '/' << c.schema << '>' << cand_out(c);
     return o.str();
 }
 
@@ -396,6 +401,7 @@ static sn_status profile_graph_on(Graph *g, const sn_profile_opts &o, cudaStream
             a.in[0] = sc.in0.ptr;
             a.in[1] = in.size() > 1 ? sc.in1.ptr : nullptr;  // a residual only where the layer has one
             a.out = sc.out.ptr;
+            a.out_schema = g->schemas[cand_out(cd)];
             a.stream = st;
             a.qs_in[0] = a.qs_in[1] = a.qs_out = kProfileQScale;
             if (k::fill_pattern(sc.in0.ptr, s.dtype, in[0].numel(), 1234u + i, 1.0f, st) != cudaSuccess ||
@@ -449,16 +455,20 @@ static sn_status profile_graph_on(Graph *g, const sn_profile_opts &o, cudaStream
             seen.emplace(sig, t);
         }
     }
-    // --- unit profiling of adapt routines: every edge, every ordered pair ---
-    std::vector<int64_t> F;
-    std::vector<int32_t> argF;
-    fastest_per_schema(*g, F, argF);
+    // --- unit profiling of adapt routines: every edge, every ordered pair of
+    // a schema its producer can write and one its consumer can read ---
+    std::vector<int64_t> Fw((size_t)n * ns, kInf), F((size_t)n * ns, kInf);
+    for (const Candidate &c : g->cands) {
+        int64_t &w = Fw[(size_t)c.layer * ns + cand_out(c)], &r = F[(size_t)c.layer * ns + c.schema];
+        w = std::min(w, c.cost);
+        r = std::min(r, c.cost);
+    }
     std::map<std::string, int64_t> seen_a;
     for (size_t e = 0; e < g->edges.size() && rc == SN_OK; ++e) {
         auto [j, i] = g->edges[e];
         const Shape s = g->layers[j].out;
         for (int32_t a = 0; a < ns && rc == SN_OK; ++a) {
-            if (F[(size_t)j * ns + a] == kInf) continue;
+            if (Fw[(size_t)j * ns + a] == kInf) continue;
             for (int32_t b = 0; b < ns && rc == SN_OK; ++b) {
                 if (a == b || F[(size_t)i * ns + b] == kInf) continue;
                 std::ostringstream key;
@@ -626,18 +636,13 @@ sn_status calibrate(Graph *g, const void *in, cudaStream_t st) {
     // candidates
     const std::vector<Candidate> saved_costs = g->cands;
     for (auto &c : g->cands)
-        if (g->schemas[c.schema].dtype == SN_QI8) c.cost = kInf;
-    std::vector<int32_t> schema_of;
+        if (g->schemas[c.schema].dtype == SN_QI8 || g->schemas[cand_out(c)].dtype == SN_QI8) c.cost = kInf;
+    std::vector<int32_t> pc;
     int64_t total = kInf;
-    sn_status rc = select_dprs(*g, schema_of, total);
-    std::vector<int64_t> F;
-    std::vector<int32_t> argF;
-    if (rc == SN_OK) fastest_per_schema(*g, F, argF);
+    sn_status rc = select_path(*g, SN_SELECT_DPRS, pc, total);
     g->cands = saved_costs;
     if (rc != SN_OK || total == kInf)
         return fail(SN_ESTATE, "sn_calibrate: no float path of finite cost (profile or set the costs first)");
-    std::vector<int32_t> pc(n);
-    for (int32_t i = 0; i < n; ++i) pc[i] = argF[(size_t)i * ns + schema_of[i]];
 
     const bool had_path = g->has_path;
     const std::vector<int32_t> saved_path = g->path_cand;

@@ -90,9 +90,11 @@ struct Layer {
 };
 
 struct Candidate {
-    int32_t routine, variant, schema, layer;
+    int32_t routine, variant, schema, layer;  // schema: the one the routine reads
     int64_t cost;
+    int32_t out_schema = -1;  // the schema it writes; -1 = the one it reads
 };
+inline int32_t cand_out(const Candidate &c) { return c.out_schema < 0 ? c.schema : c.out_schema; }
 
 struct Buffer {  // device allocation owned by the graph
     void *ptr = nullptr;
@@ -121,6 +123,7 @@ struct LaunchArgs {
     std::vector<Shape> in_shapes;
     const void *in[2] = {nullptr, nullptr};
     void *out = nullptr;
+    sn_schema out_schema{-1, -1};  // schema of `out` when the routine writes another (fused boundary)
     const void *wt = nullptr;   // prepared weights in the routine's format
     const float *bias = nullptr;
     void *ws = nullptr;         // workspace
@@ -229,10 +232,18 @@ bool stage_uses_variant(int32_t routine, int32_t stage);
 sn_status launch_routine_stage(const LaunchArgs &a, int32_t stage);
 int32_t kernels_per_launch(int32_t routine, int32_t variant, const Layer &layer, const std::vector<Shape> &in,
                            sn_schema s);
+// schemas other than `s` that the routine can write its output in, reading
+// its inputs in `s` (a fused boundary: dequantisation in a qint8 epilogue)
+std::vector<sn_schema> fused_outputs(int32_t routine, const Layer &layer, sn_schema s);
 
 // selection (section IV)
 sn_status select_dprs(const Graph &g, std::vector<int32_t> &schema_of, int64_t &total);
 sn_status select_brute(const Graph &g, std::vector<int32_t> &schema_of, int64_t &total);
+// either method on the graph's candidates: when some routine writes a schema
+// other than the one it reads, a layer's state is the pair (read, written)
+// and an edge costs the adapt from its producer's written schema to its
+// consumer's read one.  cand_of[i] = the chosen candidate of layer i.
+sn_status select_path(const Graph &g, int32_t method, std::vector<int32_t> &cand_of, int64_t &total);
 void fastest_per_schema(const Graph &g, std::vector<int64_t> &F, std::vector<int32_t> &argF);
 
 // plan + run

@@ -1,0 +1,89 @@
+"""Fused-boundary routines (routines that write a schema other than the one
+they read: a qint8 routine with the dequantisation in its epilogue): the
+candidates, and DPRS over (read, written) schema pairs against an exhaustive
+search over one candidate per layer.  CPU only: costs are injected."""
+import numpy as np
+import pytest
+
+import oracle
+from oracle.paths import brute_force_candidates
+from paper_2110_06037_gb300 import SN_SELECT_BRUTE, SN_SELECT_DPRS, SnError, build_graph
+from paper_2110_06037_gb300 import _sn
+
+from test_dprs import random_net
+
+INF = oracle.INF
+LAMBDA = [("f16", "nhwc"), ("qi8", "nhwc"), ("f16", "nchw")]
+
+
+def _graph(layers, ns):
+    return build_graph(layers, (1, 4, 3, 3), ("f16", "nhwc"), ("f16", "nhwc"), LAMBDA[:ns], torch_alloc=False)
+
+
+def test_qint8_routines_offer_float_outputs_of_their_layout():
+    rng = np.random.default_rng(1)
+    g = _graph(random_net(rng, 3), 3)
+    t = g.cost_table()
+    uni = g.schema_universe()
+    fused = [c for c in range(len(t["cost"])) if t["out_schema"][c] != t["schema"][c]]
+    assert fused
+    for c in fused:
+        rd, wr = uni[t["schema"][c]], uni[t["out_schema"][c]]
+        assert rd[0] == "qi8" and wr[0] != "qi8" and rd[1] == wr[1]
+        # the same routine and parameter exists with its ordinary output
+        assert any(t["routine"][k] == t["routine"][c] and t["variant"][k] == t["variant"][c]
+                   and t["schema"][k] == t["schema"][c] and t["out_schema"][k] == t["schema"][c]
+                   and t["layer"][k] == t["layer"][c] for k in range(len(t["cost"])))
+    # float routines never change the schema they write
+    assert all(uni[t["schema"][c]][0] == "qi8" for c in fused)
+
+
+def _random_costs(g, rng):
+    t = g.cost_table()
+    c = rng.integers(1, 1000, size=len(t["cost"])).astype(np.int64)
+    c[rng.random(len(c)) < 0.1] = INF
+    c[t["routine"] == 0] = 0
+    t["cost"] = c
+    a = rng.integers(0, 400, size=t["adapt"].shape).astype(np.int64)
+    a[rng.random(a.shape) < 0.05] = INF
+    for e in range(a.shape[0]):
+        np.fill_diagonal(a[e], 0)
+    t["adapt"] = a
+    g.set_cost_table(t)
+    return t
+
+
+def _cands_per_layer(t):
+    out = []
+    for i in range(t["n_layers"]):
+        idx = np.flatnonzero(t["layer"] == i)
+        out.append([(int(t["cost"][c]), int(t["schema"][c]), int(t["out_schema"][c])) for c in idx])
+    return out
+
+
+@pytest.mark.parametrize("seed", range(40))
+def test_dprs_over_schema_pairs_equals_exhaustive_search(seed):
+    rng = np.random.default_rng(9100 + seed)
+    ns = 2 if seed % 2 else 3
+    layers = random_net(rng, int(rng.integers(1, 4)))
+    g = _graph(layers, ns)
+    t = _random_costs(g, rng)
+    per = _cands_per_layer(t)
+    if np.prod([len(c) for c in per], dtype=float) > 3e5:
+        pytest.skip("candidate product too large to enumerate")
+    ref, pick = brute_force_candidates(per, t["edges"].tolist(), t["adapt"])
+    try:
+        tot, sch, cand = g.select_path(SN_SELECT_DPRS)
+    except SnError as e:
+        assert ref == INF and e.status == _sn.SN_EINFEASIBLE
+        return
+    assert tot == ref
+    # the chosen candidates realise the total
+    chosen = [(int(t["cost"][c]), int(t["schema"][c]), int(t["out_schema"][c])) for c in cand]
+    realised = sum(c[0] for c in chosen)
+    for e, (u, v) in enumerate(t["edges"].tolist()):
+        if chosen[u][2] != chosen[v][1]:
+            realised += int(t["adapt"][e][chosen[u][2]][chosen[v][1]])
+    assert realised == ref
+    if len(layers) <= 3:
+        assert g.select_path(SN_SELECT_BRUTE)[0] == ref

@@ -291,3 +291,75 @@ def test_hybrid_dprs_equals_brute_force_and_runs():
     ref = run_net(layers, x)
     got = from_device(y, ("f32", "nchw"))
     assert maxrel(got.reshape(ref.shape), ref) < 0.1
+
+
+# ------------------------------------------------------- fused boundaries
+FUSED_CASES = [
+    ("conv2/direct", lambda rng: conv_layer(rng, 8, 12, 3, 1, 1, act="relu6")),
+    ("conv2/igemm_dp4a", lambda rng: conv_layer(rng, 16, 20, 3, 2, 1)),
+    ("dwconv2/direct", lambda rng: conv_layer(rng, 16, 16, 3, 1, 1, dw=True)),
+    ("maxpool/direct", lambda rng: {"type": "maxpool", "inputs": [-1],
+                                    "params": dict(kh=3, kw=3, sh=2, sw=2, ph=1, pw=1)}),
+    ("gap/reduce", lambda rng: {"type": "gap", "inputs": [-1]}),
+    ("add/eltwise", lambda rng: {"type": "add", "inputs": [-1, -1], "params": dict(act="relu")}),
+]
+
+
+@pytest.mark.parametrize("out_dt", ["f16", "f32", "bf16"])
+@pytest.mark.parametrize("case", range(len(FUSED_CASES)))
+def test_fused_dequantisation_matches_oracle(case, out_dt):
+    """A qint8 routine writing a float schema: the fp32 result rounded to that
+    dtype, bit for bit."""
+    import torch
+    name, make = FUSED_CASES[case]
+    rng = np.random.default_rng(500 + case)
+    layer = make(rng)
+    c = layer["params"]["c_in"] if "c_in" in layer.get("params", {}) else 16
+    q_in = rng.integers(-127, 128, (2, c, 11, 9)).astype(np.int8)
+    s_in = F32(0.04)
+    scales = _out_scales([layer], q_in, s_in)
+    sch = [("qi8", "nhwc"), (out_dt, "nhwc")]
+    g = build_graph([layer], q_in.shape, ("qi8", "nhwc"), (out_dt, "nhwc"), sch)
+    g.set_qscale(-1, float(s_in))
+    g.set_qscale(0, float(scales[0]))
+    t = g.cost_table()
+    hit = [k for k in range(len(t["cost"])) if t["layer"][k] == 1 and routine_name(int(t["routine"][k])) == name
+           and t["schema"][k] == 0 and t["out_schema"][k] == 1]
+    assert hit, name
+    g.set_path([int(np.flatnonzero(t["layer"] == 0)[0]), hit[0], int(np.flatnonzero(t["layer"] == 2)[0])])
+    y = g.run(codes_to_device(q_in, "nhwc"))
+    torch.cuda.synchronize()
+    got = from_device(y, (out_dt, "nhwc"))
+    n_in = len(layer["inputs"])
+    want = q8.run_layer(layer, [q_in] * n_in, [s_in] * n_in, scales[0], out_dtype=out_dt).astype(np.float64)
+    assert np.array_equal(got.reshape(want.shape), want), name
+    # one launch: no dequantise adapt on the path
+    assert g.plan_stats()[0] == 1
+
+
+def test_hybrid_with_fused_boundaries_equals_exhaustive_search_and_runs():
+    import torch
+    from oracle.paths import brute_force_candidates
+    rng = np.random.default_rng(46)
+    layers = small_net(rng)[:5]  # stem, conv, residual conv, pool, depthwise
+    x = rng.standard_normal((1, 3, 16, 16)).astype(F32)
+    g = build_graph(layers, x.shape, ("f16", "nhwc"), ("f16", "nhwc"), [("f16", "nhwc"), ("qi8", "nhwc")])
+    g.profile(warmup=1, iters=3, topk=1, passes=2)
+    g.calibrate(to_device(x, ("f16", "nhwc")))
+    t = g.cost_table()
+    assert (t["out_schema"] != t["schema"]).any()
+    per = []  # per layer the fastest candidate of each (read, written) pair (Eq. 1)
+    for i in range(t["n_layers"]):
+        best = {}
+        for c in np.flatnonzero(t["layer"] == i):
+            key = (int(t["schema"][c]), int(t["out_schema"][c]))
+            if key not in best or t["cost"][c] < best[key]:
+                best[key] = int(t["cost"][c])
+        per.append([(v, k[0], k[1]) for k, v in sorted(best.items())])
+    ref, _ = brute_force_candidates(per, t["edges"].tolist(), t["adapt"])
+    tot, _, _ = g.select_path()
+    assert tot == ref
+    y = g.run(to_device(x, ("f16", "nhwc")))
+    torch.cuda.synchronize()
+    want = run_net(layers, x)
+    assert maxrel(from_device(y, ("f16", "nhwc")).reshape(want.shape), want) < 0.1

@@ -234,3 +234,23 @@ def test_qint8_net_tracks_the_float_net():
     assert got.shape == ref.reshape(2, 4).shape or got.shape == ref.shape
     err = np.abs(got.reshape(ref.shape).astype(np.float64) - ref)
     assert err.max() <= 4 * float(scales[-1]) + 1e-6
+
+
+def test_fused_dequantisation_output_is_the_unrounded_value():
+    """A qint8 routine that writes a float schema leaves act(conv + bias) in
+    that dtype instead of requantising: with unit scales and integer weights
+    that is the exact integer sum (no division by the output scale)."""
+    rng = np.random.default_rng(19)
+    x = rng.integers(-127, 128, (1, 4, 5, 5)).astype(np.int8)
+    w = _int_weights(rng, (3, 4, 3, 3))
+    qw, sw = q8.quantize_weights(w)
+    b = rng.integers(-50, 50, 3).astype(F32)
+    got = q8.conv2d(x, 1.0, qw, sw, b, 256.0, pad=(1, 1), act="relu", out_dtype="f32")
+    acc = _brute_conv(x, qw, (1, 1), (1, 1), (1, 1), 1)
+    want = np.vectorize(lambda v: float(v))(acc).astype(np.float64) + b.reshape(1, 3, 1, 1)
+    assert np.array_equal(got.astype(np.float64), np.maximum(want, 0))
+    # and in fp16 it is that value rounded to nearest even
+    h = q8.conv2d(x, 1.0, qw, sw, b, 256.0, pad=(1, 1), act="relu", out_dtype="f16")
+    assert np.array_equal(h, oracle.round_to(got.astype(np.float32), "f16"))
+    # requantising it gives the ordinary qint8 output
+    assert np.array_equal(q8.requantize(got, 256.0), q8.conv2d(x, 1.0, qw, sw, b, 256.0, pad=(1, 1), act="relu"))
