@@ -576,7 +576,7 @@ def run_hybrid(args):
                 if scales_from is not None:
                     for i in range(-1, len(layers)):
                         g.set_qscale(i, scales_from.get_qscale(i))
-                g.profile(warmup=2, iters=5, topk=1, passes=2)
+                g.profile(warmup=3, iters=10, topk=2, passes=3)
                 if scales_from is None and any(d == "qi8" for d, _ in schemas):
                     g.calibrate(xd)
                 total, sch, cands = g.select_path(sn.SN_SELECT_DPRS)
