@@ -326,27 +326,60 @@ def main():
     value = ws * args.batch / (ms / 1e3)
 
     # ---------------- e2e through the public API with host buffers ----------------
+    # Every step copies its input batch from pinned host memory and reads its
+    # logits back to the host, inside the timed region.  As a serving loop
+    # would, the next step's host->device copy runs on a copy stream into one
+    # of two staging buffers while the current step computes; the step then
+    # moves its batch into the net's input buffer (device to device) and its
+    # logits go back to the host on the copy stream.
     xh = torch.from_numpy(x).to(torch.bfloat16).pin_memory()
-    oh = torch.empty(out.shape, dtype=out.dtype).pin_memory()
+    oh = [torch.empty(out.shape, dtype=out.dtype).pin_memory() for _ in range(2)]
     xin = torch.empty_like(xd)
+    stage = [torch.empty_like(xd) for _ in range(2)]
+    ostage = [torch.empty_like(out) for _ in range(2)]
+    cstream = torch.cuda.Stream()
+
+    def e2e_steps(n):
+        ev = lambda: torch.cuda.Event()
+        h_done, used, r_done, d_done = ([ev() for _ in range(n)] for _ in range(4))
+        cstream.wait_stream(stream)
+        with torch.cuda.stream(cstream):
+            stage[0].copy_(xh, non_blocking=True)
+            h_done[0].record(cstream)
+        for k in range(n):
+            if k + 1 < n:
+                with torch.cuda.stream(cstream):
+                    if k >= 1:
+                        cstream.wait_event(used[k - 1])  # staging buffer (k+1)%2 was read by step k-1
+                    stage[(k + 1) % 2].copy_(xh, non_blocking=True)
+                    h_done[k + 1].record(cstream)
+            stream.wait_event(h_done[k])
+            with torch.cuda.stream(stream):
+                xin.copy_(stage[k % 2], non_blocking=True)
+                used[k].record(stream)
+                g.run(xin, out)
+                if k >= 2:
+                    stream.wait_event(d_done[k - 2])  # logits staging buffer k%2 read back by step k-2
+                ostage[k % 2].copy_(out, non_blocking=True)
+                r_done[k].record(stream)
+            with torch.cuda.stream(cstream):
+                cstream.wait_event(r_done[k])
+                oh[k % 2].copy_(ostage[k % 2], non_blocking=True)
+                d_done[k].record(cstream)
+        stream.wait_stream(cstream)
+
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    with torch.cuda.stream(stream):
-        for _ in range(2):
-            xin.copy_(xh, non_blocking=True)
-            g.run(xin, out)
-            oh.copy_(out, non_blocking=True)
-        stream.synchronize()
-        e0.record(stream)
-        for _ in range(args.steps):
-            xin.copy_(xh, non_blocking=True)
-            g.run(xin, out)
-            oh.copy_(out, non_blocking=True)
-        e1.record(stream)
+    e2e_steps(3)
+    stream.synchronize()
+    e0.record(stream)
+    e2e_steps(args.steps)
+    e1.record(stream)
     stream.synchronize()
     e2e_ms = e0.elapsed_time(e1) / args.steps
     e2e = {"value": args.batch / (e2e_ms / 1e3), "unit": "images/s",
            "h2d_bytes_per_step": xh.numel() * xh.element_size(),
-           "d2h_bytes_per_step": oh.numel() * oh.element_size()}
+           "d2h_bytes_per_step": oh[0].numel() * oh[0].element_size(),
+           "overlap": "next step's host->device copy overlaps this step's compute (two staging buffers)"}
 
     # ---------------- per-routine device time (events around every launch) ----------------
     g.set_option(sn.SN_OPT_CUDA_GRAPH, 0)
