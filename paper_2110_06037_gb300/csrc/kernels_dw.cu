@@ -298,7 +298,7 @@ inline int round_rows(int row_items, int sw) {
 // (one CTA per SM with a ~200 KB ring).  A round's rows must fit the ring
 // with rows to spare for prefetch; whole-channel rows are preferred, since a
 // slice reads each pixel's channels in pieces, which costs DRAM efficiency.
-RingPlan plan_ring(const ConvDims &d, int es) {
+RingPlan plan_ring(const ConvDims &d, int es, bool packed) {
     RingPlan best{0, 0, 0, -1.0};
     const int E = 16 / es;
     const int WB = (d.Q - 1) * d.sw + 3;
@@ -307,15 +307,19 @@ RingPlan plan_ring(const ConvDims &d, int es) {
         if (d.C % CS) continue;
         const size_t slot = ((size_t)WB * CS * es + 127) & ~(size_t)127;
         const int NS = (int)std::min<size_t>(DW_MAX_SLOTS, budget / slot);
-        for (int QB : {4, 2, 1}) {
-            if (QB == 4 && d.sw == 2) continue;  // a 9-column window does not fit the register budget
+        for (int QB : {8, 4, 2, 1}) {
+            // the fp32 accumulators of 4 columns at stride 2 (a 9-column window),
+            // or of 8 columns, do not fit the register budget; packed half2
+            // accumulators (fp16) take half the registers
+            if (QB == 8 && !(packed && d.sw == 1)) continue;
+            if (QB == 4 && d.sw == 2 && !packed) continue;
             const int QBLK = (d.Q + QB - 1) / QB;
             const double colutil = (double)d.Q / (QBLK * QB);
             const int need = std::min(round_rows(QBLK * (CS / E), d.sw), std::min(d.H, (d.P - 1) * d.sw + 3));
             if (NS < need + 1) continue;
             const double spare = std::min(1.0, 0.5 + 0.125 * (NS - need));  // prefetch depth
             const double score =
-                colutil * (QB == 4 ? 1.0 : QB == 2 ? 0.96 : 0.9) * spare * (CS == d.C ? 1.0 : 0.85);
+                colutil * (QB == 8 ? 1.02 : QB == 4 ? 1.0 : QB == 2 ? 0.96 : 0.9) * spare * (CS == d.C ? 1.0 : 0.85);
             if (score > best.score) best = RingPlan{CS, QB, NS, score};
         }
     }
@@ -341,6 +345,10 @@ cudaError_t dispatch_ring(const CUtensorMap &mx, const LaunchArgs &a, const DwRi
                           size_t smem) {
     const T *w = (const T *)a.wt;
     T *y = (T *)a.out;
+    if constexpr (std::is_same<T, __half>::value) {
+        if (SW == 1 && QB == 8) return launch_ring<T, 1, 8>(mx, w, y, p, grid, smem, a.stream);
+        if (SW == 2 && QB == 4) return launch_ring<T, 2, 4>(mx, w, y, p, grid, smem, a.stream);
+    }
     if (SW == 1) {
         if (QB == 4) return launch_ring<T, 1, 4>(mx, w, y, p, grid, smem, a.stream);
         if (QB == 2) return launch_ring<T, 1, 2>(mx, w, y, p, grid, smem, a.stream);
@@ -368,7 +376,7 @@ cudaError_t dw3_nhwc_ring(const LaunchArgs &a, const ConvDims &d) {
     const int es = dtype_size(a.schema.dtype);
     const int WB = (d.Q - 1) * d.sw + 3;
     const size_t hdr = 2 * DW_MAX_SLOTS * 8 + 128;  // barriers and alignment slack
-    const RingPlan pl = plan_ring(d, es);
+    const RingPlan pl = plan_ring(d, es, a.schema.dtype == SN_F16);
     if (pl.score < 0) return cudaErrorNotSupported;
     DwRing p{};
     p.H = d.H;
