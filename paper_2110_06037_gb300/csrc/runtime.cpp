@@ -631,7 +631,7 @@ static sn_status profile_graph_on(Graph *g, const sn_profile_opts &o, cudaStream
 // qint8 calibration (post-training, symmetric, one scale per blob)
 // ---------------------------------------------------------------------------
 sn_status calibrate(Graph *g, const void *in, cudaStream_t st) {
-    const int32_t n = g->n_layers(), ns = g->n_schemas();
+    const int32_t n = g->n_layers();
     // the cheapest float path: DPRS over the current costs without the qint8
     // candidates
     const std::vector<Candidate> saved_costs = g->cands;

@@ -9,7 +9,6 @@ import pytest
 
 import oracle
 from oracle import q8
-from oracle.net import run_layer as run_layer_f64
 from oracle.net import run_net
 from paper_2110_06037_gb300 import build_graph, convert_q, routine_name
 
