@@ -165,3 +165,26 @@ def test_convert_needs_a_scale_for_qint8():
     st = _sn.lib().sn_convert_q(fake, _sn.schema(("f16", "nchw")), fake, _sn.schema(("qi8", "nchw")), shp,
                                 C.c_float(0.0), None)
     assert st == _sn.SN_EINVAL  # bad scale
+
+
+def test_calibration_needs_costs_and_a_single_input():
+    import ctypes as C
+    x, layers = synth.tiny_cnn()
+    g = build_graph(layers, x.shape, ("f32", "nchw"), ("f32", "nchw"), [("f32", "nhwc"), ("qi8", "nhwc")],
+                    torch_alloc=False)
+    fake = C.c_void_p(256)  # refused before any device access
+    assert _sn.lib().sn_calibrate(g.h, fake, None) == _sn.SN_ESTATE  # nothing profiled: no finite float path
+    g2 = Graph((1, 4, 3, 3), ("f32", "nchw"), ("f32", "nchw"), [("f32", "nchw")], torch_alloc=False)
+    g2.add_input((1, 4, 3, 3))
+    w = np.zeros((4, 4, 1, 1), np.float32)
+    p = dict(c_in=4, c_out=4, kh=1, kw=1, sh=1, sw=1, ph=0, pw=0)
+    g2.add_layer(_sn.SN_L_CONV2, p, (-1,), w, None)
+    g2.add_layer(_sn.SN_L_CONV2, p, (-2,), w, None)
+    g2.add_layer(_sn.SN_L_ADD, dict(act="none"), (0, 1), None, None)
+    assert _sn.lib().sn_calibrate(g2.h, fake, None) == _sn.SN_EUNSUPPORTED
+    assert g2.io_counts() == (2, 1)
+    # a second input's scale is set by its id
+    g2.set_qscale(-2, 0.25)
+    assert g2.get_qscale(-2) == 0.25 and g2.get_qscale(-1) == 0.0
+    with pytest.raises(SnError):
+        g2.set_qscale(-3, 1.0)
