@@ -5,6 +5,11 @@ a profiler measures each routine and DPRS (Alg. 1) picks the fastest routine
 path, counting the adapt (cast / layout) conversions between layers.  The
 work happens in libsn.so behind the C ABI in include/sn.h; this package is a
 thin binding over it.
+
+Schemas are (dtype, layout) pairs: dtype "f32" | "f16" | "bf16" | "qi8"
+(symmetric int8 codes with one scale per blob: Graph.set_qscale or
+Graph.calibrate), layout "nchw" | "nhwc".  Nets may have several inputs
+(Graph.add_input) and outputs (Graph.set_outputs, Graph.run_multi).
 """
 from ._sn import (SN_SELECT_BRUTE, SN_SELECT_DPRS, SN_OPT_CHECK, SN_OPT_CUDA_GRAPH, SnError, lib,
                   routine_name, variant_name)
