@@ -87,3 +87,27 @@ def test_dprs_over_schema_pairs_equals_exhaustive_search(seed):
     assert realised == ref
     if len(layers) <= 3:
         assert g.select_path(SN_SELECT_BRUTE)[0] == ref
+
+
+@pytest.mark.parametrize("seed", range(20))
+def test_pair_problem_without_fused_choices_is_the_plain_problem(seed):
+    """With every fused candidate infeasible the pair problem keeps only the
+    diagonal pairs, so its optimum is the plain DPRS optimum over schemas
+    (checked against the oracle's exhaustive search of Def. 2)."""
+    rng = np.random.default_rng(9300 + seed)
+    layers = random_net(rng, int(rng.integers(1, 5)))
+    g = _graph(layers, 2)
+    t = _random_costs(g, rng)
+    t["cost"][t["out_schema"] != t["schema"]] = INF
+    g.set_cost_table(t)
+    ns, n = t["n_schemas"], t["n_layers"]
+    lc = np.array([oracle.fastest_per_schema(t["schema"][t["layer"] == i], t["cost"][t["layer"] == i], ns)
+                   for i in range(n)])
+    ref, _, _ = oracle.brute_force(lc, t["edges"], t["adapt"])
+    try:
+        tot, _, cand = g.select_path(SN_SELECT_DPRS)
+    except SnError as e:
+        assert ref == INF and e.status == _sn.SN_EINFEASIBLE
+        return
+    assert tot == ref
+    assert all(t["out_schema"][c] == t["schema"][c] for c in cand)
