@@ -111,3 +111,21 @@ def test_dprs_equals_brute_force_on_mimo_nets(seed):
         assert tot == lc_ref
     except SnError as e:
         assert lc_ref == oracle.INF and e.status == _sn.SN_EINFEASIBLE
+
+
+def test_oracle_net_with_two_inputs():
+    """The oracle's multi-input forward: a side input of zeros added to a
+    branch leaves the single-input result unchanged, and ids -1 / -2 pick
+    the first / second array."""
+    from oracle.net import run_net
+    rng = np.random.default_rng(3)
+    conv = dict(_conv1x1(4), inputs=[-1])
+    conv["weight"] = rng.standard_normal((4, 4, 1, 1)).astype(np.float32)
+    conv["params"] = dict(conv["params"], act="none")
+    x = rng.standard_normal(SHAPE).astype(np.float32)
+    side = rng.standard_normal(SHAPE).astype(np.float32)
+    one = run_net([conv], x)
+    two = run_net([conv, dict(_add(), inputs=[0, -2])], [x, np.zeros_like(side)])
+    assert np.array_equal(one, two)
+    swapped = run_net([dict(conv, inputs=[-2])], [side, x])
+    assert np.array_equal(swapped, one)
