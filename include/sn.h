@@ -346,9 +346,13 @@ SN_API sn_status sn_calibrate(sn_graph *g, const void *in_dev, void *stream);
  * (3x3 kernel, stride 1, dilation 1, groups 1, zero padding `pad` on both
  * axes, bias + act), using the same kernels, but its scratch (the transformed
  * filter U and the Winograd buffers V and M) lives in one fixed device array
- * of SN_NOALLOC_SCRATCH_BYTES that is part of the library image: every GPU
- * that loads the library holds that memory until the process exits.  The
- * call itself never allocates: no cudaMalloc, no cudaFree, no allocator hook.
+ * of SN_NOALLOC_SCRATCH_BYTES that is part of the library image.  A GPU
+ * takes that memory when the library's device code is loaded on it: no later
+ * than this call's first use there (earlier if CUDA loads modules eagerly,
+ * e.g. CUDA_MODULE_LOADING=EAGER, or another entry point of the library
+ * loaded them), and it keeps it until the process exits; count it in the
+ * fixed memory budget of every device the library runs on.  The call itself
+ * never allocates: no cudaMalloc, no cudaFree, no allocator hook.
  *
  *   x_dev    input, logical N x C x H x W stored in `schema` (caller-owned)
  *   w_dev    device fp32 weights [c_out][C][3][3] (caller-owned)
@@ -365,8 +369,9 @@ SN_API sn_status sn_calibrate(sn_graph *g, const void *in_dev, void *stream);
  * GPU (different streams, or host threads without ordering) race on the
  * array: serialise them.
  * Errors: SN_EINVAL (NULL pointer, bad extent, schema, pad or act),
- * SN_EUNSUPPORTED (the scratch need exceeds SN_NOALLOC_SCRATCH_BYTES; nothing
- * is launched), SN_ECUDA. */
+ * SN_EUNSUPPORTED (schema.dtype is SN_QI8, which this routine has no form
+ * for, or the scratch need exceeds SN_NOALLOC_SCRATCH_BYTES; nothing is
+ * launched), SN_ECUDA. */
 #define SN_NOALLOC_SCRATCH_BYTES (32u * 1024u * 1024u)
 SN_API sn_status sn_conv2d_wino_noalloc(const void *x_dev, sn_schema schema, const int64_t in_nchw[4],
                                         int32_t c_out, int32_t pad, int32_t act, const float *w_dev,

@@ -51,6 +51,8 @@ extern "C" sn_status sn_conv2d_wino_noalloc(const void *x_dev, sn_schema schema,
         if (!x_dev || !in_nchw || !w_dev || !bias_dev || !y_dev)
             return fail(SN_EINVAL, "sn_conv2d_wino_noalloc: NULL argument");
         if (!schema_valid(schema)) return fail(SN_EINVAL, "sn_conv2d_wino_noalloc: invalid schema");
+        if (schema.dtype == SN_QI8)
+            return fail(SN_EUNSUPPORTED, "sn_conv2d_wino_noalloc: the Winograd routine has no qint8 form");
         if (pad < 0 || pad > 2) return fail(SN_EINVAL, "sn_conv2d_wino_noalloc: pad must be 0, 1 or 2");
         if (act < SN_ACT_NONE || act > SN_ACT_HSIGMOID) return fail(SN_EINVAL, "sn_conv2d_wino_noalloc: bad act");
         for (int i = 0; i < 4; ++i)
@@ -60,15 +62,24 @@ extern "C" sn_status sn_conv2d_wino_noalloc(const void *x_dev, sn_schema schema,
         const int64_t N = in_nchw[0], C = in_nchw[1], H = in_nchw[2], W = in_nchw[3];
         const int64_t P = H + 2 * pad - 2, Q = W + 2 * pad - 2;
         if (P < 1 || Q < 1) return fail(SN_EINVAL, "sn_conv2d_wino_noalloc: empty output");
-        const int64_t tiles = N * ((P + 1) / 2) * ((Q + 1) / 2);
-        const size_t u_bytes = align256((size_t)16 * c_out * C * dtype_size(schema.dtype));
-        const size_t v_bytes = align256((size_t)16 * tiles * C * sizeof(float));
-        const size_t m_bytes = align256((size_t)16 * tiles * c_out * sizeof(float));
-        if (u_bytes + v_bytes + m_bytes > (size_t)SN_NOALLOC_SCRATCH_BYTES)
+        // Every byte count is a product of extents of up to 2^30 each, so it
+        // is formed with overflow checks: a count that does not fit in 64
+        // bits is far beyond the scratch size and is rejected as such.
+        const uint64_t limit = SN_NOALLOC_SCRATCH_BYTES;
+        auto mul = [](uint64_t a, uint64_t b, uint64_t *out) { return !__builtin_mul_overflow(a, b, out); };
+        uint64_t tiles = 0, u_raw = 0, v_raw = 0, m_raw = 0, need = 0;
+        const bool in64 =
+            mul((uint64_t)N, (uint64_t)((P + 1) / 2), &tiles) && mul(tiles, (uint64_t)((Q + 1) / 2), &tiles) &&
+            mul((uint64_t)16 * dtype_size(schema.dtype), (uint64_t)c_out, &u_raw) && mul(u_raw, (uint64_t)C, &u_raw) &&
+            mul((uint64_t)16 * sizeof(float), tiles, &v_raw) && mul(v_raw, (uint64_t)C, &v_raw) &&
+            mul((uint64_t)16 * sizeof(float), tiles, &m_raw) && mul(m_raw, (uint64_t)c_out, &m_raw) &&
+            !__builtin_add_overflow(u_raw, v_raw, &need) && !__builtin_add_overflow(need, m_raw, &need);
+        // each part is rounded up to 256 bytes: at most 3 x 255 more than `need`
+        if (!in64 || need > limit || align256(u_raw) + align256(v_raw) + align256(m_raw) > limit)
             return fail(SN_EUNSUPPORTED, "sn_conv2d_wino_noalloc: needs " +
-                                             std::to_string(u_bytes + v_bytes + m_bytes) +
-                                             " bytes of scratch, the fixed limit is " +
-                                             std::to_string((size_t)SN_NOALLOC_SCRATCH_BYTES));
+                                             (in64 ? std::to_string(need) : std::string("more than 2^64")) +
+                                             " bytes of scratch, the fixed limit is " + std::to_string(limit));
+        const size_t u_bytes = align256(u_raw), v_bytes = align256(v_raw);
         void *scratch = nullptr;
         sn_status rc = scratch_on_current_device(&scratch);
         if (rc != SN_OK) return rc;

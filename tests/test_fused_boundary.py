@@ -111,3 +111,66 @@ def test_pair_problem_without_fused_choices_is_the_plain_problem(seed):
         return
     assert tot == ref
     assert all(t["out_schema"][c] == t["schema"][c] for c in cand)
+
+
+# ---------------------------------------------------------------------------
+# pins of the oracle's exhaustive search over candidates (fused boundaries)
+# ---------------------------------------------------------------------------
+
+def _golden_fused():
+    import json
+    import os
+    here = os.path.dirname(os.path.abspath(__file__))
+    with open(os.path.join(here, "golden", "path_fused_boundary.json")) as f:
+        return json.load(f)
+
+
+def test_candidate_search_reaches_the_hand_worked_fused_optimum():
+    """Def. 1-2 read for fused boundaries: each edge is charged the adapt from
+    the producer's WRITTEN schema to the consumer's READ schema.  The golden
+    lists every choice with its cost by hand; the optimum uses the qint8
+    routine that writes f16, and charging the edge from its read schema
+    instead would move the optimum."""
+    g = _golden_fused()
+    ns = len(g["schemas"])
+    a = np.zeros((len(g["edges"]), ns, ns), np.int64)
+    a[:, 0, 1] = g["adapt"]["F->Q (quantise)"]
+    a[:, 1, 0] = g["adapt"]["Q->F (dequantise)"]
+    cands = [[tuple(c) for c in layer] for layer in g["candidates"]]
+    cost, pick = brute_force_candidates(cands, g["edges"], a)
+    assert cost == g["expect_cost"]
+    assert pick == g["expect_pick"]
+
+
+def test_candidate_search_equals_schema_search_without_fused_candidates():
+    """When every candidate writes the schema it reads, the search over one
+    candidate per layer is the plain problem of Def. 2: its optimum equals the
+    exhaustive search over schema assignments of F_i(lambda) (Eq. 1)."""
+    for seed in range(60):
+        rng = np.random.default_rng(9500 + seed)
+        n, ns = int(rng.integers(3, 7)), int(rng.integers(2, 4))
+        edges = [(i, i + 1) for i in range(n - 1)]
+        for _ in range(int(rng.integers(0, 3))):  # a few skip edges (still a DAG in index order)
+            u = int(rng.integers(0, n - 2))
+            v = int(rng.integers(u + 2, n))
+            if (u, v) not in edges:
+                edges.append((u, v))
+        cands, lc = [], np.full((n, ns), INF, np.int64)
+        for i in range(n):
+            layer = []
+            for _ in range(int(rng.integers(1, 4))):
+                s = int(rng.integers(0, ns))
+                c = 0 if i in (0, n - 1) else int(rng.integers(1, 100))
+                layer.append((c, s, s))
+                lc[i, s] = min(lc[i, s], c)
+            cands.append(layer)
+        a = rng.integers(0, 40, size=(len(edges), ns, ns)).astype(np.int64)
+        for e in range(len(edges)):
+            np.fill_diagonal(a[e], 0)
+        got, pick = brute_force_candidates(cands, edges, a)
+        ref, _, _ = oracle.brute_force(lc, edges, a)
+        assert got == ref, seed
+        if got < INF:
+            # the chosen candidates, read as a schema assignment, cost the same
+            assign = [cands[i][k][1] for i, k in enumerate(pick)]
+            assert oracle.path_cost(lc, edges, a, assign) == ref

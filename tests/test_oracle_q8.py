@@ -254,3 +254,47 @@ def test_fused_dequantisation_output_is_the_unrounded_value():
     assert np.array_equal(h, oracle.round_to(got.astype(np.float32), "f16"))
     # requantising it gives the ordinary qint8 output
     assert np.array_equal(q8.requantize(got, 256.0), q8.conv2d(x, 1.0, qw, sw, b, 256.0, pad=(1, 1), act="relu"))
+
+
+def test_absmax_scale_hand_cases():
+    """Calibration scale = max |x| / 127 in fp32 (section II-C, symmetric),
+    1 for an all-zero (or empty) blob.  127 and 254 give exactly 1 and 2."""
+    assert q8.absmax_scale(np.array([-127.0, 3.0, 50.0], F32)) == F32(1.0)
+    assert q8.absmax_scale(np.array([[1.0, 254.0], [-2.0, 0.5]], F32)) == F32(2.0)
+    # the magnitude counts, not the sign: the largest entry is negative
+    assert q8.absmax_scale(np.array([12.7, -25.4], F32)) == F32(25.4) / F32(127)
+    assert q8.absmax_scale(np.zeros((2, 3), F32)) == F32(1.0)
+    assert q8.absmax_scale(np.zeros((0,), F32)) == F32(1.0)
+    assert q8.absmax_scale(np.array([-0.0, 0.0], F32)) == F32(1.0)
+
+
+def test_calibrate_scales_each_blob_by_its_own_maximum():
+    """One float pass of a 3-layer net whose blobs have hand-known maxima:
+    x has max |x| = 127 * 4; an identity 1x1 conv (+ReLU) keeps the positive
+    part (max 127 * 3); a 2x2 max pool keeps that maximum; a GAP of the conv
+    output averages channel 0 to (381 + 1 + 2 + 0) / 4 = 96 and channel 1 to
+    254.  Scales: input 4, then 3, 3 and 2 in layer order (an off-by-one blob
+    index or a missing /127 changes one of them)."""
+    x = np.zeros((1, 2, 2, 2), F32)
+    x[0, 0] = [[127 * 3, 1], [2, -127 * 4]]      # channel 0: max |.| = 508, max(.) = 381
+    x[0, 1] = [[254, 254], [254, 254]]           # channel 1: constant 254
+    eye = np.eye(2, dtype=F32).reshape(2, 2, 1, 1)
+    layers = [
+        {"type": "conv2", "inputs": [-1], "params": dict(c_in=2, c_out=2, kh=1, kw=1, sh=1, sw=1, ph=0, pw=0,
+                                                         act="relu"),
+         "weight": eye, "bias": np.zeros(2, F32)},
+        {"type": "maxpool", "inputs": [0], "params": dict(kh=2, kw=2, sh=2, sw=2, ph=0, pw=0)},
+        {"type": "gap", "inputs": [0]},
+    ]
+    s_in, scales = q8.calibrate(layers, x)
+    assert s_in == F32(4.0)
+    # conv + ReLU: channel 0 max 381 (= 127 * 3), channel 1 254 -> blob max 381
+    assert scales[0] == F32(3.0)
+    # pool of a 2x2 map to 1x1: the maxima 381 and 254 -> blob max 381
+    assert scales[1] == F32(3.0)
+    # GAP of the conv output: channel means 96 and 254 -> blob max 254
+    assert scales[2] == F32(2.0)
+    # and a blob that is all zero gets scale 1
+    x0 = np.zeros_like(x)
+    s0, sc0 = q8.calibrate(layers, x0)
+    assert s0 == F32(1.0) and all(s == F32(1.0) for s in sc0)
