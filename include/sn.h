@@ -254,6 +254,15 @@ SN_API sn_status sn_set_path(sn_graph *g, const int32_t *candidate, int32_t n_la
 #define SN_OPT_CUDA_GRAPH 0 /* 1 = replay the launch sequence as a CUDA graph    */
 #define SN_OPT_CHECK 1      /* 1 = sync stream after sn_run and read the device
                                error word (SN_ETIMEOUT / SN_ECUDA on failure)    */
+#define SN_OPT_CHAIN 2      /* 1 (default) = run every run of two or more
+                               consecutive conv2/igemm_tc layers of the plan as
+                               one persistent launch whose tiles wait on the
+                               tiles they read (section III-A executes the tuned
+                               net layer by layer; the routine and its
+                               parameters per layer are unchanged, the launch
+                               boundaries between them go); 0 = one launch per
+                               layer.  Profiling and sn_run_timed always run
+                               one launch per layer.                             */
 SN_API sn_status sn_set_option(sn_graph *g, int32_t option, int64_t value);
 
 /* Run the net with the selected path: in_dev holds the input in in_schema,

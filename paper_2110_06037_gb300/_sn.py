@@ -22,7 +22,7 @@ SN_NCHW, SN_NHWC = 0, 1
 SN_L_CONV2, SN_L_DWCONV2, SN_L_MAXPOOL, SN_L_GAP, SN_L_ADD, SN_L_DENSE, SN_L_MUL = range(7)
 SN_ACT = {"none": 0, None: 0, "relu": 1, "relu6": 2, "hswish": 3, "hsigmoid": 4}
 SN_SELECT_DPRS, SN_SELECT_BRUTE = 0, 1
-SN_OPT_CUDA_GRAPH, SN_OPT_CHECK = 0, 1
+SN_OPT_CUDA_GRAPH, SN_OPT_CHECK, SN_OPT_CHAIN = 0, 1, 2
 COST_INF = np.iinfo(np.int64).max
 
 DTYPES = {"f32": SN_F32, "f16": SN_F16, "bf16": SN_BF16, "qi8": SN_QI8}

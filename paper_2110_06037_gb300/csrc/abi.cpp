@@ -267,6 +267,11 @@ sn_status sn_set_option(sn_graph *gg, int32_t option, int64_t value) {
             }
         } else if (option == SN_OPT_CHECK) {
             g->opt_check = value ? 1 : 0;
+        } else if (option == SN_OPT_CHAIN) {
+            if (g->opt_chain != (value ? 1 : 0)) {
+                g->opt_chain = value ? 1 : 0;
+                invalidate_plan(g);
+            }
         } else {
             return fail(SN_EINVAL, "sn_set_option: unknown option");
         }
@@ -424,8 +429,11 @@ sn_status sn_plan_stats(sn_graph *gg, int32_t *n_ops, int32_t *n_kernels, void *
             if (rc != SN_OK) return rc;
         }
         int32_t kern = 0;
-        for (const PlanOp &op : g->plan) {
-            if (op.kind == PlanOp::ADAPT) {
+        for (size_t q = 0; q < g->plan.size(); ++q) {
+            const PlanOp &op = g->plan[q];
+            if (q < g->op_chain.size() && g->op_chain[q] >= 0) {  // one launch per chain
+                kern += g->chains[g->op_chain[q]].first_op == (int32_t)q ? 1 : 0;
+            } else if (op.kind == PlanOp::ADAPT) {
                 kern += 1;
             } else {
                 const Candidate &c = g->cands[op.cand];

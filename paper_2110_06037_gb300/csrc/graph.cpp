@@ -32,6 +32,10 @@ static int64_t out_dim(int64_t in, int64_t k, int64_t s, int64_t p, int64_t d) {
 
 Graph::~Graph() {
     if (gexec) cudaGraphExecDestroy(gexec);
+    for (auto &c : chains) {
+        dev_free(this, &c.desc);
+        dev_free(this, &c.done);
+    }
     for (auto &b : slots) dev_free(this, &b);
     for (auto &kv : weight_cache) dev_free(this, &kv.second);
     for (auto &kv : bias_cache) dev_free(this, &kv.second);
@@ -73,6 +77,12 @@ void dev_free(Graph *g, Buffer *b) {
 void invalidate_plan(Graph *g) {
     g->plan_valid = false;
     g->plan.clear();
+    for (auto &c : g->chains) {
+        dev_free(g, &c.desc);
+        dev_free(g, &c.done);
+    }
+    g->chains.clear();
+    g->op_chain.clear();
     if (g->gexec) {
         cudaGraphExecDestroy(g->gexec);
         g->gexec = nullptr;

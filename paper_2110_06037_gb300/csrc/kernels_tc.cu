@@ -1008,6 +1008,34 @@ int32_t conv_tc_variants(const Layer &l, const Shape &in, sn_schema s) {
     return (int32_t)tc::configs(l, in, s).size();
 }
 
+// The tile shape a layer takes inside a chained launch (one CTA per tile of
+// 128 pixels, no K split): the selected variant's pixel formulation (plain or
+// implicit, and its tile geometry; a 256-row geometry is halved along its
+// outermost axis), the widest output-channel tile the layer fills, and two
+// channel blocks per stage only for 64-channel tiles (the chain's stage holds
+// 48 KB).  False when the variant is not a conv2/igemm_tc one.
+bool conv_tc_chain_shape(const Layer &l, const Shape &in, sn_schema s, int32_t v, bool *implicit, int *bn, int *kb,
+                         int *bw, int *bh, int *bni) {
+    const std::vector<tc::Config> cfgs = tc::configs(l, in, s);
+    if (v < 0 || v >= (int)cfgs.size()) return false;
+    const tc::Config &cf = cfgs[v];
+    *implicit = cf.implicit;
+    // the widest output-channel tile the layer fills: a stage costs its TMA
+    // boxes (about the same per box whatever its size), so a 256-wide tile
+    // does twice the MMA work of a 128-wide one for the same two boxes, and
+    // wide tiles mean fewer units to drain and fewer dependency checks
+    *bn = l.conv.c_out <= 64 ? 64 : l.conv.c_out <= 128 ? 128 : 256;
+    *kb = (*bn == 64 && l.conv.c_in % 128 == 0) ? 2 : 1;
+    int w = cf.BW, h = cf.BH, n = cf.BNI;
+    if (cf.implicit && cf.ms == 2) {
+        if (n >= 2) n /= 2;
+        else if (h >= 2) h /= 2;
+        else w /= 2;
+    }
+    *bw = w, *bh = h, *bni = n;
+    return !cf.implicit || w * h * n == tc::BM;
+}
+
 size_t conv_tc_ws(const Layer &l, const Shape &in, sn_schema s, int32_t v, int32_t a_blocks) {
     const std::vector<tc::Config> cfgs = tc::configs(l, in, s, a_blocks);
     if (v < 0 || v >= (int)cfgs.size() || cfgs[v].ksplit == 1) return 0;

@@ -156,7 +156,92 @@ sn_status build_plan(Graph *g, cudaStream_t st) {
         sn_status rc = dev_alloc(g, ws, &g->workspace);
         if (rc != SN_OK) return rc;
     }
+    if (g->opt_chain && !g->profiling) {
+        sn_status rc = build_chains(g, st);
+        if (rc != SN_OK) return rc;
+    }
     g->plan_valid = true;
+    return SN_OK;
+}
+
+// A plan op that a chained launch can run: a conv2 on the tensor-core
+// routine reading and writing graph-owned buffers (the caller's buffers may
+// change from run to run; a chain's tensor maps are encoded once).
+static bool chain_eligible(const Graph *g, const PlanOp &op) {
+    if (op.kind != PlanOp::LAYER) return false;
+    const Candidate &c = g->cands[op.cand];
+    if (c.routine != R_CONV_TC || cand_out(c) != c.schema) return false;
+    if (op.out_slot < g->n_ext) return false;
+    for (int32_t s : op.in_slots)
+        if (s < g->n_ext) return false;
+    const Layer &L = g->layers[op.layer];
+    if (L.type != SN_L_CONV2 || L.inputs.empty() || L.inputs.size() > 2) return false;
+    bool imp;
+    int bn, kb, bw, bh, bni;
+    return k::conv_tc_chain_shape(L, g->layers[L.inputs[0]].out, g->schemas[c.schema], c.variant, &imp, &bn, &kb,
+                                  &bw, &bh, &bni);
+}
+
+// Group maximal runs of two or more consecutive chain-eligible ops of one
+// dtype into chains and upload their descriptors.
+sn_status build_chains(Graph *g, cudaStream_t st) {
+    g->chains.clear();
+    g->op_chain.assign(g->plan.size(), -1);
+    const size_t n = g->plan.size();
+    auto dtype_of = [&](size_t q) { return g->schemas[g->cands[g->plan[q].cand].schema].dtype; };
+    size_t i = 0;
+    while (i < n) {
+        if (!chain_eligible(g, g->plan[i])) {
+            ++i;
+            continue;
+        }
+        size_t j = i;
+        while (j + 1 < n && chain_eligible(g, g->plan[j + 1]) && dtype_of(j + 1) == dtype_of(i)) ++j;
+        if (j > i) {
+            std::vector<ChainOp> ops;
+            for (size_t q = i; q <= j; ++q) {
+                const PlanOp &op = g->plan[q];
+                const Candidate &c = g->cands[op.cand];
+                const Layer &L = g->layers[op.layer];
+                ChainOp co;
+                co.layer = &L;
+                co.in = g->layers[L.inputs[0]].out;
+                co.schema = g->schemas[c.schema];
+                co.variant = c.variant;
+                co.in0 = g->slots[op.in_slots[0]].ptr;
+                co.res = op.in_slots.size() > 1 ? g->slots[op.in_slots[1]].ptr : nullptr;
+                co.out = g->slots[op.out_slot].ptr;
+                co.wt = op.wt;
+                co.bias = op.bias;
+                for (size_t p = i; p < q; ++p) {
+                    if (g->plan[p].out_slot == op.in_slots[0]) co.src = (int32_t)(p - i);
+                    if (op.in_slots.size() > 1 && g->plan[p].out_slot == op.in_slots[1]) co.res_src = (int32_t)(p - i);
+                }
+                ops.push_back(co);
+            }
+            ChainPlan cp;
+            cp.first_op = (int32_t)i;
+            cp.last_op = (int32_t)j;
+            cp.n_layers = (int32_t)ops.size();
+            cp.dtype = dtype_of(i);
+            std::vector<uint8_t> blob;
+            cudaError_t e = k::chain_encode(ops, blob, &cp.total_units, &cp.done_count);
+            if (e != cudaSuccess) return fail(SN_ECUDA, std::string("chain descriptors: ") + cudaGetErrorString(e));
+            sn_status rc = dev_alloc(g, blob.size(), &cp.desc);
+            if (rc == SN_OK) rc = dev_alloc(g, ((size_t)cp.done_count + 2) * sizeof(int32_t), &cp.done);
+            if (rc != SN_OK) {
+                dev_free(g, &cp.desc);
+                dev_free(g, &cp.done);
+                return rc;
+            }
+            g->chains.push_back(cp);  // owned by the graph from here on (freed with the plan)
+            SN_CUDA_TRY(cudaMemcpyAsync(cp.desc.ptr, blob.data(), blob.size(), cudaMemcpyHostToDevice, st));
+            SN_CUDA_TRY(cudaMemsetAsync(cp.done.ptr, 0, cp.done.bytes, st));
+            SN_CUDA_TRY(cudaStreamSynchronize(st));  // `blob` is freed on return
+            for (size_t q = i; q <= j; ++q) g->op_chain[q] = (int32_t)g->chains.size() - 1;
+        }
+        i = j + 1;
+    }
     return SN_OK;
 }
 
@@ -207,6 +292,15 @@ sn_status run_plan(Graph *g, const IoPtrs &io, cudaStream_t st, std::vector<cuda
     if ((int32_t)(io.in.size() + io.out.size()) != g->n_ext || (int32_t)io.in.size() != g->n_in())
         return fail(SN_EINVAL, "run: wrong number of input or output buffers");
     for (size_t i = 0; i < g->plan.size(); ++i) {
+        if (!evs && i < g->op_chain.size() && g->op_chain[i] >= 0) {  // a chained launch runs the whole chain
+            const ChainPlan &c = g->chains[g->op_chain[i]];
+            if (c.first_op == (int32_t)i) {
+                cudaError_t e = k::chain_launch(c.dtype, c.desc.ptr, c.n_layers, c.total_units,
+                                                static_cast<int32_t *>(c.done.ptr), c.done_count, st);
+                if (e != cudaSuccess) return fail(SN_ECUDA, std::string("chained launch: ") + cudaGetErrorString(e));
+            }
+            continue;
+        }
         // external records: timing nodes when the stream is being captured
         if (evs) SN_CUDA_TRY(cudaEventRecordWithFlags((*evs)[2 * i], st, cudaEventRecordExternal));
         sn_status rc = launch_op(g, g->plan[i], io, st);

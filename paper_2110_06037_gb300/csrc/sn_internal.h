@@ -114,6 +114,31 @@ struct PlanOp {
 
 struct Graph;
 
+// One layer of a chained launch (consecutive conv2/igemm_tc layers run as one
+// persistent kernel whose tiles wait on the tiles they read): the layer, its
+// selected routine parameter and its resolved buffers; src / res_src = index
+// within the chain of the layer that writes input 0 / the residual (-1: the
+// buffer is written before the chain starts).
+struct ChainOp {
+    const Layer *layer = nullptr;
+    Shape in;
+    sn_schema schema{};
+    int32_t variant = 0;
+    const void *in0 = nullptr, *res = nullptr;
+    void *out = nullptr;
+    const void *wt = nullptr;
+    const float *bias = nullptr;
+    int32_t src = -1, res_src = -1;
+};
+
+// A chain of the plan: ops [first_op, last_op] run as one launch.
+struct ChainPlan {
+    int32_t first_op = -1, last_op = -1;
+    int32_t n_layers = 0, total_units = 0, done_count = 0;
+    int32_t dtype = 0;
+    Buffer desc, done;  // layer descriptors; completion counters (+ exit counter, abort flag)
+};
+
 // A launchable routine instance: everything a kernel needs, resolved.
 struct LaunchArgs {
     const Graph *g;
@@ -180,6 +205,9 @@ struct Graph {
     std::map<int32_t, Buffer> bias_cache;        // per layer fp32 bias
     Buffer workspace;
     int opt_graph = 0, opt_check = 0;
+    int opt_chain = 0;                // run runs of tensor-core convolutions as chained launches
+    std::vector<ChainPlan> chains;    // built with the plan
+    std::vector<int32_t> op_chain;    // per plan op: its chain, or -1
     bool profiling = false;           // plans built while profiling may lack qint8 scales
     cudaGraphExec_t gexec = nullptr;
     std::vector<const void *> gexec_in;
@@ -248,6 +276,7 @@ void fastest_per_schema(const Graph &g, std::vector<int64_t> &F, std::vector<int
 
 // plan + run
 sn_status build_plan(Graph *g, cudaStream_t st);
+sn_status build_chains(Graph *g, cudaStream_t st);
 sn_status run_plan(Graph *g, const IoPtrs &io, cudaStream_t st,
                    std::vector<cudaEvent_t> *evs);
 // one run of the plan replayed from a CUDA graph with a timing node around
@@ -290,6 +319,14 @@ int32_t conv_tc_variants(const Layer &l, const Shape &in, sn_schema s);
 size_t conv_tc_ws(const Layer &l, const Shape &in, sn_schema s, int32_t v, int32_t a_blocks = 0);  // K-split partials
 size_t dense_tc_ws(const Layer &l, const Shape &in, sn_schema s, int32_t v);
 const char *conv_tc_variant_name(int32_t v);
+// chained launches of consecutive tensor-core convolutions
+bool conv_tc_chain_shape(const Layer &l, const Shape &in, sn_schema s, int32_t v, bool *implicit, int *bn, int *kb,
+                         int *bw, int *bh, int *bni);
+size_t chain_desc_bytes(int n_layers);
+cudaError_t chain_encode(const std::vector<ChainOp> &ops, std::vector<uint8_t> &blob, int32_t *total_units,
+                         int32_t *done_count);
+cudaError_t chain_launch(int dtype, const void *desc_dev, int32_t n_layers, int32_t total_units, int32_t *done_dev,
+                         int32_t done_count, cudaStream_t st);
 // im2col childnet and dense childnet on the tensor-core GEMM
 int32_t conv_im2col_tc_variants(const Layer &l, const Shape &in, sn_schema s);
 size_t conv_im2col_tc_ws(const Layer &l, const Shape &in, sn_schema s, int32_t v);
