@@ -63,15 +63,15 @@ class ClockSampler:
         self.t0 = self.t1 = None
 
     def start(self):
-        """Start sampling and wait (up to 5 s) for the first sample, so that
+        """Start sampling and wait (up to 15 s) for the first sample, so that
         the timed region that follows is covered."""
         try:
             self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.Q}",
-                                          "--format=csv,noheader,nounits", "-lms", "50"],
+                                          "--format=csv,noheader,nounits", "-lms", "10"],
                                          stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
             self.t = threading.Thread(target=self._read, daemon=True)
             self.t.start()
-            deadline = time.monotonic() + 5.0
+            deadline = time.monotonic() + 15.0
             while not self.lines and time.monotonic() < deadline:
                 time.sleep(0.01)
         except Exception:
@@ -243,6 +243,9 @@ def main():
     ap.add_argument("--batch", type=int, default=32)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-b1", action="store_true")
+    ap.add_argument("--no-extras", action="store_true",
+                    help="skip the extra rows of the benchmark line (bandwidth, MobileNetV2 / tiny CNN latency, "
+                         "sweep summary, oracle timings)")
     ap.add_argument("--config", default="r50_b32",
                     choices=["r50_b32", "bandwidth", "sweep", "mbv2_b1", "r50_b1", "tiny", "layer", "vgg16_b32",
                              "vgg16_b1", "mbv3_b1", "hybrid", "q8_dense"],
@@ -274,13 +277,14 @@ def main():
     pk, pk_kind = peaks()
 
     # ---------------- tune: profile + DPRS ----------------
-    x, layers = synth.resnet50(args.batch)
-    layers = sn.fuse_residual(layers)
+    x, layers0 = synth.resnet50(args.batch)
     sch = [("bf16", "nchw"), ("bf16", "nhwc")]
     stream = torch.cuda.Stream()
     t_tune0 = time.perf_counter()
     with torch.cuda.stream(stream):
-        g = sn.build_graph(layers, x.shape, ("bf16", "nchw"), ("bf16", "nchw"), sch)
+        # the library's residual-add fusion pass runs before tuning
+        g = sn.build_graph(layers0, x.shape, ("bf16", "nchw"), ("bf16", "nchw"), sch, fuse=True)
+        layers = sn.fused_description(layers0, g.fused_ids)
         g.profile(warmup=3, iters=10, topk=2, passes=3)
         total, schemas, cands = g.select_path(sn.SN_SELECT_DPRS)
     stream.synchronize()
@@ -325,63 +329,36 @@ def main():
         ms = float(t.item())
     value = ws * args.batch / (ms / 1e3)
 
-    # ---------------- e2e through the public API with host buffers ----------------
-    # Every step copies its input batch from pinned host memory and reads its
-    # logits back to the host, inside the timed region.  As a serving loop
-    # would, the next step's host->device copy runs on a copy stream into one
-    # of two staging buffers while the current step computes; the step then
-    # moves its batch into the net's input buffer (device to device) and its
-    # logits go back to the host on the copy stream.
+    # ---------------- e2e through the C ABI with host buffers ----------------
+    # Every step is one sn_run_host call: the library copies the batch from
+    # pinned host memory into its device staging buffer, runs the net and
+    # copies the logits back to pinned host memory, all on the stream, so the
+    # timed region holds each step's host->device and device->host copies.
     xh = torch.from_numpy(x).to(torch.bfloat16).pin_memory()
-    oh = [torch.empty(out.shape, dtype=out.dtype).pin_memory() for _ in range(2)]
-    xin = torch.empty_like(xd)
-    stage = [torch.empty_like(xd) for _ in range(2)]
-    ostage = [torch.empty_like(out) for _ in range(2)]
-    cstream = torch.cuda.Stream()
-
-    def e2e_steps(n):
-        ev = lambda: torch.cuda.Event()
-        h_done, used, r_done, d_done = ([ev() for _ in range(n)] for _ in range(4))
-        cstream.wait_stream(stream)
-        with torch.cuda.stream(cstream):
-            stage[0].copy_(xh, non_blocking=True)
-            h_done[0].record(cstream)
-        for k in range(n):
-            if k + 1 < n:
-                with torch.cuda.stream(cstream):
-                    if k >= 1:
-                        cstream.wait_event(used[k - 1])  # staging buffer (k+1)%2 was read by step k-1
-                    stage[(k + 1) % 2].copy_(xh, non_blocking=True)
-                    h_done[k + 1].record(cstream)
-            stream.wait_event(h_done[k])
-            with torch.cuda.stream(stream):
-                xin.copy_(stage[k % 2], non_blocking=True)
-                used[k].record(stream)
-                g.run(xin, out)
-                if k >= 2:
-                    stream.wait_event(d_done[k - 2])  # logits staging buffer k%2 read back by step k-2
-                ostage[k % 2].copy_(out, non_blocking=True)
-                r_done[k].record(stream)
-            with torch.cuda.stream(cstream):
-                cstream.wait_event(r_done[k])
-                oh[k % 2].copy_(ostage[k % 2], non_blocking=True)
-                d_done[k].record(cstream)
-        stream.wait_stream(cstream)
-
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e2e_steps(3)
+    oh = torch.empty(out.shape, dtype=out.dtype).pin_memory()
+    with torch.cuda.stream(stream):
+        for _ in range(3):
+            g.run_host(xh, oh)
     stream.synchronize()
-    e0.record(stream)
-    e2e_steps(args.steps)
-    e1.record(stream)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for _ in range(args.steps):
+            g.run_host(xh, oh)
+        e1.record(stream)
     stream.synchronize()
     e2e_ms = e0.elapsed_time(e1) / args.steps
     e2e = {"value": args.batch / (e2e_ms / 1e3), "unit": "images/s",
            "h2d_bytes_per_step": xh.numel() * xh.element_size(),
-           "d2h_bytes_per_step": oh[0].numel() * oh[0].element_size(),
-           "overlap": "next step's host->device copy overlaps this step's compute (two staging buffers)"}
+           "d2h_bytes_per_step": oh.numel() * oh.element_size(),
+           "path": "sn_run_host (C ABI): copies from and to pinned host memory inside each call, in stream order"}
 
-    # ---------------- per-routine device time (events around every launch) ----------------
+    # ---------------- per-op shares of the step ----------------
+    # One replay of the step with a timing node around every op gives each
+    # op's device time run on its own; the ops overlap in the timed replay
+    # (programmatic dependent launch), so these times sum to more than the
+    # step.  Each routine's time in the step is its share of that sum times
+    # the measured ms_per_step, which by construction cannot exceed the step.
     g.set_option(sn.SN_OPT_CUDA_GRAPH, 0)
     t = g.cost_table()
     layer_ms = np.zeros(t["n_layers"])
@@ -395,48 +372,75 @@ def main():
             edge_ms += em[: len(edge_ms)]
     layer_ms /= reps
     edge_ms /= reps
-    work, _ = conv_work(layers, x.shape)
+    op_sum = float(layer_ms[1:-1].sum() + edge_ms.sum())
+    scale = ms / op_sum
+    work, shapes = conv_work(layers, x.shape)
     per_routine = {}
     for i in range(1, t["n_layers"] - 1):
         c = int(cands[i])
         r = routine_name(int(t["routine"][c]))
         d = per_routine.setdefault(r, {"ms": 0.0, "flop": 0, "bytes": 0, "launches": 0})
-        d["ms"] += float(layer_ms[i])
+        d["ms"] += float(layer_ms[i]) * scale
         d["flop"] += work[i - 1][0]
         d["bytes"] += work[i - 1][1]
         d["launches"] += 1
     if edge_ms.sum() > 0:
-        per_routine["adapt/convert"] = {"ms": float(edge_ms.sum()), "flop": 0, "bytes": 0,
+        per_routine["adapt/convert"] = {"ms": float(edge_ms.sum()) * scale, "flop": 0, "bytes": 0,
                                         "launches": int((edge_ms > 0).sum())}
     dom = max(per_routine, key=lambda r: per_routine[r]["ms"])
     d = per_routine[dom]
     sustained = pk.get("bf16_tflops_sustained", pk["bf16_tflops"])
+    share = {"share_of_step": d["ms"] / ms, "time_ms": d["ms"],
+             "method": "the routine's share of the per-op device times of one replay with a timing node around "
+                       "every op (CUDA events on the launching stream), times ms_per_step"}
     if dom == "conv2/igemm_tc":
         achieved = d["flop"] / (d["ms"] / 1e3) / 1e12
         roof = {"bound": "tensor", "achieved": achieved, "peak": sustained, "unit": "TFLOP/s",
                 "frac": achieved / sustained, "traffic": tc_traffic_per_step(),
                 "traffic_unit": "DRAM bytes per step over the igemm_tc launches (ncu, cold L2 per kernel)",
-                "algorithmic_bytes": d["bytes"]}
+                "algorithmic_flop": d["flop"], "algorithmic_bytes": d["bytes"], **share}
     elif dom in ("conv2/igemm_simt", "conv2/direct", "conv2/wino_f2x2_3x3"):
         ffma_peak = 2 * 128 * 152 * pk.get("sm_max_mhz", 2070.0) / 1e6  # TFLOP/s fp32 FFMA
         achieved = d["flop"] / (d["ms"] / 1e3) / 1e12
         roof = {"bound": "alu", "achieved": achieved, "peak": ffma_peak, "unit": "TFLOP/s",
-                "frac": achieved / ffma_peak, "traffic": None}
+                "frac": achieved / ffma_peak, "traffic": None, **share}
     else:
         achieved = d["bytes"] / (d["ms"] / 1e3) / 1e9
         roof = {"bound": "hbm", "achieved": achieved, "peak": pk["hbm_gbs"], "unit": "GB/s",
-                "frac": achieved / pk["hbm_gbs"], "traffic": None}
+                "frac": achieved / pk["hbm_gbs"], "traffic": None, **share}
     roof["kernel"] = dom
     roof["peak_source"] = f"{pk_kind} (MEASURED_PEAKS.json)" if pk_kind == "measured" else "fallback"
+    # every conv layer of the path: its share-derived time, TFLOP/s and the
+    # fraction of the roofline its arithmetic intensity puts it under
+    ridge = sustained * 1e12 / (pk["hbm_gbs"] * 1e9)  # FLOP per byte where the two roofs meet
+    per_layer = []
+    for i in range(1, t["n_layers"] - 1):
+        lay = layers[i - 1]
+        if lay["type"] != "conv2":
+            continue
+        fl, by = work[i - 1]
+        us = float(layer_ms[i]) * scale * 1e3
+        if us <= 0:
+            continue
+        p_ = lay["params"]
+        ins = [x.shape if j < 0 else shapes[j] for j in lay["inputs"]]
+        ai = fl / by
+        row = {"layer": lay.get("name", str(i)),
+               "shape": f"{ins[0][1]}->{p_['c_out']} {ins[0][2]}x{ins[0][3]} k{p_['kh']} s{p_['sh']}" +
+                        (" +res" if len(lay["inputs"]) == 2 else ""),
+               "routine": g.candidate_desc(int(cands[i])), "us": round(us, 2),
+               "tflops": round(fl / us / 1e6, 1), "gbs": round(by / us / 1e3, 1), "ai": round(ai, 1),
+               "bound": "tensor" if ai > ridge else "hbm"}
+        row["frac"] = round(row["tflops"] / sustained if ai > ridge else row["gbs"] / pk["hbm_gbs"], 3)
+        per_layer.append(row)
 
     # ---------------- ResNet-50 b1 latency (fp16, CUDA graph) ----------------
     b1 = None
     if not args.no_b1:
         x1, layers1 = synth.resnet50(1)
-        layers1 = sn.fuse_residual(layers1)
         s16 = [("f16", "nchw"), ("f16", "nhwc")]
         with torch.cuda.stream(stream):
-            g1 = sn.build_graph(layers1, x1.shape, ("f16", "nchw"), ("f16", "nchw"), s16)
+            g1 = sn.build_graph(layers1, x1.shape, ("f16", "nchw"), ("f16", "nchw"), s16, fuse=True)
             g1.profile(warmup=3, iters=10, topk=2, passes=3)
             g1.select_path(sn.SN_SELECT_DPRS)
             g1.set_option(sn.SN_OPT_CUDA_GRAPH, 1)
@@ -457,6 +461,20 @@ def main():
             lat.append(a.elapsed_time(b))
         b1 = {"mean_ms": statistics.mean(lat), "std_ms": statistics.pstdev(lat), "median_ms": statistics.median(lat)}
 
+    # ---------------- the other rooflines and configurations (one GPU, rank 0) ----------------
+    extras = None
+    if rank == 0 and not args.no_extras:
+        extras = {}
+        t_ex = time.perf_counter()
+        extras["bandwidth"] = _bandwidth_rows(sn, torch, synth, pk["hbm_gbs"], compact=True)
+        lat_graphs = {}
+        for name in ("mbv2_b1", "tiny"):
+            extras[name] = _latency_config(sn, torch, synth, name, keep=lat_graphs)
+        extras["sweep"] = _sweep_summary(sn, torch, synth, pk)
+        if ws == 1:
+            extras["oracle"] = _oracle_times(sn, synth, lat_graphs, g1_table=(g1.cost_table() if b1 else None))
+        extras["seconds"] = time.perf_counter() - t_ex
+
     cpu = None
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         cpu = cpu_baseline_sample()
@@ -471,7 +489,8 @@ def main():
                 "e2e": e2e, "gpu_launches": n_kern * args.steps, "roofline": roof, "cpu_baseline": cpu,
                 "clocks": clk, "tuning_s": tune_s, "path_cost_ns": total,
                 "r50_b1_fp16_latency": b1,
-                "per_routine_ms": {k: round(v["ms"], 4) for k, v in per_routine.items()}}
+                "per_routine_ms": {k: round(v["ms"], 4) for k, v in per_routine.items()},
+                "per_layer": per_layer, "extras": extras}
         print(json.dumps(line))
     if dist:
         dist.destroy_process_group()
@@ -598,7 +617,7 @@ def run_hybrid(args):
     for name, make in nets.items():
         x, layers = make()
         if name != "vgg16":
-            layers = sn.fuse_residual(layers)
+            layers = sn.fuse_residual(layers, x.shape)
         xd = torch.from_numpy(x).to(torch.float16).cuda()
         row = {}
         outs = {}
@@ -650,6 +669,234 @@ def run_hybrid(args):
                       "data": "synthetic inputs and random weights", "nets": rows}))
 
 
+def _dw_rows(sn, torch, synth, hbm, shapes, variants=(0, 1), layouts=("nhwc", "nchw")):
+    rows = []
+    for (N, C, H, s_) in shapes:
+        for lay in layouts:
+            for var in variants:
+                sch = ("f16", lay)
+                layer = synth.dwconv(C, 3, s_, act="relu6")
+                layer["weight"] = np.zeros((C, 1, 3, 3), np.float32)
+                layer["bias"] = np.zeros(C, np.float32)
+                g = _single_layer_graph(sn, layer, (N, C, H, H), sch)
+                _forced(sn, g, "dwconv2/direct", var)
+                P = (H + 2 - 3) // s_ + 1
+                bufs = [(torch.zeros(sn.storage_shape((N, C, H, H), lay), dtype=torch.float16, device="cuda"),
+                         g.new_output()) for _ in range(_sets_for(2 * N * C * (H * H + P * P)))]
+                ms = _time_cold(torch, [(lambda xb=xb, yb=yb: g.run(xb, yb)) for xb, yb in bufs])
+                del bufs, g
+                by = 2 * (N * C * H * H + N * C * P * P) + 2 * 9 * C + 4 * C
+                rows.append({"kernel": "dwconv2/direct", "variant": sn.variant_name(5, var), "layout": lay,
+                             "shape": [N, C, H, H], "stride": s_, "us": ms * 1e3, "gbs": by / ms / 1e6,
+                             "frac": by / ms / 1e6 / hbm})
+    return rows
+
+
+def _adapt_rows(sn, torch, hbm, shapes, pairs):
+    rows = []
+    dt = {"f32": torch.float32, "bf16": torch.bfloat16, "f16": torch.float16}
+    for shp in shapes:
+        for (a_, b_) in pairs:
+            x = torch.zeros(sn.storage_shape(shp, a_[1]), dtype=dt[a_[0]], device="cuda")
+            y = torch.empty(sn.storage_shape(shp, b_[1]), dtype=dt[b_[0]], device="cuda")
+            bufs = [(x, y)] + [(torch.zeros_like(x), torch.empty_like(y))
+                               for _ in range(_sets_for(x.nbytes + y.nbytes) - 1)]
+            ms = _time_cold(torch, [(lambda xb=xb, yb=yb: sn.convert(xb, a_, b_, shp, out=yb)) for xb, yb in bufs])
+            del bufs
+            by = x.numel() * x.element_size() + y.numel() * y.element_size()
+            rows.append({"kernel": "adapt/convert", "from": "%s.%s" % a_, "to": "%s.%s" % b_, "shape": list(shp),
+                         "us": ms * 1e3, "gbs": by / ms / 1e6, "frac": by / ms / 1e6 / hbm})
+    return rows
+
+
+DW_SHAPES = [(128, 144, 56, 1), (128, 96, 112, 2), (128, 192, 28, 1), (128, 576, 14, 1), (128, 960, 7, 1)]
+ADAPT_SHAPES = [(32, 64, 112, 112), (32, 256, 56, 56), (32, 1024, 14, 14)]
+ADAPT_PAIRS = [(("bf16", "nchw"), ("bf16", "nhwc")), (("bf16", "nhwc"), ("bf16", "nchw")),
+               (("f32", "nchw"), ("bf16", "nhwc")), (("bf16", "nhwc"), ("f32", "nchw"))]
+
+
+def _bandwidth_rows(sn, torch, synth, hbm, compact=False):
+    """Depthwise 3x3 at MobileNetV2 shapes (batch 128) and the adapt conversions
+    on ResNet-50 b32 activations, each timed from CUDA-graph replays that rotate
+    through buffer sets totalling four L2 capacities (cold operands).  compact:
+    the best routine parameter and layout per depthwise shape (what DPRS would
+    take), and the conversions of the ResNet-50 b32 path."""
+    dw = _dw_rows(sn, torch, synth, hbm, DW_SHAPES)
+    ad = _adapt_rows(sn, torch, hbm, ADAPT_SHAPES, ADAPT_PAIRS)
+    if not compact:
+        return dw + ad
+    best = {}
+    for r in dw:
+        k = (tuple(r["shape"]), r["stride"])
+        if k not in best or r["gbs"] > best[k]["gbs"]:
+            best[k] = r
+    rnd = lambda r: {k: (round(v, 3) if isinstance(v, float) else v) for k, v in r.items()}
+    return {"metric": "achieved HBM GB/s (algorithmic bytes / event time), cold L2", "peak_gbs": hbm,
+            "depthwise_best": [rnd(r) for r in best.values()], "adapt": [rnd(r) for r in ad]}
+
+
+def _latency_config(sn, torch, synth, name, keep=None):
+    """Profile + DPRS + CUDA-graph latency of one net at batch 1 (or the given config)."""
+    if name == "tiny":
+        x, layers = synth.tiny_cnn()
+        sch, io, dt = [("f32", "nchw"), ("f32", "nhwc")], ("f32", "nchw"), torch.float32
+    elif name == "mbv2_b1":
+        x, layers = synth.mobilenet_v2(1)
+        sch, io, dt = [("f16", "nchw"), ("f16", "nhwc")], ("f16", "nchw"), torch.float16
+    elif name == "mbv3_b1":
+        x, layers = synth.mobilenet_v3(1)
+        sch, io, dt = [("f16", "nchw"), ("f16", "nhwc")], ("f16", "nchw"), torch.float16
+    elif name == "vgg16_b32":
+        x, layers = synth.vgg16(32)
+        sch, io, dt = [("bf16", "nchw"), ("bf16", "nhwc")], ("bf16", "nchw"), torch.bfloat16
+    elif name == "vgg16_b1":
+        x, layers = synth.vgg16(1)
+        sch, io, dt = [("f16", "nchw"), ("f16", "nhwc")], ("f16", "nchw"), torch.float16
+    else:
+        x, layers = synth.resnet50(1)
+        sch, io, dt = [("f16", "nchw"), ("f16", "nhwc")], ("f16", "nchw"), torch.float16
+    stream = torch.cuda.Stream()
+    t0 = time.perf_counter()
+    with torch.cuda.stream(stream):
+        # residual adds fused by the library's pass before tuning (no-op where there are none)
+        g = sn.build_graph(layers, x.shape, io, io, sch, fuse=True)
+        layers = sn.fused_description(layers, g.fused_ids)
+        g.profile(warmup=3, iters=10, topk=2, passes=3)
+        total, schemas, cands = g.select_path(sn.SN_SELECT_DPRS)
+    stream.synchronize()
+    tune = time.perf_counter() - t0
+    g.set_option(sn.SN_OPT_CUDA_GRAPH, 1)
+    xd = torch.from_numpy(x).to(dt).cuda()
+    y = g.new_output()
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
+    with torch.cuda.stream(stream):
+        for _ in range(5):
+            g.run(xd, y)
+    stream.synchronize()
+    lat = []
+    for _ in range(20):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(stream):
+            flush.zero_()
+            a.record(stream)
+            g.run(xd, y)
+            b.record(stream)
+        stream.synchronize()
+        lat.append(a.elapsed_time(b))
+    t = g.cost_table()
+    path = {}
+    for i in range(1, t["n_layers"] - 1):
+        r = sn.routine_name(int(t["routine"][int(cands[i])]))
+        path[r] = path.get(r, 0) + 1
+    work, _ = conv_work(layers, x.shape)
+    fl = sum(w[0] for w in work)
+    out = {"batch": int(x.shape[0]), "images_per_s": x.shape[0] / statistics.median(lat) * 1e3,
+           "gflop": fl / 1e9, "tflops": fl / statistics.median(lat) / 1e9,
+           "metric": "latency (ms), CUDA-graph replay, L2 flushed", "mean_ms": statistics.mean(lat),
+           "std_ms": statistics.pstdev(lat), "median_ms": statistics.median(lat), "tuning_s": tune,
+           "path_cost_ns": total, "routines_on_path": path,
+           "schemas_on_path": {str(s_): int((schemas == i).sum()) for i, s_ in enumerate(g.schema_universe())}}
+    if keep is not None:
+        keep[name] = (t, layers, x)
+    del g
+    return out
+
+
+def _sweep_rows(sn, torch, synth, Ns, Hs, Cs, ks, ss, lays):
+    rows = []
+    for N in Ns:
+        for H in Hs:
+            for C in Cs:
+                for k in ks:
+                    for s_ in ss:
+                        for lay in lays:
+                            sch = ("f16", lay)
+                            x, layers = synth.single_conv(N, H, C, C, k, s_)
+                            g = _single_layer_graph(sn, layers[0], x.shape, sch)
+                            g.profile(warmup=2, iters=5, topk=0, passes=1)
+                            total, schemas, cands = g.select_path(sn.SN_SELECT_DPRS)
+                            t = g.cost_table()
+                            c = int(cands[1])
+                            xd = torch.zeros(sn.storage_shape(x.shape, lay), dtype=torch.float16, device="cuda")
+                            y = g.new_output()
+                            ms = _time_back_to_back(torch, lambda: g.run(xd, y), reps=10, warm=2)
+                            P = (H + 2 * (k // 2) - k) // s_ + 1
+                            fl = 2 * N * C * P * P * C * k * k
+                            by = 2 * (N * C * H * H + N * C * P * P + C * C * k * k)
+                            rows.append({"N": N, "H": H, "C": C, "k": k, "s": s_, "layout": lay,
+                                         "routine": g.candidate_desc(c), "us": ms * 1e3,
+                                         "tflops": fl / ms / 1e9, "gbs": by / ms / 1e6, "ai": fl / by})
+                            del g
+    return rows
+
+
+def _sweep_summary(sn, torch, synth, pk):
+    """A cut of the single-layer sweep (batch 32, NHWC, stride 1, every H, C and
+    kernel size): per shape the DPRS-chosen routine, and each shape's fraction
+    of the roofline its arithmetic intensity puts it under (back-to-back
+    launches; --config sweep runs the whole sweep)."""
+    sustained = pk.get("bf16_tflops_sustained", pk["bf16_tflops"])
+    ridge = sustained * 1e12 / (pk["hbm_gbs"] * 1e9)
+    rows = _sweep_rows(sn, torch, synth, (32,), (7, 14, 28, 56), (64, 128, 256, 512), (1, 3), (1,), ("nhwc",))
+    out = []
+    for r in rows:
+        tb = r["ai"] > ridge
+        out.append({"H": r["H"], "C": r["C"], "k": r["k"], "us": round(r["us"], 2), "tflops": round(r["tflops"], 1),
+                    "bound": "tensor" if tb else "hbm",
+                    "frac": round(r["tflops"] / sustained if tb else r["gbs"] / pk["hbm_gbs"], 3),
+                    "routine": r["routine"]})
+    tens = [r["frac"] for r in out if r["bound"] == "tensor"]
+    mem = [r["frac"] for r in out if r["bound"] == "hbm"]
+    return {"metric": "single-layer conv, fp16 NHWC, batch 32, stride 1; frac of the sustained tensor peak "
+                      "(AI above the ridge) or of the HBM peak", "ridge_flop_per_byte": ridge,
+            "tensor_bound_median_frac": statistics.median(tens) if tens else None,
+            "hbm_bound_median_frac": statistics.median(mem) if mem else None, "rows": out}
+
+
+def _oracle_times(sn, synth, graphs, g1_table=None):
+    """The oracle on the host cores: one ResNet-50 image with every core and
+    with one thread (a child process with OMP_NUM_THREADS=1), the exhaustive
+    path search on the tiny CNN's profiled cost table and the block-wise exact
+    search on ResNet-50 b1's (section IV problem sizes), with the library's
+    DPRS time on the same tables for comparison."""
+    import oracle
+    from oracle.net import run_net
+    from oracle.paths import blockwise_search
+    out = {"cores": os.cpu_count()}
+    x, layers = synth.resnet50(1)
+    t0 = time.perf_counter()
+    run_net(layers, x, "bf16")
+    out["r50_image_all_cores_s"] = time.perf_counter() - t0
+    code = ("import sys, time; sys.path.insert(0, %r); import synth; from oracle.net import run_net; "
+            "x, l = synth.resnet50(1); t0 = time.perf_counter(); run_net(l, x, 'bf16'); "
+            "print(time.perf_counter() - t0)") % ROOT
+    env = dict(os.environ, OMP_NUM_THREADS="1", CUDA_VISIBLE_DEVICES="")
+    try:
+        r = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True, timeout=300)
+        out["r50_image_1_thread_s"] = float(r.stdout.strip().splitlines()[-1])
+    except Exception as e:  # noqa: BLE001
+        out["r50_image_1_thread_s"] = None
+        out["r50_image_1_thread_error"] = str(e)[:200]
+
+    def layer_cost(t):
+        n, ns = t["n_layers"], t["n_schemas"]
+        return np.array([oracle.fastest_per_schema(t["schema"][t["layer"] == i], t["cost"][t["layer"] == i], ns)
+                         for i in range(n)])
+    if "tiny" in graphs:
+        t = graphs["tiny"][0]
+        lc = layer_cost(t)
+        t0 = time.perf_counter()
+        tot, _, _ = oracle.brute_force(lc, t["edges"], t["adapt"])
+        out["tiny_exhaustive_search_s"] = time.perf_counter() - t0
+        out["tiny_assignments"] = int(t["n_schemas"]) ** int(t["n_layers"] - 2)
+    if g1_table is not None:
+        lc = layer_cost(g1_table)
+        t0 = time.perf_counter()
+        blockwise_search(lc, g1_table["edges"], g1_table["adapt"])
+        out["r50_b1_blockwise_search_s"] = time.perf_counter() - t0
+    return out
+
+
 def run_extra_config(args):
     import torch
     import synth
@@ -659,43 +906,7 @@ def run_extra_config(args):
     torch.cuda.set_device(0)
     out = {"config": args.config, "peaks": pk_kind}
     if args.config == "bandwidth":
-        # depthwise 3x3 (MobileNetV2 shapes) at batch 128 and the adapt conversion on
-        # ResNet-50 b32 activations, each timed from CUDA-graph replays that rotate
-        # through buffer sets totalling four L2 capacities (cold operands, no host
-        # launch cost)
-        rows = []
-        for (N, C, H, s_) in [(128, 144, 56, 1), (128, 96, 112, 2), (128, 192, 28, 1), (128, 576, 14, 1),
-                              (128, 960, 7, 1)]:
-            for lay in ("nhwc", "nchw"):
-                for var in (0, 1):
-                    sch = ("f16", lay)
-                    layer = synth.dwconv(C, 3, s_, act="relu6")
-                    layer["weight"] = np.zeros((C, 1, 3, 3), np.float32)
-                    layer["bias"] = np.zeros(C, np.float32)
-                    g = _single_layer_graph(sn, layer, (N, C, H, H), sch)
-                    _forced(sn, g, "dwconv2/direct", var)
-                    P = (H + 2 - 3) // s_ + 1
-                    bufs = [(torch.zeros(sn.storage_shape((N, C, H, H), lay), dtype=torch.float16, device="cuda"),
-                             g.new_output()) for _ in range(_sets_for(2 * N * C * (H * H + P * P)))]
-                    ms = _time_cold(torch, [(lambda xb=xb, yb=yb: g.run(xb, yb)) for xb, yb in bufs])
-                    del bufs
-                    by = 2 * (N * C * H * H + N * C * P * P) + 2 * 9 * C + 4 * C
-                    rows.append({"kernel": "dwconv2/direct", "variant": sn.variant_name(5, var), "layout": lay,
-                                 "shape": [N, C, H, H], "stride": s_, "us": ms * 1e3, "gbs": by / ms / 1e6,
-                                 "frac": by / ms / 1e6 / hbm})
-        for shp in [(32, 64, 112, 112), (32, 256, 56, 56), (32, 1024, 14, 14)]:
-            for (a_, b_) in [(("bf16", "nchw"), ("bf16", "nhwc")), (("bf16", "nhwc"), ("bf16", "nchw")),
-                             (("f32", "nchw"), ("bf16", "nhwc")), (("bf16", "nhwc"), ("f32", "nchw"))]:
-                dt = {"f32": torch.float32, "bf16": torch.bfloat16}
-                x = torch.zeros(sn.storage_shape(shp, a_[1]), dtype=dt[a_[0]], device="cuda")
-                y = torch.empty(sn.storage_shape(shp, b_[1]), dtype=dt[b_[0]], device="cuda")
-                bufs = [(x, y)] + [(torch.zeros_like(x), torch.empty_like(y))
-                                   for _ in range(_sets_for(x.nbytes + y.nbytes) - 1)]
-                ms = _time_cold(torch, [(lambda xb=xb, yb=yb: sn.convert(xb, a_, b_, shp, out=yb)) for xb, yb in bufs])
-                del bufs
-                by = x.numel() * x.element_size() + y.numel() * y.element_size()
-                rows.append({"kernel": "adapt/convert", "from": "%s.%s" % a_, "to": "%s.%s" % b_, "shape": list(shp),
-                             "us": ms * 1e3, "gbs": by / ms / 1e6, "frac": by / ms / 1e6 / hbm})
+        rows = _bandwidth_rows(sn, torch, synth, hbm)
         # qint8 schema: the quantise / dequantise adapts on ResNet-50 b32 activations
         # and the int8 dense routine at batch 1 (VGG16's fully connected shapes),
         # where the weight codes are the bytes that matter
@@ -775,96 +986,13 @@ def run_extra_config(args):
         out.update({"metric": "single-layer conv2/igemm_tc, bf16 NHWC, device time per launch (CUDA-graph replay)",
                     "layer": [N, C, H, K, k, s_], "gflop": fl / 1e9, "bytes": by, "best": best, "rows": rows})
     elif args.config == "sweep":
-        rows = []
-        for N in (1, 8, 32):
-            for H in (7, 14, 28, 56):
-                for C in (64, 128, 256, 512):
-                    for k in (1, 3):
-                        for s_ in (1, 2):
-                            for lay in ("nhwc", "nchw"):
-                                sch = ("f16", lay)
-                                x, layers = synth.single_conv(N, H, C, C, k, s_)
-                                g = _single_layer_graph(sn, layers[0], x.shape, sch)
-                                g.profile(warmup=2, iters=5, topk=0, passes=1)
-                                total, schemas, cands = g.select_path(sn.SN_SELECT_DPRS)
-                                t = g.cost_table()
-                                c = int(cands[1])
-                                xd = torch.zeros(sn.storage_shape(x.shape, lay), dtype=torch.float16, device="cuda")
-                                y = g.new_output()
-                                ms = _time_back_to_back(torch, lambda: g.run(xd, y), reps=10, warm=2)
-                                P = (H + 2 * (k // 2) - k) // s_ + 1
-                                fl = 2 * N * C * P * P * C * k * k
-                                by = 2 * (N * C * H * H + N * C * P * P + C * C * k * k)
-                                rows.append({"N": N, "H": H, "C": C, "k": k, "s": s_, "layout": lay,
-                                             "routine": sn.routine_name(int(t["routine"][c])),
-                                             "variant": int(t["variant"][c]), "us": ms * 1e3,
-                                             "tflops": fl / ms / 1e9, "gbs": by / ms / 1e6})
+        rows = _sweep_rows(sn, torch, synth, (1, 8, 32), (7, 14, 28, 56), (64, 128, 256, 512), (1, 3), (1, 2),
+                           ("nhwc", "nchw"))
         out.update({"metric": "single-layer conv, fp16, best routine by profiling + DPRS", "rows": rows})
     else:
-        name = args.config
-        if name == "tiny":
-            x, layers = synth.tiny_cnn()
-            sch, io, dt = [("f32", "nchw"), ("f32", "nhwc")], ("f32", "nchw"), torch.float32
-        elif name == "mbv2_b1":
-            x, layers = synth.mobilenet_v2(1)
-            layers = sn.fuse_residual(layers)
-            sch, io, dt = [("f16", "nchw"), ("f16", "nhwc")], ("f16", "nchw"), torch.float16
-        elif name == "mbv3_b1":
-            x, layers = synth.mobilenet_v3(1)
-            layers = sn.fuse_residual(layers)
-            sch, io, dt = [("f16", "nchw"), ("f16", "nhwc")], ("f16", "nchw"), torch.float16
-        elif name == "vgg16_b32":
-            x, layers = synth.vgg16(32)
-            sch, io, dt = [("bf16", "nchw"), ("bf16", "nhwc")], ("bf16", "nchw"), torch.bfloat16
-        elif name == "vgg16_b1":
-            x, layers = synth.vgg16(1)
-            sch, io, dt = [("f16", "nchw"), ("f16", "nhwc")], ("f16", "nchw"), torch.float16
-        else:
-            x, layers = synth.resnet50(1)
-            layers = sn.fuse_residual(layers)
-            sch, io, dt = [("f16", "nchw"), ("f16", "nhwc")], ("f16", "nchw"), torch.float16
-        stream = torch.cuda.Stream()
-        t0 = time.perf_counter()
-        with torch.cuda.stream(stream):
-            g = sn.build_graph(layers, x.shape, io, io, sch)
-            g.profile(warmup=3, iters=10, topk=2, passes=3)
-            total, schemas, cands = g.select_path(sn.SN_SELECT_DPRS)
-        stream.synchronize()
-        tune = time.perf_counter() - t0
-        g.set_option(sn.SN_OPT_CUDA_GRAPH, 1)
-        xd = torch.from_numpy(x).to(dt).cuda()
-        y = g.new_output()
-        flush = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
-        with torch.cuda.stream(stream):
-            for _ in range(5):
-                g.run(xd, y)
-        stream.synchronize()
-        lat = []
-        torch.cuda.nvtx.range_push("sn_timed")
-        for _ in range(20):
-            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            with torch.cuda.stream(stream):
-                flush.zero_()
-                a.record(stream)
-                g.run(xd, y)
-                b.record(stream)
-            stream.synchronize()
-            lat.append(a.elapsed_time(b))
-        torch.cuda.nvtx.range_pop()
-        t = g.cost_table()
-        path = {}
-        for i in range(1, t["n_layers"] - 1):
-            r = sn.routine_name(int(t["routine"][int(cands[i])]))
-            path[r] = path.get(r, 0) + 1
-        work, _ = conv_work(layers, x.shape)
-        fl = sum(w[0] for w in work)
-        out.update({"batch": int(x.shape[0]), "images_per_s": x.shape[0] / statistics.median(lat) * 1e3,
-                    "gflop": fl / 1e9, "tflops": fl / statistics.median(lat) / 1e9})
-        out.update({"metric": "latency (ms), CUDA-graph replay, L2 flushed", "mean_ms": statistics.mean(lat),
-                    "std_ms": statistics.pstdev(lat), "median_ms": statistics.median(lat), "tuning_s": tune,
-                    "path_cost_ns": total, "routines_on_path": path,
-                    "schemas_on_path": {str(s_): int((schemas == i).sum()) for i, s_ in enumerate(g.schema_universe())}})
+        out.update(_latency_config(sn, torch, synth, args.config))
     print(json.dumps(out))
+
 
 if __name__ == "__main__":
     main()

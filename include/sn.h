@@ -168,6 +168,22 @@ SN_API sn_status sn_add_layer(sn_graph *g, int32_t type, const void *params, con
  * sn_add_input after a layer). */
 SN_API sn_status sn_add_input(sn_graph *g, const int64_t in_nchw[4], int32_t *input_id);
 SN_API sn_status sn_set_outputs(sn_graph *g, const int32_t *layer_ids, int32_t n);
+/* Residual-add fusion, the graph optimiser pass run before tuning (section
+ * III-A: layers are fused ahead of profiling and routine selection): every
+ * SN_L_ADD one of whose inputs is an SN_L_CONV2 with SN_ACT_NONE and one
+ * input, read by nothing else and not a net output, is replaced by that
+ * conv2 with the add's other input as a residual and the add's activation,
+ * y = act(conv(x) + bias + residual) (the conv2-with-residual layer of
+ * sn_add_layer).  The fused layer takes the add's place and the conv2 is
+ * removed, so layer ids change: new_id[old] (n_ids = the number of layers
+ * added so far; may be NULL) receives each old id's new id, -1 for a conv2
+ * folded into its add; net output ids are remapped.  *n_fused (may be NULL)
+ * = the number of adds fused.  Call after the last sn_add_layer /
+ * sn_set_outputs and before anything that finalises the net (cost table,
+ * profiling, path selection, run).
+ * Errors: SN_ESTATE (net already finalised), SN_EINVAL (NULL graph, n_ids
+ * not the number of layers). */
+SN_API sn_status sn_fuse_residual(sn_graph *g, int32_t *new_id, int32_t n_ids, int32_t *n_fused);
 SN_API sn_status sn_get_io(sn_graph *g, int32_t *n_inputs, int32_t *n_outputs);
 
 /* ---------------- the cost table (profiling data, section III-C) ----------
@@ -263,6 +279,21 @@ SN_API sn_status sn_set_path(sn_graph *g, const int32_t *candidate, int32_t n_la
                                boundaries between them go); 0 = one launch per
                                layer.  Profiling and sn_run_timed always run
                                one launch per layer.                             */
+#define SN_OPT_SHARE_BUFFERS 4 /* 1 (default) = activation blobs whose live
+                               ranges do not overlap share bytes of the plan's
+                               arena (sn_plan_memory); 0 = every blob its own
+                               bytes.  The outputs are the same either way.   */
+#define SN_OPT_WAIT_LIMIT 3 /* SM clock cycles that one pipeline wait of a
+                               tensor-core routine (conv2/igemm_tc and the
+                               routines built on it) may take before the kernel
+                               stops, lets its own copies and MMAs land, frees
+                               its tensor memory, records the cause in the
+                               library's error word and returns (sn_run then
+                               reports SN_ETIMEOUT under SN_OPT_CHECK and
+                               clears the word).  0 (default) = about 2 s at
+                               the maximum clock.  A small value makes waits
+                               that would have completed expire: the run's
+                               output is then not valid.                         */
 SN_API sn_status sn_set_option(sn_graph *g, int32_t option, int64_t value);
 
 /* Run the net with the selected path: in_dev holds the input in in_schema,
@@ -271,6 +302,18 @@ SN_API sn_status sn_set_option(sn_graph *g, int32_t option, int64_t value);
  * builds the plan (adapt insertion, buffers, weight copies per schema).
  * Errors: SN_ESTATE (no path), SN_ENOMEM, SN_ECUDA, SN_ETIMEOUT. */
 SN_API sn_status sn_run(sn_graph *g, const void *in_dev, void *out_dev, void *stream);
+/* sn_run from and to host memory: the input is copied from in_host (host
+ * memory holding the input in in_schema, the full tensor) into a device
+ * buffer the graph owns, the net runs, and the output is copied back to
+ * out_host (out_schema, the full tensor), all asynchronously on `stream`:
+ * read out_host only after synchronising the stream.  Page-locked host
+ * buffers (cudaHostAlloc / cudaHostRegister) make the copies asynchronous;
+ * pageable ones work but the copies then synchronise with the host.  Both
+ * host buffers are the caller's and must stay valid until the stream has
+ * passed this call.  Nets with one input and one output only.
+ * Errors: as sn_run, plus SN_EINVAL for a net with several inputs or
+ * outputs and SN_ENOMEM when the device staging buffers cannot be made. */
+SN_API sn_status sn_run_host(sn_graph *g, const void *in_host, void *out_host, void *stream);
 /* sn_run for a net with several inputs or outputs: in_devs[0..n_in) in the
  * order of their ids (-1, -2, ...), out_devs[0..n_out) in the order given to
  * sn_set_outputs.  n_in and n_out must match the net (SN_EINVAL otherwise);
@@ -291,6 +334,15 @@ SN_API sn_status sn_run_timed(sn_graph *g, const void *in_dev, void *out_dev, vo
  * that one sn_run launches.  Either output may be NULL.
  * Errors: SN_ESTATE (no path), plus those of plan building. */
 SN_API sn_status sn_plan_stats(sn_graph *g, int32_t *n_ops, int32_t *n_kernels, void *stream);
+/* Device memory of the current plan's activations (built on `stream` if
+ * needed): *arena_bytes = the one allocation that holds every graph-owned
+ * blob, placed by liveness (a blob lives from the op that writes it to the
+ * last op that reads it; blobs live at the same time never share bytes);
+ * *unshared_bytes = what the same blobs take one allocation each.  The
+ * caller's input and output buffers, weights and the routines' workspace are
+ * not counted.  Either output may be NULL.
+ * Errors: SN_ESTATE (no path), plus those of plan building. */
+SN_API sn_status sn_plan_memory(sn_graph *g, int64_t *arena_bytes, int64_t *unshared_bytes, void *stream);
 
 /* Logical output shape of internal layer `layer` (N, C, H, W). */
 SN_API sn_status sn_layer_shape(sn_graph *g, int32_t layer, int64_t out_nchw[4]);
@@ -308,6 +360,13 @@ SN_API void sn_graph_destroy(sn_graph *g);
 SN_API const char *sn_routine_name(int32_t routine);
 /* Human-readable routine parameters of (routine, variant), e.g. "bn=128". */
 SN_API const char *sn_variant_name(int32_t routine, int32_t variant);
+/* Descriptor of candidate `cand` of a graph (section III-C: a routine is
+ * identified by its descriptor and its routine parameters): routine name,
+ * the schema it reads (and "->" the one it writes when they differ) and its
+ * parameter values, e.g. "conv2/igemm_tc bf16.nhwc [bn=128 cta=2 kb=2 ...]".
+ * The string lives in thread-local storage until the next call on the same
+ * thread.  NULL for a NULL graph, an unfinalisable graph or a bad index. */
+SN_API const char *sn_candidate_desc(sn_graph *g, int32_t cand);
 
 /* Adapt routine on its own (section III-C, jobs (2) and (3)): convert the
  * N x C x H x W blob x_dev stored in `from` into y_dev stored in `to`

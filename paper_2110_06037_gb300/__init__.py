@@ -11,10 +11,10 @@ Schemas are (dtype, layout) pairs: dtype "f32" | "f16" | "bf16" | "qi8"
 Graph.calibrate), layout "nchw" | "nhwc".  Nets may have several inputs
 (Graph.add_input) and outputs (Graph.set_outputs, Graph.run_multi).
 """
-from ._sn import (SN_SELECT_BRUTE, SN_SELECT_DPRS, SN_OPT_CHAIN, SN_OPT_CHECK, SN_OPT_CUDA_GRAPH, SnError, lib,
+from ._sn import (SN_SELECT_BRUTE, SN_SELECT_DPRS, SN_OPT_CHAIN, SN_OPT_CHECK, SN_OPT_CUDA_GRAPH, SN_OPT_WAIT_LIMIT, SN_OPT_SHARE_BUFFERS, SnError, lib,
                   routine_name, variant_name)
 from .api import Graph, convert, convert_q, storage_shape
-from .netbuild import build_graph, fuse_residual
+from .netbuild import build_graph, fuse_residual, fused_description
 
-__all__ = ["Graph", "convert", "convert_q", "build_graph", "fuse_residual", "storage_shape", "SnError", "lib", "routine_name",
-           "variant_name", "SN_SELECT_DPRS", "SN_SELECT_BRUTE", "SN_OPT_CHAIN", "SN_OPT_CHECK", "SN_OPT_CUDA_GRAPH"]
+__all__ = ["Graph", "convert", "convert_q", "build_graph", "fuse_residual", "fused_description", "storage_shape", "SnError", "lib", "routine_name",
+           "variant_name", "SN_SELECT_DPRS", "SN_SELECT_BRUTE", "SN_OPT_CHAIN", "SN_OPT_CHECK", "SN_OPT_CUDA_GRAPH", "SN_OPT_WAIT_LIMIT", "SN_OPT_SHARE_BUFFERS"]

@@ -22,7 +22,7 @@ SN_NCHW, SN_NHWC = 0, 1
 SN_L_CONV2, SN_L_DWCONV2, SN_L_MAXPOOL, SN_L_GAP, SN_L_ADD, SN_L_DENSE, SN_L_MUL = range(7)
 SN_ACT = {"none": 0, None: 0, "relu": 1, "relu6": 2, "hswish": 3, "hsigmoid": 4}
 SN_SELECT_DPRS, SN_SELECT_BRUTE = 0, 1
-SN_OPT_CUDA_GRAPH, SN_OPT_CHECK, SN_OPT_CHAIN = 0, 1, 2
+SN_OPT_CUDA_GRAPH, SN_OPT_CHECK, SN_OPT_CHAIN, SN_OPT_WAIT_LIMIT, SN_OPT_SHARE_BUFFERS = 0, 1, 2, 3, 4
 COST_INF = np.iinfo(np.int64).max
 
 DTYPES = {"f32": SN_F32, "f16": SN_F16, "bf16": SN_BF16, "qi8": SN_QI8}
@@ -87,15 +87,19 @@ SIGNATURES = {
     "sn_set_path": (C.c_int, [C.c_void_p, C.POINTER(C.c_int32), C.c_int32]),
     "sn_set_option": (C.c_int, [C.c_void_p, C.c_int32, C.c_int64]),
     "sn_run": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p]),
+    "sn_run_host": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p]),
+    "sn_fuse_residual": (C.c_int, [C.c_void_p, C.POINTER(C.c_int32), C.c_int32, C.POINTER(C.c_int32)]),
     "sn_run_timed": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.POINTER(C.c_float),
                                C.POINTER(C.c_float)]),
     "sn_layer_shape": (C.c_int, [C.c_void_p, C.c_int32, C.POINTER(C.c_int64)]),
     "sn_plan_stats": (C.c_int, [C.c_void_p, C.POINTER(C.c_int32), C.POINTER(C.c_int32), C.c_void_p]),
+    "sn_plan_memory": (C.c_int, [C.c_void_p, C.POINTER(C.c_int64), C.POINTER(C.c_int64), C.c_void_p]),
     "sn_save_plan": (C.c_int, [C.c_void_p, C.c_char_p]),
     "sn_load_plan": (C.c_int, [C.c_void_p, C.c_char_p]),
     "sn_graph_destroy": (None, [C.c_void_p]),
     "sn_routine_name": (C.c_char_p, [C.c_int32]),
     "sn_variant_name": (C.c_char_p, [C.c_int32, C.c_int32]),
+    "sn_candidate_desc": (C.c_char_p, [C.c_void_p, C.c_int32]),
     "sn_convert": (C.c_int, [C.c_void_p, sn_schema, C.c_void_p, sn_schema, C.POINTER(C.c_int64), C.c_void_p]),
     "sn_convert_q": (C.c_int, [C.c_void_p, sn_schema, C.c_void_p, sn_schema, C.POINTER(C.c_int64), C.c_float,
                                C.c_void_p]),

@@ -125,6 +125,18 @@ class Graph:
         self.n_user += 1
         return out.value
 
+    def fuse_residual(self):
+        """sn_fuse_residual: the library's residual-add fusion pass.  Returns
+        (new_id, n_fused): new_id[old] = each added layer's new id (-1 for a
+        conv2 folded into its add)."""
+        m = self.n_user
+        ids = (C.c_int32 * max(m, 1))()
+        nf = C.c_int32()
+        check(lib().sn_fuse_residual(self.h, ids, m, C.byref(nf)))
+        new_id = [int(ids[i]) for i in range(m)]
+        self.n_user = sum(1 for v in new_id if v >= 0)
+        return new_id, nf.value
+
     # ------------------------------------------------------------ cost table
     def cost_table(self):
         t = _sn.sn_cost_table()
@@ -168,6 +180,13 @@ class Graph:
             out.append((dt, ly))
         return out
 
+    def candidate_desc(self, cand):
+        """Descriptor string of candidate `cand`: routine, schema, parameter values."""
+        d = lib().sn_candidate_desc(self.h, int(cand))
+        if d is None:
+            raise _sn.SnError(_sn.SN_EINVAL, f"no candidate {cand}")
+        return d.decode()
+
     # -------------------------------------------------------- tune and select
     def profile(self, warmup=3, iters=20, topk=2, passes=5, stream=None):
         o = _sn.sn_profile_opts(warmup, iters, topk, passes)
@@ -199,6 +218,13 @@ class Graph:
         ops, kern = C.c_int32(), C.c_int32()
         check(lib().sn_plan_stats(self.h, C.byref(ops), C.byref(kern), _stream_ptr(stream)))
         return ops.value, kern.value
+
+
+    def plan_memory(self, stream=None):
+        """(arena bytes, bytes the same activations take unshared) of the plan."""
+        a, b = C.c_int64(), C.c_int64()
+        check(lib().sn_plan_memory(self.h, C.byref(a), C.byref(b), _stream_ptr(stream)))
+        return a.value, b.value
 
     def save_plan(self, path):
         check(lib().sn_save_plan(self.h, str(path).encode()))
@@ -235,6 +261,14 @@ class Graph:
             out = self.new_output()
         check(lib().sn_run(self.h, C.c_void_p(x.data_ptr()), C.c_void_p(out.data_ptr()), _stream_ptr(stream)))
         return out
+
+    def run_host(self, x_host, out_host, stream=None):
+        """sn_run_host: x_host / out_host are host tensors (pinned for asynchronous
+        copies) of the input and output; the copies run inside the library, on the
+        stream; synchronise the stream before reading out_host."""
+        check(lib().sn_run_host(self.h, C.c_void_p(x_host.data_ptr()), C.c_void_p(out_host.data_ptr()),
+                                _stream_ptr(stream)))
+        return out_host
 
     def output_shapes(self):
         """Logical shapes of the net outputs (in order)."""

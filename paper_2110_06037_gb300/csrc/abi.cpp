@@ -40,6 +40,19 @@ const char *sn_variant_name(int32_t routine, int32_t variant) {
     return variant_name(routine, variant);
 }
 
+const char *sn_candidate_desc(sn_graph *gg, int32_t cand) {
+    static thread_local std::string buf;
+    try {
+        if (!gg) return nullptr;
+        Graph *g = reinterpret_cast<Graph *>(gg);
+        if (graph_finalize(g) != SN_OK || cand < 0 || cand >= (int32_t)g->cands.size()) return nullptr;
+        buf = candidate_desc(*g, cand);
+        return buf.c_str();
+    } catch (...) {
+        return nullptr;
+    }
+}
+
 sn_status sn_graph_create(const int64_t in_nchw[4], sn_schema in_schema, sn_schema out_schema,
                           const sn_schema *schemas, int32_t n_schemas, sn_alloc_fn alloc,
                           sn_free_fn free_fn, void *alloc_ctx, sn_graph **out) {
@@ -267,6 +280,20 @@ sn_status sn_set_option(sn_graph *gg, int32_t option, int64_t value) {
             }
         } else if (option == SN_OPT_CHECK) {
             g->opt_check = value ? 1 : 0;
+        } else if (option == SN_OPT_WAIT_LIMIT) {
+            if (value < 0) return fail(SN_EINVAL, "sn_set_option: the wait limit is a cycle count >= 0");
+            if (g->opt_wait_limit != value) {
+                g->opt_wait_limit = value;
+                if (g->gexec) {  // the limit is a launch argument baked into a captured graph
+                    cudaGraphExecDestroy(g->gexec);
+                    g->gexec = nullptr;
+                }
+            }
+        } else if (option == SN_OPT_SHARE_BUFFERS) {
+            if (g->opt_share != (value ? 1 : 0)) {
+                g->opt_share = value ? 1 : 0;
+                invalidate_plan(g);
+            }
         } else if (option == SN_OPT_CHAIN) {
             if (g->opt_chain != (value ? 1 : 0)) {
                 g->opt_chain = value ? 1 : 0;
@@ -351,6 +378,36 @@ sn_status sn_run(sn_graph *gg, const void *in_dev, void *out_dev, void *stream) 
     })
 }
 
+sn_status sn_run_host(sn_graph *gg, const void *in_host, void *out_host, void *stream) {
+    SN_GUARD({
+        if (!gg || !in_host || !out_host) return fail(SN_EINVAL, "sn_run_host: NULL argument");
+        Graph *g = G(gg);
+        sn_status rc = graph_finalize(g);
+        if (rc != SN_OK) return rc;
+        if (g->n_in() != 1 || g->n_out() != 1)
+            return fail(SN_EINVAL, "sn_run_host: the net has several inputs or outputs");
+        const Shape &os = g->layers[g->layers.back().inputs[0]].out;
+        const size_t in_bytes = (size_t)g->in_shape.numel() * dtype_size(g->in_schema.dtype);
+        const size_t out_bytes = (size_t)os.numel() * dtype_size(g->out_schema.dtype);
+        if (g->host_in.bytes < in_bytes) {
+            dev_free(g, &g->host_in);
+            if ((rc = dev_alloc(g, in_bytes, &g->host_in)) != SN_OK) return rc;
+        }
+        if (g->host_out.bytes < out_bytes) {
+            dev_free(g, &g->host_out);
+            if ((rc = dev_alloc(g, out_bytes, &g->host_out)) != SN_OK) return rc;
+        }
+        cudaStream_t st = static_cast<cudaStream_t>(stream);
+        SN_CUDA_TRY(cudaMemcpyAsync(g->host_in.ptr, in_host, in_bytes, cudaMemcpyHostToDevice, st));
+        IoPtrs io;
+        io.in = {g->host_in.ptr};
+        io.out = {g->host_out.ptr};
+        if ((rc = run_io(g, io, st)) != SN_OK) return rc;
+        SN_CUDA_TRY(cudaMemcpyAsync(out_host, g->host_out.ptr, out_bytes, cudaMemcpyDeviceToHost, st));
+        return SN_OK;
+    })
+}
+
 sn_status sn_run_multi(sn_graph *gg, const void *const *in_devs, int32_t n_in, void *const *out_devs, int32_t n_out,
                        void *stream) {
     SN_GUARD({
@@ -359,6 +416,22 @@ sn_status sn_run_multi(sn_graph *gg, const void *const *in_devs, int32_t n_in, v
         io.in.assign(in_devs, in_devs + n_in);
         io.out.assign(out_devs, out_devs + n_out);
         return run_io(G(gg), io, static_cast<cudaStream_t>(stream));
+    })
+}
+
+sn_status sn_fuse_residual(sn_graph *gg, int32_t *new_id, int32_t n_ids, int32_t *n_fused) {
+    SN_GUARD({
+        if (!gg) return fail(SN_EINVAL, "sn_fuse_residual: NULL graph");
+        Graph *g = G(gg);
+        if (new_id && n_ids != (int32_t)g->user.size())
+            return fail(SN_EINVAL, "sn_fuse_residual: new_id must have one entry per layer added (" +
+                                       std::to_string(g->user.size()) + ")");
+        std::vector<int32_t> map;
+        sn_status rc = fuse_residual(g, map, n_fused);
+        if (rc != SN_OK) return rc;
+        if (new_id)
+            for (size_t i = 0; i < map.size(); ++i) new_id[i] = map[i];
+        return SN_OK;
     })
 }
 
@@ -445,6 +518,21 @@ sn_status sn_plan_stats(sn_graph *gg, int32_t *n_ops, int32_t *n_kernels, void *
         }
         if (n_ops) *n_ops = (int32_t)g->plan.size();
         if (n_kernels) *n_kernels = kern;
+        return SN_OK;
+    })
+}
+
+sn_status sn_plan_memory(sn_graph *gg, int64_t *arena_bytes, int64_t *unshared_bytes, void *stream) {
+    SN_GUARD({
+        if (!gg) return fail(SN_EINVAL, "sn_plan_memory: NULL graph");
+        Graph *g = G(gg);
+        if (!g->has_path) return fail(SN_ESTATE, "sn_plan_memory: select or set a routine path first");
+        if (!g->plan_valid) {
+            sn_status rc = build_plan(g, static_cast<cudaStream_t>(stream));
+            if (rc != SN_OK) return rc;
+        }
+        if (arena_bytes) *arena_bytes = (int64_t)g->arena.bytes;
+        if (unshared_bytes) *unshared_bytes = (int64_t)g->arena_unshared;
         return SN_OK;
     })
 }

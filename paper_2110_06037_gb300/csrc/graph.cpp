@@ -40,6 +40,9 @@ Graph::~Graph() {
     for (auto &kv : weight_cache) dev_free(this, &kv.second);
     for (auto &kv : bias_cache) dev_free(this, &kv.second);
     dev_free(this, &workspace);
+    dev_free(this, &arena);
+    dev_free(this, &host_in);
+    dev_free(this, &host_out);
 }
 
 sn_status dev_alloc(Graph *g, size_t bytes, Buffer *b) {
@@ -67,6 +70,11 @@ sn_status dev_alloc(Graph *g, size_t bytes, Buffer *b) {
 }
 
 void dev_free(Graph *g, Buffer *b) {
+    if (b->view) {
+        b->ptr = nullptr;
+        b->view = false;
+        return;
+    }
     if (!b->ptr) return;
     if (g->free_fn) g->free_fn(b->ptr, g->alloc_ctx);
     else cudaFree(b->ptr);
@@ -253,6 +261,69 @@ sn_status set_outputs(Graph *g, const int32_t *ids, int32_t n) {
         v.push_back(ids[i]);
     }
     g->outputs = v;
+    return SN_OK;
+}
+
+// Graph optimiser pass run before tuning (section III-A fuses layers ahead of
+// tuning): every add whose input is a conv2 without activation, read by
+// nothing else and not a net output, becomes that conv2 with the add's other
+// input as a residual and the add's activation, y = act(conv(x) + b + r).
+// The fused layer takes the add's place (after both of its inputs) and the
+// conv2 is dropped; the user layers are renumbered.  new_id[old] = the new
+// id of each old user layer (-1 for a conv2 folded into its add).
+sn_status fuse_residual(Graph *g, std::vector<int32_t> &new_id, int32_t *n_fused) {
+    if (g->finalized) return fail(SN_ESTATE, "sn_fuse_residual: the net is already finalised (fuse before tuning)");
+    const int32_t m = (int32_t)g->user.size(), m_in = g->n_in();
+    std::vector<std::vector<int32_t>> consumers(m);
+    for (int32_t i = 0; i < m; ++i)
+        for (int32_t j : g->user[i].inputs)
+            if (j >= m_in) consumers[j - m_in].push_back(i);
+    std::vector<char> is_output(m, 0);
+    for (int32_t u : g->outputs) is_output[u] = 1;
+    if (g->outputs.empty() && m > 0) is_output[m - 1] = 1;
+    std::vector<int32_t> fold_conv(m, -1), fold_other(m, -1);  // per add: the folded conv2, the residual
+    std::vector<char> dropped(m, 0);
+    int32_t nf = 0;
+    for (int32_t i = 0; i < m; ++i) {
+        const Layer &a = g->user[i];
+        if (a.type != SN_L_ADD || a.inputs.size() != 2) continue;
+        for (int pos = 0; pos < 2; ++pos) {
+            const int32_t jj = a.inputs[pos], other = a.inputs[1 - pos];
+            if (jj < m_in || jj == other) continue;
+            const int32_t j = jj - m_in;
+            const Layer &c = g->user[j];
+            if (c.type != SN_L_CONV2 || c.inputs.size() != 1 || c.conv.act != SN_ACT_NONE) continue;
+            if (consumers[j].size() != 1 || consumers[j][0] != i || is_output[j] || dropped[j]) continue;
+            fold_conv[i] = j;
+            fold_other[i] = other;
+            dropped[j] = 1;
+            ++nf;
+            break;
+        }
+    }
+    new_id.assign(m, -1);
+    std::vector<Layer> out;
+    for (int32_t i = 0; i < m; ++i) {
+        if (dropped[i]) continue;
+        new_id[i] = (int32_t)out.size();
+        if (fold_conv[i] >= 0) {
+            Layer f = g->user[fold_conv[i]];
+            f.inputs = {f.inputs[0], fold_other[i]};
+            f.conv.act = g->user[i].act;
+            f.act = g->user[i].act;
+            f.out = g->user[i].out;
+            f.qscale = g->user[i].qscale;
+            out.push_back(std::move(f));
+        } else {
+            out.push_back(g->user[i]);
+        }
+    }
+    for (Layer &l : out)
+        for (int32_t &j : l.inputs)
+            if (j >= m_in) j = new_id[j - m_in] + m_in;
+    for (int32_t &u : g->outputs) u = new_id[u];
+    g->user = std::move(out);
+    if (n_fused) *n_fused = nf;
     return SN_OK;
 }
 

@@ -35,6 +35,7 @@
 #include <algorithm>
 #include <cstdio>
 #include <mutex>
+#include <string>
 #include <type_traits>
 #include <vector>
 
@@ -173,7 +174,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                 krange(w);
                 const int b = lt & 1;
                 const uint32_t aph = (uint32_t)(lt >> 1) & 1u;
-                bool ok = G == 2 ? mbar_wait_cluster(&acce_bar[b], aph ^ 1u) : mbar_wait(&acce_bar[b], aph ^ 1u);
+                bool ok = G == 2 ? mbar_wait_cluster(&acce_bar[b], aph ^ 1u, p.wait_limit) : mbar_wait(&acce_bar[b], aph ^ 1u, p.wait_limit);
                 if (!ok) {
                     if (lane == 0) atomicOr(p.err, ERR_EPI_WAIT);
                     set_abort();
@@ -181,7 +182,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                 __syncwarp();  // bar.red is warp-aligned: reconverge after the polling loops
                 if (bar_red_or(BAR_MMA, 64, !ok || abort_sh)) break;
                 for (int it = w.it0; it < w.it1; ++it) {
-                    ok = mbar_wait(&full_bar[s], par);
+                    ok = mbar_wait(&full_bar[s], par, p.wait_limit);
                     if (!ok) {
                         if (lane == 0) atomicOr(p.err, ERR_MMA_WAIT);
                         set_abort();
@@ -231,7 +232,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                 int r = (int)fdiv((uint32_t)tap, p.fd_S), ss = tap - r * S;
                 for (int it = w.it0; it < w.it1; ++it, ++g) {
                     if (g % NPROD == prod) {
-                        if (!mbar_wait(&empty_bar[s], par ^ 1u)) {
+                        if (!mbar_wait(&empty_bar[s], par ^ 1u, p.wait_limit)) {
                             atomicOr(p.err, ERR_TMA_WAIT);
                             set_abort();
                         }
@@ -303,7 +304,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             const uint64_t descb = sdesc_sw128(su32(bst));   // weight-stationary B, K step 0
             int g = 0, lt = 0, s = 0;
             bool stop = false;
-            if (BST && lane == 0 && !mbar_wait(&bst_bar, 0u)) {
+            if (BST && lane == 0 && !mbar_wait(&bst_bar, 0u, p.wait_limit)) {
                 atomicOr(p.err, ERR_MMA_WAIT);
                 set_abort();
             }
@@ -353,7 +354,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             int g = 0, lt = 0, s = 0;
             uint32_t par = 0;
             bool stop = false;
-            if (BST && !mbar_wait(&bst_bar, 0u)) {
+            if (BST && !mbar_wait(&bst_bar, 0u, p.wait_limit)) {
                 atomicOr(p.err, ERR_MMA_WAIT);
                 set_abort();
                 stop = true;
@@ -363,7 +364,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                 krange(w);
                 const int b = lt & 1;
                 const uint32_t aph = (uint32_t)(lt >> 1) & 1u;
-                const bool drained = G == 2 ? mbar_wait_cluster(&acce_bar[b], aph ^ 1u) : mbar_wait(&acce_bar[b], aph ^ 1u);
+                const bool drained = G == 2 ? mbar_wait_cluster(&acce_bar[b], aph ^ 1u, p.wait_limit) : mbar_wait(&acce_bar[b], aph ^ 1u, p.wait_limit);
                 if (!drained) {
                     atomicOr(p.err, ERR_EPI_WAIT);
                     set_abort();
@@ -372,7 +373,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                 tc_fence_after();
                 const uint32_t d = tmem + (uint32_t)(b * MS * BN);
                 for (int it = w.it0; it < w.it1; ++it, ++g) {
-                    if (!mbar_wait(&full_bar[s], par)) {
+                    if (!mbar_wait(&full_bar[s], par, p.wait_limit)) {
                         atomicOr(p.err, ERR_MMA_WAIT);
                         set_abort();
                         stop = true;
@@ -420,7 +421,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             const uint32_t aph = (uint32_t)(lt >> 1) & 1u;
             const Work w = work_of(p, u, BN, IMPLICIT, G, MS, 0);
             const bool tile_live = w.mt < p.mtiles;
-            if (!mbar_wait(&accf_bar[b], aph)) {
+            if (!mbar_wait(&accf_bar[b], aph, p.wait_limit)) {
                 if (lane == 0) atomicOr(p.err, ERR_ACC_WAIT);
                 set_abort();
                 break;
@@ -434,7 +435,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                 uint32_t v[64];
                 __syncwarp();
                 tmem_ld64(taddr, v);
-                if (!mbar_wait_cluster(&xfree_bar[warp - 2], xph)) {
+                if (!mbar_wait_cluster(&xfree_bar[warp - 2], xph, p.wait_limit)) {
                     if (lane == 0) atomicOr(p.err, ERR_EPI_WAIT);
                     set_abort();
                     stop = true;
@@ -472,6 +473,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         const int cbase = (ALT || MS == 2) ? 0 : half * CPH;  // first chunk of this warp
         int lt = ALT ? half : 0;
         uint32_t rpar = 0;  // phase parity of this warp's residual barrier
+        int res_issued = 0, res_landed = 0;  // residual loads issued / waited for (warp-uniform)
         uint32_t xph = 0;   // cluster K split: phase parity of this warp's exchange block
         bool waited = false;
         for (int u = cid + (ALT ? half * ncl : 0); u < total; u += (ALT ? 2 : 1) * ncl, lt += ALT ? 2 : 1) {
@@ -513,7 +515,9 @@ __global__ void __launch_bounds__(THREADS, 1)
             }
             const bool has_res = p.res != nullptr && p.ksplit == 1;
             auto issue_res = [&](int k0) {
-                if (!has_res || !tile_live || k0 >= p.K) return;
+                // no new copies once the kernel is stopping
+                if (!has_res || !tile_live || k0 >= p.K || __shfl_sync(0xffffffffu, (int)abort_sh, 0)) return;
+                ++res_issued;
                 if (lane == 0) {
                     bulk_wait_read_0();
                     mbar_expect_tx(&res_bar[warp - 2], STG_BYTES);
@@ -524,7 +528,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                 }
             };
             issue_res(w.n0 + 64 * cbase);
-            if (!mbar_wait(&accf_bar[b], aph)) {
+            if (!mbar_wait(&accf_bar[b], aph, p.wait_limit)) {
                 if (lane == 0) atomicOr(p.err, ERR_ACC_WAIT);
                 set_abort();
                 break;
@@ -551,11 +555,14 @@ __global__ void __launch_bounds__(THREADS, 1)
                         for (int j = 0; j < 16; ++j) rv[h][j] = 0u;
                     if (!has_res && lane == 0) bulk_wait_read_0();  // the previous store has read the block
                     if (has_res) {
-                        if (!mbar_wait(&res_bar[warp - 2], rpar)) {
+                        const bool landed = mbar_wait(&res_bar[warp - 2], rpar, p.wait_limit);
+                        rpar ^= 1u;
+                        if (!__all_sync(0xffffffffu, landed)) {
                             if (lane == 0) atomicOr(p.err, ERR_EPI_WAIT);
                             set_abort();
+                            break;
                         }
-                        rpar ^= 1u;
+                        ++res_landed;
 #pragma unroll
                         for (int j = 0; j < 8; ++j) {
                             const uint4 u = *reinterpret_cast<const uint4 *>(buf + lane * 128 + ((j ^ (lane & 7)) << 4));
@@ -571,7 +578,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                     if (CSK == 2) {
                         // add CTA 1's partial of the same rows and channels, then
                         // hand its exchange block back
-                        if (!mbar_wait_cluster(&xfull_bar[warp - 2], xph)) {
+                        if (!mbar_wait_cluster(&xfull_bar[warp - 2], xph, p.wait_limit)) {
                             if (lane == 0) atomicOr(p.err, ERR_EPI_WAIT);
                             set_abort();
                         }
@@ -658,8 +665,15 @@ __global__ void __launch_bounds__(THREADS, 1)
             }
         }
         // the last stores have read their staging blocks before the CTA's shared
-        // memory is released (their global writes complete with the grid)
-        if (lane == 0) bulk_wait_read_0();
+        // memory is released (their global writes complete with the grid), and
+        // after an abort the residual loads still in flight have landed
+        if (lane == 0) {
+            bulk_wait_read_0();
+            const long long t0 = clock64();
+            for (int i = res_landed; i < res_issued; ++i)
+                while (!mbar_try(&res_bar[warp - 2], (uint32_t)i & 1u) && clock64() - t0 < WAIT_LIMIT) {
+                }
+        }
         __syncwarp();
     }
 
@@ -1036,6 +1050,23 @@ bool conv_tc_chain_shape(const Layer &l, const Shape &in, sn_schema s, int32_t v
     return !cf.implicit || w * h * n == tc::BM;
 }
 
+// the routine parameters of variant v for a layer, spelled out: output-channel
+// tile, CTAs per tile, channel blocks per stage, 128-row halves per tile, K
+// split, weight-stationary B, cluster K split, and the pixel tiling
+std::string conv_tc_config_desc(const Layer &l, const Shape &in, sn_schema s, int32_t v, int32_t a_blocks) {
+    const std::vector<tc::Config> cfgs = tc::configs(l, in, s, a_blocks);
+    if (v < 0 || v >= (int)cfgs.size()) return "?";
+    const tc::Config &c = cfgs[v];
+    char b[160];
+    if (c.implicit)
+        snprintf(b, sizeof(b), "bn=%d cta=%d kb=%d rows=%d ksplit=%d bst=%d csk=%d tile=%dx%dx%d", c.BN, c.G, c.KB,
+                 128 * c.ms * c.G, c.ksplit, c.bst ? 1 : 0, c.csk, c.BW, c.BH, c.BNI);
+    else
+        snprintf(b, sizeof(b), "bn=%d cta=%d kb=%d rows=%d ksplit=%d bst=%d csk=%d plain", c.BN, c.G, c.KB,
+                 128 * c.ms * c.G, c.ksplit, c.bst ? 1 : 0, c.csk);
+    return b;
+}
+
 size_t conv_tc_ws(const Layer &l, const Shape &in, sn_schema s, int32_t v, int32_t a_blocks) {
     const std::vector<tc::Config> cfgs = tc::configs(l, in, s, a_blocks);
     if (v < 0 || v >= (int)cfgs.size() || cfgs[v].ksplit == 1) return 0;
@@ -1070,6 +1101,7 @@ cudaError_t conv_tc(const LaunchArgs &a) {
     p.res = a.in[1];  // residual input of a fused add (null when the layer has one input)
     if (p.res && (uintptr_t)p.res % 16) return cudaErrorInvalidValue;  // read as 16-byte vectors
     p.err = device_error_word();
+    p.wait_limit = a.wait_limit > 0 ? a.wait_limit : WAIT_LIMIT;
     p.M = in.n * (int64_t)in.h * in.w;
     p.Mout = (int64_t)p.N * p.P * p.Q;
     p.ntiles = (p.K + cf.BN - 1) / cf.BN;

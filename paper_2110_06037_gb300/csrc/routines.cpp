@@ -47,6 +47,23 @@ const char *variant_name(int32_t r, int32_t v) {
     }
 }
 
+std::string candidate_desc(const Graph &g, int32_t cand) {
+    const Candidate &c = g.cands[cand];
+    const Layer &L = g.layers[c.layer];
+    std::string d = routine_name(c.routine) ? routine_name(c.routine) : "?";
+    d += " " + schema_str(g.schemas[c.schema]);
+    if (cand_out(c) != c.schema) d += "->" + schema_str(g.schemas[cand_out(c)]);
+    std::vector<Shape> in;
+    for (int32_t j : L.inputs) in.push_back(g.layers[j].out);
+    std::string params;
+    if (c.routine == R_CONV_TC && !in.empty())
+        params = k::conv_tc_config_desc(L, in[0], g.schemas[c.schema], c.variant);
+    else
+        params = variant_name(c.routine, c.variant);
+    if (!params.empty()) d += " [" + params + "]";
+    return d;
+}
+
 static bool is_conv(const Layer &l) { return l.type == SN_L_CONV2; }
 
 // qint8 schema: the routines that have an int8 kernel (one variant each)

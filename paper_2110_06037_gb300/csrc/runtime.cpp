@@ -38,10 +38,83 @@ static cudaError_t convert_blob(const void *x, sn_schema a, void *y, sn_schema b
 // stand-in scale of qint8 blobs while profiling (timing does not depend on it)
 constexpr float kProfileQScale = 1.0f / 64.0f;
 
+static bool chain_eligible(const Graph *g, const PlanOp &op);
+
+// Activation buffers by liveness (the plan step of section III-C): every
+// graph-owned blob is live from the op that writes it to the last op that
+// reads it, in plan order (an op's inputs and its output are live together,
+// so no op writes over what it reads); blobs whose live ranges overlap get
+// disjoint places in one arena, the others may share bytes.  Ops of a chained
+// launch run at once, so what they touch is live across the whole chain.
+// Placement: largest blob first, at the lowest offset (256-byte aligned) free
+// of every placed blob it is live with.
+static sn_status place_slots(Graph *g) {
+    const size_t ns = g->slots.size();
+    std::vector<int32_t> first(ns, INT32_MAX), last(ns, -1);
+    auto touch = [&](int32_t s, int32_t a, int32_t b) {
+        if (s < 0) return;
+        first[s] = std::min(first[s], a);
+        last[s] = std::max(last[s], b);
+    };
+    for (size_t q = 0; q < g->plan.size(); ++q) {
+        const PlanOp &op = g->plan[q];
+        for (int32_t s : op.in_slots) touch(s, (int32_t)q, (int32_t)q);
+        touch(op.out_slot, (int32_t)q, (int32_t)q);
+    }
+    if (g->opt_chain && !g->profiling)
+        for (const auto &r : chain_runs(g))
+            for (int32_t q = r.first; q <= r.second; ++q) {
+                for (int32_t s : g->plan[q].in_slots) touch(s, r.first, r.second);
+                touch(g->plan[q].out_slot, r.first, r.second);
+            }
+    struct Item {
+        size_t s, bytes, off;
+    };
+    std::vector<Item> items;
+    size_t unshared = 0;
+    for (size_t s = g->n_ext; s < ns; ++s) {
+        if (last[s] < 0) continue;  // never referenced
+        const size_t bytes = ((size_t)g->slot_shape[s].numel() * dtype_size(g->slot_schema[s].dtype) + 255) & ~size_t(255);
+        items.push_back({s, bytes, 0});
+        unshared += bytes;
+    }
+    std::sort(items.begin(), items.end(),
+              [](const Item &a, const Item &b) { return a.bytes != b.bytes ? a.bytes > b.bytes : a.s < b.s; });
+    size_t total = 0;
+    for (size_t i = 0; i < items.size(); ++i) {
+        Item &it = items[i];
+        std::vector<std::pair<size_t, size_t>> busy;  // [off, end) of placed blobs live with this one
+        for (size_t j = 0; j < i; ++j) {
+            const Item &o = items[j];
+            if (!g->opt_share || (first[o.s] <= last[it.s] && first[it.s] <= last[o.s]))
+                busy.push_back({o.off, o.off + o.bytes});
+        }
+        std::sort(busy.begin(), busy.end());
+        size_t off = 0;
+        for (const auto &b : busy) {
+            if (off + it.bytes <= b.first) break;
+            off = std::max(off, b.second);
+        }
+        it.off = off;
+        total = std::max(total, off + it.bytes);
+    }
+    sn_status rc = dev_alloc(g, total, &g->arena);
+    if (rc != SN_OK) return rc;
+    for (const Item &it : items) {
+        g->slots[it.s].ptr = static_cast<uint8_t *>(g->arena.ptr) + it.off;
+        g->slots[it.s].bytes = it.bytes;
+        g->slots[it.s].view = true;
+    }
+    g->arena_unshared = unshared;
+    return SN_OK;
+}
+
 sn_status build_plan(Graph *g, cudaStream_t st) {
     if (!g->has_path) return fail(SN_ESTATE, "no routine path selected");
     invalidate_plan(g);
     for (auto &b : g->slots) dev_free(g, &b);
+    dev_free(g, &g->arena);
+    g->arena_unshared = 0;
     g->slots.clear();
     g->slot_shape.clear();
     g->slot_schema.clear();
@@ -146,9 +219,8 @@ sn_status build_plan(Graph *g, cudaStream_t st) {
             return fail(SN_ESTATE, "the path keeps a blob in qi8 without a scale (sn_set_qscale or sn_calibrate)");
         }
     }
-    for (size_t s = g->n_ext; s < g->slots.size(); ++s) {
-        const size_t bytes = (size_t)g->slot_shape[s].numel() * dtype_size(g->slot_schema[s].dtype);
-        sn_status rc = dev_alloc(g, bytes, &g->slots[s]);
+    {
+        sn_status rc = place_slots(g);
         if (rc != SN_OK) return rc;
     }
     if (ws > g->workspace.bytes) {
@@ -184,9 +256,8 @@ static bool chain_eligible(const Graph *g, const PlanOp &op) {
 
 // Group maximal runs of two or more consecutive chain-eligible ops of one
 // dtype into chains and upload their descriptors.
-sn_status build_chains(Graph *g, cudaStream_t st) {
-    g->chains.clear();
-    g->op_chain.assign(g->plan.size(), -1);
+std::vector<std::pair<int32_t, int32_t>> chain_runs(const Graph *g) {
+    std::vector<std::pair<int32_t, int32_t>> runs;
     const size_t n = g->plan.size();
     auto dtype_of = [&](size_t q) { return g->schemas[g->cands[g->plan[q].cand].schema].dtype; };
     size_t i = 0;
@@ -197,7 +268,19 @@ sn_status build_chains(Graph *g, cudaStream_t st) {
         }
         size_t j = i;
         while (j + 1 < n && chain_eligible(g, g->plan[j + 1]) && dtype_of(j + 1) == dtype_of(i)) ++j;
-        if (j > i) {
+        if (j > i) runs.push_back({(int32_t)i, (int32_t)j});
+        i = j + 1;
+    }
+    return runs;
+}
+
+sn_status build_chains(Graph *g, cudaStream_t st) {
+    g->chains.clear();
+    g->op_chain.assign(g->plan.size(), -1);
+    auto dtype_of = [&](size_t q) { return g->schemas[g->cands[g->plan[q].cand].schema].dtype; };
+    for (const auto &run : chain_runs(g)) {
+        const size_t i = (size_t)run.first, j = (size_t)run.second;
+        {
             std::vector<ChainOp> ops;
             for (size_t q = i; q <= j; ++q) {
                 const PlanOp &op = g->plan[q];
@@ -240,7 +323,6 @@ sn_status build_chains(Graph *g, cudaStream_t st) {
             SN_CUDA_TRY(cudaStreamSynchronize(st));  // `blob` is freed on return
             for (size_t q = i; q <= j; ++q) g->op_chain[q] = (int32_t)g->chains.size() - 1;
         }
-        i = j + 1;
     }
     return SN_OK;
 }
@@ -280,6 +362,7 @@ static sn_status launch_op(Graph *g, const PlanOp &op, const IoPtrs &io, cudaStr
     a.bias = op.bias;
     a.ws = g->workspace.ptr;
     a.ws_bytes = g->workspace.bytes;
+    a.wait_limit = g->opt_wait_limit;
     a.stream = st;
     return launch_routine(a);
 }

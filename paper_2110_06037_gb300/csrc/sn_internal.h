@@ -99,6 +99,7 @@ inline int32_t cand_out(const Candidate &c) { return c.out_schema < 0 ? c.schema
 struct Buffer {  // device allocation owned by the graph
     void *ptr = nullptr;
     size_t bytes = 0;
+    bool view = false;  // a part of another buffer (the activation arena): not freed on its own
 };
 
 struct PlanOp {
@@ -164,6 +165,9 @@ struct LaunchArgs {
     // qint8 routines: scales of the input blobs and of the output blob
     float qs_in[2] = {0.0f, 0.0f};
     float qs_out = 0.0f;
+    // tensor-core routines: SM cycles a pipeline wait may take before the
+    // kernel gives up and reports SN_ETIMEOUT (0 = the library default)
+    int64_t wait_limit = 0;
     cudaStream_t stream = nullptr;
 };
 
@@ -204,7 +208,12 @@ struct Graph {
     std::map<std::string, Buffer> weight_cache;  // key: layer/format/dtype
     std::map<int32_t, Buffer> bias_cache;        // per layer fp32 bias
     Buffer workspace;
+    Buffer arena;                     // the plan's activation buffers, placed by liveness
+    size_t arena_unshared = 0;        // what the activation buffers would take one allocation each
+    Buffer host_in, host_out;         // device staging of sn_run_host
     int opt_graph = 0, opt_check = 0;
+    int64_t opt_wait_limit = 0;       // SN_OPT_WAIT_LIMIT (0 = default)
+    int opt_share = 1;                // SN_OPT_SHARE_BUFFERS: place activations by liveness
     int opt_chain = 0;                // run runs of tensor-core convolutions as chained launches
     std::vector<ChainPlan> chains;    // built with the plan
     std::vector<int32_t> op_chain;    // per plan op: its chain, or -1
@@ -228,6 +237,7 @@ struct Graph {
 };
 
 sn_status graph_finalize(Graph *g);
+sn_status fuse_residual(Graph *g, std::vector<int32_t> &new_id, int32_t *n_fused);
 sn_status add_input(Graph *g, const int64_t nchw[4], int32_t *id);
 sn_status set_outputs(Graph *g, const int32_t *ids, int32_t n);
 
@@ -245,6 +255,8 @@ int32_t routine_variants(int32_t routine, const Layer &layer, const std::vector<
                          sn_schema s);
 const char *routine_name(int32_t routine);
 const char *variant_name(int32_t routine, int32_t variant);
+// descriptor of one candidate of a graph: routine name, schema and routine parameters
+std::string candidate_desc(const Graph &g, int32_t cand);
 size_t routine_workspace(int32_t routine, int32_t variant, const Layer &layer,
                          const std::vector<Shape> &in, sn_schema s);
 // prepare weights for (layer, routine, variant, schema); returns device pointer
@@ -277,6 +289,8 @@ void fastest_per_schema(const Graph &g, std::vector<int64_t> &F, std::vector<int
 // plan + run
 sn_status build_plan(Graph *g, cudaStream_t st);
 sn_status build_chains(Graph *g, cudaStream_t st);
+// [first op, last op] of every run of plan ops that a chained launch would run
+std::vector<std::pair<int32_t, int32_t>> chain_runs(const Graph *g);
 sn_status run_plan(Graph *g, const IoPtrs &io, cudaStream_t st,
                    std::vector<cudaEvent_t> *evs);
 // one run of the plan replayed from a CUDA graph with a timing node around
@@ -319,6 +333,7 @@ int32_t conv_tc_variants(const Layer &l, const Shape &in, sn_schema s);
 size_t conv_tc_ws(const Layer &l, const Shape &in, sn_schema s, int32_t v, int32_t a_blocks = 0);  // K-split partials
 size_t dense_tc_ws(const Layer &l, const Shape &in, sn_schema s, int32_t v);
 const char *conv_tc_variant_name(int32_t v);
+std::string conv_tc_config_desc(const Layer &l, const Shape &in, sn_schema s, int32_t v, int32_t a_blocks = 0);
 // chained launches of consecutive tensor-core convolutions
 bool conv_tc_chain_shape(const Layer &l, const Shape &in, sn_schema s, int32_t v, bool *implicit, int *bn, int *kb,
                          int *bw, int *bh, int *bni);

@@ -63,6 +63,7 @@ struct Params {
     const void *res;               // residual added before the activation (output's layout), or null
     float *part;                   // K split: fp32 partial sums [ksplit][Mout][K]
     int *err;                      // the library's device error word
+    long long wait_limit;          // SM cycles a pipeline wait may take before the kernel gives up
 };
 
 // ---------------------------------------------------------------- PTX helpers
@@ -88,12 +89,34 @@ __device__ __forceinline__ bool mbar_try(uint64_t *b, uint32_t parity) {
         : "memory");
     return ok != 0;
 }
-// bounded wait for the phase with the given parity; false on expiry
-__device__ __forceinline__ bool mbar_wait(uint64_t *b, uint32_t parity) {
+// non-suspending test of the phase with the given parity
+__device__ __forceinline__ bool mbar_test(uint64_t *b, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(su32(b)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+// bounded wait for the phase with the given parity (limit in SM cycles);
+// false on expiry.  try_wait may suspend the thread inside the hardware for
+// a while, so a limit shorter than the default polls with test_wait instead,
+// which lets even a limit of a few cycles be honoured.
+__device__ __forceinline__ bool mbar_wait(uint64_t *b, uint32_t parity, long long limit = WAIT_LIMIT) {
+    if (limit < WAIT_LIMIT) {
+        if (mbar_test(b, parity)) return true;
+        const long long t0 = clock64();
+        while (!mbar_test(b, parity))
+            if (clock64() - t0 > limit) return false;
+        return true;
+    }
     if (mbar_try(b, parity)) return true;
     const long long t0 = clock64();
     while (!mbar_try(b, parity))
-        if (clock64() - t0 > WAIT_LIMIT) return false;
+        if (clock64() - t0 > limit) return false;
     return true;
 }
 
@@ -229,11 +252,29 @@ __device__ __forceinline__ bool mbar_try_cluster(uint64_t *b, uint32_t parity) {
         : "memory");
     return ok != 0;
 }
-__device__ __forceinline__ bool mbar_wait_cluster(uint64_t *b, uint32_t parity) {
+__device__ __forceinline__ bool mbar_test_cluster(uint64_t *b, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.test_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(su32(b)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+__device__ __forceinline__ bool mbar_wait_cluster(uint64_t *b, uint32_t parity, long long limit = WAIT_LIMIT) {
+    if (limit < WAIT_LIMIT) {
+        if (mbar_test_cluster(b, parity)) return true;
+        const long long t0 = clock64();
+        while (!mbar_test_cluster(b, parity))
+            if (clock64() - t0 > limit) return false;
+        return true;
+    }
     if (mbar_try_cluster(b, parity)) return true;
     const long long t0 = clock64();
     while (!mbar_try_cluster(b, parity))
-        if (clock64() - t0 > WAIT_LIMIT) return false;
+        if (clock64() - t0 > limit) return false;
     return true;
 }
 __device__ __forceinline__ void st_cluster_v4(uint32_t caddr, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {

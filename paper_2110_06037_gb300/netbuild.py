@@ -15,9 +15,13 @@ TYPES = {"conv2": _sn.SN_L_CONV2, "dwconv2": _sn.SN_L_DWCONV2, "maxpool": _sn.SN
 
 
 def build_graph(layers, in_shape, in_schema, out_schema, schemas, torch_alloc=True, extra_inputs=(),
-                outputs=None) -> Graph:
+                outputs=None, fuse=False) -> Graph:
     """extra_inputs: shapes of net inputs -2, -3, ...; outputs: layer indices
-    of the net outputs (default: the last layer)."""
+    of the net outputs (default: the last layer).  fuse=True runs the
+    library's residual-add fusion pass (sn_fuse_residual) before anything
+    finalises the net; the graph then has the layers of
+    fused_description(layers, g.fused_ids) and g.fused_ids maps the given
+    layer indices to the graph's."""
     g = Graph(in_shape, in_schema, out_schema, schemas, torch_alloc=torch_alloc)
     for k, shp in enumerate(extra_inputs):
         assert g.add_input(shp) == -2 - k
@@ -27,50 +31,43 @@ def build_graph(layers, in_shape, in_schema, out_schema, schemas, torch_alloc=Tr
         assert lid == i
     if outputs is not None:
         g.set_outputs(list(outputs))
+    g.fused_ids = None
+    if fuse:
+        g.fused_ids, _ = g.fuse_residual()
     return g
 
 
-def fuse_residual(layers):
-    """Fuse every residual add into the convolution that feeds it.
-
-    A graph-optimiser pass over the plain-data description, run before the
-    net is built and tuned (the paper fuses layers ahead of tuning, section
-    III-A): an 'add' whose input is a 'conv2' with no activation, read by
-    nothing else, becomes that conv2 with the add's other input as a
-    residual and the add's activation, y = act(conv(x) + b + residual).  The
-    fused layer takes the add's place in the list (after both of its inputs)
-    and the conv2 is dropped; indices are renumbered.  Returns a new list.
-    """
-    consumers = {}
+def fused_description(layers, new_id):
+    """The plain-data description of the net after the library's fusion pass,
+    read off its id map (new_id[old], -1 for a folded conv2): a kept layer is
+    copied with its inputs renumbered; an add one of whose inputs was folded
+    becomes that conv2 with the add's other input as its residual and the
+    add's activation.  This only restates, for the Python side, what
+    sn_fuse_residual did to the graph."""
+    out = [None] * (max(new_id) + 1 if new_id else 0)
     for i, l in enumerate(layers):
-        for j in l["inputs"]:
-            consumers.setdefault(j, []).append(i)
-    fold = {}  # add index -> (conv index, residual index)
-    for i, l in enumerate(layers):
-        if l["type"] != "add":
+        k = new_id[i]
+        if k < 0:
             continue
-        for pos in (0, 1):
-            j, other = l["inputs"][pos], l["inputs"][1 - pos]
-            if j < 0 or layers[j]["type"] != "conv2" or len(layers[j]["inputs"]) != 1:
-                continue
-            if layers[j]["params"].get("act", "none") != "none" or consumers.get(j) != [i]:
-                continue
-            fold[i] = (j, other)
-            break
-    dropped = {j for (j, _) in fold.values()}
-    new_index, out = {}, []
-    for i, l in enumerate(layers):
-        if i in dropped:
-            continue
-        new_index[i] = len(out)
-        if i in fold:
-            j, other = fold[i]
+        folded = [j for j in l["inputs"] if j >= 0 and new_id[j] < 0] if l["type"] == "add" else []
+        if folded:
+            j = folded[0]
+            other = l["inputs"][1] if l["inputs"][0] == j else l["inputs"][0]
             conv = layers[j]
             params = dict(conv["params"], act=l["params"].get("act", "none"))
-            out.append(dict(conv, name=conv.get("name", "conv") + "+" + l.get("name", "add"), params=params,
-                            inputs=[conv["inputs"][0], other]))
+            d = dict(conv, name=conv.get("name", "conv") + "+" + l.get("name", "add"), params=params,
+                     inputs=[conv["inputs"][0], other])
         else:
-            out.append(dict(l))
-    for l in out:
-        l["inputs"] = [j if j < 0 else new_index[j] for j in l["inputs"]]
+            d = dict(l)
+        d["inputs"] = [j if j < 0 else new_id[j] for j in d["inputs"]]
+        out[k] = d
     return out
+
+
+def fuse_residual(layers, in_shape, extra_inputs=(), outputs=None):
+    """Run the library's residual-add fusion pass (sn_fuse_residual) on a
+    host-only graph of the net and return the fused plain-data description
+    (see fused_description)."""
+    g = build_graph(layers, in_shape, ("f32", "nchw"), ("f32", "nchw"), [("f32", "nchw")], torch_alloc=False,
+                    extra_inputs=extra_inputs, outputs=outputs, fuse=True)
+    return fused_description(layers, g.fused_ids)

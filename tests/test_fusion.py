@@ -13,7 +13,7 @@ import pytest
 
 import synth
 from oracle.net import run_net
-from paper_2110_06037_gb300 import SnError, _sn, build_graph, fuse_residual
+from paper_2110_06037_gb300 import SnError, _sn, build_graph, fuse_residual, fused_description
 from paper_2110_06037_gb300.api import Graph
 
 from test_dprs import check_against_oracle, random_costs
@@ -25,12 +25,12 @@ def _counts(layers):
 
 
 def test_fuse_resnet50_and_mobilenet_v2_structure():
-    _, r50 = synth.resnet50(1, res=32)
-    f = fuse_residual(r50)
+    xr, r50 = synth.resnet50(1, res=32)
+    f = fuse_residual(r50, xr.shape)
     assert _counts(r50) == (16, 0) and _counts(f) == (0, 16)
     assert len(f) == len(r50) - 16
-    _, mb = synth.mobilenet_v2(1, res=32)
-    fm = fuse_residual(mb)
+    xm, mb = synth.mobilenet_v2(1, res=32)
+    fm = fuse_residual(mb, xm.shape)
     assert _counts(mb)[0] == 10 and _counts(fm) == (0, 10)
     for net in (f, fm):
         for i, l in enumerate(net):
@@ -40,7 +40,7 @@ def test_fuse_resnet50_and_mobilenet_v2_structure():
     # the fused layer takes the add's activation; a conv with an activation is left alone
     assert all(l["params"]["act"] == "relu" for l in f if len(l["inputs"]) == 2)
     x, tiny = synth.tiny_cnn()
-    assert fuse_residual(tiny) == tiny
+    assert fuse_residual(tiny, x.shape) == tiny
 
 
 def _residual_net(rng):
@@ -60,7 +60,7 @@ def _residual_net(rng):
 def test_oracle_fused_equals_conv_then_add():
     rng = np.random.default_rng(3)
     net = _residual_net(rng)
-    f = fuse_residual(net)
+    f = fuse_residual(net, (2, 4, 7, 5))
     assert [l["type"] for l in f] == ["conv2", "conv2", "gap"] and f[1]["inputs"] == [0, 0]
     x = rng.standard_normal((2, 4, 7, 5)).astype(np.float32)
     a = run_net(net, x, "f32")
@@ -71,7 +71,7 @@ def test_oracle_fused_equals_conv_then_add():
 def test_oracle_fused_resnet50_equals_unfused():
     x, r50 = synth.resnet50(1, res=32)
     a = run_net(r50, x, "bf16")
-    b = run_net(fuse_residual(r50), x, "bf16")
+    b = run_net(fuse_residual(r50, x.shape), x, "bf16")
     assert np.array_equal(a, b)
 
 
@@ -93,10 +93,55 @@ def test_residual_shape_checked_and_routines_offered():
 @pytest.mark.parametrize("net", ["resnet50", "mobilenet_v2"])
 def test_dprs_on_fused_nets_equals_blockwise_search(net):
     _, layers = (synth.resnet50(1, res=32) if net == "resnet50" else synth.mobilenet_v2(1, res=32))
-    layers = fuse_residual(layers)
+    layers = fuse_residual(layers, (1, 3, 32, 32))
     sch = [("f16", "nchw"), ("f16", "nhwc")]
     g = build_graph(layers, (1, 3, 32, 32), ("f32", "nchw"), ("f32", "nchw"), sch, torch_alloc=False)
     for seed in range(3):
         rng = np.random.default_rng(100 + seed)
         t = random_costs(g, rng, p_inf=0.05)
         check_against_oracle(g, t, exhaustive=False)
+
+
+def test_library_pass_through_the_c_abi():
+    """sn_fuse_residual on the graph itself (what a C caller gets): ResNet-50
+    loses its 16 adds and 16 convs, the id map sends each add to its fused
+    layer and each folded conv2 to -1, the outputs follow the map, and once
+    the net is finalised the pass is refused with SN_ESTATE."""
+    import ctypes as C
+    x, r50 = synth.resnet50(1, res=32)
+    g = build_graph(r50, x.shape, ("f16", "nchw"), ("f16", "nchw"), [("f16", "nhwc")], torch_alloc=False)
+    m = len(r50)
+    ids = (C.c_int32 * m)()
+    nf = C.c_int32()
+    assert _sn.lib().sn_fuse_residual(g.h, ids, m, C.byref(nf)) == _sn.SN_OK
+    assert nf.value == 16
+    new_id = list(ids)
+    adds = [i for i, l in enumerate(r50) if l["type"] == "add"]
+    assert sum(1 for v in new_id if v < 0) == 16
+    assert all(new_id[i] >= 0 for i in adds)
+    folded = [i for i, v in enumerate(new_id) if v < 0]
+    assert all(r50[i]["type"] == "conv2" and r50[i]["params"]["act"] == "none" for i in folded)
+    kept = [v for v in new_id if v >= 0]
+    assert kept == list(range(m - 16))  # renumbered in order
+    g.n_user = m - 16
+    t = g.cost_table()
+    assert t["n_layers"] == m - 16 + 2  # + the auxiliary input and output layers
+    # one edge per layer input of the fused description, plus the output layer's
+    assert len(t["edges"]) == sum(len(l["inputs"]) for l in fused_description(r50, new_id)) + 1
+    with pytest.raises(SnError) as e:
+        g.fuse_residual()
+    assert e.value.status == _sn.SN_ESTATE
+
+
+def test_library_pass_leaves_nets_without_residual_adds_alone():
+    x, tiny = synth.tiny_cnn()
+    g = build_graph(tiny, x.shape, ("f32", "nchw"), ("f32", "nchw"), [("f32", "nchw")], torch_alloc=False,
+                    fuse=True)
+    assert g.fused_ids == list(range(len(tiny)))
+    # an add fed by a conv2 that has an activation, or by a conv2 read twice, stays
+    rng = np.random.default_rng(5)
+    net = _residual_net(rng)
+    net[1]["params"] = dict(net[1]["params"], act="relu")
+    g = build_graph(net, (2, 4, 7, 5), ("f32", "nchw"), ("f32", "nchw"), [("f32", "nchw")], torch_alloc=False,
+                    fuse=True)
+    assert g.fused_ids == [0, 1, 2, 3]

@@ -65,7 +65,7 @@ def _run(g, xd, chain, graph=False):
 def test_chained_run_equals_per_layer_launches_bit_for_bit(dt):
     import torch
     x, layers = synth.resnet50(2, res=64)
-    fused = fuse_residual(layers)
+    fused = fuse_residual(layers, x.shape)
     sch = (dt, "nhwc")
     g = build_graph(fused, x.shape, (dt, "nchw"), (dt, "nchw"), [sch])
     n_tc = _force_tc(g, fused, lambda i, n: 0)  # variant 0: 64-channel tiles, one CTA, no K split
@@ -87,7 +87,7 @@ def test_chained_run_equals_per_layer_launches_bit_for_bit(dt):
 @pytest.mark.parametrize("seed", [1, 2, 3])
 def test_chained_run_with_mixed_variants_matches_oracle(seed):
     x, layers = synth.resnet50(2, res=96, seed=seed)
-    fused = fuse_residual(layers)
+    fused = fuse_residual(layers, x.shape)
     g = build_graph(fused, x.shape, ("bf16", "nchw"), ("bf16", "nchw"), [("bf16", "nhwc")])
     rng = np.random.default_rng(seed)
     _force_tc(g, fused, lambda i, n: int(rng.integers(0, n)))
@@ -102,7 +102,7 @@ def test_chained_run_with_mixed_variants_matches_oracle(seed):
 def test_profiled_resnet50_b32_runs_chained():
     import torch
     x, layers = synth.resnet50(32)
-    fused = fuse_residual(layers)
+    fused = fuse_residual(layers, x.shape)
     g = build_graph(fused, x.shape, ("bf16", "nchw"), ("bf16", "nchw"), [("bf16", "nchw"), ("bf16", "nhwc")])
     g.profile(warmup=1, iters=3, topk=1, passes=2)
     g.select_path(SN_SELECT_DPRS)

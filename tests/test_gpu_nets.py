@@ -157,14 +157,14 @@ def test_resnet50_b32_bf16_sampled():
 
 def test_fused_mobilenet_v2_b1_fp16():
     x, layers = synth.mobilenet_v2(1)
-    fused = fuse_residual(layers)
+    fused = fuse_residual(layers, x.shape)
     g, got = _profile_select_run(fused, x, ("f16", "nchw"), ("f16", "nchw"), F16, exhaustive=False)
     assert maxrel(got, run_net(layers, x, "f16")) <= TOL["f16"]
 
 
 def test_fused_resnet50_b1_fp16():
     x, layers = synth.resnet50(1)
-    fused = fuse_residual(layers)
+    fused = fuse_residual(layers, x.shape)
     g, got = _profile_select_run(fused, x, ("f16", "nchw"), ("f16", "nchw"), F16, exhaustive=False)
     assert maxrel(got, run_net(layers, x, "f16")) <= TOL["f16"]
 
@@ -172,7 +172,7 @@ def test_fused_resnet50_b1_fp16():
 def test_fused_resnet50_b32_bf16_sampled():
     import torch
     x, layers = synth.resnet50(32)
-    fused = fuse_residual(layers)
+    fused = fuse_residual(layers, x.shape)
     g = build_graph(fused, x.shape, ("bf16", "nchw"), ("bf16", "nchw"), BF16)
     g.profile(warmup=1, iters=3, topk=1, passes=2)
     t = g.cost_table()
@@ -186,3 +186,58 @@ def test_fused_resnet50_b32_bf16_sampled():
     for n in (0, 17):
         ref = run_net(layers, x[n:n + 1], "bf16")
         assert maxrel(got[n:n + 1], ref) <= TOL["bf16"]
+
+
+def test_run_host_copies_inside_the_call():
+    """sn_run_host: input from host memory, output to host memory, the copies
+    queued by the library on the caller's stream; same bits as sn_run on
+    device buffers, pinned or pageable host memory, eager or graph replay."""
+    import torch
+    x, layers = synth.resnet50(2, res=64)
+    fused = fuse_residual(layers, x.shape)
+    g = build_graph(fused, x.shape, ("bf16", "nchw"), ("bf16", "nchw"), BF16)
+    g.profile(warmup=1, iters=2, topk=1, passes=1)
+    g.select_path(SN_SELECT_DPRS)
+    xd = to_device(x, ("bf16", "nchw"))
+    ref = g.run(xd)
+    torch.cuda.synchronize()
+    s = torch.cuda.Stream()
+    for graph in (0, 1):
+        g.set_option(SN_OPT_CUDA_GRAPH, graph)
+        for pinned in (True, False):
+            xh = xd.cpu().pin_memory() if pinned else xd.cpu()
+            oh = torch.empty(ref.shape, dtype=ref.dtype).pin_memory() if pinned else torch.empty(ref.shape, dtype=ref.dtype)
+            for _ in range(2):
+                g.run_host(xh, oh, stream=s)
+            s.synchronize()
+            assert torch.equal(oh, ref.cpu()), (graph, pinned)
+
+
+@pytest.mark.parametrize("chain", [0, 1])
+def test_liveness_arena_same_bits_less_memory(chain):
+    """Activations placed by liveness in one arena give the same bits as one
+    place per blob, with and without chained launches, and take less memory
+    without them (ResNet-50, profiled path, batch 2)."""
+    import torch
+    from paper_2110_06037_gb300 import SN_OPT_CHAIN, SN_OPT_SHARE_BUFFERS
+    x, layers = synth.resnet50(2, res=96)
+    g = build_graph(layers, x.shape, ("bf16", "nchw"), ("bf16", "nchw"), BF16, fuse=True)
+    g.profile(warmup=1, iters=2, topk=1, passes=1)
+    g.select_path(SN_SELECT_DPRS)
+    g.set_option(SN_OPT_CHAIN, chain)
+    xd = to_device(x, ("bf16", "nchw"))
+    g.set_option(SN_OPT_SHARE_BUFFERS, 0)
+    y0 = g.run(xd).clone()
+    a0, u0 = g.plan_memory()
+    g.set_option(SN_OPT_SHARE_BUFFERS, 1)
+    y1 = g.run(xd)
+    y2 = g.run(xd)
+    torch.cuda.synchronize()
+    a1, u1 = g.plan_memory()
+    assert u0 == u1 and a0 == u0
+    # a chained launch keeps everything it touches live across the chain, so
+    # sharing then only happens outside it
+    assert a1 <= u1 if chain else a1 < 0.5 * u1, (a1, u1)
+    assert torch.equal(y0, y1) and torch.equal(y1, y2)
+    ref = run_net(layers, x, "bf16")
+    assert maxrel(from_device(y1, ("bf16", "nchw")), ref) <= TOL["bf16"]

@@ -188,3 +188,21 @@ def test_calibration_needs_costs_and_a_single_input():
     assert g2.get_qscale(-2) == 0.25 and g2.get_qscale(-1) == 0.0
     with pytest.raises(SnError):
         g2.set_qscale(-3, 1.0)
+
+
+def test_candidate_descriptors():
+    """Every candidate has a descriptor naming its routine, the schema it reads
+    and, for the tensor-core routine, the parameter values that tell its
+    variants apart (section III-C: routine descriptor + routine parameters)."""
+    x, layers = synth.single_conv(2, 14, 64, 128, 3, 1)
+    g = build_graph(layers, x.shape, ("bf16", "nhwc"), ("bf16", "nhwc"), [("bf16", "nhwc")], torch_alloc=False)
+    t = g.cost_table()
+    descs = [g.candidate_desc(c) for c in range(len(t["cost"]))]
+    for c, d in enumerate(descs):
+        assert d.startswith(_sn.routine_name(int(t["routine"][c]))), d
+        assert "bf16.nhwc" in d or t["routine"][c] == 0, d
+    tc = [d for c, d in enumerate(descs) if _sn.routine_name(int(t["routine"][c])) == "conv2/igemm_tc"]
+    assert len(tc) > 4 and len(set(tc)) == len(tc), tc  # distinct parameter values per variant
+    assert all("bn=" in d and "tile=" in d for d in tc)
+    with pytest.raises(SnError):
+        g.candidate_desc(len(t["cost"]))
