@@ -54,17 +54,25 @@ def articulation_layers(n, edges):
     return arts
 
 
-def blockwise_search(layer_cost, edges, adapt_cost, max_interior=16):
+def blockwise_search(layer_cost, edges, adapt_cost, max_interior=16, pairs=None):
     """Exact min of T(S) by block brute force + chain DP.
 
     layer_cost: int64 [n, ns] of F_i(lambda) (INF where infeasible);
     edges: (src, dst) pairs; adapt_cost: int64 [n_edges, ns, ns].
     Returns (cost, assignment).  Raises ValueError if a block is too large.
+
+    pairs (routines that write a schema other than the one they read): the
+    states of a layer are then the (read, written) schema pairs pairs[k] and
+    layer_cost is [n, len(pairs)]; an edge (u, v) costs the adapt from u's
+    written schema to v's read schema, nothing when they agree (Def. 1 read
+    for fused boundaries).  adapt_cost stays indexed by schemas.
     """
     lc = np.asarray(layer_cost, dtype=np.int64)
     n, ns = lc.shape
     edges = [tuple(map(int, e)) for e in np.asarray(edges).reshape(-1, 2)]
-    ac = np.asarray(adapt_cost, dtype=np.int64).reshape(len(edges), ns, ns)
+    ac = np.asarray(adapt_cost, dtype=np.int64)
+    nsch = ns if pairs is None else ac.shape[-1]
+    ac = ac.reshape(len(edges), nsch, nsch)
     succ = [[] for _ in range(n)]
     for u, v in edges:
         succ[u].append(v)
@@ -75,6 +83,8 @@ def blockwise_search(layer_cost, edges, adapt_cost, max_interior=16):
         return INF if a == INF or b == INF else a + b
 
     def adapt(e, x, y):
+        if pairs is not None:
+            x, y = pairs[x][1], pairs[y][0]  # written by the producer, read by the consumer
         return 0 if x == y else int(ac[e, x, y])
 
     # assign every layer and edge to the block that contains it
@@ -109,7 +119,8 @@ def blockwise_search(layer_cost, edges, adapt_cost, max_interior=16):
         for x in range(ns):
             for y in range(ns):
                 best, best_asg = INF, None
-                for asg in itertools.product(range(ns), repeat=len(interior)):
+                # only states a layer can take (finite F): the others give INF anyway
+                for asg in itertools.product(*[[z for z in range(ns) if lc[v, z] < INF] for v in interior]):
                     t = 0
                     for v, lam in zip(interior, asg):
                         t = add(t, int(lc[v, lam]))

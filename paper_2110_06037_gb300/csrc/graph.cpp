@@ -403,6 +403,7 @@ sn_status graph_finalize(Graph *g) {
                     for (int32_t so = 0; so < g->n_lambda; ++so)
                         if (so != s && schema_eq(g->schemas[so], o))
                             for (int32_t v = 0; v < nv; ++v) {
+                                if (!fused_variant_ok(r, L[i], in, g->schemas[s], v)) continue;
                                 Candidate c{r, v, s, i, kInf};
                                 c.out_schema = so;
                                 cands.push_back(c);

@@ -502,6 +502,15 @@ __global__ void __launch_bounds__(THREADS, 1)
                 pix = w.m0 + row;
                 valid = pix < p.Mout;
             }
+            // NCHW output (a routine that writes the next layer's layout): this
+            // row's first element of output channel k0 sits at
+            // ((n K + k0) P + p) Q + q; channel c adds c P Q
+            T *ynchw = nullptr;
+            if (p.y_nchw && valid) {
+                const int64_t PQ = (int64_t)p.P * p.Q;
+                const int64_t n_img = pix / PQ;
+                ynchw = static_cast<T *>(p.y) + n_img * p.K * PQ + (pix - n_img * PQ);
+            }
             // the idle CTA of a pair whose group has one tile stores nothing
             const bool tile_live = w.mt < p.mtiles;
             // residual (fused add): the warp's 32 x 64 block of it is loaded by
@@ -624,13 +633,31 @@ __global__ void __launch_bounds__(THREADS, 1)
                         stage_rows([act = p.act](float x) { return act_apply(x, act); });
                     fence_proxy_async_smem();
                     __syncwarp();
-                    if (lane == 0) {
-                        if (IMPLICIT)
-                            tma_store_4d(&mY, buf, k0, w.q0 + wq0, w.p0 + hp0, w.i0 + ni0);
-                        else
-                            tma_store_2d(&mY, buf, k0, (int)(w.m0 + r0));
-                        bulk_commit();
+                    if (!p.y_nchw) {
+                        if (lane == 0) {
+                            if (IMPLICIT)
+                                tma_store_4d(&mY, buf, k0, w.q0 + wq0, w.p0 + hp0, w.i0 + ni0);
+                            else
+                                tma_store_2d(&mY, buf, k0, (int)(w.m0 + r0));
+                            bulk_commit();
+                        }
+                    } else if (ynchw) {
+                        // NCHW output: each lane reads its own row of the staged
+                        // block back, channel by channel (the same rounded values),
+                        // and stores it at its pixel of that channel's plane; a
+                        // warp's rows are consecutive pixels, so each store
+                        // instruction writes neighbouring elements
+                        const int64_t pq = (int64_t)p.P * p.Q;
+                        T *yc = ynchw + (int64_t)k0 * pq;
+                        const int kmax = min(64, p.K - k0);
+                        for (int j = 0; j < kmax; ++j) {
+                            const T val = *reinterpret_cast<const T *>(buf + lane * 128 + (((j >> 3) ^ (lane & 7)) << 4) +
+                                                                       (j & 7) * 2);
+                            yc[(int64_t)j * pq] = val;
+                        }
+                        fence_proxy_async_smem();  // these reads before TMA writes the block again
                     }
+                    __syncwarp();
                     if (cj + 1 < CPH) issue_res(k0 + 64);
                 } else {
 #pragma unroll
@@ -1067,6 +1094,11 @@ std::string conv_tc_config_desc(const Layer &l, const Shape &in, sn_schema s, in
     return b;
 }
 
+int32_t conv_tc_ksplit(const Layer &l, const Shape &in, sn_schema s, int32_t v) {
+    const std::vector<tc::Config> cfgs = tc::configs(l, in, s);
+    return v >= 0 && v < (int)cfgs.size() ? cfgs[v].ksplit : 0;
+}
+
 size_t conv_tc_ws(const Layer &l, const Shape &in, sn_schema s, int32_t v, int32_t a_blocks) {
     const std::vector<tc::Config> cfgs = tc::configs(l, in, s, a_blocks);
     if (v < 0 || v >= (int)cfgs.size() || cfgs[v].ksplit == 1) return 0;
@@ -1102,6 +1134,15 @@ cudaError_t conv_tc(const LaunchArgs &a) {
     if (p.res && (uintptr_t)p.res % 16) return cudaErrorInvalidValue;  // read as 16-byte vectors
     p.err = device_error_word();
     p.wait_limit = a.wait_limit > 0 ? a.wait_limit : WAIT_LIMIT;
+    // a routine that writes the next layer's layout: the same dtype in NCHW
+    // (one CTA's epilogue per tile, so no K split through fp32 partials)
+    p.y_nchw = 0;
+    if (a.out_schema.dtype >= 0 && !schema_eq(a.out_schema, a.schema)) {
+        if (a.out_schema.dtype != a.schema.dtype || a.out_schema.layout != SN_NCHW || cf.ksplit != 1 ||
+            a.a_blocks > 0)
+            return cudaErrorInvalidValue;
+        p.y_nchw = 1;
+    }
     p.M = in.n * (int64_t)in.h * in.w;
     p.Mout = (int64_t)p.N * p.P * p.Q;
     p.ntiles = (p.K + cf.BN - 1) / cf.BN;
@@ -1412,6 +1453,7 @@ cudaError_t conv_im2col_tc_stage(const LaunchArgs &a, int stage) {
     LaunchArgs g = a;
     g.layer = &gl;
     g.routine = R_CONV_TC;
+    g.out_schema = g.schema;
     g.in_shapes = {Shape{l.out.n, kpad, l.out.h, l.out.w}};
     g.in[0] = a.ws;
     g.ws = static_cast<uint8_t *>(a.ws) + im2col_bytes(l, a.schema);
@@ -1531,6 +1573,7 @@ cudaError_t conv_s2d_tc_stage(const LaunchArgs &a, int stage) {
     LaunchArgs g = a;
     g.layer = &gl;
     g.routine = R_CONV_TC;
+    g.out_schema = g.schema;
     g.in_shapes = {gin};
     g.in[0] = a.ws;
     const int64_t pix = 16 * (int64_t)dtype_size(a.schema.dtype);  // 32 bytes: one X pixel
@@ -1565,6 +1608,7 @@ cudaError_t dense_tc(const LaunchArgs &a) {
     g.layer = &gl;
     g.routine = R_CONV_TC;
     g.schema = sn_schema{a.schema.dtype, SN_NHWC};
+    g.out_schema = g.schema;  // N x C x 1 x 1: the same bytes in either layout
     return conv_tc(g);
 }
 

@@ -249,11 +249,14 @@ int32_t kernels_per_launch(int32_t r, int32_t v, const Layer &l, const std::vect
 }
 
 std::vector<sn_schema> fused_outputs(int32_t r, const Layer &l, sn_schema s) {
+    // the tensor-core convolution can write its NHWC result straight in the
+    // NCHW layout of the same dtype (the permutation fused into its epilogue)
+    if (r == R_CONV_TC && l.type == SN_L_CONV2 && s.layout == SN_NHWC && (s.dtype == SN_F16 || s.dtype == SN_BF16))
+        return {{s.dtype, SN_NCHW}};
     // qint8 routines can leave their fp32 result in a float schema of the
     // same layout instead of requantising it (dequantisation fused into the
     // epilogue)
     if (s.dtype != SN_QI8) return {};
-    (void)l;
     switch (r) {
     case R_CONV_DIRECT:
     case R_CONV_DP4A:
@@ -265,6 +268,14 @@ std::vector<sn_schema> fused_outputs(int32_t r, const Layer &l, sn_schema s) {
     case R_DENSE: return {{SN_F16, s.layout}, {SN_BF16, s.layout}, {SN_F32, s.layout}};
     default: return {};
     }
+}
+
+bool fused_variant_ok(int32_t r, const Layer &l, const std::vector<Shape> &in, sn_schema s, int32_t v) {
+    if (s.dtype == SN_QI8) return true;
+    // the NCHW writer drains each tile in one CTA's epilogue: no K split
+    // through fp32 partials
+    if (r == R_CONV_TC && !in.empty()) return k::conv_tc_ksplit(l, in[0], s, v) == 1;
+    return false;
 }
 
 int32_t childnet_stages(int32_t r, sn_schema s) {

@@ -275,6 +275,8 @@ int32_t kernels_per_launch(int32_t routine, int32_t variant, const Layer &layer,
 // schemas other than `s` that the routine can write its output in, reading
 // its inputs in `s` (a fused boundary: dequantisation in a qint8 epilogue)
 std::vector<sn_schema> fused_outputs(int32_t routine, const Layer &layer, sn_schema s);
+// whether variant v of the routine can write those other schemas
+bool fused_variant_ok(int32_t routine, const Layer &layer, const std::vector<Shape> &in, sn_schema s, int32_t v);
 
 // selection (section IV)
 sn_status select_dprs(const Graph &g, std::vector<int32_t> &schema_of, int64_t &total);
@@ -333,6 +335,7 @@ int32_t conv_tc_variants(const Layer &l, const Shape &in, sn_schema s);
 size_t conv_tc_ws(const Layer &l, const Shape &in, sn_schema s, int32_t v, int32_t a_blocks = 0);  // K-split partials
 size_t dense_tc_ws(const Layer &l, const Shape &in, sn_schema s, int32_t v);
 const char *conv_tc_variant_name(int32_t v);
+int32_t conv_tc_ksplit(const Layer &l, const Shape &in, sn_schema s, int32_t v);  // K split of variant v
 std::string conv_tc_config_desc(const Layer &l, const Shape &in, sn_schema s, int32_t v, int32_t a_blocks = 0);
 // chained launches of consecutive tensor-core convolutions
 bool conv_tc_chain_shape(const Layer &l, const Shape &in, sn_schema s, int32_t v, bool *implicit, int *bn, int *kb,

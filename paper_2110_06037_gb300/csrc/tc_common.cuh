@@ -64,6 +64,7 @@ struct Params {
     float *part;                   // K split: fp32 partial sums [ksplit][Mout][K]
     int *err;                      // the library's device error word
     long long wait_limit;          // SM cycles a pipeline wait may take before the kernel gives up
+    int32_t y_nchw;                // 1: the output is written in NCHW (same dtype)
 };
 
 // ---------------------------------------------------------------- PTX helpers

@@ -92,7 +92,47 @@ def oracle_layer_cost(t):
     return lc
 
 
+def oracle_pair_cost(t):
+    """Per layer, the cheapest candidate of every (read, written) schema pair
+    (INF where none): the states of the pair problem."""
+    n, ns = t["n_layers"], t["n_schemas"]
+    pairs = [(r, w) for r in range(ns) for w in range(ns)]
+    lc = np.full((n, len(pairs)), INF, np.int64)
+    for c in range(len(t["cost"])):
+        k = int(t["schema"][c]) * ns + int(t["out_schema"][c])
+        lc[t["layer"][c], k] = min(lc[t["layer"][c], k], int(t["cost"][c]))
+    return lc, pairs
+
+
+def has_fused(t):
+    return bool((t["out_schema"] != t["schema"]).any())
+
+
+def realised_cost(t, cand):
+    """T of a choice of one candidate per layer: their times plus, on every
+    edge, the adapt from the producer's written schema to the consumer's read
+    schema (Def. 1, fused boundaries)."""
+    tot = sum(int(t["cost"][c]) for c in cand)
+    for e, (u, v) in enumerate(t["edges"].tolist()):
+        w, r = int(t["out_schema"][cand[u]]), int(t["schema"][cand[v]])
+        if w != r:
+            tot += int(t["adapt"][e][w][r])
+    return tot
+
+
 def check_against_oracle(g, t, exhaustive=True):
+    if has_fused(t):
+        # some routine writes another schema: the exact pair-state search
+        lcp, pairs = oracle_pair_cost(t)
+        ref, _ = blockwise_search(lcp, t["edges"], t["adapt"], pairs=pairs)
+        try:
+            tot, sch, cand = g.select_path(SN_SELECT_DPRS)
+        except SnError as e:
+            assert e.status == _sn.SN_EINFEASIBLE and ref == INF
+            return None
+        assert tot == ref, (tot, ref)
+        assert realised_cost(t, cand) == ref
+        return None
     lc = oracle_layer_cost(t)
     if exhaustive:
         ref, asg, nmin = oracle.brute_force(lc, t["edges"], t["adapt"])

@@ -174,3 +174,39 @@ def test_candidate_search_equals_schema_search_without_fused_candidates():
             # the chosen candidates, read as a schema assignment, cost the same
             assign = [cands[i][k][1] for i, k in enumerate(pick)]
             assert oracle.path_cost(lc, edges, a, assign) == ref
+
+
+def test_pair_blockwise_search_equals_candidate_search():
+    """The oracle's block-wise exact search over (read, written) pair states
+    (used on nets too large to enumerate) equals the exhaustive search over
+    one candidate per layer, on random nets with fused candidates."""
+    from oracle.paths import blockwise_search
+    from test_dprs import oracle_pair_cost
+    for seed in range(40):
+        rng = np.random.default_rng(9700 + seed)
+        layers = random_net(rng, int(rng.integers(1, 4)))
+        g = _graph(layers, 3 if seed % 2 else 2)
+        t = _random_costs(g, rng)
+        per = _cands_per_layer(t)
+        if np.prod([len(c) for c in per], dtype=float) > 2e5:
+            continue
+        ref, _ = brute_force_candidates(per, t["edges"].tolist(), t["adapt"])
+        lcp, pairs = oracle_pair_cost(t)
+        got, _ = blockwise_search(lcp, t["edges"], t["adapt"], pairs=pairs)
+        assert got == ref, seed
+
+
+def test_pair_blockwise_search_without_fused_states_is_the_plain_search():
+    from oracle.paths import blockwise_search
+    rng = np.random.default_rng(4)
+    for _ in range(20):
+        n, ns = int(rng.integers(3, 8)), 2
+        edges = [(i, i + 1) for i in range(n - 1)]
+        lc = rng.integers(1, 50, size=(n, ns)).astype(np.int64)
+        lc[0] = lc[-1] = 0
+        ac = rng.integers(0, 30, size=(len(edges), ns, ns)).astype(np.int64)
+        pairs = [(r, w) for r in range(ns) for w in range(ns)]
+        lcp = np.full((n, len(pairs)), INF, np.int64)
+        for r in range(ns):
+            lcp[:, r * ns + r] = lc[:, r]
+        assert blockwise_search(lcp, edges, ac, pairs=pairs)[0] == blockwise_search(lc, edges, ac)[0]

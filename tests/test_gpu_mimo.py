@@ -10,7 +10,8 @@ from oracle.net import run_net
 from paper_2110_06037_gb300 import SN_OPT_CUDA_GRAPH, SN_SELECT_BRUTE, SN_SELECT_DPRS, build_graph
 
 from gpu_helpers import TOL, from_device, maxrel, to_device
-from test_dprs import oracle_layer_cost
+from oracle.paths import blockwise_search
+from test_dprs import has_fused, oracle_layer_cost, oracle_pair_cost
 
 pytestmark = pytest.mark.gpu
 
@@ -46,8 +47,11 @@ def test_two_inputs_two_outputs_match_the_oracle():
     assert g.io_counts() == (2, 2)
     g.profile(warmup=1, iters=5, topk=2, passes=3)
     t = g.cost_table()
-    lc = oracle_layer_cost(t)
-    ref_cost, _, _ = oracle.brute_force(lc, t["edges"], t["adapt"])
+    if has_fused(t):  # a routine that writes another schema: the exact pair-state search
+        lcp, pairs = oracle_pair_cost(t)
+        ref_cost, _ = blockwise_search(lcp, t["edges"], t["adapt"], pairs=pairs)
+    else:
+        ref_cost, _, _ = oracle.brute_force(oracle_layer_cost(t), t["edges"], t["adapt"])
     tot, _, _ = g.select_path(SN_SELECT_DPRS)
     assert tot == ref_cost
     assert g.select_path(SN_SELECT_BRUTE)[0] == tot

@@ -22,7 +22,7 @@ from oracle.paths import blockwise_search
 from paper_2110_06037_gb300 import SN_OPT_CUDA_GRAPH, SN_SELECT_BRUTE, SN_SELECT_DPRS, build_graph, fuse_residual
 
 from gpu_helpers import TOL, from_device, maxrel, to_device
-from test_dprs import oracle_layer_cost
+from test_dprs import has_fused, oracle_layer_cost, oracle_pair_cost, realised_cost
 
 pytestmark = pytest.mark.gpu
 
@@ -31,11 +31,25 @@ F16 = [("f16", "nchw"), ("f16", "nhwc")]
 BF16 = [("bf16", "nchw"), ("bf16", "nhwc")]
 
 
+def _exact_pair_total(t):
+    """The exact optimum of the pair problem (some routine writes another
+    schema): the oracle's block-wise search over (read, written) states."""
+    lcp, pairs = oracle_pair_cost(t)
+    return blockwise_search(lcp, t["edges"], t["adapt"], pairs=pairs)[0]
+
+
 def _profile_select_run(layers, x, in_schema, out_schema, schemas, exhaustive, warmup=1, iters=5):
     import torch
     g = build_graph(layers, x.shape, in_schema, out_schema, schemas)
     g.profile(warmup=warmup, iters=iters, topk=2, passes=3)
     t = g.cost_table()
+    if has_fused(t):
+        total, sch, cand = g.select_path(SN_SELECT_DPRS)
+        assert total == _exact_pair_total(t)
+        assert realised_cost(t, cand) == total
+        y = g.run(to_device(x, in_schema))
+        torch.cuda.synchronize()
+        return g, from_device(y, out_schema)
     lc = oracle_layer_cost(t)
     if exhaustive:
         ref_total, ref_asg, nmin = oracle.brute_force(lc, t["edges"], t["adapt"])
@@ -143,8 +157,10 @@ def test_resnet50_b32_bf16_sampled():
     g = build_graph(layers, x.shape, ("bf16", "nchw"), ("bf16", "nchw"), BF16)
     g.profile(warmup=1, iters=3, topk=1, passes=2)
     t = g.cost_table()
-    lc = oracle_layer_cost(t)
-    ref_total, _ = blockwise_search(lc, t["edges"], t["adapt"])
+    if has_fused(t):
+        ref_total = _exact_pair_total(t)
+    else:
+        ref_total, _ = blockwise_search(oracle_layer_cost(t), t["edges"], t["adapt"])
     total, sch, _ = g.select_path(SN_SELECT_DPRS)
     assert total == ref_total
     y = g.run(to_device(x, ("bf16", "nchw")))
@@ -176,8 +192,10 @@ def test_fused_resnet50_b32_bf16_sampled():
     g = build_graph(fused, x.shape, ("bf16", "nchw"), ("bf16", "nchw"), BF16)
     g.profile(warmup=1, iters=3, topk=1, passes=2)
     t = g.cost_table()
-    lc = oracle_layer_cost(t)
-    ref_total, _ = blockwise_search(lc, t["edges"], t["adapt"])
+    if has_fused(t):
+        ref_total = _exact_pair_total(t)
+    else:
+        ref_total, _ = blockwise_search(oracle_layer_cost(t), t["edges"], t["adapt"])
     total, sch, _ = g.select_path(SN_SELECT_DPRS)
     assert total == ref_total
     y = g.run(to_device(x, ("bf16", "nchw")))
