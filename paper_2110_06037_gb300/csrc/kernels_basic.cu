@@ -670,6 +670,135 @@ __global__ void __launch_bounds__(256, 2) dw_nhwc_vec(const T *__restrict__ x, c
     }
 }
 
+// asynchronous 16-byte global -> shared copy, zero-filled when !valid
+__device__ __forceinline__ void cp_async16(void *smem, const void *gmem, bool valid) {
+    const uint32_t sa = (uint32_t)__cvta_generic_to_shared(smem);
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(sa), "l"(gmem), "r"(valid ? 16 : 0)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
+
+// 3x3 depthwise, NHWC, small maps (stride 1 or 2, padding 1): one CTA per
+// (image, 128-byte channel slice, band of PB output rows).  The band's input
+// rows -- every column of the slice, with the zero padding around -- are read
+// once, 16 bytes a thread and 128 bytes a pixel (coalesced), into shared
+// memory; each thread then keeps one channel vector's nine tap weights in
+// registers and produces that vector for output pixel after pixel from the
+// shared tile, writing 16-byte vectors.  Input bytes cross HBM once (plus the
+// two halo rows of a band), so the kernel needs no cross-thread reuse through
+// L1 and no per-thread windows.  The accumulation order is that of the other
+// NHWC kernels (bias, then rows inside the image, then columns), so the
+// results agree with them bit for bit.
+template <typename T, int SW>
+__global__ void __launch_bounds__(256, 4) dw3_nhwc_band(const T *__restrict__ x, const T *__restrict__ w,
+                                                     const float *__restrict__ bias, T *__restrict__ y, ConvDims d,
+                                                     int PB) {
+    griddep_launch();
+    griddep_wait();
+    constexpr int E = 16 / sizeof(T);  // elements per 16-byte vector
+    constexpr int VS = 8;              // vectors per 128-byte slice
+    extern __shared__ uint4 band_smem[];
+    const int slices = (d.C * (int)sizeof(T) + 127) / 128;
+    const int slice = (int)(blockIdx.x % slices), band = (int)(blockIdx.x / slices);
+    const int n = blockIdx.y;
+    const int p0 = band * PB, p1 = min(p0 + PB, d.P);
+    const int h0 = p0 * SW - 1;              // input row of band row 0 (padding 1)
+    const int rows = (p1 - p0 - 1) * SW + 3;
+    const int WP = d.W + 2;                  // band columns, padding included
+    const int nv = min(VS, (d.C * (int)sizeof(T) - slice * 128) / 16);  // vectors of this slice
+    const int cs = slice * (128 / (int)sizeof(T));
+    // asynchronous 16-byte copies (zero-filled outside the image and the
+    // slice): every load of the band is in flight at once, none holds a
+    // register
+    for (int i = threadIdx.x; i < rows * WP * VS; i += blockDim.x) {
+        const int v = i % VS, pix = i / VS, rr = pix / WP, cc = pix - rr * WP;
+        const int h = h0 + rr, ww = cc - 1;
+        const bool ok = v < nv && h >= 0 && h < d.H && ww >= 0 && ww < d.W;
+        const T *src = ok ? x + (((int64_t)n * d.H + h) * d.W + ww) * d.C + cs + v * E : x;
+        cp_async16(band_smem + i, src, ok);
+    }
+    cp_async_commit();
+    cp_async_wait<0>();
+    __syncthreads();
+    const int v = threadIdx.x % VS;
+    if (v >= nv) return;  // no barrier follows
+    const int c0 = cs + v * E;
+    uint4 wv[9];
+#pragma unroll
+    for (int k = 0; k < 9; ++k) wv[k] = *reinterpret_cast<const uint4 *>(w + (int64_t)k * d.C + c0);
+    float b[E];
+#pragma unroll
+    for (int e = 0; e < E; ++e) b[e] = bias[c0 + e];
+    for (int o = threadIdx.x / VS; o < (p1 - p0) * d.Q; o += blockDim.x / VS) {
+        const int pr = o / d.Q, q = o - pr * d.Q;
+        const int hb = (p0 + pr) * SW - 1;  // input row of tap row 0
+        uint4 out;
+        if constexpr (std::is_same<T, __half>::value) {
+            __half2 hacc[4];
+#pragma unroll
+            for (int k = 0; k < 4; ++k) hacc[k] = __floats2half2_rn(b[2 * k], b[2 * k + 1]);
+#pragma unroll
+            for (int r = 0; r < 3; ++r) {
+                if (hb + r < 0 || hb + r >= d.H) continue;
+                const uint4 *row = band_smem + ((pr * SW + r) * WP + q * SW) * VS + v;
+#pragma unroll
+                for (int s_ = 0; s_ < 3; ++s_) {
+                    const uint4 xv4 = row[s_ * VS];
+                    const __half2 *xv = reinterpret_cast<const __half2 *>(&xv4);
+                    const __half2 *wq = reinterpret_cast<const __half2 *>(&wv[r * 3 + s_]);
+#pragma unroll
+                    for (int k = 0; k < 4; ++k) hacc[k] = __hfma2(xv[k], wq[k], hacc[k]);
+                }
+            }
+            __half2 *oh = reinterpret_cast<__half2 *>(&out);
+            const __half2 z2 = __float2half2_rn(0.0f), six2 = __float2half2_rn(6.0f);
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                __half2 vv = hacc[k];
+                if (d.act == SN_ACT_RELU) {
+                    vv = __hmax2(vv, z2);
+                } else if (d.act == SN_ACT_RELU6) {
+                    vv = __hmin2(__hmax2(vv, z2), six2);
+                } else if (d.act != SN_ACT_NONE) {
+                    const float2 f = __half22float2(vv);
+                    vv = __floats2half2_rn(act_apply(f.x, d.act), act_apply(f.y, d.act));
+                }
+                oh[k] = vv;
+            }
+        } else {
+            float acc[E];
+#pragma unroll
+            for (int e = 0; e < E; ++e) acc[e] = b[e];
+#pragma unroll
+            for (int r = 0; r < 3; ++r) {
+                if (hb + r < 0 || hb + r >= d.H) continue;
+                const uint4 *row = band_smem + ((pr * SW + r) * WP + q * SW) * VS + v;
+#pragma unroll
+                for (int s_ = 0; s_ < 3; ++s_) fma16<T>(acc, row[s_ * VS], wv[r * 3 + s_]);
+            }
+            T *op = reinterpret_cast<T *>(&out);
+#pragma unroll
+            for (int e = 0; e < E; ++e) op[e] = cvt<T>(act_apply(acc[e], d.act));
+        }
+        *reinterpret_cast<uint4 *>(y + (((int64_t)n * d.P + p0 + pr) * d.Q + q) * d.C + c0) = out;
+    }
+}
+
+// band height and shared-memory bytes of dw3_nhwc_band for a layer (PB = 0:
+// the kernel does not apply: a 3-row band of the map would not fit)
+static int dw3_band_rows(const ConvDims &d, size_t *smem) {
+    const size_t row_bytes = (size_t)(d.W + 2) * 128;
+    const size_t budget = d.W <= 64 ? 32768 : 49152;
+    const int max_rows = (int)(budget / row_bytes);
+    if (max_rows < 3) return 0;
+    int PB = (max_rows - 3) / d.sh + 1;
+    if (PB > d.P) PB = d.P;
+    *smem = (size_t)((PB - 1) * d.sh + 3) * row_bytes;
+    return PB;
+}
+
 // NCHW: one thread per (n, c, p) and 8 consecutive output columns; consecutive
 // threads take consecutive column blocks, so every load and store is
 // coalesced across the warp; weights are [C][R][S].
@@ -735,14 +864,6 @@ __global__ void __launch_bounds__(256) dw_nchw_row(const T *__restrict__ x, cons
 constexpr int DW_TP = 8;
 template <int SW> struct DwTQ { static constexpr int v = SW == 1 ? 16 : 8; };  // output columns per unit
 
-__device__ __forceinline__ void cp_async16(void *smem, const void *gmem, bool valid) {
-    const uint32_t sa = (uint32_t)__cvta_generic_to_shared(smem);
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(sa), "l"(gmem), "r"(valid ? 16 : 0)
-                 : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
 
 template <typename T, int SW, int STAGES>
 __global__ void __launch_bounds__(256, 2) dw3_nhwc_halo(const T *__restrict__ x, const T *__restrict__ w,
@@ -881,6 +1002,18 @@ __global__ void __launch_bounds__(256) dw3_nchw_tile(const T *__restrict__ x, co
     }
 }
 
+bool dw3_band_applies(const Layer &l, const Shape &in, sn_schema s) {
+    const sn_conv_params &c = l.conv;
+    if (s.dtype == SN_QI8 || s.layout != SN_NHWC || c.kh != 3 || c.kw != 3 || c.dh != 1 || c.dw != 1 ||
+        c.ph != 1 || c.pw != 1 || c.sh != c.sw || (c.sh != 1 && c.sh != 2) || (in.c * dtype_size(s.dtype)) % 16 ||
+        in.n > 65535)
+        return false;
+    const ConvDims d{(int32_t)in.n, (int32_t)in.c, (int32_t)in.h, (int32_t)in.w, c.c_out, (int32_t)l.out.h,
+                     (int32_t)l.out.w, 3, 3, c.sh, c.sw, 1, 1, 1, 1, c.groups, c.act};
+    size_t smem = 0;
+    return dw3_band_rows(d, &smem) > 0;
+}
+
 cudaError_t dwconv(const LaunchArgs &a) {
     // routine parameter (variant): NHWC 0 = register window (4 columns per
     // thread), 1 = input rows staged by TMA in a shared-memory ring (3x3,
@@ -900,7 +1033,21 @@ cudaError_t dwconv(const LaunchArgs &a) {
         const T *x = (const T *)a.in[0];
         const T *w = (const T *)a.wt;
         T *y = (T *)a.out;
-        if (a.schema.layout == SN_NHWC && vec_ok) {
+        const bool band_ok = k3 && d.dh == 1 && d.ph == 1 && d.pw == 1 && d.sh == d.sw && (d.sh == 1 || d.sh == 2);
+        size_t band_smem = 0;
+        const int PB = band_ok && a.schema.layout == SN_NHWC && vec_ok ? dw3_band_rows(d, &band_smem) : 0;
+        if (a.variant == 2 && PB > 0 && d.N <= 65535) {
+            const int slices = (int)((d.C * (int64_t)es + 127) / 128);
+            const dim3 gb((unsigned)(slices * ((d.P + PB - 1) / PB)), (unsigned)d.N);
+            static bool attr = false;
+            if (!attr) {
+                cudaFuncSetAttribute(dw3_nhwc_band<T, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, 49152);
+                cudaFuncSetAttribute(dw3_nhwc_band<T, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, 49152);
+                attr = true;
+            }
+            if (d.sh == 1) launch_pdl(dw3_nhwc_band<T, 1>, gb, 256, band_smem, a.stream, x, w, a.bias, y, d, PB);
+            else launch_pdl(dw3_nhwc_band<T, 2>, gb, 256, band_smem, a.stream, x, w, a.bias, y, d, PB);
+        } else if (a.schema.layout == SN_NHWC && vec_ok) {
             const int64_t cvec = d.C * es / 16;
             const bool halo = k3 && d.dh == 1 && (d.sw == 1 || d.sw == 2) && d.sh == d.sw;
             if (a.variant == 1 && halo) {

@@ -38,7 +38,7 @@ const char *variant_name(int32_t r, int32_t v) {
     switch (r) {
     case R_CONV_IGEMM: return v == 0 ? "tile=64x64" : "tile=128x64";
     case R_CONV_WINO: return v == 0 ? "gemm=simt" : "gemm=tc";
-    case R_DW_DIRECT: return v == 0 ? "nhwc:window|nchw:rows" : "nhwc:tma_rows|nchw:plane_tile";
+    case R_DW_DIRECT: return v == 0 ? "nhwc:window|nchw:rows" : v == 1 ? "nhwc:tma_rows|nchw:plane_tile" : "nhwc:band";
     case R_CONV_TC:
     case R_CONV_IM2COL_TC:
     case R_CONV_S2D_TC:
@@ -103,7 +103,9 @@ int32_t routine_variants(int32_t r, const Layer &l, const std::vector<Shape> &in
     case R_CONV_TC:
         return is_conv(l) ? k::conv_tc_variants(l, in[0], s) : 0;
     case R_DW_DIRECT:
-        return l.type == SN_L_DWCONV2 ? 2 : 0;
+        if (l.type != SN_L_DWCONV2) return 0;
+        // NHWC 3x3 of small maps: a third parameter, the shared-memory band kernel
+        return (s.layout == SN_NHWC && k::dw3_band_applies(l, in[0], s)) ? 3 : 2;
     case R_MAXPOOL:
         return l.type == SN_L_MAXPOOL ? 1 : 0;
     case R_GAP:

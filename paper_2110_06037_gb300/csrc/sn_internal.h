@@ -356,6 +356,7 @@ size_t conv_s2d_tc_ws(const Layer &l, const Shape &in, sn_schema s, int32_t v);
 cudaError_t conv_s2d_tc(const LaunchArgs &a);
 cudaError_t dense_tc(const LaunchArgs &a);
 cudaError_t dwconv(const LaunchArgs &a);
+bool dw3_band_applies(const Layer &l, const Shape &in, sn_schema s);  // NHWC small-map depthwise kernel
 cudaError_t maxpool(const LaunchArgs &a);
 cudaError_t gap(const LaunchArgs &a);
 cudaError_t add(const LaunchArgs &a);

@@ -105,16 +105,25 @@ def test_depthwise(case, schema):
     layer["weight"] = (rng.standard_normal((C, 1, 3, 3)) * np.sqrt(2 / 9)).astype(np.float32)
     layer["bias"] = (rng.standard_normal(C) * 0.1).astype(np.float32)
     ref = ref_one(layer, x, schema[0])
-    outs = []
-    for v in (0, 1):  # routine parameters: register window / rows in shared memory (NHWC), row / plane tile (NCHW)
+    outs = {}
+    # routine parameters: register window / rows in shared memory / (small maps)
+    # band tiles in shared memory (NHWC); row / plane tile (NCHW)
+    variants = (0, 1, 2) if schema[1] == "nhwc" else (0, 1)
+    for v in variants:
         got = run_one(layer, x, schema, "dwconv2/direct", v)
+        if got is None:  # the band kernel does not apply to this map (a 3-row band would not fit)
+            assert v == 2 and W > 110
+            continue
         assert maxrel(got, ref) <= TOL[schema[0]], v
-        outs.append(got)
-    if schema[1] == "nhwc" and schema[0] != "f32":
-        # both NHWC kernels accumulate the nine taps in the same order (bias,
+        outs[v] = got
+    if schema[1] == "nhwc":
+        # the NHWC kernels accumulate the nine taps in the same order (bias,
         # then rows, then columns): in f32 with exact products for bf16, in
-        # packed half2 for f16: equal results
-        assert np.array_equal(outs[0], outs[1])
+        # packed half2 for f16: equal results (the f32 ring fallback differs)
+        if schema[0] != "f32":
+            assert np.array_equal(outs[0], outs[1])
+        if 2 in outs:
+            assert np.array_equal(outs[0], outs[2])
 
 
 @pytest.mark.parametrize("schema", SCHEMAS)
