@@ -307,13 +307,14 @@ sn_status sn_set_option(sn_graph *gg, int32_t option, int64_t value) {
 }
 
 static sn_status check_device(Graph *g, cudaStream_t st) {
-    (void)g;
     SN_CUDA_TRY(cudaStreamSynchronize(st));
     int word = 0;
     SN_CUDA_TRY(cudaMemcpy(&word, k::device_error_word(), sizeof(int), cudaMemcpyDeviceToHost));
     if (word) {
         const int zero = 0;
         cudaMemcpy(k::device_error_word(), &zero, sizeof(int), cudaMemcpyHostToDevice);
+        // a stopped stream-K launch may have left tile counts behind
+        if (g->tile_counts.ptr) cudaMemset(g->tile_counts.ptr, 0, g->tile_counts.bytes);
         return fail(SN_ETIMEOUT, "device error word set: " + std::to_string(word) +
                                      " (a bounded wait in a kernel gave up)");
     }

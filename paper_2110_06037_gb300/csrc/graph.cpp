@@ -40,6 +40,7 @@ Graph::~Graph() {
     for (auto &kv : weight_cache) dev_free(this, &kv.second);
     for (auto &kv : bias_cache) dev_free(this, &kv.second);
     dev_free(this, &workspace);
+    dev_free(this, &tile_counts);
     dev_free(this, &arena);
     dev_free(this, &host_in);
     dev_free(this, &host_out);

@@ -275,8 +275,8 @@ std::vector<sn_schema> fused_outputs(int32_t r, const Layer &l, sn_schema s) {
 bool fused_variant_ok(int32_t r, const Layer &l, const std::vector<Shape> &in, sn_schema s, int32_t v) {
     if (s.dtype == SN_QI8) return true;
     // the NCHW writer drains each tile in one CTA's epilogue: no K split
-    // through fp32 partials
-    if (r == R_CONV_TC && !in.empty()) return k::conv_tc_ksplit(l, in[0], s, v) == 1;
+    // through fp32 partials, no stream-K parts
+    if (r == R_CONV_TC && !in.empty()) return k::conv_tc_nchw_ok(l, in[0], s, v);
     return false;
 }
 

@@ -48,6 +48,17 @@ static bool chain_eligible(const Graph *g, const PlanOp &op);
 // launch run at once, so what they touch is live across the whole chain.
 // Placement: largest blob first, at the lowest offset (256-byte aligned) free
 // of every placed blob it is live with.
+// The zeroed counters of the stream-K tensor-core routines (one per tile and
+// epilogue warp; every launch leaves them zeroed): allocated once per graph.
+sn_status ensure_tile_counts(Graph *g, cudaStream_t st) {
+    if (g->tile_counts.ptr) return SN_OK;
+    sn_status rc = dev_alloc(g, kTileCounts * sizeof(int), &g->tile_counts);
+    if (rc != SN_OK) return rc;
+    if (cudaMemsetAsync(g->tile_counts.ptr, 0, g->tile_counts.bytes, st) != cudaSuccess)
+        return fail(SN_ECUDA, "stream-K counters: memset failed");
+    return SN_OK;
+}
+
 static sn_status place_slots(Graph *g) {
     const size_t ns = g->slots.size();
     std::vector<int32_t> first(ns, INT32_MAX), last(ns, -1);
@@ -228,6 +239,10 @@ sn_status build_plan(Graph *g, cudaStream_t st) {
         sn_status rc = dev_alloc(g, ws, &g->workspace);
         if (rc != SN_OK) return rc;
     }
+    {
+        sn_status rc = ensure_tile_counts(g, st);
+        if (rc != SN_OK) return rc;
+    }
     if (g->opt_chain && !g->profiling) {
         sn_status rc = build_chains(g, st);
         if (rc != SN_OK) return rc;
@@ -363,6 +378,8 @@ static sn_status launch_op(Graph *g, const PlanOp &op, const IoPtrs &io, cudaStr
     a.ws = g->workspace.ptr;
     a.ws_bytes = g->workspace.bytes;
     a.wait_limit = g->opt_wait_limit;
+    a.tile_counts = static_cast<int *>(g->tile_counts.ptr);
+    a.tile_counts_n = (int64_t)(g->tile_counts.bytes / sizeof(int));
     a.stream = st;
     return launch_routine(a);
 }
@@ -546,7 +563,7 @@ static sn_status profile_graph_on(Graph *g, const sn_profile_opts &o, cudaStream
         dev_free(g, &sc.out);
     };
     if ((rc = ensure(g, sc.in0, max_bytes)) != SN_OK || (rc = ensure(g, sc.in1, max_bytes)) != SN_OK ||
-        (rc = ensure(g, sc.out, max_bytes)) != SN_OK) {
+        (rc = ensure(g, sc.out, max_bytes)) != SN_OK || (rc = ensure_tile_counts(g, st)) != SN_OK) {
         cleanup();
         return rc;
     }
@@ -597,6 +614,8 @@ static sn_status profile_graph_on(Graph *g, const sn_profile_opts &o, cudaStream
             }
             a.ws = g->workspace.ptr;
             a.ws_bytes = g->workspace.bytes;
+            a.tile_counts = static_cast<int *>(g->tile_counts.ptr);
+            a.tile_counts_n = (int64_t)(g->tile_counts.bytes / sizeof(int));
             int64_t t = kInf;
             const int32_t nst = childnet_stages(cd.routine, s);
             if (nst == 1) {

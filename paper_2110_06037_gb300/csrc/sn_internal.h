@@ -168,6 +168,10 @@ struct LaunchArgs {
     // tensor-core routines: SM cycles a pipeline wait may take before the
     // kernel gives up and reports SN_ETIMEOUT (0 = the library default)
     int64_t wait_limit = 0;
+    // tensor-core stream-K routines: the graph's zeroed counter array (the
+    // kernels leave it zeroed) and its length in ints
+    int *tile_counts = nullptr;
+    int64_t tile_counts_n = 0;
     cudaStream_t stream = nullptr;
 };
 
@@ -208,6 +212,7 @@ struct Graph {
     std::map<std::string, Buffer> weight_cache;  // key: layer/format/dtype
     std::map<int32_t, Buffer> bias_cache;        // per layer fp32 bias
     Buffer workspace;
+    Buffer tile_counts;               // kTileCounts zeroed ints for the stream-K tensor-core routines
     Buffer arena;                     // the plan's activation buffers, placed by liveness
     size_t arena_unshared = 0;        // what the activation buffers would take one allocation each
     Buffer host_in, host_out;         // device staging of sn_run_host
@@ -247,6 +252,9 @@ struct IoPtrs {
     std::vector<void *> out;
 };
 sn_status dev_alloc(Graph *g, size_t bytes, Buffer *b);
+// stream-K counters: one int per (tile, epilogue warp), 1024 tiles of 8 warps
+constexpr int64_t kTileCounts = 8192;
+sn_status ensure_tile_counts(Graph *g, cudaStream_t st);
 void dev_free(Graph *g, Buffer *b);
 void invalidate_plan(Graph *g);
 
@@ -335,7 +343,7 @@ int32_t conv_tc_variants(const Layer &l, const Shape &in, sn_schema s);
 size_t conv_tc_ws(const Layer &l, const Shape &in, sn_schema s, int32_t v, int32_t a_blocks = 0);  // K-split partials
 size_t dense_tc_ws(const Layer &l, const Shape &in, sn_schema s, int32_t v);
 const char *conv_tc_variant_name(int32_t v);
-int32_t conv_tc_ksplit(const Layer &l, const Shape &in, sn_schema s, int32_t v);  // K split of variant v
+bool conv_tc_nchw_ok(const Layer &l, const Shape &in, sn_schema s, int32_t v);  // variant v can write NCHW
 std::string conv_tc_config_desc(const Layer &l, const Shape &in, sn_schema s, int32_t v, int32_t a_blocks = 0);
 // chained launches of consecutive tensor-core convolutions
 bool conv_tc_chain_shape(const Layer &l, const Shape &in, sn_schema s, int32_t v, bool *implicit, int *bn, int *kb,

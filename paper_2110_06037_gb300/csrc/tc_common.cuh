@@ -65,6 +65,11 @@ struct Params {
     int *err;                      // the library's device error word
     long long wait_limit;          // SM cycles a pipeline wait may take before the kernel gives up
     int32_t y_nchw;                // 1: the output is written in NCHW (same dtype)
+    // stream-K (one-CTA tiles): the tiles' K steps laid end to end, sk_steps =
+    // mtiles * ntiles * kiters in all, CTA c taking [c sk_len, (c + 1) sk_len)
+    int32_t sk_len, sk_steps;      // 0: off
+    int *sk_count;                 // per (tile, epilogue warp): parts arrived; zero between launches
+    float *sk_part;                // fp32 partial tiles, two slots of 128 x BN per CTA
 };
 
 // ---------------------------------------------------------------- PTX helpers
@@ -405,6 +410,10 @@ struct Work {
     int q0, p0, i0;  // implicit mode: box origin (q, p, image)
     int sp, it0, it1;
     int mt;          // pixel tile index (>= mtiles: the idle half of a CTA pair)
+    // stream-K: the tile, its number of parts (CTAs that take some of its K
+    // steps; 1 = this CTA takes all), the first of those CTAs, and this
+    // CTA's partial slot for it (0 when the tile is the first of the CTA's range)
+    int sk_t, sk_n, sk_c0, sk_slot;
 };
 
 // work unit u: K-split part sp of output-channel tile nt of pixel-tile group
@@ -418,6 +427,7 @@ __device__ __forceinline__ Work work_of(const Params &p, int u, int bn, bool imp
     const int mg = (int)fdiv((uint32_t)t, p.fd_ntiles), nt = t - mg * p.ntiles;
     const int mt = mg * ctas + rank;
     w.mt = mt;
+    w.sk_t = t, w.sk_n = 1, w.sk_c0 = 0, w.sk_slot = 0;
     w.n0 = nt * bn;
     w.m0 = 0;
     w.q0 = w.p0 = w.i0 = 0;
