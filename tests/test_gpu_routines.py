@@ -201,10 +201,12 @@ def test_conv_hard_activations(act, schema):
     assert ran >= 2
 
 
-# planes of 196 (8-byte bf16 rows, 16-byte f32 rows), 49 (element-wide rows)
-# and 130 channels (ragged tiles on both axes, element-wide channel rows)
+# planes of 196 (8-byte bf16 rows, 16-byte f32 rows), 49 (element-wide rows),
+# 81 and 60 (ragged tiles per image) and 130 channels (ragged tiles on both
+# axes, element-wide channel rows)
 CONVERT_SHAPES = [(2, 5, 7, 9), (1, 64, 56, 56), (3, 130, 1, 1), (1, 3, 65, 67), (2, 24, 14, 14),
-                  (2, 40, 7, 7), (2, 130, 14, 14), (1, 1024, 14, 14)]
+                  (2, 40, 7, 7), (2, 130, 14, 14), (1, 1024, 14, 14), (5, 64, 9, 9), (4, 256, 14, 14),
+                  (3, 72, 10, 6)]
 
 
 @pytest.mark.parametrize("shape", CONVERT_SHAPES)
