@@ -70,6 +70,7 @@ struct Config {
     int ms = 1;        // 128-row halves per one-CTA tile (2: 256 x BN, one A box, B shared)
     int csk = 1;       // 2: a cluster of two CTAs splits each tile's K steps, reducing on chip
     int sk = 0;        // 1: stream-K, one equal range of the tiles' K steps per SM
+    int halo = 0;      // 1: 3x3 stride 1, 8 x 16 pixel tiles, one A box per row of taps
 };
 
 constexpr int kSmCount = 152;  // GB300; only used to decide which K splits to offer
@@ -231,6 +232,21 @@ static std::vector<Config> configs(const Layer &l, const Shape &in, sn_schema s,
     if (a_blocks == 0) {
         for (const Geo &gg : geos(2 * BM)) push_ms2({true, 0, gg.bw, gg.bh, gg.bni, 1, 1, 1}, tiles_of(gg));
         for (const Geo &gg : geos(BM)) push_sk({true, 0, gg.bw, gg.bh, gg.bni, 1, 1, 1}, tiles_of(gg));
+        // halo tiles for 3x3 stride-1 layers (appended last, like stream-K):
+        // one CTA per tile (BN <= 128), and CTA pairs that share B
+        if (c.kh == 3 && c.kw == 3 && c.sh == 1 && c.dh == 1 && c.dw == 1) {
+            for (int bn : bns)
+                if (bn <= 128) {
+                    Config cf{true, bn, HALO_BW, HALO_BH, 1, 1, 1, 1};
+                    cf.halo = 1;
+                    out.push_back(cf);
+                }
+            for (int bn : bns) {
+                Config cf{true, bn, HALO_BW, HALO_BH, 1, 1, 2, 1};
+                cf.halo = 1;
+                out.push_back(cf);
+            }
+        }
     }
     return out;
 }
@@ -280,7 +296,8 @@ std::string conv_tc_config_desc(const Layer &l, const Shape &in, sn_schema s, in
     char b[160];
     if (c.implicit)
         snprintf(b, sizeof(b), "bn=%d cta=%d kb=%d rows=%d ksplit=%d bst=%d csk=%d%s tile=%dx%dx%d", c.BN, c.G,
-                 c.KB, 128 * c.ms * c.G, c.ksplit, c.bst ? 1 : 0, c.csk, c.sk ? " streamk" : "", c.BW, c.BH, c.BNI);
+                 c.KB, 128 * c.ms * c.G, c.ksplit, c.bst ? 1 : 0, c.csk,
+                 c.sk ? " streamk" : c.halo ? " halo" : "", c.BW, c.BH, c.BNI);
     else
         snprintf(b, sizeof(b), "bn=%d cta=%d kb=%d rows=%d ksplit=%d bst=%d csk=%d%s plain", c.BN, c.G, c.KB,
                  128 * c.ms * c.G, c.ksplit, c.bst ? 1 : 0, c.csk, c.sk ? " streamk" : "");
@@ -365,7 +382,25 @@ cudaError_t conv_tc(const LaunchArgs &a) {
     // one box lands KB consecutive 128-B-row blocks in shared memory
     const bool blk = cf.KB > 1;
     const uint64_t CB = (uint64_t)p.cblocks;
-    {  // B: weights [K][R*S][C]
+    if (cf.halo) {
+        // halo tiles: a K step is one row of three taps of one channel block
+        if (p.R != 3 || p.S != 3 || p.stride != 1 || p.dh != 1 || p.dw != 1 || cf.KB != 1 || cf.ms != 1)
+            return cudaErrorInvalidValue;
+        p.kiters = p.R * p.cblocks;
+        {  // B: weights [K][R*S][C] read as [R*S][K][C], one box = a row's three taps x BN x 64
+            const uint64_t dims[3] = {(uint64_t)p.C, (uint64_t)p.K, (uint64_t)(p.R * p.S)};
+            const uint64_t str[2] = {(uint64_t)p.R * p.S * p.C * es, p.C * es};
+            const uint32_t box[3] = {BK, (uint32_t)(cf.BN / cf.G), 3};  // a CTA's share of the BN rows
+            if (!encode(&mB, dt, 3, a.wt, dims, str, box)) return cudaErrorInvalidValue;
+        }
+        {  // A: [N][H][W][C], one box = 16 rows x 10 columns of one image
+            const uint64_t dims[4] = {(uint64_t)p.C, (uint64_t)p.W, (uint64_t)p.H, (uint64_t)p.N};
+            const uint64_t str[3] = {p.C * es, (uint64_t)p.W * p.C * es, (uint64_t)p.H * p.W * p.C * es};
+            const uint32_t box[4] = {BK, (uint32_t)HALO_W, (uint32_t)HALO_BH, 1};
+            if (!encode(&mA[0], dt, 4, a.in[0], dims, str, box)) return cudaErrorInvalidValue;
+            mA[1] = mA[2] = mA[3] = mA[0];
+        }
+    } else {  // B: weights [K][R*S][C]
         const uint64_t dims[4] = {blk ? 64 : (uint64_t)p.C, (uint64_t)(p.R * p.S), (uint64_t)p.K, CB};
         const uint64_t str[3] = {p.C * es, (uint64_t)p.R * p.S * p.C * es, 128};
         const uint32_t box[4] = {BK, 1, (uint32_t)(cf.BN / cf.G), (uint32_t)cf.KB};  // a CTA's share of the BN rows
@@ -393,7 +428,9 @@ cudaError_t conv_tc(const LaunchArgs &a) {
         const int tn = (p.N + cf.BNI - 1) / cf.BNI;
         const uint32_t box[5] = {BK, (uint32_t)cf.BW, (uint32_t)cf.BH, (uint32_t)cf.BNI, (uint32_t)cf.KB};
         const uint64_t c0dim = blk ? 64 : (uint64_t)p.C;
-        if (p.stride == 1) {
+        if (cf.halo) {
+            // A was encoded above (one box per row of taps)
+        } else if (p.stride == 1) {
             const uint64_t dims[5] = {c0dim, (uint64_t)p.W, (uint64_t)p.H, (uint64_t)p.N, CB};
             uint64_t str[4] = {p.C * es, (uint64_t)p.W * p.C * es, (uint64_t)p.H * p.W * p.C * es, 128};
             if (a.a_strides[0] > 0)  // a caller-laid-out A (overlapping pixel rows)
@@ -441,7 +478,7 @@ cudaError_t conv_tc(const LaunchArgs &a) {
     p.fd_tq = make_fastdiv((uint32_t)std::max(p.tq, 1));
     p.fd_tp = make_fastdiv((uint32_t)std::max(p.tp, 1));
     p.fd_spt = make_fastdiv((uint32_t)(p.cblocks / cf.KB));
-    p.fd_S = make_fastdiv((uint32_t)p.S);
+    p.fd_S = make_fastdiv((uint32_t)(cf.halo ? 1 : p.S));  // halo: a K step's "tap" is a row of taps
     p.lbw = p.lbwh = 0;
     if (cf.implicit) {
         while ((1 << p.lbw) < cf.BW) ++p.lbw;
@@ -452,6 +489,7 @@ cudaError_t conv_tc(const LaunchArgs &a) {
     return cf.implicit ? launch<TT, BNV, true, GV, KBV>(mA, mB, mY, mR, p, a.stream)               \
                        : launch<TT, BNV, false, GV, KBV>(mA, mB, mY, mR, p, a.stream)
 #define SN_TC_LAUNCH_T(TT)                                                                          \
+    if (cf.halo) return launch_halo(dt, cf.BN, cf.G, mA, mB, mY, mR, p, a.stream);                 \
     if (cf.sk) {                                                                                    \
         if (cf.G != 1 || cf.ms != 1 || cf.bst || cf.ksplit != 1 || cf.csk != 1) return cudaErrorInvalidValue; \
         return launch_sk(dt, cf.BN, cf.KB, cf.implicit, mA, mB, mY, mR, p, a.stream);              \

@@ -36,6 +36,12 @@ constexpr int stages_for(int bn, int g, int kb, int ms = 1, int extra = 0) {
                ? (198656 - extra) / (kb * (16384 * ms + bn / g * 128))
                : 8;
 }
+// halo tiles (3x3, stride 1): 8 x 16 output pixels of one image; a stage
+// holds the 10 x 16 input pixels one tap row reads (all three column taps)
+constexpr int HALO_BW = 8, HALO_BH = 16, HALO_W = HALO_BW + 2, HALO_ROWS = HALO_W * HALO_BH;
+constexpr int halo_stages(int bn) {
+    return 198656 / (HALO_ROWS * 128 + 3 * bn * 128) < 8 ? 198656 / (HALO_ROWS * 128 + 3 * bn * 128) : 8;
+}
 // weight-stationary tiles: the layer's whole B (K steps x BN rows x 128 B) is
 // loaded once per CTA and stays in shared memory beside this many A stages
 constexpr int BST_STAGES = 4;
@@ -332,6 +338,20 @@ __device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr) {
     d |= (uint64_t)(1024 >> 4) << 32;
     d |= (uint64_t)1 << 46;  // descriptor version for tcgen05
     d |= (uint64_t)2 << 61;  // 128-byte swizzle
+    return d;
+}
+
+// the same with 8-row groups sbo bytes apart (a multiple of 128 B): the
+// 128-byte swizzle is a function of the absolute shared-memory address, so a
+// matrix may start at any row of a box TMA wrote and step by any whole number
+// of rows per group
+__device__ __forceinline__ uint64_t sdesc_sw128_sbo(uint32_t saddr, uint32_t sbo) {
+    uint64_t d = 0;
+    d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
+    d |= (uint64_t)1 << 16;
+    d |= (uint64_t)((sbo >> 4) & 0x3FFFu) << 32;
+    d |= (uint64_t)1 << 46;
+    d |= (uint64_t)2 << 61;
     return d;
 }
 

@@ -59,7 +59,15 @@ namespace tc {
 // tile's counter (one per epilogue warp) sums the parts in CTA order and
 // finishes the tile (bias, residual, activation, store).  No CTA waits for
 // another, so the split needs no co-residency.
-template <typename T, int BN, int STAGES, bool IMPLICIT, int G, int KB, bool BST, int MS, int CSK, bool SK>
+// HALO (3x3, stride 1, one-CTA tiles of 8 x 16 output pixels of one image):
+// a K step is one tap row r of one 64-channel block; its stage holds A = the
+// 10 x 16 input pixels the row's three column taps read, as one TMA box, and
+// B = the three taps' weight rows.  Tap s reads A from box row s on, with
+// 8-row groups 10 rows apart (the swizzle follows the absolute address, so
+// any row offset and group stride work): one A box per three taps instead of
+// three, and 10/8 of the rows instead of three times them.
+template <typename T, int BN, int STAGES, bool IMPLICIT, int G, int KB, bool BST, int MS, int CSK, bool SK,
+          bool HALO>
 __global__ void __launch_bounds__(THREADS, 1)
     conv_tc_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ CUtensorMap mA1,
                    const __grid_constant__ CUtensorMap mA2, const __grid_constant__ CUtensorMap mA3,
@@ -69,9 +77,10 @@ __global__ void __launch_bounds__(THREADS, 1)
     // 128 rows x 128 B, of B (BN / G) rows x 128 B (this CTA's share)
     // MS = 2: a one-CTA tile of 256 rows, one TMA box of A for both 128-row
     // halves and two MMAs (one per half, one TMEM accumulator each) sharing B
-    constexpr uint32_t A_SUB = BM * BK * 2;  // one 128-row half
+    constexpr uint32_t A_SUB = HALO ? HALO_ROWS * BK * 2 : BM * BK * 2;  // one 128-row half (or the halo box)
     constexpr uint32_t A_BLK = MS * A_SUB;
-    constexpr uint32_t B_BLK = (BN / G) * BK * 2;
+    constexpr uint32_t B_TAP = (BN / G) * BK * 2;          // one tap's weight rows
+    constexpr uint32_t B_BLK = B_TAP * (HALO ? 3 : 1);
     constexpr uint32_t A_BYTES = KB * A_BLK;
     constexpr uint32_t B_BYTES = KB * B_BLK;
     // BST (weight-stationary, G = 1, one N tile, no K split): a stage holds A
@@ -233,7 +242,9 @@ __global__ void __launch_bounds__(THREADS, 1)
             // thread's issue loop is slower than the MMAs of a stage.  The
             // tap / channel-block position advances incrementally for every
             // K step, with no division per step.
-            const int cblocks = p.cblocks, S = p.S, dh = p.dh, dw = p.dw, ph0 = p.ph, pw0 = p.pw;
+            // (halo tiles: a "tap" is a row of three taps, and the box starts
+            // at the row's first column tap)
+            const int cblocks = p.cblocks, S = HALO ? 1 : p.S, dh = p.dh, dw = p.dw, ph0 = p.ph, pw0 = p.pw;
             const int brow = (int)rank * (BN / G);
             int g = 0, s = prod, issued = 0;
             uint32_t par = 0;
@@ -298,7 +309,9 @@ __global__ void __launch_bounds__(THREADS, 1)
                             else
                                 tma_3d<G>(sa, &mA0, bar, 0, (int)w.m0, cb);
                         }
-                        if (!BST) {  // weight-stationary B is already resident
+                        if (HALO) {  // the three taps of row `tap`: map [C][K][R*S], box 64 x BN x 3
+                            tma_3d<G>(sa + A_BYTES, &mB, bar, c0, w.n0 + brow, tap * 3);
+                        } else if (!BST) {  // weight-stationary B is already resident
                             if (KB == 1)
                                 tma_3d<G>(sa + A_BYTES, &mB, bar, c0, tap, w.n0 + brow);
                             else
@@ -326,8 +339,10 @@ __global__ void __launch_bounds__(THREADS, 1)
     } else if (warp == 1 && WAITER) {
         if (leader) {  // ---------------- MMA issuer (lane 0; the whole warp meets the waiter)
             const uint32_t idesc = idesc_f16<T>(BM * G, BN);
-            const uint64_t desc0 = sdesc_sw128(su32(smem));  // stage 0, A; offsets add to the address field
+            // stage 0, A; offsets add to the address field (halo: 8-row groups one box row apart)
+            const uint64_t desc0 = HALO ? sdesc_sw128_sbo(su32(smem), HALO_W * 128u) : sdesc_sw128(su32(smem));
             const uint64_t descb = sdesc_sw128(su32(bst));   // weight-stationary B, K step 0
+            const uint64_t deschb = sdesc_sw128(su32(smem) + A_BYTES);  // halo: stage 0, B
             int g = 0, lt = 0, s = 0;
             bool stop = false;
             if (BST && lane == 0 && !mbar_wait(&bst_bar, 0u, p.wait_limit)) {
@@ -350,17 +365,29 @@ __global__ void __launch_bounds__(THREADS, 1)
                     if (lane == 0) {
                         // descriptors of this stage; a K step of 16 is 32 bytes (2 units)
                         const uint64_t da = desc0 + (uint64_t)((s * STAGE_BYTES) >> 4);
-                        const uint64_t db =
-                            BST ? descb + (uint64_t)(((uint32_t)it * B_BYTES) >> 4) : da + (A_BYTES >> 4);
+                        if constexpr (HALO) {
+                            // tap s_ of the row: A from box row s_ on (128 B = 8 units), B its own rows
+                            const uint64_t db = deschb + (uint64_t)((s * STAGE_BYTES) >> 4);
 #pragma unroll
-                        for (int j = 0; j < KB; ++j)
+                            for (int s_ = 0; s_ < 3; ++s_)
 #pragma unroll
-                            for (int k = 0; k < BK / 16; ++k)
+                                for (int k = 0; k < BK / 16; ++k)
+                                    umma<G>(d, da + 8 * s_ + 2 * k, db + s_ * (B_TAP >> 4) + 2 * k, idesc,
+                                            (it > w.it0 || s_ > 0 || k > 0) ? 1u : 0u);
+                        } else {
+                            const uint64_t db =
+                                BST ? descb + (uint64_t)(((uint32_t)it * B_BYTES) >> 4) : da + (A_BYTES >> 4);
 #pragma unroll
-                                for (int m = 0; m < MS; ++m)
-                                    umma<G>(d + (uint32_t)(m * BN), da + j * (A_BLK >> 4) + m * (A_SUB >> 4) + 2 * k,
-                                            db + j * (B_BLK >> 4) + 2 * k, idesc,
-                                            (it > w.it0 || j > 0 || k > 0) ? 1u : 0u);
+                            for (int j = 0; j < KB; ++j)
+#pragma unroll
+                                for (int k = 0; k < BK / 16; ++k)
+#pragma unroll
+                                    for (int m = 0; m < MS; ++m)
+                                        umma<G>(d + (uint32_t)(m * BN),
+                                                da + j * (A_BLK >> 4) + m * (A_SUB >> 4) + 2 * k,
+                                                db + j * (B_BLK >> 4) + 2 * k, idesc,
+                                                (it > w.it0 || j > 0 || k > 0) ? 1u : 0u);
+                        }
                         umma_commit<G>(&empty_bar[s]);  // frees the stage (in both CTAs) once read
                     }
                     __syncwarp();
@@ -374,8 +401,10 @@ __global__ void __launch_bounds__(THREADS, 1)
     } else if (warp == 1) {
         if (lane == 0 && leader) {  // ---------------- MMA issuer (the pair's leader)
             const uint32_t idesc = idesc_f16<T>(BM * G, BN);
-            const uint64_t desc0 = sdesc_sw128(su32(smem));  // stage 0, A; offsets add to the address field
+            // stage 0, A; offsets add to the address field (halo: 8-row groups one box row apart)
+            const uint64_t desc0 = HALO ? sdesc_sw128_sbo(su32(smem), HALO_W * 128u) : sdesc_sw128(su32(smem));
             const uint64_t descb = sdesc_sw128(su32(bst));   // weight-stationary B, K step 0
+            const uint64_t deschb = sdesc_sw128(su32(smem) + A_BYTES);  // halo: stage 0, B
             int g = 0, lt = 0, s = 0;
             uint32_t par = 0;
             bool stop = false;
@@ -406,16 +435,27 @@ __global__ void __launch_bounds__(THREADS, 1)
                     tc_fence_after();
                     // descriptors of this stage; a K step of 16 is 32 bytes (2 units)
                     const uint64_t da = desc0 + (uint64_t)((s * STAGE_BYTES) >> 4);
-                    const uint64_t db = BST ? descb + (uint64_t)(((uint32_t)it * B_BYTES) >> 4) : da + (A_BYTES >> 4);
+                    if constexpr (HALO) {
+                        const uint64_t db = deschb + (uint64_t)((s * STAGE_BYTES) >> 4);
 #pragma unroll
-                    for (int j = 0; j < KB; ++j)
+                        for (int s_ = 0; s_ < 3; ++s_)
 #pragma unroll
-                        for (int k = 0; k < BK / 16; ++k)
+                            for (int k = 0; k < BK / 16; ++k)
+                                umma<G>(d, da + 8 * s_ + 2 * k, db + s_ * (B_TAP >> 4) + 2 * k, idesc,
+                                        (it > w.it0 || s_ > 0 || k > 0) ? 1u : 0u);
+                    } else {
+                        const uint64_t db =
+                            BST ? descb + (uint64_t)(((uint32_t)it * B_BYTES) >> 4) : da + (A_BYTES >> 4);
 #pragma unroll
-                            for (int m = 0; m < MS; ++m)
-                                umma<G>(d + (uint32_t)(m * BN), da + j * (A_BLK >> 4) + m * (A_SUB >> 4) + 2 * k,
-                                        db + j * (B_BLK >> 4) + 2 * k, idesc,
-                                        (it > w.it0 || j > 0 || k > 0) ? 1u : 0u);
+                        for (int j = 0; j < KB; ++j)
+#pragma unroll
+                            for (int k = 0; k < BK / 16; ++k)
+#pragma unroll
+                                for (int m = 0; m < MS; ++m)
+                                    umma<G>(d + (uint32_t)(m * BN), da + j * (A_BLK >> 4) + m * (A_SUB >> 4) + 2 * k,
+                                            db + j * (B_BLK >> 4) + 2 * k, idesc,
+                                            (it > w.it0 || j > 0 || k > 0) ? 1u : 0u);
+                    }
                     umma_commit<G>(&empty_bar[s]);  // frees the stage (in both CTAs) once read
                     if (++s == STAGES) {
                         s = 0;
@@ -916,27 +956,29 @@ __global__ void splitk_reduce_kernel(const float *__restrict__ part, const float
 }
 
 template <typename T, int BN, bool IMPLICIT, int G, int KB, bool BST = false, int MS = 1, int CSK = 1,
-          bool SK = false>
+          bool SK = false, bool HALO = false>
 static cudaError_t launch(const CUtensorMap *mA, const CUtensorMap &mB, const CUtensorMap &mY, const CUtensorMap &mR,
                           const Params &p,
                           cudaStream_t st) {
-    constexpr int STAGES = BST ? BST_STAGES : stages_for(BN, G, KB, MS);
+    constexpr int STAGES = BST ? BST_STAGES : HALO ? halo_stages(BN / G) : stages_for(BN, G, KB, MS);
+    // bytes of one pipeline stage (A and this CTA's share of B), as the kernel lays them out
+    constexpr size_t STAGE = HALO ? (size_t)HALO_ROWS * BK * 2 + 3 * (size_t)(BN / G) * BK * 2
+                                  : (size_t)KB * (MS * BM * BK * 2 + (BN / G) * BK * 2);
     static_assert(CSK == 1 || (size_t)STAGES * KB * (BM * BK * 2 + BN * BK * 2) >= EPI_WARPS * XBLK_BYTES,
                   "cluster K split: the exchange blocks live in the stage memory");
     constexpr size_t smem_max = 227 * 1024;
     const size_t smem = BST ? (size_t)STAGES * BM * BK * 2 + p.bst_bytes + EPI_WARPS * STG_BYTES + 1024
-                            : (size_t)STAGES * KB * (MS * BM * BK * 2 + (BN / G) * BK * 2) + EPI_WARPS * STG_BYTES + 1024;
-    static_assert(BST ||
-                      (size_t)STAGES * KB * (MS * BM * BK * 2 + (BN / G) * BK * 2) + EPI_WARPS * STG_BYTES + 1024 <=
-                          smem_max,
-                  "shared memory per CTA");
+                            : (size_t)STAGES * STAGE + EPI_WARPS * STG_BYTES + 1024;
+    static_assert(BST || (size_t)STAGES * STAGE + EPI_WARPS * STG_BYTES + 1024 <= smem_max, "shared memory per CTA");
+    static_assert(!HALO || (IMPLICIT && KB == 1 && MS == 1 && !BST && CSK == 1 && !SK),
+                  "halo tiles: implicit tiles of one CTA or a pair, one channel block per stage");
     static_assert(!BST || (G == 1 && KB == 1 && MS == 1), "weight-stationary tiles are one-CTA, one block per stage");
     static_assert(MS == 1 || (G == 1 && KB == 1 && !BST && 2 * MS * BN <= 512), "two-half tiles: one CTA, TMEM");
     static_assert(CSK == 1 || (G == 1 && MS == 1 && !BST && BN >= 128), "cluster K split: one-CTA tiles of >= 2 chunks");
     static_assert(!SK || (G == 1 && MS == 1 && !BST && CSK == 1 && BN >= 128), "stream-K: one-CTA tiles of >= 2 chunks");
     static_assert(STAGES >= 2, "pipeline depth");
     if (smem > smem_max) return cudaErrorInvalidValue;
-    auto kern = conv_tc_kernel<T, BN, STAGES, IMPLICIT, G, KB, BST, MS, CSK, SK>;
+    auto kern = conv_tc_kernel<T, BN, STAGES, IMPLICIT, G, KB, BST, MS, CSK, SK, HALO>;
     constexpr bool CLUSTER = G == 2 || CSK == 2;
     static int max_groups = 0;  // co-resident CTAs (G = 1) or clusters of two (pairs, K split)
     cudaLaunchConfig_t cfg = {};
@@ -994,6 +1036,11 @@ static cudaError_t launch(const CUtensorMap *mA, const CUtensorMap &mB, const CU
                                                                p.ksplit, p.act);
     return cudaGetLastError();
 }
+
+// halo launches (kernels_tc_halo.cu): 3x3 stride-1 tiles of 8 x 16 pixels per
+// CTA; one CTA (g = 1, bn in {64, 128}) or a pair sharing B (g = 2, bn in {64, 128, 256})
+cudaError_t launch_halo(int dtype, int bn, int g, const CUtensorMap *mA, const CUtensorMap &mB,
+                        const CUtensorMap &mY, const CUtensorMap &mR, const Params &p, cudaStream_t st);
 
 // stream-K launches (kernels_tc_sk.cu): one-CTA tiles of bn in {128, 256}
 // output channels, kb channel blocks per stage
