@@ -252,6 +252,9 @@ def main():
                     help="r50_b32 is the benchmark line; the others print one extra JSON line each")
     ap.add_argument("--layer", default="32,512,56,512,3,1",
                     help="--config layer: N,C,H,K,k,s of one bf16 NHWC conv (C -> K channels, HxH input)")
+    ap.add_argument("--plan", default="",
+                    help="tuned-state file (cost table + path): loaded if it exists, else written after tuning, "
+                         "so that a profiler run times the same path as a plain run")
     ap.add_argument("--variant", type=int, default=-1,
                     help="--config layer: conv2/igemm_tc routine parameter index (-1: every one)")
     args = ap.parse_args()
@@ -285,8 +288,14 @@ def main():
         # the library's residual-add fusion pass runs before tuning
         g = sn.build_graph(layers0, x.shape, ("bf16", "nchw"), ("bf16", "nchw"), sch, fuse=True)
         layers = sn.fused_description(layers0, g.fused_ids)
-        g.profile(warmup=3, iters=10, topk=2, passes=3)
+        plan_loaded = bool(args.plan) and os.path.exists(args.plan)
+        if plan_loaded:  # the saved cost table; DPRS on it gives the saved path again
+            g.load_plan(args.plan)
+        else:
+            g.profile(warmup=3, iters=10, topk=2, passes=3)
         total, schemas, cands = g.select_path(sn.SN_SELECT_DPRS)
+        if args.plan and not plan_loaded:
+            g.save_plan(args.plan)
     stream.synchronize()
     tune_s = time.perf_counter() - t_tune0
 
@@ -489,6 +498,7 @@ def main():
                            "timing": "CUDA events around each step on the launching stream, CUDA-graph replay"},
                 "e2e": e2e, "gpu_launches": n_kern * args.steps, "roofline": roof, "cpu_baseline": cpu,
                 "clocks": clk, "tuning_s": tune_s, "path_cost_ns": total,
+                "plan": ("loaded from " + os.path.basename(args.plan)) if plan_loaded else "tuned in this run",
                 "r50_b1_fp16_latency": b1,
                 "activation_memory": {"arena_bytes": arena_b, "unshared_bytes": unshared_b},
                 "per_routine_ms": {k: round(v["ms"], 4) for k, v in per_routine.items()},
