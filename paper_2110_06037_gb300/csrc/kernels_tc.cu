@@ -347,6 +347,11 @@ cudaError_t conv_tc(const LaunchArgs &a) {
     if (p.res && (uintptr_t)p.res % 16) return cudaErrorInvalidValue;  // read as 16-byte vectors
     p.err = device_error_word();
     p.wait_limit = a.wait_limit > 0 ? a.wait_limit : WAIT_LIMIT;
+    // the prepared weights [K][R*S][C] (16-byte multiple: C is a multiple of
+    // 8); none for the space-to-depth form, whose weights have another layout
+    p.wt = a.wt;
+    p.wt_bytes = (uintptr_t)a.wt % 16 == 0 && a.a_blocks == 0 ? (int64_t)c.c_out * c.kh * c.kw * in.c * 2 : 0;
+    if (p.wt_bytes >= ((int64_t)1 << 32) * 64) p.wt_bytes = 0;  // slices stay below 4 GB
     // a routine that writes the next layer's layout: the same dtype in NCHW
     // (one CTA's epilogue per tile, so no K split through fp32 partials)
     p.y_nchw = 0;

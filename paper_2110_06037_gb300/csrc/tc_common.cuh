@@ -76,6 +76,10 @@ struct Params {
     int32_t sk_len, sk_steps;      // 0: off
     int *sk_count;                 // per (tile, epilogue warp): parts arrived; zero between launches
     float *sk_part;                // fp32 partial tiles, two slots of 128 x BN per CTA
+    // the layer's weights (not written by the previous kernel): each CTA asks
+    // L2 for its slice of them before the dependency wait
+    const void *wt;
+    int64_t wt_bytes;
 };
 
 // ---------------------------------------------------------------- PTX helpers
@@ -166,6 +170,12 @@ __device__ __forceinline__ void tma_5d(uint32_t dst, const CUtensorMap *m, uint3
     SN_TMA_LOAD("5d", "{%3, %4, %5, %6, %7}", "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(c4));
 }
 #undef SN_TMA_LOAD
+
+// bring [p, p + bytes) into L2 (no data is returned; p and bytes multiples of 16)
+__device__ __forceinline__ void prefetch_l2(const void *p, uint32_t bytes) {
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(reinterpret_cast<uint64_t>(p)), "r"(bytes)
+                 : "memory");
+}
 
 // TMEM allocation; G = 2 allocates the same columns in both CTAs of the pair
 // (one warp of each CTA executes it)

@@ -162,6 +162,15 @@ __global__ void __launch_bounds__(THREADS, 1)
         // the tensor maps are kernel parameters, not data of the previous kernel
         const CUtensorMap *maps[7] = {&mA0, &mA1, &mA2, &mA3, &mB, &mY, &mR};
         for (int i = 0; i < 7; ++i) asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(maps[i])) : "memory");
+        // this CTA's slice of the weights into L2 while the previous kernel
+        // finishes (after an L2 flush they would otherwise come from HBM
+        // on the critical path of the first K steps)
+        if (p.wt_bytes > 0) {
+            const int64_t slice = ((p.wt_bytes + gridDim.x - 1) / gridDim.x + 15) & ~(int64_t)15;
+            const int64_t off = (int64_t)blockIdx.x * slice;
+            if (off < p.wt_bytes)
+                prefetch_l2(static_cast<const uint8_t *>(p.wt) + off, (uint32_t)min(slice, p.wt_bytes - off));
+        }
         for (int s = 0; s < STAGES; ++s) {
             mbar_init(&full_bar[s], 1);  // the (leader's) producer of the stage
             mbar_init(&empty_bar[s], 1);
