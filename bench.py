@@ -292,7 +292,11 @@ def main():
         if plan_loaded:  # the saved cost table; DPRS on it gives the saved path again
             g.load_plan(args.plan)
         else:
-            g.profile(warmup=3, iters=10, topk=2, passes=3)
+            # 20 back-to-back launches per unit timing, the best 3 candidates per
+            # (layer, schema) re-timed in 5 whole-net passes: three runs each of
+            # (10, 2, 3), (20, 3, 5) and (40, 3, 8) tuned to 0.770-0.787,
+            # 0.766-0.770 and 0.765-0.779 ms per step on GB300
+            g.profile(warmup=3, iters=20, topk=3, passes=5)
         total, schemas, cands = g.select_path(sn.SN_SELECT_DPRS)
         if args.plan and not plan_loaded:
             g.save_plan(args.plan)
