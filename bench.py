@@ -124,7 +124,7 @@ def tc_sources_digest():
     """sha256 over the tensor-core conv kernel sources: a DRAM-traffic figure
     measured with ncu is reported only while these are unchanged."""
     h = hashlib.sha256()
-    for f in ("tc_conv.cuh", "kernels_tc.cu", "kernels_tc_sk.cu", "tc_common.cuh"):
+    for f in ("tc_conv.cuh", "kernels_tc.cu", "kernels_tc_sk.cu", "kernels_tc_halo.cu", "tc_common.cuh"):
         with open(os.path.join(ROOT, "paper_2110_06037_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()
