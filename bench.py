@@ -344,10 +344,12 @@ def main():
     value = ws * args.batch / (ms / 1e3)
 
     # ---------------- e2e through the C ABI with host buffers ----------------
-    # Every step is one sn_run_host call: the library copies the batch from
-    # pinned host memory into its device staging buffer, runs the net and
-    # copies the logits back to pinned host memory, all on the stream, so the
-    # timed region holds each step's host->device and device->host copies.
+    # Every step is one sn_run_host call: the library uploads the batch from
+    # pinned host memory (on its own copy stream, into one of two landing
+    # buffers, so that the upload overlaps the previous step's net), runs the
+    # net and copies the logits back to pinned host memory, in order on the
+    # stream, so the timed region holds each step's host->device and
+    # device->host copies.
     xh = torch.from_numpy(x).to(torch.bfloat16).pin_memory()
     oh = torch.empty(out.shape, dtype=out.dtype).pin_memory()
     with torch.cuda.stream(stream):
@@ -365,7 +367,8 @@ def main():
     e2e = {"value": args.batch / (e2e_ms / 1e3), "unit": "images/s",
            "h2d_bytes_per_step": xh.numel() * xh.element_size(),
            "d2h_bytes_per_step": oh.numel() * oh.element_size(),
-           "path": "sn_run_host (C ABI): copies from and to pinned host memory inside each call, in stream order"}
+           "path": "sn_run_host (C ABI): copies from and to pinned host memory inside each call; the upload of "
+                   "one call overlaps the net of the previous one (library copy stream, two landing buffers)"}
 
     # ---------------- per-op shares of the step ----------------
     # One replay of the step with a timing node around every op gives each

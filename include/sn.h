@@ -305,12 +305,16 @@ SN_API sn_status sn_run(sn_graph *g, const void *in_dev, void *out_dev, void *st
 /* sn_run from and to host memory: the input is copied from in_host (host
  * memory holding the input in in_schema, the full tensor) into a device
  * buffer the graph owns, the net runs, and the output is copied back to
- * out_host (out_schema, the full tensor), all asynchronously on `stream`:
- * read out_host only after synchronising the stream.  Page-locked host
+ * out_host (out_schema, the full tensor), all asynchronously and in order
+ * on `stream`: read out_host only after synchronising the stream.  The
+ * upload itself runs on a stream the graph owns, into one of two device
+ * landing buffers used in turn, so that the upload of one call overlaps the
+ * net of the call before it; `stream` waits for it.  Page-locked host
  * buffers (cudaHostAlloc / cudaHostRegister) make the copies asynchronous;
  * pageable ones work but the copies then synchronise with the host.  Both
- * host buffers are the caller's and must stay valid until the stream has
- * passed this call.  Nets with one input and one output only.
+ * host buffers are the caller's and must stay valid (in_host unchanged)
+ * until the stream has passed this call.  Nets with one input and one
+ * output only.
  * Errors: as sn_run, plus SN_EINVAL for a net with several inputs or
  * outputs and SN_ENOMEM when the device staging buffers cannot be made. */
 SN_API sn_status sn_run_host(sn_graph *g, const void *in_host, void *out_host, void *stream);

@@ -399,7 +399,34 @@ sn_status sn_run_host(sn_graph *gg, const void *in_host, void *out_host, void *s
             if ((rc = dev_alloc(g, out_bytes, &g->host_out)) != SN_OK) return rc;
         }
         cudaStream_t st = static_cast<cudaStream_t>(stream);
-        SN_CUDA_TRY(cudaMemcpyAsync(g->host_in.ptr, in_host, in_bytes, cudaMemcpyHostToDevice, st));
+        // the upload runs on the graph's copy stream into one of two landing
+        // buffers (alternating per call), after the call two before this one
+        // has copied that buffer out; the caller's stream waits for it and
+        // copies it into the net's input buffer (the captured CUDA graph keeps
+        // one input address).  So the upload of one call overlaps the net of
+        // the previous one, and everything stays in order on `stream`.
+        if (!g->copy_stream) {
+            SN_CUDA_TRY(cudaStreamCreateWithFlags(&g->copy_stream, cudaStreamNonBlocking));
+            for (int i = 0; i < 2; ++i) {
+                SN_CUDA_TRY(cudaEventCreateWithFlags(&g->land_done[i], cudaEventDisableTiming));
+                SN_CUDA_TRY(cudaEventCreateWithFlags(&g->land_free[i], cudaEventDisableTiming));
+            }
+        }
+        const int b = g->land_next;
+        if (g->host_land[b].bytes < in_bytes) {
+            if (g->land_used[b]) SN_CUDA_TRY(cudaEventSynchronize(g->land_free[b]));
+            dev_free(g, &g->host_land[b]);
+            g->land_used[b] = false;
+            if ((rc = dev_alloc(g, in_bytes, &g->host_land[b])) != SN_OK) return rc;
+        }
+        if (g->land_used[b]) SN_CUDA_TRY(cudaStreamWaitEvent(g->copy_stream, g->land_free[b], 0));
+        SN_CUDA_TRY(cudaMemcpyAsync(g->host_land[b].ptr, in_host, in_bytes, cudaMemcpyHostToDevice, g->copy_stream));
+        SN_CUDA_TRY(cudaEventRecord(g->land_done[b], g->copy_stream));
+        SN_CUDA_TRY(cudaStreamWaitEvent(st, g->land_done[b], 0));
+        SN_CUDA_TRY(cudaMemcpyAsync(g->host_in.ptr, g->host_land[b].ptr, in_bytes, cudaMemcpyDeviceToDevice, st));
+        SN_CUDA_TRY(cudaEventRecord(g->land_free[b], st));
+        g->land_used[b] = true;
+        g->land_next = b ^ 1;
         IoPtrs io;
         io.in = {g->host_in.ptr};
         io.out = {g->host_out.ptr};

@@ -42,6 +42,13 @@ Graph::~Graph() {
     dev_free(this, &workspace);
     dev_free(this, &tile_counts);
     dev_free(this, &arena);
+    if (copy_stream) cudaStreamSynchronize(copy_stream);  // no upload still writes a landing buffer
+    for (int b = 0; b < 2; ++b) {
+        dev_free(this, &host_land[b]);
+        if (land_done[b]) cudaEventDestroy(land_done[b]);
+        if (land_free[b]) cudaEventDestroy(land_free[b]);
+    }
+    if (copy_stream) cudaStreamDestroy(copy_stream);
     dev_free(this, &host_in);
     dev_free(this, &host_out);
 }

@@ -216,6 +216,15 @@ struct Graph {
     Buffer arena;                     // the plan's activation buffers, placed by liveness
     size_t arena_unshared = 0;        // what the activation buffers would take one allocation each
     Buffer host_in, host_out;         // device staging of sn_run_host
+    // sn_run_host's input upload: two landing buffers filled on the graph's
+    // own copy stream (so that a call's upload overlaps the previous call's
+    // net), each copied into host_in on the caller's stream
+    Buffer host_land[2];
+    cudaStream_t copy_stream = nullptr;
+    cudaEvent_t land_done[2] = {nullptr, nullptr};  // upload into landing buffer b finished
+    cudaEvent_t land_free[2] = {nullptr, nullptr};  // landing buffer b copied out (may be refilled)
+    bool land_used[2] = {false, false};
+    int land_next = 0;
     int opt_graph = 0, opt_check = 0;
     int64_t opt_wait_limit = 0;       // SN_OPT_WAIT_LIMIT (0 = default)
     int opt_share = 1;                // SN_OPT_SHARE_BUFFERS: place activations by liveness

@@ -231,6 +231,34 @@ def test_run_host_copies_inside_the_call():
             assert torch.equal(oh, ref.cpu()), (graph, pinned)
 
 
+def test_run_host_back_to_back_calls_keep_their_inputs():
+    """Consecutive sn_run_host calls without a synchronisation in between,
+    each on its own pinned input and output: the uploads go through two
+    landing buffers used in turn on the graph's copy stream, so a call's
+    upload overlaps the previous call's net; every output must still be the
+    one of its own input (same bits as sn_run on that input)."""
+    import torch
+    x, layers = synth.resnet50(2, res=64)
+    g = build_graph(layers, x.shape, ("bf16", "nchw"), ("bf16", "nchw"), BF16, fuse=True)
+    g.profile(warmup=1, iters=2, topk=1, passes=1)
+    g.select_path(SN_SELECT_DPRS)
+    rng = np.random.default_rng(3)
+    xs = [to_device((x * rng.uniform(0.5, 1.5)).astype(np.float32), ("bf16", "nchw")) for _ in range(5)]
+    refs = [g.run(xd).clone() for xd in xs]
+    torch.cuda.synchronize()
+    s = torch.cuda.Stream()
+    for graph in (0, 1):
+        g.set_option(SN_OPT_CUDA_GRAPH, graph)
+        xh = [xd.cpu().pin_memory() for xd in xs]
+        oh = [torch.empty(refs[0].shape, dtype=refs[0].dtype).pin_memory() for _ in xs]
+        for _ in range(2):
+            for i in range(len(xs)):
+                g.run_host(xh[i], oh[i], stream=s)
+        s.synchronize()
+        for i in range(len(xs)):
+            assert torch.equal(oh[i], refs[i].cpu()), (graph, i)
+
+
 @pytest.mark.parametrize("chain", [0, 1])
 def test_liveness_arena_same_bits_less_memory(chain):
     """Activations placed by liveness in one arena give the same bits as one
