@@ -356,8 +356,7 @@ cudaError_t conv_tc(const LaunchArgs &a) {
     // (one CTA's epilogue per tile, so no K split through fp32 partials)
     p.y_nchw = 0;
     if (a.out_schema.dtype >= 0 && !schema_eq(a.out_schema, a.schema)) {
-        if (a.out_schema.dtype != a.schema.dtype || a.out_schema.layout != SN_NCHW || cf.ksplit != 1 || cf.sk ||
-            a.a_blocks > 0)
+        if (a.out_schema.dtype != a.schema.dtype || a.out_schema.layout != SN_NCHW || cf.ksplit != 1 || cf.sk)
             return cudaErrorInvalidValue;
         p.y_nchw = 1;
     }
@@ -748,7 +747,7 @@ static bool s2d_applies(const Layer &l, sn_schema s) {
     const sn_conv_params &c = l.conv;
     return l.type == SN_L_CONV2 && c.groups == 1 && c.sh == 2 && c.sw == 2 && c.dh == 1 && c.dw == 1 &&
            4 * c.c_in <= 16 && c.kh >= 3 && c.kh <= 8 && c.kw <= 8 && c.c_out % 8 == 0 && s.dtype != SN_F32 &&
-           s.layout == SN_NHWC;
+           s.dtype != SN_QI8;  // input in either layout (the re-layout reads both)
 }
 
 // rows of taps A = ceil(kh/2) rounded up to 2 or 4 (zero weights beyond kh);
@@ -774,17 +773,19 @@ static size_t s2d_bytes(const Layer &l, sn_schema s) {
 
 int32_t conv_s2d_tc_variants(const Layer &l, const Shape &in, sn_schema s) {
     (void)in;
-    if (!s2d_applies(l, s)) return 0;
-    return (int32_t)tc::configs(s2d_gemm_layer(l), s2d_gemm_in(l), s, s2d_rows(l)).size();
+    if (!s2d_applies(l, s)) return 0;  // the GEMM on X is NHWC-like whatever the input layout
+    return (int32_t)tc::configs(s2d_gemm_layer(l), s2d_gemm_in(l), sn_schema{s.dtype, SN_NHWC}, s2d_rows(l)).size();
 }
 
 size_t conv_s2d_tc_ws(const Layer &l, const Shape &in, sn_schema s, int32_t v) {
     (void)in;
-    return s2d_bytes(l, s) + conv_tc_ws(s2d_gemm_layer(l), s2d_gemm_in(l), s, v, s2d_rows(l));
+    return s2d_bytes(l, s) + conv_tc_ws(s2d_gemm_layer(l), s2d_gemm_in(l), sn_schema{s.dtype, SN_NHWC}, v, s2d_rows(l));
 }
 
-// X[n][u][v][16]: one thread per X pixel, two 16-byte stores
-template <typename T>
+// X[n][u][v][16]: one thread per X pixel, two 16-byte stores; the input is
+// NHWC, or NCHW (NCHW_IN: the layout change fused into the re-layout, so an
+// NCHW net input needs no separate adapt)
+template <typename T, bool NCHW_IN>
 __global__ void __launch_bounds__(256) s2d_kernel(const T *__restrict__ x, T *__restrict__ X, S2dDims d) {
     griddep_launch();
     griddep_wait();
@@ -798,8 +799,13 @@ __global__ void __launch_bounds__(256) s2d_kernel(const T *__restrict__ x, T *__
         for (int ij = 0; ij < 4; ++ij) {
             const int h = 2 * u + (ij >> 1) - d.ph, w = 2 * v + (ij & 1) - d.pw;
             if (h < 0 || h >= d.H || w < 0 || w >= d.W) continue;
-            const T *xp = x + ((n * d.H + h) * d.W + w) * d.C;
-            for (int c = 0; c < d.C; ++c) po[ij * d.C + c] = xp[c];
+            if (NCHW_IN) {
+                const T *xp = x + (n * d.C * d.H + h) * d.W + w;
+                for (int c = 0; c < d.C; ++c) po[ij * d.C + c] = xp[(int64_t)c * d.H * d.W];
+            } else {
+                const T *xp = x + ((n * d.H + h) * d.W + w) * d.C;
+                for (int c = 0; c < d.C; ++c) po[ij * d.C + c] = xp[c];
+            }
         }
         uint4 *dst = reinterpret_cast<uint4 *>(X + t * 16);
         dst[0] = o[0];
@@ -821,9 +827,15 @@ cudaError_t conv_s2d_tc_stage(const LaunchArgs &a, int stage) {
     if (!a.ws || a.ws_bytes < xb || (uintptr_t)a.ws % 256) return cudaErrorInvalidValue;
     const int64_t total = (int64_t)d.N * d.Pp * d.Qp;
     if (stage != 1) {
-        SN_DT_SWITCH(a.schema.dtype, T,
-                     launch_pdl(s2d_kernel<T>, grid_for(total, 256), 256, 0, a.stream, (const T *)a.in[0], (T *)a.ws,
-                                d));
+        if (a.schema.layout == SN_NCHW) {
+            SN_DT_SWITCH(a.schema.dtype, T,
+                         launch_pdl(s2d_kernel<T, true>, grid_for(total, 256), 256, 0, a.stream, (const T *)a.in[0],
+                                    (T *)a.ws, d));
+        } else {
+            SN_DT_SWITCH(a.schema.dtype, T,
+                         launch_pdl(s2d_kernel<T, false>, grid_for(total, 256), 256, 0, a.stream, (const T *)a.in[0],
+                                    (T *)a.ws, d));
+        }
         cudaError_t e = cudaGetLastError();
         if (e != cudaSuccess || stage == 0) return e;
     }
@@ -831,7 +843,10 @@ cudaError_t conv_s2d_tc_stage(const LaunchArgs &a, int stage) {
     LaunchArgs g = a;
     g.layer = &gl;
     g.routine = R_CONV_TC;
-    g.out_schema = g.schema;
+    // the GEMM reads X (its own layout) and writes the output in the
+    // candidate's written schema: NHWC, or NCHW through the NCHW epilogue
+    g.schema = sn_schema{a.schema.dtype, SN_NHWC};
+    g.out_schema = a.out_schema.dtype >= 0 ? a.out_schema : a.schema;
     g.in_shapes = {gin};
     g.in[0] = a.ws;
     const int64_t pix = 16 * (int64_t)dtype_size(a.schema.dtype);  // 32 bytes: one X pixel

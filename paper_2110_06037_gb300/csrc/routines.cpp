@@ -255,6 +255,10 @@ std::vector<sn_schema> fused_outputs(int32_t r, const Layer &l, sn_schema s) {
     // NCHW layout of the same dtype (the permutation fused into its epilogue)
     if (r == R_CONV_TC && l.type == SN_L_CONV2 && s.layout == SN_NHWC && (s.dtype == SN_F16 || s.dtype == SN_BF16))
         return {{s.dtype, SN_NCHW}};
+    // the space-to-depth stem reads either layout and its GEMM writes either
+    // (NHWC from its TMA store, NCHW from the NCHW epilogue)
+    if (r == R_CONV_S2D_TC && l.type == SN_L_CONV2 && (s.dtype == SN_F16 || s.dtype == SN_BF16))
+        return {{s.dtype, s.layout == SN_NHWC ? SN_NCHW : SN_NHWC}};
     // qint8 routines can leave their fp32 result in a float schema of the
     // same layout instead of requantising it (dequantisation fused into the
     // epilogue)
@@ -277,6 +281,7 @@ bool fused_variant_ok(int32_t r, const Layer &l, const std::vector<Shape> &in, s
     // the NCHW writer drains each tile in one CTA's epilogue: no K split
     // through fp32 partials, no stream-K parts
     if (r == R_CONV_TC && !in.empty()) return k::conv_tc_nchw_ok(l, in[0], s, v);
+    if (r == R_CONV_S2D_TC) return true;  // one-CTA tiles without a K split
     return false;
 }
 

@@ -627,10 +627,12 @@ static sn_status profile_graph_on(Graph *g, const sn_profile_opts &o, cudaStream
                 // chain whose sub-layer schemas the parent routine fixes)
                 t = 0;
                 for (int32_t stg = 0; stg < nst && rc == SN_OK && t != kInf; ++stg) {
+                    // (the last sub-layer writes the candidate's output schema)
+                    Candidate sc_{cd.routine, stage_uses_variant(cd.routine, stg) ? cd.variant : -1, cd.schema,
+                                  cd.layer, 0};
+                    if (stg == nst - 1) sc_.out_schema = cd.out_schema;
                     std::ostringstream sk;
-                    sk << signature(g, i, Candidate{cd.routine, stage_uses_variant(cd.routine, stg) ? cd.variant : -1,
-                                                    cd.schema, cd.layer, 0})
-                       << "#stage" << stg;
+                    sk << signature(g, i, sc_) << "#stage" << stg;
                     auto hit = seen_stage.find(sk.str());
                     int64_t ts = kInf;
                     if (hit != seen_stage.end()) {
