@@ -43,6 +43,20 @@ def peaks():
     return FALLBACK, "fallback"
 
 
+def job_throughput(ms_local, ws, batch, dist=None, device="cpu"):
+    """Replicas: every rank runs its own batch with no exchange on the data
+    path; the job's step time is the slowest rank's (max over ranks, the one
+    collective) and its throughput the images of all ranks over that time.
+    Returns (ms_per_step, images_per_s)."""
+    ms = ms_local
+    if dist is not None:
+        import torch
+        t = torch.tensor([ms_local], dtype=torch.float64, device=device)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    return ms, ws * batch / (ms / 1e3)
+
+
 def dist_env():
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -336,12 +350,7 @@ def main():
         dist.barrier()
     clk = clocks.stop()
     step_ms = [a.elapsed_time(b) for a, b in ev]
-    ms = sum(step_ms) / len(step_ms)
-    if dist:
-        t = torch.tensor([ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
-    value = ws * args.batch / (ms / 1e3)
+    ms, value = job_throughput(sum(step_ms) / len(step_ms), ws, args.batch, dist, "cuda")
 
     # ---------------- e2e through the C ABI with host buffers ----------------
     # Every step is one sn_run_host call: the library uploads the batch from
